@@ -1,0 +1,17 @@
+"""fp64 CPU oracle for the REAL-Q per-layer quantization sweep.
+
+TEST INFRASTRUCTURE ONLY.  Nothing in the product path may import, call, link
+or execute anything in this package: only the tests, ``__graft_entry__.smoke``
+and the CPU-baseline leg of ``bench.py`` use it.  It shares no code with the
+CUDA path (``paper_2609_00049_gb300``); the two meet only through the seeded
+input generators in ``synth``.
+
+Contents
+--------
+realq.py   the sweep in the paper's order and notation, fp64 throughout except
+           where a floating-point value decides an integer (the int4 code and
+           the zero point), which is taken in fp32 on both sides.
+brute.c    exhaustive search over all int4 codes of a tiny layer (the
+           brute-force pin of the quantizer + surrogate), built by build.py.
+"""
+from .realq import *  # noqa: F401,F403

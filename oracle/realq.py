@@ -1,0 +1,338 @@
+"""Plain fp64 statement of the REAL-Q per-layer sweep (test infrastructure only).
+
+Notation follows the paper: W (m x n, out x in), calibration inputs x̂_t
+(perturbed) and x_t (full precision), H the input second-moment matrix,
+F the aggregated Fisher on the module-output space, B the column block size.
+
+Sections cited:
+  Sec. 3.2 "GPTQ Recap", Eq. (gptq_update) and the lazy batch update after it
+  Sec. 4.2 "Objective", Eq. (fisher_full), Eq. (fisher_loss)
+  Sec. 4.3 "Dynamic Block-wise Gradient Descent", Eq. (block_gd_update)
+  Sec. 4.4 "Loss Sliding Window", Eq. (slide_window)
+  Algorithm 1 "REAL-Q Quantization"
+  App. "Reconstruction error of GPTQ" theorem and the Schur-complement proof
+  App. "Full Setup": Adam hyper-parameters, Eq. (reverse_cosine)
+
+Everything is fp64 except the integer decisions of the quantizer (the code and
+the zero point), which are taken in fp32 arithmetic: the paper does not fix the
+precision of quant(.), and the CUDA path decides in fp32, so both sides decide
+in fp32 on their own fp32-rounded operands.
+
+Readings of points the paper leaves open are listed with each function.
+The oracle performs the OBS compensation of every column immediately on all
+remaining columns and downdates H^-1 explicitly (no lazy batching, no Cholesky
+shortcut): the column sweep is the literal recursion of Eq. (gptq_update) with
+the Schur-complement downdate named in the theorem's proof.
+"""
+from __future__ import annotations
+
+import math
+from typing import Iterable, Optional
+
+import numpy as np
+
+__all__ = [
+    "hessian_sum", "cross_moment_sum", "prepare", "inverse_upper_cholesky",
+    "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
+    "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
+]
+
+
+# ---------------------------------------------------------------------------
+# Step a2: Hessian accumulation.  Sec. 3.2 defines H from the calibration
+# inputs; REAL-Q feeds the perturbed inputs x̂ (Sec. 1, Sec. 2 on GPTAQ).
+# ---------------------------------------------------------------------------
+def hessian_sum(xhat_chunks: Iterable[np.ndarray]):
+    """H_sum = sum_t x̂_t x̂_t^T over all chunks, and the token count T."""
+    H, T = None, 0
+    for c in xhat_chunks:
+        c = np.asarray(c, dtype=np.float64)
+        if H is None:
+            H = np.zeros((c.shape[1], c.shape[1]))
+        H += c.T @ c
+        T += c.shape[0]
+    return H, T
+
+
+def cross_moment_sum(xhat_chunks: Iterable[np.ndarray], x_chunks: Iterable[np.ndarray]):
+    """D_sum[i, j] = sum_t (x̂_ti - x_ti) x̂_tj.
+
+    With Δy_t = Ŵ x̂_t - W0 x_t, the surrogate gradient needs
+    (1/T) sum_t Δy_t x̂_t^T = (Ŵ - W0) H̄ + W0 D̄ with D̄ = D_sum / T.
+    """
+    D = None
+    for ch, cx in zip(xhat_chunks, x_chunks):
+        ch = np.asarray(ch, dtype=np.float64)
+        cx = np.asarray(cx, dtype=np.float64)
+        if D is None:
+            D = np.zeros((ch.shape[1], ch.shape[1]))
+        D += (ch - cx).T @ ch
+    return D
+
+
+# ---------------------------------------------------------------------------
+# Step a3: preparation of the OBS Hessian (Alg. 1, "Compute ... H_g and its
+# inverse").  Readings: H̄ = H_sum / T (the factor 2/T of Sec. 3.2 cancels in
+# every ratio the OBS step uses); channels that never fire (H_jj = 0) get
+# H_jj = 1 and their weights are zeroed; damping lambda = damp * mean(diag H̄).
+# ---------------------------------------------------------------------------
+def prepare(H_sum: np.ndarray, T: int, damp_frac: float = 0.01):
+    H_sum = np.asarray(H_sum, dtype=np.float64)
+    n = H_sum.shape[0]
+    Hbar = H_sum / float(T)
+    dead = np.diag(H_sum) == 0.0
+    Hd = Hbar.copy()
+    idx = np.arange(n)
+    Hd[idx[dead], idx[dead]] = 1.0
+    lam = damp_frac * float(np.mean(np.diag(Hd)))
+    Hd[idx, idx] += lam
+    return {"Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": lam}
+
+
+def inverse_upper_cholesky(Hd: np.ndarray) -> np.ndarray:
+    """U upper triangular with Hd^-1 = U^T U (the 'Cholesky-based inverse')."""
+    Hinv = np.linalg.inv(Hd)
+    L = np.linalg.cholesky(Hinv)       # Hinv = L L^T, L lower
+    return L.T.copy()                  # U = L^T  =>  Hinv = U^T U
+
+
+# ---------------------------------------------------------------------------
+# quant(.) of Alg. 1: uniform b-bit grid.  Reading: asymmetric
+# min/max grid that always contains 0 (xmin <= 0 <= xmax, degenerate rows get
+# [-1, 1]), scale = (xmax - xmin) / (2^b - 1), integer zero point; symmetric
+# variant: xmax = max(|xmin|, xmax), xmin = -xmax, zero = 2^(b-1).  Rounding is
+# round-half-to-even.  Decisions in fp32 (module docstring).
+# ---------------------------------------------------------------------------
+def quant_params(w_rows: np.ndarray, bits: int = 4, symmetric: bool = False):
+    """Per-row (scale fp32, zero int) for a group of columns w_rows (m x g)."""
+    w = np.asarray(w_rows, dtype=np.float64).astype(np.float32)
+    maxq = np.float32(2 ** bits - 1)
+    xmin = np.minimum(w.min(axis=1), np.float32(0.0))
+    xmax = np.maximum(w.max(axis=1), np.float32(0.0))
+    if symmetric:
+        xmax = np.maximum(-xmin, xmax)
+        xmin = -xmax
+    both0 = (xmin == 0) & (xmax == 0)
+    xmin = np.where(both0, np.float32(-1.0), xmin).astype(np.float32)
+    xmax = np.where(both0, np.float32(1.0), xmax).astype(np.float32)
+    scale = ((xmax - xmin) / maxq).astype(np.float32)
+    if symmetric:
+        zero = np.full(w.shape[0], 2 ** (bits - 1), dtype=np.int64)
+        zmargin = np.full(w.shape[0], 0.5)
+    else:
+        zf = (-xmin / scale).astype(np.float32)
+        zero = np.rint(zf).astype(np.int64)
+        zmargin = np.abs(np.abs(zf.astype(np.float64) - np.floor(zf)) - 0.5)
+    return scale, zero, zmargin
+
+
+def quantize(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int = 4):
+    """q = clamp(rint(w / scale) + zero, 0, 2^b - 1); deq = scale * (q - zero).
+
+    Returns (q int64, deq as fp64 of the fp32 value, margin) where margin is the
+    distance of w/scale from the nearest rounding boundary, in grid steps.
+    """
+    maxq = 2 ** bits - 1
+    x = (np.asarray(w, dtype=np.float64).astype(np.float32) / scale.astype(np.float32)).astype(np.float32)
+    r = np.rint(x)
+    q = np.clip(r.astype(np.int64) + zero, 0, maxq)
+    deq = (scale.astype(np.float32) * (q.astype(np.float32) - zero.astype(np.float32))).astype(np.float32)
+    x64 = x.astype(np.float64)
+    margin = np.abs(np.abs(x64 - np.floor(x64)) - 0.5)
+    return q, deq.astype(np.float64), margin
+
+
+def rtn(W: np.ndarray, bits: int = 4, group_size: int = 128, symmetric: bool = False):
+    """Round-to-nearest baseline: every group quantized from the original weights."""
+    W = np.asarray(W, dtype=np.float64)
+    m, n = W.shape
+    g = group_size if group_size > 0 else n
+    codes = np.zeros((m, n), dtype=np.int64)
+    deq = np.zeros((m, n))
+    scales, zeros = [], []
+    for j0 in range(0, n, g):
+        s, z, _ = quant_params(W[:, j0:j0 + g], bits, symmetric)
+        for j in range(j0, min(j0 + g, n)):
+            codes[:, j], deq[:, j], _ = quantize(W[:, j], s, z, bits)
+        scales.append(s)
+        zeros.append(z)
+    return codes, deq, np.stack(scales, 1), np.stack(zeros, 1)
+
+
+# ---------------------------------------------------------------------------
+# Schedules.  Eq. (slide_window) and Eq. (reverse_cosine).
+# ---------------------------------------------------------------------------
+def sliding_alpha(b_global: int, B_total: int) -> float:
+    """alpha = 1 - (b_global - 1) / (B_total - 1); 1 when there is one step only."""
+    if B_total <= 1:
+        return 1.0
+    return 1.0 - (b_global - 1) / (B_total - 1)
+
+
+def reverse_cosine_lr(i: int, L: int, eta_final: float, eta_base: Optional[float] = None) -> float:
+    """Learning rate of transformer block i (1-based) of L; eta_base = 0.01 eta_final."""
+    if eta_base is None:
+        eta_base = 0.01 * eta_final
+    if L <= 1:
+        return eta_final
+    return eta_base + (eta_final - eta_base) * math.sin(0.5 * math.pi * (i - 1) / (L - 1))
+
+
+# ---------------------------------------------------------------------------
+# Adam (App. "Full Setup": beta1 0.9, beta2 0.999, eps 1e-8, bias correction
+# at every block step).  Reading: PyTorch placement of eps (outside the sqrt),
+# no weight decay; one state per weight, reset per module.
+# ---------------------------------------------------------------------------
+class Adam:
+    def __init__(self, shape, lr, beta1=0.9, beta2=0.999, eps=1e-8):
+        self.m = np.zeros(shape)
+        self.v = np.zeros(shape)
+        self.t = 0
+        self.lr, self.beta1, self.beta2, self.eps = lr, beta1, beta2, eps
+
+    def direction(self, g: np.ndarray, cols: slice) -> np.ndarray:
+        """Advance the moments of columns `cols` with gradient g; return the step."""
+        self.t += 1
+        m = self.m[:, cols]
+        v = self.v[:, cols]
+        m[...] = self.beta1 * m + (1.0 - self.beta1) * g
+        v[...] = self.beta2 * v + (1.0 - self.beta2) * g * g
+        mhat = m / (1.0 - self.beta1 ** self.t)
+        vhat = v / (1.0 - self.beta2 ** self.t)
+        return self.lr * mhat / (np.sqrt(vhat) + self.eps)
+
+
+# ---------------------------------------------------------------------------
+# Surrogate, Eq. (fisher_loss), read at the layer level: Δy_t = Ŵ x̂_t - W0 x_t
+# on the module-output space with an m x m Fisher F.
+# ---------------------------------------------------------------------------
+def surrogate_tokens(What, W0, Xhat, X, F) -> float:
+    """(1/2)(1/T) sum_t Δy_t^T F Δy_t, evaluated token by token (matmul per chunk)."""
+    What = np.asarray(What, dtype=np.float64)
+    W0 = np.asarray(W0, dtype=np.float64)
+    F = np.asarray(F, dtype=np.float64)
+    Xhat = np.asarray(Xhat)
+    X = Xhat if X is None else np.asarray(X)
+    T = Xhat.shape[0]
+    acc = 0.0
+    for t0 in range(0, T, 4096):
+        xh = Xhat[t0:t0 + 4096].astype(np.float64)
+        xx = X[t0:t0 + 4096].astype(np.float64)
+        dY = xh @ What.T - xx @ W0.T
+        acc += float(np.sum((dY @ F) * dY))
+    return 0.5 * acc / T
+
+
+def surrogate_moment(What, W0, Hbar, F) -> float:
+    """Same loss when X = X̂: (1/2) tr(F ΔW H̄ ΔW^T) with ΔW = Ŵ - W0."""
+    dW = np.asarray(What, dtype=np.float64) - np.asarray(W0, dtype=np.float64)
+    return 0.5 * float(np.sum((np.asarray(F, dtype=np.float64) @ dW) * (dW @ np.asarray(Hbar, dtype=np.float64))))
+
+
+def gradient(What, W0, Hbar, Dbar, F) -> np.ndarray:
+    """dL/dŴ = F P with P = (1/T) sum_t Δy_t x̂_t^T = (Ŵ - W0) H̄ + W0 D̄ (m x n)."""
+    W0 = np.asarray(W0, dtype=np.float64)
+    P = (np.asarray(What, dtype=np.float64) - W0) @ np.asarray(Hbar, dtype=np.float64)
+    if Dbar is not None:
+        P = P + W0 @ np.asarray(Dbar, dtype=np.float64)
+    return np.asarray(F, dtype=np.float64) @ P
+
+
+def pack_codes(codes: np.ndarray) -> np.ndarray:
+    """Two int4 codes per byte, even column in the low nibble (m x ceil(n/2) uint8)."""
+    m, n = codes.shape
+    c = np.zeros((m, n + (n & 1)), dtype=np.uint8)
+    c[:, :n] = codes
+    return (c[:, 0::2] | (c[:, 1::2] << 4)).astype(np.uint8)
+
+
+# ---------------------------------------------------------------------------
+# The sweep: Algorithm 1, inner loops for one linear module.
+# ---------------------------------------------------------------------------
+def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetric=False,
+                damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True):
+    """Quantize W0 column by column with OBS feedback and Block-GD after each block.
+
+    bgd: None for the plain column sweep (GPTQ), else a dict with keys
+      steps_per_block (1 in the paper), lr, beta1, beta2, eps,
+      optimizer ("adam" | "sgd"), b_global_start (1-based cumulative block index
+      of this module's first block), B_total (column-block steps in the
+      transformer block; 1 disables the sliding window).
+
+    Readings: group parameters are computed at the first column of each group
+    from the current (compensated, Block-GD-updated) weights; group_size 0
+    means one group per row; the gradient is the full-batch moment form of the
+    layer-level surrogate; Block-GD updates all rows jointly on the columns
+    after the block; the block after the last column is skipped (no columns
+    remain).  Returns a dict of codes, scale, zero, deq (fp32 values as fp64),
+    per-column residuals, tie margins and per-block surrogate values.
+    """
+    W0 = np.asarray(W0, dtype=np.float64)
+    m, n = W0.shape
+    B = block_size
+    g = group_size if group_size > 0 else n
+    if not (g % B == 0 or B % g == 0 or g == n):
+        raise ValueError("group size must divide the block size or be a multiple of it")
+    prep = prepare(H_sum, T, damp_frac)
+    Hbar, Hd, dead = prep["Hbar"], prep["Hd"], prep["dead"]
+    Dbar = None if D_sum is None else np.asarray(D_sum, dtype=np.float64) / float(T)
+
+    W = W0.copy()
+    W[:, dead] = 0.0
+    Hinv = np.linalg.inv(Hd)
+    ngroups = -(-n // g)
+    codes = np.zeros((m, n), dtype=np.int64)
+    scale = np.zeros((m, ngroups), dtype=np.float32)
+    zero = np.zeros((m, ngroups), dtype=np.int64)
+    margin = np.zeros((m, n))
+    zmargin = np.zeros((m, ngroups))
+    eps_cols = np.zeros((m, n))
+    hinv_diag = np.zeros(n)
+    block_loss = []
+    opt = None
+    if bgd is not None:
+        opt = Adam((m, n), bgd["lr"], bgd.get("beta1", 0.9), bgd.get("beta2", 0.999), bgd.get("eps", 1e-8))
+    Fm = None if F is None else np.asarray(F, dtype=np.float64)
+    Fn = None if F_next is None else np.asarray(F_next, dtype=np.float64)
+
+    for j in range(n):
+        if j % g == 0:
+            gi = j // g
+            scale[:, gi], zero[:, gi], zmargin[:, gi] = quant_params(W[:, j:j + g], bits, symmetric)
+        gi = j // g
+        q, dq, mg = quantize(W[:, j], scale[:, gi], zero[:, gi], bits)
+        e = W[:, j] - dq                       # residual delta_j of Eq. (gptq_update)
+        d = Hinv[j, j]
+        codes[:, j] = q
+        margin[:, j] = mg
+        eps_cols[:, j] = e
+        hinv_diag[j] = d
+        # Eq. (gptq_update): W[:, j+1:] -= delta_j H^-1[j, j+1:] / [H^-1]_jj
+        W[:, j + 1:] -= np.outer(e / d, Hinv[j, j + 1:])
+        # remove j from the free set: Schur-complement downdate of H^-1
+        Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d
+        W[:, j] = dq
+
+        be = j + 1
+        if opt is not None and (be % B == 0 or be == n) and be < n:
+            b = j // B
+            b_global = bgd.get("b_global_start", 1) + b
+            alpha = sliding_alpha(b_global, bgd.get("B_total", 1))
+            Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
+            before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
+            for _ in range(bgd.get("steps_per_block", 1)):
+                G = gradient(W, W0, Hbar, Dbar, Feff)[:, be:]
+                if bgd.get("optimizer", "adam") == "sgd":
+                    opt.t += 1
+                    W[:, be:] -= bgd["lr"] * G
+                else:
+                    W[:, be:] -= opt.direction(G, slice(be, n))
+            after = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
+            block_loss.append((b, alpha, before, after))
+
+    return {
+        "codes": codes, "scale": scale, "zero": zero, "deq": W.copy(),
+        "margin": margin, "zero_margin": zmargin, "eps": eps_cols, "hinv_diag": hinv_diag,
+        "block_loss": block_loss, "adam_t": 0 if opt is None else opt.t,
+        "Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": prep["lam"], "Dbar": Dbar,
+    }

@@ -1,0 +1,378 @@
+"""Pins of the fp64 oracle against what the paper and the mathematics fix.
+
+Each test checks the oracle against something other than itself: a closed
+form, a brute-force search, a special case that reduces to a textbook routine,
+an independent route to the same quantity, or a library implementation.
+"""
+import math
+
+import numpy as np
+import pytest
+
+import oracle
+import synth
+from oracle import brute
+
+
+def _correlated_case(seed, m, n, T, w_std=0.02):
+    r = synth.rng(seed, "pin-corr", m, n, T)
+    Z = r.standard_normal((T, n))
+    M = np.eye(n) + 0.6 * r.standard_normal((n, n)) / math.sqrt(n)
+    X = Z @ M
+    W0 = r.standard_normal((m, n)) * w_std
+    return W0.astype(np.float32).astype(np.float64), X
+
+
+# ---------------------------------------------------------------------------
+# quantizer: the grid point chosen is the nearest one among all 2^b codes
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("bits,sym", [(4, False), (4, True), (3, False), (2, True)])
+def test_quantizer_is_nearest_grid_point(bits, sym):
+    r = synth.rng(1, "quant", bits, int(sym))
+    w = r.standard_normal((64, 128)) * 0.02
+    w[:, 5] *= 4.0                      # values outside the grid range get clamped
+    s, z, _ = oracle.quant_params(w[:, :100], bits, sym)
+    levels = 2 ** bits
+    grid = (s[:, None].astype(np.float32) * (np.arange(levels, dtype=np.float32)[None, :] - z[:, None].astype(np.float32)))
+    for j in range(w.shape[1]):
+        q, dq, _ = oracle.quantize(w[:, j], s, z, bits)
+        dist = np.abs(grid.astype(np.float64) - w[:, j:j + 1].astype(np.float32).astype(np.float64))
+        chosen = dist[np.arange(64), q]
+        # the chosen code is a nearest grid point (up to fp32 rounding of w/scale)
+        assert np.all(chosen <= dist.min(axis=1) + 1e-6 * s)
+        assert np.array_equal(dq, grid[np.arange(64), q].astype(np.float64))
+        unique = np.sort(dist, axis=1)[:, 1] - dist.min(axis=1) > 1e-6 * s
+        assert np.array_equal(q[unique], np.argmin(dist, axis=1)[unique])
+    # the grid holds 0 exactly and spans the group's range
+    assert np.all(np.min(np.abs(grid), axis=1) == 0.0)
+    lo = np.minimum(w[:, :100].min(1), 0)
+    hi = np.maximum(w[:, :100].max(1), 0)
+    assert np.all(grid.min(1) <= lo + s) and np.all(grid.max(1) >= hi - s)
+
+
+def test_degenerate_group_gets_unit_range():
+    s, z, _ = oracle.quant_params(np.zeros((3, 8)), 4, False)
+    # -xmin/scale = 1/(2/15) evaluates to 7.4999997 in fp32, so the zero point is 7
+    assert np.allclose(s, 2.0 / 15.0) and np.all(z == 7)
+
+
+# ---------------------------------------------------------------------------
+# RTN special case: no Block-GD and H = I leave no error feedback
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("group,sym,bits", [(128, False, 4), (0, True, 4), (32, False, 3)])
+def test_identity_hessian_reduces_to_rtn(group, sym, bits):
+    r = synth.rng(2, "rtn")
+    W0 = r.standard_normal((48, 256)) * 0.02
+    T = 1000
+    res = oracle.realq_sweep(W0, T * np.eye(256), T, bits=bits, group_size=group, symmetric=sym, damp_frac=0.01)
+    codes, deq, s, z = oracle.rtn(W0, bits, group, sym)
+    assert np.array_equal(res["codes"], codes)
+    assert np.array_equal(res["deq"], deq)
+    assert np.array_equal(res["scale"], s) and np.array_equal(res["zero"], z)
+
+
+# ---------------------------------------------------------------------------
+# OBS step against the definition: at column j the compensation uses row j of
+# the inverse of H restricted to the columns still free (Schur complement),
+# and the same sweep through rows of the upper Cholesky factor of H^-1,
+# immediate or lazily batched, gives the same result.
+# ---------------------------------------------------------------------------
+def _sweep_submatrix_inverse(W0, Hd, bits, g, sym):
+    W = W0.copy()
+    m, n = W.shape
+    codes = np.zeros((m, n), dtype=np.int64)
+    for j in range(n):
+        if j % g == 0:
+            s, z, _ = oracle.quant_params(W[:, j:j + g], bits, sym)
+        q, dq, _ = oracle.quantize(W[:, j], s, z, bits)
+        eps = W[:, j] - dq
+        Hinv_free = np.linalg.inv(Hd[j:, j:])          # free set {j, ..., n-1}
+        v = np.zeros(n)
+        v[j] = -1.0
+        v[j + 1:] = -Hinv_free[0, 1:] / Hinv_free[0, 0]  # the lemma's compensation vector
+        W += np.outer(eps, v)                          # ΔW^(j) = eps_j v_j^T
+        W[:, j] = dq
+        codes[:, j] = q
+    return codes, W
+
+
+def _sweep_cholesky_lazy(W0, Hd, bits, g, sym, B):
+    U = np.linalg.cholesky(np.linalg.inv(Hd)).T
+    W = W0.copy()
+    m, n = W.shape
+    codes = np.zeros((m, n), dtype=np.int64)
+    for b0 in range(0, n, B):
+        b1 = min(b0 + B, n)
+        E = np.zeros((m, b1 - b0))
+        for j in range(b0, b1):
+            if j % g == 0:
+                s, z, _ = oracle.quant_params(W[:, j:j + g], bits, sym)
+            q, dq, _ = oracle.quantize(W[:, j], s, z, bits)
+            err = (W[:, j] - dq) / U[j, j]
+            W[:, j + 1:b1] -= np.outer(err, U[j, j + 1:b1])
+            W[:, j] = dq
+            E[:, j - b0] = err
+            codes[:, j] = q
+        W[:, b1:] -= E @ U[b0:b1, b1:]
+    return codes, W
+
+
+@pytest.mark.parametrize("n,g,B", [(3, 3, 1), (8, 8, 2), (12, 4, 4), (16, 8, 4)])
+def test_obs_recursion_matches_definitions(n, g, B):
+    W0, X = _correlated_case(3, 4, n, 200)
+    H = X.T @ X
+    ref = oracle.realq_sweep(W0, H, 200, bits=4, group_size=g, block_size=B, damp_frac=0.01)
+    Hd = ref["Hd"]
+    c1, w1 = _sweep_submatrix_inverse(W0, Hd, 4, g, False)
+    c2, w2 = _sweep_cholesky_lazy(W0, Hd, 4, g, False, B)
+    assert np.array_equal(ref["codes"], c1) and np.array_equal(ref["codes"], c2)
+    assert np.allclose(ref["deq"], w1, rtol=0, atol=1e-12)
+    assert np.allclose(ref["deq"], w2, rtol=0, atol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Theorem "Reconstruction error of GPTQ": sum_j ||eps_j||^2 / [H^-1]_jj equals
+# tr(ΔW H ΔW^T) exactly under the fixed Hessian.
+# ---------------------------------------------------------------------------
+@pytest.mark.parametrize("seed,m,n,g", [(4, 16, 64, 16), (5, 8, 96, 32), (6, 32, 40, 0)])
+def test_gptq_error_theorem(seed, m, n, g):
+    W0, X = _correlated_case(seed, m, n, 500)
+    res = oracle.realq_sweep(W0, X.T @ X, 500, bits=3, group_size=g, block_size=8)
+    lhs = np.sum(np.sum(res["eps"] ** 2, axis=0) / res["hinv_diag"])
+    dW = res["deq"] - W0
+    rhs = np.trace(dW @ res["Hd"] @ dW.T)
+    assert abs(lhs - rhs) <= 1e-10 * abs(rhs)
+
+
+# ---------------------------------------------------------------------------
+# Closed-form inverse: the Kac-Murdock-Szego matrix A_ij = rho^|i-j| has a
+# tridiagonal inverse, and every trailing principal block is again KMS.
+# ---------------------------------------------------------------------------
+def _kms_inverse(n, rho):
+    Ainv = np.zeros((n, n))
+    c = 1.0 / (1.0 - rho * rho)
+    for i in range(n):
+        Ainv[i, i] = c * (1.0 + rho * rho) if 0 < i < n - 1 else c
+        if i + 1 < n:
+            Ainv[i, i + 1] = Ainv[i + 1, i] = -rho * c
+    if n == 1:
+        Ainv[0, 0] = 1.0
+    return Ainv
+
+
+def test_kms_closed_form_inverse_and_downdate():
+    n, rho, T = 24, 0.7, 10
+    A = rho ** np.abs(np.subtract.outer(np.arange(n), np.arange(n)))
+    U = oracle.inverse_upper_cholesky(A)
+    assert np.allclose(U.T @ U, _kms_inverse(n, rho), atol=1e-12)
+    assert np.allclose(np.tril(U, -1), 0.0)
+    r = synth.rng(7, "kms")
+    W0 = r.standard_normal((5, n)) * 0.02
+    res = oracle.realq_sweep(W0, T * A, T, damp_frac=0.0, group_size=0)
+    want = np.array([_kms_inverse(n - j, rho)[0, 0] for j in range(n)])
+    assert np.allclose(res["hinv_diag"], want, rtol=1e-12)
+
+
+# ---------------------------------------------------------------------------
+# Hessian: integer inputs give an exact H; compare with exact integer sums.
+# ---------------------------------------------------------------------------
+def test_hessian_exact_on_integer_inputs():
+    r = synth.rng(8, "hint")
+    X = r.integers(-2, 3, size=(300, 7))
+    H, T = oracle.hessian_sum([X[:128], X[128:]])
+    assert T == 300
+    for i in range(7):
+        for j in range(7):
+            assert H[i, j] == sum(int(X[t, i]) * int(X[t, j]) for t in range(300))
+    Xfp = r.integers(-2, 3, size=(300, 7))
+    D = oracle.cross_moment_sum([X], [Xfp])
+    for i in range(7):
+        for j in range(7):
+            assert D[i, j] == sum((int(X[t, i]) - int(Xfp[t, i])) * int(X[t, j]) for t in range(300))
+
+
+def test_dead_columns():
+    case = synth.layer_case(9, 6, 20, 64, dead_cols=(3, 11))
+    H, T = oracle.hessian_sum([case.Xhat])
+    res = oracle.realq_sweep(case.W0, H, T, group_size=0)
+    assert list(np.nonzero(res["dead"])[0]) == [3, 11]
+    assert np.all(res["deq"][:, [3, 11]] == 0.0)
+    assert np.all(res["codes"][:, [3, 11]] == res["zero"][:, [0]])
+    Hd = res["Hd"]
+    assert Hd[3, 3] == 1.0 + res["lam"] and np.all(Hd[3, :3] == 0.0)
+    # reading: the damping mean is taken after the dead channels got H_jj = 1
+    d = np.where(res["dead"], 1.0, np.diag(H) / T)
+    assert res["lam"] == pytest.approx(0.01 * d.mean(), rel=1e-15)
+
+
+# ---------------------------------------------------------------------------
+# Surrogate and gradient: token form vs moment form; finite differences.
+# ---------------------------------------------------------------------------
+def test_surrogate_two_routes():
+    case = synth.layer_case(10, 12, 20, 300)
+    H, T = oracle.hessian_sum([case.Xhat])
+    r = synth.rng(10, "what")
+    What = case.W0 + 0.003 * r.standard_normal(case.W0.shape)
+    a = oracle.surrogate_tokens(What, case.W0, case.Xhat, None, case.F)
+    b = oracle.surrogate_moment(What, case.W0, H / T, case.F)
+    assert abs(a - b) <= 1e-12 * abs(a)
+
+
+def test_gradient_finite_differences_with_perturbed_inputs():
+    case = synth.layer_case(11, 5, 7, 200, perturbed=True)
+    H, T = oracle.hessian_sum([case.Xhat])
+    D = oracle.cross_moment_sum([case.Xhat], [case.X])
+    r = synth.rng(11, "what")
+    What = case.W0 + 0.01 * r.standard_normal(case.W0.shape)
+    G = oracle.gradient(What, case.W0, H / T, D / T, case.F)
+    h = 1e-6
+    for (i, j) in [(0, 0), (2, 3), (4, 6), (1, 5)]:
+        Wp = What.copy(); Wp[i, j] += h
+        Wm = What.copy(); Wm[i, j] -= h
+        fd = (oracle.surrogate_tokens(Wp, case.W0, case.Xhat, case.X, case.F)
+              - oracle.surrogate_tokens(Wm, case.W0, case.Xhat, case.X, case.F)) / (2 * h)
+        assert abs(fd - G[i, j]) <= 1e-6 * max(1e-3, abs(G[i, j]))
+
+
+# ---------------------------------------------------------------------------
+# Descent lemma (Sec. 5, SGD form): the surrogate is quadratic in the free
+# columns, so one SGD step changes it by exactly
+#   -eta ||G||^2 + (eta^2/2) <G, F G H̄_rr>,
+# negative whenever eta < 2 / (lambda_max(F) lambda_max(H̄_rr)).
+# ---------------------------------------------------------------------------
+def test_sgd_step_descent_lemma():
+    case = synth.layer_case(12, 16, 48, 400, outliers=2)
+    H, T = oracle.hessian_sum([case.Xhat])
+    Hbar = H / T
+    F = case.F.astype(np.float64)
+    B = 16
+    be = B
+    lmax = np.linalg.eigvalsh(F)[-1] * np.linalg.eigvalsh(Hbar[be:, be:])[-1]
+    eta = 1.0 / lmax
+    res = oracle.realq_sweep(case.W0, H, T, block_size=B, group_size=16,
+                             bgd={"lr": eta, "optimizer": "sgd"}, F=F)
+    assert len(res["block_loss"]) == 2
+    for (b, alpha, before, after) in res["block_loss"]:
+        assert after < before
+    # quadratic identity at a random point, loss evaluated token by token
+    r = synth.rng(12, "quad")
+    What = case.W0 + 0.004 * r.standard_normal(case.W0.shape)
+    G = oracle.gradient(What, case.W0, Hbar, None, F)[:, be:]
+    Wn = What.copy(); Wn[:, be:] -= eta * G
+    d_loss = oracle.surrogate_tokens(Wn, case.W0, case.Xhat, None, F) - oracle.surrogate_tokens(What, case.W0, case.Xhat, None, F)
+    pred = -eta * np.sum(G * G) + 0.5 * eta * eta * np.sum(G * (F @ G @ Hbar[be:, be:]))
+    assert abs(d_loss - pred) <= 1e-9 * abs(pred)
+    assert pred < 0
+
+
+# ---------------------------------------------------------------------------
+# Adam against torch.optim.Adam in fp64 (library implementation).
+# ---------------------------------------------------------------------------
+def test_adam_matches_torch():
+    torch = pytest.importorskip("torch")
+    r = synth.rng(13, "adam")
+    p0 = r.standard_normal((6, 9))
+    grads = [r.standard_normal((6, 9)) * 10 ** r.uniform(-3, 1) for _ in range(6)]
+    opt = oracle.Adam(p0.shape, lr=3e-4)
+    p = p0.copy()
+    tp = torch.tensor(p0, dtype=torch.float64, requires_grad=True)
+    topt = torch.optim.Adam([tp], lr=3e-4, betas=(0.9, 0.999), eps=1e-8)
+    for g in grads:
+        p -= opt.direction(g, slice(0, 9))
+        tp.grad = torch.tensor(g, dtype=torch.float64)
+        topt.step()
+    assert np.allclose(p, tp.detach().numpy(), rtol=0, atol=1e-15)
+    # first step is lr * g / (|g| + eps): a sign step
+    o2 = oracle.Adam((1, 3), lr=0.5)
+    d = o2.direction(np.array([[2.0, -1e-3, 0.0]]), slice(0, 3))
+    assert np.allclose(d, [[0.5 * 2 / (2 + 1e-8), -0.5 * 1e-3 / (1e-3 + 1e-8), 0.0]], rtol=1e-14)
+
+
+# ---------------------------------------------------------------------------
+# Schedules: Eq. (slide_window) and Eq. (reverse_cosine).
+# ---------------------------------------------------------------------------
+def test_schedules():
+    assert oracle.sliding_alpha(1, 304) == 1.0
+    assert oracle.sliding_alpha(304, 304) == 0.0
+    a = [oracle.sliding_alpha(b, 11) for b in range(1, 12)]
+    assert np.allclose(np.diff(a), -0.1)
+    assert oracle.sliding_alpha(1, 1) == 1.0
+    assert math.isclose(oracle.reverse_cosine_lr(1, 32, 1e-5), 1e-7)
+    assert math.isclose(oracle.reverse_cosine_lr(32, 32, 1e-5), 1e-5)
+    mid = oracle.reverse_cosine_lr(17, 33, 1.0)
+    assert math.isclose(mid, 0.01 + 0.99 * math.sin(math.pi / 4))
+
+
+def test_sliding_window_blends_fishers():
+    case = synth.layer_case(14, 8, 24, 100, with_next=True)
+    H, T = oracle.hessian_sum([case.Xhat])
+    bgd = {"lr": 1e-4, "b_global_start": 3, "B_total": 7}
+    res = oracle.realq_sweep(case.W0, H, T, block_size=8, group_size=8, bgd=bgd, F=case.F, F_next=case.F_next)
+    alphas = [x[1] for x in res["block_loss"]]
+    assert np.allclose(alphas, [1 - 2 / 6, 1 - 3 / 6])
+    assert res["adam_t"] == 2
+
+
+# ---------------------------------------------------------------------------
+# Output invariants of a full sweep.
+# ---------------------------------------------------------------------------
+def test_sweep_output_invariants():
+    case = synth.layer_case(15, 20, 300, 400, outliers=3)
+    H, T = oracle.hessian_sum([case.Xhat])
+    res = oracle.realq_sweep(case.W0, H, T, block_size=128, group_size=128,
+                             bgd={"lr": 1e-4}, F=case.F)
+    codes, s, z = res["codes"], res["scale"], res["zero"]
+    assert codes.min() >= 0 and codes.max() <= 15
+    gi = np.arange(300) // 128
+    deq = (s[:, gi] * (codes.astype(np.float32) - z[:, gi].astype(np.float32))).astype(np.float64)
+    assert np.array_equal(deq, res["deq"])
+    assert res["adam_t"] == 2
+    packed = oracle.pack_codes(codes)
+    assert packed.shape == (20, 150)
+    assert np.array_equal(packed[:, 7] & 15, codes[:, 14]) and np.array_equal(packed[:, 7] >> 4, codes[:, 15])
+
+
+# ---------------------------------------------------------------------------
+# Brute force over all int4 codes of a 4 x 8 layer (diagonal Fisher: rows
+# decouple).  The surrogate evaluator agrees with the independent C evaluator;
+# no code vector beats the global minimum; the sweep does not lose to RTN; with
+# one column the sweep is the exact minimiser.
+# ---------------------------------------------------------------------------
+@pytest.mark.slow
+def test_brute_force_4x8():
+    W0, X = _correlated_case(16, 4, 8, 64)
+    T = X.shape[0]
+    H = X.T @ X
+    F = np.diag(synth.rng(16, "fd").uniform(0.5, 2.0, size=4))
+    gptq = oracle.realq_sweep(W0, H, T, group_size=0, block_size=8)
+    realq = oracle.realq_sweep(W0, H, T, group_size=0, block_size=2, bgd={"lr": 2e-4}, F=F)
+    codes_rtn, _, s_rtn, z_rtn = oracle.rtn(W0, 4, 0)
+    s, z = gptq["scale"][:, 0], gptq["zero"][:, 0]
+    assert np.array_equal(s, s_rtn[:, 0]) and np.array_equal(z, z_rtn[:, 0])
+    Hbar = H / T
+    mins, argmins = brute.layer_min(W0, s, z, Hbar)
+    f = np.diag(F)
+    for name, res in (("gptq", gptq), ("realq", realq)):
+        per_row = np.array([brute.row_eval(W0[i], s[i], z[i], Hbar, res["codes"][i]) for i in range(4)])
+        L_or = oracle.surrogate_moment(res["deq"], W0, Hbar, F)
+        assert abs(0.5 * np.sum(f * per_row) - L_or) <= 1e-12 * L_or, name
+        assert np.all(mins <= per_row * (1 + 1e-12)), name
+    # n = 8 is small enough that the greedy sweep may lose to RTN on a row; over
+    # many rows of the same input it must win (a sign or index error would not)
+    Wm, _ = _correlated_case(16, 256, 8, 64)
+    gm = oracle.realq_sweep(Wm, H, T, group_size=0, block_size=8)
+    cr, dr, _, _ = oracle.rtn(Wm, 4, 0)
+    Fi = np.eye(256)
+    assert oracle.surrogate_moment(gm["deq"], Wm, Hbar, Fi) < 0.9 * oracle.surrogate_moment(dr, Wm, Hbar, Fi)
+
+
+def test_single_column_sweep_is_exact_minimiser():
+    r = synth.rng(17, "n1")
+    W0 = r.standard_normal((32, 1)) * 0.02
+    H = np.array([[3.7]])
+    res = oracle.realq_sweep(W0, H, 1, group_size=0)
+    s, z = res["scale"][:, 0], res["zero"][:, 0]
+    for i in range(32):
+        best, arg = brute.row_min(W0[i], s[i], z[i], H / 1.0)
+        val = brute.row_eval(W0[i], s[i], z[i], H / 1.0, res["codes"][i])
+        assert val <= best * (1 + 1e-12) + 1e-300
