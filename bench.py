@@ -1,0 +1,472 @@
+"""Throughput of the REAL-Q per-layer quantization sweep on GB300.
+
+One step = the whole sweep of one synthetic decoder block (default: the
+Qwen3-0.6B-shaped block, 128 x 2048 calibration tokens): for each of its four
+distinct inputs the Hessian over all tokens and its preparation, then the
+column sweep with Block-GD of its seven linear modules.  Metric: quantized
+weight-columns per second (whole job; N GPUs run N independent replicas).
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
+
+Prints one JSON line (rank 0).  --impl reference times the fp64 CPU oracle on
+a bounded sample of the same workload instead.
+"""
+from __future__ import annotations
+
+import argparse
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+import synth  # noqa: E402
+
+METRIC = "quantized weight-columns/sec per layer on 1 GB300; % tensor-core peak / % HBM BW"
+UNIT = "columns/s"
+
+# dram bytes per launch from ncu captures (profiles/), keyed by kernel; None
+# when the kernel changed after its capture.
+NCU_TRAFFIC = {}
+
+
+def load_peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        with open(p) as f:
+            d = json.load(f)
+        return {"hbm_gbs": d["hbm_gbs"], "bf16_tflops": d["bf16_tflops"],
+                "bf16_tflops_sustained": d.get("bf16_tflops_sustained", d["bf16_tflops"]),
+                "sm_max_mhz": d.get("sm_max_mhz", 2070.0), "source": "measured"}
+    except Exception:
+        return {"hbm_gbs": 6800.0, "bf16_tflops": 1900.0, "bf16_tflops_sustained": 1700.0, "sm_max_mhz": 2070.0,
+                "source": "fallback"}
+
+
+# --------------------------------------------------------------------------
+# clocks sampled during the timed region
+# --------------------------------------------------------------------------
+class ClockSampler:
+    FIELDS = ("index,uuid,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, uuid):
+        self.uuid = uuid
+        self.proc = None
+        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+
+    def start(self):
+        try:
+            os.makedirs(os.path.dirname(self.path), exist_ok=True)
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
+                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if self.proc is None:
+            return None
+        time.sleep(0.25)
+        self.proc.terminate()
+        try:
+            self.proc.wait(timeout=5)
+        except Exception:
+            self.proc.kill()
+        self.f.close()
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in open(self.path):
+            parts = [p.strip() for p in line.split(",")]
+            if len(parts) < 10:
+                continue
+            if self.uuid and self.uuid not in parts[1]:
+                continue
+            try:
+                sm.append(float(parts[2]))
+                mx = float(parts[3])
+            except ValueError:
+                continue
+            for nm, v in zip(names, parts[6:10]):
+                if v.lower() == "active":
+                    reasons.add(nm)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# --------------------------------------------------------------------------
+# the GPU arm
+# --------------------------------------------------------------------------
+def gpu_arm(args, wl, rank, world):
+    import torch
+    import paper_2609_00049_gb300 as rq
+    from paper_2609_00049_gb300 import build as rqbuild
+
+    rqbuild.build()
+    dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
+    torch.cuda.set_device(dev)
+    rq.lib()
+    stream = torch.cuda.current_stream()
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        dist.init_process_group("nccl", device_id=dev)
+
+    def barrier():
+        if dist is not None:
+            dist.barrier()
+
+    t_gen = time.time()
+    # ---- inputs: generated on the host (seeded), pinned, then resident on the device
+    host_x, dev_x = {}, {}
+    for name, spec in wl.inputs.items():
+        bits = synth.xhat_full(wl, name, as_bits=True)
+        t = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).pin_memory()
+        host_x[name] = t
+        dev_x[name] = t.to(dev, non_blocking=True)
+    host_w, dev_w, host_f, dev_f = {}, {}, {}, {}
+    for mod in wl.modules:
+        t = torch.from_numpy(synth.weights(wl, mod).view(np.int16)).view(torch.bfloat16).pin_memory()
+        host_w[mod.name] = t
+        dev_w[mod.name] = t.to(dev, non_blocking=True)
+        f = torch.from_numpy(synth.fisher(wl, mod)).pin_memory()
+        host_f[mod.name] = f
+        dev_f[mod.name] = f.to(dev, non_blocking=True)
+    torch.cuda.synchronize()
+    t_gen = time.time() - t_gen
+
+    qcfg = rq.quant_cfg(wl.bits, wl.group_size, wl.block_size, wl.symmetric, wl.damp_frac)
+    B_total = wl.total_column_blocks
+    # ---- state buffers (allocated once)
+    st = {}
+    for name, spec in wl.inputs.items():
+        n = spec.n
+        st[name] = dict(H=torch.empty(n, n, device=dev), U=torch.empty(n, n, device=dev),
+                        Hbar=torch.empty(n, n, device=dev), dead=torch.empty(n, dtype=torch.uint8, device=dev),
+                        pws=rq.workspace(rq.realq_prepare_workspace_size(n), dev),
+                        hws=rq.workspace(rq.realq_hessian_workspace_size(n, spec.T), dev))
+    mods, bstart = {}, 1
+    for mod in wl.modules:
+        m, n = mod.m, mod.n
+        g = wl.group_size or n
+        ng = -(-n // g)
+        nb = -(-n // wl.block_size)
+        bc = rq.bgd_cfg(wl.lr, wl.steps_per_block, b_global_start=bstart, B_total=B_total if wl.sliding_window else 1)
+        bstart += nb
+        mods[mod.name] = dict(
+            W=torch.empty(m, n, device=dev), codes=torch.empty(m, (n + 1) // 2, dtype=torch.uint8, device=dev),
+            scale=torch.empty(m, ng, device=dev), zero=torch.empty(m, ng, dtype=torch.uint8, device=dev),
+            am=torch.empty(m, n, device=dev), av=torch.empty(m, n, device=dev), bcfg=bc,
+            ws=rq.workspace(rq.realq_quantize_workspace_size(m, n, qcfg, bc, False, False), dev))
+    # e2e-only buffers: pinned host outputs, device staging for chunked inputs
+    E2E_CHUNK = 32768
+    stage = {}
+    for name, spec in wl.inputs.items():
+        stage[name] = [torch.empty(E2E_CHUNK, spec.n, dtype=torch.bfloat16, device=dev) for _ in range(2)]
+    host_out = {mod.name: dict(codes=torch.empty_like(mods[mod.name]["codes"], device="cpu").pin_memory(),
+                               scale=torch.empty_like(mods[mod.name]["scale"], device="cpu").pin_memory(),
+                               zero=torch.empty_like(mods[mod.name]["zero"], device="cpu").pin_memory())
+                for mod in wl.modules}
+    copy_stream = torch.cuda.Stream(device=dev)
+
+    def sweep_modules(wsrc, fsrc):
+        for mod in wl.modules:
+            p, s_in = mods[mod.name], st[mod.input]
+            rq.realq_quantize_layer(wsrc[mod.name], s_in["U"], s_in["Hbar"], qcfg, p["W"], p["codes"], p["scale"],
+                                    p["zero"], dead=s_in["dead"], bcfg=p["bcfg"], F=fsrc[mod.name],
+                                    adam_m=p["am"], adam_v=p["av"], ws=p["ws"])
+
+    def step_device():
+        for name, spec in wl.inputs.items():
+            s_in = st[name]
+            s_in["H"].zero_()
+            rq.realq_hessian_accumulate(dev_x[name], s_in["H"], ws=s_in["hws"])
+            rq.realq_hessian_prepare(s_in["H"], spec.T, wl.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
+                                     s_in["pws"])
+        sweep_modules(dev_w, dev_f)
+        for mod in wl.modules:
+            rq.realq_workspace_status(mods[mod.name]["ws"])
+
+    e2e_bytes = {"h2d": 0, "d2h": 0}
+    dev_w_e2e = {k: torch.empty_like(v) for k, v in dev_w.items()}
+    dev_f_e2e = {k: torch.empty_like(v) for k, v in dev_f.items()}
+    e2e_ws = {name: rq.workspace(rq.realq_hessian_workspace_size(spec.n, E2E_CHUNK), dev)
+              for name, spec in wl.inputs.items()}
+
+    def step_e2e():
+        h2d = d2h = 0
+        for mod in wl.modules:
+            dev_w_e2e[mod.name].copy_(host_w[mod.name], non_blocking=True)
+            dev_f_e2e[mod.name].copy_(host_f[mod.name], non_blocking=True)
+            h2d += host_w[mod.name].numel() * 2 + host_f[mod.name].numel() * 4
+        for name, spec in wl.inputs.items():
+            s_in = st[name]
+            s_in["H"].zero_()
+            xs = host_x[name]
+            nch = -(-spec.T // E2E_CHUNK)
+            ev = [None, None]
+            for c in range(nch):
+                buf = stage[name][c % 2]
+                rows = min(E2E_CHUNK, spec.T - c * E2E_CHUNK)
+                with torch.cuda.stream(copy_stream):
+                    if ev[c % 2] is not None:
+                        copy_stream.wait_event(ev[c % 2])
+                    buf[:rows].copy_(xs[c * E2E_CHUNK:c * E2E_CHUNK + rows], non_blocking=True)
+                    done = torch.cuda.Event()
+                    done.record(copy_stream)
+                stream.wait_event(done)
+                rq.realq_hessian_accumulate(buf[:rows], s_in["H"], ws=e2e_ws[name])
+                used = torch.cuda.Event()
+                used.record(stream)
+                ev[c % 2] = used
+                h2d += rows * spec.n * 2
+            rq.realq_hessian_prepare(s_in["H"], spec.T, wl.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
+                                     s_in["pws"])
+        sweep_modules(dev_w_e2e, dev_f_e2e)
+        for mod in wl.modules:
+            p, o = mods[mod.name], host_out[mod.name]
+            for k in ("codes", "scale", "zero"):
+                o[k].copy_(p[k], non_blocking=True)
+                d2h += o[k].numel() * o[k].element_size()
+        for mod in wl.modules:
+            rq.realq_workspace_status(mods[mod.name]["ws"])
+        torch.cuda.current_stream().synchronize()
+        e2e_bytes["h2d"], e2e_bytes["d2h"] = h2d, d2h
+
+    # ---- warm-up
+    for _ in range(args.warmup):
+        step_device()
+    torch.cuda.synchronize()
+    barrier()
+
+    # ---- timed region (device-resident inputs)
+    uuid = None
+    try:
+        uuid = str(torch.cuda.get_device_properties(dev).uuid)
+    except Exception:
+        pass
+    clocks = ClockSampler(uuid)
+    rq.realq_profile_collect()          # drop anything pending
+    rq.realq_profile_enable(True)
+    launches0 = rq.realq_launch_count()
+    clocks.start()
+    torch.cuda.synchronize()
+    barrier()
+    t0 = torch.cuda.Event(enable_timing=True)
+    t1 = torch.cuda.Event(enable_timing=True)
+    t0.record(stream)
+    for _ in range(args.steps):
+        step_device()
+    t1.record(stream)
+    torch.cuda.synchronize()
+    barrier()
+    ms_total = t0.elapsed_time(t1)
+    clk = clocks.stop()
+    launches = rq.realq_launch_count() - launches0
+    rq.realq_profile_enable(False)
+    prof = rq.realq_profile_collect(256)
+    if dist is not None:
+        tt = torch.tensor([ms_total], device=dev)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        ms_total = float(tt.item())
+    cols = wl.total_columns * args.steps * world
+    value = cols / (ms_total / 1e3)
+
+    # ---- end to end through host buffers
+    e2e = None
+    if not args.no_e2e:
+        step_e2e()
+        torch.cuda.synchronize()
+        barrier()
+        e0 = time.perf_counter()
+        a0 = torch.cuda.Event(enable_timing=True)
+        a1 = torch.cuda.Event(enable_timing=True)
+        a0.record(stream)
+        for _ in range(args.steps):
+            step_e2e()
+        a1.record(stream)
+        torch.cuda.synchronize()
+        barrier()
+        e_ms = (time.perf_counter() - e0) * 1e3
+        if dist is not None:
+            tt = torch.tensor([e_ms], device=dev)
+            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+            e_ms = float(tt.item())
+        e2e = {"value": cols / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": e2e_bytes["h2d"],
+               "d2h_bytes_per_step": e2e_bytes["d2h"], "ms_per_step": e_ms / args.steps}
+
+    result = None
+    if rank == 0:
+        peaks = load_peaks()
+        roof = roofline(wl, prof, args.steps, peaks)
+        result = {
+            "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "data": "synthetic (seeded; bf16 weights ~N(0,0.02^2), Gaussian activations with 1% outlier channels x20)",
+            "config": {"workload": wl.name, "description": wl.description, "modules": len(wl.modules),
+                       "calibration_tokens": wl.inputs[wl.modules[0].input].T,
+                       "columns_per_step": wl.total_columns, "column_blocks_per_step": wl.total_column_blocks,
+                       "quantizer": f"W{wl.bits} {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}",
+                       "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}",
+                       "parallelism": f"replicas x{world}",
+                       "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
+                             (sum(s.T * s.n * 2 for s in wl.inputs.values()) / 1e9),
+                       "input_generation_s": round(t_gen, 1)},
+            "roofline": roof, "kernels": {k: {"launches": v[0], "ms": round(v[1], 3)} for k, v in
+                                           sorted(prof.items(), key=lambda kv: -kv[1][1])},
+            "gpu_launches": int(launches), "clocks": clk, "e2e": e2e,
+        }
+    if dist is not None:
+        dist.destroy_process_group()
+    return result
+
+
+def roofline(wl, prof, steps, peaks):
+    """Roofline entry for the kernel with the largest share of device time."""
+    if not prof:
+        return None
+    name, (launches, ms) = max(prof.items(), key=lambda kv: kv[1][1])
+    per_step = {}
+    # algorithmic work per step of each kernel family
+    hess_flops = sum(s.T * s.n * (s.n + 1) for s in wl.inputs.values())       # symmetric X^T X
+    per_step["hessian_syrk_simt"] = ("tensor", hess_flops, "TFLOP/s")
+    per_step["hessian_syrk"] = ("tensor", hess_flops, "TFLOP/s")
+    bgd_p = bgd_g = trail = 0
+    serial_bytes = 0
+    for md in wl.modules:
+        m, n, B = md.m, md.n, wl.block_size
+        for b in range(-(-n // B)):
+            be = min((b + 1) * B, n)
+            r = n - be
+            bgd_p += 2 * m * n * r
+            bgd_g += 2 * m * m * r
+            trail += 2 * m * (be - b * B) * r
+            serial_bytes += m * (be - b * B) * (4 + 4 + 4) + m * (be - b * B) // 2
+    per_step["bgd_p_gemm"] = ("alu", bgd_p, "TFLOP/s")
+    per_step["bgd_g_gemm"] = ("alu", bgd_g, "TFLOP/s")
+    per_step["trailing_update"] = ("alu", trail, "TFLOP/s")
+    per_step["quant_block"] = ("hbm", serial_bytes, "GB/s")
+    if name not in per_step:
+        return {"kernel": name, "bound": None, "achieved": None, "peak": None, "unit": None, "frac": None,
+                "traffic": None, "note": "no algorithmic model for this kernel"}
+    bound, work, unit = per_step[name]
+    secs = ms / 1e3
+    total = work * steps
+    fp32_alu_tflops = 152 * 128 * 2 * peaks["sm_max_mhz"] * 1e6 / 1e12
+    if bound == "tensor":
+        achieved = total / secs / 1e12
+        peak = peaks["bf16_tflops_sustained"]
+        peak_note = f"bf16 dense, sustained, {peaks['source']}"
+    elif bound == "alu":
+        achieved = total / secs / 1e12
+        peak = fp32_alu_tflops
+        peak_note = "fp32 FFMA: 152 SMs x 128 lanes x 2 flop x max SM clock"
+    else:
+        achieved = total / secs / 1e9
+        peak = peaks["hbm_gbs"]
+        peak_note = f"HBM copy, {peaks['source']}"
+    traffic = NCU_TRAFFIC.get(name)
+    return {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
+            "frac": achieved / peak, "traffic": traffic, "peak_source": peak_note,
+            "launches": launches, "avg_launch_ms": ms / launches,
+            "work_per_step": work}
+
+
+# --------------------------------------------------------------------------
+# the CPU oracle (cpu_baseline leg and the reference arm)
+# --------------------------------------------------------------------------
+def oracle_sample(wl, token_sample=8192):
+    """Times the fp64 oracle on module k_proj (or the first module) end to end;
+    the Hessian is accumulated over token_sample tokens and its time scaled to
+    the full token count.  Returns (columns/s, description)."""
+    import oracle
+    mod = next((md for md in wl.modules if md.name == "k_proj"), wl.modules[0])
+    spec = wl.inputs[mod.input]
+    X = synth.xhat_full(wl, mod.input, as_bits=False, max_tokens=min(token_sample, spec.T))
+    W0 = synth.weights(wl, mod, as_bits=False)
+    F = synth.fisher(wl, mod)
+    t0 = time.perf_counter()
+    Hs, T = oracle.hessian_sum([X])
+    t_h = time.perf_counter() - t0
+    scale = spec.T / T
+    t1 = time.perf_counter()
+    oracle.realq_sweep(W0, Hs * scale, spec.T, bits=wl.bits, group_size=wl.group_size, block_size=wl.block_size,
+                       symmetric=bool(wl.symmetric), damp_frac=wl.damp_frac,
+                       bgd={"lr": wl.lr, "steps_per_block": wl.steps_per_block}, F=F, record=False)
+    t_s = time.perf_counter() - t1
+    total = t_h * scale + t_s
+    desc = (f"{mod.name} ({mod.n}->{mod.m}) of {wl.name}: Hessian over {T} of {spec.T} tokens "
+            f"({t_h:.2f} s, scaled x{scale:g}), prepare + sweep with Block-GD {t_s:.2f} s")
+    return mod.n / total, desc, total
+
+
+def cpu_cores():
+    for k in ("OMP_NUM_THREADS", "OPENBLAS_NUM_THREADS"):
+        if os.environ.get(k):
+            return int(os.environ[k])
+    try:
+        from threadpoolctl import threadpool_info
+        n = [i.get("num_threads") for i in threadpool_info() if i.get("user_api") == "blas"]
+        if n:
+            return int(n[0])
+    except Exception:
+        pass
+    return os.cpu_count()
+
+
+def reference_arm(args, wl, rank, world):
+    if rank != 0:
+        return None
+    vals, descs, secs = [], None, []
+    for _ in range(max(0, min(args.warmup, 1))):
+        oracle_sample(wl)
+    for _ in range(args.steps):
+        v, descs, s = oracle_sample(wl)
+        vals.append(v)
+        secs.append(s)
+    value = statistics.mean(vals)
+    cb = {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": descs}
+    return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(secs),
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": {"workload": wl.name, "description": wl.description}, "cpu_baseline": cb,
+            "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=10)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
+    ap.add_argument("--workload", default="qwen3-0.6b")
+    ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    args = ap.parse_args()
+    rank = int(os.environ.get("RANK", 0))
+    world = int(os.environ.get("WORLD_SIZE", 1))
+    wl = synth.workloads()[args.workload]
+    if args.impl == "reference":
+        res = reference_arm(args, wl, rank, world)
+    else:
+        res = gpu_arm(args, wl, rank, world)
+        if res is not None and rank == 0 and world == 1 and not args.no_cpu_baseline:
+            v, desc, _ = oracle_sample(wl)
+            res["cpu_baseline"] = {"value": v, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": desc}
+        elif res is not None:
+            res["cpu_baseline"] = None
+    if rank == 0 and res is not None:
+        print(json.dumps(res))
+
+
+if __name__ == "__main__":
+    main()

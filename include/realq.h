@@ -1,0 +1,225 @@
+/*
+ * realq.h - C ABI of the GB300 (sm_103a) REAL-Q per-layer quantization sweep.
+ *
+ * The library quantizes one linear module W (m x n, out x in, row-major) to
+ * b-bit integer codes with per-group scale and zero point.  The sweep is the
+ * per-module part of Algorithm 1 of "REAL-Q: E2E LLM Quantization via Dynamic
+ * Gradient Descent":
+ *   1. accumulate the input second moment H = sum_t x̂_t x̂_t^T of the perturbed
+ *      calibration inputs (Sec. 3.2, "GPTQ Recap");
+ *   2. damp H and form the upper Cholesky factor U of H^-1 (Alg. 1, "compute
+ *      ... H_g and its inverse");
+ *   3. sweep the columns in blocks of B: quantize each column and feed its error
+ *      back into the later columns of the block (Eq. gptq_update), then apply
+ *      the batched update to all columns after the block (Sec. 3.2);
+ *   4. after every block take one Adam step on the columns after the block,
+ *      descending the aggregated-Fisher surrogate (Eq. fisher_loss,
+ *      Eq. block_gd_update), optionally blended with the next transformer
+ *      block's Fisher (Eq. slide_window).
+ *
+ * Conventions shared by every entry point
+ *   - Pointers are DEVICE pointers unless marked (host).  Matrices are dense,
+ *     row-major, without padding (leading dimension = number of columns).
+ *   - The caller owns every buffer; the library allocates no device memory.
+ *     Scratch comes from a caller-provided workspace whose size is returned by
+ *     the matching *_workspace_size function (256-byte aligned pointer).
+ *   - All work is enqueued on `stream` (a cudaStream_t passed as void*; NULL
+ *     is the legacy default stream).  Calls are asynchronous unless stated.
+ *   - Argument errors are detected on the host before anything is enqueued and
+ *     leave every buffer untouched: REALQ_ERR_INVALID_ARG /
+ *     REALQ_ERR_WORKSPACE / REALQ_ERR_UNSUPPORTED.  realq_last_error() gives a
+ *     thread-local description of the last failure.
+ *   - No exception crosses the ABI.  The library keeps no per-call state
+ *     besides the thread-local error string and the optional profiling
+ *     counters.
+ */
+#ifndef REALQ_H
+#define REALQ_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef void *realq_stream_t; /* cudaStream_t */
+
+typedef enum {
+    REALQ_OK = 0,
+    REALQ_ERR_INVALID_ARG = 1, /* null pointer, bad size or bad config value */
+    REALQ_ERR_WORKSPACE = 2,   /* workspace missing, too small or misaligned */
+    REALQ_ERR_NOT_SPD = 3,     /* damped Hessian not positive definite (prepare) */
+    REALQ_ERR_NONFINITE = 4,   /* NaN/Inf met in the weights during the sweep */
+    REALQ_ERR_TIMEOUT = 5,     /* a bounded device-side wait gave up */
+    REALQ_ERR_CUDA = 6,        /* a CUDA runtime call or launch failed */
+    REALQ_ERR_UNSUPPORTED = 7  /* valid but not implemented combination */
+} realq_status_t;
+
+typedef enum { REALQ_F32 = 0, REALQ_BF16 = 1 } realq_dtype_t;
+
+/* Quantizer and sweep geometry.
+ *   bits        2..4 (codes are stored as 4-bit nibbles).
+ *   group_size  columns sharing one (scale, zero) per row; 0 = one group per
+ *               row.  Must divide block_size or be a multiple of it.
+ *   block_size  column block B of the sweep: 32, 64 or 128 (paper: 128).
+ *   symmetric   0: asymmetric min/max grid containing 0 with an integer zero
+ *               point; 1: symmetric grid, zero = 2^(bits-1).
+ *   damp_frac   lambda = damp_frac * mean(diag(H̄)) is added to the diagonal. */
+typedef struct {
+    int bits;
+    int group_size;
+    int block_size;
+    int symmetric;
+    float damp_frac;
+} realq_quant_cfg_t;
+
+enum { REALQ_OPT_ADAM = 0, REALQ_OPT_SGD = 1 };
+
+/* Block-wise gradient descent (Sec. 4.3, App. "Full Setup").
+ *   steps_per_block  optimizer steps after each column block (paper: 1; 0
+ *                    turns Block-GD off and the sweep is plain GPTQ).
+ *   optimizer        REALQ_OPT_ADAM (paper) or REALQ_OPT_SGD.
+ *   lr, beta1, beta2, eps   paper: lr per model, 0.9, 0.999, 1e-8.
+ *   b_global_start   1-based cumulative column-block index of this module's
+ *                    first block within the transformer block (Eq. slide_window).
+ *   B_total          column-block steps of the whole transformer block; with
+ *                    B_total > 1 and F_next given, the Fisher used after block
+ *                    b is alpha F + (1 - alpha) F_next,
+ *                    alpha = 1 - (b_global - 1) / (B_total - 1). */
+typedef struct {
+    int steps_per_block;
+    int optimizer;
+    float lr;
+    float beta1;
+    float beta2;
+    float eps;
+    int b_global_start;
+    int B_total;
+} realq_bgd_cfg_t;
+
+/* ------------------------------------------------------------------------ */
+/* Step 1. Hessian accumulation (Sec. 3.2: H is the second moment of the
+ * calibration inputs; REAL-Q uses the perturbed inputs x̂).
+ *   H_sum += X̂^T X̂                      (n x n fp32, full symmetric matrix)
+ *   D_sum += (X̂ - X)^T X̂   if X_fp != NULL (n x n fp32; D_sum[i][j] =
+ *            sum_t (x̂_ti - x_ti) x̂_tj), needed by the surrogate when the
+ *            reference output W0 x uses unperturbed inputs.
+ * X_hat, X_fp: T_chunk x n, token-major, dtype x_dtype.  T_chunk = 0 is a
+ * no-op.  Call once per chunk of calibration tokens; the caller zeroes H_sum
+ * (and D_sum) before the first chunk and keeps the token count. Asynchronous.
+ * x_dtype = REALQ_BF16: products are exact in fp32, sums are fp32. */
+realq_status_t realq_hessian_accumulate(realq_stream_t stream, int64_t n, int64_t T_chunk,
+                                        const void *X_hat, const void *X_fp, realq_dtype_t x_dtype,
+                                        float *H_sum, float *D_sum, void *ws, size_t ws_bytes);
+/* Workspace for one accumulate call (token-split partial sums, reduced in a
+ * fixed order so results are bitwise repeatable); 0 means ws may be NULL. */
+size_t realq_hessian_workspace_size(int64_t n, int64_t T_chunk, realq_dtype_t x_dtype, int has_X_fp);
+
+/* Step 2. Preparation (Alg. 1: Hessian and its inverse; the inverse used by
+ * the column step is the Cholesky factorisation of H^-1, whose rows equal the
+ * Schur-complement-downdated rows of H^-1 used by Eq. gptq_update).
+ *   Hbar_out = H_sum / T_total                       (n x n, undamped)
+ *   dead_out[j] = (H_sum[j][j] == 0)                 (n bytes; channel never fires)
+ *   Hd = Hbar with Hd[j][j] = 1 on dead channels, plus lambda I,
+ *        lambda = damp_frac * mean(diag(Hd before damping))
+ *   U_out: upper triangular, Hd^-1 = U^T U           (n x n; strictly lower part = 0)
+ * H_sum must be symmetric.  Hbar_out may alias H_sum (in-place).  This call
+ * SYNCHRONIZES `stream` once to read the factorisation status: if a pivot is
+ * not positive it returns REALQ_ERR_NOT_SPD and *fail_col (host) holds the
+ * column, else *fail_col = -1.  Outputs are unspecified after NOT_SPD. */
+realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                     const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                     int64_t *fail_col, void *ws, size_t ws_bytes);
+size_t realq_prepare_workspace_size(int64_t n);
+
+/* Dbar = D_sum / T_total (n x n); may alias D_sum.  Asynchronous. */
+realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum,
+                                  float *Dbar);
+
+/* Steps 3-4. The column sweep with Block-GD for one module (Alg. 1, loop over
+ * blocks b; Eq. gptq_update inside the block, the lazy batch update after it,
+ * Eq. block_gd_update on the remaining columns).
+ *   W0        m x n, original weights (w_dtype); also the surrogate's reference.
+ *   U         n x n from realq_hessian_prepare; Hbar the undamped H / T.
+ *   Dbar      n x n or NULL (X = X̂): the gradient is
+ *             F_eff [ (Ŵ - W0) Hbar + W0 Dbar ] restricted to the free columns.
+ *   dead      n bytes from prepare, or NULL (no dead channels).
+ *   bcfg      NULL or steps_per_block = 0: plain GPTQ sweep (F, adam_* unused).
+ *   F         m x m symmetric Fisher of the module-output space; F_next the
+ *             next transformer block's (NULL: no sliding window).
+ *   W_work    m x n fp32 state.  On a sweep starting at block 0 it is
+ *             initialised from W0 (dead channels zeroed); on return its columns
+ *             < min(block_end*B, n) hold the dequantized weights.
+ *   adam_m, adam_v  m x n fp32 Adam moments (zeroed at block 0); adam_t (host)
+ *             step counter in/out (set to 0 at block 0).
+ *   codes     m x ceil(n/2) bytes, two codes per byte, even column in the low
+ *             nibble.  scale (fp32) and zero (uint8): m x ngroups, ngroups =
+ *             ceil(n / group_size) (1 when group_size = 0).
+ *   W_deq     optional m x n copy of the dequantized weights in deq_dtype
+ *             (written for the processed columns), or NULL.
+ *   block_begin, block_end  blocks [block_begin, block_end) of the
+ *             ceil(n / B) blocks are processed; a sweep interrupted after block k
+ *             resumes with block_begin = k + 1 and the same state buffers.
+ * Asynchronous.  A NaN/Inf weight met by the column step is recorded in the
+ * workspace status word, read by realq_workspace_status(). */
+realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
+                                    const void *W0, realq_dtype_t w_dtype,
+                                    const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
+                                    const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg,
+                                    const float *F, const float *F_next,
+                                    float *W_work, float *adam_m, float *adam_v, int64_t *adam_t,
+                                    uint8_t *codes, float *scale, uint8_t *zero,
+                                    void *W_deq, realq_dtype_t deq_dtype,
+                                    int64_t block_begin, int64_t block_end,
+                                    void *ws, size_t ws_bytes);
+size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg_t *qcfg,
+                                     const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar);
+
+/* Step 4 alone: bcfg->steps_per_block optimizer steps of Eq. block_gd_update
+ * on the columns col_start..n-1 of W (columns < col_start are locked; they
+ * hold dequantized values).  alpha blends F and F_next (ignored when F_next is
+ * NULL).  adam_t (host) is advanced by the number of steps.  Asynchronous. */
+realq_status_t realq_bgd_refine(realq_stream_t stream, int64_t m, int64_t n, int64_t col_start,
+                                float *W, const void *W0, realq_dtype_t w_dtype,
+                                const float *Hbar, const float *Dbar,
+                                const float *F, const float *F_next, float alpha,
+                                float *adam_m, float *adam_v, int64_t *adam_t,
+                                const realq_bgd_cfg_t *bcfg, void *ws, size_t ws_bytes);
+size_t realq_bgd_workspace_size(int64_t m, int64_t n, int has_F_next, int has_Dbar);
+
+/* Surrogate of Eq. fisher_loss at the layer level with X = X̂:
+ *   *loss_out (device fp32) = 1/2 tr(F (W_hat - W0) Hbar (W_hat - W0)^T).
+ * Asynchronous. */
+realq_status_t realq_surrogate_loss(realq_stream_t stream, int64_t m, int64_t n,
+                                    const float *W_hat, const void *W0, realq_dtype_t w_dtype,
+                                    const float *Hbar, const float *F, float *loss_out,
+                                    void *ws, size_t ws_bytes);
+size_t realq_surrogate_workspace_size(int64_t m, int64_t n);
+
+/* Synchronizes `stream`, returns the device status word recorded in a
+ * quantize workspace (REALQ_OK, REALQ_ERR_NONFINITE) and clears it. */
+realq_status_t realq_workspace_status(realq_stream_t stream, void *ws, size_t ws_bytes);
+
+/* Diagnostics. */
+const char *realq_status_string(realq_status_t s);
+const char *realq_last_error(void);
+
+/* Launch accounting and per-kernel timing.
+ * realq_launch_count(): number of kernels this library has launched since load.
+ * With profiling on, every launch is bracketed by CUDA events recorded on its
+ * own stream; realq_profile_collect synchronizes those events, writes up to
+ * max_entries per-kernel totals and clears them. */
+typedef struct {
+    char name[48];
+    int64_t launches;
+    double total_ms;
+} realq_kernel_stat_t;
+int64_t realq_launch_count(void);
+void realq_profile_enable(int on);
+int realq_profile_collect(realq_kernel_stat_t *out, int max_entries);
+
+#ifdef __cplusplus
+}
+#endif
+#endif /* REALQ_H */

@@ -1,0 +1,292 @@
+"""Python binding of librealq.so, the GB300 (sm_103a) REAL-Q per-layer sweep.
+
+Every function here marshals torch tensors (device memory, current stream)
+into the C ABI declared in include/realq.h and calls it; all computation runs
+in the library's CUDA kernels.  There is no CPU fallback: if the library is
+missing, importing the binding works but every call raises.
+
+Names match the C entry points.  Errors come back as RealqError carrying the
+status code and the library's message.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+from typing import Optional
+
+import torch
+
+__all__ = [
+    "RealqError", "QuantCfg", "BgdCfg", "lib", "library_path", "quant_cfg", "bgd_cfg", "workspace",
+    "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
+    "realq_prepare_workspace_size", "realq_scale_moment", "realq_quantize_layer",
+    "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
+    "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
+    "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
+    "realq_profile_collect",
+]
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+library_path = os.path.join(_HERE, "_lib", "librealq.so")
+
+REALQ_OK, REALQ_ERR_INVALID_ARG, REALQ_ERR_WORKSPACE, REALQ_ERR_NOT_SPD = 0, 1, 2, 3
+REALQ_ERR_NONFINITE, REALQ_ERR_TIMEOUT, REALQ_ERR_CUDA, REALQ_ERR_UNSUPPORTED = 4, 5, 6, 7
+REALQ_F32, REALQ_BF16 = 0, 1
+REALQ_OPT_ADAM, REALQ_OPT_SGD = 0, 1
+
+
+class RealqError(RuntimeError):
+    def __init__(self, status: int, message: str, **extra):
+        super().__init__(f"realq status {status}: {message}")
+        self.status = status
+        self.message = message
+        for k, v in extra.items():
+            setattr(self, k, v)
+
+
+class QuantCfg(ctypes.Structure):
+    _fields_ = [("bits", ctypes.c_int), ("group_size", ctypes.c_int), ("block_size", ctypes.c_int),
+                ("symmetric", ctypes.c_int), ("damp_frac", ctypes.c_float)]
+
+
+class BgdCfg(ctypes.Structure):
+    _fields_ = [("steps_per_block", ctypes.c_int), ("optimizer", ctypes.c_int), ("lr", ctypes.c_float),
+                ("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
+                ("b_global_start", ctypes.c_int), ("B_total", ctypes.c_int)]
+
+
+class KernelStat(ctypes.Structure):
+    _fields_ = [("name", ctypes.c_char * 48), ("launches", ctypes.c_int64), ("total_ms", ctypes.c_double)]
+
+
+def quant_cfg(bits=4, group_size=128, block_size=128, symmetric=0, damp_frac=0.01) -> QuantCfg:
+    return QuantCfg(bits, group_size, block_size, int(symmetric), damp_frac)
+
+
+def bgd_cfg(lr, steps_per_block=1, optimizer=REALQ_OPT_ADAM, beta1=0.9, beta2=0.999, eps=1e-8,
+            b_global_start=1, B_total=1) -> BgdCfg:
+    return BgdCfg(steps_per_block, optimizer, lr, beta1, beta2, eps, b_global_start, B_total)
+
+
+_lib = None
+_vp, _i64, _sz, _int, _f32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t, ctypes.c_int, ctypes.c_float
+_P_i64 = ctypes.POINTER(ctypes.c_int64)
+_SIGS = {
+    "realq_hessian_accumulate": ([_vp, _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _sz], _int),
+    "realq_hessian_workspace_size": ([_i64, _i64, _int, _int], _sz),
+    "realq_hessian_prepare": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
+    "realq_prepare_workspace_size": ([_i64], _sz),
+    "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
+    "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
+                              ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
+                              _i64, _i64, _vp, _sz], _int),
+    "realq_quantize_workspace_size": ([_i64, _i64, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _int, _int],
+                                      _sz),
+    "realq_bgd_refine": ([_vp, _i64, _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _vp, _f32, _vp, _vp, _P_i64,
+                          ctypes.POINTER(BgdCfg), _vp, _sz], _int),
+    "realq_bgd_workspace_size": ([_i64, _i64, _int, _int], _sz),
+    "realq_surrogate_loss": ([_vp, _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _vp, _sz], _int),
+    "realq_surrogate_workspace_size": ([_i64, _i64], _sz),
+    "realq_workspace_status": ([_vp, _vp, _sz], _int),
+    "realq_status_string": ([_int], ctypes.c_char_p),
+    "realq_last_error": ([], ctypes.c_char_p),
+    "realq_launch_count": ([], _i64),
+    "realq_profile_enable": ([_int], None),
+    "realq_profile_collect": ([ctypes.POINTER(KernelStat), _int], _int),
+}
+
+
+def lib():
+    """The loaded CUDA library (raises if it has not been built)."""
+    global _lib
+    if _lib is None:
+        if not os.path.exists(library_path):
+            raise RuntimeError(f"{library_path} is missing: build it with paper_2609_00049_gb300.build.build() "
+                               "(the CUDA library is required; there is no CPU fallback)")
+        L = ctypes.CDLL(library_path)
+        for name, (args, res) in _SIGS.items():
+            fn = getattr(L, name)
+            fn.argtypes = args
+            fn.restype = res
+        _lib = L
+    return _lib
+
+
+def _check(status: int, **extra):
+    if status != REALQ_OK:
+        raise RealqError(status, lib().realq_last_error().decode(errors="replace"), **extra)
+
+
+def _ptr(t: Optional[torch.Tensor]):
+    if t is None:
+        return None
+    if not t.is_cuda:
+        raise ValueError("expected a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError("expected a contiguous tensor")
+    return ctypes.c_void_p(t.data_ptr())
+
+
+def _dtype(t: torch.Tensor) -> int:
+    if t.dtype == torch.float32:
+        return REALQ_F32
+    if t.dtype == torch.bfloat16:
+        return REALQ_BF16
+    raise ValueError(f"unsupported dtype {t.dtype}")
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    s = torch.cuda.current_stream() if stream is None else stream
+    return ctypes.c_void_p(s.cuda_stream)
+
+
+def _need(t, dtype, shape, name):
+    if t is None:
+        return
+    if t.dtype != dtype or tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name}: expected {dtype} {tuple(shape)}, got {t.dtype} {tuple(t.shape)}")
+
+
+def workspace(nbytes: int, device=None) -> Optional[torch.Tensor]:
+    """Caller-owned workspace buffer (torch allocations are >= 256-byte aligned)."""
+    if nbytes == 0:
+        return None
+    return torch.empty(int(nbytes), dtype=torch.uint8, device=device or "cuda")
+
+
+def _ws(ws):
+    return (None, 0) if ws is None else (_ptr(ws), ws.numel())
+
+
+# ----------------------------------------------------------------- Hessian ---
+def realq_hessian_workspace_size(n: int, T_chunk: int, x_dtype: int = REALQ_BF16, has_X_fp: bool = False) -> int:
+    return int(lib().realq_hessian_workspace_size(n, T_chunk, x_dtype, int(has_X_fp)))
+
+
+def realq_hessian_accumulate(X_hat: torch.Tensor, H_sum: torch.Tensor, D_sum: Optional[torch.Tensor] = None,
+                             X_fp: Optional[torch.Tensor] = None, ws: Optional[torch.Tensor] = None, stream=None):
+    T, n = X_hat.shape
+    _need(H_sum, torch.float32, (n, n), "H_sum")
+    _need(D_sum, torch.float32, (n, n), "D_sum")
+    if X_fp is not None and (X_fp.dtype != X_hat.dtype or X_fp.shape != X_hat.shape):
+        raise ValueError("X_fp must match X_hat")
+    wp, wb = _ws(ws)
+    _check(lib().realq_hessian_accumulate(_stream(stream), n, T, _ptr(X_hat), _ptr(X_fp), _dtype(X_hat),
+                                          _ptr(H_sum), _ptr(D_sum), wp, wb))
+
+
+# ----------------------------------------------------------------- prepare ---
+def realq_prepare_workspace_size(n: int) -> int:
+    return int(lib().realq_prepare_workspace_size(n))
+
+
+def realq_hessian_prepare(H_sum: torch.Tensor, T_total: int, damp_frac: float, U_out: torch.Tensor,
+                          Hbar_out: Optional[torch.Tensor], dead_out: torch.Tensor, ws: torch.Tensor,
+                          stream=None) -> int:
+    """Returns -1; raises RealqError(status=NOT_SPD, fail_col=j) on a failed pivot."""
+    n = H_sum.shape[0]
+    _need(U_out, torch.float32, (n, n), "U_out")
+    _need(Hbar_out, torch.float32, (n, n), "Hbar_out")
+    _need(dead_out, torch.uint8, (n,), "dead_out")
+    fc = ctypes.c_int64(-1)
+    wp, wb = _ws(ws)
+    st = lib().realq_hessian_prepare(_stream(stream), n, int(T_total), float(damp_frac), _ptr(H_sum), _ptr(U_out),
+                                     _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc), wp, wb)
+    _check(st, fail_col=fc.value)
+    return fc.value
+
+
+def realq_scale_moment(D_sum: torch.Tensor, T_total: int, Dbar: torch.Tensor, stream=None):
+    n = D_sum.shape[0]
+    _check(lib().realq_scale_moment(_stream(stream), n, int(T_total), _ptr(D_sum), _ptr(Dbar)))
+
+
+# ------------------------------------------------------------------- sweep ---
+def realq_quantize_workspace_size(m: int, n: int, qcfg: QuantCfg, bcfg: Optional[BgdCfg] = None,
+                                  has_F_next: bool = False, has_Dbar: bool = False) -> int:
+    return int(lib().realq_quantize_workspace_size(m, n, ctypes.byref(qcfg),
+                                                   ctypes.byref(bcfg) if bcfg is not None else None,
+                                                   int(has_F_next), int(has_Dbar)))
+
+
+def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch.Tensor], qcfg: QuantCfg,
+                         W_work: torch.Tensor, codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *,
+                         Dbar=None, dead=None, bcfg: Optional[BgdCfg] = None, F=None, F_next=None,
+                         adam_m=None, adam_v=None, adam_t: int = 0, W_deq=None,
+                         block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None) -> int:
+    """Runs blocks [block_begin, block_end) of the sweep; returns the Adam step counter."""
+    m, n = W0.shape
+    nb = -(-n // qcfg.block_size)
+    if block_end is None:
+        block_end = nb
+    _need(W_work, torch.float32, (m, n), "W_work")
+    _need(U, torch.float32, (n, n), "U")
+    _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
+    _need(adam_m, torch.float32, (m, n), "adam_m")
+    _need(adam_v, torch.float32, (m, n), "adam_v")
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    _check(lib().realq_quantize_layer(
+        _stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar), _ptr(Dbar), _ptr(dead),
+        ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
+        _ptr(W_work), _ptr(adam_m), _ptr(adam_v), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
+        _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
+    return t.value
+
+
+def realq_bgd_workspace_size(m: int, n: int, has_F_next: bool = False, has_Dbar: bool = False) -> int:
+    return int(lib().realq_bgd_workspace_size(m, n, int(has_F_next), int(has_Dbar)))
+
+
+def realq_bgd_refine(W: torch.Tensor, W0: torch.Tensor, col_start: int, Hbar: torch.Tensor, F: torch.Tensor,
+                     bcfg: BgdCfg, *, Dbar=None, F_next=None, alpha: float = 1.0, adam_m=None, adam_v=None,
+                     adam_t: int = 0, ws=None, stream=None) -> int:
+    m, n = W.shape
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    _check(lib().realq_bgd_refine(_stream(stream), m, n, int(col_start), _ptr(W), _ptr(W0), _dtype(W0), _ptr(Hbar),
+                                  _ptr(Dbar), _ptr(F), _ptr(F_next), float(alpha), _ptr(adam_m), _ptr(adam_v),
+                                  ctypes.byref(t), ctypes.byref(bcfg), wp, wb))
+    return t.value
+
+
+def realq_surrogate_workspace_size(m: int, n: int) -> int:
+    return int(lib().realq_surrogate_workspace_size(m, n))
+
+
+def realq_surrogate_loss(W_hat: torch.Tensor, W0: torch.Tensor, Hbar: torch.Tensor, F: torch.Tensor,
+                         loss_out: torch.Tensor, ws: torch.Tensor, stream=None):
+    m, n = W_hat.shape
+    wp, wb = _ws(ws)
+    _check(lib().realq_surrogate_loss(_stream(stream), m, n, _ptr(W_hat), _ptr(W0), _dtype(W0), _ptr(Hbar), _ptr(F),
+                                      _ptr(loss_out), wp, wb))
+
+
+def realq_workspace_status(ws: torch.Tensor, stream=None) -> int:
+    """Synchronizes; raises RealqError if the sweep recorded a non-finite weight."""
+    wp, wb = _ws(ws)
+    _check(lib().realq_workspace_status(_stream(stream), wp, wb))
+    return REALQ_OK
+
+
+def realq_status_string(status: int) -> str:
+    return lib().realq_status_string(status).decode()
+
+
+def realq_last_error() -> str:
+    return lib().realq_last_error().decode(errors="replace")
+
+
+def realq_launch_count() -> int:
+    return int(lib().realq_launch_count())
+
+
+def realq_profile_enable(on: bool = True):
+    lib().realq_profile_enable(int(on))
+
+
+def realq_profile_collect(max_entries: int = 64) -> dict:
+    """{kernel name: (launches, total_ms)} since the last collect (synchronizes the recorded events)."""
+    arr = (KernelStat * max_entries)()
+    k = lib().realq_profile_collect(arr, max_entries)
+    return {arr[i].name.decode(): (int(arr[i].launches), float(arr[i].total_ms)) for i in range(k)}

@@ -1,0 +1,347 @@
+// C ABI of the library (include/realq.h): argument validation, workspace
+// checks, sequencing of the kernels of one call, error reporting, launch
+// accounting and optional per-kernel event timing.
+#include "kernels.cuh"
+
+#include <atomic>
+#include <cmath>
+#include <cstdarg>
+#include <cstdio>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <string>
+#include <vector>
+
+namespace realq {
+
+// ------------------------------------------------------------ error text ---
+static thread_local char g_err[512] = "";
+
+void set_error(const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+}
+
+realq_status_t fail(realq_status_t s, const char *fmt, ...) {
+    va_list ap;
+    va_start(ap, fmt);
+    vsnprintf(g_err, sizeof(g_err), fmt, ap);
+    va_end(ap);
+    return s;
+}
+
+realq_status_t check_launch(const char *what) {
+    cudaError_t e = cudaGetLastError();
+    if (e != cudaSuccess) return fail(REALQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+    return REALQ_OK;
+}
+
+// ------------------------------------------------------ launch accounting ---
+static std::atomic<int64_t> g_launches{0};
+static std::atomic<int> g_prof_on{0};
+struct ProfRec {
+    const char *name;
+    cudaEvent_t a, b;
+};
+static std::mutex g_prof_mu;
+static std::vector<ProfRec> g_pending;
+static std::vector<cudaEvent_t> g_pool;
+
+static cudaEvent_t pool_get() {
+    if (!g_pool.empty()) {
+        cudaEvent_t e = g_pool.back();
+        g_pool.pop_back();
+        return e;
+    }
+    cudaEvent_t e = nullptr;
+    if (cudaEventCreate(&e) != cudaSuccess) return nullptr;
+    return e;
+}
+
+Launch::Launch(const char *n, cudaStream_t s) : name(n), stream(s), slot(-1) {
+    g_launches.fetch_add(1, std::memory_order_relaxed);
+    if (!g_prof_on.load(std::memory_order_relaxed)) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    ProfRec r{n, pool_get(), pool_get()};
+    if (!r.a || !r.b) return;
+    cudaEventRecord(r.a, s);
+    g_pending.push_back(r);
+    slot = (int)g_pending.size() - 1;
+}
+
+Launch::~Launch() {
+    if (slot < 0) return;
+    std::lock_guard<std::mutex> lk(g_prof_mu);
+    if (slot < (int)g_pending.size()) cudaEventRecord(g_pending[slot].b, stream);
+}
+
+}  // namespace realq
+
+using namespace realq;
+
+namespace {
+
+cudaStream_t S(realq_stream_t s) { return static_cast<cudaStream_t>(s); }
+
+realq_status_t check_ws(void *ws, size_t have, size_t need, const char *who) {
+    if (need == 0) return REALQ_OK;
+    if (ws == nullptr) return fail(REALQ_ERR_WORKSPACE, "%s: workspace of %zu bytes required", who, need);
+    if (reinterpret_cast<uintptr_t>(ws) % kAlign != 0)
+        return fail(REALQ_ERR_WORKSPACE, "%s: workspace must be %zu-byte aligned", who, kAlign);
+    if (have < need) return fail(REALQ_ERR_WORKSPACE, "%s: workspace %zu < %zu bytes", who, have, need);
+    return REALQ_OK;
+}
+
+bool valid_dtype(realq_dtype_t d) { return d == REALQ_F32 || d == REALQ_BF16; }
+
+realq_status_t check_qcfg(const realq_quant_cfg_t *q, int64_t n) {
+    if (!q) return fail(REALQ_ERR_INVALID_ARG, "qcfg is NULL");
+    if (q->bits < 2 || q->bits > 4) return fail(REALQ_ERR_INVALID_ARG, "bits must be in [2, 4] (got %d)", q->bits);
+    if (q->block_size != 32 && q->block_size != 64 && q->block_size != 128)
+        return fail(REALQ_ERR_INVALID_ARG, "block_size must be 32, 64 or 128 (got %d)", q->block_size);
+    if (q->group_size < 0) return fail(REALQ_ERR_INVALID_ARG, "group_size must be >= 0");
+    if (q->symmetric != 0 && q->symmetric != 1) return fail(REALQ_ERR_INVALID_ARG, "symmetric must be 0 or 1");
+    if (!(q->damp_frac >= 0.f) || !std::isfinite(q->damp_frac)) return fail(REALQ_ERR_INVALID_ARG, "damp_frac must be >= 0");
+    const int B = q->block_size;
+    const int g = q->group_size == 0 ? (int)std::min<int64_t>(n, 1 << 30) : q->group_size;
+    if (q->group_size != 0) {
+        if (g <= B) {
+            if (B % g != 0 || (g != B && g != B / 2 && g != B / 4) || g < 32)
+                return fail(REALQ_ERR_UNSUPPORTED, "group_size %d inside block %d (supported: B, B/2, B/4, >= 32)", g, B);
+        } else if (g % B != 0) {
+            return fail(REALQ_ERR_INVALID_ARG, "group_size %d must be a multiple of block_size %d", g, B);
+        }
+    }
+    return REALQ_OK;
+}
+
+realq_status_t check_bcfg(const realq_bgd_cfg_t *b) {
+    if (!b) return REALQ_OK;
+    if (b->steps_per_block < 0) return fail(REALQ_ERR_INVALID_ARG, "steps_per_block must be >= 0");
+    if (b->optimizer != REALQ_OPT_ADAM && b->optimizer != REALQ_OPT_SGD)
+        return fail(REALQ_ERR_INVALID_ARG, "optimizer must be REALQ_OPT_ADAM or REALQ_OPT_SGD");
+    if (!std::isfinite(b->lr) || b->lr < 0.f) return fail(REALQ_ERR_INVALID_ARG, "lr must be finite and >= 0");
+    if (b->optimizer == REALQ_OPT_ADAM) {
+        if (!(b->beta1 >= 0.f && b->beta1 < 1.f) || !(b->beta2 >= 0.f && b->beta2 < 1.f))
+            return fail(REALQ_ERR_INVALID_ARG, "betas must be in [0, 1)");
+        if (!(b->eps > 0.f)) return fail(REALQ_ERR_INVALID_ARG, "eps must be > 0");
+    }
+    if (b->b_global_start < 1 || b->B_total < 1) return fail(REALQ_ERR_INVALID_ARG, "b_global_start and B_total must be >= 1");
+    return REALQ_OK;
+}
+
+int effective_group(const realq_quant_cfg_t *q, int64_t n) {
+    return q->group_size == 0 ? (int)n : q->group_size;
+}
+
+}  // namespace
+
+extern "C" {
+
+const char *realq_status_string(realq_status_t s) {
+    switch (s) {
+        case REALQ_OK: return "ok";
+        case REALQ_ERR_INVALID_ARG: return "invalid argument";
+        case REALQ_ERR_WORKSPACE: return "workspace missing, too small or misaligned";
+        case REALQ_ERR_NOT_SPD: return "damped Hessian not positive definite";
+        case REALQ_ERR_NONFINITE: return "non-finite value in the weights";
+        case REALQ_ERR_TIMEOUT: return "bounded device wait timed out";
+        case REALQ_ERR_CUDA: return "CUDA error";
+        case REALQ_ERR_UNSUPPORTED: return "unsupported configuration";
+    }
+    return "unknown status";
+}
+
+const char *realq_last_error(void) { return g_err; }
+
+int64_t realq_launch_count(void) { return g_launches.load(); }
+
+void realq_profile_enable(int on) { g_prof_on.store(on ? 1 : 0); }
+
+int realq_profile_collect(realq_kernel_stat_t *out, int max_entries) {
+    std::vector<ProfRec> recs;
+    {
+        std::lock_guard<std::mutex> lk(g_prof_mu);
+        recs.swap(g_pending);
+    }
+    std::map<std::string, std::pair<int64_t, double>> acc;
+    for (auto &r : recs) {
+        float ms = 0.f;
+        if (cudaEventSynchronize(r.b) == cudaSuccess && cudaEventElapsedTime(&ms, r.a, r.b) == cudaSuccess) {
+            auto &e = acc[r.name];
+            e.first += 1;
+            e.second += ms;
+        }
+    }
+    {
+        std::lock_guard<std::mutex> lk(g_prof_mu);
+        for (auto &r : recs) {
+            g_pool.push_back(r.a);
+            g_pool.push_back(r.b);
+        }
+    }
+    int k = 0;
+    for (auto &kv : acc) {
+        if (k >= max_entries || out == nullptr) break;
+        std::memset(out[k].name, 0, sizeof(out[k].name));
+        std::strncpy(out[k].name, kv.first.c_str(), sizeof(out[k].name) - 1);
+        out[k].launches = kv.second.first;
+        out[k].total_ms = kv.second.second;
+        ++k;
+    }
+    return k;
+}
+
+// -------------------------------------------------------------- Hessian ---
+size_t realq_hessian_workspace_size(int64_t n, int64_t T_chunk, realq_dtype_t x_dtype, int has_X_fp) {
+    (void)x_dtype;
+    if (n <= 0 || T_chunk <= 0) return 0;
+    return hessian_ws_bytes(n, T_chunk, has_X_fp);
+}
+
+realq_status_t realq_hessian_accumulate(realq_stream_t stream, int64_t n, int64_t T_chunk, const void *X_hat,
+                                        const void *X_fp, realq_dtype_t x_dtype, float *H_sum, float *D_sum, void *ws,
+                                        size_t ws_bytes) {
+    if (n <= 0 || T_chunk < 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate: n > 0, T_chunk >= 0 required");
+    if (!valid_dtype(x_dtype)) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate: bad x_dtype");
+    if (!H_sum || (T_chunk > 0 && !X_hat)) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate: NULL X_hat or H_sum");
+    if (X_fp && !D_sum) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate: D_sum required with X_fp");
+    if (ws && reinterpret_cast<uintptr_t>(ws) % kAlign)
+        return fail(REALQ_ERR_WORKSPACE, "hessian_accumulate: workspace must be %zu-byte aligned", kAlign);
+    if (T_chunk == 0) return REALQ_OK;
+    return hessian_accumulate(S(stream), n, T_chunk, X_hat, X_fp, x_dtype, H_sum, D_sum, ws, ws ? ws_bytes : 0);
+}
+
+// -------------------------------------------------------------- prepare ---
+size_t realq_prepare_workspace_size(int64_t n) { return n > 0 ? prepare_ws_bytes(n) : 0; }
+
+realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                     const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                     int64_t *fail_col, void *ws, size_t ws_bytes) {
+    if (n <= 0 || T_total <= 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare: n > 0, T_total > 0 required");
+    if (!H_sum || !U_out || !dead_out || !fail_col) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare: NULL argument");
+    if ((const void *)U_out == (const void *)H_sum) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare: U_out may not alias H_sum");
+    if (!(damp_frac >= 0.f) || !std::isfinite(damp_frac)) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare: damp_frac >= 0");
+    REALQ_TRY(check_ws(ws, ws_bytes, prepare_ws_bytes(n), "hessian_prepare"));
+    *fail_col = -1;
+    return prepare(S(stream), n, T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col, ws, ws_bytes);
+}
+
+realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum, float *Dbar) {
+    if (n <= 0 || T_total <= 0 || !D_sum || !Dbar) return fail(REALQ_ERR_INVALID_ARG, "scale_moment: bad argument");
+    return scale_copy(S(stream), n * n, (float)T_total, D_sum, Dbar);
+}
+
+// ---------------------------------------------------------------- sweep ---
+size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg,
+                                     int has_F_next, int has_Dbar) {
+    if (m <= 0 || n <= 0 || !qcfg) return 0;
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, has_Dbar);
+}
+
+realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
+                                    const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
+                                    const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg, const float *F,
+                                    const float *F_next, float *W_work, float *adam_m, float *adam_v, int64_t *adam_t,
+                                    uint8_t *codes, float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
+                                    int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
+    if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: m, n must be > 0");
+    if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: m, n too large");
+    if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: bad dtype");
+    if (!W0 || !U || !W_work || !codes || !scale || !zero)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: NULL W0, U, W_work, codes, scale or zero");
+    REALQ_TRY(check_qcfg(qcfg, n));
+    REALQ_TRY(check_bcfg(bcfg));
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    if (bgd) {
+        if (!Hbar || !F || !adam_t) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Block-GD needs Hbar, F and adam_t");
+        if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
+            return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Adam needs adam_m and adam_v");
+    }
+    const int64_t nb = (n + qcfg->block_size - 1) / qcfg->block_size;
+    if (block_begin < 0 || block_end > nb || block_begin > block_end)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: block range [%lld, %lld) outside [0, %lld)",
+                    (long long)block_begin, (long long)block_end, (long long)nb);
+    const int has_fn = bgd && F_next != nullptr;
+    const int has_db = bgd && Dbar != nullptr;
+    REALQ_TRY(check_ws(ws, ws_bytes, sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db), "quantize_layer"));
+
+    SweepPlan p{};
+    p.m = m; p.n = n; p.W0 = W0; p.w_dtype = w_dtype;
+    p.U = U; p.Hbar = Hbar; p.Dbar = has_db ? Dbar : nullptr; p.dead = dead;
+    p.bits = qcfg->bits; p.block = qcfg->block_size; p.sym = qcfg->symmetric;
+    p.group = effective_group(qcfg, n);
+    p.ngroups = (int)((n + p.group - 1) / p.group);
+    p.bgd_steps = bgd ? bcfg->steps_per_block : 0;
+    if (bgd) {
+        p.optimizer = bcfg->optimizer; p.lr = bcfg->lr; p.beta1 = bcfg->beta1; p.beta2 = bcfg->beta2; p.eps = bcfg->eps;
+        p.b_global_start = bcfg->b_global_start; p.B_total = bcfg->B_total;
+    }
+    p.F = F; p.F_next = has_fn ? F_next : nullptr;
+    p.W = W_work; p.adam_m = adam_m; p.adam_v = adam_v; p.adam_t = adam_t;
+    p.codes = codes; p.scale = scale; p.zero = zero; p.W_deq = W_deq; p.deq_dtype = deq_dtype;
+    sweep_carve(p, ws, bgd, has_fn, has_db);
+    cudaStream_t s = S(stream);
+    REALQ_CUDA_TRY(cudaMemsetAsync(p.status, 0, sizeof(int), s));
+    if (block_begin == 0) REALQ_TRY(sweep_init(s, p));
+    REALQ_TRY(sweep_prologue_r0(s, p));
+    for (int64_t b = block_begin; b < block_end; ++b) REALQ_TRY(sweep_block(s, p, b));
+    return REALQ_OK;
+}
+
+// ---------------------------------------------------------------- BGD -----
+size_t realq_bgd_workspace_size(int64_t m, int64_t n, int has_F_next, int has_Dbar) {
+    if (m <= 0 || n <= 0) return 0;
+    return sweep_ws_bytes(m, n, 0, 1, has_F_next, has_Dbar);
+}
+
+realq_status_t realq_bgd_refine(realq_stream_t stream, int64_t m, int64_t n, int64_t col_start, float *W, const void *W0,
+                                realq_dtype_t w_dtype, const float *Hbar, const float *Dbar, const float *F,
+                                const float *F_next, float alpha, float *adam_m, float *adam_v, int64_t *adam_t,
+                                const realq_bgd_cfg_t *bcfg, void *ws, size_t ws_bytes) {
+    if (m <= 0 || n <= 0 || col_start < 0 || col_start > n) return fail(REALQ_ERR_INVALID_ARG, "bgd_refine: bad sizes");
+    if (!W || !W0 || !Hbar || !F || !bcfg || !adam_t) return fail(REALQ_ERR_INVALID_ARG, "bgd_refine: NULL argument");
+    if (!valid_dtype(w_dtype)) return fail(REALQ_ERR_INVALID_ARG, "bgd_refine: bad dtype");
+    REALQ_TRY(check_bcfg(bcfg));
+    if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v)) return fail(REALQ_ERR_INVALID_ARG, "bgd_refine: Adam state");
+    if (!(alpha >= 0.f && alpha <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "bgd_refine: alpha must be in [0, 1]");
+    const int has_fn = F_next != nullptr, has_db = Dbar != nullptr;
+    REALQ_TRY(check_ws(ws, ws_bytes, sweep_ws_bytes(m, n, 0, 1, has_fn, has_db), "bgd_refine"));
+    SweepPlan p{};
+    p.m = m; p.n = n; p.W0 = W0; p.w_dtype = w_dtype; p.Hbar = Hbar; p.Dbar = Dbar;
+    p.bgd_steps = bcfg->steps_per_block; p.optimizer = bcfg->optimizer; p.lr = bcfg->lr;
+    p.beta1 = bcfg->beta1; p.beta2 = bcfg->beta2; p.eps = bcfg->eps;
+    p.F = F; p.F_next = F_next; p.W = W; p.adam_m = adam_m; p.adam_v = adam_v; p.adam_t = adam_t;
+    p.block = 0;
+    sweep_carve(p, ws, 1, has_fn, has_db);
+    return bgd_step(S(stream), p, col_start, alpha);
+}
+
+// ------------------------------------------------------------ surrogate ---
+size_t realq_surrogate_workspace_size(int64_t m, int64_t n) { return (m > 0 && n > 0) ? surrogate_ws_bytes(m, n) : 0; }
+
+realq_status_t realq_surrogate_loss(realq_stream_t stream, int64_t m, int64_t n, const float *W_hat, const void *W0,
+                                    realq_dtype_t w_dtype, const float *Hbar, const float *F, float *loss_out, void *ws,
+                                    size_t ws_bytes) {
+    if (m <= 0 || n <= 0 || !W_hat || !W0 || !Hbar || !F || !loss_out)
+        return fail(REALQ_ERR_INVALID_ARG, "surrogate_loss: bad argument");
+    if (!valid_dtype(w_dtype)) return fail(REALQ_ERR_INVALID_ARG, "surrogate_loss: bad dtype");
+    REALQ_TRY(check_ws(ws, ws_bytes, surrogate_ws_bytes(m, n), "surrogate_loss"));
+    return surrogate(S(stream), m, n, W_hat, W0, w_dtype, Hbar, F, loss_out, ws);
+}
+
+realq_status_t realq_workspace_status(realq_stream_t stream, void *ws, size_t ws_bytes) {
+    if (!ws || ws_bytes < sizeof(int)) return fail(REALQ_ERR_INVALID_ARG, "workspace_status: bad workspace");
+    int st = 0;
+    REALQ_CUDA_TRY(cudaMemcpyAsync(&st, ws, sizeof(int), cudaMemcpyDeviceToHost, S(stream)));
+    REALQ_CUDA_TRY(cudaStreamSynchronize(S(stream)));
+    REALQ_CUDA_TRY(cudaMemsetAsync(ws, 0, sizeof(int), S(stream)));
+    if (st & ST_NONFINITE) return fail(REALQ_ERR_NONFINITE, "non-finite weight met during the sweep");
+    return REALQ_OK;
+}
+
+}  // extern "C"

@@ -1,0 +1,77 @@
+// Host-side launchers of the library's kernels (internal interface).
+#pragma once
+
+#include "common.cuh"
+
+namespace realq {
+
+// ------------------------------------------------------------------ GEMM ---
+// C[M x N] (ldc) <- epilogue(alpha * A[M x K] * B[K x N]), fp32 FFMA, fp32
+// accumulation.  B is row-major (B[k * ldb + j]).  A modes:
+enum AMode {
+    A_ROW = 0,        // A[i][k] = Af[i * lda + k]
+    A_ROW_BF16 = 1,   // A[i][k] = bf16 Ab[i * lda + k]
+    A_DIFF_F32 = 2,   // A[i][k] = Af[i * lda + k] - Yf[i * ldy + k]
+    A_DIFF_BF16 = 3,  // A[i][k] = Af[i * lda + k] - bf16 Yb[i * ldy + k]
+    A_KMAJOR = 4,     // A[i][k] = Af[k * lda + i]
+};
+enum EpiMode {
+    EPI_STORE = 0,    // C = alpha * acc
+    EPI_SUB = 1,      // C = C - alpha * acc
+    EPI_BIAS = 2,     // C = alpha * acc + R[i * ldr + j]
+};
+struct GemmArgs {
+    int64_t M, N, K;
+    const void *A; int64_t lda;
+    const void *Y; int64_t ldy;
+    const float *B; int64_t ldb;
+    float *C; int64_t ldc;
+    const float *R; int64_t ldr;
+    float alpha;
+};
+realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name);
+
+// --------------------------------------------------------------- Hessian ---
+int hessian_splits(int64_t n, int64_t T, int num_sms);
+size_t hessian_ws_bytes(int64_t n, int64_t T, int has_xfp);
+realq_status_t hessian_accumulate(cudaStream_t s, int64_t n, int64_t T, const void *X, const void *Xfp,
+                                  realq_dtype_t dt, float *H, float *D, void *ws, size_t ws_bytes);
+
+// --------------------------------------------------------------- prepare ---
+size_t prepare_ws_bytes(int64_t n);
+realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+                       uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes);
+realq_status_t scale_copy(cudaStream_t s, int64_t count, float mul, const float *in, float *out);
+
+// ----------------------------------------------------------------- sweep ---
+struct SweepPlan {
+    int64_t m, n;
+    const void *W0; realq_dtype_t w_dtype;
+    const float *U, *Hbar, *Dbar;
+    const uint8_t *dead;
+    int bits, group, block, sym;           // group = effective group size (n when per-row)
+    int ngroups;
+    // Block-GD
+    int bgd_steps, optimizer;
+    float lr, beta1, beta2, eps;
+    int b_global_start, B_total;
+    const float *F, *F_next;
+    float *W, *adam_m, *adam_v;
+    int64_t *adam_t;
+    uint8_t *codes; float *scale; uint8_t *zero;
+    void *W_deq; realq_dtype_t deq_dtype;
+    // workspace pieces
+    int *status;
+    float *Et, *P, *G, *Feff, *R0;
+};
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar);
+void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);
+realq_status_t sweep_init(cudaStream_t s, SweepPlan &p);
+realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b);
+realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p);
+realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha);
+realq_status_t surrogate(cudaStream_t s, int64_t m, int64_t n, const float *What, const void *W0,
+                         realq_dtype_t w_dtype, const float *Hbar, const float *F, float *loss, void *ws);
+size_t surrogate_ws_bytes(int64_t m, int64_t n);
+
+}  // namespace realq

@@ -1,0 +1,277 @@
+// Step a3 (Alg. 1: "Compute ... H and its inverse"): H̄ = H_sum / T, dead
+// channels, relative damping, and the upper factor U with Hd^-1 = U^T U.
+//
+// U is obtained without forming Hd^-1: factor Hd = R R^T with R upper
+// triangular (Cholesky taken from the last index backwards), then U = R^-1,
+// because Hd^-1 = R^-T R^-1 = U^T U.  Row j of U, scaled by U_jj, is row j of
+// the inverse Hessian after the Schur-complement downdates of columns < j,
+// which is what the OBS step of Eq. (gptq_update) consumes.
+//
+// Both factorizations are blocked with 64-wide blocks: a one-CTA kernel
+// factors / inverts the diagonal block in shared memory, the off-diagonal work
+// runs as fp32 GEMMs.  A pivot that is not positive (or not finite) records its
+// column in the workspace status word; the host reads it once at the end.
+#include "kernels.cuh"
+
+namespace realq {
+namespace {
+
+constexpr int NB = 64;
+
+__global__ void prep_init_kernel(int64_t n, float Tf, const float *H, float *Hbar, float *A, uint8_t *dead) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= n * n) return;
+    const int64_t i = idx / n, j = idx % n;
+    const float h = H[idx];
+    const float hb = h / Tf;
+    float a = 0.f;
+    if (j > i) a = hb;
+    else if (j == i) {
+        const bool d = (h == 0.f);
+        dead[i] = d ? 1 : 0;
+        a = d ? 1.f : hb;
+    }
+    if (Hbar) Hbar[idx] = hb;
+    A[idx] = a;
+}
+
+// lambda = damp * mean(diag A) (fp64 reduction in a fixed order); A_jj += lambda
+__global__ void prep_damp_kernel(int64_t n, float *A, float damp, float *lam_out) {
+    __shared__ double red[1024];
+    double s = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x) s += (double)A[j * n + j];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+        if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+        __syncthreads();
+    }
+    const float lam = (float)((double)damp * (red[0] / (double)n));
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x) A[j * n + j] += lam;
+    if (threadIdx.x == 0) *lam_out = lam;
+}
+
+// Diagonal block [k0, k0 + kb): A_KK = R_KK R_KK^T, R_KK upper (in place).
+__global__ void chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status) {
+    __shared__ float S[NB][NB + 1];
+    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
+        const int r = idx / NB, c = idx % NB;
+        S[r][c] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
+    }
+    __syncthreads();
+    for (int k = kb - 1; k >= 0; --k) {
+        if (threadIdx.x == 0) {
+            float d = S[k][k];
+            if (!(d > 0.f) || !isfinite(d)) {
+                atomicCAS(status, -1, (int)(k0 + k));
+                d = 1.f;
+            }
+            S[k][k] = sqrtf(d);
+        }
+        __syncthreads();
+        const float r = S[k][k];
+        for (int i = threadIdx.x; i < k; i += blockDim.x) S[i][k] = S[i][k] / r;
+        __syncthreads();
+        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
+            const int i = idx / k, j = idx % k;
+            if (j >= i) S[i][j] -= S[i][k] * S[j][k];
+        }
+        __syncthreads();
+    }
+    for (int idx = threadIdx.x; idx < kb * kb; idx += blockDim.x) {
+        const int r = idx / kb, c = idx % kb;
+        if (c >= r) A[(k0 + r) * n + k0 + c] = S[r][c];
+    }
+}
+
+// Rows i < k0 of the block column: solve x R_KK^T = A[i, k0:k0+kb] (one thread per row).
+__global__ void chol_panel_kernel(int64_t n, float *A, int64_t k0, int kb) {
+    __shared__ float R[NB][NB + 1];
+    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
+        const int r = idx / NB, c = idx % NB;
+        R[r][c] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
+    }
+    __syncthreads();
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= k0) return;
+    float x[NB];
+#pragma unroll
+    for (int c = 0; c < NB; ++c) x[c] = (c < kb) ? A[i * n + k0 + c] : 0.f;
+#pragma unroll
+    for (int c = NB - 1; c >= 0; --c) {
+        if (c < kb) {
+            float v = x[c];
+#pragma unroll
+            for (int d = c + 1; d < NB; ++d) v -= x[d] * R[c][d];
+            x[c] = v / R[c][c];
+        }
+    }
+#pragma unroll
+    for (int c = 0; c < NB; ++c)
+        if (c < kb) A[i * n + k0 + c] = x[c];
+}
+
+// A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles).
+__global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, int64_t k0, int kb) {
+    __shared__ __align__(16) float Pi[NB][NB + 4];
+    __shared__ __align__(16) float Pj[NB][NB + 4];
+    const int64_t idx = blockIdx.x;
+    int r = (int)((sqrt(8.0 * (double)idx + 1.0) - 1.0) * 0.5);
+    while ((int64_t)(r + 1) * (r + 2) / 2 <= idx) ++r;
+    while ((int64_t)r * (r + 1) / 2 > idx) --r;
+    const int tj = r, ti = (int)(idx - (int64_t)r * (r + 1) / 2);  // ti <= tj
+    const int64_t i0 = (int64_t)ti * NB, j0 = (int64_t)tj * NB;
+    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
+        const int rr = e / NB, c = e % NB;
+        Pi[c][rr] = (c < kb && i0 + rr < k0) ? A[(i0 + rr) * n + k0 + c] : 0.f;
+        Pj[c][rr] = (c < kb && j0 + rr < k0) ? A[(j0 + rr) * n + k0 + c] : 0.f;
+    }
+    __syncthreads();
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float acc[4][4] = {};
+    for (int c = 0; c < kb; ++c) {
+        const float4 a = *reinterpret_cast<const float4 *>(&Pi[c][ty * 4]);
+        const float4 b = *reinterpret_cast<const float4 *>(&Pj[c][tx * 4]);
+        const float av[4] = {a.x, a.y, a.z, a.w}, bv[4] = {b.x, b.y, b.z, b.w};
+#pragma unroll
+        for (int p = 0; p < 4; ++p)
+#pragma unroll
+            for (int q = 0; q < 4; ++q) acc[p][q] = fmaf(av[p], bv[q], acc[p][q]);
+    }
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+        const int64_t gi = i0 + ty * 4 + p;
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+            const int64_t gj = j0 + tx * 4 + q;
+            if (gi < k0 && gj < k0 && gj >= gi) A[gi * n + gj] -= acc[p][q];
+        }
+    }
+}
+
+// V = R_JJ^-1 (upper) by back substitution, one thread per column; written to
+// A[J, J] and to the dense 64 x 64 buffer Vd (zeros below the diagonal).
+__global__ void trtri_diag_kernel(int64_t n, float *A, int64_t j0, int jb, float *Vd) {
+    __shared__ float R[NB][NB + 1];
+    __shared__ float V[NB][NB + 1];
+    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
+        const int r = idx / NB, c = idx % NB;
+        R[r][c] = (r < jb && c < jb && c >= r) ? A[(j0 + r) * n + j0 + c] : 0.f;
+        V[r][c] = 0.f;
+    }
+    __syncthreads();
+    const int c = threadIdx.x;
+    if (c < jb) {
+        V[c][c] = 1.f / R[c][c];
+        for (int i = c - 1; i >= 0; --i) {
+            float s = 0.f;
+            for (int l = i + 1; l <= c; ++l) s += R[i][l] * V[l][c];
+            V[i][c] = -s / R[i][i];
+        }
+    }
+    __syncthreads();
+    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
+        const int r = idx / NB, cc = idx % NB;
+        Vd[idx] = V[r][cc];
+        if (r < jb && cc < jb && cc >= r) A[(j0 + r) * n + j0 + cc] = V[r][cc];
+    }
+}
+
+__global__ void scale_kernel(int64_t count, float div, const float *in, float *out) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i < count) out[i] = in[i] / div;
+}
+
+}  // namespace
+
+size_t prepare_ws_bytes(int64_t n) {
+    return align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)n * NB * sizeof(float)) +
+           align_up((size_t)NB * NB * sizeof(float));
+}
+
+realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+                       uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes) {
+    Carve cv(ws);
+    int *status = cv.take<int>(1);
+    float *lam = cv.take<float>(1);
+    float *panel = cv.take<float>((size_t)n * NB);
+    float *Vd = cv.take<float>((size_t)NB * NB);
+    (void)ws_bytes;
+    REALQ_CUDA_TRY(cudaMemsetAsync(status, 0xFF, sizeof(int), s));
+    const int64_t tot = n * n;
+    {
+        Launch L("prepare_init", s);
+        prep_init_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(n, (float)T, H, Hbar, U, dead);
+    }
+    REALQ_TRY(check_launch("prepare_init"));
+    {
+        Launch L("prepare_damp", s);
+        prep_damp_kernel<<<1, 1024, 0, s>>>(n, U, damp, lam);
+    }
+    REALQ_TRY(check_launch("prepare_damp"));
+    // reverse-order blocked Cholesky: Hd = R R^T
+    const int nbk = ceil_div(n, NB);
+    for (int K = nbk - 1; K >= 0; --K) {
+        const int64_t k0 = (int64_t)K * NB;
+        const int kb = (int)std::min<int64_t>(NB, n - k0);
+        {
+            Launch L("chol_diag", s);
+            chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status);
+        }
+        REALQ_TRY(check_launch("chol_diag"));
+        if (k0 == 0) continue;
+        {
+            Launch L("chol_panel", s);
+            chol_panel_kernel<<<ceil_div(k0, 128), 128, 0, s>>>(n, U, k0, kb);
+        }
+        REALQ_TRY(check_launch("chol_panel"));
+        const int64_t nt0 = k0 / NB;
+        {
+            Launch L("chol_update", s);
+            chol_update_kernel<<<(unsigned)(nt0 * (nt0 + 1) / 2), 256, 0, s>>>(n, U, k0, kb);
+        }
+        REALQ_TRY(check_launch("chol_update"));
+    }
+    // U = R^-1, block columns left to right
+    for (int J = 0; J < nbk; ++J) {
+        const int64_t j0 = (int64_t)J * NB;
+        const int jb = (int)std::min<int64_t>(NB, n - j0);
+        {
+            Launch L("trtri_diag", s);
+            trtri_diag_kernel<<<1, NB, 0, s>>>(n, U, j0, jb, Vd);
+        }
+        REALQ_TRY(check_launch("trtri_diag"));
+        if (j0 == 0) continue;
+        GemmArgs g{};
+        g.M = j0; g.N = jb; g.K = j0;
+        g.A = U; g.lda = n;
+        g.B = U + j0; g.ldb = n;
+        g.C = panel; g.ldc = NB;
+        g.alpha = 1.f;
+        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "trtri_trmm"));
+        GemmArgs h{};
+        h.M = j0; h.N = jb; h.K = jb;
+        h.A = panel; h.lda = NB;
+        h.B = Vd; h.ldb = NB;
+        h.C = U + j0; h.ldc = n;
+        h.alpha = -1.f;
+        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, h, "trtri_panel"));
+    }
+    int host_status = -1;
+    REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
+    REALQ_CUDA_TRY(cudaStreamSynchronize(s));
+    *fail_col = host_status;
+    if (host_status >= 0) return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", host_status);
+    return REALQ_OK;
+}
+
+realq_status_t scale_copy(cudaStream_t s, int64_t count, float div, const float *in, float *out) {
+    if (count == 0) return REALQ_OK;
+    {
+        Launch L("scale_moment", s);
+        scale_kernel<<<(unsigned)((count + 255) / 256), 256, 0, s>>>(count, div, in, out);
+    }
+    return check_launch("scale_moment");
+}
+
+}  // namespace realq

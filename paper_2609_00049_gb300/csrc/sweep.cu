@@ -1,0 +1,456 @@
+// Steps a4-a8 of the sweep for one module (Alg. 1, loop over column blocks):
+//   quantize the B columns of block b with OBS error feedback inside the block
+//   (Eq. gptq_update, written with rows of U: err_j = (w_j - deq_j) / U_jj,
+//   W[:, k] -= err_j U_jk), the lazy batch update of all later columns
+//   (Sec. 3.2: W[:, rest] -= E_b U[b, rest]), then Block-GD on the later columns
+//   (Eq. block_gd_update) with the layer-level Fisher surrogate, optionally
+//   blended with the next block's Fisher (Eq. slide_window).
+#include "kernels.cuh"
+
+#include <cmath>
+
+namespace realq {
+namespace {
+
+constexpr int QB_THREADS = 32;
+
+// quant(.) grid of one group from its min / max (the reading fixed by the
+// oracle: the grid contains 0; degenerate groups get [-1, 1]).  fp32, IEEE
+// division, round-half-to-even.
+__device__ __forceinline__ void grid_params(float mn, float mx, int bits, int sym, float &sc, float &zr) {
+    const float maxq = (float)((1 << bits) - 1);
+    float xmin = fminf(mn, 0.f), xmax = fmaxf(mx, 0.f);
+    if (sym) {
+        xmax = fmaxf(-xmin, xmax);
+        xmin = -xmax;
+    }
+    if (xmin == 0.f && xmax == 0.f) {
+        xmin = -1.f;
+        xmax = 1.f;
+    }
+    sc = (xmax - xmin) / maxq;
+    zr = sym ? (float)(1 << (bits - 1)) : rintf(-xmin / sc);
+}
+
+template <typename TW>
+__global__ void init_work_kernel(int64_t m, int64_t n, const TW *W0, const uint8_t *dead, float *W) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * n) return;
+    const int64_t j = idx % n;
+    W[idx] = (dead && dead[j]) ? 0.f : load_as_float(W0, idx);
+}
+
+// one warp per row: min / max of W[i, c0:c1) -> (scale, zero) of group gi
+__global__ void group_params_kernel(int64_t m, int64_t n, const float *W, int64_t c0, int64_t c1, int gi,
+                                    int ngroups, int bits, int sym, float *scale, uint8_t *zero) {
+    const int64_t i = (int64_t)blockIdx.x * (blockDim.x / 32) + threadIdx.x / 32;
+    const int lane = threadIdx.x & 31;
+    if (i >= m) return;
+    float mn = 0.f, mx = 0.f;
+    for (int64_t c = c0 + lane; c < c1; c += 32) {
+        const float w = W[i * n + c];
+        mn = fminf(mn, w);
+        mx = fmaxf(mx, w);
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        mn = fminf(mn, __shfl_xor_sync(0xffffffffu, mn, o));
+        mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    }
+    if (lane == 0) {
+        float sc, zr;
+        grid_params(mn, mx, bits, sym, sc, zr);
+        scale[i * ngroups + gi] = sc;
+        zero[i * ngroups + gi] = (uint8_t)zr;
+    }
+}
+
+struct QArgs {
+    int64_t m, n, bs;
+    int kb;
+    float *W;
+    const float *U;
+    int g, ngroups, bits, sym;
+    float *scale;
+    uint8_t *zero;
+    uint8_t *codes;
+    int64_t ncb;
+    float *Et;
+    int *status;
+};
+
+// Column-serial quantize + in-block OBS propagation for block [bs, bs + kb).
+// One thread owns one row; the row's B columns live in registers (fully
+// unrolled), the B x B diagonal block of U is staged once per CTA in shared
+// memory and read as broadcasts.  G > 0: group parameters are computed here
+// at every G-th column from the current (compensated) weights; G = 0: they
+// were computed before the block for a group spanning whole blocks.
+template <int B, int G>
+__global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) {
+    extern __shared__ __align__(16) float qsm[];
+    float *Us = qsm;           // B x B
+    float *invd = qsm + B * B; // B
+    const int kb = a.kb;
+    for (int idx = threadIdx.x; idx < B * B; idx += blockDim.x) {
+        const int r = idx / B, c = idx % B;
+        Us[idx] = (r < kb && c < kb && c > r) ? a.U[(a.bs + r) * a.n + a.bs + c] : 0.f;
+    }
+    for (int j = threadIdx.x; j < B; j += blockDim.x)
+        invd[j] = (j < kb) ? 1.f / a.U[(a.bs + j) * a.n + a.bs + j] : 0.f;
+    __syncthreads();
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= a.m) return;
+
+    float r[B];
+    const float *wrow = a.W + i * a.n + a.bs;
+#pragma unroll
+    for (int c = 0; c < B; ++c) r[c] = (c < kb) ? wrow[c] : 0.f;
+
+    float sc = 1.f, zr = 0.f;
+    if (G == 0) {
+        const int gi = (int)(a.bs / a.g);
+        sc = a.scale[i * a.ngroups + gi];
+        zr = (float)a.zero[i * a.ngroups + gi];
+    }
+    const float maxq = (float)((1 << a.bits) - 1);
+    uint8_t *crow = a.codes + i * a.ncb + a.bs / 2;
+    bool bad = false;
+    unsigned lo = 0;
+#pragma unroll
+    for (int j = 0; j < B; ++j) {
+        if (j < kb) {
+            if (G > 0 && (j % (G > 0 ? G : 1)) == 0) {
+                float mn = 0.f, mx = 0.f;
+#pragma unroll
+                for (int c = j; c < j + G && c < B; ++c)
+                    if (c < kb) {
+                        mn = fminf(mn, r[c]);
+                        mx = fmaxf(mx, r[c]);
+                    }
+                grid_params(mn, mx, a.bits, a.sym, sc, zr);
+                const int gi = (int)((a.bs + j) / a.g);
+                a.scale[i * a.ngroups + gi] = sc;
+                a.zero[i * a.ngroups + gi] = (uint8_t)zr;
+            }
+            const float w = r[j];
+            bad |= !isfinite(w);
+            float q = rintf(w / sc) + zr;
+            q = fminf(fmaxf(q, 0.f), maxq);
+            const float dq = sc * (q - zr);
+            const float e = (w - dq) * invd[j];
+            a.Et[(int64_t)j * a.m + i] = e;
+            r[j] = dq;
+#pragma unroll
+            for (int k = j + 1; k < B; ++k) r[k] = fmaf(-e, Us[j * B + k], r[k]);
+            const unsigned qi = (unsigned)q;
+            if ((j & 1) == 0) {
+                lo = qi;
+                if (j == kb - 1) crow[j / 2] = (uint8_t)lo;
+            } else {
+                crow[j / 2] = (uint8_t)(lo | (qi << 4));
+            }
+        }
+    }
+    float *wout = a.W + i * a.n + a.bs;
+#pragma unroll
+    for (int c = 0; c < B; ++c)
+        if (c < kb) wout[c] = r[c];
+    if (bad) atomicOr(a.status, ST_NONFINITE);
+}
+
+__global__ void adam_kernel(int64_t m, int64_t r, int64_t n, int64_t c0, const float *G, float *W, float *mA,
+                            float *vA, float lr, float b1, float b2, float eps, float bc1, float bc2, int sgd) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * r) return;
+    const int64_t i = idx / r, c = idx % r;
+    const int64_t w = i * n + c0 + c;
+    const float g = G[idx];
+    if (sgd) {
+        W[w] -= lr * g;
+        return;
+    }
+    const float mv = b1 * mA[w] + (1.f - b1) * g;
+    const float vv = b2 * vA[w] + (1.f - b2) * g * g;
+    mA[w] = mv;
+    vA[w] = vv;
+    W[w] -= lr * (mv / bc1) / (sqrtf(vv / bc2) + eps);
+}
+
+__global__ void feff_kernel(int64_t count, const float *F, const float *Fn, float alpha, float *out) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx < count) out[idx] = alpha * F[idx] + (1.f - alpha) * Fn[idx];
+}
+
+template <typename TO>
+__global__ void copy_cols_kernel(int64_t m, int64_t n, int64_t c0, int64_t c1, const float *W, TO *out) {
+    const int64_t w = c1 - c0;
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * w) return;
+    const int64_t i = idx / w, c = c0 + idx % w;
+    if constexpr (sizeof(TO) == 2) out[i * n + c] = __float2bfloat16_rn(W[i * n + c]);
+    else out[i * n + c] = W[i * n + c];
+}
+
+template <typename TW>
+__global__ void diff_kernel(int64_t count, const float *A, const TW *W0, float *out) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx < count) out[idx] = A[idx] - load_as_float(W0, idx);
+}
+
+// 1/2 sum X1 .* X2 in fp64, two fixed-order stages
+constexpr int RED_BLOCKS = 512;
+__global__ void dot_partial_kernel(int64_t count, const float *X1, const float *X2, double *part) {
+    __shared__ double red[256];
+    double s = 0.0;
+    for (int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x; idx < count; idx += (int64_t)gridDim.x * blockDim.x)
+        s += (double)X1[idx] * (double)X2[idx];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = 128; w > 0; w >>= 1) {
+        if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) part[blockIdx.x] = red[0];
+}
+__global__ void dot_final_kernel(const double *part, int nparts, float *out) {
+    __shared__ double red[RED_BLOCKS];
+    red[threadIdx.x] = threadIdx.x < nparts ? part[threadIdx.x] : 0.0;
+    __syncthreads();
+    for (int w = RED_BLOCKS / 2; w > 0; w >>= 1) {
+        if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *out = (float)(0.5 * red[0]);
+}
+
+inline unsigned blocks_for(int64_t count, int threads = 256) { return (unsigned)((count + threads - 1) / threads); }
+
+template <int B, int G>
+realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
+    const size_t smem = (size_t)(B * B + B) * sizeof(float);
+    static bool configured = false;
+    if (!configured) {
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(quant_block_kernel<B, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
+        configured = true;
+    }
+    {
+        Launch L("quant_block", s);
+        quant_block_kernel<B, G><<<ceil_div(qa.m, QB_THREADS), QB_THREADS, smem, s>>>(qa);
+    }
+    return check_launch("quant_block");
+}
+
+template <int B>
+realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
+    if (Gk == 0) return launch_qb<B, 0>(s, qa);
+    if (Gk == B) return launch_qb<B, B>(s, qa);
+    if (B >= 64 && Gk == B / 2) return launch_qb<B, (B >= 64 ? B / 2 : B)>(s, qa);
+    if (B >= 128 && Gk == B / 4) return launch_qb<B, (B >= 128 ? B / 4 : B)>(s, qa);
+    return fail(REALQ_ERR_UNSUPPORTED, "group size %d inside block %d", Gk, B);
+}
+
+}  // namespace
+
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar) {
+    size_t b = align_up(sizeof(int)) + align_up((size_t)block * m * sizeof(float));
+    if (has_bgd) {
+        b += 2 * align_up((size_t)m * n * sizeof(float));
+        if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
+        if (has_dbar) b += align_up((size_t)m * n * sizeof(float));
+    }
+    return b;
+}
+
+void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar) {
+    Carve cv(ws);
+    p.status = cv.take<int>(1);
+    p.Et = cv.take<float>((size_t)p.block * p.m);
+    p.P = p.G = p.Feff = p.R0 = nullptr;
+    if (has_bgd) {
+        p.P = cv.take<float>((size_t)p.m * p.n);
+        p.G = cv.take<float>((size_t)p.m * p.n);
+        if (has_fnext) p.Feff = cv.take<float>((size_t)p.m * p.m);
+        if (has_dbar) p.R0 = cv.take<float>((size_t)p.m * p.n);
+    }
+}
+
+realq_status_t sweep_init(cudaStream_t s, SweepPlan &p) {
+    const int64_t mn = p.m * p.n;
+    {
+        Launch L("init_work", s);
+        if (p.w_dtype == REALQ_BF16)
+            init_work_kernel<<<blocks_for(mn), 256, 0, s>>>(p.m, p.n, static_cast<const __nv_bfloat16 *>(p.W0), p.dead, p.W);
+        else
+            init_work_kernel<<<blocks_for(mn), 256, 0, s>>>(p.m, p.n, static_cast<const float *>(p.W0), p.dead, p.W);
+    }
+    REALQ_TRY(check_launch("init_work"));
+    if (p.bgd_steps > 0) {
+        if (p.optimizer == REALQ_OPT_ADAM) {
+            REALQ_CUDA_TRY(cudaMemsetAsync(p.adam_m, 0, (size_t)mn * sizeof(float), s));
+            REALQ_CUDA_TRY(cudaMemsetAsync(p.adam_v, 0, (size_t)mn * sizeof(float), s));
+        }
+        *p.adam_t = 0;
+    }
+    return REALQ_OK;
+}
+
+static realq_status_t compute_r0(cudaStream_t s, SweepPlan &p) {
+    GemmArgs g{};
+    g.M = p.m; g.N = p.n; g.K = p.n;
+    g.A = p.W0; g.lda = p.n;
+    g.B = p.Dbar; g.ldb = p.n;
+    g.C = p.R0; g.ldc = p.n;
+    g.alpha = 1.f;
+    return gemm_f32(s, p.w_dtype == REALQ_BF16 ? A_ROW_BF16 : A_ROW, EPI_STORE, g, "bgd_r0_gemm");
+}
+
+static realq_status_t fisher_for(cudaStream_t s, SweepPlan &p, float alpha, const float **Fuse) {
+    *Fuse = p.F;
+    if (p.F_next == nullptr || alpha == 1.f) return REALQ_OK;
+    if (alpha == 0.f) {
+        *Fuse = p.F_next;
+        return REALQ_OK;
+    }
+    {
+        Launch L("fisher_blend", s);
+        feff_kernel<<<blocks_for(p.m * p.m), 256, 0, s>>>(p.m * p.m, p.F, p.F_next, alpha, p.Feff);
+    }
+    *Fuse = p.Feff;
+    return check_launch("fisher_blend");
+}
+
+static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const float *Fuse) {
+    const int64_t r = p.n - c0;
+    GemmArgs g{};
+    g.M = p.m; g.N = r; g.K = p.n;
+    g.A = p.W; g.lda = p.n;
+    g.Y = p.W0; g.ldy = p.n;
+    g.B = p.Hbar + c0; g.ldb = p.n;
+    g.C = p.P; g.ldc = r;
+    g.R = p.R0 ? p.R0 + c0 : nullptr; g.ldr = p.n;
+    g.alpha = 1.f;
+    REALQ_TRY(gemm_f32(s, p.w_dtype == REALQ_BF16 ? A_DIFF_BF16 : A_DIFF_F32, p.R0 ? EPI_BIAS : EPI_STORE, g,
+                       "bgd_p_gemm"));
+    GemmArgs h{};
+    h.M = p.m; h.N = r; h.K = p.m;
+    h.A = Fuse; h.lda = p.m;
+    h.B = p.P; h.ldb = r;
+    h.C = p.G; h.ldc = r;
+    h.alpha = 1.f;
+    REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, h, "bgd_g_gemm"));
+    const int64_t t = ++(*p.adam_t);
+    const double bc1 = 1.0 - std::pow((double)p.beta1, (double)t);
+    const double bc2 = 1.0 - std::pow((double)p.beta2, (double)t);
+    {
+        Launch L("bgd_adam", s);
+        adam_kernel<<<blocks_for(p.m * r), 256, 0, s>>>(p.m, r, p.n, c0, p.G, p.W, p.adam_m, p.adam_v, p.lr, p.beta1,
+                                                         p.beta2, p.eps, (float)bc1, (float)bc2,
+                                                         p.optimizer == REALQ_OPT_SGD);
+    }
+    return check_launch("bgd_adam");
+}
+
+realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
+    if (col_start >= p.n) return REALQ_OK;
+    if (p.Dbar) REALQ_TRY(compute_r0(s, p));
+    const float *Fuse = nullptr;
+    REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
+    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, col_start, Fuse));
+    return REALQ_OK;
+}
+
+realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
+    const int B = p.block;
+    const int64_t bs = b * B;
+    const int64_t be = std::min<int64_t>(bs + B, p.n);
+    const int kb = (int)(be - bs);
+    const int params_here = p.group <= B;
+    if (!params_here && bs % p.group == 0) {
+        Launch L("group_params", s);
+        group_params_kernel<<<ceil_div(p.m, 8), 256, 0, s>>>(p.m, p.n, p.W, bs, std::min<int64_t>(bs + p.group, p.n),
+                                                              (int)(bs / p.group), p.ngroups, p.bits, p.sym, p.scale,
+                                                              p.zero);
+    }
+    if (!params_here) REALQ_TRY(check_launch("group_params"));
+    QArgs qa{};
+    qa.m = p.m; qa.n = p.n; qa.bs = bs; qa.kb = kb;
+    qa.W = p.W; qa.U = p.U;
+    qa.g = p.group; qa.ngroups = p.ngroups; qa.bits = p.bits; qa.sym = p.sym;
+    qa.scale = p.scale; qa.zero = p.zero; qa.codes = p.codes; qa.ncb = (p.n + 1) / 2;
+    qa.Et = p.Et; qa.status = p.status;
+    const int Gk = params_here ? p.group : 0;
+    if (B == 128) REALQ_TRY(launch_qb_g<128>(s, qa, Gk));
+    else if (B == 64) REALQ_TRY(launch_qb_g<64>(s, qa, Gk));
+    else REALQ_TRY(launch_qb_g<32>(s, qa, Gk));
+    if (p.W_deq) {
+        Launch L("copy_deq", s);
+        if (p.deq_dtype == REALQ_BF16)
+            copy_cols_kernel<<<blocks_for(p.m * kb), 256, 0, s>>>(p.m, p.n, bs, be, p.W, static_cast<__nv_bfloat16 *>(p.W_deq));
+        else
+            copy_cols_kernel<<<blocks_for(p.m * kb), 256, 0, s>>>(p.m, p.n, bs, be, p.W, static_cast<float *>(p.W_deq));
+    }
+    if (p.W_deq) REALQ_TRY(check_launch("copy_deq"));
+    if (be >= p.n) return REALQ_OK;
+    // lazy batch update of every later column: W[:, be:] -= E_b U[bs:be, be:]
+    GemmArgs g{};
+    g.M = p.m; g.N = p.n - be; g.K = kb;
+    g.A = p.Et; g.lda = p.m;
+    g.B = p.U + bs * p.n + be; g.ldb = p.n;
+    g.C = p.W + be; g.ldc = p.n;
+    g.alpha = 1.f;
+    REALQ_TRY(gemm_f32(s, A_KMAJOR, EPI_SUB, g, "trailing_update"));
+    if (p.bgd_steps <= 0) return REALQ_OK;
+    const int64_t b_global = p.b_global_start + b;
+    float alpha = 1.f;
+    if (p.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(p.B_total - 1));
+    const float *Fuse = nullptr;
+    REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
+    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, be, Fuse));
+    return REALQ_OK;
+}
+
+realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p) {
+    if (p.Dbar && p.bgd_steps > 0) return compute_r0(s, p);
+    return REALQ_OK;
+}
+
+size_t surrogate_ws_bytes(int64_t m, int64_t n) {
+    return 3 * align_up((size_t)m * n * sizeof(float)) + align_up(RED_BLOCKS * sizeof(double));
+}
+
+realq_status_t surrogate(cudaStream_t s, int64_t m, int64_t n, const float *What, const void *W0,
+                         realq_dtype_t w_dtype, const float *Hbar, const float *F, float *loss, void *ws) {
+    Carve cv(ws);
+    float *dW = cv.take<float>((size_t)m * n);
+    float *X1 = cv.take<float>((size_t)m * n);
+    float *X2 = cv.take<float>((size_t)m * n);
+    double *part = cv.take<double>(RED_BLOCKS);
+    {
+        Launch L("surrogate_diff", s);
+        if (w_dtype == REALQ_BF16)
+            diff_kernel<<<blocks_for(m * n), 256, 0, s>>>(m * n, What, static_cast<const __nv_bfloat16 *>(W0), dW);
+        else
+            diff_kernel<<<blocks_for(m * n), 256, 0, s>>>(m * n, What, static_cast<const float *>(W0), dW);
+    }
+    REALQ_TRY(check_launch("surrogate_diff"));
+    GemmArgs g{};
+    g.M = m; g.N = n; g.K = n;
+    g.A = dW; g.lda = n; g.B = Hbar; g.ldb = n; g.C = X1; g.ldc = n; g.alpha = 1.f;
+    REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "surrogate_gemm"));
+    GemmArgs h{};
+    h.M = m; h.N = n; h.K = m;
+    h.A = F; h.lda = m; h.B = dW; h.ldb = n; h.C = X2; h.ldc = n; h.alpha = 1.f;
+    REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, h, "surrogate_gemm"));
+    {
+        Launch L("surrogate_reduce", s);
+        dot_partial_kernel<<<RED_BLOCKS, 256, 0, s>>>(m * n, X1, X2, part);
+    }
+    REALQ_TRY(check_launch("surrogate_reduce"));
+    {
+        Launch L("surrogate_reduce", s);
+        dot_final_kernel<<<1, RED_BLOCKS, 0, s>>>(part, RED_BLOCKS, loss);
+    }
+    return check_launch("surrogate_reduce");
+}
+
+}  // namespace realq

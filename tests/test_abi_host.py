@@ -1,0 +1,106 @@
+"""Host-side checks of the C ABI: the library builds, loads, exports every
+declared entry point, and rejects bad arguments before touching the GPU."""
+import ctypes
+import os
+import re
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+@pytest.fixture(scope="module")
+def L():
+    from paper_2609_00049_gb300 import build as b
+    b.build()
+    import paper_2609_00049_gb300 as rq
+    return rq.lib()
+
+
+def _declared():
+    src = open(os.path.join(ROOT, "include", "realq.h")).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(realq_\w+)\s*\(", src)))
+
+
+def test_exports_every_declared_symbol(L):
+    names = _declared()
+    assert len(names) >= 15
+    for n in names:
+        assert hasattr(L, n), n
+
+
+def test_status_strings(L):
+    import paper_2609_00049_gb300 as rq
+    for s in range(8):
+        assert rq.realq_status_string(s)
+    assert rq.realq_status_string(3) == "damped Hessian not positive definite"
+
+
+def test_workspace_sizes(L):
+    import paper_2609_00049_gb300 as rq
+    q = rq.quant_cfg()
+    b = rq.bgd_cfg(1e-4)
+    w0 = rq.realq_quantize_workspace_size(256, 512, q, None)
+    w1 = rq.realq_quantize_workspace_size(256, 512, q, b)
+    w2 = rq.realq_quantize_workspace_size(256, 512, q, b, has_F_next=True, has_Dbar=True)
+    assert 0 < w0 < w1 < w2
+    assert w1 >= 2 * 256 * 512 * 4
+    assert rq.realq_prepare_workspace_size(1000) >= 1000 * 64 * 4
+    assert rq.realq_quantize_workspace_size(0, 512, q, None) == 0
+    # a small Hessian on many tokens splits the token range; a large one does not
+    assert rq.realq_hessian_workspace_size(128, 65536) > 0
+    assert rq.realq_hessian_workspace_size(8192, 8192) == 0
+
+
+FAKE = ctypes.c_void_p(0x10000)   # never dereferenced: every call below fails validation first
+
+
+def _ql(L, m=256, n=512, qcfg=None, bcfg=None, F=FAKE, W0=FAKE, ws=FAKE, ws_bytes=1 << 30, blocks=(0, 4)):
+    import paper_2609_00049_gb300 as rq
+    q = qcfg or rq.quant_cfg()
+    t = ctypes.c_int64(0)
+    return L.realq_quantize_layer(None, m, n, W0, 0, FAKE, FAKE, None, None, ctypes.byref(q),
+                                  ctypes.byref(bcfg) if bcfg is not None else None, F, None, FAKE, FAKE, FAKE,
+                                  ctypes.byref(t), FAKE, FAKE, FAKE, None, 0, blocks[0], blocks[1], ws, ws_bytes)
+
+
+def test_argument_validation(L):
+    import paper_2609_00049_gb300 as rq
+    assert _ql(L, m=0) == rq.REALQ_ERR_INVALID_ARG
+    assert "m, n" in rq.realq_last_error()
+    assert _ql(L, W0=None) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, qcfg=rq.quant_cfg(bits=5)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, qcfg=rq.quant_cfg(block_size=96)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, qcfg=rq.quant_cfg(group_size=16)) == rq.REALQ_ERR_UNSUPPORTED
+    assert _ql(L, qcfg=rq.quant_cfg(group_size=192)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, bcfg=rq.bgd_cfg(1e-4), F=None) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, bcfg=rq.bgd_cfg(1e-4, beta1=1.0)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, bcfg=rq.bgd_cfg(float("nan"))) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, blocks=(0, 5)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, blocks=(3, 2)) == rq.REALQ_ERR_INVALID_ARG
+    assert _ql(L, ws=None) == rq.REALQ_ERR_WORKSPACE
+    assert _ql(L, ws=ctypes.c_void_p(0x10010)) == rq.REALQ_ERR_WORKSPACE
+    assert _ql(L, ws_bytes=100) == rq.REALQ_ERR_WORKSPACE
+    fc = ctypes.c_int64(7)
+    assert L.realq_hessian_prepare(None, 0, 10, 0.01, FAKE, FAKE, FAKE, FAKE, ctypes.byref(fc), FAKE, 1 << 20) == 1
+    assert L.realq_hessian_prepare(None, 64, 10, 0.01, FAKE, ctypes.c_void_p(0x20000), FAKE, FAKE, ctypes.byref(fc),
+                                   None, 0) == 2
+    assert L.realq_hessian_prepare(None, 64, 10, 0.01, FAKE, FAKE, FAKE, FAKE, ctypes.byref(fc), FAKE, 1 << 20) == 1
+    assert L.realq_hessian_prepare(None, 64, 10, -1.0, FAKE, ctypes.c_void_p(0x20000), FAKE, FAKE,
+                                   ctypes.byref(fc), FAKE, 1 << 20) == 1
+    assert L.realq_hessian_accumulate(None, 64, 100, FAKE, FAKE, 1, FAKE, None, None, 0) == 1
+    assert L.realq_hessian_accumulate(None, 64, 100, FAKE, None, 9, FAKE, None, None, 0) == 1
+    assert L.realq_hessian_accumulate(None, 64, 0, None, None, 1, FAKE, None, None, 0) == 0  # empty chunk
+    assert L.realq_bgd_refine(None, 4, 4, 5, FAKE, FAKE, 0, FAKE, None, FAKE, None, 1.0, FAKE, FAKE,
+                              ctypes.byref(ctypes.c_int64(0)), ctypes.byref(rq.bgd_cfg(1e-3)), FAKE, 1 << 20) == 1
+    assert L.realq_bgd_refine(None, 4, 4, 0, FAKE, FAKE, 0, FAKE, None, FAKE, None, 1.5, FAKE, FAKE,
+                              ctypes.byref(ctypes.c_int64(0)), ctypes.byref(rq.bgd_cfg(1e-3)), FAKE, 1 << 20) == 1
+
+
+def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
+    import paper_2609_00049_gb300 as rq
+    monkeypatch.setattr(rq, "_lib", None)
+    monkeypatch.setattr(rq, "library_path", str(tmp_path / "missing.so"))
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        rq.lib()

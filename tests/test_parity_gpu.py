@@ -1,0 +1,298 @@
+"""CUDA path vs the fp64 oracle on the same seeded inputs, through the C ABI.
+
+Tolerances (derived in the design notes from the arithmetic):
+  Hessian   bit-exact on integer inputs; otherwise |ΔH| <= 1e-5 * rms-scaled
+            bound of fp32 accumulation over the token count.
+  U         max |ΔU| <= 2e-4 * max |U| (fp32 blocked factorisation, damped H).
+  codes     >= 99.9 % identical, every mismatch a rounding tie or downstream
+            of one (tests/parity.py).
+  scale     relative error <= 1e-5 on >= 99.9 % of groups.
+  surrogate relative error <= 1e-3 (the path's own loss vs the oracle's).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+import paper_2609_00049_gb300 as rq
+from paper_2609_00049_gb300 import layer
+from parity import compare_codes, scale_agreement, unpack
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_00049_gb300 import build as b
+    b.build()
+    rq.lib()
+
+
+def dev(a, dtype=torch.float32):
+    return torch.from_numpy(np.ascontiguousarray(a)).to("cuda", dtype)
+
+
+def bf16_dev(bits):
+    return torch.from_numpy(np.ascontiguousarray(bits).view(np.int16)).to("cuda").view(torch.bfloat16)
+
+
+def gpu_loss(Wq, W0, Hbar, F):
+    m, n = Wq.shape
+    out = torch.zeros(1, dtype=torch.float32, device="cuda")
+    ws = rq.workspace(rq.realq_surrogate_workspace_size(m, n))
+    rq.realq_surrogate_loss(Wq, W0, Hbar, F, out, ws)
+    return float(out.item())
+
+
+# --------------------------------------------------------------- Hessian ---
+def test_hessian_exact_on_integer_inputs():
+    case = synth.layer_case(20, 4, 200, 3000, integer_x=True)
+    H = torch.zeros(200, 200, device="cuda")
+    X = dev(case.Xhat)
+    rq.realq_hessian_accumulate(X[:1700], H)
+    rq.realq_hessian_accumulate(X[1700:], H)
+    Href, _ = oracle.hessian_sum([case.Xhat])
+    assert np.array_equal(H.cpu().numpy().astype(np.float64), Href)
+
+
+@pytest.mark.parametrize("n,T", [(300, 5000), (128, 65536), (97, 4099)])
+def test_hessian_bf16_and_cross_moment(n, T):
+    case = synth.layer_case(21, 4, n, T, perturbed=True, bf16=True, outliers=2)
+    Xh = dev(case.Xhat, torch.bfloat16)
+    Xf = dev(case.X, torch.bfloat16)
+    H, D, T_ = layer.accumulate([Xh], n, [Xf])
+    Href, _ = oracle.hessian_sum([case.Xhat])
+    Dref = oracle.cross_moment_sum([case.Xhat], [case.X])
+    scale = np.sqrt(np.outer(np.diag(Href), np.diag(Href)))
+    err = np.abs(H.cpu().numpy() - Href) / scale
+    assert err.max() < 2e-6 * np.sqrt(T)
+    dscale = np.sqrt(np.outer(np.diag(Dref @ Dref.T / T) + 1e-30, np.diag(Href)))
+    derr = np.abs(D.cpu().numpy() - Dref) / (np.abs(Dref).max())
+    assert derr.max() < 1e-4, dscale.shape
+    # bitwise repeatable (fixed-order split reduction)
+    H2, _, _ = layer.accumulate([Xh], n)
+    assert torch.equal(H, H2)
+
+
+# --------------------------------------------------------------- prepare ---
+@pytest.mark.parametrize("n,dead", [(256, ()), (300, (5, 77, 299)), (64, ())])
+def test_prepare_matches_oracle(n, dead):
+    case = synth.layer_case(22, 4, n, 4 * n, outliers=3, dead_cols=dead)
+    Href, T = oracle.hessian_sum([case.Xhat])
+    prep = layer.prepare(dev(Href), T, 0.01)
+    ref = oracle.prepare(Href, T, 0.01)
+    Uref = oracle.inverse_upper_cholesky(ref["Hd"])
+    U = prep.U.cpu().numpy().astype(np.float64)
+    assert np.abs(U - Uref).max() <= 2e-4 * np.abs(Uref).max()
+    assert np.all(np.tril(U, -1) == 0)
+    assert np.array_equal(prep.dead.cpu().numpy().astype(bool), ref["dead"])
+    assert np.allclose(prep.Hbar.cpu().numpy(), ref["Hbar"], rtol=1e-6, atol=0)
+
+
+def test_prepare_reports_not_spd():
+    n = 96
+    H = -torch.eye(n, device="cuda") * 10.0
+    with pytest.raises(rq.RealqError) as ei:
+        layer.prepare(H, 10, 0.01)
+    assert ei.value.status == rq.REALQ_ERR_NOT_SPD
+    assert ei.value.fail_col == n - 1
+
+
+# ------------------------------------------------------------ the sweep ---
+def _oracle_and_gpu(case, qkw, bgd=None, steps=1, with_next=False, b_global_start=1, B_total=1, use_dbar=False,
+                    w_bf16=False):
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    Ds = oracle.cross_moment_sum([case.Xhat], [case.X]) if use_dbar else None
+    obgd = None if bgd is None else {"lr": bgd, "steps_per_block": steps, "b_global_start": b_global_start,
+                                     "B_total": B_total}
+    orc = oracle.realq_sweep(case.W0, Hs, T, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
+                             block_size=qkw.get("block_size", 128), symmetric=bool(qkw.get("symmetric", 0)),
+                             bgd=obgd, F=case.F, F_next=case.F_next if with_next else None, D_sum=Ds)
+    Xh = dev(case.Xhat)
+    Xf = dev(case.X) if use_dbar else None
+    H, D, T_ = layer.accumulate([Xh], case.Xhat.shape[1], [Xf] if use_dbar else None)
+    prep = layer.prepare(H, T_, qkw.get("damp_frac", 0.01), D_sum=D)
+    q = rq.quant_cfg(**qkw)
+    b = None if bgd is None else rq.bgd_cfg(bgd, steps_per_block=steps, b_global_start=b_global_start,
+                                            B_total=B_total)
+    W0 = dev(case.W0, torch.bfloat16) if w_bf16 else dev(case.W0)
+    F = dev(case.F) if bgd is not None else None
+    Fn = dev(case.F_next) if (with_next and bgd is not None) else None
+    out = layer.quantize(W0, prep, q, b, F=F, F_next=Fn, use_dbar=use_dbar)
+    torch.cuda.synchronize()
+    return orc, out, prep, W0
+
+
+def _check(orc, out, case, qkw, bgd, loss_tol=1e-3, prep=None, W0=None):
+    n = case.W0.shape[1]
+    codes = unpack(out.codes.cpu().numpy(), n)
+    rep = compare_codes(codes, orc, qkw.get("block_size", 128), qkw.get("group_size", 128), bgd)
+    assert rep["frac_equal"] >= 0.999, rep
+    assert rep["n_unexplained"] == 0, rep
+    frac, med = scale_agreement(out.scale.cpu().numpy(), orc["scale"])
+    assert frac >= 0.999, (frac, med)
+    zero_eq = (out.zero.cpu().numpy().astype(np.int64) == orc["zero"]).mean()
+    assert zero_eq >= 0.999
+    # dequantized values are the grid points of the returned codes
+    g = qkw.get("group_size", 128) or n
+    s = out.scale.cpu().numpy()[:, np.arange(n) // g]
+    z = out.zero.cpu().numpy()[:, np.arange(n) // g].astype(np.float32)
+    deq = (s * (codes.astype(np.float32) - z)).astype(np.float32)
+    assert np.array_equal(deq, out.W.cpu().numpy())
+    L_or = oracle.surrogate_tokens(orc["deq"], case.W0, case.Xhat, case.X, case.F)
+    if prep is not None and case.X is None:
+        L_gpu = gpu_loss(out.W, W0, prep.Hbar, dev(case.F))
+        assert abs(L_gpu - L_or) <= loss_tol * L_or, (L_gpu, L_or)
+    return rep
+
+
+def test_identity_hessian_gives_rtn_codes():
+    r = synth.rng(23, "rtn-gpu")
+    m, n, T = 64, 384, 1000
+    W0 = (r.standard_normal((m, n)) * 0.02).astype(np.float32)
+    prep = layer.prepare(torch.eye(n, device="cuda") * T, T, 0.01)
+    for qkw in (dict(group_size=128), dict(group_size=0, symmetric=1), dict(group_size=32, bits=3),
+                dict(group_size=256, block_size=64)):
+        out = layer.quantize(dev(W0), prep, rq.quant_cfg(**qkw))
+        codes, deq, s, z = oracle.rtn(W0, qkw.get("bits", 4), qkw.get("group_size", 128), bool(qkw.get("symmetric", 0)))
+        assert np.array_equal(unpack(out.codes.cpu().numpy(), n), codes), qkw
+        assert np.array_equal(out.scale.cpu().numpy(), s)
+        assert np.array_equal(out.W.cpu().numpy().astype(np.float64), deq)
+
+
+def _fc_case():
+    wl = synth.workloads()["fc256x512"]
+    mod = wl.modules[0]
+    W0 = synth.weights(wl, mod)
+    X = synth.xhat_full(wl, "x")
+    return wl, synth.LayerCase(W0=W0, Xhat=X, X=None, F=synth.fisher(wl, mod))
+
+
+def test_fc256x512_gptq_mode():
+    wl, case = _fc_case()
+    qkw = dict(group_size=128, block_size=128)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw)
+    _check(orc, out, case, qkw, False, prep=prep, W0=W0)
+
+
+@pytest.mark.parametrize("steps", [1, 4])
+def test_fc256x512_realq(steps):
+    wl, case = _fc_case()
+    qkw = dict(group_size=128, block_size=128)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=wl.lr, steps=steps)
+    assert out.adam_t == orc["adam_t"] == 3 * steps
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+
+
+@pytest.mark.parametrize("qkw", [dict(group_size=64, block_size=64), dict(group_size=0, symmetric=1),
+                                 dict(group_size=32, block_size=128, bits=3), dict(group_size=256, block_size=128)])
+def test_ragged_shapes_and_quantizer_modes(qkw):
+    case = synth.layer_case(24, 200, 300, 1500, outliers=2, dead_cols=(7,))
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+
+
+def test_block_narrower_than_layer_and_single_block():
+    case = synth.layer_case(25, 40, 100, 800)
+    qkw = dict(group_size=0, block_size=128)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=1e-4)
+    assert out.adam_t == 0
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+
+
+def test_sliding_window():
+    case = synth.layer_case(26, 96, 320, 1200, with_next=True)
+    qkw = dict(group_size=64, block_size=64)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, with_next=True, b_global_start=3, B_total=9)
+    assert [round(x[1], 6) for x in orc["block_loss"]] == [round(1 - k / 8, 6) for k in range(2, 6)]
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+
+
+def test_perturbed_inputs_cross_moment():
+    case = synth.layer_case(27, 64, 192, 900, perturbed=True)
+    qkw = dict(group_size=64, block_size=64)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, use_dbar=True)
+    _check(orc, out, case, qkw, True)
+
+
+def test_bf16_weights():
+    case = synth.layer_case(28, 128, 256, 1024, bf16=True)
+    qkw = dict(group_size=128, block_size=128)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=3e-4, w_bf16=True)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+
+
+def test_resume_matches_single_call():
+    case = synth.layer_case(29, 64, 384, 1000)
+    Xh = dev(case.Xhat)
+    H, _, T = layer.accumulate([Xh], 384)
+    prep = layer.prepare(H, T)
+    q = rq.quant_cfg(group_size=128, block_size=128)
+    b = rq.bgd_cfg(1e-4)
+    F = dev(case.F)
+    W0 = dev(case.W0)
+    full = layer.quantize(W0, prep, q, b, F=F)
+    m, n = 64, 384
+    W = torch.empty(m, n, device="cuda")
+    codes = torch.empty(m, n // 2, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(m, 3, device="cuda")
+    zero = torch.empty(m, 3, dtype=torch.uint8, device="cuda")
+    am, av = torch.empty(m, n, device="cuda"), torch.empty(m, n, device="cuda")
+    ws = rq.workspace(rq.realq_quantize_workspace_size(m, n, q, b))
+    t = 0
+    for (b0, b1) in ((0, 1), (1, 3)):
+        t = rq.realq_quantize_layer(W0, prep.U, prep.Hbar, q, W, codes, scale, zero, dead=prep.dead, bcfg=b, F=F,
+                                    adam_m=am, adam_v=av, adam_t=t, block_begin=b0, block_end=b1, ws=ws)
+    assert t == full.adam_t == 2
+    assert torch.equal(codes, full.codes) and torch.equal(W, full.W)
+
+
+def test_nonfinite_weight_is_reported():
+    case = synth.layer_case(30, 32, 128, 400)
+    W0 = case.W0.copy()
+    W0[3, 5] = np.nan
+    H, _, T = layer.accumulate([dev(case.Xhat)], 128)
+    prep = layer.prepare(H, T)
+    q = rq.quant_cfg()
+    ws = rq.workspace(rq.realq_quantize_workspace_size(32, 128, q))
+    layer.quantize(dev(W0), prep, q, ws=ws)
+    with pytest.raises(rq.RealqError) as ei:
+        rq.realq_workspace_status(ws)
+    assert ei.value.status == rq.REALQ_ERR_NONFINITE
+
+
+def test_bgd_refine_single_adam_step():
+    case = synth.layer_case(31, 96, 256, 900)
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    r = synth.rng(31, "what")
+    What = (case.W0 + 0.004 * r.standard_normal(case.W0.shape)).astype(np.float32)
+    c0 = 100
+    Hbar = Hs / T
+    G = oracle.gradient(What.astype(np.float64), case.W0, Hbar, None, case.F)[:, c0:]
+    opt = oracle.Adam(What.shape, lr=1e-3)
+    ref = What.astype(np.float64).copy()
+    ref[:, c0:] -= opt.direction(G, slice(c0, 256))
+    W = dev(What)
+    am, av = torch.zeros_like(W), torch.zeros_like(W)
+    b = rq.bgd_cfg(1e-3)
+    ws = rq.workspace(rq.realq_bgd_workspace_size(96, 256))
+    t = rq.realq_bgd_refine(W, dev(case.W0), c0, dev(Hbar), dev(case.F), b, adam_m=am, adam_v=av, ws=ws)
+    assert t == 1
+    got = W.cpu().numpy().astype(np.float64)
+    assert np.array_equal(got[:, :c0], What[:, :c0].astype(np.float64))
+    # the first Adam step is lr * sign(g) unless |g| is near the fp32 rounding level of the gradient
+    sure = np.abs(G) > 1e-5 * np.abs(G).max()
+    d = np.abs(got[:, c0:] - ref[:, c0:])
+    assert d[sure].max() <= 1e-3 * 1e-3 + 2e-7 * np.abs(What).max()
+    assert d[~sure].max(initial=0.0) <= 2.0 * 1e-3 + 1e-6
+
+
+def test_surrogate_loss_matches_oracle():
+    case = synth.layer_case(32, 80, 160, 700)
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    r = synth.rng(32, "what")
+    What = (case.W0 + 0.003 * r.standard_normal(case.W0.shape)).astype(np.float32)
+    L_or = oracle.surrogate_tokens(What, case.W0, case.Xhat, None, case.F)
+    L_gpu = gpu_loss(dev(What), dev(case.W0), dev(Hs / T), dev(case.F))
+    assert abs(L_gpu - L_or) <= 1e-4 * L_or
