@@ -164,7 +164,8 @@ def gpu_arm(args, wl, rank, world):
         mods[mod.name] = dict(
             W=torch.empty(m, n, device=dev), codes=torch.empty(m, (n + 1) // 2, dtype=torch.uint8, device=dev),
             scale=torch.empty(m, ng, device=dev), zero=torch.empty(m, ng, dtype=torch.uint8, device=dev),
-            am=torch.empty(m, n, device=dev), av=torch.empty(m, n, device=dev), bcfg=bc,
+            am=torch.empty(m, n, device=dev), av=torch.empty(m, n, device=dev), disp=torch.empty(m, n, device=dev),
+            bcfg=bc,
             ws=rq.workspace(rq.realq_quantize_workspace_size(m, n, qcfg, bc, False, False), dev))
     # e2e-only buffers: pinned host outputs, device staging for chunked inputs
     E2E_CHUNK = 32768
@@ -182,7 +183,7 @@ def gpu_arm(args, wl, rank, world):
             p, s_in = mods[mod.name], st[mod.input]
             rq.realq_quantize_layer(wsrc[mod.name], s_in["U"], s_in["Hbar"], qcfg, p["W"], p["codes"], p["scale"],
                                     p["zero"], dead=s_in["dead"], bcfg=p["bcfg"], F=fsrc[mod.name],
-                                    adam_m=p["am"], adam_v=p["av"], ws=p["ws"])
+                                    adam_m=p["am"], adam_v=p["av"], bgd_disp=p["disp"], ws=p["ws"])
 
     def step_device():
         for name, spec in wl.inputs.items():

@@ -153,6 +153,14 @@ realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_to
  *             < min(block_end*B, n) hold the dequantized weights.
  *   adam_m, adam_v  m x n fp32 Adam moments (zeroed at block 0); adam_t (host)
  *             step counter in/out (set to 0 at block 0).
+ *   bgd_disp  m x n fp32: sum of all optimizer steps applied so far (zeroed
+ *             at block 0).  After the lazy batch update the OBS compensation
+ *             leaves the free columns at a stationary point of the damped
+ *             layer-local quadratic, so the surrogate gradient there is
+ *               P_R = (bgd_disp Hbar)_R + lambda (bgd_disp - (W - W0))_R
+ *                     (+ (W0 Dbar)_R),  0 on dead channels,
+ *             the same value as ((W - W0) Hbar)_R without its cancellation;
+ *             G = F_eff P_R.
  *   codes     m x ceil(n/2) bytes, two codes per byte, even column in the low
  *             nibble.  scale (fp32) and zero (uint8): m x ngroups, ngroups =
  *             ceil(n / group_size) (1 when group_size = 0).
@@ -168,7 +176,7 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
                                     const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
                                     const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg,
                                     const float *F, const float *F_next,
-                                    float *W_work, float *adam_m, float *adam_v, int64_t *adam_t,
+                                    float *W_work, float *adam_m, float *adam_v, float *bgd_disp, int64_t *adam_t,
                                     uint8_t *codes, float *scale, uint8_t *zero,
                                     void *W_deq, realq_dtype_t deq_dtype,
                                     int64_t block_begin, int64_t block_end,

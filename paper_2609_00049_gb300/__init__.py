@@ -78,7 +78,7 @@ _SIGS = {
     "realq_prepare_workspace_size": ([_i64], _sz),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
-                              ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
+                              ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
                               _i64, _i64, _vp, _sz], _int),
     "realq_quantize_workspace_size": ([_i64, _i64, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _int, _int],
                                       _sz),
@@ -212,7 +212,7 @@ def realq_quantize_workspace_size(m: int, n: int, qcfg: QuantCfg, bcfg: Optional
 def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch.Tensor], qcfg: QuantCfg,
                          W_work: torch.Tensor, codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *,
                          Dbar=None, dead=None, bcfg: Optional[BgdCfg] = None, F=None, F_next=None,
-                         adam_m=None, adam_v=None, adam_t: int = 0, W_deq=None,
+                         adam_m=None, adam_v=None, bgd_disp=None, adam_t: int = 0, W_deq=None,
                          block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None) -> int:
     """Runs blocks [block_begin, block_end) of the sweep; returns the Adam step counter."""
     m, n = W0.shape
@@ -224,12 +224,13 @@ def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch
     _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
     _need(adam_m, torch.float32, (m, n), "adam_m")
     _need(adam_v, torch.float32, (m, n), "adam_v")
+    _need(bgd_disp, torch.float32, (m, n), "bgd_disp")
     t = ctypes.c_int64(adam_t)
     wp, wb = _ws(ws)
     _check(lib().realq_quantize_layer(
         _stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar), _ptr(Dbar), _ptr(dead),
         ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
-        _ptr(W_work), _ptr(adam_m), _ptr(adam_v), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
+        _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
         _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
     return t.value
 

@@ -246,7 +246,8 @@ size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg
 realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
                                     const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
                                     const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg, const float *F,
-                                    const float *F_next, float *W_work, float *adam_m, float *adam_v, int64_t *adam_t,
+                                    const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                    int64_t *adam_t,
                                     uint8_t *codes, float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
                                     int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
     if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: m, n must be > 0");
@@ -258,7 +259,8 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
     REALQ_TRY(check_bcfg(bcfg));
     const int bgd = bcfg && bcfg->steps_per_block > 0;
     if (bgd) {
-        if (!Hbar || !F || !adam_t) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Block-GD needs Hbar, F and adam_t");
+        if (!Hbar || !F || !adam_t || !bgd_disp)
+            return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Block-GD needs Hbar, F, bgd_disp and adam_t");
         if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
             return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Adam needs adam_m and adam_v");
     }
@@ -282,7 +284,8 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
         p.b_global_start = bcfg->b_global_start; p.B_total = bcfg->B_total;
     }
     p.F = F; p.F_next = has_fn ? F_next : nullptr;
-    p.W = W_work; p.adam_m = adam_m; p.adam_v = adam_v; p.adam_t = adam_t;
+    p.W = W_work; p.adam_m = adam_m; p.adam_v = adam_v; p.disp = bgd ? bgd_disp : nullptr; p.adam_t = adam_t;
+    p.damp = qcfg->damp_frac;
     p.codes = codes; p.scale = scale; p.zero = zero; p.W_deq = W_deq; p.deq_dtype = deq_dtype;
     sweep_carve(p, ws, bgd, has_fn, has_db);
     cudaStream_t s = S(stream);

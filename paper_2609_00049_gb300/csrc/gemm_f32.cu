@@ -83,7 +83,17 @@ __global__ void __launch_bounds__(THREADS) sgemm_kernel(const GemmArgs g) {
             const float v = g.alpha * acc[i][j];
             if (EM == EPI_STORE) *c = v;
             else if (EM == EPI_SUB) *c = *c - v;
-            else *c = v + g.R[gi * g.ldr + gj];
+            else if (EM == EPI_BIAS) *c = v + g.R[gi * g.ldr + gj];
+            else {
+                const int64_t col = g.col0 + gj;
+                const int64_t w = gi * g.ldw + col;
+                const float w0 = g.w0_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16 *>(g.W0c)[w])
+                                           : static_cast<const float *>(g.W0c)[w];
+                float p = v + (*g.lam) * (g.Ad[w] - (g.Wc[w] - w0));
+                if (g.R) p += g.R[gi * g.ldr + gj];
+                if (g.dead && g.dead[col]) p = 0.f;
+                *c = p;
+            }
         }
     }
 }
@@ -95,7 +105,8 @@ realq_status_t dispatch_epi(cudaStream_t s, EpiMode em, const GemmArgs &g, const
         Launch L(name, s);
         if (em == EPI_STORE) sgemm_kernel<AM, EPI_STORE><<<grid, THREADS, 0, s>>>(g);
         else if (em == EPI_SUB) sgemm_kernel<AM, EPI_SUB><<<grid, THREADS, 0, s>>>(g);
-        else sgemm_kernel<AM, EPI_BIAS><<<grid, THREADS, 0, s>>>(g);
+        else if (em == EPI_BIAS) sgemm_kernel<AM, EPI_BIAS><<<grid, THREADS, 0, s>>>(g);
+        else sgemm_kernel<AM, EPI_BGD_P><<<grid, THREADS, 0, s>>>(g);
     }
     return check_launch(name);
 }

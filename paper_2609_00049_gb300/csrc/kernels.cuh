@@ -19,6 +19,10 @@ enum EpiMode {
     EPI_STORE = 0,    // C = alpha * acc
     EPI_SUB = 1,      // C = C - alpha * acc
     EPI_BIAS = 2,     // C = alpha * acc + R[i * ldr + j]
+    // Block-GD gradient after the lazy OBS update (column c = col0 + j):
+    // C = alpha * acc + lam * (Ad[i][c] - (Wc[i][c] - W0c[i][c])) (+ R[i * ldr + j]),
+    // and C = 0 on dead channels; Ad, Wc, W0c have leading dimension ldw.
+    EPI_BGD_P = 3,
 };
 struct GemmArgs {
     int64_t M, N, K;
@@ -28,6 +32,9 @@ struct GemmArgs {
     float *C; int64_t ldc;
     const float *R; int64_t ldr;
     float alpha;
+    // EPI_BGD_P operands
+    const float *Ad; const float *Wc; const void *W0c; int w0_bf16;
+    const uint8_t *dead; const float *lam; int64_t col0; int64_t ldw;
 };
 realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name);
 
@@ -56,12 +63,14 @@ struct SweepPlan {
     float lr, beta1, beta2, eps;
     int b_global_start, B_total;
     const float *F, *F_next;
-    float *W, *adam_m, *adam_v;
+    float damp;
+    float *W, *adam_m, *adam_v, *disp;
     int64_t *adam_t;
     uint8_t *codes; float *scale; uint8_t *zero;
     void *W_deq; realq_dtype_t deq_dtype;
     // workspace pieces
     int *status;
+    float *lam;
     float *Et, *P, *G, *Feff, *R0;
 };
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar);

@@ -158,22 +158,44 @@ __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) 
     if (bad) atomicOr(a.status, ST_NONFINITE);
 }
 
+// One optimizer step on the free columns c0..n-1; the applied step is also
+// accumulated into D (the optimizer displacement) when D is given.
 __global__ void adam_kernel(int64_t m, int64_t r, int64_t n, int64_t c0, const float *G, float *W, float *mA,
-                            float *vA, float lr, float b1, float b2, float eps, float bc1, float bc2, int sgd) {
+                            float *vA, float *D, float lr, float b1, float b2, float eps, float bc1, float bc2,
+                            int sgd) {
     const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (idx >= m * r) return;
     const int64_t i = idx / r, c = idx % r;
     const int64_t w = i * n + c0 + c;
     const float g = G[idx];
+    float step;
     if (sgd) {
-        W[w] -= lr * g;
-        return;
+        step = lr * g;
+    } else {
+        const float mv = b1 * mA[w] + (1.f - b1) * g;
+        const float vv = b2 * vA[w] + (1.f - b2) * g * g;
+        mA[w] = mv;
+        vA[w] = vv;
+        step = lr * (mv / bc1) / (sqrtf(vv / bc2) + eps);
     }
-    const float mv = b1 * mA[w] + (1.f - b1) * g;
-    const float vv = b2 * vA[w] + (1.f - b2) * g * g;
-    mA[w] = mv;
-    vA[w] = vv;
-    W[w] -= lr * (mv / bc1) / (sqrtf(vv / bc2) + eps);
+    W[w] -= step;
+    if (D) D[w] -= step;
+}
+
+// lambda = damp * mean(diag(Hbar) with dead channels counted as 1), the same
+// fixed-order fp64 reduction as the preparation step.
+__global__ void lambda_kernel(int64_t n, const float *Hbar, const uint8_t *dead, float damp, float *lam_out) {
+    __shared__ double red[1024];
+    double s = 0.0;
+    for (int64_t j = threadIdx.x; j < n; j += blockDim.x)
+        s += (dead && dead[j]) ? 1.0 : (double)Hbar[j * n + j];
+    red[threadIdx.x] = s;
+    __syncthreads();
+    for (int w = blockDim.x / 2; w > 0; w >>= 1) {
+        if ((int)threadIdx.x < w) red[threadIdx.x] += red[threadIdx.x + w];
+        __syncthreads();
+    }
+    if (threadIdx.x == 0) *lam_out = (float)((double)damp * (red[0] / (double)n));
 }
 
 __global__ void feff_kernel(int64_t count, const float *F, const float *Fn, float alpha, float *out) {
@@ -252,7 +274,7 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 }  // namespace
 
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar) {
-    size_t b = align_up(sizeof(int)) + align_up((size_t)block * m * sizeof(float));
+    size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
     if (has_bgd) {
         b += 2 * align_up((size_t)m * n * sizeof(float));
         if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
@@ -264,6 +286,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar) {
     Carve cv(ws);
     p.status = cv.take<int>(1);
+    p.lam = cv.take<float>(1);
     p.Et = cv.take<float>((size_t)p.block * p.m);
     p.P = p.G = p.Feff = p.R0 = nullptr;
     if (has_bgd) {
@@ -289,6 +312,7 @@ realq_status_t sweep_init(cudaStream_t s, SweepPlan &p) {
             REALQ_CUDA_TRY(cudaMemsetAsync(p.adam_m, 0, (size_t)mn * sizeof(float), s));
             REALQ_CUDA_TRY(cudaMemsetAsync(p.adam_v, 0, (size_t)mn * sizeof(float), s));
         }
+        if (p.disp) REALQ_CUDA_TRY(cudaMemsetAsync(p.disp, 0, (size_t)mn * sizeof(float), s));
         *p.adam_t = 0;
     }
     return REALQ_OK;
@@ -319,18 +343,33 @@ static realq_status_t fisher_for(cudaStream_t s, SweepPlan &p, float alpha, cons
     return check_launch("fisher_blend");
 }
 
-static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const float *Fuse) {
+// One Block-GD step on columns c0..n-1.  identity = 1 (inside the sweep, right
+// after the lazy batch update): P from the optimizer displacement through the
+// OBS stationarity identity; identity = 0: P = (W - W0) Hbar (+ W0 Dbar).
+static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const float *Fuse, int identity) {
     const int64_t r = p.n - c0;
     GemmArgs g{};
-    g.M = p.m; g.N = r; g.K = p.n;
-    g.A = p.W; g.lda = p.n;
-    g.Y = p.W0; g.ldy = p.n;
-    g.B = p.Hbar + c0; g.ldb = p.n;
+    g.M = p.m; g.N = r;
     g.C = p.P; g.ldc = r;
     g.R = p.R0 ? p.R0 + c0 : nullptr; g.ldr = p.n;
     g.alpha = 1.f;
-    REALQ_TRY(gemm_f32(s, p.w_dtype == REALQ_BF16 ? A_DIFF_BF16 : A_DIFF_F32, p.R0 ? EPI_BIAS : EPI_STORE, g,
-                       "bgd_p_gemm"));
+    if (identity) {
+        // columns of the first block never received a step: skip them in K
+        const int64_t k0 = std::min<int64_t>(p.block, c0);
+        g.K = p.n - k0;
+        g.A = p.disp + k0; g.lda = p.n;
+        g.B = p.Hbar + k0 * p.n + c0; g.ldb = p.n;
+        g.Ad = p.disp; g.Wc = p.W; g.W0c = p.W0; g.w0_bf16 = p.w_dtype == REALQ_BF16;
+        g.dead = p.dead; g.lam = p.lam; g.col0 = c0; g.ldw = p.n;
+        REALQ_TRY(gemm_f32(s, A_ROW, EPI_BGD_P, g, "bgd_p_gemm"));
+    } else {
+        g.K = p.n;
+        g.A = p.W; g.lda = p.n;
+        g.Y = p.W0; g.ldy = p.n;
+        g.B = p.Hbar + c0; g.ldb = p.n;
+        REALQ_TRY(gemm_f32(s, p.w_dtype == REALQ_BF16 ? A_DIFF_BF16 : A_DIFF_F32, p.R0 ? EPI_BIAS : EPI_STORE, g,
+                           "bgd_p_gemm"));
+    }
     GemmArgs h{};
     h.M = p.m; h.N = r; h.K = p.m;
     h.A = Fuse; h.lda = p.m;
@@ -343,8 +382,8 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
     const double bc2 = 1.0 - std::pow((double)p.beta2, (double)t);
     {
         Launch L("bgd_adam", s);
-        adam_kernel<<<blocks_for(p.m * r), 256, 0, s>>>(p.m, r, p.n, c0, p.G, p.W, p.adam_m, p.adam_v, p.lr, p.beta1,
-                                                         p.beta2, p.eps, (float)bc1, (float)bc2,
+        adam_kernel<<<blocks_for(p.m * r), 256, 0, s>>>(p.m, r, p.n, c0, p.G, p.W, p.adam_m, p.adam_v, p.disp, p.lr,
+                                                         p.beta1, p.beta2, p.eps, (float)bc1, (float)bc2,
                                                          p.optimizer == REALQ_OPT_SGD);
     }
     return check_launch("bgd_adam");
@@ -355,7 +394,7 @@ realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float a
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
     const float *Fuse = nullptr;
     REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
-    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, col_start, Fuse));
+    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, col_start, Fuse, 0));
     return REALQ_OK;
 }
 
@@ -364,7 +403,8 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     const int64_t bs = b * B;
     const int64_t be = std::min<int64_t>(bs + B, p.n);
     const int kb = (int)(be - bs);
-    const int params_here = p.group <= B;
+    // a single group no wider than a block is handled inside the block kernel
+    const int params_here = p.group <= B || (p.group >= p.n && p.n <= B);
     if (!params_here && bs % p.group == 0) {
         Launch L("group_params", s);
         group_params_kernel<<<ceil_div(p.m, 8), 256, 0, s>>>(p.m, p.n, p.W, bs, std::min<int64_t>(bs + p.group, p.n),
@@ -378,7 +418,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     qa.g = p.group; qa.ngroups = p.ngroups; qa.bits = p.bits; qa.sym = p.sym;
     qa.scale = p.scale; qa.zero = p.zero; qa.codes = p.codes; qa.ncb = (p.n + 1) / 2;
     qa.Et = p.Et; qa.status = p.status;
-    const int Gk = params_here ? p.group : 0;
+    const int Gk = !params_here ? 0 : (p.group <= B ? p.group : B);
     if (B == 128) REALQ_TRY(launch_qb_g<128>(s, qa, Gk));
     else if (B == 64) REALQ_TRY(launch_qb_g<64>(s, qa, Gk));
     else REALQ_TRY(launch_qb_g<32>(s, qa, Gk));
@@ -405,12 +445,18 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     if (p.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(p.B_total - 1));
     const float *Fuse = nullptr;
     REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
-    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, be, Fuse));
+    for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, be, Fuse, 1));
     return REALQ_OK;
 }
 
 realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p) {
-    if (p.Dbar && p.bgd_steps > 0) return compute_r0(s, p);
+    if (p.bgd_steps <= 0) return REALQ_OK;
+    {
+        Launch L("bgd_lambda", s);
+        lambda_kernel<<<1, 1024, 0, s>>>(p.n, p.Hbar, p.dead, p.damp, p.lam);
+    }
+    REALQ_TRY(check_launch("bgd_lambda"));
+    if (p.Dbar) return compute_r0(s, p);
     return REALQ_OK;
 }
 

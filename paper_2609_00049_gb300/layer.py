@@ -79,10 +79,12 @@ def quantize(W0: torch.Tensor, prep: Prepared, qcfg: QuantCfg, bcfg: Optional[Bg
     zero = torch.empty((m, ngroups), dtype=torch.uint8, device=dev)
     am = torch.empty((m, n), dtype=torch.float32, device=dev) if bgd else None
     av = torch.empty((m, n), dtype=torch.float32, device=dev) if bgd else None
+    disp = torch.empty((m, n), dtype=torch.float32, device=dev) if bgd else None
     if ws is None:
         ws = workspace(realq_quantize_workspace_size(m, n, qcfg, bcfg, F_next is not None, Dbar is not None), dev)
     t = realq_quantize_layer(W0, prep.U, prep.Hbar, qcfg, W, codes, scale, zero, Dbar=Dbar, dead=prep.dead,
-                             bcfg=bcfg, F=F, F_next=F_next, adam_m=am, adam_v=av, ws=ws, stream=stream)
+                             bcfg=bcfg, F=F, F_next=F_next, adam_m=am, adam_v=av, bgd_disp=disp, ws=ws,
+                             stream=stream)
     return Quantized(codes, scale, zero, W, t)
 
 

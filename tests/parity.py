@@ -43,6 +43,7 @@ def compare_codes(gpu_codes: np.ndarray, orc: dict, block_size: int, group_size:
     if bgd and first_block is not None:
         explained[:, (first_block + 1) * block_size:] = True
     unexpl = mism & ~explained
+    compare_codes.last_explained = explained
     return {
         "frac_equal": 1.0 - float(mism.mean()),
         "n_mismatch": int(mism.sum()),
@@ -52,6 +53,16 @@ def compare_codes(gpu_codes: np.ndarray, orc: dict, block_size: int, group_size:
     }
 
 
-def scale_agreement(gpu_scale: np.ndarray, orc_scale: np.ndarray, rtol: float = 1e-5):
+def scale_agreement(gpu_scale: np.ndarray, orc_scale: np.ndarray, group_size: int, rtol: float = 1e-5,
+                    explained: np.ndarray = None):
+    """(fraction of groups within rtol, median relative error, groups off by more
+    than rtol that are not downstream of an accepted tie)."""
     rel = np.abs(gpu_scale.astype(np.float64) - orc_scale.astype(np.float64)) / np.abs(orc_scale.astype(np.float64))
-    return float((rel <= rtol).mean()), float(np.median(rel))
+    bad = rel > rtol
+    n_unexpl = int(bad.sum())
+    if explained is not None:
+        m, n = explained.shape
+        g = group_size if group_size > 0 else n
+        first_cols = np.arange(gpu_scale.shape[1]) * g
+        n_unexpl = int((bad & ~explained[:, first_cols]).sum())
+    return float((~bad).mean()), float(np.median(rel)), n_unexpl

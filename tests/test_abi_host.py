@@ -62,7 +62,8 @@ def _ql(L, m=256, n=512, qcfg=None, bcfg=None, F=FAKE, W0=FAKE, ws=FAKE, ws_byte
     t = ctypes.c_int64(0)
     return L.realq_quantize_layer(None, m, n, W0, 0, FAKE, FAKE, None, None, ctypes.byref(q),
                                   ctypes.byref(bcfg) if bcfg is not None else None, F, None, FAKE, FAKE, FAKE,
-                                  ctypes.byref(t), FAKE, FAKE, FAKE, None, 0, blocks[0], blocks[1], ws, ws_bytes)
+                                  FAKE, ctypes.byref(t), FAKE, FAKE, FAKE, None, 0, blocks[0], blocks[1], ws,
+                                  ws_bytes)
 
 
 def test_argument_validation(L):

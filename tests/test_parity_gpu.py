@@ -128,10 +128,13 @@ def _check(orc, out, case, qkw, bgd, loss_tol=1e-3, prep=None, W0=None):
     n = case.W0.shape[1]
     codes = unpack(out.codes.cpu().numpy(), n)
     rep = compare_codes(codes, orc, qkw.get("block_size", 128), qkw.get("group_size", 128), bgd)
+    frac, med, s_unexpl = scale_agreement(out.scale.cpu().numpy(), orc["scale"], qkw.get("group_size", 128),
+                                          explained=compare_codes.last_explained)
+    print(f"\nparity {qkw} bgd={bgd}: {rep} scale_within_1e-5={frac:.5f} median_rel={med:.2e} "
+          f"scale_unexplained={s_unexpl}")
     assert rep["frac_equal"] >= 0.999, rep
     assert rep["n_unexplained"] == 0, rep
-    frac, med = scale_agreement(out.scale.cpu().numpy(), orc["scale"])
-    assert frac >= 0.999, (frac, med)
+    assert s_unexpl == 0 and frac >= 0.99, (frac, med, s_unexpl)
     zero_eq = (out.zero.cpu().numpy().astype(np.int64) == orc["zero"]).mean()
     assert zero_eq >= 0.999
     # dequantized values are the grid points of the returned codes
@@ -239,11 +242,13 @@ def test_resume_matches_single_call():
     scale = torch.empty(m, 3, device="cuda")
     zero = torch.empty(m, 3, dtype=torch.uint8, device="cuda")
     am, av = torch.empty(m, n, device="cuda"), torch.empty(m, n, device="cuda")
+    disp = torch.empty(m, n, device="cuda")
     ws = rq.workspace(rq.realq_quantize_workspace_size(m, n, q, b))
     t = 0
     for (b0, b1) in ((0, 1), (1, 3)):
         t = rq.realq_quantize_layer(W0, prep.U, prep.Hbar, q, W, codes, scale, zero, dead=prep.dead, bcfg=b, F=F,
-                                    adam_m=am, adam_v=av, adam_t=t, block_begin=b0, block_end=b1, ws=ws)
+                                    adam_m=am, adam_v=av, bgd_disp=disp, adam_t=t, block_begin=b0, block_end=b1,
+                                    ws=ws)
     assert t == full.adam_t == 2
     assert torch.equal(codes, full.codes) and torch.equal(W, full.W)
 
