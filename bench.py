@@ -340,7 +340,7 @@ def roofline(wl, prof, steps, peaks):
     # algorithmic work per step of each kernel family
     hess_flops = sum(s.T * s.n * (s.n + 1) for s in wl.inputs.values())       # symmetric X^T X
     per_step["hessian_syrk_simt"] = ("tensor", hess_flops, "TFLOP/s")
-    per_step["hessian_syrk"] = ("tensor", hess_flops, "TFLOP/s")
+    per_step["hessian_syrk_tc"] = ("tensor", hess_flops, "TFLOP/s")
     bgd_p = bgd_g = trail = 0
     serial_bytes = 0
     for md in wl.modules:

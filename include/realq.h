@@ -112,8 +112,12 @@ typedef struct {
 realq_status_t realq_hessian_accumulate(realq_stream_t stream, int64_t n, int64_t T_chunk,
                                         const void *X_hat, const void *X_fp, realq_dtype_t x_dtype,
                                         float *H_sum, float *D_sum, void *ws, size_t ws_bytes);
-/* Workspace for one accumulate call (token-split partial sums, reduced in a
- * fixed order so results are bitwise repeatable); 0 means ws may be NULL. */
+/* Workspace for one accumulate call: a status word (first 256 bytes) and the
+ * token-split partial sums, reduced in a fixed order so results are bitwise
+ * repeatable.  ws may be NULL (no split, no status word).  bf16 inputs with
+ * n % 8 == 0 and a 16-byte aligned X_hat run on the tensor cores; a tile whose
+ * bounded pipeline wait gave up is written as NaN and the status word gets a
+ * timeout bit, read with realq_workspace_status(). */
 size_t realq_hessian_workspace_size(int64_t n, int64_t T_chunk, realq_dtype_t x_dtype, int has_X_fp);
 
 /* Step 2. Preparation (Alg. 1: Hessian and its inverse; the inverse used by
@@ -205,8 +209,9 @@ realq_status_t realq_surrogate_loss(realq_stream_t stream, int64_t m, int64_t n,
                                     void *ws, size_t ws_bytes);
 size_t realq_surrogate_workspace_size(int64_t m, int64_t n);
 
-/* Synchronizes `stream`, returns the device status word recorded in a
- * quantize workspace (REALQ_OK, REALQ_ERR_NONFINITE) and clears it. */
+/* Synchronizes `stream`, returns the device status word recorded at the start
+ * of a Hessian or quantize workspace (REALQ_OK, REALQ_ERR_TIMEOUT,
+ * REALQ_ERR_NONFINITE) and clears it. */
 realq_status_t realq_workspace_status(realq_stream_t stream, void *ws, size_t ws_bytes);
 
 /* Diagnostics. */

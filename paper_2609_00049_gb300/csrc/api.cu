@@ -343,6 +343,7 @@ realq_status_t realq_workspace_status(realq_stream_t stream, void *ws, size_t ws
     REALQ_CUDA_TRY(cudaMemcpyAsync(&st, ws, sizeof(int), cudaMemcpyDeviceToHost, S(stream)));
     REALQ_CUDA_TRY(cudaStreamSynchronize(S(stream)));
     REALQ_CUDA_TRY(cudaMemsetAsync(ws, 0, sizeof(int), S(stream)));
+    if (st & ST_TIMEOUT) return fail(REALQ_ERR_TIMEOUT, "a bounded device-side wait gave up");
     if (st & ST_NONFINITE) return fail(REALQ_ERR_NONFINITE, "non-finite weight met during the sweep");
     return REALQ_OK;
 }

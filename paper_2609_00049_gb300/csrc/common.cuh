@@ -33,6 +33,7 @@ enum : int {
     ST_OK = 0,
     ST_NONFINITE = 1,
     ST_NOT_SPD = 2,
+    ST_TIMEOUT = 4,
 };
 
 constexpr size_t kAlign = 256;

@@ -119,18 +119,6 @@ __global__ void hess_reduce_kernel(int64_t n, int splits, const float *part, flo
     if (MODE == 0 && ti > tj) out[j * n + i] += s;
 }
 
-int g_num_sms = 0;
-int num_sms() {
-    if (g_num_sms == 0) {
-        int dev = 0, v = 0;
-        if (cudaGetDevice(&dev) == cudaSuccess && cudaDeviceGetAttribute(&v, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess)
-            g_num_sms = v;
-        else
-            g_num_sms = 152;
-    }
-    return g_num_sms;
-}
-
 template <typename TX>
 realq_status_t run(cudaStream_t s, int64_t n, int64_t T, const TX *X, const TX *Xf, float *H, float *D, void *ws,
                    size_t ws_bytes) {
@@ -144,43 +132,57 @@ realq_status_t run(cudaStream_t s, int64_t n, int64_t T, const TX *X, const TX *
     float *partH = static_cast<float *>(ws);
     float *partD = partH + (size_t)splits * n * n;
     const int direct = splits == 1;
-    {
-        Launch L("hessian_syrk_simt", s);
-        hess_kernel<TX, 0><<<dim3((unsigned)lower, splits), THREADS, 0, s>>>(n, T, X, nullptr, H, partH, tper, direct);
-    }
-    REALQ_TRY(check_launch("hessian_syrk_simt"));
-    if (Xf) {
-        Launch L("hessian_cross_simt", s);
-        hess_kernel<TX, 1><<<dim3((unsigned)((int64_t)nt * nt), splits), THREADS, 0, s>>>(n, T, X, Xf, D, partD, tper,
-                                                                                         direct);
-    }
-    REALQ_TRY(check_launch("hessian_cross_simt"));
-    if (!direct) {
-        const int64_t tot = n * n;
-        const unsigned blocks = (unsigned)((tot + 255) / 256);
+    if (H) {
         {
-            Launch L("hessian_reduce", s);
-            hess_reduce_kernel<0><<<blocks, 256, 0, s>>>(n, splits, partH, H);
+            Launch L("hessian_syrk_simt", s);
+            hess_kernel<TX, 0><<<dim3((unsigned)lower, splits), THREADS, 0, s>>>(n, T, X, nullptr, H, partH, tper,
+                                                                                 direct);
         }
-        REALQ_TRY(check_launch("hessian_reduce"));
-        if (Xf) {
-            {
-                Launch L("hessian_reduce", s);
-                hess_reduce_kernel<1><<<blocks, 256, 0, s>>>(n, splits, partD, D);
-            }
-            REALQ_TRY(check_launch("hessian_reduce"));
+        REALQ_TRY(check_launch("hessian_syrk_simt"));
+        if (!direct) REALQ_TRY(hessian_reduce(s, n, splits, partH, H, 0));
+    }
+    if (Xf) {
+        {
+            Launch L("hessian_cross_simt", s);
+            hess_kernel<TX, 1><<<dim3((unsigned)((int64_t)nt * nt), splits), THREADS, 0, s>>>(n, T, X, Xf, D, partD,
+                                                                                             tper, direct);
         }
+        REALQ_TRY(check_launch("hessian_cross_simt"));
+        if (!direct) REALQ_TRY(hessian_reduce(s, n, splits, partD, D, 1));
     }
     return REALQ_OK;
 }
 
 }  // namespace
 
+int num_sms() {
+    static int v = 0;
+    if (v == 0) {
+        int dev = 0, c = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && c > 0)
+            v = c;
+        else
+            v = 152;
+    }
+    return v;
+}
+
+realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float *part, float *out, int mode) {
+    const unsigned blocks = (unsigned)((n * n + 255) / 256);
+    {
+        Launch L("hessian_reduce", s);
+        if (mode == 0) hess_reduce_kernel<0><<<blocks, 256, 0, s>>>(n, splits, part, out);
+        else hess_reduce_kernel<1><<<blocks, 256, 0, s>>>(n, splits, part, out);
+    }
+    return check_launch("hessian_reduce");
+}
+
 int hessian_splits(int64_t n, int64_t T, int sms) {
     const int nt = ceil_div(n, TB);
     const int64_t lower = (int64_t)nt * (nt + 1) / 2;
-    int64_t want = (2 * (int64_t)sms + lower - 1) / lower;
-    const int64_t by_tokens = T / 2048;
+    int64_t want = (sms + lower / 2) / lower;       // nearest whole number of waves
+    const int64_t by_tokens = T / 4096;              // at least 4096 tokens per split
     if (want > by_tokens) want = by_tokens;
     if (want > 16) want = 16;
     if (want < 1) want = 1;
@@ -188,18 +190,30 @@ int hessian_splits(int64_t n, int64_t T, int sms) {
 }
 
 size_t hessian_ws_bytes(int64_t n, int64_t T, int has_xfp) {
+    size_t b = align_up(sizeof(int));
     const int splits = hessian_splits(n, T, 152);
-    if (splits <= 1) return 0;
-    return (size_t)splits * n * n * sizeof(float) * (has_xfp ? 2 : 1);
+    if (splits > 1) b += (size_t)splits * n * n * sizeof(float) * (has_xfp ? 2 : 1);
+    return b;
 }
 
 realq_status_t hessian_accumulate(cudaStream_t s, int64_t n, int64_t T, const void *X, const void *Xfp,
                                   realq_dtype_t dt, float *H, float *D, void *ws, size_t ws_bytes) {
     if (T == 0) return REALQ_OK;
+    int *err = nullptr;
+    char *pw = nullptr;
+    size_t pbytes = 0;
+    if (ws && ws_bytes >= align_up(sizeof(int))) {
+        err = static_cast<int *>(ws);
+        pw = static_cast<char *>(ws) + align_up(sizeof(int));
+        pbytes = ws_bytes - align_up(sizeof(int));
+    }
+    const bool tc_path = dt == REALQ_BF16 && hessian_tc_eligible(n, T, X);
+    if (tc_path) REALQ_TRY(hessian_syrk_tc(s, n, T, X, H, err, pw, pbytes, num_sms()));
+    float *Hs = tc_path ? nullptr : H;
     if (dt == REALQ_BF16)
         return run<__nv_bfloat16>(s, n, T, static_cast<const __nv_bfloat16 *>(X),
-                                  static_cast<const __nv_bfloat16 *>(Xfp), H, D, ws, ws_bytes);
-    return run<float>(s, n, T, static_cast<const float *>(X), static_cast<const float *>(Xfp), H, D, ws, ws_bytes);
+                                  static_cast<const __nv_bfloat16 *>(Xfp), Hs, D, pw, pbytes);
+    return run<float>(s, n, T, static_cast<const float *>(X), static_cast<const float *>(Xfp), Hs, D, pw, pbytes);
 }
 
 }  // namespace realq

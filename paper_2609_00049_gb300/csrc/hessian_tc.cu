@@ -1,0 +1,245 @@
+// Step a2 (Sec. 3.2) on the 5th-generation tensor cores: H_sum += X̂^T X̂ for
+// bf16 calibration activations, fp32 accumulation in TMEM.
+//
+// One CTA owns one 128 x 128 tile (i-block >= j-block) of H and a contiguous
+// range of tokens.  X̂ is token-major (T x n), so both MMA operands are read
+// MN-major straight from the activation rows: a TMA box of 64 tokens x 64
+// channels (128-byte rows, 128-byte swizzle) is one canonical MN-major atom
+// stack; two boxes make the 128-channel operand (LBO = 8 KB between them,
+// SBO = 1 KB between 8-token groups).  Diagonal tiles load one operand.
+//
+// Roles (128 threads): warp 0 lane 0 issues TMA into a STAGES-deep ring,
+// warp 1 lane 0 issues tcgen05.mma (4 x K16 per 64-token stage) and frees
+// stages with tcgen05.commit; afterwards all four warps drain the 128 x 128
+// fp32 accumulator from TMEM (warp w owns lanes 32w..32w+31) and add it to H
+// and its mirror, or store it as a partial sum when tokens are split.
+// Every wait is bounded; on a timeout the tile is written as NaN (so the
+// factorisation of H reports a non-finite pivot), the workspace status word
+// gets ST_TIMEOUT, and the kernel still frees TMEM and returns.
+#include "kernels.cuh"
+#include "tc.cuh"
+
+#include <mutex>
+
+namespace realq {
+namespace {
+
+constexpr int TILE = 128;
+constexpr int KSTAGE = 64;                       // tokens per pipeline stage
+constexpr int STAGES = 6;
+constexpr int OP_BYTES = TILE * KSTAGE * 2;      // one 128 x 64 bf16 operand tile
+constexpr int BOX_BYTES = 64 * KSTAGE * 2;       // one TMA box (64 channels x 64 tokens)
+constexpr int STAGE_BYTES = 2 * OP_BYTES;
+constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr uint32_t IDESC = tc::idesc_bf16_f32(TILE, TILE, 1, 1);
+
+__device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
+    int r = (int)((sqrt(8.0 * (double)idx + 1.0) - 1.0) * 0.5);
+    while ((int64_t)(r + 1) * (r + 2) / 2 <= idx) ++r;
+    while ((int64_t)r * (r + 1) / 2 > idx) --r;
+    ti = r;
+    tj = (int)(idx - (int64_t)r * (r + 1) / 2);
+}
+
+__global__ void __launch_bounds__(128, 1)
+    hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, int64_t n, int64_t T, int64_t tper, float *H,
+                   float *part, int direct, int *err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
+    uint64_t *empty = full + STAGES;
+    uint64_t *accb = empty + STAGES;
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(accb + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    int ti, tj;
+    lower_tile(blockIdx.x, ti, tj);
+    const bool diag = ti == tj;
+    const int i0 = ti * TILE, j0 = tj * TILE;
+    const int64_t t_begin = (int64_t)blockIdx.y * tper;
+    const int64_t t_end = min(T, t_begin + tper);
+    const int nk = t_end > t_begin ? (int)((t_end - t_begin + KSTAGE - 1) / KSTAGE) : 0;
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            tc::mbar_init(tc::smem_u32(&full[s]), 1);
+            tc::mbar_init(tc::smem_u32(&empty[s]), 1);
+        }
+        tc::mbar_init(tc::smem_u32(accb), 1);
+        *abort_flag = 0;
+        tc::fence_barrier_init();
+        tc::prefetch_tmap(&tmap);
+    }
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), TILE);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        int it = 0;
+        for (; it < nk; ++it) {
+            const int s = it % STAGES;
+            const uint32_t r = (uint32_t)(it / STAGES);
+            if (!tc::mbar_wait(tc::smem_u32(&empty[s]), (r & 1u) ^ 1u, abort_flag)) {
+                *abort_flag = 1;
+                break;
+            }
+            const uint32_t fb = tc::smem_u32(&full[s]);
+            tc::mbar_arrive_expect_tx(fb, diag ? OP_BYTES : 2 * OP_BYTES);
+            const int y = (int)(t_begin + (int64_t)it * KSTAGE);
+            const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
+            tc::tma_load_2d(a, &tmap, fb, i0, y);
+            tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
+            if (!diag) {
+                tc::tma_load_2d(a + OP_BYTES, &tmap, fb, j0, y);
+                tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, &tmap, fb, j0 + 64, y);
+            }
+        }
+        // on abort, let the copies already issued land before the CTA exits
+        if (*abort_flag) {
+            int never = 0;
+            for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k)
+                tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (uint32_t)(k / STAGES) & 1u, &never, 100000000ull);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        for (int it = 0; it < nk; ++it) {
+            const int s = it % STAGES;
+            const uint32_t r = (uint32_t)(it / STAGES);
+            if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc::fence_after_sync();
+            const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
+            const uint32_t b = diag ? a : a + OP_BYTES;
+#pragma unroll
+            for (int k = 0; k < KSTAGE / 16; ++k) {
+                const uint64_t da = tc::smem_desc(a + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
+                const uint64_t db = tc::smem_desc(b + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
+                tc::mma_bf16_ss(tmem, da, db, IDESC, (it > 0 || k > 0) ? 1u : 0u);
+            }
+            tc::mma_commit(tc::smem_u32(&empty[s]));
+        }
+        tc::mma_commit(tc::smem_u32(accb));
+    }
+    __syncwarp();
+
+    // ---------------- epilogue: TMEM -> registers -> global ----------------
+    const bool ok = tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
+    tc::fence_after_sync();
+    const bool good = __all_sync(0xffffffffu, ok && !*abort_flag);
+    if (!good) {
+        // poison the tile: the factorisation of H then reports a non-finite pivot
+        const int row = warp * 32 + lane;
+        const int64_t gi = i0 + row;
+        if (gi < n) {
+            for (int c = 0; c < TILE && j0 + c < n; ++c) {
+                const int64_t gj = j0 + c;
+                if (direct) {
+                    H[gi * n + gj] = __int_as_float(0x7fc00000);
+                    H[gj * n + gi] = __int_as_float(0x7fc00000);
+                } else {
+                    part[(int64_t)blockIdx.y * n * n + gi * n + gj] = __int_as_float(0x7fc00000);
+                }
+            }
+        }
+    }
+    __syncwarp();
+    if (good && nk > 0) {
+        const int row = warp * 32 + lane;
+        const int64_t gi = i0 + row;
+#pragma unroll 1
+        for (int c0 = 0; c0 < TILE; c0 += 32) {
+            uint32_t v[32];
+            tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+            if (gi < n) {
+#pragma unroll
+                for (int q = 0; q < 32; ++q) {
+                    const int64_t gj = j0 + c0 + q;
+                    if (gj >= n) break;
+                    const float x = __uint_as_float(v[q]);
+                    if (direct) {
+                        H[gi * n + gj] += x;
+                        if (!diag) H[gj * n + gi] += x;
+                    } else {
+                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = x;
+                    }
+                }
+            }
+        }
+    }
+    if (!good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 0) tc::tmem_dealloc(tmem, TILE);
+}
+
+using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
+                              const cuuint64_t *, const cuuint32_t *, const cuuint32_t *, CUtensorMapInterleave,
+                              CUtensorMapSwizzle, CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+EncodeFn g_encode = nullptr;
+std::once_flag g_encode_once;
+
+}  // namespace
+
+CUresult encode_tmap_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
+                             uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128) {
+    std::call_once(g_encode_once, [] {
+        void *fn = nullptr;
+        cudaDriverEntryPointQueryResult q;
+        if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &fn, 12000, cudaEnableDefault, &q) ==
+                cudaSuccess &&
+            q == cudaDriverEntryPointSuccess)
+            g_encode = reinterpret_cast<EncodeFn>(fn);
+    });
+    if (!g_encode) return CUDA_ERROR_NOT_FOUND;
+    cuuint64_t dims[2] = {inner, outer};
+    cuuint64_t strides[1] = {row_stride_bytes};
+    cuuint32_t box[2] = {box_inner, box_outer};
+    cuuint32_t estr[2] = {1, 1};
+    return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+                    CU_TENSOR_MAP_INTERLEAVE_NONE,
+                    swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                    CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
+}
+
+bool hessian_tc_eligible(int64_t n, int64_t T, const void *X) {
+    return n >= 64 && n % 8 == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0 && T > 0 && T < (1ll << 31) &&
+           n < (1ll << 31);
+}
+
+realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
+                               size_t ws_bytes, int sms) {
+    CUtensorMap map;
+    CUresult cr = encode_tmap_2d_bf16(&map, X, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
+    if (cr != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)cr);
+    const int nt = ceil_div(n, TILE);
+    const int64_t lower = (int64_t)nt * (nt + 1) / 2;
+    int splits = hessian_splits(n, T, sms);
+    const size_t per = (size_t)n * n * sizeof(float);
+    if (splits > 1 && (ws == nullptr || ws_bytes < 2 * per)) splits = 1;
+    if (splits > 1 && (size_t)splits * per > ws_bytes) splits = (int)(ws_bytes / per);
+    int64_t tper = (T + splits - 1) / splits;
+    tper = (tper + KSTAGE - 1) / KSTAGE * KSTAGE;
+    splits = (int)((T + tper - 1) / tper);
+    static bool configured = false;
+    if (!configured) {
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(hess_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
+        configured = true;
+    }
+    float *part = static_cast<float *>(ws);
+    {
+        Launch L("hessian_syrk_tc", s);
+        hess_tc_kernel<<<dim3((unsigned)lower, (unsigned)splits), 128, SMEM_BYTES, s>>>(map, n, T, tper, H, part,
+                                                                                       splits == 1, err);
+    }
+    REALQ_TRY(check_launch("hessian_syrk_tc"));
+    if (splits > 1) REALQ_TRY(hessian_reduce(s, n, splits, part, H, 0));
+    return REALQ_OK;
+}
+
+}  // namespace realq

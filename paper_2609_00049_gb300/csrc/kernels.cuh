@@ -40,9 +40,14 @@ realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g,
 
 // --------------------------------------------------------------- Hessian ---
 int hessian_splits(int64_t n, int64_t T, int num_sms);
+int num_sms();
 size_t hessian_ws_bytes(int64_t n, int64_t T, int has_xfp);
 realq_status_t hessian_accumulate(cudaStream_t s, int64_t n, int64_t T, const void *X, const void *Xfp,
                                   realq_dtype_t dt, float *H, float *D, void *ws, size_t ws_bytes);
+realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float *part, float *out, int mode);
+bool hessian_tc_eligible(int64_t n, int64_t T, const void *X);
+realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
+                               size_t ws_bytes, int sms);
 
 // --------------------------------------------------------------- prepare ---
 size_t prepare_ws_bytes(int64_t n);

@@ -418,7 +418,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     qa.g = p.group; qa.ngroups = p.ngroups; qa.bits = p.bits; qa.sym = p.sym;
     qa.scale = p.scale; qa.zero = p.zero; qa.codes = p.codes; qa.ncb = (p.n + 1) / 2;
     qa.Et = p.Et; qa.status = p.status;
-    const int Gk = !params_here ? 0 : (p.group <= B ? p.group : B);
+    const int Gk = !params_here ? 0 : (p.group >= p.n ? B : p.group);
     if (B == 128) REALQ_TRY(launch_qb_g<128>(s, qa, Gk));
     else if (B == 64) REALQ_TRY(launch_qb_g<64>(s, qa, Gk));
     else REALQ_TRY(launch_qb_g<32>(s, qa, Gk));

@@ -56,7 +56,17 @@ def test_hessian_exact_on_integer_inputs():
     assert np.array_equal(H.cpu().numpy().astype(np.float64), Href)
 
 
-@pytest.mark.parametrize("n,T", [(300, 5000), (128, 65536), (97, 4099)])
+def test_hessian_tensor_core_exact_on_integer_inputs():
+    # integer activations are exact in bf16 and every partial sum is exact in fp32
+    for n, T in ((256, 4160), (384, 20000), (136, 777), (1024, 65536)):
+        case = synth.layer_case(33, 4, n, T, integer_x=True)
+        X = dev(case.Xhat, torch.bfloat16)
+        H, _, _ = layer.accumulate([X], n)
+        Href, _ = oracle.hessian_sum([case.Xhat])
+        assert np.array_equal(H.cpu().numpy().astype(np.float64), Href), (n, T)
+
+
+@pytest.mark.parametrize("n,T", [(300, 5000), (128, 65536), (97, 4099), (512, 70000)])
 def test_hessian_bf16_and_cross_moment(n, T):
     case = synth.layer_case(21, 4, n, T, perturbed=True, bf16=True, outliers=2)
     Xh = dev(case.Xhat, torch.bfloat16)
