@@ -137,6 +137,29 @@ realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T
                                      int64_t *fail_col, void *ws, size_t ws_bytes);
 size_t realq_prepare_workspace_size(int64_t n);
 
+/* Allocation-free variant of realq_hessian_prepare.  The paper has no
+ * counterpart: this exists for callers that cannot allocate device memory,
+ * e.g. a plugin running inside a host application that owns every device
+ * allocation and exposes no allocator through this C interface, or a
+ * long-running service that reserves all of its memory up front and must not
+ * allocate (or let cudaMalloc / cudaFree synchronize the device) once it runs.
+ * Same arguments, results, synchronization and NOT_SPD behaviour as
+ * realq_hessian_prepare, without the workspace: its scratch is a file-scope
+ * device array of the library sized for n <= REALQ_PREPARE_NOALLOC_MAX_N
+ * (about 8.4 MB, held by every GPU that loads the library until the process
+ * exits).  Larger n returns REALQ_ERR_INVALID_ARG before any work is queued.
+ * The call allocates nothing (no cudaMalloc / cudaFree, no allocating library
+ * routine).  The first call on a device, with that device current, looks up
+ * the array's device address once; make that first call before any stream
+ * capture.  All calls share the one array, which keeps the last call's
+ * contents (the status word is cleared at the start of each call, the rest is
+ * overwritten before it is read), so calls that overlap on the GPU race: do
+ * not run two of them concurrently on one device. */
+#define REALQ_PREPARE_NOALLOC_MAX_N 32768
+realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                             const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                             int64_t *fail_col);
+
 /* Dbar = D_sum / T_total (n x n); may alias D_sum.  Asynchronous. */
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum,
                                   float *Dbar);

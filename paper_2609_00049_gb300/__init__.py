@@ -19,7 +19,7 @@ import torch
 __all__ = [
     "RealqError", "QuantCfg", "BgdCfg", "lib", "library_path", "quant_cfg", "bgd_cfg", "workspace",
     "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
-    "realq_prepare_workspace_size", "realq_scale_moment", "realq_quantize_layer",
+    "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -76,6 +76,7 @@ _SIGS = {
     "realq_hessian_workspace_size": ([_i64, _i64, _int, _int], _sz),
     "realq_hessian_prepare": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
     "realq_prepare_workspace_size": ([_i64], _sz),
+    "realq_hessian_prepare_noalloc": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64], _int),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
                               ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
@@ -192,6 +193,25 @@ def realq_hessian_prepare(H_sum: torch.Tensor, T_total: int, damp_frac: float, U
     wp, wb = _ws(ws)
     st = lib().realq_hessian_prepare(_stream(stream), n, int(T_total), float(damp_frac), _ptr(H_sum), _ptr(U_out),
                                      _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc), wp, wb)
+    _check(st, fail_col=fc.value)
+    return fc.value
+
+
+PREPARE_NOALLOC_MAX_N = 32768
+
+
+def realq_hessian_prepare_noalloc(H_sum: torch.Tensor, T_total: int, damp_frac: float, U_out: torch.Tensor,
+                                  Hbar_out: Optional[torch.Tensor], dead_out: torch.Tensor, stream=None) -> int:
+    """realq_hessian_prepare without a workspace, for callers that cannot allocate
+    device memory (its scratch is a fixed device array of the library, n <= 32768).
+    Returns -1; raises RealqError(status=NOT_SPD, fail_col=j) on a failed pivot."""
+    n = H_sum.shape[0]
+    _need(U_out, torch.float32, (n, n), "U_out")
+    _need(Hbar_out, torch.float32, (n, n), "Hbar_out")
+    _need(dead_out, torch.uint8, (n,), "dead_out")
+    fc = ctypes.c_int64(-1)
+    st = lib().realq_hessian_prepare_noalloc(_stream(stream), n, int(T_total), float(damp_frac), _ptr(H_sum),
+                                             _ptr(U_out), _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc))
     _check(st, fail_col=fc.value)
     return fc.value
 

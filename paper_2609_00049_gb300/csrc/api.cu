@@ -230,6 +230,25 @@ realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T
     return prepare(S(stream), n, T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col, ws, ws_bytes);
 }
 
+realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                             const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                             int64_t *fail_col) {
+    if (n <= 0 || T_total <= 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_noalloc: n > 0, T_total > 0 required");
+    if (n > REALQ_PREPARE_NOALLOC_MAX_N)
+        return fail(REALQ_ERR_INVALID_ARG,
+                    "hessian_prepare_noalloc: n = %lld exceeds the allocation-free maximum %d; use "
+                    "realq_hessian_prepare with a workspace",
+                    (long long)n, REALQ_PREPARE_NOALLOC_MAX_N);
+    if (!H_sum || !U_out || !dead_out || !fail_col)
+        return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_noalloc: NULL argument");
+    if ((const void *)U_out == (const void *)H_sum)
+        return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_noalloc: U_out may not alias H_sum");
+    if (!(damp_frac >= 0.f) || !std::isfinite(damp_frac))
+        return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_noalloc: damp_frac >= 0");
+    *fail_col = -1;
+    return prepare_noalloc(S(stream), n, T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col);
+}
+
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum, float *Dbar) {
     if (n <= 0 || T_total <= 0 || !D_sum || !Dbar) return fail(REALQ_ERR_INVALID_ARG, "scale_moment: bad argument");
     return scale_copy(S(stream), n * n, (float)T_total, D_sum, Dbar);

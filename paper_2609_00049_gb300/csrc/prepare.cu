@@ -13,6 +13,8 @@
 // column in the workspace status word; the host reads it once at the end.
 #include "kernels.cuh"
 
+#include <mutex>
+
 namespace realq {
 namespace {
 
@@ -182,11 +184,46 @@ __global__ void scale_kernel(int64_t count, float div, const float *in, float *o
     if (i < count) out[i] = in[i] / div;
 }
 
+constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
+constexpr size_t prepare_bytes(int64_t n) {
+    return align256(sizeof(int)) + align256(sizeof(float)) + align256((size_t)n * NB * sizeof(float)) +
+           align256((size_t)NB * NB * sizeof(float));
+}
+
+// Scratch of the allocation-free entry point, sized for n <= REALQ_PREPARE_NOALLOC_MAX_N.
+// Every GPU that loads the library holds it until the process exits.
+constexpr size_t kNoAllocBytes = prepare_bytes(REALQ_PREPARE_NOALLOC_MAX_N);
+static __device__ __align__(256) unsigned char g_prepare_scratch[kNoAllocBytes];
+
+std::mutex g_noalloc_mu;
+void *g_noalloc_ptr[256] = {};
+
+// Device address of g_prepare_scratch on the current device (looked up once per device).
+realq_status_t noalloc_scratch(void **out) {
+    int dev = 0;
+    REALQ_CUDA_TRY(cudaGetDevice(&dev));
+    if (dev < 0 || dev >= 256) return fail(REALQ_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
+    std::lock_guard<std::mutex> lk(g_noalloc_mu);
+    if (g_noalloc_ptr[dev] == nullptr) {
+        void *p = nullptr;
+        const cudaError_t e = cudaGetSymbolAddress(&p, g_prepare_scratch);
+        if (e != cudaSuccess || p == nullptr)
+            return fail(REALQ_ERR_CUDA, "cudaGetSymbolAddress(prepare scratch): %s", cudaGetErrorString(e));
+        g_noalloc_ptr[dev] = p;
+    }
+    *out = g_noalloc_ptr[dev];
+    return REALQ_OK;
+}
+
 }  // namespace
 
-size_t prepare_ws_bytes(int64_t n) {
-    return align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)n * NB * sizeof(float)) +
-           align_up((size_t)NB * NB * sizeof(float));
+size_t prepare_ws_bytes(int64_t n) { return prepare_bytes(n); }
+
+realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+                               uint8_t *dead, int64_t *fail_col) {
+    void *scratch = nullptr;
+    REALQ_TRY(noalloc_scratch(&scratch));
+    return prepare(s, n, T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes);
 }
 
 realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
