@@ -443,6 +443,40 @@ def reference_arm(args, wl, rank, world):
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
+def kernel_bench(args):
+    """Times one kernel family alone on a synthetic case sized by --n / --tokens
+    (the small-case target of ncu captures).  Prints one JSON line."""
+    import torch
+    import paper_2609_00049_gb300 as rq
+    from paper_2609_00049_gb300 import build as rqbuild
+    rqbuild.build()
+    rq.lib()
+    peaks = load_peaks()
+    n, T = args.n, args.tokens
+    wl = synth.Workload("kernel", {"x": synth.InputSpec("x", n, T, "gauss", outlier_frac=0.01, outlier_scale=20.0)},
+                        [], seed=1)
+    X = torch.from_numpy(synth.xhat_full(wl, "x").view(np.int16)).view(torch.bfloat16).cuda()
+    H = torch.zeros(n, n, device="cuda")
+    ws = rq.workspace(rq.realq_hessian_workspace_size(n, T))
+    stream = torch.cuda.current_stream()
+    for _ in range(args.warmup):
+        rq.realq_hessian_accumulate(X, H, ws=ws)
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        rq.realq_hessian_accumulate(X, H, ws=ws)
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    flops = T * n * (n + 1)
+    tf = flops / (ms / 1e3) / 1e12
+    print(json.dumps({"kernel": "hessian_syrk_tc", "n": n, "tokens": T, "ms_per_launch": ms, "achieved": tf,
+                      "unit": "TFLOP/s", "peak": peaks["bf16_tflops"], "frac": tf / peaks["bf16_tflops"],
+                      "peak_source": f"bf16 dense burst, {peaks['source']}",
+                      "input_bytes": T * n * 2}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -452,7 +486,13 @@ def main():
     ap.add_argument("--workload", default="qwen3-0.6b")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--kernel", choices=["hessian"], default=None, help="time one kernel alone (small case)")
+    ap.add_argument("--n", type=int, default=2048)
+    ap.add_argument("--tokens", type=int, default=65536)
     args = ap.parse_args()
+    if args.kernel:
+        kernel_bench(args)
+        return
     rank = int(os.environ.get("RANK", 0))
     world = int(os.environ.get("WORLD_SIZE", 1))
     wl = synth.workloads()[args.workload]

@@ -80,16 +80,20 @@ struct QArgs {
 };
 
 // Column-serial quantize + in-block OBS propagation for block [bs, bs + kb).
-// One thread owns one row; the row's B columns live in registers (fully
-// unrolled), the B x B diagonal block of U is staged once per CTA in shared
-// memory and read as broadcasts.  G > 0: group parameters are computed here
-// at every G-th column from the current (compensated) weights; G = 0: they
-// were computed before the block for a group spanning whole blocks.
+// One thread owns one row; the row's B columns live in registers, the B x B
+// diagonal block of U is staged once per CTA in shared memory and read as
+// broadcasts.  The block is walked in sub-blocks of 32 columns: inside a
+// sub-block every column's error is fed to the later columns at once, and
+// after it the 32 errors are applied to the columns of the later sub-blocks,
+// column by column in the same order, so the arithmetic is that of the plain
+// column loop (this shape keeps the row in registers).  G > 0: group
+// parameters are computed here at every G-th column (G a multiple of 32) from
+// the current weights; G = 0: they were computed before the block.
 template <int B, int G>
 __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) {
     extern __shared__ __align__(16) float qsm[];
-    float *Us = qsm;           // B x B
-    float *invd = qsm + B * B; // B
+    float *Us = qsm;            // B x B, strictly upper part
+    float *invd = qsm + B * B;  // B
     const int kb = a.kb;
     for (int idx = threadIdx.x; idx < B * B; idx += blockDim.x) {
         const int r = idx / B, c = idx % B;
@@ -117,38 +121,52 @@ __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) 
     bool bad = false;
     unsigned lo = 0;
 #pragma unroll
-    for (int j = 0; j < B; ++j) {
-        if (j < kb) {
-            if (G > 0 && (j % (G > 0 ? G : 1)) == 0) {
-                float mn = 0.f, mx = 0.f;
+    for (int s = 0; s < B / 32; ++s) {
+        float e[32];
+        if (G > 0 && ((s * 32) % (G > 0 ? G : 1)) == 0 && s * 32 < kb) {
+            float mn = 0.f, mx = 0.f;
 #pragma unroll
-                for (int c = j; c < j + G && c < B; ++c)
-                    if (c < kb) {
-                        mn = fminf(mn, r[c]);
-                        mx = fmaxf(mx, r[c]);
-                    }
-                grid_params(mn, mx, a.bits, a.sym, sc, zr);
-                const int gi = (int)((a.bs + j) / a.g);
-                a.scale[i * a.ngroups + gi] = sc;
-                a.zero[i * a.ngroups + gi] = (uint8_t)zr;
-            }
-            const float w = r[j];
-            bad |= !isfinite(w);
-            float q = rintf(w / sc) + zr;
-            q = fminf(fmaxf(q, 0.f), maxq);
-            const float dq = sc * (q - zr);
-            const float e = (w - dq) * invd[j];
-            a.Et[(int64_t)j * a.m + i] = e;
-            r[j] = dq;
+            for (int c = s * 32; c < s * 32 + G && c < B; ++c)
+                if (c < kb) {
+                    mn = fminf(mn, r[c]);
+                    mx = fmaxf(mx, r[c]);
+                }
+            grid_params(mn, mx, a.bits, a.sym, sc, zr);
+            const int gi = (int)((a.bs + s * 32) / a.g);
+            a.scale[i * a.ngroups + gi] = sc;
+            a.zero[i * a.ngroups + gi] = (uint8_t)zr;
+        }
 #pragma unroll
-            for (int k = j + 1; k < B; ++k) r[k] = fmaf(-e, Us[j * B + k], r[k]);
-            const unsigned qi = (unsigned)q;
-            if ((j & 1) == 0) {
-                lo = qi;
-                if (j == kb - 1) crow[j / 2] = (uint8_t)lo;
-            } else {
-                crow[j / 2] = (uint8_t)(lo | (qi << 4));
+        for (int jj = 0; jj < 32; ++jj) {
+            const int j = s * 32 + jj;
+            e[jj] = 0.f;
+            if (j < kb) {
+                const float w = r[j];
+                bad |= !isfinite(w);
+                float q = rintf(w / sc) + zr;
+                q = fminf(fmaxf(q, 0.f), maxq);
+                const float dq = sc * (q - zr);
+                const float err = (w - dq) * invd[j];
+                e[jj] = err;
+                a.Et[(int64_t)j * a.m + i] = err;
+                r[j] = dq;
+#pragma unroll
+                for (int kk = jj + 1; kk < 32; ++kk) r[s * 32 + kk] = fmaf(-err, Us[j * B + s * 32 + kk], r[s * 32 + kk]);
+                const unsigned qi = (unsigned)q;
+                if ((j & 1) == 0) {
+                    lo = qi;
+                    if (j == kb - 1) crow[j / 2] = (uint8_t)lo;
+                } else {
+                    crow[j / 2] = (uint8_t)(lo | (qi << 4));
+                }
             }
+        }
+#pragma unroll
+        for (int k = (s + 1) * 32; k < B; ++k) {
+            float acc = r[k];
+#pragma unroll
+            for (int jj = 0; jj < 32; ++jj) acc = fmaf(-e[jj], Us[(s * 32 + jj) * B + k], acc);
+            r[k] = acc;
         }
     }
     float *wout = a.W + i * a.n + a.bs;
