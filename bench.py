@@ -255,8 +255,6 @@ def gpu_arm(args, wl, rank, world):
     except Exception:
         pass
     clocks = ClockSampler(uuid)
-    rq.realq_profile_collect()          # drop anything pending
-    rq.realq_profile_enable(True)
     launches0 = rq.realq_launch_count()
     clocks.start()
     torch.cuda.synchronize()
@@ -272,8 +270,18 @@ def gpu_arm(args, wl, rank, world):
     ms_total = t0.elapsed_time(t1)
     clk = clocks.stop()
     launches = rq.realq_launch_count() - launches0
-    rq.realq_profile_enable(False)
-    prof = rq.realq_profile_collect(256)
+
+    # the same K steps again with every library launch bracketed by CUDA events
+    # on its own stream: per-kernel device time for the breakdown and roofline
+    prof = {}
+    if not args.no_profile:
+        rq.realq_profile_collect()          # drop anything pending
+        rq.realq_profile_enable(True)
+        for _ in range(args.steps):
+            step_device()
+        torch.cuda.synchronize()
+        rq.realq_profile_enable(False)
+        prof = rq.realq_profile_collect(256)
     if dist is not None:
         tt = torch.tensor([ms_total], device=dev)
         dist.all_reduce(tt, op=dist.ReduceOp.MAX)
@@ -451,24 +459,47 @@ def kernel_bench(args):
     from paper_2609_00049_gb300 import build as rqbuild
     rqbuild.build()
     rq.lib()
+    from paper_2609_00049_gb300 import layer
     peaks = load_peaks()
     n, T = args.n, args.tokens
     wl = synth.Workload("kernel", {"x": synth.InputSpec("x", n, T, "gauss", outlier_frac=0.01, outlier_scale=20.0)},
-                        [], seed=1)
+                        [synth.ModuleSpec("w", args.m, n, "x")], seed=1, lr=3e-4)
     X = torch.from_numpy(synth.xhat_full(wl, "x").view(np.int16)).view(torch.bfloat16).cuda()
+    stream = torch.cuda.current_stream()
     H = torch.zeros(n, n, device="cuda")
     ws = rq.workspace(rq.realq_hessian_workspace_size(n, T))
-    stream = torch.cuda.current_stream()
-    for _ in range(args.warmup):
+    if args.kernel == "hessian":
+        def run():
+            rq.realq_hessian_accumulate(X, H, ws=ws)
+    else:
         rq.realq_hessian_accumulate(X, H, ws=ws)
+        prep = layer.prepare(H, T)
+        if args.kernel == "prepare":
+            def run():
+                layer.prepare(H, T)
+        else:
+            mod = wl.modules[0]
+            W0 = torch.from_numpy(synth.weights(wl, mod).view(np.int16)).view(torch.bfloat16).cuda()
+            F = torch.from_numpy(synth.fisher(wl, mod)).cuda()
+            q = rq.quant_cfg()
+            b = rq.bgd_cfg(wl.lr)
+            qws = rq.workspace(rq.realq_quantize_workspace_size(mod.m, n, q, b))
+
+            def run():
+                layer.quantize(W0, prep, q, b, F=F, ws=qws)
+    for _ in range(args.warmup):
+        run()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
     for _ in range(args.steps):
-        rq.realq_hessian_accumulate(X, H, ws=ws)
+        run()
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
+    if args.kernel != "hessian":
+        print(json.dumps({"kernel": args.kernel, "m": args.m, "n": n, "ms_per_call": ms}))
+        return
     flops = T * n * (n + 1)
     tf = flops / (ms / 1e3) / 1e12
     print(json.dumps({"kernel": "hessian_syrk_tc", "n": n, "tokens": T, "ms_per_launch": ms, "achieved": tf,
@@ -486,8 +517,11 @@ def main():
     ap.add_argument("--workload", default="qwen3-0.6b")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--kernel", choices=["hessian"], default=None, help="time one kernel alone (small case)")
+    ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
+    ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep"], default=None,
+                    help="time one stage alone on a small synthetic case")
     ap.add_argument("--n", type=int, default=2048)
+    ap.add_argument("--m", type=int, default=1024)
     ap.add_argument("--tokens", type=int, default=65536)
     args = ap.parse_args()
     if args.kernel:

@@ -53,64 +53,133 @@ __global__ void prep_damp_kernel(int64_t n, float *A, float damp, float *lam_out
     if (threadIdx.x == 0) *lam_out = lam;
 }
 
-// Diagonal block [k0, k0 + kb): A_KK = R_KK R_KK^T, R_KK upper (in place).
-__global__ void chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status) {
-    __shared__ float S[NB][NB + 1];
-    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
-        const int r = idx / NB, c = idx % NB;
-        S[r][c] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
-    }
-    __syncthreads();
+// The 64 x 64 diagonal-block kernels below use 256 threads as a 16 x 16 grid;
+// thread (ty, tx) keeps the 4 x 4 block rows 4ty.., columns 4tx.. in
+// registers, and only the pivot and the pivot column / row travel through
+// double-buffered shared memory.
+
+// V = R^-1 for the kb x kb upper triangle in Rs, by row operations on the
+// identity (back substitution applied to all columns at once); v is this
+// thread's 4 x 4 block of V.  One barrier per pivot.
+__device__ __forceinline__ void upper_inverse_regs(const float (*Rs)[NB + 1], int kb, float (&v)[4][4],
+                                                   float (*rowk)[NB]) {
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) v[a][b] = (ty * 4 + a == tx * 4 + b && ty * 4 + a < kb) ? 1.f : 0.f;
     for (int k = kb - 1; k >= 0; --k) {
-        if (threadIdx.x == 0) {
-            float d = S[k][k];
-            if (!(d > 0.f) || !isfinite(d)) {
-                atomicCAS(status, -1, (int)(k0 + k));
-                d = 1.f;
+        const int kt = k >> 2, kq = k & 3, p = k & 1;
+        if (ty == kt) {
+            const float rkk = Rs[k][k];
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+                if (a == kq) {
+#pragma unroll
+                    for (int b = 0; b < 4; ++b) {
+                        v[a][b] = v[a][b] / rkk;
+                        rowk[p][tx * 4 + b] = v[a][b];
+                    }
+                }
+        }
+        __syncthreads();
+        float rv[4];
+#pragma unroll
+        for (int b = 0; b < 4; ++b) rv[b] = rowk[p][tx * 4 + b];
+#pragma unroll
+        for (int a = 0; a < 4; ++a) {
+            const int i = ty * 4 + a;
+            if (i < k) {
+                const float rik = Rs[i][k];
+#pragma unroll
+                for (int b = 0; b < 4; ++b) v[a][b] -= rik * rv[b];
             }
-            S[k][k] = sqrtf(d);
         }
-        __syncthreads();
-        const float r = S[k][k];
-        for (int i = threadIdx.x; i < k; i += blockDim.x) S[i][k] = S[i][k] / r;
-        __syncthreads();
-        for (int idx = threadIdx.x; idx < k * k; idx += blockDim.x) {
-            const int i = idx / k, j = idx % k;
-            if (j >= i) S[i][j] -= S[i][k] * S[j][k];
-        }
-        __syncthreads();
-    }
-    for (int idx = threadIdx.x; idx < kb * kb; idx += blockDim.x) {
-        const int r = idx / kb, c = idx % kb;
-        if (c >= r) A[(k0 + r) * n + k0 + c] = S[r][c];
     }
 }
 
-// Rows i < k0 of the block column: solve x R_KK^T = A[i, k0:k0+kb] (one thread per row).
-__global__ void chol_panel_kernel(int64_t n, float *A, int64_t k0, int kb) {
-    __shared__ float R[NB][NB + 1];
-    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
-        const int r = idx / NB, c = idx % NB;
-        R[r][c] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
-    }
-    __syncthreads();
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= k0) return;
-    float x[NB];
+// Diagonal block [k0, k0 + kb): A_KK = R_KK R_KK^T with R_KK upper (in place),
+// and Vt = (R_KK^-1)^T (dense 64 x 64, row-major) for the panel solve.
+// Two barriers per Cholesky pivot, one per inverse pivot.
+__global__ void __launch_bounds__(256) chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status,
+                                                        float *Vt) {
+    __shared__ float Rs[NB][NB + 1];
+    __shared__ float colk[2][NB];
+    __shared__ float rk_s[2];
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+    float sv[4][4];
 #pragma unroll
-    for (int c = 0; c < NB; ++c) x[c] = (c < kb) ? A[i * n + k0 + c] : 0.f;
+    for (int a = 0; a < 4; ++a)
 #pragma unroll
-    for (int c = NB - 1; c >= 0; --c) {
-        if (c < kb) {
-            float v = x[c];
+        for (int b = 0; b < 4; ++b) {
+            const int r = ty * 4 + a, c = tx * 4 + b;
+            sv[a][b] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
+        }
+    for (int k = kb - 1; k >= 0; --k) {
+        const int kt = k >> 2, kq = k & 3, p = k & 1;
+        if (ty == kt && tx == kt) {
 #pragma unroll
-            for (int d = c + 1; d < NB; ++d) v -= x[d] * R[c][d];
-            x[c] = v / R[c][c];
+            for (int a = 0; a < 4; ++a)
+                if (a == kq) {
+                    float d = sv[a][a];
+                    const bool bad = !(d > 0.f) || !isfinite(d);
+                    if (bad) {
+                        atomicCAS(status, -1, (int)(k0 + k));
+                        d = 1.f;
+                    }
+                    const float rk = sqrtf(d);
+                    sv[a][a] = rk;
+                    rk_s[p] = rk;
+                }
+        }
+        __syncthreads();
+        if (tx == kt) {
+            const float rk = rk_s[p];
+#pragma unroll
+            for (int b = 0; b < 4; ++b)
+                if (b == kq) {
+#pragma unroll
+                    for (int a = 0; a < 4; ++a) {
+                        const int i = ty * 4 + a;
+                        if (i < k) {
+                            sv[a][b] = sv[a][b] / rk;
+                            colk[p][i] = sv[a][b];
+                        }
+                    }
+                }
+        }
+        __syncthreads();
+        if (ty * 4 < k && tx * 4 < k) {
+            float ci[4], cj[4];
+#pragma unroll
+            for (int a = 0; a < 4; ++a) ci[a] = colk[p][ty * 4 + a];
+#pragma unroll
+            for (int b = 0; b < 4; ++b) cj[b] = colk[p][tx * 4 + b];
+#pragma unroll
+            for (int a = 0; a < 4; ++a)
+#pragma unroll
+                for (int b = 0; b < 4; ++b) {
+                    const int i = ty * 4 + a, j = tx * 4 + b;
+                    if (i <= j && j < k) sv[a][b] -= ci[a] * cj[b];
+                }
         }
     }
 #pragma unroll
-    for (int c = 0; c < NB; ++c)
-        if (c < kb) A[i * n + k0 + c] = x[c];
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int r = ty * 4 + a, c = tx * 4 + b;
+            Rs[r][c] = sv[a][b];
+            if (r < kb && c < kb && c >= r) A[(k0 + r) * n + k0 + c] = sv[a][b];
+        }
+    __syncthreads();
+    __shared__ float rowk[2][NB];
+    float v[4][4];
+    upper_inverse_regs(Rs, kb, v, rowk);
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) Vt[(tx * 4 + b) * NB + ty * 4 + a] = v[a][b];
 }
 
 // A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles).
@@ -151,32 +220,27 @@ __global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, i
     }
 }
 
-// V = R_JJ^-1 (upper) by back substitution, one thread per column; written to
-// A[J, J] and to the dense 64 x 64 buffer Vd (zeros below the diagonal).
-__global__ void trtri_diag_kernel(int64_t n, float *A, int64_t j0, int jb, float *Vd) {
-    __shared__ float R[NB][NB + 1];
-    __shared__ float V[NB][NB + 1];
+// V = R_JJ^-1 (upper); written to A[J, J] and to the dense 64 x 64 buffer Vd
+// (zeros below the diagonal).
+__global__ void __launch_bounds__(256) trtri_diag_kernel(int64_t n, float *A, int64_t j0, int jb, float *Vd) {
+    __shared__ float Rs[NB][NB + 1];
+    __shared__ float rowk[2][NB];
     for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
         const int r = idx / NB, c = idx % NB;
-        R[r][c] = (r < jb && c < jb && c >= r) ? A[(j0 + r) * n + j0 + c] : 0.f;
-        V[r][c] = 0.f;
+        Rs[r][c] = (r < jb && c < jb && c >= r) ? A[(j0 + r) * n + j0 + c] : 0.f;
     }
     __syncthreads();
-    const int c = threadIdx.x;
-    if (c < jb) {
-        V[c][c] = 1.f / R[c][c];
-        for (int i = c - 1; i >= 0; --i) {
-            float s = 0.f;
-            for (int l = i + 1; l <= c; ++l) s += R[i][l] * V[l][c];
-            V[i][c] = -s / R[i][i];
+    float v[4][4];
+    upper_inverse_regs(Rs, jb, v, rowk);
+    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+#pragma unroll
+    for (int a = 0; a < 4; ++a)
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int r = ty * 4 + a, c = tx * 4 + b;
+            Vd[r * NB + c] = v[a][b];
+            if (r < jb && c < jb && c >= r) A[(j0 + r) * n + j0 + c] = v[a][b];
         }
-    }
-    __syncthreads();
-    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
-        const int r = idx / NB, cc = idx % NB;
-        Vd[idx] = V[r][cc];
-        if (r < jb && cc < jb && cc >= r) A[(j0 + r) * n + j0 + cc] = V[r][cc];
-    }
 }
 
 __global__ void scale_kernel(int64_t count, float div, const float *in, float *out) {
@@ -253,15 +317,19 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
         const int kb = (int)std::min<int64_t>(NB, n - k0);
         {
             Launch L("chol_diag", s);
-            chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status);
+            chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status, Vd);
         }
         REALQ_TRY(check_launch("chol_diag"));
         if (k0 == 0) continue;
-        {
-            Launch L("chol_panel", s);
-            chol_panel_kernel<<<ceil_div(k0, 128), 128, 0, s>>>(n, U, k0, kb);
-        }
-        REALQ_TRY(check_launch("chol_panel"));
+        // rows above the block: R[0:k0, K] = A[0:k0, K] R_KK^-T (in place; one
+        // column tile, so every CTA reads only the rows it writes)
+        GemmArgs pg{};
+        pg.M = k0; pg.N = kb; pg.K = kb;
+        pg.A = U + k0; pg.lda = n;
+        pg.B = Vd; pg.ldb = NB;
+        pg.C = U + k0; pg.ldc = n;
+        pg.alpha = 1.f;
+        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, pg, "chol_panel"));
         const int64_t nt0 = k0 / NB;
         {
             Launch L("chol_update", s);
@@ -275,7 +343,7 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
         const int jb = (int)std::min<int64_t>(NB, n - j0);
         {
             Launch L("trtri_diag", s);
-            trtri_diag_kernel<<<1, NB, 0, s>>>(n, U, j0, jb, Vd);
+            trtri_diag_kernel<<<1, 256, 0, s>>>(n, U, j0, jb, Vd);
         }
         REALQ_TRY(check_launch("trtri_diag"));
         if (j0 == 0) continue;

@@ -12,7 +12,7 @@
 namespace realq {
 namespace {
 
-constexpr int QB_THREADS = 32;
+constexpr int QB_THREADS = 128;
 
 // quant(.) grid of one group from its min / max (the reading fixed by the
 // oracle: the grid contains 0; degenerate groups get [-1, 1]).  fp32, IEEE
@@ -65,6 +65,11 @@ __global__ void group_params_kernel(int64_t m, int64_t n, const float *W, int64_
     }
 }
 
+__device__ __forceinline__ void cp_async4(float *dst, const float *src) {
+    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
+    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src) : "memory");
+}
+
 struct QArgs {
     int64_t m, n, bs;
     int kb;
@@ -80,68 +85,84 @@ struct QArgs {
 };
 
 // Column-serial quantize + in-block OBS propagation for block [bs, bs + kb).
-// One thread owns one row; the row's B columns live in registers, the B x B
-// diagonal block of U is staged once per CTA in shared memory and read as
-// broadcasts.  The block is walked in sub-blocks of 32 columns: inside a
-// sub-block every column's error is fed to the later columns at once, and
-// after it the 32 errors are applied to the columns of the later sub-blocks,
-// column by column in the same order, so the arithmetic is that of the plain
-// column loop (this shape keeps the row in registers).  G > 0: group
+// One thread owns one row.  The block is walked in sub-blocks of 32 columns:
+// the current sub-block lives in registers (unrolled), the rest of the row in
+// shared memory (thread-major, conflict-free); inside the sub-block every
+// column's error is fed to the later columns of the sub-block at once, and
+// after it the 32 errors are applied to every later column in column order,
+// so the arithmetic is that of the plain column loop.  U's diagonal block is
+// staged transposed (Ut[k][j] = U[j][k]) so the 32 coefficients of a later
+// column are contiguous.  The sub-block loop is not unrolled: the whole kernel
+// body stays small enough for the instruction cache.  G > 0: group
 // parameters are computed here at every G-th column (G a multiple of 32) from
 // the current weights; G = 0: they were computed before the block.
 template <int B, int G>
 __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) {
     extern __shared__ __align__(16) float qsm[];
-    float *Us = qsm;            // B x B, strictly upper part
-    float *invd = qsm + B * B;  // B
+    constexpr int UP = B + 4;             // row pitch of Ut: aligned float4 rows, 4-way store conflicts
+    float *Ut = qsm;                      // B x UP, Ut[k * UP + j] = U[j][k] for j < k, else 0
+    float *invd = Ut + B * UP;            // B
+    constexpr int RP = QB_THREADS + 1;    // row pitch of rs (conflict-free both ways)
+    float *rs = invd + B;                 // B x RP, rs[k * RP + row]
     const int kb = a.kb;
+    // Stage U's diagonal block (transposed) and the CTA's rows x kb slab of W
+    // (read along rows) with asynchronous 4-byte copies, all in flight at once;
+    // the entries that must be zero are written directly.
     for (int idx = threadIdx.x; idx < B * B; idx += blockDim.x) {
-        const int r = idx / B, c = idx % B;
-        Us[idx] = (r < kb && c < kb && c > r) ? a.U[(a.bs + r) * a.n + a.bs + c] : 0.f;
+        const int j = idx / B, k = idx % B;   // U row j, contiguous in k
+        float *dst = Ut + k * UP + j;
+        if (j < kb && k < kb && k > j) cp_async4(dst, a.U + (a.bs + j) * a.n + a.bs + k);
+        else *dst = 0.f;
+    }
+    const int64_t row0 = (int64_t)blockIdx.x * blockDim.x;
+    for (int rr = 0; rr < QB_THREADS; ++rr) {
+        const int64_t gi = row0 + rr;
+        for (int c = threadIdx.x; c < B; c += blockDim.x) {
+            float *dst = rs + c * RP + rr;
+            if (gi < a.m && c < kb) cp_async4(dst, a.W + gi * a.n + a.bs + c);
+            else *dst = 0.f;
+        }
     }
     for (int j = threadIdx.x; j < B; j += blockDim.x)
         invd[j] = (j < kb) ? 1.f / a.U[(a.bs + j) * a.n + a.bs + j] : 0.f;
+    asm volatile("cp.async.wait_all;" ::: "memory");
     __syncthreads();
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= a.m) return;
-
-    float r[B];
-    const float *wrow = a.W + i * a.n + a.bs;
-#pragma unroll
-    for (int c = 0; c < B; ++c) r[c] = (c < kb) ? wrow[c] : 0.f;
+    const int64_t i = row0 + threadIdx.x;
+    const bool live = i < a.m;
 
     float sc = 1.f, zr = 0.f;
-    if (G == 0) {
+    if (live && G == 0) {
         const int gi = (int)(a.bs / a.g);
         sc = a.scale[i * a.ngroups + gi];
         zr = (float)a.zero[i * a.ngroups + gi];
     }
     const float maxq = (float)((1 << a.bits) - 1);
-    uint8_t *crow = a.codes + i * a.ncb + a.bs / 2;
+    uint8_t *crow = a.codes + (live ? i : 0) * a.ncb + a.bs / 2;
     bool bad = false;
-    unsigned lo = 0;
+#pragma unroll 1
+    for (int s0 = 0; live && s0 < kb; s0 += 32) {
+        float r[32], e[32];
 #pragma unroll
-    for (int s = 0; s < B / 32; ++s) {
-        float e[32];
-        if (G > 0 && ((s * 32) % (G > 0 ? G : 1)) == 0 && s * 32 < kb) {
+        for (int jj = 0; jj < 32; ++jj) r[jj] = rs[(s0 + jj) * RP + threadIdx.x];
+        if (G > 0 && (s0 % (G > 0 ? G : 1)) == 0) {
             float mn = 0.f, mx = 0.f;
-#pragma unroll
-            for (int c = s * 32; c < s * 32 + G && c < B; ++c)
-                if (c < kb) {
-                    mn = fminf(mn, r[c]);
-                    mx = fmaxf(mx, r[c]);
-                }
+            for (int c = s0; c < s0 + G && c < kb; ++c) {
+                const float w = rs[c * RP + threadIdx.x];
+                mn = fminf(mn, w);
+                mx = fmaxf(mx, w);
+            }
             grid_params(mn, mx, a.bits, a.sym, sc, zr);
-            const int gi = (int)((a.bs + s * 32) / a.g);
+            const int gi = (int)((a.bs + s0) / a.g);
             a.scale[i * a.ngroups + gi] = sc;
             a.zero[i * a.ngroups + gi] = (uint8_t)zr;
         }
+        unsigned lo = 0;
 #pragma unroll
         for (int jj = 0; jj < 32; ++jj) {
-            const int j = s * 32 + jj;
+            const int j = s0 + jj;
             e[jj] = 0.f;
             if (j < kb) {
-                const float w = r[j];
+                const float w = r[jj];
                 bad |= !isfinite(w);
                 float q = rintf(w / sc) + zr;
                 q = fminf(fmaxf(q, 0.f), maxq);
@@ -149,11 +170,11 @@ __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) 
                 const float err = (w - dq) * invd[j];
                 e[jj] = err;
                 a.Et[(int64_t)j * a.m + i] = err;
-                r[j] = dq;
+                r[jj] = dq;
 #pragma unroll
-                for (int kk = jj + 1; kk < 32; ++kk) r[s * 32 + kk] = fmaf(-err, Us[j * B + s * 32 + kk], r[s * 32 + kk]);
+                for (int kk = jj + 1; kk < 32; ++kk) r[kk] = fmaf(-err, Ut[(s0 + kk) * UP + j], r[kk]);
                 const unsigned qi = (unsigned)q;
-                if ((j & 1) == 0) {
+                if ((jj & 1) == 0) {
                     lo = qi;
                     if (j == kb - 1) crow[j / 2] = (uint8_t)lo;
                 } else {
@@ -162,17 +183,29 @@ __global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) 
             }
         }
 #pragma unroll
-        for (int k = (s + 1) * 32; k < B; ++k) {
-            float acc = r[k];
+        for (int jj = 0; jj < 32; ++jj) rs[(s0 + jj) * RP + threadIdx.x] = r[jj];
+        // the 32 errors, column by column in order, into every later column
+#pragma unroll 2
+        for (int k = s0 + 32; k < kb; ++k) {
+            float acc = rs[k * RP + threadIdx.x];
+            const float4 *u4 = reinterpret_cast<const float4 *>(Ut + k * UP + s0);
 #pragma unroll
-            for (int jj = 0; jj < 32; ++jj) acc = fmaf(-e[jj], Us[(s * 32 + jj) * B + k], acc);
-            r[k] = acc;
+            for (int q4 = 0; q4 < 8; ++q4) {
+                const float4 u = u4[q4];
+                acc = fmaf(-e[q4 * 4 + 0], u.x, acc);
+                acc = fmaf(-e[q4 * 4 + 1], u.y, acc);
+                acc = fmaf(-e[q4 * 4 + 2], u.z, acc);
+                acc = fmaf(-e[q4 * 4 + 3], u.w, acc);
+            }
+            rs[k * RP + threadIdx.x] = acc;
         }
     }
-    float *wout = a.W + i * a.n + a.bs;
-#pragma unroll
-    for (int c = 0; c < B; ++c)
-        if (c < kb) wout[c] = r[c];
+    __syncthreads();
+    for (int rr = 0; rr < QB_THREADS; ++rr) {
+        const int64_t gi = row0 + rr;
+        if (gi >= a.m) break;
+        for (int c = threadIdx.x; c < kb; c += blockDim.x) a.W[gi * a.n + a.bs + c] = rs[c * RP + rr];
+    }
     if (bad) atomicOr(a.status, ST_NONFINITE);
 }
 
@@ -267,7 +300,7 @@ inline unsigned blocks_for(int64_t count, int threads = 256) { return (unsigned)
 
 template <int B, int G>
 realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
-    const size_t smem = (size_t)(B * B + B) * sizeof(float);
+    const size_t smem = (size_t)(B * (B + 4) + B + B * (QB_THREADS + 1)) * sizeof(float);
     static bool configured = false;
     if (!configured) {
         REALQ_CUDA_TRY(cudaFuncSetAttribute(quant_block_kernel<B, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
