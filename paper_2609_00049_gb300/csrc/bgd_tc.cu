@@ -1,0 +1,374 @@
+// Block-GD contractions (Eq. block_gd_update) on the 5th-generation tensor
+// cores with fp32-level accuracy: three tf32 products per term,
+//   a b ~= a_hi b_hi + a_hi b_lo + a_lo b_hi,
+// where a_hi keeps a's top 11 significand bits (exact in tf32) and
+// a_lo = a - a_hi.  The dropped a_lo b_lo and the tf32 rounding of the lo
+// parts leave ~2^-20 relative error per product, below the fp32 rounding of
+// the K-long accumulation itself; the gradient's sign, which Adam's first
+// step depends on, is then as reliable as with fp32 FFMA.
+//
+// C[M x N] = A[M x K] B[N x K]^T with both operands K-major in global memory
+// (rows of A, rows of B), each as a hi and a lo plane.  One CTA computes a
+// 128 x 128 tile: TMA loads 32-wide K slices of the four planes (128-byte
+// rows, 128-byte swizzle) into a 3-stage ring, one thread issues
+// 3 x 4 tcgen05.mma (kind::tf32, K = 8) per stage into a TMEM accumulator,
+// and four warps drain it through one of the epilogues:
+//   TC_STORE  C = acc
+//   TC_BGD_P  the Block-GD gradient factor after the lazy OBS update,
+//             p = acc + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead
+//             channels, written transposed and split (P^T hi / lo planes)
+//   TC_ADAM   g = acc: one Adam (or SGD) step on W[:, col0 + j], updating the
+//             moments and the displacement (full value and hi / lo planes)
+#include "kernels.cuh"
+#include "tc.cuh"
+
+namespace realq {
+namespace {
+
+constexpr int TB = 128;                       // tile rows (M) and columns (N)
+constexpr int KS = 32;                        // fp32 elements per K slice (128 bytes)
+constexpr int STAGES = 3;
+constexpr int PLANE = TB * KS * 4;            // 16 KB
+constexpr int STAGE_BYTES = 4 * PLANE;        // A hi, A lo, B hi, B lo
+constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+constexpr uint32_t IDESC = tc::idesc_tf32_f32(TB, TB);
+
+struct Maps {
+    CUtensorMap a_hi, a_lo, b_hi, b_lo;
+};
+
+// p = acc + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead channels
+__device__ __forceinline__ float bgd_p_value(const TcEpi &e, int64_t i, int64_t j, float v) {
+    const int64_t col = e.col0 + j;
+    const int64_t w = i * e.ldw + col;
+    const float w0 = e.w0_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16 *>(e.W0)[w])
+                               : static_cast<const float *>(e.W0)[w];
+    float p = v + (*e.lam) * (e.Ad[w] - (e.W[w] - w0));
+    if (e.R0) p += e.R0[w];
+    if (e.dead && e.dead[col]) p = 0.f;
+    return p;
+}
+
+__device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
+__device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
+__device__ __forceinline__ float4 ld4_w0(const TcEpi &e, int64_t w) {
+    if (e.w0_bf16) {
+        const uint2 u = *reinterpret_cast<const uint2 *>(static_cast<const __nv_bfloat16 *>(e.W0) + w);
+        return make_float4(__uint_as_float(u.x << 16), __uint_as_float(u.x & 0xFFFF0000u),
+                           __uint_as_float(u.y << 16), __uint_as_float(u.y & 0xFFFF0000u));
+    }
+    return ld4(static_cast<const float *>(e.W0) + w);
+}
+
+// Gradient factor for 4 rows x 4 columns (columns gj..gj+3 all < N); t points
+// at the tile entry of row 0, column 0 of the 4x4 patch, pitch tp.
+__device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, float *t, int tp) {
+    const int64_t col = e.col0 + gj;
+    float4 a[4], w[4], w0[4], r0[4];
+    uchar4 dd = make_uchar4(0, 0, 0, 0);
+    if (e.dead) dd = *reinterpret_cast<const uchar4 *>(e.dead + col);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        if (gi0 + u >= M) break;
+        const int64_t wi = (gi0 + u) * e.ldw + col;
+        a[u] = ld4(e.Ad + wi);
+        w[u] = ld4(e.W + wi);
+        w0[u] = ld4_w0(e, wi);
+        r0[u] = e.R0 ? ld4(e.R0 + wi) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    const float lam = *e.lam;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        if (gi0 + u >= M) break;
+        float *tr = t + u * tp;
+        tr[0] = dd.x ? 0.f : tr[0] + lam * (a[u].x - (w[u].x - w0[u].x)) + r0[u].x;
+        tr[1] = dd.y ? 0.f : tr[1] + lam * (a[u].y - (w[u].y - w0[u].y)) + r0[u].y;
+        tr[2] = dd.z ? 0.f : tr[2] + lam * (a[u].z - (w[u].z - w0[u].z)) + r0[u].z;
+        tr[3] = dd.w ? 0.f : tr[3] + lam * (a[u].w - (w[u].w - w0[u].w)) + r0[u].w;
+    }
+}
+
+__device__ __forceinline__ float adam_step(const TcEpi &e, float g, float &m, float &v) {
+    if (e.sgd) return e.lr * g;
+    m = e.b1 * m + (1.f - e.b1) * g;
+    v = e.b2 * v + (1.f - e.b2) * g * g;
+    return e.lr * (m / e.bc1) / (sqrtf(v / e.bc2) + e.eps);
+}
+
+// Optimizer step for 4 rows x 4 columns of the free block.
+__device__ __forceinline__ void adam_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, const float *t, int tp) {
+    const int64_t col = e.col0 + gj;
+    float4 m[4], v[4], w[4], d[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        if (gi0 + u >= M) break;
+        const int64_t wi = (gi0 + u) * e.ldw + col;
+        if (!e.sgd) {
+            m[u] = ld4(e.mA + wi);
+            v[u] = ld4(e.vA + wi);
+        }
+        w[u] = ld4(e.Wm + wi);
+        d[u] = ld4(e.D + wi);
+    }
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        if (gi0 + u >= M) break;
+        const int64_t wi = (gi0 + u) * e.ldw + col;
+        const float *tr = t + u * tp;
+        float4 st;
+        st.x = adam_step(e, tr[0], m[u].x, v[u].x);
+        st.y = adam_step(e, tr[1], m[u].y, v[u].y);
+        st.z = adam_step(e, tr[2], m[u].z, v[u].z);
+        st.w = adam_step(e, tr[3], m[u].w, v[u].w);
+        if (!e.sgd) {
+            st4(e.mA + wi, m[u]);
+            st4(e.vA + wi, v[u]);
+        }
+        st4(e.Wm + wi, make_float4(w[u].x - st.x, w[u].y - st.y, w[u].z - st.z, w[u].w - st.w));
+        const float4 dn = make_float4(d[u].x - st.x, d[u].y - st.y, d[u].z - st.z, d[u].w - st.w);
+        st4(e.D + wi, dn);
+        const float4 dh = make_float4(tc::tf32_hi(dn.x), tc::tf32_hi(dn.y), tc::tf32_hi(dn.z), tc::tf32_hi(dn.w));
+        st4(e.Dh + wi, dh);
+        st4(e.Dl + wi, make_float4(dn.x - dh.x, dn.y - dh.y, dn.z - dh.z, dn.w - dh.w));
+    }
+}
+
+__device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, float v) {
+    if (e.mode == TC_STORE) {
+        e.C[i * e.ldc + j] = v;
+        return;
+    }
+    const int64_t col = e.col0 + j;
+    const int64_t w = i * e.ldw + col;
+    // TC_ADAM
+    float step;
+    if (e.sgd) {
+        step = e.lr * v;
+    } else {
+        const float mv = e.b1 * e.mA[w] + (1.f - e.b1) * v;
+        const float vv = e.b2 * e.vA[w] + (1.f - e.b2) * v * v;
+        e.mA[w] = mv;
+        e.vA[w] = vv;
+        step = e.lr * (mv / e.bc1) / (sqrtf(vv / e.bc2) + e.eps);
+    }
+    e.Wm[w] -= step;
+    const float d = e.D[w] - step;
+    e.D[w] = d;
+    const float dh = tc::tf32_hi(d);
+    e.Dh[w] = dh;
+    e.Dl[w] = d - dh;
+}
+
+__global__ void __launch_bounds__(128, 1)
+    gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
+                       const TcEpi e, int *err) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
+    uint64_t *empty = full + STAGES;
+    uint64_t *accb = empty + STAGES;
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(accb + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TB;
+    const int nk = (int)((K + KS - 1) / KS);
+
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            tc::mbar_init(tc::smem_u32(&full[s]), 1);
+            tc::mbar_init(tc::smem_u32(&empty[s]), 1);
+        }
+        tc::mbar_init(tc::smem_u32(accb), 1);
+        *abort_flag = 0;
+        tc::fence_barrier_init();
+        tc::prefetch_tmap(&maps.a_hi);
+        tc::prefetch_tmap(&maps.a_lo);
+        tc::prefetch_tmap(&maps.b_hi);
+        tc::prefetch_tmap(&maps.b_lo);
+    }
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), TB);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0 && lane == 0) {
+        // ---------------- TMA producer ----------------
+        int it = 0;
+        for (; it < nk; ++it) {
+            const int s = it % STAGES;
+            const uint32_t r = (uint32_t)(it / STAGES);
+            if (!tc::mbar_wait(tc::smem_u32(&empty[s]), (r & 1u) ^ 1u, abort_flag)) {
+                *abort_flag = 1;
+                break;
+            }
+            const uint32_t fb = tc::smem_u32(&full[s]);
+            tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+            const int x = k_off + it * KS;
+            const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
+            tc::tma_load_2d(base, &maps.a_hi, fb, x, (int)i0);
+            tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, (int)i0);
+            tc::tma_load_2d(base + 2 * PLANE, &maps.b_hi, fb, x, b_row0 + (int)j0);
+            tc::tma_load_2d(base + 3 * PLANE, &maps.b_lo, fb, x, b_row0 + (int)j0);
+        }
+        if (*abort_flag) {
+            int never = 0;
+            for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k)
+                tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (uint32_t)(k / STAGES) & 1u, &never, 100000000ull);
+        }
+    } else if (warp == 1 && lane == 0) {
+        // ---------------- MMA issuer ----------------
+        for (int it = 0; it < nk; ++it) {
+            const int s = it % STAGES;
+            const uint32_t r = (uint32_t)(it / STAGES);
+            if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc::fence_after_sync();
+            const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
+#pragma unroll
+            for (int k = 0; k < KS / 8; ++k) {
+                const uint64_t ah = tc::smem_desc(base + k * 32, 16, 1024, tc::SW_128B);
+                const uint64_t al = tc::smem_desc(base + PLANE + k * 32, 16, 1024, tc::SW_128B);
+                const uint64_t bh = tc::smem_desc(base + 2 * PLANE + k * 32, 16, 1024, tc::SW_128B);
+                const uint64_t bl = tc::smem_desc(base + 3 * PLANE + k * 32, 16, 1024, tc::SW_128B);
+                tc::mma_tf32_ss(tmem, ah, bh, IDESC, (it > 0 || k > 0) ? 1u : 0u);
+                tc::mma_tf32_ss(tmem, ah, bl, IDESC, 1u);
+                tc::mma_tf32_ss(tmem, al, bh, IDESC, 1u);
+            }
+            tc::mma_commit(tc::smem_u32(&empty[s]));
+        }
+        tc::mma_commit(tc::smem_u32(accb));
+    }
+    __syncwarp();
+
+    // ---------------- epilogue ----------------
+    // The accumulator tile goes TMEM -> registers -> shared memory (the
+    // pipeline buffers are free once the last MMA committed), so that global
+    // reads and writes walk rows (or, for P^T, columns) with consecutive lanes.
+    const bool ok = tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
+    tc::fence_after_sync();
+    const bool good = __syncthreads_and(ok && !*abort_flag) != 0 && nk > 0;
+    constexpr int TP = TB + 1;
+    float *T = reinterpret_cast<float *>(smem);
+    if (good) {
+        const int row = warp * 32 + lane;
+#pragma unroll 1
+        for (int c0 = 0; c0 < TB; c0 += 32) {
+            uint32_t v[32];
+            tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+#pragma unroll
+            for (int q = 0; q < 32; ++q) T[row * TP + c0 + q] = __uint_as_float(v[q]);
+        }
+    }
+    __syncthreads();
+    if (good) {
+        // rows of the tile, each lane on 4 consecutive columns; the loads of
+        // 4 rows are issued before any store so they overlap
+        const int cc = lane * 4;
+        const int64_t gj = j0 + cc;
+        const bool vec = e.mode != TC_STORE && gj + 3 < N;
+        for (int rb = warp * 32; rb < warp * 32 + 32; rb += 4) {
+            if (vec) {
+                if (e.mode == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                else bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+            } else {
+                for (int u = 0; u < 4; ++u) {
+                    const int rr = rb + u;
+                    const int64_t gi = i0 + rr;
+                    if (gi >= M) break;
+                    for (int q = 0; q < 4; ++q) {
+                        if (gj + q >= N) break;
+                        float &t = T[rr * TP + cc + q];
+                        if (e.mode == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
+                        else epi_apply(e, gi, gj + q, t);
+                    }
+                }
+            }
+        }
+    }
+    __syncthreads();
+    if (good && e.mode == TC_BGD_P) {
+        // columns of the tile, lanes over rows: P^T rows are contiguous
+        for (int cc = warp * 32; cc < warp * 32 + 32; ++cc) {
+            const int64_t gj = j0 + cc;
+            if (gj >= N) break;
+            for (int rr = lane; rr < TB; rr += 32) {
+                const int64_t gi = i0 + rr;
+                if (gi >= M) break;
+                const float pv = T[rr * TP + cc];
+                const float hi = tc::tf32_hi(pv);
+                e.Pth[gj * e.ldp + gi] = hi;
+                e.Ptl[gj * e.ldp + gi] = pv - hi;
+            }
+        }
+    }
+    if (!good && nk > 0 && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
+    tc::fence_before_sync();
+    __syncthreads();
+    if (warp == 0) tc::tmem_dealloc(tmem, TB);
+}
+
+// hi / lo planes of x (or of alpha x + (1 - alpha) y when y is given)
+__global__ void split_kernel(int64_t count, const float *x, const float *y, float alpha, float *hi, float *lo) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= count) return;
+    const float v = y ? alpha * x[i] + (1.f - alpha) * y[i] : x[i];
+    const float h = tc::tf32_hi(v);
+    hi[i] = h;
+    lo[i] = v - h;
+}
+
+}  // namespace
+
+bool tc_gemm_eligible(int64_t m, int64_t n) {
+    return m % 4 == 0 && n % 4 == 0 && m >= 32 && n >= 32 && m < (1ll << 31) && n < (1ll << 31);
+}
+
+realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const float *y, float alpha, float *hi,
+                        float *lo) {
+    if (count <= 0) return REALQ_OK;
+    {
+        Launch L("tf32_split", s);
+        split_kernel<<<(unsigned)((count + 255) / 256), 256, 0, s>>>(count, x, y, alpha, hi, lo);
+    }
+    return check_launch("tf32_split");
+}
+
+realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
+                            int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
+                            int64_t ldb) {
+    static_assert(sizeof(Maps) <= sizeof(TcMaps), "map storage");
+    Maps *m = reinterpret_cast<Maps *>(out->storage);
+    CUresult r = encode_tmap_2d_f32(&m->a_hi, a_hi, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, KS, TB, 1);
+    if (r == CUDA_SUCCESS)
+        r = encode_tmap_2d_f32(&m->a_lo, a_lo, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, KS, TB, 1);
+    if (r == CUDA_SUCCESS)
+        r = encode_tmap_2d_f32(&m->b_hi, b_hi, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, KS, TB, 1);
+    if (r == CUDA_SUCCESS)
+        r = encode_tmap_2d_f32(&m->b_lo, b_lo, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, KS, TB, 1);
+    if (r != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled (tf32 planes) failed (%d)", (int)r);
+    return REALQ_OK;
+}
+
+realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
+                              int b_row0, const TcEpi &e, int *err, const char *name) {
+    if (M <= 0 || N <= 0) return REALQ_OK;
+    if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
+    static bool configured = false;
+    if (!configured) {
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM));
+        configured = true;
+    }
+    const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
+    {
+        Launch L(name, s);
+        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB)), 128, SMEM, s>>>(
+            m, M, N, K, k_off, b_row0, e, err);
+    }
+    return check_launch(name);
+}
+
+}  // namespace realq

@@ -186,8 +186,25 @@ std::once_flag g_encode_once;
 
 }  // namespace
 
+static CUresult encode_tmap_2d(CUtensorMapDataType dt, CUtensorMap *map, const void *base, uint64_t inner,
+                               uint64_t outer, uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer,
+                               int swizzle128);
+
 CUresult encode_tmap_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
                              uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128) {
+    return encode_tmap_2d(CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, map, base, inner, outer, row_stride_bytes, box_inner,
+                          box_outer, swizzle128);
+}
+
+CUresult encode_tmap_2d_f32(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
+                            uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128) {
+    return encode_tmap_2d(CU_TENSOR_MAP_DATA_TYPE_FLOAT32, map, base, inner, outer, row_stride_bytes, box_inner,
+                          box_outer, swizzle128);
+}
+
+static CUresult encode_tmap_2d(CUtensorMapDataType dt, CUtensorMap *map, const void *base, uint64_t inner,
+                               uint64_t outer, uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer,
+                               int swizzle128) {
     std::call_once(g_encode_once, [] {
         void *fn = nullptr;
         cudaDriverEntryPointQueryResult q;
@@ -201,7 +218,7 @@ CUresult encode_tmap_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner,
     cuuint64_t strides[1] = {row_stride_bytes};
     cuuint32_t box[2] = {box_inner, box_outer};
     cuuint32_t estr[2] = {1, 1};
-    return g_encode(map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void *>(base), dims, strides, box, estr,
+    return g_encode(map, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE,
                     swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);

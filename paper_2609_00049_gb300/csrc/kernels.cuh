@@ -38,6 +38,29 @@ struct GemmArgs {
 };
 realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name);
 
+// ------------------------------------------- tensor-core tf32x3 GEMM ---
+enum TcMode { TC_STORE = 0, TC_BGD_P = 1, TC_ADAM = 2 };
+struct TcEpi {
+    int mode;
+    float *C; int64_t ldc;                                   // TC_STORE
+    const float *Ad; const float *W; const void *W0; int w0_bf16;  // TC_BGD_P
+    const uint8_t *dead; const float *lam; const float *R0; int64_t ldw; int64_t col0;
+    float *Pth; float *Ptl; int64_t ldp;
+    float *Wm; float *mA; float *vA; float *D; float *Dh; float *Dl;  // TC_ADAM (ldw, col0 shared)
+    float lr, b1, b2, eps, bc1, bc2; int sgd;
+};
+struct TcMaps {
+    alignas(64) unsigned char storage[4 * 128];
+};
+bool tc_gemm_eligible(int64_t m, int64_t n);
+realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const float *y, float alpha, float *hi,
+                        float *lo);
+realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
+                            int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
+                            int64_t ldb);
+realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
+                              int b_row0, const TcEpi &e, int *err, const char *name);
+
 // --------------------------------------------------------------- Hessian ---
 int hessian_splits(int64_t n, int64_t T, int num_sms);
 int num_sms();
@@ -79,6 +102,12 @@ struct SweepPlan {
     int *status;
     float *lam;
     float *Et, *P, *G, *Feff, *R0;
+    // tensor-core path: hi / lo planes and tensor maps
+    int tc;
+    float *Dh, *Dl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;
+    TcMaps mapsP, mapsG;
+    int f_split_alpha_valid;
+    float f_split_alpha;
 };
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar);
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);

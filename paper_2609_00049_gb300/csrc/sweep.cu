@@ -324,27 +324,52 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 
 }  // namespace
 
+// Workspace of a sweep.  With Block-GD on shapes the tensor-core path can
+// address (m, n multiples of 4), the gradient GEMMs run as tf32x3 on tcgen05
+// and need hi / lo planes of the displacement, H̄, F and P^T; otherwise the
+// fp32 SIMT path needs P, G (and F_eff).  block = 0: Block-GD only (literal
+// gradient form, SIMT).
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar) {
+    const size_t mn = align_up((size_t)m * n * sizeof(float));
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
     if (has_bgd) {
-        b += 2 * align_up((size_t)m * n * sizeof(float));
-        if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
-        if (has_dbar) b += align_up((size_t)m * n * sizeof(float));
+        if (block > 0 && tc_gemm_eligible(m, n)) {
+            b += 4 * mn + 2 * align_up((size_t)n * n * sizeof(float)) + 2 * align_up((size_t)m * m * sizeof(float));
+        } else {
+            b += 2 * mn;
+            if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
+        }
+        if (has_dbar) b += mn;
     }
     return b;
 }
 
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar) {
     Carve cv(ws);
+    const size_t mn = (size_t)p.m * p.n;
     p.status = cv.take<int>(1);
     p.lam = cv.take<float>(1);
     p.Et = cv.take<float>((size_t)p.block * p.m);
     p.P = p.G = p.Feff = p.R0 = nullptr;
+    p.Dh = p.Dl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = nullptr;
+    p.tc = 0;
     if (has_bgd) {
-        p.P = cv.take<float>((size_t)p.m * p.n);
-        p.G = cv.take<float>((size_t)p.m * p.n);
-        if (has_fnext) p.Feff = cv.take<float>((size_t)p.m * p.m);
-        if (has_dbar) p.R0 = cv.take<float>((size_t)p.m * p.n);
+        if (p.block > 0 && tc_gemm_eligible(p.m, p.n)) {
+            p.tc = 1;
+            p.Dh = cv.take<float>(mn);
+            p.Dl = cv.take<float>(mn);
+            p.Pth = cv.take<float>(mn);
+            p.Ptl = cv.take<float>(mn);
+            p.Hh = cv.take<float>((size_t)p.n * p.n);
+            p.Hl = cv.take<float>((size_t)p.n * p.n);
+            p.Fh = cv.take<float>((size_t)p.m * p.m);
+            p.Fl = cv.take<float>((size_t)p.m * p.m);
+        } else {
+            p.P = cv.take<float>(mn);
+            p.G = cv.take<float>(mn);
+            if (has_fnext) p.Feff = cv.take<float>((size_t)p.m * p.m);
+        }
+        if (has_dbar) p.R0 = cv.take<float>(mn);
     }
 }
 
@@ -440,6 +465,30 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
     return check_launch("bgd_adam");
 }
 
+// One Block-GD step on columns c0..n-1 on the tensor cores (identity form):
+// P^T planes from the displacement planes and H̄ planes, then G = F_eff P with
+// the optimizer step fused into the epilogue.
+static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
+    const int64_t r = p.n - c0;
+    const int64_t k0 = std::min<int64_t>(p.block, c0);   // displacement columns < B are zero
+    TcEpi e{};
+    e.mode = TC_BGD_P;
+    e.Ad = p.disp; e.W = p.W; e.W0 = p.W0; e.w0_bf16 = p.w_dtype == REALQ_BF16;
+    e.dead = p.dead; e.lam = p.lam; e.R0 = p.R0; e.ldw = p.n; e.col0 = c0;
+    e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
+    const int64_t t = ++(*p.adam_t);
+    TcEpi g{};
+    g.mode = TC_ADAM;
+    g.ldw = p.n; g.col0 = c0;
+    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Dh = p.Dh; g.Dl = p.Dl;
+    g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
+    g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
+    g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
+    g.sgd = p.optimizer == REALQ_OPT_SGD;
+    return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
+}
+
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
     if (col_start >= p.n) return REALQ_OK;
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
@@ -494,6 +543,18 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     const int64_t b_global = p.b_global_start + b;
     float alpha = 1.f;
     if (p.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(p.B_total - 1));
+    if (p.tc) {
+        // F_eff planes: split once for a plain F, per block under the sliding window
+        const float a_eff = p.F_next ? alpha : 1.f;
+        if (!p.f_split_alpha_valid || p.f_split_alpha != a_eff) {
+            REALQ_TRY(tc_split(s, p.m * p.m, p.F, (p.F_next && a_eff != 1.f) ? p.F_next : nullptr, a_eff, p.Fh,
+                               p.Fl));
+            p.f_split_alpha_valid = 1;
+            p.f_split_alpha = a_eff;
+        }
+        for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one_tc(s, p, be));
+        return REALQ_OK;
+    }
     const float *Fuse = nullptr;
     REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
     for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, be, Fuse, 1));
@@ -507,7 +568,16 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p) {
         lambda_kernel<<<1, 1024, 0, s>>>(p.n, p.Hbar, p.dead, p.damp, p.lam);
     }
     REALQ_TRY(check_launch("bgd_lambda"));
-    if (p.Dbar) return compute_r0(s, p);
+    if (p.Dbar) REALQ_TRY(compute_r0(s, p));
+    if (p.tc) {
+        // planes of H̄ and of the caller's displacement (so a resumed sweep needs
+        // nothing from an earlier workspace), and the tensor maps of both GEMMs
+        REALQ_TRY(tc_split(s, p.n * p.n, p.Hbar, nullptr, 1.f, p.Hh, p.Hl));
+        REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Dh, p.Dl));
+        REALQ_TRY(tc_make_maps(&p.mapsP, p.Dh, p.Dl, p.m, p.n, p.n, p.Hh, p.Hl, p.n, p.n, p.n));
+        REALQ_TRY(tc_make_maps(&p.mapsG, p.Fh, p.Fl, p.m, p.m, p.m, p.Pth, p.Ptl, p.n, p.m, p.m));
+        p.f_split_alpha_valid = 0;
+    }
     return REALQ_OK;
 }
 

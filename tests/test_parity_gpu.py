@@ -134,12 +134,23 @@ def _oracle_and_gpu(case, qkw, bgd=None, steps=1, with_next=False, b_global_star
     return orc, out, prep, W0
 
 
-def _check(orc, out, case, qkw, bgd, loss_tol=1e-3, prep=None, W0=None):
+def _adam_scale_bound(orc, n, qkw, lr, steps):
+    # per group: optimizer steps applied to its columns before its parameters
+    B = qkw.get("block_size", 128)
+    g = qkw.get("group_size", 128) or n
+    maxq = 2 ** qkw.get("bits", 4) - 1
+    first_cols = np.arange(orc["scale"].shape[1]) * g
+    taken = np.minimum(first_cols // B, max(0, -(-n // B) - 1)) * steps
+    return np.broadcast_to(4.0 * lr * taken / maxq + 1e-12, orc["scale"].shape)
+
+
+def _check(orc, out, case, qkw, bgd, loss_tol=1e-3, prep=None, W0=None, lr=0.0, steps=1):
     n = case.W0.shape[1]
     codes = unpack(out.codes.cpu().numpy(), n)
     rep = compare_codes(codes, orc, qkw.get("block_size", 128), qkw.get("group_size", 128), bgd)
     frac, med, s_unexpl = scale_agreement(out.scale.cpu().numpy(), orc["scale"], qkw.get("group_size", 128),
-                                          explained=compare_codes.last_explained)
+                                          explained=compare_codes.last_explained,
+                                          adam_bound=_adam_scale_bound(orc, n, qkw, lr, steps) if bgd else None)
     print(f"\nparity {qkw} bgd={bgd}: {rep} scale_within_1e-5={frac:.5f} median_rel={med:.2e} "
           f"scale_unexplained={s_unexpl}")
     assert rep["frac_equal"] >= 0.999, rep
@@ -195,7 +206,7 @@ def test_fc256x512_realq(steps):
     qkw = dict(group_size=128, block_size=128)
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=wl.lr, steps=steps)
     assert out.adam_t == orc["adam_t"] == 3 * steps
-    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=wl.lr, steps=steps)
 
 
 @pytest.mark.parametrize("qkw", [dict(group_size=64, block_size=64), dict(group_size=0, symmetric=1),
@@ -203,7 +214,15 @@ def test_fc256x512_realq(steps):
 def test_ragged_shapes_and_quantizer_modes(qkw):
     case = synth.layer_case(24, 200, 300, 1500, outliers=2, dead_cols=(7,))
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4)
-    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=2e-4)
+
+
+def test_simt_fallback_shape():
+    # n not a multiple of 4: the Block-GD GEMMs take the fp32 CUDA-core path
+    case = synth.layer_case(34, 60, 197, 900, outliers=2)
+    qkw = dict(group_size=64, block_size=64)
+    orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=2e-4)
 
 
 def test_block_narrower_than_layer_and_single_block():
@@ -211,7 +230,7 @@ def test_block_narrower_than_layer_and_single_block():
     qkw = dict(group_size=0, block_size=128)
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=1e-4)
     assert out.adam_t == 0
-    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=1e-4)
 
 
 def test_sliding_window():
@@ -219,21 +238,21 @@ def test_sliding_window():
     qkw = dict(group_size=64, block_size=64)
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, with_next=True, b_global_start=3, B_total=9)
     assert [round(x[1], 6) for x in orc["block_loss"]] == [round(1 - k / 8, 6) for k in range(2, 6)]
-    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=2e-4)
 
 
 def test_perturbed_inputs_cross_moment():
     case = synth.layer_case(27, 64, 192, 900, perturbed=True)
     qkw = dict(group_size=64, block_size=64)
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, use_dbar=True)
-    _check(orc, out, case, qkw, True)
+    _check(orc, out, case, qkw, True, lr=2e-4)
 
 
 def test_bf16_weights():
     case = synth.layer_case(28, 128, 256, 1024, bf16=True)
     qkw = dict(group_size=128, block_size=128)
     orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=3e-4, w_bf16=True)
-    _check(orc, out, case, qkw, True, prep=prep, W0=W0)
+    _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=3e-4)
 
 
 def test_resume_matches_single_call():
