@@ -16,7 +16,12 @@ constexpr int BK = 16, THREADS = 256;
 
 template <int AM>
 __device__ __forceinline__ float load_a(const GemmArgs &g, int64_t i, int64_t k) {
-    if (AM == A_ROW) return static_cast<const float *>(g.A)[i * g.lda + k];
+    if (AM == A_ROW) {
+        const float *a = static_cast<const float *>(g.A) + i * g.lda + k;
+        float v = a[0];
+        for (int s = 1; s < g.nsum; ++s) v += a[s * g.aplane];
+        return v;
+    }
     if (AM == A_ROW_BF16) return __bfloat162float(static_cast<const __nv_bfloat16 *>(g.A)[i * g.lda + k]);
     if (AM == A_DIFF_F32)
         return static_cast<const float *>(g.A)[i * g.lda + k] - static_cast<const float *>(g.Y)[i * g.ldy + k];
@@ -28,7 +33,7 @@ __device__ __forceinline__ float load_a(const GemmArgs &g, int64_t i, int64_t k)
 
 template <int EM>
 __device__ __forceinline__ void epilogue(const GemmArgs &g, int64_t gi, int64_t gj, float acc) {
-    float *c = g.C + gi * g.ldc + gj;
+    float *c = g.C + (int64_t)blockIdx.z * g.cplane + gi * g.ldc + gj;
     const float v = g.alpha * acc;
     if (EM == EPI_STORE) *c = v;
     else if (EM == EPI_SUB) *c = *c - v;
@@ -57,7 +62,9 @@ __global__ void __launch_bounds__(THREADS) sgemm_kernel(const GemmArgs g) {
     const int tx = tid & 15, ty = tid >> 4;
     const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
     const int64_t kz = (g.K + gridDim.z - 1) / gridDim.z;
-    const int64_t kbeg = (int64_t)blockIdx.z * kz, kend = min(g.K, kbeg + kz);
+    int64_t kbeg = (int64_t)blockIdx.z * kz;
+    const int64_t kend = min(g.K, kbeg + kz);
+    if (g.a_upper && kbeg < m0) kbeg = m0;
 
     float acc[TM][TN];
 #pragma unroll
@@ -166,15 +173,19 @@ realq_status_t dispatch(cudaStream_t s, EpiMode em, const GemmArgs &g, const cha
     const bool small = big_tiles < num_sms();
     {
         Launch L(name, s);
-        if (small) launch_epi<64, 64, AM>(s, em, g, dim3(ceil_div(g.N, 64), ceil_div(g.M, 64), 1));
-        else launch_epi<128, 128, AM>(s, em, g, dim3(ceil_div(g.N, 128), ceil_div(g.M, 128), 1));
+        const unsigned z = g.ksplit > 1 ? (unsigned)g.ksplit : 1u;
+        if (small) launch_epi<64, 64, AM>(s, em, g, dim3(ceil_div(g.N, 64), ceil_div(g.M, 64), z));
+        else launch_epi<128, 128, AM>(s, em, g, dim3(ceil_div(g.N, 128), ceil_div(g.M, 128), z));
     }
     return check_launch(name);
 }
 
 }  // namespace
 
-realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name) {
+realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g0, const char *name) {
+    GemmArgs g = g0;
+    if (g.nsum < 1) g.nsum = 1;
+    if (g.ksplit > 1 && em != EPI_STORE) return fail(REALQ_ERR_UNSUPPORTED, "%s: split K needs a plain store", name);
     if (g.M <= 0 || g.N <= 0) return REALQ_OK;
     if (g.M > 64LL * 65535LL) return fail(REALQ_ERR_UNSUPPORTED, "%s: GEMM M too large (%lld)", name, (long long)g.M);
     switch (am) {

@@ -32,6 +32,12 @@ struct GemmArgs {
     float *C; int64_t ldc;
     const float *R; int64_t ldr;
     float alpha;
+    // A_ROW only: A(i, k) = sum over s < nsum of A[s * aplane + i * lda + k]
+    int nsum; int64_t aplane;
+    // K split over gridDim.z; EPI_STORE writes slice z to C + z * cplane
+    int ksplit; int64_t cplane;
+    // A(i, k) = 0 for k < i: start each CTA's K range at its first row
+    int a_upper;
     // EPI_BGD_P operands
     const float *Ad; const float *Wc; const void *W0c; int w0_bf16;
     const uint8_t *dead; const float *lam; int64_t col0; int64_t ldw;

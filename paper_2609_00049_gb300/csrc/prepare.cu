@@ -71,13 +71,13 @@ __device__ __forceinline__ void upper_inverse_regs(const float (*Rs)[NB + 1], in
     for (int k = kb - 1; k >= 0; --k) {
         const int kt = k >> 2, kq = k & 3, p = k & 1;
         if (ty == kt) {
-            const float rkk = Rs[k][k];
+            const float rinv = 1.f / Rs[k][k];
 #pragma unroll
             for (int a = 0; a < 4; ++a)
                 if (a == kq) {
 #pragma unroll
                     for (int b = 0; b < 4; ++b) {
-                        v[a][b] = v[a][b] / rkk;
+                        v[a][b] = v[a][b] * rinv;
                         rowk[p][tx * 4 + b] = v[a][b];
                     }
                 }
@@ -134,7 +134,7 @@ __global__ void __launch_bounds__(256) chol_diag_kernel(int64_t n, float *A, int
         }
         __syncthreads();
         if (tx == kt) {
-            const float rk = rk_s[p];
+            const float rinv = 1.f / rk_s[p];
 #pragma unroll
             for (int b = 0; b < 4; ++b)
                 if (b == kq) {
@@ -142,7 +142,7 @@ __global__ void __launch_bounds__(256) chol_diag_kernel(int64_t n, float *A, int
                     for (int a = 0; a < 4; ++a) {
                         const int i = ty * 4 + a;
                         if (i < k) {
-                            sv[a][b] = sv[a][b] / rk;
+                            sv[a][b] = sv[a][b] * rinv;
                             colk[p][i] = sv[a][b];
                         }
                     }
@@ -249,10 +249,12 @@ __global__ void scale_kernel(int64_t count, float div, const float *in, float *o
 }
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
-constexpr size_t prepare_bytes(int64_t n) {
-    return align256(sizeof(int)) + align256(sizeof(float)) + align256((size_t)n * NB * sizeof(float)) +
-           align256((size_t)NB * NB * sizeof(float));
+constexpr int KSPLIT_MAX = 8;    // K slices of the triangular-inverse panel product
+constexpr size_t prepare_bytes_split(int64_t n, int slices) {
+    return align256(sizeof(int)) + align256(sizeof(float)) + align256((size_t)NB * NB * sizeof(float)) +
+           align256((size_t)slices * n * NB * sizeof(float));
 }
+constexpr size_t prepare_bytes(int64_t n) { return prepare_bytes_split(n, 1); }
 
 // Scratch of the allocation-free entry point, sized for n <= REALQ_PREPARE_NOALLOC_MAX_N.
 // Every GPU that loads the library holds it until the process exits.
@@ -281,7 +283,7 @@ realq_status_t noalloc_scratch(void **out) {
 
 }  // namespace
 
-size_t prepare_ws_bytes(int64_t n) { return prepare_bytes(n); }
+size_t prepare_ws_bytes(int64_t n) { return prepare_bytes_split(n, KSPLIT_MAX); }
 
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                                uint8_t *dead, int64_t *fail_col) {
@@ -295,9 +297,12 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
     Carve cv(ws);
     int *status = cv.take<int>(1);
     float *lam = cv.take<float>(1);
-    float *panel = cv.take<float>((size_t)n * NB);
     float *Vd = cv.take<float>((size_t)NB * NB);
-    (void)ws_bytes;
+    float *panel = cv.take<float>(0);
+    // as many K slices of the panel product as the workspace holds
+    int slices = 1;
+    while (slices < KSPLIT_MAX && prepare_bytes_split(n, slices + 1) <= ws_bytes) ++slices;
+    const int64_t plane = n * NB;
     REALQ_CUDA_TRY(cudaMemsetAsync(status, 0xFF, sizeof(int), s));
     const int64_t tot = n * n;
     {
@@ -347,16 +352,20 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
         }
         REALQ_TRY(check_launch("trtri_diag"));
         if (j0 == 0) continue;
+        // X = U[0:j0, 0:j0] R[0:j0, J] (U upper: row block i starts its K at i),
+        // K split into fixed-order slices summed by the next product's A load
+        const int ks = (int)std::max<int64_t>(1, std::min<int64_t>(slices, j0 / 512));
         GemmArgs g{};
         g.M = j0; g.N = jb; g.K = j0;
         g.A = U; g.lda = n;
         g.B = U + j0; g.ldb = n;
         g.C = panel; g.ldc = NB;
+        g.ksplit = ks; g.cplane = plane; g.a_upper = 1;
         g.alpha = 1.f;
         REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "trtri_trmm"));
         GemmArgs h{};
         h.M = j0; h.N = jb; h.K = jb;
-        h.A = panel; h.lda = NB;
+        h.A = panel; h.lda = NB; h.nsum = ks; h.aplane = plane;
         h.B = Vd; h.ldb = NB;
         h.C = U + j0; h.ldc = n;
         h.alpha = -1.f;
