@@ -12,7 +12,6 @@
 namespace realq {
 namespace {
 
-constexpr int QB_THREADS = 128;
 
 // quant(.) grid of one group from its min / max (the reading fixed by the
 // oracle: the grid contains 0; degenerate groups get [-1, 1]).  fp32, IEEE
@@ -85,126 +84,179 @@ struct QArgs {
 };
 
 // Column-serial quantize + in-block OBS propagation for block [bs, bs + kb).
-// One thread owns one row.  The block is walked in sub-blocks of 32 columns:
-// the current sub-block lives in registers (unrolled), the rest of the row in
-// shared memory (thread-major, conflict-free); inside the sub-block every
-// column's error is fed to the later columns of the sub-block at once, and
-// after it the 32 errors are applied to every later column in column order,
-// so the arithmetic is that of the plain column loop.  U's diagonal block is
-// staged transposed (Ut[k][j] = U[j][k]) so the 32 coefficients of a later
-// column are contiguous.  The sub-block loop is not unrolled: the whole kernel
-// body stays small enough for the instruction cache.  G > 0: group
-// parameters are computed here at every G-th column (G a multiple of 32) from
-// the current weights; G = 0: they were computed before the block.
+// A CTA takes QB_ROWS rows and B/32 warps: warp w keeps columns
+// [32w, 32w + 32) of the CTA's rows in registers (lane = row).  Phase s: warp
+// s quantizes its 32 columns one after the other, feeding each column's error
+// to its later columns at once, and publishes the 32 errors of every row;
+// then every warp w > s applies them to its columns, column by column in
+// order, so each weight sees exactly the updates of the plain column loop.
+// U's B x B diagonal block is staged once in shared memory (rows padded to
+// keep float4 reads aligned).  G > 0: group parameters are computed at every
+// G-th column (a multiple of 32) from the current weights, with the min / max
+// of the group's sub-blocks gathered through shared memory; G = 0: they were
+// computed before the block.
+constexpr int QB_ROWS = 32;
+
 template <int B, int G>
-__global__ void __launch_bounds__(QB_THREADS) quant_block_kernel(const QArgs a) {
+__global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
+    constexpr int NW = B / 32;            // warps = sub-blocks
+    constexpr int UP = B + 4;             // U row pitch (floats)
     extern __shared__ __align__(16) float qsm[];
-    constexpr int UP = B + 4;             // row pitch of Ut: aligned float4 rows, 4-way store conflicts
-    float *Ut = qsm;                      // B x UP, Ut[k * UP + j] = U[j][k] for j < k, else 0
-    float *invd = Ut + B * UP;            // B
-    constexpr int RP = QB_THREADS + 1;    // row pitch of rs (conflict-free both ways)
-    float *rs = invd + B;                 // B x RP, rs[k * RP + row]
+    float *Us = qsm;                      // B x UP: U[j][k] for j < k, else 0
+    float *invd = Us + B * UP;            // B
+    float *Es = invd + B;                 // QB_ROWS x 33: errors of the current sub-block
+    float *mm = Es + QB_ROWS * 33;        // 2 x NW x QB_ROWS: group min / max partials
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int kb = a.kb;
-    // Stage U's diagonal block (transposed) and the CTA's rows x kb slab of W
-    // (read along rows) with asynchronous 4-byte copies, all in flight at once;
-    // the entries that must be zero are written directly.
-    for (int idx = threadIdx.x; idx < B * B; idx += blockDim.x) {
-        const int j = idx / B, k = idx % B;   // U row j, contiguous in k
-        float *dst = Ut + k * UP + j;
-        if (j < kb && k < kb && k > j) cp_async4(dst, a.U + (a.bs + j) * a.n + a.bs + k);
-        else *dst = 0.f;
-    }
-    const int64_t row0 = (int64_t)blockIdx.x * blockDim.x;
-    for (int rr = 0; rr < QB_THREADS; ++rr) {
-        const int64_t gi = row0 + rr;
-        for (int c = threadIdx.x; c < B; c += blockDim.x) {
-            float *dst = rs + c * RP + rr;
-            if (gi < a.m && c < kb) cp_async4(dst, a.W + gi * a.n + a.bs + c);
-            else *dst = 0.f;
+    if ((a.n & 3) == 0 && kb == B) {
+        for (int idx = threadIdx.x; idx < B * B / 4; idx += blockDim.x) {
+            const int j = (idx * 4) / B, k = (idx * 4) % B;
+            const float4 v = *reinterpret_cast<const float4 *>(a.U + (a.bs + j) * a.n + a.bs + k);
+            float *d = Us + j * UP + k;
+            d[0] = (k + 0 > j) ? v.x : 0.f;
+            d[1] = (k + 1 > j) ? v.y : 0.f;
+            d[2] = (k + 2 > j) ? v.z : 0.f;
+            d[3] = (k + 3 > j) ? v.w : 0.f;
+        }
+    } else {
+        for (int idx = threadIdx.x; idx < B * B; idx += blockDim.x) {
+            const int j = idx / B, k = idx % B;
+            Us[j * UP + k] = (j < kb && k < kb && k > j) ? a.U[(a.bs + j) * a.n + a.bs + k] : 0.f;
         }
     }
     for (int j = threadIdx.x; j < B; j += blockDim.x)
         invd[j] = (j < kb) ? 1.f / a.U[(a.bs + j) * a.n + a.bs + j] : 0.f;
-    asm volatile("cp.async.wait_all;" ::: "memory");
-    __syncthreads();
-    const int64_t i = row0 + threadIdx.x;
-    const bool live = i < a.m;
 
+    const int64_t i = (int64_t)blockIdx.x * QB_ROWS + lane;   // this lane's row
+    const bool live = i < a.m;
+    const int c0 = warp * 32;                                   // this warp's first column
+    float r[32];
+    {
+        const float *wrow = a.W + (live ? i : 0) * a.n + a.bs + c0;
+        if ((a.n & 3) == 0 && c0 + 32 <= kb) {
+#pragma unroll
+            for (int c = 0; c < 32; c += 4) {
+                const float4 v = live ? *reinterpret_cast<const float4 *>(wrow + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                r[c] = v.x; r[c + 1] = v.y; r[c + 2] = v.z; r[c + 3] = v.w;
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) r[c] = (live && c0 + c < kb) ? wrow[c] : 0.f;
+        }
+    }
     float sc = 1.f, zr = 0.f;
-    if (live && G == 0) {
+    if (G == 0 && live) {
         const int gi = (int)(a.bs / a.g);
         sc = a.scale[i * a.ngroups + gi];
         zr = (float)a.zero[i * a.ngroups + gi];
     }
+    __syncthreads();
+
     const float maxq = (float)((1 << a.bits) - 1);
-    uint8_t *crow = a.codes + (live ? i : 0) * a.ncb + a.bs / 2;
     bool bad = false;
 #pragma unroll 1
-    for (int s0 = 0; live && s0 < kb; s0 += 32) {
-        float r[32], e[32];
+    for (int s = 0; s < NW && s * 32 < kb; ++s) {
+        if (G > 0 && ((s * 32) % (G > 0 ? G : 1)) == 0) {
+            // min / max of the group's columns (sub-blocks s .. s + G/32 - 1)
+            constexpr int GS = (G > 0 ? G : 32) / 32;
+            if (warp >= s && warp < s + GS) {
+                float mn = 0.f, mx = 0.f;
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) r[jj] = rs[(s0 + jj) * RP + threadIdx.x];
-        if (G > 0 && (s0 % (G > 0 ? G : 1)) == 0) {
-            float mn = 0.f, mx = 0.f;
-            for (int c = s0; c < s0 + G && c < kb; ++c) {
-                const float w = rs[c * RP + threadIdx.x];
-                mn = fminf(mn, w);
-                mx = fmaxf(mx, w);
+                for (int c = 0; c < 32; ++c)
+                    if (c0 + c < kb) {
+                        mn = fminf(mn, r[c]);
+                        mx = fmaxf(mx, r[c]);
+                    }
+                mm[warp * QB_ROWS + lane] = mn;
+                mm[(NW + warp) * QB_ROWS + lane] = mx;
             }
-            grid_params(mn, mx, a.bits, a.sym, sc, zr);
-            const int gi = (int)((a.bs + s0) / a.g);
-            a.scale[i * a.ngroups + gi] = sc;
-            a.zero[i * a.ngroups + gi] = (uint8_t)zr;
+            __syncthreads();
+            if (warp == s) {
+                float mn = 0.f, mx = 0.f;
+                for (int w = s; w < s + GS && w < NW; ++w) {
+                    mn = fminf(mn, mm[w * QB_ROWS + lane]);
+                    mx = fmaxf(mx, mm[(NW + w) * QB_ROWS + lane]);
+                }
+                grid_params(mn, mx, a.bits, a.sym, sc, zr);
+                if (live) {
+                    const int gi = (int)((a.bs + s * 32) / a.g);
+                    a.scale[i * a.ngroups + gi] = sc;
+                    a.zero[i * a.ngroups + gi] = (uint8_t)zr;
+                }
+                // the next sub-blocks of the same group quantize with these parameters
+                mm[lane] = sc;
+                mm[QB_ROWS + lane] = zr;
+            }
+            __syncthreads();
+            if (warp > s && warp < s + GS) {
+                sc = mm[lane];
+                zr = mm[QB_ROWS + lane];
+            }
         }
-        unsigned lo = 0;
+        if (warp == s) {
+            uint32_t packed[4] = {0u, 0u, 0u, 0u};
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) {
-            const int j = s0 + jj;
-            e[jj] = 0.f;
-            if (j < kb) {
-                const float w = r[jj];
-                bad |= !isfinite(w);
-                float q = rintf(w / sc) + zr;
-                q = fminf(fmaxf(q, 0.f), maxq);
-                const float dq = sc * (q - zr);
-                const float err = (w - dq) * invd[j];
-                e[jj] = err;
-                a.Et[(int64_t)j * a.m + i] = err;
-                r[jj] = dq;
+            for (int jj = 0; jj < 32; ++jj) {
+                const int j = c0 + jj;
+                float err = 0.f;
+                uint32_t qi = 0;
+                if (j < kb) {
+                    const float w = r[jj];
+                    bad |= !isfinite(w);
+                    float q = rintf(w / sc) + zr;
+                    q = fminf(fmaxf(q, 0.f), maxq);
+                    const float dq = sc * (q - zr);
+                    err = (w - dq) * invd[j];
+                    r[jj] = dq;
+                    qi = (uint32_t)q;
 #pragma unroll
-                for (int kk = jj + 1; kk < 32; ++kk) r[kk] = fmaf(-err, Ut[(s0 + kk) * UP + j], r[kk]);
-                const unsigned qi = (unsigned)q;
-                if ((jj & 1) == 0) {
-                    lo = qi;
-                    if (j == kb - 1) crow[j / 2] = (uint8_t)lo;
+                    for (int kk = jj + 1; kk < 32; ++kk) r[kk] = fmaf(-err, Us[j * UP + c0 + kk], r[kk]);
+                }
+                Es[lane * 33 + jj] = err;
+                if (live && j < kb) a.Et[(int64_t)j * a.m + i] = err;
+                packed[jj >> 3] |= (qi & 15u) << ((jj & 7) * 4);
+            }
+            if (live) {
+                uint8_t *crow = a.codes + i * a.ncb + (a.bs + c0) / 2;
+                if (c0 + 32 <= kb && (((uintptr_t)crow) & 15) == 0) {
+                    *reinterpret_cast<uint4 *>(crow) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
                 } else {
-                    crow[j / 2] = (uint8_t)(lo | (qi << 4));
+                    for (int jj = 0; jj < 32 && c0 + jj < kb; jj += 2)
+                        crow[jj / 2] = (uint8_t)((packed[jj >> 3] >> ((jj & 7) * 4)) & 0xFFu);
                 }
             }
         }
+        __syncthreads();
+        if (warp > s) {
+            // the 32 errors of sub-block s, column by column in order
+            float e[32];
 #pragma unroll
-        for (int jj = 0; jj < 32; ++jj) rs[(s0 + jj) * RP + threadIdx.x] = r[jj];
-        // the 32 errors, column by column in order, into every later column
-#pragma unroll 2
-        for (int k = s0 + 32; k < kb; ++k) {
-            float acc = rs[k * RP + threadIdx.x];
-            const float4 *u4 = reinterpret_cast<const float4 *>(Ut + k * UP + s0);
+            for (int jj = 0; jj < 32; ++jj) e[jj] = Es[lane * 33 + jj];
 #pragma unroll
-            for (int q4 = 0; q4 < 8; ++q4) {
-                const float4 u = u4[q4];
-                acc = fmaf(-e[q4 * 4 + 0], u.x, acc);
-                acc = fmaf(-e[q4 * 4 + 1], u.y, acc);
-                acc = fmaf(-e[q4 * 4 + 2], u.z, acc);
-                acc = fmaf(-e[q4 * 4 + 3], u.w, acc);
+            for (int jj = 0; jj < 32; ++jj) {
+                const float *urow = Us + (s * 32 + jj) * UP + c0;
+#pragma unroll
+                for (int c = 0; c < 32; c += 4) {
+                    const float4 u = *reinterpret_cast<const float4 *>(urow + c);
+                    r[c] = fmaf(-e[jj], u.x, r[c]);
+                    r[c + 1] = fmaf(-e[jj], u.y, r[c + 1]);
+                    r[c + 2] = fmaf(-e[jj], u.z, r[c + 2]);
+                    r[c + 3] = fmaf(-e[jj], u.w, r[c + 3]);
+                }
             }
-            rs[k * RP + threadIdx.x] = acc;
         }
+        __syncthreads();
     }
-    __syncthreads();
-    for (int rr = 0; rr < QB_THREADS; ++rr) {
-        const int64_t gi = row0 + rr;
-        if (gi >= a.m) break;
-        for (int c = threadIdx.x; c < kb; c += blockDim.x) a.W[gi * a.n + a.bs + c] = rs[c * RP + rr];
+    if (live) {
+        float *wout = a.W + i * a.n + a.bs + c0;
+        if ((a.n & 3) == 0 && c0 + 32 <= kb) {
+#pragma unroll
+            for (int c = 0; c < 32; c += 4) *reinterpret_cast<float4 *>(wout + c) = make_float4(r[c], r[c + 1], r[c + 2], r[c + 3]);
+        } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+                if (c0 + c < kb) wout[c] = r[c];
+        }
     }
     if (bad) atomicOr(a.status, ST_NONFINITE);
 }
@@ -300,7 +352,7 @@ inline unsigned blocks_for(int64_t count, int threads = 256) { return (unsigned)
 
 template <int B, int G>
 realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
-    const size_t smem = (size_t)(B * (B + 4) + B + B * (QB_THREADS + 1)) * sizeof(float);
+    const size_t smem = (size_t)(B * (B + 4) + B + QB_ROWS * 33 + 2 * (B / 32) * QB_ROWS) * sizeof(float);
     static bool configured = false;
     if (!configured) {
         REALQ_CUDA_TRY(cudaFuncSetAttribute(quant_block_kernel<B, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
@@ -308,7 +360,7 @@ realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
     }
     {
         Launch L("quant_block", s);
-        quant_block_kernel<B, G><<<ceil_div(qa.m, QB_THREADS), QB_THREADS, smem, s>>>(qa);
+        quant_block_kernel<B, G><<<ceil_div(qa.m, QB_ROWS), B, smem, s>>>(qa);
     }
     return check_launch("quant_block");
 }
