@@ -63,8 +63,9 @@ __global__ void __launch_bounds__(THREADS) sgemm_kernel(const GemmArgs g) {
     const int64_t m0 = (int64_t)blockIdx.y * BM, n0 = (int64_t)blockIdx.x * BN;
     const int64_t kz = (g.K + gridDim.z - 1) / gridDim.z;
     int64_t kbeg = (int64_t)blockIdx.z * kz;
-    const int64_t kend = min(g.K, kbeg + kz);
+    int64_t kend = min(g.K, kbeg + kz);
     if (g.a_upper && kbeg < m0) kbeg = m0;
+    if (g.b_upper && kend > n0 + BN) kend = n0 + BN;
 
     float acc[TM][TN];
 #pragma unroll
@@ -88,7 +89,13 @@ __global__ void __launch_bounds__(THREADS) sgemm_kernel(const GemmArgs g) {
             const int idx = tid + r * THREADS;
             const int kk = idx / BN, jj = idx % BN;
             const int64_t gk = k0 + kk, gj = n0 + jj;
-            rb[r] = (gk < kend && gj < g.N) ? g.B[gk * g.ldb + gj] : 0.f;
+            float bv = 0.f;
+            if (gk < kend && gj < g.N) {
+                const float *bp = g.B + gk * g.ldb + gj;
+                bv = bp[0];
+                for (int s2 = 1; s2 < g.nsum_b; ++s2) bv += bp[s2 * g.bplane];
+            }
+            rb[r] = bv;
         }
     };
     auto stash = [&](int buf) {
@@ -185,6 +192,7 @@ realq_status_t dispatch(cudaStream_t s, EpiMode em, const GemmArgs &g, const cha
 realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g0, const char *name) {
     GemmArgs g = g0;
     if (g.nsum < 1) g.nsum = 1;
+    if (g.nsum_b < 1) g.nsum_b = 1;
     if (g.ksplit > 1 && em != EPI_STORE) return fail(REALQ_ERR_UNSUPPORTED, "%s: split K needs a plain store", name);
     if (g.M <= 0 || g.N <= 0) return REALQ_OK;
     if (g.M > 64LL * 65535LL) return fail(REALQ_ERR_UNSUPPORTED, "%s: GEMM M too large (%lld)", name, (long long)g.M);

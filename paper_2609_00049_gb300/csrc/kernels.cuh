@@ -38,6 +38,10 @@ struct GemmArgs {
     int ksplit; int64_t cplane;
     // A(i, k) = 0 for k < i: start each CTA's K range at its first row
     int a_upper;
+    // B(k, j) = 0 for k > j: end each CTA's K range at its last column
+    int b_upper;
+    // B(k, j) = sum over s < nsum_b of B[s * bplane + k * ldb + j]
+    int nsum_b; int64_t bplane;
     // EPI_BGD_P operands
     const float *Ad; const float *Wc; const void *W0c; int w0_bf16;
     const uint8_t *dead; const float *lam; int64_t col0; int64_t ldw;

@@ -167,19 +167,20 @@ __global__ void __launch_bounds__(256) chol_diag_kernel(int64_t n, float *A, int
 #pragma unroll
     for (int a = 0; a < 4; ++a)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int r = ty * 4 + a, c = tx * 4 + b;
-            Rs[r][c] = sv[a][b];
-            if (r < kb && c < kb && c >= r) A[(k0 + r) * n + k0 + c] = sv[a][b];
-        }
+        for (int b = 0; b < 4; ++b) Rs[ty * 4 + a][tx * 4 + b] = sv[a][b];
     __syncthreads();
     __shared__ float rowk[2][NB];
     float v[4][4];
     upper_inverse_regs(Rs, kb, v, rowk);
+    // U_KK = R_KK^-1 goes to A[K, K]; Vt = U_KK^T feeds the panel solve
 #pragma unroll
     for (int a = 0; a < 4; ++a)
 #pragma unroll
-        for (int b = 0; b < 4; ++b) Vt[(tx * 4 + b) * NB + ty * 4 + a] = v[a][b];
+        for (int b = 0; b < 4; ++b) {
+            const int r = ty * 4 + a, c = tx * 4 + b;
+            if (r < kb && c < kb && c >= r) A[(k0 + r) * n + k0 + c] = v[a][b];
+            Vt[c * NB + r] = v[a][b];
+        }
 }
 
 // A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles).
@@ -218,29 +219,6 @@ __global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, i
             if (gi < k0 && gj < k0 && gj >= gi) A[gi * n + gj] -= acc[p][q];
         }
     }
-}
-
-// V = R_JJ^-1 (upper); written to A[J, J] and to the dense 64 x 64 buffer Vd
-// (zeros below the diagonal).
-__global__ void __launch_bounds__(256) trtri_diag_kernel(int64_t n, float *A, int64_t j0, int jb, float *Vd) {
-    __shared__ float Rs[NB][NB + 1];
-    __shared__ float rowk[2][NB];
-    for (int idx = threadIdx.x; idx < NB * NB; idx += blockDim.x) {
-        const int r = idx / NB, c = idx % NB;
-        Rs[r][c] = (r < jb && c < jb && c >= r) ? A[(j0 + r) * n + j0 + c] : 0.f;
-    }
-    __syncthreads();
-    float v[4][4];
-    upper_inverse_regs(Rs, jb, v, rowk);
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-#pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int r = ty * 4 + a, c = tx * 4 + b;
-            Vd[r * NB + c] = v[a][b];
-            if (r < jb && c < jb && c >= r) A[(j0 + r) * n + j0 + c] = v[a][b];
-        }
 }
 
 __global__ void scale_kernel(int64_t count, float div, const float *in, float *out) {
@@ -315,61 +293,59 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
         prep_damp_kernel<<<1, 1024, 0, s>>>(n, U, damp, lam);
     }
     REALQ_TRY(check_launch("prepare_damp"));
-    // reverse-order blocked Cholesky: Hd = R R^T
+    // Reverse-order blocked Cholesky Hd = R R^T, with U = R^-1 formed block row
+    // by block row as soon as a row block of R is final: after step K no later
+    // step reads row block K of R, and
+    //   U[K, K] = R_KK^-1,  U[K, K+1:] = -U[K, K] (R[K, K+1:] U[K+1:, K+1:]).
     const int nbk = ceil_div(n, NB);
     for (int K = nbk - 1; K >= 0; --K) {
         const int64_t k0 = (int64_t)K * NB;
         const int kb = (int)std::min<int64_t>(NB, n - k0);
+        const int64_t k1 = k0 + kb;
         {
             Launch L("chol_diag", s);
             chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status, Vd);
         }
         REALQ_TRY(check_launch("chol_diag"));
-        if (k0 == 0) continue;
-        // rows above the block: R[0:k0, K] = A[0:k0, K] R_KK^-T (in place; one
-        // column tile, so every CTA reads only the rows it writes)
-        GemmArgs pg{};
-        pg.M = k0; pg.N = kb; pg.K = kb;
-        pg.A = U + k0; pg.lda = n;
-        pg.B = Vd; pg.ldb = NB;
-        pg.C = U + k0; pg.ldc = n;
-        pg.alpha = 1.f;
-        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, pg, "chol_panel"));
-        const int64_t nt0 = k0 / NB;
-        {
-            Launch L("chol_update", s);
-            chol_update_kernel<<<(unsigned)(nt0 * (nt0 + 1) / 2), 256, 0, s>>>(n, U, k0, kb);
+        if (k0 > 0) {
+            // rows above the block: R[0:k0, K] = A[0:k0, K] R_KK^-T (in place; one
+            // column tile, so every CTA reads only the rows it writes)
+            GemmArgs pg{};
+            pg.M = k0; pg.N = kb; pg.K = kb;
+            pg.A = U + k0; pg.lda = n;
+            pg.B = Vd; pg.ldb = NB;
+            pg.C = U + k0; pg.ldc = n;
+            pg.alpha = 1.f;
+            REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, pg, "chol_panel"));
+            const int64_t nt0 = k0 / NB;
+            {
+                Launch L("chol_update", s);
+                chol_update_kernel<<<(unsigned)(nt0 * (nt0 + 1) / 2), 256, 0, s>>>(n, U, k0, kb);
+            }
+            REALQ_TRY(check_launch("chol_update"));
         }
-        REALQ_TRY(check_launch("chol_update"));
-    }
-    // U = R^-1, block columns left to right
-    for (int J = 0; J < nbk; ++J) {
-        const int64_t j0 = (int64_t)J * NB;
-        const int jb = (int)std::min<int64_t>(NB, n - j0);
-        {
-            Launch L("trtri_diag", s);
-            trtri_diag_kernel<<<1, 256, 0, s>>>(n, U, j0, jb, Vd);
+        if (k1 < n) {
+            const int64_t r = n - k1;
+            // X = R[K, K+1:] U[K+1:, K+1:] (U upper: a column tile's K range ends
+            // at its last column), K split into fixed-order slices
+            const int ks = (int)std::max<int64_t>(1, std::min<int64_t>(slices, r / 512));
+            GemmArgs g{};
+            g.M = kb; g.N = r; g.K = r;
+            g.A = U + k0 * n + k1; g.lda = n;
+            g.B = U + k1 * n + k1; g.ldb = n;
+            g.C = panel; g.ldc = n;
+            g.ksplit = ks; g.cplane = plane; g.b_upper = 1;
+            g.alpha = 1.f;
+            REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "trtri_trmm"));
+            // U[K, K+1:] = -U_KK X  (U_KK = Vt^T, read K-major from Vt)
+            GemmArgs h{};
+            h.M = kb; h.N = r; h.K = kb;
+            h.A = Vd; h.lda = NB;
+            h.B = panel; h.ldb = n; h.nsum_b = ks; h.bplane = plane;
+            h.C = U + k0 * n + k1; h.ldc = n;
+            h.alpha = -1.f;
+            REALQ_TRY(gemm_f32(s, A_KMAJOR, EPI_STORE, h, "trtri_panel"));
         }
-        REALQ_TRY(check_launch("trtri_diag"));
-        if (j0 == 0) continue;
-        // X = U[0:j0, 0:j0] R[0:j0, J] (U upper: row block i starts its K at i),
-        // K split into fixed-order slices summed by the next product's A load
-        const int ks = (int)std::max<int64_t>(1, std::min<int64_t>(slices, j0 / 512));
-        GemmArgs g{};
-        g.M = j0; g.N = jb; g.K = j0;
-        g.A = U; g.lda = n;
-        g.B = U + j0; g.ldb = n;
-        g.C = panel; g.ldc = NB;
-        g.ksplit = ks; g.cplane = plane; g.a_upper = 1;
-        g.alpha = 1.f;
-        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "trtri_trmm"));
-        GemmArgs h{};
-        h.M = j0; h.N = jb; h.K = jb;
-        h.A = panel; h.lda = NB; h.nsum = ks; h.aplane = plane;
-        h.B = Vd; h.ldb = NB;
-        h.C = U + j0; h.ldc = n;
-        h.alpha = -1.f;
-        REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, h, "trtri_panel"));
     }
     int host_status = -1;
     REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
