@@ -14,6 +14,7 @@
 #include "kernels.cuh"
 
 #include <mutex>
+#include <vector>
 
 namespace realq {
 namespace {
@@ -263,15 +264,54 @@ realq_status_t noalloc_scratch(void **out) {
 
 size_t prepare_ws_bytes(int64_t n) { return prepare_bytes_split(n, KSPLIT_MAX); }
 
+realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap);
+
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                                uint8_t *dead, int64_t *fail_col) {
     void *scratch = nullptr;
     REALQ_TRY(noalloc_scratch(&scratch));
-    return prepare(s, n, T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes);
+    // single stream: this entry point creates no stream or event
+    return prepare_impl(s, n, T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes, false);
+}
+
+// Auxiliary stream of the calling thread (and its events) for the U row
+// work, created on first use per device and kept for the life of the thread.
+struct AuxStream {
+    int device = -1;
+    cudaStream_t stream = nullptr;
+    cudaEvent_t ev[2] = {nullptr, nullptr};
+    std::vector<cudaEvent_t> steps;
+};
+static thread_local AuxStream g_aux;
+
+realq_status_t aux_for(int64_t nsteps, AuxStream **out) {
+    int dev = 0;
+    REALQ_CUDA_TRY(cudaGetDevice(&dev));
+    AuxStream &a = g_aux;
+    if (a.device != dev) {
+        a = AuxStream{};
+        REALQ_CUDA_TRY(cudaStreamCreateWithFlags(&a.stream, cudaStreamNonBlocking));
+        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[0], cudaEventDisableTiming));
+        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[1], cudaEventDisableTiming));
+        a.device = dev;
+    }
+    while ((int64_t)a.steps.size() < nsteps) {
+        cudaEvent_t e;
+        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+        a.steps.push_back(e);
+    }
+    *out = &a;
+    return REALQ_OK;
 }
 
 realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes) {
+    return prepare_impl(s, n, T, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true);
+}
+
+realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap) {
     Carve cv(ws);
     int *status = cv.take<int>(1);
     float *lam = cv.take<float>(1);
@@ -298,6 +338,16 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
     // step reads row block K of R, and
     //   U[K, K] = R_KK^-1,  U[K, K+1:] = -U[K, K] (R[K, K+1:] U[K+1:, K+1:]).
     const int nbk = ceil_div(n, NB);
+    // Row block K of U touches rows >= k0 only, the later Cholesky steps rows
+    // < k0 only: with overlap, the U row work runs on an auxiliary stream that
+    // starts after the diagonal step of K (which wrote U_KK into A[K, K]).
+    AuxStream *aux = nullptr;
+    if (overlap && nbk > 1) REALQ_TRY(aux_for(nbk, &aux));
+    cudaStream_t rs = aux ? aux->stream : s;
+    if (aux) {
+        REALQ_CUDA_TRY(cudaEventRecord(aux->ev[0], s));
+        REALQ_CUDA_TRY(cudaStreamWaitEvent(rs, aux->ev[0], 0));
+    }
     for (int K = nbk - 1; K >= 0; --K) {
         const int64_t k0 = (int64_t)K * NB;
         const int kb = (int)std::min<int64_t>(NB, n - k0);
@@ -307,6 +357,10 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
             chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status, Vd);
         }
         REALQ_TRY(check_launch("chol_diag"));
+        if (aux && k1 < n) {
+            REALQ_CUDA_TRY(cudaEventRecord(aux->steps[K], s));
+            REALQ_CUDA_TRY(cudaStreamWaitEvent(rs, aux->steps[K], 0));
+        }
         if (k0 > 0) {
             // rows above the block: R[0:k0, K] = A[0:k0, K] R_KK^-T (in place; one
             // column tile, so every CTA reads only the rows it writes)
@@ -336,16 +390,20 @@ realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const f
             g.C = panel; g.ldc = n;
             g.ksplit = ks; g.cplane = plane; g.b_upper = 1;
             g.alpha = 1.f;
-            REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, g, "trtri_trmm"));
-            // U[K, K+1:] = -U_KK X  (U_KK = Vt^T, read K-major from Vt)
+            REALQ_TRY(gemm_f32(rs, A_ROW, EPI_STORE, g, "trtri_trmm"));
+            // U[K, K+1:] = -U_KK X, U_KK read from A[K, K] (upper, zeros below)
             GemmArgs h{};
             h.M = kb; h.N = r; h.K = kb;
-            h.A = Vd; h.lda = NB;
+            h.A = U + k0 * n + k0; h.lda = n;
             h.B = panel; h.ldb = n; h.nsum_b = ks; h.bplane = plane;
             h.C = U + k0 * n + k1; h.ldc = n;
             h.alpha = -1.f;
-            REALQ_TRY(gemm_f32(s, A_KMAJOR, EPI_STORE, h, "trtri_panel"));
+            REALQ_TRY(gemm_f32(rs, A_ROW, EPI_STORE, h, "trtri_panel"));
         }
+    }
+    if (aux) {
+        REALQ_CUDA_TRY(cudaEventRecord(aux->ev[1], rs));
+        REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[1], 0));
     }
     int host_status = -1;
     REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
