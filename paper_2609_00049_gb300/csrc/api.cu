@@ -310,7 +310,7 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
     cudaStream_t s = S(stream);
     REALQ_CUDA_TRY(cudaMemsetAsync(p.status, 0, sizeof(int), s));
     if (block_begin == 0) REALQ_TRY(sweep_init(s, p));
-    REALQ_TRY(sweep_prologue_r0(s, p));
+    REALQ_TRY(sweep_prologue_r0(s, p, block_begin == 0));
     for (int64_t b = block_begin; b < block_end; ++b) REALQ_TRY(sweep_block(s, p, b));
     return REALQ_OK;
 }

@@ -14,11 +14,13 @@
 // 3 x 4 tcgen05.mma (kind::tf32, K = 8) per stage into a TMEM accumulator,
 // and four warps drain it through one of the epilogues:
 //   TC_STORE  C = acc
-//   TC_BGD_P  the Block-GD gradient factor after the lazy OBS update,
-//             p = acc + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead
-//             channels, written transposed and split (P^T hi / lo planes)
+//   TC_BGD_P  the Block-GD gradient factor after the lazy OBS update: the
+//             running product M = A_disp H̄ takes the latest step (acc),
+//             M += acc, and p = M + lambda (A_disp - (W - W0)) (+ W0 Dbar),
+//             0 on dead channels, written transposed and split (P^T hi / lo)
 //   TC_ADAM   g = acc: one Adam (or SGD) step on W[:, col0 + j], updating the
-//             moments and the displacement (full value and hi / lo planes)
+//             moments and the displacement, and writing the step's hi / lo
+//             planes for the next M update
 #include "kernels.cuh"
 #include "tc.cuh"
 
@@ -37,12 +39,14 @@ struct Maps {
     CUtensorMap a_hi, a_lo, b_hi, b_lo;
 };
 
-// p = acc + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead channels
+// M += acc; p = M + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead channels
 __device__ __forceinline__ float bgd_p_value(const TcEpi &e, int64_t i, int64_t j, float v) {
     const int64_t col = e.col0 + j;
     const int64_t w = i * e.ldw + col;
     const float w0 = e.w0_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16 *>(e.W0)[w])
                                : static_cast<const float *>(e.W0)[w];
+    v += e.M[w];
+    e.M[w] = v;
     float p = v + (*e.lam) * (e.Ad[w] - (e.W[w] - w0));
     if (e.R0) p += e.R0[w];
     if (e.dead && e.dead[col]) p = 0.f;
@@ -64,13 +68,14 @@ __device__ __forceinline__ float4 ld4_w0(const TcEpi &e, int64_t w) {
 // at the tile entry of row 0, column 0 of the 4x4 patch, pitch tp.
 __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, float *t, int tp) {
     const int64_t col = e.col0 + gj;
-    float4 a[4], w[4], w0[4], r0[4];
+    float4 a[4], w[4], w0[4], r0[4], mp[4];
     uchar4 dd = make_uchar4(0, 0, 0, 0);
     if (e.dead) dd = *reinterpret_cast<const uchar4 *>(e.dead + col);
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
         if (gi0 + u >= M) break;
         const int64_t wi = (gi0 + u) * e.ldw + col;
+        mp[u] = ld4(e.M + wi);
         a[u] = ld4(e.Ad + wi);
         w[u] = ld4(e.W + wi);
         w0[u] = ld4_w0(e, wi);
@@ -81,6 +86,9 @@ __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t
     for (int u = 0; u < 4; ++u) {
         if (gi0 + u >= M) break;
         float *tr = t + u * tp;
+        const float4 mn = make_float4(tr[0] + mp[u].x, tr[1] + mp[u].y, tr[2] + mp[u].z, tr[3] + mp[u].w);
+        st4(e.M + (gi0 + u) * e.ldw + col, mn);
+        tr[0] = mn.x; tr[1] = mn.y; tr[2] = mn.z; tr[3] = mn.w;
         tr[0] = dd.x ? 0.f : tr[0] + lam * (a[u].x - (w[u].x - w0[u].x)) + r0[u].x;
         tr[1] = dd.y ? 0.f : tr[1] + lam * (a[u].y - (w[u].y - w0[u].y)) + r0[u].y;
         tr[2] = dd.z ? 0.f : tr[2] + lam * (a[u].z - (w[u].z - w0[u].z)) + r0[u].z;
@@ -125,11 +133,11 @@ __device__ __forceinline__ void adam_rows4(const TcEpi &e, int64_t gi0, int64_t 
             st4(e.vA + wi, v[u]);
         }
         st4(e.Wm + wi, make_float4(w[u].x - st.x, w[u].y - st.y, w[u].z - st.z, w[u].w - st.w));
-        const float4 dn = make_float4(d[u].x - st.x, d[u].y - st.y, d[u].z - st.z, d[u].w - st.w);
-        st4(e.D + wi, dn);
-        const float4 dh = make_float4(tc::tf32_hi(dn.x), tc::tf32_hi(dn.y), tc::tf32_hi(dn.z), tc::tf32_hi(dn.w));
-        st4(e.Dh + wi, dh);
-        st4(e.Dl + wi, make_float4(dn.x - dh.x, dn.y - dh.y, dn.z - dh.z, dn.w - dh.w));
+        st4(e.D + wi, make_float4(d[u].x - st.x, d[u].y - st.y, d[u].z - st.z, d[u].w - st.w));
+        // the displacement moved by -st: its planes feed the next M update
+        const float4 sh = make_float4(tc::tf32_hi(-st.x), tc::tf32_hi(-st.y), tc::tf32_hi(-st.z), tc::tf32_hi(-st.w));
+        st4(e.Sh + wi, sh);
+        st4(e.Sl + wi, make_float4(-st.x - sh.x, -st.y - sh.y, -st.z - sh.z, -st.w - sh.w));
     }
 }
 
@@ -152,11 +160,10 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
         step = e.lr * (mv / e.bc1) / (sqrtf(vv / e.bc2) + e.eps);
     }
     e.Wm[w] -= step;
-    const float d = e.D[w] - step;
-    e.D[w] = d;
-    const float dh = tc::tf32_hi(d);
-    e.Dh[w] = dh;
-    e.Dl[w] = d - dh;
+    e.D[w] -= step;
+    const float sh = tc::tf32_hi(-step);
+    e.Sh[w] = sh;
+    e.Sl[w] = -step - sh;
 }
 
 __global__ void __launch_bounds__(128, 1)
@@ -217,7 +224,7 @@ __global__ void __launch_bounds__(128, 1)
             for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k)
                 tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (uint32_t)(k / STAGES) & 1u, &never, 100000000ull);
         }
-    } else if (warp == 1 && lane == 0) {
+    } else if (warp == 1 && lane == 0 && nk > 0) {
         // ---------------- MMA issuer ----------------
         for (int it = 0; it < nk; ++it) {
             const int s = it % STAGES;
@@ -248,9 +255,10 @@ __global__ void __launch_bounds__(128, 1)
     // The accumulator tile goes TMEM -> registers -> shared memory (the
     // pipeline buffers are free once the last MMA committed), so that global
     // reads and writes walk rows (or, for P^T, columns) with consecutive lanes.
-    const bool ok = tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
+    // (K = 0: nothing was issued and the accumulator is zero)
+    const bool ok = nk == 0 || tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
     tc::fence_after_sync();
-    const bool good = __syncthreads_and(ok && !*abort_flag) != 0 && nk > 0;
+    const bool good = __syncthreads_and(ok && !*abort_flag) != 0;
     constexpr int TP = TB + 1;
     float *T = reinterpret_cast<float *>(smem);
     if (good) {
@@ -258,7 +266,12 @@ __global__ void __launch_bounds__(128, 1)
 #pragma unroll 1
         for (int c0 = 0; c0 < TB; c0 += 32) {
             uint32_t v[32];
-            tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+            if (nk > 0) {
+                tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+            } else {
+#pragma unroll
+                for (int q = 0; q < 32; ++q) v[q] = 0u;
+            }
 #pragma unroll
             for (int q = 0; q < 32; ++q) T[row * TP + c0 + q] = __uint_as_float(v[q]);
         }
@@ -305,7 +318,7 @@ __global__ void __launch_bounds__(128, 1)
             }
         }
     }
-    if (!good && nk > 0 && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
+    if (!good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
     tc::fence_before_sync();
     __syncthreads();
     if (warp == 0) tc::tmem_dealloc(tmem, TB);

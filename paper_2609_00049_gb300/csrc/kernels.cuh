@@ -56,7 +56,8 @@ struct TcEpi {
     const float *Ad; const float *W; const void *W0; int w0_bf16;  // TC_BGD_P
     const uint8_t *dead; const float *lam; const float *R0; int64_t ldw; int64_t col0;
     float *Pth; float *Ptl; int64_t ldp;
-    float *Wm; float *mA; float *vA; float *D; float *Dh; float *Dl;  // TC_ADAM (ldw, col0 shared)
+    float *M;                                                // running A H̄ (acc += M, M = acc)
+    float *Wm; float *mA; float *vA; float *D; float *Sh; float *Sl;  // TC_ADAM (ldw, col0 shared)
     float lr, b1, b2, eps, bc1, bc2; int sgd;
 };
 struct TcMaps {
@@ -114,7 +115,9 @@ struct SweepPlan {
     float *Et, *P, *G, *Feff, *R0;
     // tensor-core path: hi / lo planes and tensor maps
     int tc;
-    float *Dh, *Dl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;
+    float *Sh, *Sl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;
+    float *M;        // M = A H̄, kept current for the free columns
+    int64_t step_c;  // first column of the last optimizer step not yet in M (n: none)
     TcMaps mapsP, mapsG;
     int f_split_alpha_valid;
     float f_split_alpha;
@@ -123,7 +126,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);
 realq_status_t sweep_init(cudaStream_t s, SweepPlan &p);
 realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b);
-realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p);
+realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh);
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha);
 realq_status_t surrogate(cudaStream_t s, int64_t m, int64_t n, const float *What, const void *W0,
                          realq_dtype_t w_dtype, const float *Hbar, const float *F, float *loss, void *ws);

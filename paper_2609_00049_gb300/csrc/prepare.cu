@@ -276,26 +276,34 @@ realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp,
 }
 
 // Auxiliary stream of the calling thread (and its events) for the U row
-// work, created on first use per device and kept for the life of the thread.
+// work, one per (device, priority of the caller's stream), created on first
+// use and kept for the life of the thread.
 struct AuxStream {
-    int device = -1;
+    int device = -1, priority = 0;
     cudaStream_t stream = nullptr;
     cudaEvent_t ev[2] = {nullptr, nullptr};
     std::vector<cudaEvent_t> steps;
 };
-static thread_local AuxStream g_aux;
+static thread_local std::vector<AuxStream> g_aux;
 
-realq_status_t aux_for(int64_t nsteps, AuxStream **out) {
-    int dev = 0;
+realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
+    int dev = 0, prio = 0;
     REALQ_CUDA_TRY(cudaGetDevice(&dev));
-    AuxStream &a = g_aux;
-    if (a.device != dev) {
-        a = AuxStream{};
-        REALQ_CUDA_TRY(cudaStreamCreateWithFlags(&a.stream, cudaStreamNonBlocking));
+    REALQ_CUDA_TRY(cudaStreamGetPriority(s, &prio));
+    AuxStream *found = nullptr;
+    for (AuxStream &x : g_aux)
+        if (x.device == dev && x.priority == prio) found = &x;
+    if (!found) {
+        AuxStream a;
+        REALQ_CUDA_TRY(cudaStreamCreateWithPriority(&a.stream, cudaStreamNonBlocking, prio));
         REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[0], cudaEventDisableTiming));
         REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[1], cudaEventDisableTiming));
         a.device = dev;
+        a.priority = prio;
+        g_aux.push_back(a);
+        found = &g_aux.back();
     }
+    AuxStream &a = *found;
     while ((int64_t)a.steps.size() < nsteps) {
         cudaEvent_t e;
         REALQ_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
@@ -342,7 +350,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, co
     // < k0 only: with overlap, the U row work runs on an auxiliary stream that
     // starts after the diagonal step of K (which wrote U_KK into A[K, K]).
     AuxStream *aux = nullptr;
-    if (overlap && nbk > 1) REALQ_TRY(aux_for(nbk, &aux));
+    if (overlap && nbk > 1) REALQ_TRY(aux_for(s, nbk, &aux));
     cudaStream_t rs = aux ? aux->stream : s;
     if (aux) {
         REALQ_CUDA_TRY(cudaEventRecord(aux->ev[0], s));

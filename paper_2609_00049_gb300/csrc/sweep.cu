@@ -386,7 +386,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
     if (has_bgd) {
         if (block > 0 && tc_gemm_eligible(m, n)) {
-            b += 4 * mn + 2 * align_up((size_t)n * n * sizeof(float)) + 2 * align_up((size_t)m * m * sizeof(float));
+            b += 5 * mn + 2 * align_up((size_t)n * n * sizeof(float)) + 2 * align_up((size_t)m * m * sizeof(float));
         } else {
             b += 2 * mn;
             if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
@@ -403,13 +403,15 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
     p.lam = cv.take<float>(1);
     p.Et = cv.take<float>((size_t)p.block * p.m);
     p.P = p.G = p.Feff = p.R0 = nullptr;
-    p.Dh = p.Dl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = nullptr;
+    p.Sh = p.Sl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = p.M = nullptr;
+    p.step_c = p.n;
     p.tc = 0;
     if (has_bgd) {
         if (p.block > 0 && tc_gemm_eligible(p.m, p.n)) {
             p.tc = 1;
-            p.Dh = cv.take<float>(mn);
-            p.Dl = cv.take<float>(mn);
+            p.Sh = cv.take<float>(mn);
+            p.Sl = cv.take<float>(mn);
+            p.M = cv.take<float>(mn);
             p.Pth = cv.take<float>(mn);
             p.Ptl = cv.take<float>(mn);
             p.Hh = cv.take<float>((size_t)p.n * p.n);
@@ -520,25 +522,31 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
 // One Block-GD step on columns c0..n-1 on the tensor cores (identity form):
 // P^T planes from the displacement planes and H̄ planes, then G = F_eff P with
 // the optimizer step fused into the epilogue.
+// One optimizer step on the free columns [c0, n).  The first product brings
+// M = A H̄ up to date for them: the last step moved A only in its own free
+// columns [step_c, n), so M[:, c0:] += step[:, step_c:] H̄[step_c:, c0:]
+// (K = n - step_c instead of n), then the epilogue forms P from M.
 static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
     const int64_t r = p.n - c0;
-    const int64_t k0 = std::min<int64_t>(p.block, c0);   // displacement columns < B are zero
+    const int64_t k0 = p.step_c;
     TcEpi e{};
     e.mode = TC_BGD_P;
     e.Ad = p.disp; e.W = p.W; e.W0 = p.W0; e.w0_bf16 = p.w_dtype == REALQ_BF16;
     e.dead = p.dead; e.lam = p.lam; e.R0 = p.R0; e.ldw = p.n; e.col0 = c0;
-    e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m;
+    e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m; e.M = p.M;
     REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
     const int64_t t = ++(*p.adam_t);
     TcEpi g{};
     g.mode = TC_ADAM;
     g.ldw = p.n; g.col0 = c0;
-    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Dh = p.Dh; g.Dl = p.Dl;
+    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
     g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
     g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
     g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
     g.sgd = p.optimizer == REALQ_OPT_SGD;
-    return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    p.step_c = c0;
+    return REALQ_OK;
 }
 
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
@@ -613,7 +621,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     return REALQ_OK;
 }
 
-realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p) {
+realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
     if (p.bgd_steps <= 0) return REALQ_OK;
     {
         Launch L("bgd_lambda", s);
@@ -622,13 +630,23 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p) {
     REALQ_TRY(check_launch("bgd_lambda"));
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
     if (p.tc) {
-        // planes of H̄ and of the caller's displacement (so a resumed sweep needs
-        // nothing from an earlier workspace), and the tensor maps of both GEMMs
+        // planes of H̄ and the tensor maps of both GEMMs; M = A H̄ from the
+        // caller's displacement (zero on a fresh sweep; a resumed sweep takes
+        // nothing from an earlier workspace)
         REALQ_TRY(tc_split(s, p.n * p.n, p.Hbar, nullptr, 1.f, p.Hh, p.Hl));
-        REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Dh, p.Dl));
-        REALQ_TRY(tc_make_maps(&p.mapsP, p.Dh, p.Dl, p.m, p.n, p.n, p.Hh, p.Hl, p.n, p.n, p.n));
+        REALQ_TRY(tc_make_maps(&p.mapsP, p.Sh, p.Sl, p.m, p.n, p.n, p.Hh, p.Hl, p.n, p.n, p.n));
         REALQ_TRY(tc_make_maps(&p.mapsG, p.Fh, p.Fl, p.m, p.m, p.m, p.Pth, p.Ptl, p.n, p.m, p.m));
         p.f_split_alpha_valid = 0;
+        p.step_c = p.n;
+        if (fresh) {
+            REALQ_CUDA_TRY(cudaMemsetAsync(p.M, 0, (size_t)p.m * p.n * sizeof(float), s));
+        } else {
+            REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Sh, p.Sl));
+            TcEpi e{};
+            e.mode = TC_STORE;
+            e.C = p.M; e.ldc = p.n;
+            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm"));
+        }
     }
     return REALQ_OK;
 }
