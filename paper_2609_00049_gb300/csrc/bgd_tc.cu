@@ -12,7 +12,9 @@
 // 128 x 128 tile: TMA loads 32-wide K slices of the four planes (128-byte
 // rows, 128-byte swizzle) into a 3-stage ring, one thread issues
 // 3 x 4 tcgen05.mma (kind::tf32, K = 8) per stage into a TMEM accumulator,
-// and four warps drain it through one of the epilogues:
+// and eight warps drain it through one of the epilogues (the epilogues are
+// bound by the latency of their global loads, so every warp of the CTA
+// takes part):
 //   TC_STORE  C = acc
 //   TC_BGD_P  the Block-GD gradient factor after the lazy OBS update: the
 //             running product M = A_disp H̄ takes the latest step (acc),
@@ -30,6 +32,7 @@ namespace {
 constexpr int TB = 128;                       // tile rows (M) and columns (N)
 constexpr int KS = 32;                        // fp32 elements per K slice (128 bytes)
 constexpr int STAGES = 3;
+constexpr int THREADS = 256;                  // 8 warps; warp 0 lane 0 loads, warp 1 lane 0 issues MMAs
 constexpr int PLANE = TB * KS * 4;            // 16 KB
 constexpr int STAGE_BYTES = 4 * PLANE;        // A hi, A lo, B hi, B lo
 constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
@@ -64,8 +67,9 @@ __device__ __forceinline__ float4 ld4_w0(const TcEpi &e, int64_t w) {
     return ld4(static_cast<const float *>(e.W0) + w);
 }
 
-// Gradient factor for 4 rows x 4 columns (columns gj..gj+3 all < N); t points
-// at the tile entry of row 0, column 0 of the 4x4 patch, pitch tp.
+// Gradient factor for 4 rows x 4 columns (rows gi0..gi0+3 all < M, as M is a
+// multiple of 4; columns gj..gj+3 all < N); t points at the tile entry of row
+// 0, column 0 of the 4x4 patch, pitch tp.  All loads are issued first.
 __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, float *t, int tp) {
     const int64_t col = e.col0 + gj;
     float4 a[4], w[4], w0[4], r0[4], mp[4];
@@ -73,7 +77,6 @@ __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t
     if (e.dead) dd = *reinterpret_cast<const uchar4 *>(e.dead + col);
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-        if (gi0 + u >= M) break;
         const int64_t wi = (gi0 + u) * e.ldw + col;
         mp[u] = ld4(e.M + wi);
         a[u] = ld4(e.Ad + wi);
@@ -84,7 +87,6 @@ __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t
     const float lam = *e.lam;
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-        if (gi0 + u >= M) break;
         float *tr = t + u * tp;
         const float4 mn = make_float4(tr[0] + mp[u].x, tr[1] + mp[u].y, tr[2] + mp[u].z, tr[3] + mp[u].w);
         st4(e.M + (gi0 + u) * e.ldw + col, mn);
@@ -103,13 +105,12 @@ __device__ __forceinline__ float adam_step(const TcEpi &e, float g, float &m, fl
     return e.lr * (m / e.bc1) / (sqrtf(v / e.bc2) + e.eps);
 }
 
-// Optimizer step for 4 rows x 4 columns of the free block.
+// Optimizer step for 4 rows x 4 columns of the free block (same shape rules).
 __device__ __forceinline__ void adam_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, const float *t, int tp) {
     const int64_t col = e.col0 + gj;
     float4 m[4], v[4], w[4], d[4];
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-        if (gi0 + u >= M) break;
         const int64_t wi = (gi0 + u) * e.ldw + col;
         if (!e.sgd) {
             m[u] = ld4(e.mA + wi);
@@ -120,7 +121,6 @@ __device__ __forceinline__ void adam_rows4(const TcEpi &e, int64_t gi0, int64_t 
     }
 #pragma unroll
     for (int u = 0; u < 4; ++u) {
-        if (gi0 + u >= M) break;
         const int64_t wi = (gi0 + u) * e.ldw + col;
         const float *tr = t + u * tp;
         float4 st;
@@ -166,7 +166,7 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
     e.Sl[w] = -step - sh;
 }
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
                        const TcEpi e, int *err) {
     extern __shared__ uint8_t smem_raw[];
@@ -262,12 +262,15 @@ __global__ void __launch_bounds__(128, 1)
     constexpr int TP = TB + 1;
     float *T = reinterpret_cast<float *>(smem);
     if (good) {
-        const int row = warp * 32 + lane;
+        // warp w reads TMEM lanes 32 (w % 4) .. (its lane quarter), columns
+        // 64 (w / 4) ..
+        const int quarter = warp & 3, half = warp >> 2;
+        const int row = quarter * 32 + lane;
 #pragma unroll 1
-        for (int c0 = 0; c0 < TB; c0 += 32) {
+        for (int c0 = half * (TB / 2); c0 < (half + 1) * (TB / 2); c0 += 32) {
             uint32_t v[32];
             if (nk > 0) {
-                tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+                tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
             } else {
 #pragma unroll
                 for (int q = 0; q < 32; ++q) v[q] = 0u;
@@ -280,11 +283,13 @@ __global__ void __launch_bounds__(128, 1)
     if (good) {
         // rows of the tile, each lane on 4 consecutive columns; the loads of
         // 4 rows are issued before any store so they overlap
+        constexpr int RPW = TB / (THREADS / 32);   // tile rows per warp
         const int cc = lane * 4;
         const int64_t gj = j0 + cc;
         const bool vec = e.mode != TC_STORE && gj + 3 < N;
-        for (int rb = warp * 32; rb < warp * 32 + 32; rb += 4) {
+        for (int rb = warp * RPW; rb < warp * RPW + RPW; rb += 4) {
             if (vec) {
+                if (i0 + rb >= M) break;
                 if (e.mode == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
                 else bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
             } else {
@@ -305,7 +310,8 @@ __global__ void __launch_bounds__(128, 1)
     __syncthreads();
     if (good && e.mode == TC_BGD_P) {
         // columns of the tile, lanes over rows: P^T rows are contiguous
-        for (int cc = warp * 32; cc < warp * 32 + 32; ++cc) {
+        constexpr int CPW = TB / (THREADS / 32);   // tile columns per warp
+        for (int cc = warp * CPW; cc < warp * CPW + CPW; ++cc) {
             const int64_t gj = j0 + cc;
             if (gj >= N) break;
             for (int rr = lane; rr < TB; rr += 32) {
@@ -378,7 +384,7 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
     {
         Launch L(name, s);
-        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB)), 128, SMEM, s>>>(
+        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB)), THREADS, SMEM, s>>>(
             m, M, N, K, k_off, b_row0, e, err);
     }
     return check_launch(name);
