@@ -54,134 +54,158 @@ __global__ void prep_damp_kernel(int64_t n, float *A, float damp, float *lam_out
     if (threadIdx.x == 0) *lam_out = lam;
 }
 
-// The 64 x 64 diagonal-block kernels below use 256 threads as a 16 x 16 grid;
-// thread (ty, tx) keeps the 4 x 4 block rows 4ty.., columns 4tx.. in
-// registers, and only the pivot and the pivot column / row travel through
-// double-buffered shared memory.
-
-// V = R^-1 for the kb x kb upper triangle in Rs, by row operations on the
-// identity (back substitution applied to all columns at once); v is this
-// thread's 4 x 4 block of V.  One barrier per pivot.
-__device__ __forceinline__ void upper_inverse_regs(const float (*Rs)[NB + 1], int kb, float (&v)[4][4],
-                                                   float (*rowk)[NB]) {
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
+// One warp, a 32 x 32 block As (pitch 33, upper triangle): reverse-order
+// Cholesky As = R R^T (R upper) fused with the back substitution V = R^-1,
+// written to Vs (row-major, zeros below the diagonal).  Lane j keeps column j
+// of the block and row j of V in registers.  Pivot k needs only column k of R
+// and row k of V: lane k publishes both (unscaled) through a double-buffered
+// 64-float slot bf[(k & 1) * 64 ..] in shared memory, every lane reads them
+// back with 16-byte broadcast loads and applies
+//   a_ij -= r_ik r_jk (i <= j < k),   V[j] -= r_jk V[k] (j < k),
+// with r_ik = a_ik / sqrt(a_kk).  Row k of V is scaled by its own 1 / r_kk
+// once, at the end (no later pivot reads it).  A pivot that is not positive
+// (or not finite) is recorded (the first one wins; columns >= valid are
+// padding) and replaced by 1 to keep going.  Single-warp code issues slowly,
+// so the pivot step avoids shuffles and keeps to ~100 instructions.
+__device__ __forceinline__ void warp_rchol_inv32(const float (*As)[33], float (*Vs)[33], float *bf, int lane,
+                                                 int *status, int64_t col0, int valid) {
+    float c[32], v[32];
 #pragma unroll
-    for (int a = 0; a < 4; ++a)
+    for (int i = 0; i < 32; ++i) {
+        c[i] = As[i][lane];
+        v[i] = (i == lane) ? 1.f : 0.f;
+    }
+    float rown = 1.f;
+#pragma unroll 1
+    for (int k = 31; k >= 0; --k) {
+        float *b = bf + (k & 1) * 64;
+        if (lane == k) {
 #pragma unroll
-        for (int b = 0; b < 4; ++b) v[a][b] = (ty * 4 + a == tx * 4 + b && ty * 4 + a < kb) ? 1.f : 0.f;
-    for (int k = kb - 1; k >= 0; --k) {
-        const int kt = k >> 2, kq = k & 3, p = k & 1;
-        if (ty == kt) {
-            const float rinv = 1.f / Rs[k][k];
-#pragma unroll
-            for (int a = 0; a < 4; ++a)
-                if (a == kq) {
-#pragma unroll
-                    for (int b = 0; b < 4; ++b) {
-                        v[a][b] = v[a][b] * rinv;
-                        rowk[p][tx * 4 + b] = v[a][b];
-                    }
-                }
+            for (int q = 0; q < 32; q += 4) {
+                *reinterpret_cast<float4 *>(b + q) = make_float4(c[q], c[q + 1], c[q + 2], c[q + 3]);
+                *reinterpret_cast<float4 *>(b + 32 + q) = make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]);
+            }
         }
-        __syncthreads();
-        float rv[4];
+        __syncwarp();
+        float d = b[k];
+        if (!(d > 0.f) || !isfinite(d)) {
+            if (lane == 0 && k < valid) atomicCAS(status, -1, (int)(col0 + k));
+            d = 1.f;
+        }
+        const float rinv = rsqrtf(d);
+        if (lane == k) rown = rinv;
+        const float rjk = lane < k ? b[lane] * rinv : 0.f;   // r_jk on lanes j < k
+        const float cf = -rjk * rinv;                          // r_ik = b[i] rinv
 #pragma unroll
-        for (int b = 0; b < 4; ++b) rv[b] = rowk[p][tx * 4 + b];
+        for (int q = 0; q < 32; q += 4) {
+            const float4 bc = *reinterpret_cast<const float4 *>(b + q);
+            const float4 bv = *reinterpret_cast<const float4 *>(b + 32 + q);
+            if (q + 0 <= lane) c[q + 0] = fmaf(bc.x, cf, c[q + 0]);
+            if (q + 1 <= lane) c[q + 1] = fmaf(bc.y, cf, c[q + 1]);
+            if (q + 2 <= lane) c[q + 2] = fmaf(bc.z, cf, c[q + 2]);
+            if (q + 3 <= lane) c[q + 3] = fmaf(bc.w, cf, c[q + 3]);
+            v[q + 0] = fmaf(bv.x, cf, v[q + 0]);
+            v[q + 1] = fmaf(bv.y, cf, v[q + 1]);
+            v[q + 2] = fmaf(bv.z, cf, v[q + 2]);
+            v[q + 3] = fmaf(bv.w, cf, v[q + 3]);
+        }
+    }
 #pragma unroll
-        for (int a = 0; a < 4; ++a) {
-            const int i = ty * 4 + a;
-            if (i < k) {
-                const float rik = Rs[i][k];
+    for (int q = 0; q < 32; ++q) Vs[lane][q] = v[q] * rown;
+}
+
+// Diagonal block [k0, k0 + kb) of the reverse-order blocked Cholesky, 128
+// threads.  With the block split 2 x 2 into 32 x 32 pieces,
+//   A22 = R22 R22^T,  R12 = A12 R22^-T,  A11 - R12 R12^T = R11 R11^T,
+//   V = R^-1 = [[V11, -V11 R12 V22], [0, V22]].
+// Warp 0 factors and inverts the two diagonal pieces, all four warps form the
+// 32 x 32 products (warps 1-3 form R12 V22 while warp 0 works on the second
+// piece).  Out: U_KK = V into A[K, K] (upper, in place of the block) and
+// Vt = V^T (dense 64 x 64, row-major) for the panel solve.  Rows / columns
+// >= kb are padded with the identity.
+__global__ void __launch_bounds__(128) chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status,
+                                                        float *Vt) {
+    __shared__ float S11[32][33], S22[32][33], A12[32][33];
+    __shared__ float V11[32][33], V22[32][33], V12[32][33];
+    __shared__ float R12[32][33], X[32][33];   // X = R12 V22
+    __shared__ __align__(16) float bf[128];     // pivot broadcast slots
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    {
+        // all loads of a thread are issued before the first use
+        float x[NB * NB / 128];
 #pragma unroll
-                for (int b = 0; b < 4; ++b) v[a][b] -= rik * rv[b];
+        for (int t = 0; t < NB * NB / 128; ++t) {
+            const int e = tid + t * 128, i = e >> 6, j = e & 63;
+            x[t] = (i < kb && j < kb && j >= i) ? A[(k0 + i) * n + k0 + j] : 0.f;
+        }
+#pragma unroll
+        for (int t = 0; t < NB * NB / 128; ++t) {
+            const int e = tid + t * 128, i = e >> 6, j = e & 63;
+            const float v = (i == j && i >= kb) ? 1.f : x[t];
+            if (i < 32) {
+                if (j < 32) S11[i][j] = v;
+                else A12[i][j - 32] = v;
+            } else if (j >= 32) {
+                S22[i - 32][j - 32] = v;
             }
         }
     }
-}
-
-// Diagonal block [k0, k0 + kb): A_KK = R_KK R_KK^T with R_KK upper (in place),
-// and Vt = (R_KK^-1)^T (dense 64 x 64, row-major) for the panel solve.
-// Two barriers per Cholesky pivot, one per inverse pivot.
-__global__ void __launch_bounds__(256) chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status,
-                                                        float *Vt) {
-    __shared__ float Rs[NB][NB + 1];
-    __shared__ float colk[2][NB];
-    __shared__ float rk_s[2];
-    const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
-    float sv[4][4];
-#pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int r = ty * 4 + a, c = tx * 4 + b;
-            sv[a][b] = (r < kb && c < kb && c >= r) ? A[(k0 + r) * n + k0 + c] : 0.f;
-        }
-    for (int k = kb - 1; k >= 0; --k) {
-        const int kt = k >> 2, kq = k & 3, p = k & 1;
-        if (ty == kt && tx == kt) {
-#pragma unroll
-            for (int a = 0; a < 4; ++a)
-                if (a == kq) {
-                    float d = sv[a][a];
-                    const bool bad = !(d > 0.f) || !isfinite(d);
-                    if (bad) {
-                        atomicCAS(status, -1, (int)(k0 + k));
-                        d = 1.f;
-                    }
-                    const float rk = sqrtf(d);
-                    sv[a][a] = rk;
-                    rk_s[p] = rk;
-                }
-        }
-        __syncthreads();
-        if (tx == kt) {
-            const float rinv = 1.f / rk_s[p];
-#pragma unroll
-            for (int b = 0; b < 4; ++b)
-                if (b == kq) {
-#pragma unroll
-                    for (int a = 0; a < 4; ++a) {
-                        const int i = ty * 4 + a;
-                        if (i < k) {
-                            sv[a][b] = sv[a][b] * rinv;
-                            colk[p][i] = sv[a][b];
-                        }
-                    }
-                }
-        }
-        __syncthreads();
-        if (ty * 4 < k && tx * 4 < k) {
-            float ci[4], cj[4];
-#pragma unroll
-            for (int a = 0; a < 4; ++a) ci[a] = colk[p][ty * 4 + a];
-#pragma unroll
-            for (int b = 0; b < 4; ++b) cj[b] = colk[p][tx * 4 + b];
-#pragma unroll
-            for (int a = 0; a < 4; ++a)
-#pragma unroll
-                for (int b = 0; b < 4; ++b) {
-                    const int i = ty * 4 + a, j = tx * 4 + b;
-                    if (i <= j && j < k) sv[a][b] -= ci[a] * cj[b];
-                }
+    __syncthreads();
+    if (warp == 0) warp_rchol_inv32(S22, V22, bf, lane, status, k0 + 32, kb - 32);
+    __syncthreads();
+    // R12[i][j] = sum_l A12[i][l] V22[j][l]   (V22 upper, zeros below)
+#pragma unroll 1
+    for (int e = tid; e < 32 * 32; e += 128) {
+        const int i = e >> 5, j = e & 31;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int l = 0; l < 32; ++l) acc = fmaf(A12[i][l], V22[j][l], acc);
+        R12[i][j] = acc;
+    }
+    __syncthreads();
+    // A11 -= R12 R12^T
+#pragma unroll 1
+    for (int e = tid; e < 32 * 32; e += 128) {
+        const int i = e >> 5, j = e & 31;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int l = 0; l < 32; ++l) acc = fmaf(R12[i][l], R12[j][l], acc);
+        S11[i][j] -= acc;
+    }
+    __syncthreads();
+    if (warp == 0) {
+        warp_rchol_inv32(S11, V11, bf, lane, status, k0, kb);
+    } else {
+        // X = R12 V22
+#pragma unroll 1
+        for (int e = tid - 32; e < 32 * 32; e += 96) {
+            const int i = e >> 5, j = e & 31;
+            float acc = 0.f;
+#pragma unroll 8
+            for (int l = 0; l < 32; ++l) acc = fmaf(R12[i][l], V22[l][j], acc);
+            X[i][j] = acc;
         }
     }
-#pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) Rs[ty * 4 + a][tx * 4 + b] = sv[a][b];
     __syncthreads();
-    __shared__ float rowk[2][NB];
-    float v[4][4];
-    upper_inverse_regs(Rs, kb, v, rowk);
-    // U_KK = R_KK^-1 goes to A[K, K]; Vt = U_KK^T feeds the panel solve
-#pragma unroll
-    for (int a = 0; a < 4; ++a)
-#pragma unroll
-        for (int b = 0; b < 4; ++b) {
-            const int r = ty * 4 + a, c = tx * 4 + b;
-            if (r < kb && c < kb && c >= r) A[(k0 + r) * n + k0 + c] = v[a][b];
-            Vt[c * NB + r] = v[a][b];
-        }
+    // V12 = -V11 X   (V11 upper, zeros below)
+#pragma unroll 1
+    for (int e = tid; e < 32 * 32; e += 128) {
+        const int i = e >> 5, j = e & 31;
+        float acc = 0.f;
+#pragma unroll 8
+        for (int l = 0; l < 32; ++l) acc = fmaf(V11[i][l], X[l][j], acc);
+        V12[i][j] = -acc;
+    }
+    __syncthreads();
+#pragma unroll 4
+    for (int e = tid; e < NB * NB; e += 128) {
+        const int r = e >> 6, c = e & 63;
+        float x;
+        if (r < 32) x = c < 32 ? V11[r][c] : V12[r][c - 32];
+        else x = c < 32 ? 0.f : V22[r - 32][c - 32];
+        if (r < kb && c < kb && c >= r) A[(k0 + r) * n + k0 + c] = x;
+        Vt[c * NB + r] = x;
+    }
 }
 
 // A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles).
@@ -194,10 +218,22 @@ __global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, i
     while ((int64_t)r * (r + 1) / 2 > idx) --r;
     const int tj = r, ti = (int)(idx - (int64_t)r * (r + 1) / 2);  // ti <= tj
     const int64_t i0 = (int64_t)ti * NB, j0 = (int64_t)tj * NB;
-    for (int e = threadIdx.x; e < NB * NB; e += blockDim.x) {
-        const int rr = e / NB, c = e % NB;
-        Pi[c][rr] = (c < kb && i0 + rr < k0) ? A[(i0 + rr) * n + k0 + c] : 0.f;
-        Pj[c][rr] = (c < kb && j0 + rr < k0) ? A[(j0 + rr) * n + k0 + c] : 0.f;
+    {
+        // all loads of a thread are issued before the first use
+        constexpr int PER = NB * NB / 256;
+        float xi[PER], xj[PER];
+#pragma unroll
+        for (int t = 0; t < PER; ++t) {
+            const int e = threadIdx.x + t * 256, rr = e / NB, c = e % NB;
+            xi[t] = (c < kb && i0 + rr < k0) ? A[(i0 + rr) * n + k0 + c] : 0.f;
+            xj[t] = (c < kb && j0 + rr < k0) ? A[(j0 + rr) * n + k0 + c] : 0.f;
+        }
+#pragma unroll
+        for (int t = 0; t < PER; ++t) {
+            const int e = threadIdx.x + t * 256, rr = e / NB, c = e % NB;
+            Pi[c][rr] = xi[t];
+            Pj[c][rr] = xj[t];
+        }
     }
     __syncthreads();
     const int tx = threadIdx.x & 15, ty = threadIdx.x >> 4;
@@ -362,7 +398,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, co
         const int64_t k1 = k0 + kb;
         {
             Launch L("chol_diag", s);
-            chol_diag_kernel<<<1, 256, 0, s>>>(n, U, k0, kb, status, Vd);
+            chol_diag_kernel<<<1, 128, 0, s>>>(n, U, k0, kb, status, Vd);
         }
         REALQ_TRY(check_launch("chol_diag"));
         if (aux && k1 < n) {
