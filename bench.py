@@ -109,6 +109,7 @@ def gpu_arm(args, wl, rank, world):
     import torch
     import paper_2609_00049_gb300 as rq
     from paper_2609_00049_gb300 import build as rqbuild
+    from paper_2609_00049_gb300.block import BlockInput, BlockModule, BlockQuantizer
 
     rqbuild.build()
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
@@ -144,164 +145,29 @@ def gpu_arm(args, wl, rank, world):
     t_gen = time.time() - t_gen
 
     qcfg = rq.quant_cfg(wl.bits, wl.group_size, wl.block_size, wl.symmetric, wl.damp_frac)
-    B_total = wl.total_column_blocks
-    # ---- state buffers (allocated once)
-    st = {}
-    for name, spec in wl.inputs.items():
-        n = spec.n
-        st[name] = dict(H=torch.empty(n, n, device=dev), U=torch.empty(n, n, device=dev),
-                        Hbar=torch.empty(n, n, device=dev), dead=torch.empty(n, dtype=torch.uint8, device=dev),
-                        pws=rq.workspace(rq.realq_prepare_workspace_size(n), dev),
-                        hws=rq.workspace(rq.realq_hessian_workspace_size(n, spec.T), dev))
-    mods, bstart = {}, 1
-    for mod in wl.modules:
-        m, n = mod.m, mod.n
-        g = wl.group_size or n
-        ng = -(-n // g)
-        nb = -(-n // wl.block_size)
-        bc = rq.bgd_cfg(wl.lr, wl.steps_per_block, b_global_start=bstart, B_total=B_total if wl.sliding_window else 1)
-        bstart += nb
-        mods[mod.name] = dict(
-            W=torch.empty(m, n, device=dev), codes=torch.empty(m, (n + 1) // 2, dtype=torch.uint8, device=dev),
-            scale=torch.empty(m, ng, device=dev), zero=torch.empty(m, ng, dtype=torch.uint8, device=dev),
-            am=torch.empty(m, n, device=dev), av=torch.empty(m, n, device=dev), disp=torch.empty(m, n, device=dev),
-            bcfg=bc,
-            ws=rq.workspace(rq.realq_quantize_workspace_size(m, n, qcfg, bc, False, False), dev))
-    # e2e-only buffers: pinned host outputs, device staging for chunked inputs
-    E2E_CHUNK = 32768
-    stage = {}
-    for name, spec in wl.inputs.items():
-        stage[name] = [torch.empty(E2E_CHUNK, spec.n, dtype=torch.bfloat16, device=dev) for _ in range(2)]
-    host_out = {mod.name: dict(codes=torch.empty_like(mods[mod.name]["codes"], device="cpu").pin_memory(),
-                               scale=torch.empty_like(mods[mod.name]["scale"], device="cpu").pin_memory(),
-                               zero=torch.empty_like(mods[mod.name]["zero"], device="cpu").pin_memory())
-                for mod in wl.modules}
-    copy_stream = torch.cuda.Stream(device=dev)
-
-    # Concurrency: the block's inputs are independent, and so are its modules
-    # once their input is prepared.  One host thread per input drives its own
-    # stream (accumulate -> prepare, which synchronizes that stream only), then
-    # issues each of its modules on a stream of its own.
-    from concurrent.futures import ThreadPoolExecutor
-    in_streams = {name: torch.cuda.Stream(device=dev) for name in wl.inputs}
-    mod_streams = {mod.name: torch.cuda.Stream(device=dev) for mod in wl.modules}
-    pool = ThreadPoolExecutor(len(wl.inputs))
-    mods_of = {name: [md for md in wl.modules if md.input == name] for name in wl.inputs}
-
-    def input_pipeline(name, start_ev, wsrc, fsrc):
-        torch.cuda.set_device(dev)
-        spec = wl.inputs[name]
-        s_in = st[name]
-        si = in_streams[name]
-        si.wait_event(start_ev)
-        with torch.cuda.stream(si):
-            s_in["H"].zero_()
-        rq.realq_hessian_accumulate(dev_x[name], s_in["H"], ws=s_in["hws"], stream=si)
-        rq.realq_hessian_prepare(s_in["H"], spec.T, wl.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                                 s_in["pws"], stream=si)
-        for mod in mods_of[name]:
-            p, sm = mods[mod.name], mod_streams[mod.name]
-            rq.realq_quantize_layer(wsrc[mod.name], s_in["U"], s_in["Hbar"], qcfg, p["W"], p["codes"],
-                                    p["scale"], p["zero"], dead=s_in["dead"], bcfg=p["bcfg"], F=fsrc[mod.name],
-                                    adam_m=p["am"], adam_v=p["av"], bgd_disp=p["disp"], ws=p["ws"], stream=sm)
-
-    def run_block(wsrc, fsrc):
-        start = torch.cuda.Event()
-        start.record(stream)
-        futs = [pool.submit(input_pipeline, name, start, wsrc, fsrc) for name in wl.inputs]
-        for f in futs:
-            f.result()
-        for mod in wl.modules:
-            stream.wait_stream(mod_streams[mod.name])
-        for name in wl.inputs:
-            stream.wait_stream(in_streams[name])
+    dev_fn = None
+    if wl.sliding_window:
+        dev_fn = {mod.name: torch.from_numpy(synth.fisher(wl, mod, "F_next")).to(dev) for mod in wl.modules}
+    # the block's modules, scheduled concurrently by the library's block scheduler
+    bq = BlockQuantizer([BlockInput(nm, sp.n, sp.T) for nm, sp in wl.inputs.items()],
+                        [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
+                        wl.steps_per_block, sliding_window=wl.sliding_window, device=dev)
+    host_out = {mod.name: {k: torch.empty_like(bq.out[mod.name][k], device="cpu").pin_memory()
+                           for k in ("codes", "scale", "zero")} for mod in wl.modules}
+    e2e_bytes = {"h2d": 0, "d2h": 0}
 
     def step_device():
-        run_block(dev_w, dev_f)
-        for mod in wl.modules:
-            rq.realq_workspace_status(mods[mod.name]["ws"])
+        bq.run(dev_x, dev_w, dev_f, dev_fn)
+        bq.check_status()
 
     def step_serial():
-        for name, spec in wl.inputs.items():
-            s_in = st[name]
-            s_in["H"].zero_()
-            rq.realq_hessian_accumulate(dev_x[name], s_in["H"], ws=s_in["hws"])
-            rq.realq_hessian_prepare(s_in["H"], spec.T, wl.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                                     s_in["pws"])
-            for mod in mods_of[name]:
-                p = mods[mod.name]
-                rq.realq_quantize_layer(dev_w[mod.name], s_in["U"], s_in["Hbar"], qcfg, p["W"], p["codes"],
-                                        p["scale"], p["zero"], dead=s_in["dead"], bcfg=p["bcfg"], F=dev_f[mod.name],
-                                        adam_m=p["am"], adam_v=p["av"], bgd_disp=p["disp"], ws=p["ws"])
-
-    e2e_bytes = {"h2d": 0, "d2h": 0}
-    dev_w_e2e = {k: torch.empty_like(v) for k, v in dev_w.items()}
-    dev_f_e2e = {k: torch.empty_like(v) for k, v in dev_f.items()}
-    e2e_ws = {name: rq.workspace(rq.realq_hessian_workspace_size(spec.n, E2E_CHUNK), dev)
-              for name, spec in wl.inputs.items()}
-
-    copy_streams = {name: torch.cuda.Stream(device=dev) for name in wl.inputs}
-
-    def input_pipeline_e2e(name, start_ev, counts):
-        torch.cuda.set_device(dev)
-        spec = wl.inputs[name]
-        s_in = st[name]
-        si, cs = in_streams[name], copy_streams[name]
-        si.wait_event(start_ev)
-        cs.wait_event(start_ev)
-        with torch.cuda.stream(si):
-            s_in["H"].zero_()
-        xs = host_x[name]
-        nch = -(-spec.T // E2E_CHUNK)
-        used = [None, None]
-        h2d = 0
-        for c in range(nch):
-            buf = stage[name][c % 2]
-            rows = min(E2E_CHUNK, spec.T - c * E2E_CHUNK)
-            if used[c % 2] is not None:
-                cs.wait_event(used[c % 2])
-            with torch.cuda.stream(cs):
-                buf[:rows].copy_(xs[c * E2E_CHUNK:c * E2E_CHUNK + rows], non_blocking=True)
-            done = torch.cuda.Event()
-            done.record(cs)
-            si.wait_event(done)
-            rq.realq_hessian_accumulate(buf[:rows], s_in["H"], ws=e2e_ws[name], stream=si)
-            ev = torch.cuda.Event()
-            ev.record(si)
-            used[c % 2] = ev
-            h2d += rows * spec.n * 2
-        rq.realq_hessian_prepare(s_in["H"], spec.T, wl.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                                 s_in["pws"], stream=si)
-        d2h = 0
-        for mod in mods_of[name]:
-            p, sm, o = mods[mod.name], mod_streams[mod.name], host_out[mod.name]
-            with torch.cuda.stream(sm):
-                dev_w_e2e[mod.name].copy_(host_w[mod.name], non_blocking=True)
-                dev_f_e2e[mod.name].copy_(host_f[mod.name], non_blocking=True)
-            h2d += host_w[mod.name].numel() * 2 + host_f[mod.name].numel() * 4
-            rq.realq_quantize_layer(dev_w_e2e[mod.name], s_in["U"], s_in["Hbar"], qcfg, p["W"], p["codes"],
-                                    p["scale"], p["zero"], dead=s_in["dead"], bcfg=p["bcfg"], F=dev_f_e2e[mod.name],
-                                    adam_m=p["am"], adam_v=p["av"], bgd_disp=p["disp"], ws=p["ws"], stream=sm)
-            with torch.cuda.stream(sm):
-                for k in ("codes", "scale", "zero"):
-                    o[k].copy_(p[k], non_blocking=True)
-                    d2h += o[k].numel() * o[k].element_size()
-        counts[name] = (h2d, d2h)
+        bq.run_serial(dev_x, dev_w, dev_f, dev_fn)
 
     def step_e2e():
-        start = torch.cuda.Event()
-        start.record(stream)
-        counts = {}
-        futs = [pool.submit(input_pipeline_e2e, name, start, counts) for name in wl.inputs]
-        for f in futs:
-            f.result()
-        for mod in wl.modules:
-            stream.wait_stream(mod_streams[mod.name])
-        for mod in wl.modules:
-            rq.realq_workspace_status(mods[mod.name]["ws"])
+        h2d, d2h = bq.run_host(host_x, host_w, host_f, host_out)
+        bq.check_status()
         torch.cuda.current_stream().synchronize()
-        e2e_bytes["h2d"] = sum(v[0] for v in counts.values())
-        e2e_bytes["d2h"] = sum(v[1] for v in counts.values())
+        e2e_bytes["h2d"], e2e_bytes["d2h"] = h2d, d2h
 
     # ---- warm-up
     for _ in range(args.warmup):
@@ -419,7 +285,9 @@ def roofline(wl, prof, steps, peaks):
         for b in range(-(-n // B)):
             be = min((b + 1) * B, n)
             r = n - be
-            bgd_p += 2 * m * n * r
+            # M = A H̄ is kept current: the product takes the previous step's
+            # free columns (K = n - b B; none before the first step)
+            bgd_p += 2 * m * (n - b * B) * r if b > 0 else 0
             bgd_g += 2 * m * m * r
             trail += 2 * m * (be - b * B) * r
             serial_bytes += m * (be - b * B) * (4 + 4 + 4) + m * (be - b * B) // 2

@@ -1,5 +1,5 @@
 // Step a2 (Sec. 3.2) on the 5th-generation tensor cores: H_sum += X̂^T X̂ for
-// bf16 calibration activations, fp32 accumulation in TMEM.
+// bf16 calibration activations.
 //
 // One CTA owns one 128 x 128 tile (i-block >= j-block) of H and a contiguous
 // range of tokens.  X̂ is token-major (T x n), so both MMA operands are read
@@ -8,10 +8,18 @@
 // stack; two boxes make the 128-channel operand (LBO = 8 KB between them,
 // SBO = 1 KB between 8-token groups).  Diagonal tiles load one operand.
 //
-// Roles (128 threads): warp 0 lane 0 issues TMA into a STAGES-deep ring,
-// warp 1 lane 0 issues tcgen05.mma (4 x K16 per 64-token stage) and frees
-// stages with tcgen05.commit; afterwards all four warps drain the 128 x 128
-// fp32 accumulator from TMEM (warp w owns lanes 32w..32w+31) and add it to H
+// Precision: the tensor core's fp32 accumulation loses about one unit in the
+// last place per accumulated MMA, in one direction, so a TMEM accumulator that
+// takes all 2^18 tokens of a calibration set (2^14 MMAs) drifts by ~1e-3 of
+// the entry.  The accumulation is therefore promoted: TMEM holds two 128 x 128
+// accumulators, the MMA issuer switches between them every CHUNK tokens, and
+// the four drain warps add each finished chunk into fp32 registers (IEEE
+// adds) while the other accumulator fills.
+//
+// Roles (192 threads): warp 4 lane 0 issues TMA into a STAGES-deep ring,
+// warp 5 lane 0 issues tcgen05.mma (4 x K16 per 64-token stage) and frees
+// stages with tcgen05.commit; warps 0-3 drain the accumulators (warp w owns
+// TMEM lanes 32w..32w+31, i.e. tile rows 32w..) and finally add the tile to H
 // and its mirror, or store it as a partial sum when tokens are split.
 // Every wait is bounded; on a timeout the tile is written as NaN (so the
 // factorisation of H reports a non-finite pivot), the workspace status word
@@ -27,11 +35,14 @@ namespace {
 constexpr int TILE = 128;
 constexpr int KSTAGE = 64;                       // tokens per pipeline stage
 constexpr int STAGES = 6;
+constexpr int CHUNK_STAGES = 8;                  // 512 tokens per TMEM accumulator pass
+constexpr int THREADS = 192;
 constexpr int OP_BYTES = TILE * KSTAGE * 2;      // one 128 x 64 bf16 operand tile
 constexpr int BOX_BYTES = 64 * KSTAGE * 2;       // one TMA box (64 channels x 64 tokens)
 constexpr int STAGE_BYTES = 2 * OP_BYTES;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
 constexpr uint32_t IDESC = tc::idesc_bf16_f32(TILE, TILE, 1, 1);
+constexpr unsigned FULL = 0xFFFFFFFFu;
 
 __device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
     int r = (int)((sqrt(8.0 * (double)idx + 1.0) - 1.0) * 0.5);
@@ -41,15 +52,16 @@ __device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
     tj = (int)(idx - (int64_t)r * (r + 1) / 2);
 }
 
-__global__ void __launch_bounds__(128, 1)
+__global__ void __launch_bounds__(THREADS, 1)
     hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, int64_t n, int64_t T, int64_t tper, float *H,
                    float *part, int direct, int *err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
     uint64_t *empty = full + STAGES;
-    uint64_t *accb = empty + STAGES;
-    uint32_t *tslot = reinterpret_cast<uint32_t *>(accb + 1);
+    uint64_t *accf = empty + STAGES;             // [2] accumulator b holds a finished chunk
+    uint64_t *acce = accf + 2;                   // [2] accumulator b has been drained
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(acce + 2);
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
@@ -60,122 +72,158 @@ __global__ void __launch_bounds__(128, 1)
     const int64_t t_begin = (int64_t)blockIdx.y * tper;
     const int64_t t_end = min(T, t_begin + tper);
     const int nk = t_end > t_begin ? (int)((t_end - t_begin + KSTAGE - 1) / KSTAGE) : 0;
+    const int nch = (nk + CHUNK_STAGES - 1) / CHUNK_STAGES;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
             tc::mbar_init(tc::smem_u32(&full[s]), 1);
             tc::mbar_init(tc::smem_u32(&empty[s]), 1);
         }
-        tc::mbar_init(tc::smem_u32(accb), 1);
+        for (int b = 0; b < 2; ++b) {
+            tc::mbar_init(tc::smem_u32(&accf[b]), 1);
+            tc::mbar_init(tc::smem_u32(&acce[b]), 4);
+        }
         *abort_flag = 0;
         tc::fence_barrier_init();
         tc::prefetch_tmap(&tmap);
     }
-    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), TILE);
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 2 * TILE);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = *tslot;
 
-    if (warp == 0 && lane == 0) {
-        // ---------------- TMA producer ----------------
-        int it = 0;
-        for (; it < nk; ++it) {
-            const int s = it % STAGES;
-            const uint32_t r = (uint32_t)(it / STAGES);
-            if (!tc::mbar_wait(tc::smem_u32(&empty[s]), (r & 1u) ^ 1u, abort_flag)) {
-                *abort_flag = 1;
-                break;
+    float acc[TILE];
+#pragma unroll
+    for (int c = 0; c < TILE; ++c) acc[c] = 0.f;
+    bool good = true;
+
+    if (warp == 4) {
+        if (lane == 0) {
+            // ---------------- TMA producer ----------------
+            int it = 0;
+            for (; it < nk; ++it) {
+                const int s = it % STAGES;
+                const uint32_t r = (uint32_t)(it / STAGES);
+                if (!tc::mbar_wait(tc::smem_u32(&empty[s]), (r & 1u) ^ 1u, abort_flag)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                const uint32_t fb = tc::smem_u32(&full[s]);
+                tc::mbar_arrive_expect_tx(fb, diag ? OP_BYTES : 2 * OP_BYTES);
+                const int y = (int)(t_begin + (int64_t)it * KSTAGE);
+                const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
+                tc::tma_load_2d(a, &tmap, fb, i0, y);
+                tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
+                if (!diag) {
+                    tc::tma_load_2d(a + OP_BYTES, &tmap, fb, j0, y);
+                    tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, &tmap, fb, j0 + 64, y);
+                }
             }
-            const uint32_t fb = tc::smem_u32(&full[s]);
-            tc::mbar_arrive_expect_tx(fb, diag ? OP_BYTES : 2 * OP_BYTES);
-            const int y = (int)(t_begin + (int64_t)it * KSTAGE);
-            const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
-            tc::tma_load_2d(a, &tmap, fb, i0, y);
-            tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
-            if (!diag) {
-                tc::tma_load_2d(a + OP_BYTES, &tmap, fb, j0, y);
-                tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, &tmap, fb, j0 + 64, y);
+            // on abort, let the copies already issued land before the CTA exits
+            if (*abort_flag) {
+                int never = 0;
+                for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k)
+                    tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (uint32_t)(k / STAGES) & 1u, &never,
+                                  100000000ull);
             }
         }
-        // on abort, let the copies already issued land before the CTA exits
-        if (*abort_flag) {
-            int never = 0;
-            for (int k = (it > STAGES ? it - STAGES : 0); k < it; ++k)
-                tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (uint32_t)(k / STAGES) & 1u, &never, 100000000ull);
+    } else if (warp == 5) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            for (int c = 0; c < nch && !*abort_flag; ++c) {
+                const int b = c & 1;
+                if (c >= 2 && !tc::mbar_wait(tc::smem_u32(&acce[b]), (uint32_t)((c >> 1) - 1) & 1u, abort_flag)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc::fence_after_sync();
+                const uint32_t d = tmem + (uint32_t)(b * TILE);
+                const int it_end = min(nk, (c + 1) * CHUNK_STAGES);
+                for (int it = c * CHUNK_STAGES; it < it_end; ++it) {
+                    const int s = it % STAGES;
+                    const uint32_t r = (uint32_t)(it / STAGES);
+                    if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
+                        *abort_flag = 1;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
+                    const uint32_t bop = diag ? a : a + OP_BYTES;
+                    const bool first = it == c * CHUNK_STAGES;
+#pragma unroll
+                    for (int k = 0; k < KSTAGE / 16; ++k) {
+                        const uint64_t da = tc::smem_desc(a + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
+                        const uint64_t db = tc::smem_desc(bop + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
+                        tc::mma_bf16_ss(d, da, db, IDESC, (first && k == 0) ? 0u : 1u);
+                    }
+                    tc::mma_commit(tc::smem_u32(&empty[s]));
+                }
+                tc::mma_commit(tc::smem_u32(&accf[b]));
+            }
         }
-    } else if (warp == 1 && lane == 0) {
-        // ---------------- MMA issuer ----------------
-        for (int it = 0; it < nk; ++it) {
-            const int s = it % STAGES;
-            const uint32_t r = (uint32_t)(it / STAGES);
-            if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
-                *abort_flag = 1;
+    } else {
+        // ---------------- drain warps: TMEM chunk -> fp32 registers ----------------
+        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        for (int c = 0; c < nch; ++c) {
+            const int b = c & 1;
+            const bool ok = tc::mbar_wait(tc::smem_u32(&accf[b]), (uint32_t)(c >> 1) & 1u, abort_flag);
+            if (!__all_sync(FULL, ok)) {
+                good = false;
                 break;
             }
             tc::fence_after_sync();
-            const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
-            const uint32_t b = diag ? a : a + OP_BYTES;
 #pragma unroll
-            for (int k = 0; k < KSTAGE / 16; ++k) {
-                const uint64_t da = tc::smem_desc(a + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
-                const uint64_t db = tc::smem_desc(b + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
-                tc::mma_bf16_ss(tmem, da, db, IDESC, (it > 0 || k > 0) ? 1u : 0u);
+            for (int c0 = 0; c0 < TILE; c0 += 32) {
+                uint32_t v[32];
+                tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(b * TILE + c0), v);
+#pragma unroll
+                for (int q = 0; q < 32; ++q) acc[c0 + q] += __uint_as_float(v[q]);
             }
-            tc::mma_commit(tc::smem_u32(&empty[s]));
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) tc::mbar_arrive(tc::smem_u32(&acce[b]));
         }
-        tc::mma_commit(tc::smem_u32(accb));
     }
     __syncwarp();
+    const bool all_good = __syncthreads_and(good && !*abort_flag) != 0;
 
-    // ---------------- epilogue: TMEM -> registers -> global ----------------
-    const bool ok = tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
-    tc::fence_after_sync();
-    const bool good = __all_sync(0xffffffffu, ok && !*abort_flag);
-    if (!good) {
-        // poison the tile: the factorisation of H then reports a non-finite pivot
+    // ---------------- epilogue: registers -> global (drain warps) ----------------
+    if (warp < 4) {
         const int row = warp * 32 + lane;
         const int64_t gi = i0 + row;
-        if (gi < n) {
-            for (int c = 0; c < TILE && j0 + c < n; ++c) {
-                const int64_t gj = j0 + c;
-                if (direct) {
-                    H[gi * n + gj] = __int_as_float(0x7fc00000);
-                    H[gj * n + gi] = __int_as_float(0x7fc00000);
-                } else {
-                    part[(int64_t)blockIdx.y * n * n + gi * n + gj] = __int_as_float(0x7fc00000);
+        if (!all_good) {
+            // poison the tile: the factorisation of H then reports a non-finite pivot
+            if (gi < n) {
+                for (int c = 0; c < TILE && j0 + c < n; ++c) {
+                    const int64_t gj = j0 + c;
+                    if (direct) {
+                        H[gi * n + gj] = __int_as_float(0x7fc00000);
+                        H[gj * n + gi] = __int_as_float(0x7fc00000);
+                    } else {
+                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = __int_as_float(0x7fc00000);
+                    }
                 }
             }
-        }
-    }
-    __syncwarp();
-    if (good && nk > 0) {
-        const int row = warp * 32 + lane;
-        const int64_t gi = i0 + row;
-#pragma unroll 1
-        for (int c0 = 0; c0 < TILE; c0 += 32) {
-            uint32_t v[32];
-            tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
-            if (gi < n) {
+        } else if (nk > 0 && gi < n) {
 #pragma unroll
-                for (int q = 0; q < 32; ++q) {
-                    const int64_t gj = j0 + c0 + q;
-                    if (gj >= n) break;
-                    const float x = __uint_as_float(v[q]);
+            for (int q = 0; q < TILE; ++q) {
+                const int64_t gj = j0 + q;
+                if (gj < n) {
                     if (direct) {
-                        H[gi * n + gj] += x;
-                        if (!diag) H[gj * n + gi] += x;
+                        H[gi * n + gj] += acc[q];
+                        if (!diag) H[gj * n + gi] += acc[q];
                     } else {
-                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = x;
+                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = acc[q];
                     }
                 }
             }
         }
     }
-    if (!good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
+    if (!all_good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
     tc::fence_before_sync();
     __syncthreads();
-    if (warp == 0) tc::tmem_dealloc(tmem, TILE);
+    if (warp == 0) tc::tmem_dealloc(tmem, 2 * TILE);
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -251,7 +299,7 @@ realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void 
     float *part = static_cast<float *>(ws);
     {
         Launch L("hessian_syrk_tc", s);
-        hess_tc_kernel<<<dim3((unsigned)lower, (unsigned)splits), 128, SMEM_BYTES, s>>>(map, n, T, tper, H, part,
+        hess_tc_kernel<<<dim3((unsigned)lower, (unsigned)splits), THREADS, SMEM_BYTES, s>>>(map, n, T, tper, H, part,
                                                                                        splits == 1, err);
     }
     REALQ_TRY(check_launch("hessian_syrk_tc"));
