@@ -12,7 +12,7 @@
 // last place per accumulated MMA, in one direction, so a TMEM accumulator that
 // takes all 2^18 tokens of a calibration set (2^14 MMAs) drifts by ~1e-3 of
 // the entry.  The accumulation is therefore promoted: TMEM holds two 128 x 128
-// accumulators, the MMA issuer switches between them every CHUNK tokens, and
+// accumulators, the MMA issuer switches between them every 1024 tokens, and
 // the four drain warps add each finished chunk into fp32 registers (IEEE
 // adds) while the other accumulator fills.
 //
@@ -35,7 +35,7 @@ namespace {
 constexpr int TILE = 128;
 constexpr int KSTAGE = 64;                       // tokens per pipeline stage
 constexpr int STAGES = 6;
-constexpr int CHUNK_STAGES = 8;                  // 512 tokens per TMEM accumulator pass
+constexpr int CHUNK_STAGES = 16;                 // 1024 tokens per TMEM accumulator pass
 constexpr int THREADS = 192;
 constexpr int OP_BYTES = TILE * KSTAGE * 2;      // one 128 x 64 bf16 operand tile
 constexpr int BOX_BYTES = 64 * KSTAGE * 2;       // one TMA box (64 channels x 64 tokens)

@@ -264,7 +264,7 @@ __global__ void scale_kernel(int64_t count, float div, const float *in, float *o
 }
 
 constexpr size_t align256(size_t x) { return (x + 255) / 256 * 256; }
-constexpr int KSPLIT_MAX = 8;    // K slices of the triangular-inverse panel product
+constexpr int KSPLIT_MAX = 16;   // K slices of the triangular-inverse panel product
 constexpr size_t prepare_bytes_split(int64_t n, int slices) {
     return align256(sizeof(int)) + align256(sizeof(float)) + align256((size_t)NB * NB * sizeof(float)) +
            align256((size_t)slices * n * NB * sizeof(float));
@@ -426,7 +426,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, co
             const int64_t r = n - k1;
             // X = R[K, K+1:] U[K+1:, K+1:] (U upper: a column tile's K range ends
             // at its last column), K split into fixed-order slices
-            const int ks = (int)std::max<int64_t>(1, std::min<int64_t>(slices, r / 512));
+            const int ks = (int)std::max<int64_t>(1, std::min<int64_t>(slices, r / 256));
             GemmArgs g{};
             g.M = kb; g.N = r; g.K = r;
             g.A = U + k0 * n + k1; g.lda = n;
