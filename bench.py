@@ -31,12 +31,12 @@ import synth  # noqa: E402
 METRIC = "quantized weight-columns/sec per layer on 1 GB300; % tensor-core peak / % HBM BW"
 UNIT = "columns/s"
 
-# dram bytes per launch from ncu captures (profiles/), keyed by kernel; None
+# dram bytes per launch from ncu captures (profiles/), keyed by (workload, kernel); None
 # when the kernel changed after its capture.
 NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
-    "hessian_syrk_tc": 1523751616,
+    ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
 }
 
 
@@ -329,7 +329,7 @@ def roofline(wl, prof, steps, peaks):
         achieved = total / secs / 1e9
         peak = peaks["hbm_gbs"]
         peak_note = f"HBM copy, {peaks['source']}"
-    traffic = NCU_TRAFFIC.get(name)
+    traffic = NCU_TRAFFIC.get((wl.name, name))
     return {"kernel": name, "bound": bound, "achieved": achieved, "peak": peak, "unit": unit,
             "frac": achieved / peak, "traffic": traffic, "peak_source": peak_note,
             "launches": launches, "avg_launch_ms": ms / launches,
