@@ -35,6 +35,7 @@ __all__ = [
     "hessian_sum", "cross_moment_sum", "prepare", "inverse_upper_cholesky",
     "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
     "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
+    "round_bf16", "quantize_activations",
 ]
 
 
@@ -336,3 +337,42 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         "block_loss": block_loss, "adam_t": 0 if opt is None else opt.t,
         "Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": prep["lam"], "Dbar": Dbar,
     }
+
+
+# ---------------------------------------------------------------------------
+# Weight-activation setting (Sec. 5, "Weight-Activation Quantization"):
+# activations are quantized per token with a clipping ratio (a_clip = 0.9 in
+# the paper), and in the activation-aware variant the weights are quantized
+# against the already-quantized activations (they are the x̂ of the Hessian,
+# and the full-precision x stay the reference of the surrogate).
+# Readings: the activation grid is the symmetric grid of quant(.) ("symmetric
+# throughout", Sec. 5.1) on the clipped range [-a_clip max|x_t|, a_clip
+# max|x_t|] of each token; values beyond it take the end levels; a token of
+# all zeros gets the range [-1, 1]; the dequantized value is formed in fp32
+# and stored in the input's format (bf16, round to nearest even).  As for the
+# weights, the integer decisions are taken in fp32.
+# ---------------------------------------------------------------------------
+def round_bf16(a: np.ndarray) -> np.ndarray:
+    """fp32 values rounded to the nearest bf16 (ties to even), as fp32."""
+    u = np.ascontiguousarray(a, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = (u + np.uint64(0x7FFF) + ((u >> np.uint64(16)) & np.uint64(1))) & np.uint64(0xFFFF0000)
+    return u.astype(np.uint32).view(np.float32)
+
+
+def quantize_activations(X: np.ndarray, bits: int = 4, a_clip: float = 0.9, out_bf16: bool = True):
+    """Per-token symmetric b-bit quantization of X (T x n).
+
+    Returns (codes int64 T x n, scale fp32 per token, dequantized X as fp64 of
+    its stored value)."""
+    x = np.asarray(X, dtype=np.float64).astype(np.float32)
+    maxq = np.float32(2 ** bits - 1)
+    zero = 2 ** (bits - 1)
+    xmax = (np.float32(a_clip) * np.abs(x).max(axis=1)).astype(np.float32)
+    xmax = np.where(xmax == 0, np.float32(1.0), xmax).astype(np.float32)
+    scale = ((xmax - (-xmax)) / maxq).astype(np.float32)
+    r = np.rint((x / scale[:, None]).astype(np.float32))
+    q = np.clip(r.astype(np.int64) + zero, 0, 2 ** bits - 1)
+    xq = (scale[:, None] * (q - zero).astype(np.float32)).astype(np.float32)
+    if out_bf16:
+        xq = round_bf16(xq)
+    return q, scale, xq.astype(np.float64)

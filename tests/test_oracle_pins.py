@@ -376,3 +376,53 @@ def test_single_column_sweep_is_exact_minimiser():
         best, arg = brute.row_min(W0[i], s[i], z[i], H / 1.0)
         val = brute.row_eval(W0[i], s[i], z[i], H / 1.0, res["codes"][i])
         assert val <= best * (1 + 1e-12) + 1e-300
+
+
+# ------------------------------------------------ activation quantizer ---
+def test_activation_quantizer_worked_example():
+    # Sec. 5 weight-activation setting, per-token symmetric 4-bit, a_clip 0.9:
+    # max|x| = 2 -> clipped range 1.8 -> step 3.6 / 15 = 0.24, zero point 8;
+    # x / 0.24 = (2.08, -4.17, 1.04, 8.33) -> (2, -4, 1, 8), and 8 + 8 = 16 is
+    # clamped to the last level 15; the dequantized values 0.48, -0.96, 0.24,
+    # 1.68 stored in bf16 (steps 2^-9, 2^-8, 2^-10, 2^-7) are
+    # 246 * 2^-9, -246 * 2^-8, 246 * 2^-10 and 215 * 2^-7.
+    x = np.array([[0.5, -1.0, 0.25, 2.0]])
+    q, scale, xq = oracle.quantize_activations(x, bits=4, a_clip=0.9)
+    assert q.tolist() == [[10, 4, 9, 15]]
+    assert abs(float(scale[0]) - 0.24) < 1e-7
+    assert xq.tolist() == [[246 / 512, -246 / 256, 246 / 1024, 215 / 128]]
+
+
+def test_activation_quantizer_nearest_level_and_clipping():
+    r = np.random.default_rng(5)
+    X = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(r.standard_normal((64, 200)) * np.exp(r.standard_normal((64, 1)))))
+    X[3] = 0.0
+    for bits, clip in ((4, 0.9), (4, 1.0), (3, 0.8), (8, 0.9)):
+        q, scale, xq = oracle.quantize_activations(X, bits=bits, a_clip=clip, out_bf16=False)
+        z = 2 ** (bits - 1)
+        levels = np.arange(2 ** bits) - z
+        x = X.astype(np.float64)
+        # brute force over all 2^b levels of each token's grid
+        cand = scale[:, None, None].astype(np.float64) * levels[None, None, :]
+        dist = np.abs(x[:, :, None] - cand)
+        best = dist.argmin(axis=2)
+        srt = np.sort(dist, axis=2)
+        # not a tie, beyond the fp32 rounding of x / scale (2^-24 relative)
+        clear = (srt[:, :, 1] - srt[:, :, 0]) > 1e-6 * scale[:, None] + 2.0 ** -22 * np.abs(x)
+        assert np.array_equal(q[clear], best[clear])
+        # the clipped range: values beyond +-(levels) sit on the end levels
+        amax = np.abs(x).max(axis=1)
+        assert np.all(q[3] == z) and abs(float(scale[3]) - 2.0 / (2 ** bits - 1)) < 1e-7
+        xmax = np.where(amax == 0, 1.0, clip * amax)
+        np.testing.assert_allclose(scale, 2 * xmax / (2 ** bits - 1), rtol=1e-6)
+        ref = scale[:, None].astype(np.float64) * (q - z)
+        assert np.all(np.abs(xq - ref) <= 2.0 ** -24 * np.abs(ref))
+        inside = np.abs(x) <= (z - 1) * scale[:, None]
+        half = 0.5 * scale[:, None] * (1 + 1e-6) + 2.0 ** -22 * np.abs(x)
+        assert np.all((np.abs(x - xq) <= half)[inside])
+
+
+def test_bf16_rounding_matches_the_input_generator_cast():
+    r = np.random.default_rng(6)
+    a = (r.standard_normal(10000) * 10 ** r.uniform(-3, 3, 10000)).astype(np.float32)
+    assert np.array_equal(oracle.round_bf16(a), synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(a)))
