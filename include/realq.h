@@ -160,6 +160,27 @@ realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, i
                                              const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
                                              int64_t *fail_col);
 
+/* Weight-activation setting (Sec. 5, "Weight-Activation Quantization";
+ * W4A4 uses 4 bits and a_clip = 0.9).  Per-token symmetric quantization of
+ * the calibration activations X (T x n, row-major, REALQ_BF16 or REALQ_F32):
+ * for each token t, xmax = a_clip * max_j |X[t, j]| (1 for a row of zeros),
+ * scale[t] = 2 xmax / (2^bits - 1), zero point 2^(bits-1), and
+ *   codes[t, j] = clamp(rint(X[t, j] / scale[t]) + 2^(bits-1), 0, 2^bits - 1),
+ *   X_q[t, j]   = scale[t] * (codes[t, j] - 2^(bits-1)),
+ * formed in fp32 with IEEE-rounded operations and stored in x_dtype (bf16:
+ * round to nearest even).  In the activation-aware variant X_q is the x̂ given
+ * to realq_hessian_accumulate (with X as X_fp, so that the surrogate keeps
+ * the full-precision reference).
+ *   X_q     T x n, x_dtype, may alias X.
+ *   codes   NULL, or T x ceil(n/2) bytes for bits <= 4 (two codes per byte,
+ *           even column in the low nibble), T x n bytes for bits 5..8.
+ *   scale   NULL, or T floats.
+ * bits in [2, 8], 0 < a_clip <= 1, inputs finite.  Asynchronous; allocates
+ * nothing. */
+realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int64_t n, const void *X,
+                                          realq_dtype_t x_dtype, int bits, float a_clip, void *X_q, uint8_t *codes,
+                                          float *scale);
+
 /* Dbar = D_sum / T_total (n x n); may alias D_sum.  Asynchronous. */
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum,
                                   float *Dbar);

@@ -20,6 +20,7 @@ __all__ = [
     "RealqError", "QuantCfg", "BgdCfg", "lib", "library_path", "quant_cfg", "bgd_cfg", "workspace",
     "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
     "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
+    "realq_quantize_activations",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -78,6 +79,7 @@ _SIGS = {
     "realq_prepare_workspace_size": ([_i64], _sz),
     "realq_hessian_prepare_noalloc": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64], _int),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
+    "realq_quantize_activations": ([_vp, _i64, _i64, _vp, _int, _int, _f32, _vp, _vp, _vp], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
                               ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
                               _i64, _i64, _vp, _sz], _int),
@@ -214,6 +216,23 @@ def realq_hessian_prepare_noalloc(H_sum: torch.Tensor, T_total: int, damp_frac: 
                                              _ptr(U_out), _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc))
     _check(st, fail_col=fc.value)
     return fc.value
+
+
+def realq_quantize_activations(X: torch.Tensor, bits: int = 4, a_clip: float = 0.9,
+                               X_q: Optional[torch.Tensor] = None, codes: Optional[torch.Tensor] = None,
+                               scale: Optional[torch.Tensor] = None, stream=None) -> torch.Tensor:
+    """Per-token symmetric activation quantization (weight-activation setting).
+    Returns X_q (allocated like X when not given; may be X itself)."""
+    T, n = X.shape
+    if X_q is None:
+        X_q = torch.empty_like(X)
+    _need(X_q, X.dtype, (T, n), "X_q")
+    if codes is not None:
+        _need(codes, torch.uint8, (T, (n + 1) // 2 if bits <= 4 else n), "codes")
+    _need(scale, torch.float32, (T,), "scale")
+    _check(lib().realq_quantize_activations(_stream(stream), T, n, _ptr(X), _dtype(X), bits, a_clip, _ptr(X_q),
+                                            _ptr(codes), _ptr(scale)))
+    return X_q
 
 
 def realq_scale_moment(D_sum: torch.Tensor, T_total: int, Dbar: torch.Tensor, stream=None):

@@ -249,6 +249,18 @@ realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, i
     return prepare_noalloc(S(stream), n, T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col);
 }
 
+realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int64_t n, const void *X,
+                                          realq_dtype_t x_dtype, int bits, float a_clip, void *X_q, uint8_t *codes,
+                                          float *scale) {
+    if (T < 0 || n <= 0 || !X || !X_q) return fail(REALQ_ERR_INVALID_ARG, "quantize_activations: bad argument");
+    if (x_dtype != REALQ_BF16 && x_dtype != REALQ_F32)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_activations: x_dtype must be REALQ_BF16 or REALQ_F32");
+    if (bits < 2 || bits > 8) return fail(REALQ_ERR_INVALID_ARG, "quantize_activations: bits must be in [2, 8]");
+    if (!(a_clip > 0.f && a_clip <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "quantize_activations: 0 < a_clip <= 1");
+    if (T > (int64_t)INT32_MAX * 8) return fail(REALQ_ERR_UNSUPPORTED, "quantize_activations: too many tokens");
+    return act_quant(S(stream), T, n, X, x_dtype, bits, a_clip, X_q, codes, scale);
+}
+
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum, float *Dbar) {
     if (n <= 0 || T_total <= 0 || !D_sum || !Dbar) return fail(REALQ_ERR_INVALID_ARG, "scale_moment: bad argument");
     return scale_copy(S(stream), n * n, (float)T_total, D_sum, Dbar);

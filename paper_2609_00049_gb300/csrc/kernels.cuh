@@ -72,6 +72,10 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
                               int b_row0, const TcEpi &e, int *err, const char *name);
 
+// ------------------------------------------------- activation quantizer ---
+realq_status_t act_quant(cudaStream_t s, int64_t T, int64_t n, const void *X, realq_dtype_t dt, int bits, float a_clip,
+                         void *Xq, uint8_t *codes, float *scale);
+
 // --------------------------------------------------------------- Hessian ---
 int hessian_splits(int64_t n, int64_t T, int num_sms);
 int num_sms();

@@ -64,11 +64,6 @@ __global__ void group_params_kernel(int64_t m, int64_t n, const float *W, int64_
     }
 }
 
-__device__ __forceinline__ void cp_async4(float *dst, const float *src) {
-    const uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(dst));
-    asm volatile("cp.async.ca.shared.global [%0], [%1], 4;" ::"r"(d), "l"(src) : "memory");
-}
-
 struct QArgs {
     int64_t m, n, bs;
     int kb;

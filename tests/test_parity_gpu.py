@@ -330,3 +330,64 @@ def test_surrogate_loss_matches_oracle():
     L_or = oracle.surrogate_tokens(What, case.W0, case.Xhat, None, case.F)
     L_gpu = gpu_loss(dev(What), dev(case.W0), dev(Hs / T), dev(case.F))
     assert abs(L_gpu - L_or) <= 1e-4 * L_or
+
+
+# ------------------------------------------------ activation quantizer ---
+@pytest.mark.parametrize("T,n,bits,clip", [(1000, 1024, 4, 0.9), (333, 197, 4, 0.9), (64, 4096, 3, 0.8),
+                                           (50, 96, 8, 1.0), (1, 31, 4, 0.9)])
+def test_activation_quantizer_bit_exact(T, n, bits, clip):
+    r = synth.rng(41, "act-quant", T, n)
+    x = r.standard_normal((T, n)) * np.exp(r.standard_normal((T, 1)))
+    x[:, r.integers(0, n, 3)] *= 30.0                      # outlier channels
+    x[T // 2] = 0.0                                        # a token of zeros
+    bits16 = synth.f32_to_bf16_bits(x)
+    xb = synth.bf16_bits_to_f32(bits16)
+    q_or, s_or, xq_or = oracle.quantize_activations(xb, bits=bits, a_clip=clip)
+    X = bf16_dev(bits16)
+    ncb = (n + 1) // 2 if bits <= 4 else n
+    codes = torch.empty(T, ncb, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(T, dtype=torch.float32, device="cuda")
+    Xq = rq.realq_quantize_activations(X, bits, clip, codes=codes, scale=scale)
+    assert np.array_equal(scale.cpu().numpy(), s_or)
+    assert np.array_equal(Xq.float().cpu().numpy().astype(np.float64), xq_or)
+    c = codes.cpu().numpy()
+    q = unpack(c, n) if bits <= 4 else c.astype(np.int64)
+    assert np.array_equal(q, q_or)
+    # fp32 activations: the same codes, the dequantized values kept in fp32
+    Xf = dev(xb)
+    Xqf = rq.realq_quantize_activations(Xf, bits, clip)
+    _, _, xq32 = oracle.quantize_activations(xb, bits=bits, a_clip=clip, out_bf16=False)
+    assert np.array_equal(Xqf.cpu().numpy().astype(np.float64), xq32)
+    # in place
+    rq.realq_quantize_activations(X, bits, clip, X_q=X)
+    assert torch.equal(X, Xq)
+
+
+def test_activation_aware_sweep():
+    # W4A4 activation-aware: the weights see the quantized activations (x̂), the
+    # surrogate keeps the full-precision ones (x) through the cross moment
+    case = synth.layer_case(42, 96, 256, 1500, bf16=True, outliers=3)
+    x_bits = synth.f32_to_bf16_bits(case.Xhat)
+    _, _, xhat = oracle.quantize_activations(case.Xhat, bits=4, a_clip=0.9)
+    X = bf16_dev(x_bits)
+    Xq = rq.realq_quantize_activations(X, 4, 0.9)
+    assert np.array_equal(Xq.float().cpu().numpy().astype(np.float64), xhat)
+    qkw = dict(group_size=128, block_size=128)
+    Hs, T = oracle.hessian_sum([xhat])
+    Ds = oracle.cross_moment_sum([xhat], [case.Xhat])
+    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128,
+                             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}, F=case.F,
+                             D_sum=Ds)
+    H, D, T_ = layer.accumulate([Xq], 256, [X])
+    prep = layer.prepare(H, T_, 0.01, D_sum=D)
+    out = layer.quantize(dev(case.W0), prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4), F=dev(case.F), use_dbar=True)
+    torch.cuda.synchronize()
+    n = 256
+    codes = unpack(out.codes.cpu().numpy(), n)
+    rep = compare_codes(codes, orc, 128, 128, True)
+    frac, med, s_unexpl = scale_agreement(out.scale.cpu().numpy(), orc["scale"], 128,
+                                          explained=compare_codes.last_explained,
+                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, 1))
+    print(f"\nactivation-aware: {rep} scale_within_1e-5={frac:.5f}")
+    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
+    assert s_unexpl == 0
