@@ -155,7 +155,8 @@ def gpu_arm(args, wl, rank, world):
     # the block's modules, scheduled concurrently by the library's block scheduler
     bq = BlockQuantizer([BlockInput(nm, sp.n, sp.T) for nm, sp in wl.inputs.items()],
                         [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
-                        wl.steps_per_block, sliding_window=wl.sliding_window, device=dev)
+                        wl.steps_per_block, sliding_window=wl.sliding_window, device=dev,
+                        act_quant=(args.act_bits, args.a_clip) if args.act_bits else None)
     host_out = {mod.name: {k: torch.empty_like(bq.out[mod.name][k], device="cpu").pin_memory()
                            for k in ("codes", "scale", "zero")} for mod in wl.modules}
     e2e_bytes = {"h2d": 0, "d2h": 0}
@@ -224,7 +225,7 @@ def gpu_arm(args, wl, rank, world):
 
     # ---- end to end through host buffers
     e2e = None
-    if not args.no_e2e:
+    if not args.no_e2e and not args.act_bits:
         step_e2e()
         torch.cuda.synchronize()
         barrier()
@@ -257,7 +258,9 @@ def gpu_arm(args, wl, rank, world):
             "config": {"workload": wl.name, "description": wl.description, "modules": len(wl.modules),
                        "calibration_tokens": wl.inputs[wl.modules[0].input].T,
                        "columns_per_step": wl.total_columns, "column_blocks_per_step": wl.total_column_blocks,
-                       "quantizer": f"W{wl.bits} {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}",
+                       "quantizer": f"W{wl.bits}" + (f"A{args.act_bits} (activation-aware, a_clip {args.a_clip})"
+                                                     if args.act_bits else "") +
+                                    f" {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}",
                        "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}",
                        "parallelism": f"replicas x{world}",
                        "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
@@ -462,6 +465,9 @@ def main():
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
     ap.add_argument("--workload", default="qwen3-0.6b")
     ap.add_argument("--no-e2e", action="store_true")
+    ap.add_argument("--act-bits", type=int, default=0,
+                    help="activation-aware weight-activation variant: per-token activation bits (0: weights only)")
+    ap.add_argument("--a-clip", type=float, default=0.9, help="activation clipping ratio for --act-bits")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep"], default=None,

@@ -22,9 +22,10 @@ from typing import Dict, List, Optional, Sequence
 
 import torch
 
-from . import (QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_hessian_prepare, realq_hessian_workspace_size,
-               realq_prepare_workspace_size, realq_quantize_layer, realq_quantize_workspace_size,
-               realq_workspace_status, workspace)
+from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_hessian_prepare,
+               realq_hessian_workspace_size, realq_prepare_workspace_size, realq_quantize_activations,
+               realq_quantize_layer, realq_quantize_workspace_size, realq_scale_moment, realq_workspace_status,
+               workspace)
 
 
 @dataclass
@@ -52,11 +53,16 @@ class BlockQuantizer:
     over all modules' blocks).  lr and steps_per_block configure Block-GD (0
     steps disables it); sliding_window=True uses F_eff = alpha F + (1-alpha) F'
     with alpha decaying over the block's B_total column blocks.
+
+    act_quant=(bits, a_clip) selects the activation-aware weight-activation
+    variant (Sec. 5): each input is quantized per token first, the Hessian is
+    taken over the quantized activations, and the Block-GD surrogate keeps
+    the full-precision ones through the cross moment D.
     """
 
     def __init__(self, inputs: Sequence[BlockInput], modules: Sequence[BlockModule], qcfg: QuantCfg, lr: float,
                  steps_per_block: int = 1, sliding_window: bool = False, device="cuda",
-                 host_chunk_tokens: int = 32768):
+                 host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None):
         self.inputs: Dict[str, BlockInput] = {i.name: i for i in inputs}
         self.modules: List[BlockModule] = list(modules)
         for md in self.modules:
@@ -64,7 +70,10 @@ class BlockQuantizer:
                 raise ValueError(f"module {md.name}: input {md.input!r} missing or of the wrong width")
         self.qcfg = qcfg
         self.device = torch.device(device)
+        if self.device.index is None:
+            self.device = torch.device(self.device.type, torch.cuda.current_device())
         self.sliding_window = sliding_window
+        self.act_quant = act_quant
         self.mods_of = {name: [md for md in self.modules if md.input == name] for name in self.inputs}
         B = qcfg.block_size
         self.B_total = sum(-(-md.n // B) for md in self.modules)
@@ -76,7 +85,10 @@ class BlockQuantizer:
                 H=torch.empty(n, n, device=dev), U=torch.empty(n, n, device=dev), Hbar=torch.empty(n, n, device=dev),
                 dead=torch.empty(n, dtype=torch.uint8, device=dev),
                 pws=workspace(realq_prepare_workspace_size(n), dev),
-                hws=workspace(realq_hessian_workspace_size(n, spec.T), dev))
+                hws=workspace(realq_hessian_workspace_size(n, spec.T, REALQ_BF16, act_quant is not None), dev))
+            if act_quant is not None:
+                self.state[name].update(Xq=torch.empty(spec.T, n, dtype=torch.bfloat16, device=dev),
+                                        D=torch.empty(n, n, device=dev), Dbar=torch.empty(n, n, device=dev))
         self.out = {}
         bstart = 1
         g_eff = qcfg.group_size
@@ -94,8 +106,8 @@ class BlockQuantizer:
                 scale=torch.empty(m, ng, device=dev), zero=torch.empty(m, ng, dtype=torch.uint8, device=dev),
                 am=torch.empty(m, n, device=dev) if bgd else None, av=torch.empty(m, n, device=dev) if bgd else None,
                 disp=torch.empty(m, n, device=dev) if bgd else None, bcfg=bc if bgd else None,
-                ws=workspace(realq_quantize_workspace_size(m, n, qcfg, bc if bgd else None, sliding_window, False),
-                             dev),
+                ws=workspace(realq_quantize_workspace_size(m, n, qcfg, bc if bgd else None, sliding_window,
+                                                           act_quant is not None and bgd), dev),
                 adam_t=0)
         self.in_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
         self.copy_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
@@ -111,7 +123,8 @@ class BlockQuantizer:
     def _quantize_module(self, md: BlockModule, s_in, W0, F, F_next, stream):
         o = self.out[md.name]
         o["adam_t"] = realq_quantize_layer(
-            W0, s_in["U"], s_in["Hbar"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"], dead=s_in["dead"],
+            W0, s_in["U"], s_in["Hbar"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"],
+            Dbar=s_in.get("Dbar") if o["bcfg"] is not None else None, dead=s_in["dead"],
             bcfg=o["bcfg"], F=F, F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"],
             bgd_disp=o["disp"], ws=o["ws"], stream=stream)
 
@@ -119,15 +132,29 @@ class BlockQuantizer:
         torch.cuda.set_device(self.device)
         spec, s_in, si = self.inputs[name], self.state[name], self.in_streams[name]
         si.wait_event(start)
-        with torch.cuda.stream(si):
-            s_in["H"].zero_()
-        realq_hessian_accumulate(X[name], s_in["H"], ws=s_in["hws"], stream=si)
-        realq_hessian_prepare(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                              s_in["pws"], stream=si)
+        self._hessian(name, X[name], si)
         for md in self.mods_of[name]:
             sm = self.mod_streams[md.name]
             sm.wait_stream(si)
             self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), sm)
+
+    def _hessian(self, name, X, stream):
+        """H (and, activation-aware, D) of one input, then its preparation."""
+        spec, s_in = self.inputs[name], self.state[name]
+        with torch.cuda.stream(stream if stream is not None else torch.cuda.current_stream(self.device)):
+            s_in["H"].zero_()
+            if self.act_quant is not None:
+                s_in["D"].zero_()
+        if self.act_quant is None:
+            realq_hessian_accumulate(X, s_in["H"], ws=s_in["hws"], stream=stream)
+        else:
+            bits, clip = self.act_quant
+            realq_quantize_activations(X, bits, clip, X_q=s_in["Xq"], stream=stream)
+            realq_hessian_accumulate(s_in["Xq"], s_in["H"], s_in["D"], X, ws=s_in["hws"], stream=stream)
+        realq_hessian_prepare(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
+                              s_in["pws"], stream=stream)
+        if self.act_quant is not None:
+            realq_scale_moment(s_in["D"], spec.T, s_in["Dbar"], stream=stream)
 
     def _join(self, start_stream):
         for md in self.modules:
@@ -153,10 +180,7 @@ class BlockQuantizer:
         """The same work, one call after another on the current stream."""
         for name, spec in self.inputs.items():
             s_in = self.state[name]
-            s_in["H"].zero_()
-            realq_hessian_accumulate(X[name], s_in["H"], ws=s_in["hws"])
-            realq_hessian_prepare(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                                  s_in["pws"])
+            self._hessian(name, X[name], None)
             for md in self.mods_of[name]:
                 self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), None)
 
@@ -214,7 +238,10 @@ class BlockQuantizer:
         """End to end from pinned host memory: X̂ streams in chunks on a copy
         stream per input (double-buffered, overlapped with accumulation), W0
         and F are copied per module, codes / scale / zero are copied back into
-        out_host[module][...] (pinned).  Returns (h2d bytes, d2h bytes)."""
+        out_host[module][...] (pinned).  Returns (h2d bytes, d2h bytes).
+        The activation-aware variant is not streamed (it runs with run())."""
+        if self.act_quant is not None:
+            raise NotImplementedError("run_host: the activation-aware variant runs from device-resident inputs")
         dev = self.device
         if self._stage is None:
             self._stage = {name: [torch.empty(self.host_chunk, spec.n, dtype=X_host[name].dtype, device=dev)

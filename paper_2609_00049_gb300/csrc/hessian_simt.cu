@@ -180,7 +180,10 @@ realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float
 
 int hessian_splits(int64_t n, int64_t T, int sms) {
     const int nt = ceil_div(n, TB);
-    const int64_t lower = (int64_t)nt * (nt + 1) / 2;
+    return hessian_splits_tiles((int64_t)nt * (nt + 1) / 2, T, sms);
+}
+
+int hessian_splits_tiles(int64_t lower, int64_t T, int sms) {
     int64_t want = (sms + lower / 2) / lower;       // nearest whole number of waves
     const int64_t by_tokens = T / 4096;              // at least 4096 tokens per split
     if (want > by_tokens) want = by_tokens;
@@ -208,8 +211,15 @@ realq_status_t hessian_accumulate(cudaStream_t s, int64_t n, int64_t T, const vo
         pbytes = ws_bytes - align_up(sizeof(int));
     }
     const bool tc_path = dt == REALQ_BF16 && hessian_tc_eligible(n, T, X);
-    if (tc_path) REALQ_TRY(hessian_syrk_tc(s, n, T, X, H, err, pw, pbytes, num_sms()));
+    const bool tc_cross = tc_path && Xfp && hessian_tc_eligible(n, T, Xfp);
+    // tensor cores: H += X̂ᵀX̂ (and D += X̂ᵀX̂ from the same pass), D -= XᵀX̂
+    if (tc_path) REALQ_TRY(hessian_syrk_tc(s, n, T, X, H, err, pw, pbytes, num_sms(), tc_cross ? D : nullptr));
+    if (tc_cross) REALQ_TRY(hessian_cross_tc(s, n, T, Xfp, X, D, -1.f, err, pw, pbytes, num_sms()));
     float *Hs = tc_path ? nullptr : H;
+    if (tc_cross) {
+        Xfp = nullptr;
+        D = nullptr;
+    }
     if (dt == REALQ_BF16)
         return run<__nv_bfloat16>(s, n, T, static_cast<const __nv_bfloat16 *>(X),
                                   static_cast<const __nv_bfloat16 *>(Xfp), Hs, D, pw, pbytes);

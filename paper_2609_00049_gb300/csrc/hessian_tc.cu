@@ -21,6 +21,10 @@
 // stages with tcgen05.commit; warps 0-3 drain the accumulators (warp w owns
 // TMEM lanes 32w..32w+31, i.e. tile rows 32w..) and finally add the tile to H
 // and its mirror, or store it as a partial sum when tokens are split.
+// The cross mode computes the full (non-symmetric) product X_Aᵀ X_B of two
+// token-major inputs over all tiles, scaled by a sign and added to the output
+// without mirroring: the cross moment of the perturbed-input surrogate is
+// D = X̂ᵀX̂ - XᵀX̂, the symmetric pass (also added into D) minus this one.
 // Every wait is bounded; on a timeout the tile is written as NaN (so the
 // factorisation of H reports a non-finite pivot), the workspace status word
 // gets ST_TIMEOUT, and the kernel still frees TMEM and returns.
@@ -53,8 +57,9 @@ __device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
-    hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, int64_t n, int64_t T, int64_t tper, float *H,
-                   float *part, int direct, int *err) {
+    hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmapB, int64_t n,
+                   int64_t T, int64_t tper, float *H, float *H2, float *part, int direct, int cross, float sign,
+                   int *err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -66,8 +71,14 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     int ti, tj;
-    lower_tile(blockIdx.x, ti, tj);
-    const bool diag = ti == tj;
+    if (cross) {
+        const int nt = (int)((n + TILE - 1) / TILE);
+        ti = (int)(blockIdx.x / nt);
+        tj = (int)(blockIdx.x % nt);
+    } else {
+        lower_tile(blockIdx.x, ti, tj);
+    }
+    const bool diag = !cross && ti == tj;
     const int i0 = ti * TILE, j0 = tj * TILE;
     const int64_t t_begin = (int64_t)blockIdx.y * tper;
     const int64_t t_end = min(T, t_begin + tper);
@@ -86,6 +97,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         *abort_flag = 0;
         tc::fence_barrier_init();
         tc::prefetch_tmap(&tmap);
+        if (cross) tc::prefetch_tmap(&tmapB);
     }
     if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 2 * TILE);
     tc::fence_before_sync();
@@ -116,8 +128,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                 tc::tma_load_2d(a, &tmap, fb, i0, y);
                 tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
                 if (!diag) {
-                    tc::tma_load_2d(a + OP_BYTES, &tmap, fb, j0, y);
-                    tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, &tmap, fb, j0 + 64, y);
+                    const CUtensorMap *mb = cross ? &tmapB : &tmap;
+                    tc::tma_load_2d(a + OP_BYTES, mb, fb, j0, y);
+                    tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, mb, fb, j0 + 64, y);
                 }
             }
             // on abort, let the copies already issued land before the CTA exits
@@ -199,7 +212,11 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const int64_t gj = j0 + c;
                     if (direct) {
                         H[gi * n + gj] = __int_as_float(0x7fc00000);
-                        H[gj * n + gi] = __int_as_float(0x7fc00000);
+                        if (!cross) H[gj * n + gi] = __int_as_float(0x7fc00000);
+                        if (H2) {
+                            H2[gi * n + gj] = __int_as_float(0x7fc00000);
+                            H2[gj * n + gi] = __int_as_float(0x7fc00000);
+                        }
                     } else {
                         part[(int64_t)blockIdx.y * n * n + gi * n + gj] = __int_as_float(0x7fc00000);
                     }
@@ -210,11 +227,16 @@ __global__ void __launch_bounds__(THREADS, 1)
             for (int q = 0; q < TILE; ++q) {
                 const int64_t gj = j0 + q;
                 if (gj < n) {
+                    const float v = sign * acc[q];
                     if (direct) {
-                        H[gi * n + gj] += acc[q];
-                        if (!diag) H[gj * n + gi] += acc[q];
+                        H[gi * n + gj] += v;
+                        if (!diag && !cross) H[gj * n + gi] += v;
+                        if (H2) {
+                            H2[gi * n + gj] += v;
+                            if (!diag) H2[gj * n + gi] += v;
+                        }
                     } else {
-                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = acc[q];
+                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = v;
                     }
                 }
             }
@@ -277,14 +299,22 @@ bool hessian_tc_eligible(int64_t n, int64_t T, const void *X) {
            n < (1ll << 31);
 }
 
-realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
-                               size_t ws_bytes, int sms) {
-    CUtensorMap map;
-    CUresult cr = encode_tmap_2d_bf16(&map, X, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
+// out (+= sign X_Aᵀ X_B); symmetric (X_B null): lower tiles mirrored, and
+// out2 (if given) receives the same sum.  Token splits go through the
+// workspace partials and a fixed-order reduction.
+static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
+                                     float *out2, float sign, int *err, void *ws, size_t ws_bytes, int sms,
+                                     const char *name) {
+    CUtensorMap mapA, mapB;
+    CUresult cr = encode_tmap_2d_bf16(&mapA, XA, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
+    if (cr == CUDA_SUCCESS && XB)
+        cr = encode_tmap_2d_bf16(&mapB, XB, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
     if (cr != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)cr);
+    if (!XB) mapB = mapA;
+    const int cross = XB != nullptr;
     const int nt = ceil_div(n, TILE);
-    const int64_t lower = (int64_t)nt * (nt + 1) / 2;
-    int splits = hessian_splits(n, T, sms);
+    const int64_t tiles = cross ? (int64_t)nt * nt : (int64_t)nt * (nt + 1) / 2;
+    int splits = cross ? hessian_splits_tiles(tiles, T, sms) : hessian_splits(n, T, sms);
     const size_t per = (size_t)n * n * sizeof(float);
     if (splits > 1 && (ws == nullptr || ws_bytes < 2 * per)) splits = 1;
     if (splits > 1 && (size_t)splits * per > ws_bytes) splits = (int)(ws_bytes / per);
@@ -298,13 +328,26 @@ realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void 
     }
     float *part = static_cast<float *>(ws);
     {
-        Launch L("hessian_syrk_tc", s);
-        hess_tc_kernel<<<dim3((unsigned)lower, (unsigned)splits), THREADS, SMEM_BYTES, s>>>(map, n, T, tper, H, part,
-                                                                                       splits == 1, err);
+        Launch L(name, s);
+        hess_tc_kernel<<<dim3((unsigned)tiles, (unsigned)splits), THREADS, SMEM_BYTES, s>>>(
+            mapA, mapB, n, T, tper, out, out2, part, splits == 1, cross, sign, err);
     }
-    REALQ_TRY(check_launch("hessian_syrk_tc"));
-    if (splits > 1) REALQ_TRY(hessian_reduce(s, n, splits, part, H, 0));
+    REALQ_TRY(check_launch(name));
+    if (splits > 1) {
+        REALQ_TRY(hessian_reduce(s, n, splits, part, out, cross ? 1 : 0));
+        if (out2) REALQ_TRY(hessian_reduce(s, n, splits, part, out2, cross ? 1 : 0));
+    }
     return REALQ_OK;
+}
+
+realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
+                               size_t ws_bytes, int sms, float *H2) {
+    return hess_tc_launch(s, n, T, X, nullptr, H, H2, 1.f, err, ws, ws_bytes, sms, "hessian_syrk_tc");
+}
+
+realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms) {
+    return hess_tc_launch(s, n, T, XA, XB, out, nullptr, sign, err, ws, ws_bytes, sms, "hessian_cross_tc");
 }
 
 }  // namespace realq

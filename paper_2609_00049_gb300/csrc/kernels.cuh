@@ -85,7 +85,10 @@ realq_status_t hessian_accumulate(cudaStream_t s, int64_t n, int64_t T, const vo
 realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float *part, float *out, int mode);
 bool hessian_tc_eligible(int64_t n, int64_t T, const void *X);
 realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
-                               size_t ws_bytes, int sms);
+                               size_t ws_bytes, int sms, float *H2 = nullptr);
+realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms);
+int hessian_splits_tiles(int64_t tiles, int64_t T, int sms);
 
 // --------------------------------------------------------------- prepare ---
 size_t prepare_ws_bytes(int64_t n);
