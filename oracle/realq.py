@@ -35,7 +35,7 @@ __all__ = [
     "hessian_sum", "cross_moment_sum", "prepare", "inverse_upper_cholesky",
     "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
     "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
-    "round_bf16", "quantize_activations",
+    "round_bf16", "quantize_activations", "saliency_clip", "weighted_hessian_sum",
 ]
 
 
@@ -251,7 +251,7 @@ def pack_codes(codes: np.ndarray) -> np.ndarray:
 # The sweep: Algorithm 1, inner loops for one linear module.
 # ---------------------------------------------------------------------------
 def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetric=False,
-                damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True):
+                damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True, obs_hessians=None):
     """Quantize W0 column by column with OBS feedback and Block-GD after each block.
 
     bgd: None for the plain column sweep (GPTQ), else a dict with keys
@@ -267,6 +267,13 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     after the block; the block after the last column is skipped (no columns
     remain).  Returns a dict of codes, scale, zero, deq (fp32 values as fp64),
     per-column residuals, tie margins and per-block surrogate values.
+
+    obs_hessians: None (one Hessian for every row), or the row-grouped OBS of
+    Alg. 1 ("for all row-groups g"): a list of N_g pairs (H_g_sum, norm_g).
+    The rows are split into N_g contiguous groups of ceil(m / N_g) rows; group
+    g's OBS step and lazy update use H̄_g = H_g_sum / norm_g (damped and with
+    its own dead channels, as in prepare), while Block-GD keeps the
+    surrogate's plain H̄ = H_sum / T.
     """
     W0 = np.asarray(W0, dtype=np.float64)
     m, n = W0.shape
@@ -279,8 +286,17 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     Dbar = None if D_sum is None else np.asarray(D_sum, dtype=np.float64) / float(T)
 
     W = W0.copy()
-    W[:, dead] = 0.0
-    Hinv = np.linalg.inv(Hd)
+    if obs_hessians is None:
+        groups = [(slice(0, m), Hd, dead)]
+    else:
+        mg = -(-m // len(obs_hessians))
+        groups = []
+        for k, (Hg, normg) in enumerate(obs_hessians):
+            pg = prepare(Hg, normg, damp_frac)
+            groups.append((slice(k * mg, min((k + 1) * mg, m)), pg["Hd"], pg["dead"]))
+    for rows, _, dg in groups:
+        W[rows, dg] = 0.0
+    Hinvs = [np.linalg.inv(Hdg) for _, Hdg, _ in groups]
     ngroups = -(-n // g)
     codes = np.zeros((m, n), dtype=np.int64)
     scale = np.zeros((m, ngroups), dtype=np.float32)
@@ -288,7 +304,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     margin = np.zeros((m, n))
     zmargin = np.zeros((m, ngroups))
     eps_cols = np.zeros((m, n))
-    hinv_diag = np.zeros(n)
+    hinv_diag = np.zeros((len(groups), n))
     block_loss = []
     opt = None
     if bgd is not None:
@@ -303,15 +319,16 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         gi = j // g
         q, dq, mg = quantize(W[:, j], scale[:, gi], zero[:, gi], bits)
         e = W[:, j] - dq                       # residual delta_j of Eq. (gptq_update)
-        d = Hinv[j, j]
         codes[:, j] = q
         margin[:, j] = mg
         eps_cols[:, j] = e
-        hinv_diag[j] = d
-        # Eq. (gptq_update): W[:, j+1:] -= delta_j H^-1[j, j+1:] / [H^-1]_jj
-        W[:, j + 1:] -= np.outer(e / d, Hinv[j, j + 1:])
-        # remove j from the free set: Schur-complement downdate of H^-1
-        Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d
+        for k, ((rows, _, _), Hinv) in enumerate(zip(groups, Hinvs)):
+            d = Hinv[j, j]
+            hinv_diag[k, j] = d
+            # Eq. (gptq_update): W[:, j+1:] -= delta_j H^-1[j, j+1:] / [H^-1]_jj
+            W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])
+            # remove j from the free set: Schur-complement downdate of H^-1
+            Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d
         W[:, j] = dq
 
         be = j + 1
@@ -333,7 +350,8 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
 
     return {
         "codes": codes, "scale": scale, "zero": zero, "deq": W.copy(),
-        "margin": margin, "zero_margin": zmargin, "eps": eps_cols, "hinv_diag": hinv_diag,
+        "margin": margin, "zero_margin": zmargin, "eps": eps_cols,
+        "hinv_diag": hinv_diag[0] if obs_hessians is None else hinv_diag,
         "block_loss": block_loss, "adam_t": 0 if opt is None else opt.t,
         "Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": prep["lam"], "Dbar": Dbar,
     }
@@ -376,3 +394,37 @@ def quantize_activations(X: np.ndarray, bits: int = 4, a_clip: float = 0.9, out_
     if out_bf16:
         xq = round_bf16(xq)
     return q, scale, xq.astype(np.float64)
+
+
+# ---------------------------------------------------------------------------
+# Saliency-weighted grouped Hessian (Sec. 3.3 Eq. saliency_hessian, used by
+# Alg. 1 "for all row-groups g" with N_g = 4; App. "Hessian-side saliency
+# clipping": per-token saliency clipped to the 99th percentile first).
+# Readings: the rows of W form N_g contiguous groups, s[t, g] >= 0 is token
+# t's saliency for group g; the percentile is the nearest-rank one (the
+# smallest saliency value with at least pct of the tokens at or below it),
+# taken per group over the T tokens; H̄_g = H_g / sum_t s'[t, g] (the
+# saliency-weighted mean of x x^T; the OBS step does not depend on the scale).
+# ---------------------------------------------------------------------------
+def saliency_clip(S: np.ndarray, pct: float = 0.99):
+    """Returns (S clipped, per-group thresholds)."""
+    S = np.asarray(S, dtype=np.float64)
+    T = S.shape[0]
+    k = min(max(int(math.ceil(pct * T)) - 1, 0), T - 1)
+    c = np.sort(S, axis=0)[k]
+    return np.minimum(S, c[None, :]), c
+
+
+def weighted_hessian_sum(xhat_chunks: Iterable[np.ndarray], s_chunks: Iterable[np.ndarray]):
+    """H_g = sum_t s[t, g] x̂_t x̂_t^T for every group g, and sum_t s[t, g]."""
+    H, wsum = None, None
+    for c, sc in zip(xhat_chunks, s_chunks):
+        c = np.asarray(c, dtype=np.float64)
+        sc = np.asarray(sc, dtype=np.float64)
+        if H is None:
+            H = np.zeros((sc.shape[1], c.shape[1], c.shape[1]))
+            wsum = np.zeros(sc.shape[1])
+        for g in range(sc.shape[1]):
+            H[g] += (c * sc[:, g:g + 1]).T @ c
+            wsum[g] += sc[:, g].sum()
+    return H, wsum

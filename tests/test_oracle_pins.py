@@ -426,3 +426,93 @@ def test_bf16_rounding_matches_the_input_generator_cast():
     r = np.random.default_rng(6)
     a = (r.standard_normal(10000) * 10 ** r.uniform(-3, 3, 10000)).astype(np.float32)
     assert np.array_equal(oracle.round_bf16(a), synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(a)))
+
+
+# ------------------------------------------ saliency-weighted grouped OBS ---
+def _grouped_case(seed, m=32, n=48, T=400):
+    r = np.random.default_rng(seed)
+    X = r.standard_normal((T, n))
+    X[:, 3] *= 6.0
+    W0 = r.standard_normal((m, n)) * 0.02
+    Z = r.standard_normal((m, 4))
+    F = 0.5 * np.eye(m) + Z @ Z.T / 8
+    return r, X, W0, F
+
+
+def test_grouped_sweep_reduces_to_one_hessian_for_uniform_saliency():
+    r, X, W0, F = _grouped_case(61)
+    H, T = oracle.hessian_sum([X])
+    S = np.full((X.shape[0], 4), 3.0)
+    Hg, wsum = oracle.weighted_hessian_sum([X], [S])
+    np.testing.assert_allclose(Hg, 3.0 * np.broadcast_to(H, Hg.shape), rtol=0, atol=1e-12 * np.abs(Hg).max())
+    bgd = {"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
+    a = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, bgd=bgd, F=F)
+    b = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, bgd=bgd, F=F,
+                           obs_hessians=[(Hg[g], wsum[g]) for g in range(4)])
+    assert np.array_equal(a["codes"], b["codes"])
+    np.testing.assert_allclose(b["deq"], a["deq"], rtol=0, atol=1e-12)
+
+
+def test_grouped_gptq_rows_are_independent_sweeps():
+    # without Block-GD every row group is GPTQ on its own rows with its own H_g
+    r, X, W0, F = _grouped_case(62, m=30)
+    H, T = oracle.hessian_sum([X])
+    S = np.exp(2.0 * r.standard_normal((X.shape[0], 3)))
+    Hg, wsum = oracle.weighted_hessian_sum([X], [S])
+    b = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, obs_hessians=[(Hg[g], wsum[g]) for g in range(3)])
+    for g in range(3):
+        rows = slice(10 * g, 10 * (g + 1))
+        a = oracle.realq_sweep(W0[rows], Hg[g], wsum[g], group_size=16, block_size=16)
+        assert np.array_equal(a["codes"], b["codes"][rows])
+        assert np.array_equal(a["deq"], b["deq"][rows])
+    # and the groups really differ from the unweighted sweep
+    u = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16)
+    assert not np.array_equal(u["codes"], b["codes"])
+
+
+def test_weighted_hessian_exact_on_integers():
+    r = np.random.default_rng(63)
+    X = r.integers(-3, 4, (50, 7)).astype(np.float64)
+    S = r.integers(0, 5, (50, 2)).astype(np.float64)
+    Hg, wsum = oracle.weighted_hessian_sum([X[:20], X[20:]], [S[:20], S[20:]])
+    for g in range(2):
+        ref = np.zeros((7, 7))
+        for t in range(50):
+            for i in range(7):
+                for j in range(7):
+                    ref[i, j] += S[t, g] * X[t, i] * X[t, j]
+        assert np.array_equal(Hg[g], ref)
+        assert wsum[g] == S[:, g].sum()
+
+
+def test_saliency_clip_is_the_nearest_rank_percentile():
+    r = np.random.default_rng(64)
+    S = np.exp(3.0 * r.standard_normal((1000, 4)))
+    S[r.integers(0, 1000, 50), 1] = 7.0                 # ties
+    S[5, 2] = 1e15                                       # an extreme outlier
+    for pct in (0.99, 0.5, 1.0, 1e-9):
+        Sc, c = oracle.saliency_clip(S, pct)
+        for g in range(4):
+            v = S[:, g]
+            cand = [x for x in np.unique(v) if (v <= x).sum() >= pct * len(v)]
+            assert c[g] == min(cand)
+            assert np.array_equal(Sc[:, g], np.minimum(v, c[g]))
+    Sc, c = oracle.saliency_clip(S, 0.99)
+    assert c[2] < 1e15 and Sc[5, 2] == c[2]
+
+
+def test_saliency_clipping_prevents_rank_one_collapse():
+    # App. "Hessian-side saliency clipping": one token with a saliency ~1e12 x
+    # the median makes H_g nearly rank one; clipping at the 99th percentile
+    # restores a well-spread spectrum
+    r = np.random.default_rng(65)
+    X = r.standard_normal((2000, 16))
+    S = np.exp(r.standard_normal((2000, 1)))
+    S[17, 0] = 1e12
+    Hg, _ = oracle.weighted_hessian_sum([X], [S])
+    ev = np.linalg.eigvalsh(Hg[0])
+    assert ev[-1] / ev.sum() > 0.99
+    Sc, _ = oracle.saliency_clip(S, 0.99)
+    Hc, _ = oracle.weighted_hessian_sum([X], [Sc])
+    ev = np.linalg.eigvalsh(Hc[0])
+    assert ev[-1] / ev.sum() < 0.2
