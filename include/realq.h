@@ -181,6 +181,39 @@ realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int6
                                           realq_dtype_t x_dtype, int bits, float a_clip, void *X_q, uint8_t *codes,
                                           float *scale);
 
+/* Saliency-weighted Hessians of the coarse stage (Sec. 3.3 Eq.
+ * saliency_hessian, used by Alg. 1 for every row group g; N_g = 4 in the
+ * paper), and the Hessian-side saliency clipping of the appendix.
+ *
+ * realq_saliency_clip: S is T x n_groups fp32 (row-major: S[t * n_groups + g]
+ * is token t's saliency for row group g, >= 0 and finite).  clip_out[g] is the
+ * nearest-rank pct-percentile of column g over the T tokens (the smallest
+ * value with at least pct * T values at or below it: an input value, bit for
+ * bit); S_out = min(S, clip_out[g]) elementwise (may alias S, may be NULL to
+ * get the thresholds only).  0 < pct <= 1.  Asynchronous; allocates nothing. */
+realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *S, float pct,
+                                   float *S_out, float *clip_out);
+
+/* H_g += sum_t S[t, g] x̂_t x̂_t^T for every group g (H_g: n_groups x n x n
+ * fp32, group g at H_g + g n^2) and wsum[g] += sum_t S[t, g] (fp64), for a
+ * chunk of T_chunk bf16 tokens X_hat (T_chunk x n).  Each product is formed
+ * as bf16(sqrt(s) x_i) bf16(sqrt(s) x_j), within 2^-8 relative of s x_i x_j,
+ * and accumulated in fp32 as realq_hessian_accumulate does.  ws: at least
+ * realq_hessian_weighted_workspace_size(n, T_chunk) bytes, 256-byte aligned;
+ * its first word is the status that realq_workspace_status reads.
+ * Asynchronous. */
+size_t realq_hessian_weighted_workspace_size(int64_t n, int64_t T_chunk);
+realq_status_t realq_hessian_accumulate_weighted(realq_stream_t stream, int64_t n, int64_t T_chunk,
+                                                 const void *X_hat, int n_groups, const float *S, float *H_g,
+                                                 double *wsum, void *ws, size_t ws_bytes);
+
+/* realq_hessian_prepare with a real normaliser: Hbar = H_sum / norm (for a
+ * weighted Hessian, norm = the weight sum; the OBS step does not depend on
+ * it).  Everything else as realq_hessian_prepare. */
+realq_status_t realq_hessian_prepare_scaled(realq_stream_t stream, int64_t n, double norm, float damp_frac,
+                                            const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                            int64_t *fail_col, void *ws, size_t ws_bytes);
+
 /* Dbar = D_sum / T_total (n x n); may alias D_sum.  Asynchronous. */
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum,
                                   float *Dbar);

@@ -20,7 +20,8 @@ __all__ = [
     "RealqError", "QuantCfg", "BgdCfg", "lib", "library_path", "quant_cfg", "bgd_cfg", "workspace",
     "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
     "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
-    "realq_quantize_activations",
+    "realq_quantize_activations", "realq_saliency_clip", "realq_hessian_weighted_workspace_size",
+    "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -80,6 +81,10 @@ _SIGS = {
     "realq_hessian_prepare_noalloc": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64], _int),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
     "realq_quantize_activations": ([_vp, _i64, _i64, _vp, _int, _int, _f32, _vp, _vp, _vp], _int),
+    "realq_saliency_clip": ([_vp, _i64, _int, _vp, _f32, _vp, _vp], _int),
+    "realq_hessian_weighted_workspace_size": ([_i64, _i64], _sz),
+    "realq_hessian_accumulate_weighted": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _sz], _int),
+    "realq_hessian_prepare_scaled": ([_vp, _i64, ctypes.c_double, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
                               ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
                               _i64, _i64, _vp, _sz], _int),
@@ -233,6 +238,51 @@ def realq_quantize_activations(X: torch.Tensor, bits: int = 4, a_clip: float = 0
     _check(lib().realq_quantize_activations(_stream(stream), T, n, _ptr(X), _dtype(X), bits, a_clip, _ptr(X_q),
                                             _ptr(codes), _ptr(scale)))
     return X_q
+
+
+def realq_saliency_clip(S: torch.Tensor, pct: float = 0.99, S_out: Optional[torch.Tensor] = None,
+                        clip_out: Optional[torch.Tensor] = None, stream=None):
+    """Nearest-rank percentile of each saliency column and S clipped to it.
+    Returns (S_out, clip_out); S_out may be S itself."""
+    T, ng = S.shape
+    _need(S, torch.float32, (T, ng), "S")
+    if clip_out is None:
+        clip_out = torch.empty(ng, dtype=torch.float32, device=S.device)
+    if S_out is None:
+        S_out = torch.empty_like(S)
+    _need(S_out, torch.float32, (T, ng), "S_out")
+    _check(lib().realq_saliency_clip(_stream(stream), T, ng, _ptr(S), pct, _ptr(S_out), _ptr(clip_out)))
+    return S_out, clip_out
+
+
+def realq_hessian_weighted_workspace_size(n: int, T_chunk: int) -> int:
+    return int(lib().realq_hessian_weighted_workspace_size(n, T_chunk))
+
+
+def realq_hessian_accumulate_weighted(X_hat: torch.Tensor, S: torch.Tensor, H_g: torch.Tensor, wsum: torch.Tensor,
+                                      ws: torch.Tensor, stream=None):
+    T, n = X_hat.shape
+    ng = S.shape[1]
+    if X_hat.dtype != torch.bfloat16:
+        raise ValueError("X_hat: bf16 activations expected")
+    _need(S, torch.float32, (T, ng), "S")
+    _need(H_g, torch.float32, (ng, n, n), "H_g")
+    _need(wsum, torch.float64, (ng,), "wsum")
+    wp, wb = _ws(ws)
+    _check(lib().realq_hessian_accumulate_weighted(_stream(stream), n, T, _ptr(X_hat), ng, _ptr(S), _ptr(H_g),
+                                                   _ptr(wsum), wp, wb))
+
+
+def realq_hessian_prepare_scaled(H_sum: torch.Tensor, norm: float, damp_frac: float, U_out: torch.Tensor,
+                                 Hbar_out: Optional[torch.Tensor], dead_out: torch.Tensor, ws: torch.Tensor,
+                                 stream=None) -> int:
+    n = H_sum.shape[0]
+    wp, wb = _ws(ws)
+    fc = ctypes.c_int64(-1)
+    _check(lib().realq_hessian_prepare_scaled(_stream(stream), n, float(norm), damp_frac, _ptr(H_sum), _ptr(U_out),
+                                              _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc), wp, wb),
+           fail_col=fc.value)
+    return fc.value
 
 
 def realq_scale_moment(D_sum: torch.Tensor, T_total: int, Dbar: torch.Tensor, stream=None):

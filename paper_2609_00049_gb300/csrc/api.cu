@@ -261,6 +261,44 @@ realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int6
     return act_quant(S(stream), T, n, X, x_dtype, bits, a_clip, X_q, codes, scale);
 }
 
+realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *sal, float pct,
+                                   float *sal_out, float *clip_out) {
+    if (T <= 0 || n_groups <= 0 || !sal || !clip_out) return fail(REALQ_ERR_INVALID_ARG, "saliency_clip: bad argument");
+    if (!(pct > 0.f && pct <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "saliency_clip: 0 < pct <= 1");
+    return saliency_clip(S(stream), T, n_groups, sal, pct, sal_out, clip_out);
+}
+
+size_t realq_hessian_weighted_workspace_size(int64_t n, int64_t T_chunk) {
+    return (n > 0 && T_chunk >= 0) ? weighted_ws_bytes(n, T_chunk) : 0;
+}
+
+realq_status_t realq_hessian_accumulate_weighted(realq_stream_t stream, int64_t n, int64_t T_chunk,
+                                                 const void *X_hat, int n_groups, const float *sal, float *H_g,
+                                                 double *wsum, void *ws, size_t ws_bytes) {
+    if (n <= 0 || T_chunk < 0 || n_groups <= 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate_weighted: bad size");
+    if (T_chunk > 0 && (!X_hat || !sal)) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate_weighted: NULL input");
+    if (!H_g || !wsum || !ws) return fail(REALQ_ERR_INVALID_ARG, "hessian_accumulate_weighted: NULL output or workspace");
+    if (reinterpret_cast<uintptr_t>(ws) % kAlign)
+        return fail(REALQ_ERR_WORKSPACE, "hessian_accumulate_weighted: workspace must be %zu-byte aligned", kAlign);
+    if (ws_bytes < weighted_ws_bytes(n, T_chunk))
+        return fail(REALQ_ERR_WORKSPACE, "hessian_accumulate_weighted: workspace too small");
+    if (T_chunk == 0) return REALQ_OK;
+    return hessian_weighted(S(stream), n, T_chunk, X_hat, n_groups, sal, H_g, wsum, ws, ws_bytes);
+}
+
+realq_status_t realq_hessian_prepare_scaled(realq_stream_t stream, int64_t n, double norm, float damp_frac,
+                                            const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                            int64_t *fail_col, void *ws, size_t ws_bytes) {
+    if (!(norm > 0.0) || !std::isfinite(norm)) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_scaled: norm > 0");
+    if (n <= 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_scaled: n > 0 required");
+    if (!H_sum || !U_out || !dead_out || !fail_col) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_scaled: NULL argument");
+    if ((const void *)U_out == (const void *)H_sum) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_scaled: U_out may not alias H_sum");
+    if (!(damp_frac >= 0.f) || !std::isfinite(damp_frac)) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_scaled: damp_frac >= 0");
+    REALQ_TRY(check_ws(ws, ws_bytes, prepare_ws_bytes(n), "hessian_prepare_scaled"));
+    *fail_col = -1;
+    return prepare(S(stream), n, norm, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col, ws, ws_bytes);
+}
+
 realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_total, const float *D_sum, float *Dbar) {
     if (n <= 0 || T_total <= 0 || !D_sum || !Dbar) return fail(REALQ_ERR_INVALID_ARG, "scale_moment: bad argument");
     return scale_copy(S(stream), n * n, (float)T_total, D_sum, Dbar);

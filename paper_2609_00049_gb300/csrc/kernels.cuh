@@ -76,6 +76,14 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
 realq_status_t act_quant(cudaStream_t s, int64_t T, int64_t n, const void *X, realq_dtype_t dt, int bits, float a_clip,
                          void *Xq, uint8_t *codes, float *scale);
 
+// ------------------------------------------- saliency-weighted Hessians ---
+size_t saliency_clip_ws_bytes();
+realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, float pct, float *S_out,
+                             float *clip_out);
+size_t weighted_ws_bytes(int64_t n, int64_t T);
+realq_status_t hessian_weighted(cudaStream_t s, int64_t n, int64_t T, const void *X, int ng, const float *S,
+                                float *Hg, double *wsum, void *ws, size_t ws_bytes);
+
 // --------------------------------------------------------------- Hessian ---
 int hessian_splits(int64_t n, int64_t T, int num_sms);
 int num_sms();
@@ -92,7 +100,7 @@ int hessian_splits_tiles(int64_t tiles, int64_t T, int sms);
 
 // --------------------------------------------------------------- prepare ---
 size_t prepare_ws_bytes(int64_t n);
-realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes);
 realq_status_t scale_copy(cudaStream_t s, int64_t count, float mul, const float *in, float *out);
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,

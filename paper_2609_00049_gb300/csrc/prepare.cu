@@ -300,7 +300,7 @@ realq_status_t noalloc_scratch(void **out) {
 
 size_t prepare_ws_bytes(int64_t n) { return prepare_bytes_split(n, KSPLIT_MAX); }
 
-realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                             uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap);
 
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
@@ -308,7 +308,7 @@ realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp,
     void *scratch = nullptr;
     REALQ_TRY(noalloc_scratch(&scratch));
     // single stream: this entry point creates no stream or event
-    return prepare_impl(s, n, T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes, false);
+    return prepare_impl(s, n, (double)T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes, false);
 }
 
 // Auxiliary stream of the calling thread (and its events) for the U row
@@ -349,12 +349,12 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
     return REALQ_OK;
 }
 
-realq_status_t prepare(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes) {
-    return prepare_impl(s, n, T, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true);
+    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true);
 }
 
-realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
+realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                             uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap) {
     Carve cv(ws);
     int *status = cv.take<int>(1);
@@ -369,7 +369,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, int64_t T, float damp, co
     const int64_t tot = n * n;
     {
         Launch L("prepare_init", s);
-        prep_init_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(n, (float)T, H, Hbar, U, dead);
+        prep_init_kernel<<<(unsigned)((tot + 255) / 256), 256, 0, s>>>(n, (float)norm, H, Hbar, U, dead);
     }
     REALQ_TRY(check_launch("prepare_init"));
     {

@@ -436,3 +436,87 @@ def test_block_scheduler_activation_aware():
         print(f"\nblock W4A4 {nm}: {rep} scale_within_1e-5={frac:.5f}")
         assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (nm, rep)
         assert s_unexpl == 0
+
+
+# ------------------------------------------ saliency-weighted Hessians ---
+@pytest.mark.parametrize("T,pct", [(4096, 0.99), (999, 0.99), (1000, 0.5), (77, 1.0), (1, 0.99)])
+def test_saliency_clip_bit_exact(T, pct):
+    r = synth.rng(51, "saliency-clip", T)
+    S = np.exp(3.0 * r.standard_normal((T, 4))).astype(np.float32)
+    S[r.integers(0, T, max(1, T // 20)), 1] = 7.0
+    S[0, 2] = 1e30
+    S[T // 2, 3] = 0.0
+    Sc_or, c_or = oracle.saliency_clip(S.astype(np.float64), pct)
+    Sd = dev(S)
+    Sc, c = rq.realq_saliency_clip(Sd, pct)
+    assert np.array_equal(c.cpu().numpy().astype(np.float64), c_or)
+    assert np.array_equal(Sc.cpu().numpy().astype(np.float64), Sc_or)
+    rq.realq_saliency_clip(Sd, pct, S_out=Sd)          # in place
+    assert torch.equal(Sd, Sc)
+
+
+def _weighted_gpu(Xb, S, n, ng, chunks=(0,)):
+    Hg = torch.zeros(ng, n, n, device="cuda")
+    wsum = torch.zeros(ng, dtype=torch.float64, device="cuda")
+    T = Xb.shape[0]
+    bounds = list(chunks) + [T]
+    ws = rq.workspace(rq.realq_hessian_weighted_workspace_size(n, max(b - a for a, b in zip(bounds[:-1], bounds[1:]))))
+    for a, b in zip(bounds[:-1], bounds[1:]):
+        rq.realq_hessian_accumulate_weighted(Xb[a:b], S[a:b], Hg, wsum, ws)
+    rq.realq_workspace_status(ws)
+    return Hg, wsum
+
+
+def test_weighted_hessian_exact_on_perfect_squares():
+    # sqrt(s) x is an integer that bf16 holds exactly, every product and partial
+    # sum is an integer below 2^24: the tensor-core result is exact
+    r = synth.rng(52, "weighted-exact")
+    for n, T in ((128, 3000), (256, 5000), (96, 777)):
+        X = r.integers(-7, 8, (T, n)).astype(np.float64)
+        S = r.choice([0.0, 1.0, 4.0, 9.0, 16.0], size=(T, 4))
+        Hg, wsum = _weighted_gpu(bf16_dev(synth.f32_to_bf16_bits(X)), dev(S), n, 4, chunks=(0, T // 3))
+        Href, wref = oracle.weighted_hessian_sum([X], [S])
+        assert np.array_equal(Hg.cpu().numpy().astype(np.float64), Href), (n, T)
+        assert np.array_equal(wsum.cpu().numpy(), wref)
+
+
+def test_weighted_hessian_within_two_bf16_roundings():
+    r = synth.rng(53, "weighted-real")
+    n, T = 256, 20000
+    X = synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(r.standard_normal((T, n)))).astype(np.float64)
+    X[:, 7] *= 15.0
+    S, _ = oracle.saliency_clip(np.exp(2.0 * r.standard_normal((T, 4))), 0.99)
+    S = S.astype(np.float32).astype(np.float64)
+    Hg, wsum = _weighted_gpu(bf16_dev(synth.f32_to_bf16_bits(X)), dev(S), n, 4)
+    Href, wref = oracle.weighted_hessian_sum([X], [S])
+    A = np.abs(X)
+    for g in range(4):
+        absum = (A * S[:, g:g + 1]).T @ A                  # sum_t s |x_i x_j|
+        d = np.sqrt(np.diag(Href[g]))
+        bound = 2.0 ** -8 * absum + 2e-6 * np.sqrt(T) * np.outer(d, d)
+        err = np.abs(Hg[g].cpu().numpy() - Href[g])
+        assert np.all(err <= bound), (g, (err / bound).max())
+        print(f"\ngroup {g}: max error / bound = {(err / bound).max():.3e}")
+    np.testing.assert_allclose(wsum.cpu().numpy(), wref, rtol=1e-12)
+
+
+def test_prepare_scaled_matches_oracle():
+    # integer activations and perfect-square weights: the weighted Hessians are
+    # exact on both sides, so this compares the scaled preparation alone
+    r = synth.rng(54, "prepare-scaled")
+    n, T = 192, 6000
+    X = r.integers(-7, 8, (T, n)).astype(np.float64)
+    X[:, 5] *= 3.0
+    S = r.choice([1.0, 4.0, 9.0, 16.0], size=(T, 2), p=[0.7, 0.2, 0.07, 0.03])
+    Hg, wsum = _weighted_gpu(bf16_dev(synth.f32_to_bf16_bits(X)), dev(S), n, 2)
+    Href, wref = oracle.weighted_hessian_sum([X], [S])
+    ws = rq.workspace(rq.realq_prepare_workspace_size(n))
+    for g in range(2):
+        U = torch.empty(n, n, device="cuda")
+        Hb = torch.empty(n, n, device="cuda")
+        dead = torch.empty(n, dtype=torch.uint8, device="cuda")
+        rq.realq_hessian_prepare_scaled(Hg[g], float(wsum[g].item()), 0.01, U, Hb, dead, ws)
+        ref = oracle.prepare(Href[g], wref[g], 0.01)
+        Uref = oracle.inverse_upper_cholesky(ref["Hd"])
+        assert np.abs(U.cpu().numpy() - Uref).max() <= 2e-4 * np.abs(Uref).max()
+        np.testing.assert_allclose(Hb.cpu().numpy(), ref["Hbar"], rtol=1e-5, atol=1e-6 * np.abs(ref["Hbar"]).max())
