@@ -402,15 +402,18 @@ def quantize_activations(X: np.ndarray, bits: int = 4, a_clip: float = 0.9, out_
 # clipping": per-token saliency clipped to the 99th percentile first).
 # Readings: the rows of W form N_g contiguous groups, s[t, g] >= 0 is token
 # t's saliency for group g; the percentile is the nearest-rank one (the
-# smallest saliency value with at least pct of the tokens at or below it),
-# taken per group over the T tokens; H̄_g = H_g / sum_t s'[t, g] (the
+# smallest saliency value with at least pct of the tokens at or below it,
+# pct as a single-precision value), taken per group over the T tokens; H̄_g = H_g / sum_t s'[t, g] (the
 # saliency-weighted mean of x x^T; the OBS step does not depend on the scale).
 # ---------------------------------------------------------------------------
 def saliency_clip(S: np.ndarray, pct: float = 0.99):
-    """Returns (S clipped, per-group thresholds)."""
+    """Returns (S clipped, per-group thresholds).  pct is the single-precision
+    value the interface carries (0.99 -> 0.99000000953...); the rank
+    ceil(pct T) - 1 is evaluated exactly from it."""
     S = np.asarray(S, dtype=np.float64)
     T = S.shape[0]
-    k = min(max(int(math.ceil(pct * T)) - 1, 0), T - 1)
+    p32 = float(np.float32(pct))
+    k = min(max(int(math.ceil(p32 * T)) - 1, 0), T - 1)
     c = np.sort(S, axis=0)[k]
     return np.minimum(S, c[None, :]), c
 

@@ -492,13 +492,16 @@ def test_saliency_clip_is_the_nearest_rank_percentile():
     S[5, 2] = 1e15                                       # an extreme outlier
     for pct in (0.99, 0.5, 1.0, 1e-9):
         Sc, c = oracle.saliency_clip(S, pct)
+        p32 = float(np.float32(pct))
         for g in range(4):
             v = S[:, g]
-            cand = [x for x in np.unique(v) if (v <= x).sum() >= pct * len(v)]
+            cand = [x for x in np.unique(v) if (v <= x).sum() >= p32 * len(v)]
             assert c[g] == min(cand)
             assert np.array_equal(Sc[:, g], np.minimum(v, c[g]))
     Sc, c = oracle.saliency_clip(S, 0.99)
     assert c[2] < 1e15 and Sc[5, 2] == c[2]
+    # the rank comes from the single-precision pct: 0.99f * 8000 = 7920.00008
+    assert oracle.saliency_clip(np.arange(8000.0)[:, None], 0.99)[1][0] == 7920.0
 
 
 def test_saliency_clipping_prevents_rank_one_collapse():
