@@ -196,9 +196,11 @@ realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_group
 
 /* H_g += sum_t S[t, g] x̂_t x̂_t^T for every group g (H_g: n_groups x n x n
  * fp32, group g at H_g + g n^2) and wsum[g] += sum_t S[t, g] (fp64), for a
- * chunk of T_chunk bf16 tokens X_hat (T_chunk x n).  Each product is formed
- * as bf16(sqrt(s) x_i) bf16(sqrt(s) x_j), within 2^-8 relative of s x_i x_j,
- * and accumulated in fp32 as realq_hessian_accumulate does.  ws: at least
+ * chunk of T_chunk bf16 tokens X_hat (T_chunk x n; n a multiple of 8, at
+ * least 64).  Each product is formed as x_i (s x_j) with s x_j split into two
+ * bf16 parts, within 2^-17 relative of s x_i x_j, and accumulated in fp32 as
+ * realq_hessian_accumulate does (both triangles are computed; prepare reads
+ * the upper one).  ws: at least
  * realq_hessian_weighted_workspace_size(n, T_chunk) bytes, 256-byte aligned;
  * its first word is the status that realq_workspace_status reads.
  * Asynchronous. */
@@ -262,6 +264,30 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
                                     void *W_deq, realq_dtype_t deq_dtype,
                                     int64_t block_begin, int64_t block_end,
                                     void *ws, size_t ws_bytes);
+
+/* The sweep with a row-grouped OBS (Alg. 1: "for all row-groups g"; the
+ * saliency-weighted Hessians of Sec. 3.3 Eq. saliency_hessian): the rows of W
+ * form n_row_groups contiguous groups of ceil(m / n_row_groups) rows, and
+ * group g runs the OBS step and the lazy update against its own factor
+ * (U_g + g n^2, from realq_hessian_prepare_scaled of H_g) with its own dead
+ * channels (dead_g + g n).  Block-GD still descends the layer surrogate with
+ * the plain Hbar for all rows jointly; it needs Hbar_g (the groups' undamped
+ * H̄_g = H_g / weight sum, n_row_groups x n x n) and, with row groups, m and
+ * n multiples of 4 and at least 32 (REALQ_ERR_UNSUPPORTED otherwise).
+ * Everything else (outputs, state, workspace rules, resume) as
+ * realq_quantize_layer; the workspace comes from
+ * realq_quantize_grouped_workspace_size. */
+size_t realq_quantize_grouped_workspace_size(int64_t m, int64_t n, int n_row_groups, const realq_quant_cfg_t *qcfg,
+                                             const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar);
+realq_status_t realq_quantize_layer_grouped(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                            realq_dtype_t w_dtype, int n_row_groups, const float *U_g,
+                                            const float *Hbar_g, const uint8_t *dead_g, const float *Hbar,
+                                            const float *Dbar, const realq_quant_cfg_t *qcfg,
+                                            const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                            float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                            int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero,
+                                            void *W_deq, realq_dtype_t deq_dtype, int64_t block_begin,
+                                            int64_t block_end, void *ws, size_t ws_bytes);
 size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg_t *qcfg,
                                      const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar);
 

@@ -21,7 +21,8 @@ __all__ = [
     "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
     "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
     "realq_quantize_activations", "realq_saliency_clip", "realq_hessian_weighted_workspace_size",
-    "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled",
+    "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled", "realq_quantize_layer_grouped",
+    "realq_quantize_grouped_workspace_size",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -85,6 +86,11 @@ _SIGS = {
     "realq_hessian_weighted_workspace_size": ([_i64, _i64], _sz),
     "realq_hessian_accumulate_weighted": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _sz], _int),
     "realq_hessian_prepare_scaled": ([_vp, _i64, ctypes.c_double, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
+    "realq_quantize_grouped_workspace_size": ([_i64, _i64, _int, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
+                                               _int, _int], _sz),
+    "realq_quantize_layer_grouped": ([_vp, _i64, _i64, _vp, _int, _int, _vp, _vp, _vp, _vp, _vp,
+                                      ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp,
+                                      _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
                               ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
                               _i64, _i64, _vp, _sz], _int),
@@ -156,10 +162,12 @@ def _need(t, dtype, shape, name):
 
 
 def workspace(nbytes: int, device=None) -> Optional[torch.Tensor]:
-    """Caller-owned workspace buffer (torch allocations are >= 256-byte aligned)."""
+    """Caller-owned workspace buffer (torch allocations are >= 256-byte aligned).
+    Zeroed: its first word is the status that the kernels accumulate into and
+    realq_workspace_status reads and clears."""
     if nbytes == 0:
         return None
-    return torch.empty(int(nbytes), dtype=torch.uint8, device=device or "cuda")
+    return torch.zeros(int(nbytes), dtype=torch.uint8, device=device or "cuda")
 
 
 def _ws(ws):
@@ -321,6 +329,45 @@ def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch
         ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
         _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
         _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
+    return t.value
+
+
+def realq_quantize_grouped_workspace_size(m: int, n: int, n_row_groups: int, qcfg: QuantCfg,
+                                          bcfg: Optional[BgdCfg] = None, has_F_next: bool = False,
+                                          has_Dbar: bool = False) -> int:
+    return int(lib().realq_quantize_grouped_workspace_size(m, n, n_row_groups, ctypes.byref(qcfg),
+                                                           ctypes.byref(bcfg) if bcfg is not None else None,
+                                                           int(has_F_next), int(has_Dbar)))
+
+
+def realq_quantize_layer_grouped(W0: torch.Tensor, U_g: torch.Tensor, Hbar_g: Optional[torch.Tensor],
+                                 dead_g: torch.Tensor, Hbar: Optional[torch.Tensor], qcfg: QuantCfg,
+                                 W_work: torch.Tensor, codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *,
+                                 Dbar=None, bcfg: Optional[BgdCfg] = None, F=None, F_next=None, adam_m=None,
+                                 adam_v=None, bgd_disp=None, adam_t: int = 0, W_deq=None, block_begin: int = 0,
+                                 block_end: Optional[int] = None, ws=None, stream=None) -> int:
+    """The sweep with row groups, group g against U_g[g]; returns the Adam step counter."""
+    m, n = W0.shape
+    ng = U_g.shape[0]
+    nb = -(-n // qcfg.block_size)
+    if block_end is None:
+        block_end = nb
+    _need(U_g, torch.float32, (ng, n, n), "U_g")
+    _need(Hbar_g, torch.float32, (ng, n, n), "Hbar_g")
+    _need(dead_g, torch.uint8, (ng, n), "dead_g")
+    _need(W_work, torch.float32, (m, n), "W_work")
+    _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
+    _need(adam_m, torch.float32, (m, n), "adam_m")
+    _need(adam_v, torch.float32, (m, n), "adam_v")
+    _need(bgd_disp, torch.float32, (m, n), "bgd_disp")
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    _check(lib().realq_quantize_layer_grouped(
+        _stream(stream), m, n, _ptr(W0), _dtype(W0), ng, _ptr(U_g), _ptr(Hbar_g), _ptr(dead_g), _ptr(Hbar),
+        _ptr(Dbar), ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
+        _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale),
+        _ptr(zero), _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end),
+        wp, wb))
     return t.value
 
 

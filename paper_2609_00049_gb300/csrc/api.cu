@@ -312,38 +312,50 @@ size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg
     return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, has_Dbar);
 }
 
-realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
+static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
+                                    int grouped, int rgroups, const float *Ug, const float *Hbar_g,
+                                    const uint8_t *dead_g,
                                     const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
                                     const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg, const float *F,
                                     const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
-                                    int64_t *adam_t,
-                                    uint8_t *codes, float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
-                                    int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
-    if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: m, n must be > 0");
-    if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: m, n too large");
-    if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: bad dtype");
+                                    int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                    realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
+                                    size_t ws_bytes, const char *who) {
+    if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n must be > 0", who);
+    if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n too large", who);
+    if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "%s: bad dtype", who);
     if (!W0 || !U || !W_work || !codes || !scale || !zero)
-        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: NULL W0, U, W_work, codes, scale or zero");
+        return fail(REALQ_ERR_INVALID_ARG, "%s: NULL W0, U, W_work, codes, scale or zero", who);
     REALQ_TRY(check_qcfg(qcfg, n));
     REALQ_TRY(check_bcfg(bcfg));
     const int bgd = bcfg && bcfg->steps_per_block > 0;
     if (bgd) {
         if (!Hbar || !F || !adam_t || !bgd_disp)
-            return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Block-GD needs Hbar, F, bgd_disp and adam_t");
+            return fail(REALQ_ERR_INVALID_ARG, "%s: Block-GD needs Hbar, F, bgd_disp and adam_t", who);
         if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
-            return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: Adam needs adam_m and adam_v");
+            return fail(REALQ_ERR_INVALID_ARG, "%s: Adam needs adam_m and adam_v", who);
+        if (grouped && !(qcfg->block_size > 0 && tc_gemm_eligible(m, n)))
+            return fail(REALQ_ERR_UNSUPPORTED,
+                        "%s: Block-GD with row groups needs m and n multiples of 4 and at least 32", who);
     }
     const int64_t nb = (n + qcfg->block_size - 1) / qcfg->block_size;
     if (block_begin < 0 || block_end > nb || block_begin > block_end)
-        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer: block range [%lld, %lld) outside [0, %lld)",
+        return fail(REALQ_ERR_INVALID_ARG, "%s: block range [%lld, %lld) outside [0, %lld)", who,
                     (long long)block_begin, (long long)block_end, (long long)nb);
     const int has_fn = bgd && F_next != nullptr;
     const int has_db = bgd && Dbar != nullptr;
-    REALQ_TRY(check_ws(ws, ws_bytes, sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db), "quantize_layer"));
+    REALQ_TRY(check_ws(ws, ws_bytes,
+                       sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db, grouped ? rgroups : 0), who));
 
     SweepPlan p{};
     p.m = m; p.n = n; p.W0 = W0; p.w_dtype = w_dtype;
     p.U = U; p.Hbar = Hbar; p.Dbar = has_db ? Dbar : nullptr; p.dead = dead;
+    p.rgroups = grouped ? rgroups : 1;
+    p.grouped = grouped;
+    p.rg_rows = (m + p.rgroups - 1) / p.rgroups;
+    p.Ug = grouped ? Ug : U;
+    p.Hbar_g = grouped ? Hbar_g : nullptr;
+    p.dead_g = grouped ? dead_g : nullptr;
     p.bits = qcfg->bits; p.block = qcfg->block_size; p.sym = qcfg->symmetric;
     p.group = effective_group(qcfg, n);
     p.ngroups = (int)((n + p.group - 1) / p.group);
@@ -363,6 +375,44 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
     REALQ_TRY(sweep_prologue_r0(s, p, block_begin == 0));
     for (int64_t b = block_begin; b < block_end; ++b) REALQ_TRY(sweep_block(s, p, b));
     return REALQ_OK;
+}
+
+realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
+                                    const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
+                                    const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg, const float *F,
+                                    const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                    int64_t *adam_t,
+                                    uint8_t *codes, float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
+                                    int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
+    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, U, Hbar, Dbar, dead, qcfg, bcfg, F,
+                         F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq, deq_dtype,
+                         block_begin, block_end, ws, ws_bytes, "quantize_layer");
+}
+
+size_t realq_quantize_grouped_workspace_size(int64_t m, int64_t n, int n_row_groups, const realq_quant_cfg_t *qcfg,
+                                             const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar) {
+    if (m <= 0 || n <= 0 || !qcfg || n_row_groups <= 0) return 0;
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, has_Dbar, n_row_groups);
+}
+
+realq_status_t realq_quantize_layer_grouped(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                            realq_dtype_t w_dtype, int n_row_groups, const float *U_g,
+                                            const float *Hbar_g, const uint8_t *dead_g, const float *Hbar,
+                                            const float *Dbar, const realq_quant_cfg_t *qcfg,
+                                            const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                            float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                            int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero,
+                                            void *W_deq, realq_dtype_t deq_dtype, int64_t block_begin,
+                                            int64_t block_end, void *ws, size_t ws_bytes) {
+    if (n_row_groups <= 0 || (int64_t)n_row_groups > m)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_grouped: 1 <= n_row_groups <= m required");
+    if (!U_g || !dead_g) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_grouped: NULL U_g or dead_g");
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    if (bgd && !Hbar_g) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_grouped: Block-GD needs Hbar_g");
+    return quantize_impl(stream, m, n, W0, w_dtype, 1, n_row_groups, U_g, Hbar_g, dead_g, U_g, Hbar, Dbar, dead_g, qcfg,
+                         bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq,
+                         deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_grouped");
 }
 
 // ---------------------------------------------------------------- BGD -----

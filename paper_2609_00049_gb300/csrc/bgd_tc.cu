@@ -23,6 +23,12 @@
 //   TC_ADAM   g = acc: one Adam (or SGD) step on W[:, col0 + j], updating the
 //             moments and the displacement, and writing the step's hi / lo
 //             planes for the next M update
+//   TC_ACCUM  M += acc (the running product of one row group)
+//   TC_BGD_PG the gradient factor of a row group whose OBS used its own
+//             H̄_g:  p = M + lambda_g (A_disp - (W - W0)) - acc (+ W0 Dbar),
+//             acc = ΔW (H̄_g - H̄); written like TC_BGD_P
+// The A operand starts at row a_row0 of its planes (a row group), and the
+// epilogue pointers are offset to that row by the caller.
 #include "kernels.cuh"
 #include "tc.cuh"
 
@@ -56,6 +62,18 @@ __device__ __forceinline__ float bgd_p_value(const TcEpi &e, int64_t i, int64_t 
     return p;
 }
 
+// TC_BGD_PG: p = M + lambda (A_disp - (W - W0)) - acc (+ W0 Dbar), 0 on dead channels
+__device__ __forceinline__ float bgd_pg_value(const TcEpi &e, int64_t i, int64_t j, float v) {
+    const int64_t col = e.col0 + j;
+    const int64_t w = i * e.ldw + col;
+    const float w0 = e.w0_bf16 ? __bfloat162float(static_cast<const __nv_bfloat16 *>(e.W0)[w])
+                               : static_cast<const float *>(e.W0)[w];
+    float p = e.M[w] - v + (*e.lam) * (e.Ad[w] - (e.W[w] - w0));
+    if (e.R0) p += e.R0[w];
+    if (e.dead && e.dead[col]) p = 0.f;
+    return p;
+}
+
 __device__ __forceinline__ float4 ld4(const float *p) { return *reinterpret_cast<const float4 *>(p); }
 __device__ __forceinline__ void st4(float *p, float4 v) { *reinterpret_cast<float4 *>(p) = v; }
 __device__ __forceinline__ float4 ld4_w0(const TcEpi &e, int64_t w) {
@@ -67,9 +85,9 @@ __device__ __forceinline__ float4 ld4_w0(const TcEpi &e, int64_t w) {
     return ld4(static_cast<const float *>(e.W0) + w);
 }
 
-// Gradient factor for 4 rows x 4 columns (rows gi0..gi0+3 all < M, as M is a
-// multiple of 4; columns gj..gj+3 all < N); t points at the tile entry of row
-// 0, column 0 of the 4x4 patch, pitch tp.  All loads are issued first.
+// Gradient factor for 4 rows x 4 columns (rows gi0..gi0+3 and columns
+// gj..gj+3 all inside the output); t points at the tile entry of row 0,
+// column 0 of the 4x4 patch, pitch tp.  All loads are issued first.
 __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t M, int64_t gj, float *t, int tp) {
     const int64_t col = e.col0 + gj;
     float4 a[4], w[4], w0[4], r0[4], mp[4];
@@ -95,6 +113,46 @@ __device__ __forceinline__ void bgd_p_rows4(const TcEpi &e, int64_t gi0, int64_t
         tr[1] = dd.y ? 0.f : tr[1] + lam * (a[u].y - (w[u].y - w0[u].y)) + r0[u].y;
         tr[2] = dd.z ? 0.f : tr[2] + lam * (a[u].z - (w[u].z - w0[u].z)) + r0[u].z;
         tr[3] = dd.w ? 0.f : tr[3] + lam * (a[u].w - (w[u].w - w0[u].w)) + r0[u].w;
+    }
+}
+
+// TC_BGD_PG for 4 rows x 4 columns (same shape rules as bgd_p_rows4).
+__device__ __forceinline__ void bgd_pg_rows4(const TcEpi &e, int64_t gi0, int64_t gj, float *t, int tp) {
+    const int64_t col = e.col0 + gj;
+    float4 a[4], w[4], w0[4], r0[4], mp[4];
+    uchar4 dd = make_uchar4(0, 0, 0, 0);
+    if (e.dead) dd = *reinterpret_cast<const uchar4 *>(e.dead + col);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const int64_t wi = (gi0 + u) * e.ldw + col;
+        mp[u] = ld4(e.M + wi);
+        a[u] = ld4(e.Ad + wi);
+        w[u] = ld4(e.W + wi);
+        w0[u] = ld4_w0(e, wi);
+        r0[u] = e.R0 ? ld4(e.R0 + wi) : make_float4(0.f, 0.f, 0.f, 0.f);
+    }
+    const float lam = *e.lam;
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        float *tr = t + u * tp;
+        tr[0] = dd.x ? 0.f : mp[u].x - tr[0] + lam * (a[u].x - (w[u].x - w0[u].x)) + r0[u].x;
+        tr[1] = dd.y ? 0.f : mp[u].y - tr[1] + lam * (a[u].y - (w[u].y - w0[u].y)) + r0[u].y;
+        tr[2] = dd.z ? 0.f : mp[u].z - tr[2] + lam * (a[u].z - (w[u].z - w0[u].z)) + r0[u].z;
+        tr[3] = dd.w ? 0.f : mp[u].w - tr[3] + lam * (a[u].w - (w[u].w - w0[u].w)) + r0[u].w;
+    }
+}
+
+// TC_ACCUM for 4 rows x 4 columns: M += acc
+__device__ __forceinline__ void accum_rows4(const TcEpi &e, int64_t gi0, int64_t gj, const float *t, int tp) {
+    const int64_t col = e.col0 + gj;
+    float4 mp[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) mp[u] = ld4(e.M + (gi0 + u) * e.ldw + col);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const float *tr = t + u * tp;
+        st4(e.M + (gi0 + u) * e.ldw + col,
+            make_float4(mp[u].x + tr[0], mp[u].y + tr[1], mp[u].z + tr[2], mp[u].w + tr[3]));
     }
 }
 
@@ -146,6 +204,10 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
         e.C[i * e.ldc + j] = v;
         return;
     }
+    if (e.mode == TC_ACCUM) {
+        e.M[i * e.ldw + e.col0 + j] += v;
+        return;
+    }
     const int64_t col = e.col0 + j;
     const int64_t w = i * e.ldw + col;
     // TC_ADAM
@@ -168,7 +230,7 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
 
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
-                       const TcEpi e, int *err) {
+                       int a_row0, const TcEpi e, int *err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -214,8 +276,8 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
             const int x = k_off + it * KS;
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
-            tc::tma_load_2d(base, &maps.a_hi, fb, x, (int)i0);
-            tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, (int)i0);
+            tc::tma_load_2d(base, &maps.a_hi, fb, x, a_row0 + (int)i0);
+            tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, a_row0 + (int)i0);
             tc::tma_load_2d(base + 2 * PLANE, &maps.b_hi, fb, x, b_row0 + (int)j0);
             tc::tma_load_2d(base + 3 * PLANE, &maps.b_lo, fb, x, b_row0 + (int)j0);
         }
@@ -288,10 +350,14 @@ __global__ void __launch_bounds__(THREADS, 1)
         const int64_t gj = j0 + cc;
         const bool vec = e.mode != TC_STORE && gj + 3 < N;
         for (int rb = warp * RPW; rb < warp * RPW + RPW; rb += 4) {
-            if (vec) {
-                if (i0 + rb >= M) break;
+            if (i0 + rb >= M) break;
+            // a batch of 4 rows runs vectorized when all 4 exist (M need not be
+            // a multiple of 4 for a row group)
+            if (vec && i0 + rb + 3 < M) {
                 if (e.mode == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
-                else bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                else if (e.mode == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                else if (e.mode == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
+                else accum_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
             } else {
                 for (int u = 0; u < 4; ++u) {
                     const int rr = rb + u;
@@ -301,6 +367,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                         if (gj + q >= N) break;
                         float &t = T[rr * TP + cc + q];
                         if (e.mode == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
+                        else if (e.mode == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
                         else epi_apply(e, gi, gj + q, t);
                     }
                 }
@@ -308,7 +375,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
     }
     __syncthreads();
-    if (good && e.mode == TC_BGD_P) {
+    if (good && (e.mode == TC_BGD_P || e.mode == TC_BGD_PG)) {
         // columns of the tile, lanes over rows: P^T rows are contiguous
         constexpr int CPW = TB / (THREADS / 32);   // tile columns per warp
         for (int cc = warp * CPW; cc < warp * CPW + CPW; ++cc) {
@@ -340,7 +407,31 @@ __global__ void split_kernel(int64_t count, const float *x, const float *y, floa
     lo[i] = v - h;
 }
 
+// hi / lo planes of x - y (y fp32 or bf16)
+template <typename TY>
+__global__ void split_diff_kernel(int64_t count, const float *x, const TY *y, float *hi, float *lo) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= count) return;
+    const float v = x[i] - load_as_float(y, i);
+    const float h = tc::tf32_hi(v);
+    hi[i] = h;
+    lo[i] = v - h;
+}
+
 }  // namespace
+
+template <typename TY>
+realq_status_t tc_split_diff(cudaStream_t s, int64_t count, const float *x, const TY *y, float *hi, float *lo) {
+    if (count <= 0) return REALQ_OK;
+    {
+        Launch L("tf32_split", s);
+        split_diff_kernel<<<(unsigned)((count + 255) / 256), 256, 0, s>>>(count, x, y, hi, lo);
+    }
+    return check_launch("tf32_split");
+}
+template realq_status_t tc_split_diff<float>(cudaStream_t, int64_t, const float *, const float *, float *, float *);
+template realq_status_t tc_split_diff<__nv_bfloat16>(cudaStream_t, int64_t, const float *, const __nv_bfloat16 *,
+                                                     float *, float *);
 
 bool tc_gemm_eligible(int64_t m, int64_t n) {
     return m % 4 == 0 && n % 4 == 0 && m >= 32 && n >= 32 && m < (1ll << 31) && n < (1ll << 31);
@@ -373,7 +464,7 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
 }
 
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name) {
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0) {
     if (M <= 0 || N <= 0) return REALQ_OK;
     if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
     static bool configured = false;
@@ -385,7 +476,7 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     {
         Launch L(name, s);
         gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB)), THREADS, SMEM, s>>>(
-            m, M, N, K, k_off, b_row0, e, err);
+            m, M, N, K, k_off, b_row0, a_row0, e, err);
     }
     return check_launch(name);
 }

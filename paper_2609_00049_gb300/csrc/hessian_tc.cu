@@ -39,7 +39,7 @@ namespace {
 constexpr int TILE = 128;
 constexpr int KSTAGE = 64;                       // tokens per pipeline stage
 constexpr int STAGES = 6;
-constexpr int CHUNK_STAGES = 16;                 // 1024 tokens per TMEM accumulator pass
+constexpr int CHUNK_STAGES = 16;                 // default: 1024 tokens per TMEM accumulator pass
 constexpr int THREADS = 192;
 constexpr int OP_BYTES = TILE * KSTAGE * 2;      // one 128 x 64 bf16 operand tile
 constexpr int BOX_BYTES = 64 * KSTAGE * 2;       // one TMA box (64 channels x 64 tokens)
@@ -59,7 +59,7 @@ __device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
 __global__ void __launch_bounds__(THREADS, 1)
     hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmapB, int64_t n,
                    int64_t T, int64_t tper, float *H, float *H2, float *part, int direct, int cross, float sign,
-                   int *err) {
+                   int chunk_stages, int *err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -83,7 +83,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     const int64_t t_begin = (int64_t)blockIdx.y * tper;
     const int64_t t_end = min(T, t_begin + tper);
     const int nk = t_end > t_begin ? (int)((t_end - t_begin + KSTAGE - 1) / KSTAGE) : 0;
-    const int nch = (nk + CHUNK_STAGES - 1) / CHUNK_STAGES;
+    const int nch = (nk + chunk_stages - 1) / chunk_stages;
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -152,8 +152,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 }
                 tc::fence_after_sync();
                 const uint32_t d = tmem + (uint32_t)(b * TILE);
-                const int it_end = min(nk, (c + 1) * CHUNK_STAGES);
-                for (int it = c * CHUNK_STAGES; it < it_end; ++it) {
+                const int it_end = min(nk, (c + 1) * chunk_stages);
+                for (int it = c * chunk_stages; it < it_end; ++it) {
                     const int s = it % STAGES;
                     const uint32_t r = (uint32_t)(it / STAGES);
                     if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
@@ -163,7 +163,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     tc::fence_after_sync();
                     const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
                     const uint32_t bop = diag ? a : a + OP_BYTES;
-                    const bool first = it == c * CHUNK_STAGES;
+                    const bool first = it == c * chunk_stages;
 #pragma unroll
                     for (int k = 0; k < KSTAGE / 16; ++k) {
                         const uint64_t da = tc::smem_desc(a + k * 2048, BOX_BYTES, 1024, tc::SW_128B);
@@ -304,7 +304,7 @@ bool hessian_tc_eligible(int64_t n, int64_t T, const void *X) {
 // workspace partials and a fixed-order reduction.
 static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
                                      float *out2, float sign, int *err, void *ws, size_t ws_bytes, int sms,
-                                     const char *name) {
+                                     const char *name, int chunk_stages = CHUNK_STAGES) {
     CUtensorMap mapA, mapB;
     CUresult cr = encode_tmap_2d_bf16(&mapA, XA, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
     if (cr == CUDA_SUCCESS && XB)
@@ -330,7 +330,7 @@ static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const
     {
         Launch L(name, s);
         hess_tc_kernel<<<dim3((unsigned)tiles, (unsigned)splits), THREADS, SMEM_BYTES, s>>>(
-            mapA, mapB, n, T, tper, out, out2, part, splits == 1, cross, sign, err);
+            mapA, mapB, n, T, tper, out, out2, part, splits == 1, cross, sign, chunk_stages, err);
     }
     REALQ_TRY(check_launch(name));
     if (splits > 1) {
@@ -346,8 +346,9 @@ realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void 
 }
 
 realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
-                                float sign, int *err, void *ws, size_t ws_bytes, int sms) {
-    return hess_tc_launch(s, n, T, XA, XB, out, nullptr, sign, err, ws, ws_bytes, sms, "hessian_cross_tc");
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages) {
+    return hess_tc_launch(s, n, T, XA, XB, out, nullptr, sign, err, ws, ws_bytes, sms, "hessian_cross_tc",
+                          chunk_stages > 0 ? chunk_stages : CHUNK_STAGES);
 }
 
 }  // namespace realq

@@ -1,6 +1,8 @@
 // Host-side launchers of the library's kernels (internal interface).
 #pragma once
 
+#include <vector>
+
 #include "common.cuh"
 
 namespace realq {
@@ -49,7 +51,7 @@ struct GemmArgs {
 realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name);
 
 // ------------------------------------------- tensor-core tf32x3 GEMM ---
-enum TcMode { TC_STORE = 0, TC_BGD_P = 1, TC_ADAM = 2 };
+enum TcMode { TC_STORE = 0, TC_BGD_P = 1, TC_ADAM = 2, TC_ACCUM = 3, TC_BGD_PG = 4 };
 struct TcEpi {
     int mode;
     float *C; int64_t ldc;                                   // TC_STORE
@@ -70,7 +72,9 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb);
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name);
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0);
+template <typename TY>
+realq_status_t tc_split_diff(cudaStream_t s, int64_t count, const float *x, const TY *y, float *hi, float *lo);
 
 // ------------------------------------------------- activation quantizer ---
 realq_status_t act_quant(cudaStream_t s, int64_t T, int64_t n, const void *X, realq_dtype_t dt, int bits, float a_clip,
@@ -94,8 +98,9 @@ realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float
 bool hessian_tc_eligible(int64_t n, int64_t T, const void *X);
 realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
                                size_t ws_bytes, int sms, float *H2 = nullptr);
+// chunk_stages: 64-token stages per TMEM accumulator pass before promotion (0: default)
 realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
-                                float sign, int *err, void *ws, size_t ws_bytes, int sms);
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages = 0);
 int hessian_splits_tiles(int64_t tiles, int64_t T, int sms);
 
 // --------------------------------------------------------------- prepare ---
@@ -131,13 +136,24 @@ struct SweepPlan {
     // tensor-core path: hi / lo planes and tensor maps
     int tc;
     float *Sh, *Sl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;
-    float *M;        // M = A H̄, kept current for the free columns
+    float *M;        // M = A H̄ (per row group: A H̄_g), kept current for the free columns
     int64_t step_c;  // first column of the last optimizer step not yet in M (n: none)
     TcMaps mapsP, mapsG;
+    // row-grouped OBS (Alg. 1 "for all row-groups g"): rgroups contiguous row
+    // groups of rg_rows rows, group g quantized against U_g; rgroups == 1
+    // means U, Hbar and dead for every row
+    int rgroups;
+    int grouped;     // OBS of the row groups on their own H̄_g (the grouped entry point)
+    int64_t rg_rows;
+    const float *Ug, *Hbar_g;
+    const uint8_t *dead_g;
+    float *lam_g;                               // lambda_g per group (workspace)
+    float *HGh, *HGl, *GGh, *GGl, *DWh, *DWl;   // tf32 planes of H̄_g, H̄_g - H̄, W - W0
+    std::vector<TcMaps> mapsMg, mapsQg;
     int f_split_alpha_valid;
     float f_split_alpha;
 };
-size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar);
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0);
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);
 realq_status_t sweep_init(cudaStream_t s, SweepPlan &p);
 realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b);

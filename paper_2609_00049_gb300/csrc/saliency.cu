@@ -8,16 +8,25 @@
 // The percentile is an exact order statistic: one CTA per group runs a radix
 // select over the bit patterns of the (non-negative) saliencies, 8 bits per
 // pass from the top, so the threshold is one of the inputs, bit for bit.
-// The weighted product reuses the bf16 tensor-core Hessian: the rows
-// y_t = bf16(sqrt(s'_t) x̂_t) of one group are formed in a workspace and
-// accumulated as y^T y (each product is within two bf16 roundings, 2^-8
-// relative, of s' x_i x_j); the weight sums are fixed-order fp64 reductions.
+// The weighted product runs on the bf16 tensor cores as H_g = X̂ᵀ (s' X̂):
+// the scaled rows y_t = s'_t x̂_t of one group are split into two bf16 parts,
+// y = y_hi + y_lo (16 significant bits together), and accumulated by two
+// full-tile cross passes X̂ᵀ y_hi + X̂ᵀ y_lo; x̂ is exact in bf16, so each
+// product is within 2^-17 relative of s' x_i x_j, and the accumulation is
+// promoted to fp32 registers every 128 tokens.  A single bf16 rounding
+// (2^-9) is not enough: with heavy-tailed saliency a few dozen tokens carry
+// most of the weight and the rounding does not average out.  The weight sums
+// are fixed-order fp64 reductions.
 #include "kernels.cuh"
 
 namespace realq {
 namespace {
 
 constexpr int SEL_THREADS = 1024;
+// Saliency spreads token magnitudes over decades, so a TMEM accumulator loses
+// the low bits of small terms against a running sum dominated by a few large
+// ones; promote to fp32 registers every 2 stages (128 tokens) instead of 16.
+constexpr int kPromoteStages = 2;
 
 __device__ __forceinline__ uint32_t key_of(float v) { return __float_as_uint(fmaxf(v, 0.f)); }
 
@@ -62,14 +71,16 @@ __global__ void clip_kernel(int64_t count, int ng, const float *S, const float *
     if (i < count) out[i] = fminf(S[i], c[i % ng]);
 }
 
-// y[t, :] = bf16(sqrt(s[t, g]) x[t, :])
+// y = s[t, g] x[t, :] (fp32, exact up to one rounding), split into bf16 parts
 __global__ void wscale_kernel(int64_t T, int64_t n, const __nv_bfloat16 *X, const float *S, int g, int ng,
-                              __nv_bfloat16 *Y) {
+                              __nv_bfloat16 *Yhi, __nv_bfloat16 *Ylo) {
     const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
     if (i >= T * n) return;
     const int64_t t = i / n;
-    const float w = sqrtf(fmaxf(S[t * ng + g], 0.f));
-    Y[i] = __float2bfloat16_rn(w * __bfloat162float(X[i]));
+    const float y = fmaxf(S[t * ng + g], 0.f) * __bfloat162float(X[i]);
+    const __nv_bfloat16 hi = __float2bfloat16_rn(y);
+    Yhi[i] = hi;
+    Ylo[i] = __float2bfloat16_rn(y - __bfloat162float(hi));
 }
 
 // wsum[g] += sum_t s[t, g] in fp64, one CTA per group, fixed order
@@ -111,24 +122,32 @@ realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, 
 }
 
 size_t weighted_ws_bytes(int64_t n, int64_t T) {
-    return align_up(hessian_ws_bytes(n, T, 0)) + align_up((size_t)T * n * sizeof(__nv_bfloat16));
+    return align_up(hessian_ws_bytes(n, T, 0)) + 2 * align_up((size_t)T * n * sizeof(__nv_bfloat16));
 }
 
 realq_status_t hessian_weighted(cudaStream_t s, int64_t n, int64_t T, const void *X, int ng, const float *S,
                                 float *Hg, double *wsum, void *ws, size_t ws_bytes) {
     if (T == 0) return REALQ_OK;
-    // [Hessian workspace: status word, token-split partials][rows y of one group]
+    // [Hessian workspace: status word, token-split partials][y_hi][y_lo] of one group
     const size_t hbytes = hessian_ws_bytes(n, T, 0);
-    void *hws = ws;
-    __nv_bfloat16 *Y = reinterpret_cast<__nv_bfloat16 *>(static_cast<char *>(ws) + align_up(hbytes));
+    char *base = static_cast<char *>(ws);
+    int *err = reinterpret_cast<int *>(base);
+    void *part = base + align_up(sizeof(int));
+    const size_t pbytes = hbytes - align_up(sizeof(int));
+    __nv_bfloat16 *Yhi = reinterpret_cast<__nv_bfloat16 *>(base + align_up(hbytes));
+    __nv_bfloat16 *Ylo = Yhi + align_up((size_t)T * n * sizeof(__nv_bfloat16)) / sizeof(__nv_bfloat16);
+    const bool tc = hessian_tc_eligible(n, T, X) && hessian_tc_eligible(n, T, Yhi) && hessian_tc_eligible(n, T, Ylo);
+    if (!tc) return fail(REALQ_ERR_UNSUPPORTED, "weighted Hessian: n must be a multiple of 8 and >= 64");
     for (int g = 0; g < ng; ++g) {
         {
             Launch L("saliency_scale", s);
             wscale_kernel<<<(unsigned)((T * n + 255) / 256), 256, 0, s>>>(T, n, static_cast<const __nv_bfloat16 *>(X),
-                                                                          S, g, ng, Y);
+                                                                          S, g, ng, Yhi, Ylo);
         }
         REALQ_TRY(check_launch("saliency_scale"));
-        REALQ_TRY(hessian_accumulate(s, n, T, Y, nullptr, REALQ_BF16, Hg + (size_t)g * n * n, nullptr, hws, hbytes));
+        float *Hout = Hg + (size_t)g * n * n;
+        REALQ_TRY(hessian_cross_tc(s, n, T, X, Yhi, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages));
+        REALQ_TRY(hessian_cross_tc(s, n, T, X, Ylo, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages));
     }
     {
         Launch L("saliency_wsum", s);

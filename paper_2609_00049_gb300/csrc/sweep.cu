@@ -75,6 +75,7 @@ struct QArgs {
     uint8_t *codes;
     int64_t ncb;
     float *Et;
+    int64_t ldet;          // leading dimension of Et (all rows of the layer)
     int *status;
 };
 
@@ -208,7 +209,7 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
                     for (int kk = jj + 1; kk < 32; ++kk) r[kk] = fmaf(-err, Us[j * UP + c0 + kk], r[kk]);
                 }
                 Es[lane * 33 + jj] = err;
-                if (live && j < kb) a.Et[(int64_t)j * a.m + i] = err;
+                if (live && j < kb) a.Et[(int64_t)j * a.ldet + i] = err;
                 packed[jj >> 3] |= (qi & 15u) << ((jj & 7) * 4);
             }
             if (live) {
@@ -376,12 +377,15 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 // and need hi / lo planes of the displacement, H̄, F and P^T; otherwise the
 // fp32 SIMT path needs P, G (and F_eff).  block = 0: Block-GD only (literal
 // gradient form, SIMT).
-size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar) {
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups) {
     const size_t mn = align_up((size_t)m * n * sizeof(float));
+    const size_t nn = align_up((size_t)n * n * sizeof(float));
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
+    if (rgroups > 0) b += align_up((size_t)rgroups * sizeof(float));
     if (has_bgd) {
         if (block > 0 && tc_gemm_eligible(m, n)) {
-            b += 5 * mn + 2 * align_up((size_t)n * n * sizeof(float)) + 2 * align_up((size_t)m * m * sizeof(float));
+            b += 5 * mn + 2 * nn + 2 * align_up((size_t)m * m * sizeof(float));
+            if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
         } else {
             b += 2 * mn;
             if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
@@ -399,6 +403,8 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
     p.Et = cv.take<float>((size_t)p.block * p.m);
     p.P = p.G = p.Feff = p.R0 = nullptr;
     p.Sh = p.Sl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = p.M = nullptr;
+    p.HGh = p.HGl = p.GGh = p.GGl = p.DWh = p.DWl = nullptr;
+    p.lam_g = p.grouped ? cv.take<float>((size_t)p.rgroups) : nullptr;
     p.step_c = p.n;
     p.tc = 0;
     if (has_bgd) {
@@ -413,6 +419,15 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
             p.Hl = cv.take<float>((size_t)p.n * p.n);
             p.Fh = cv.take<float>((size_t)p.m * p.m);
             p.Fl = cv.take<float>((size_t)p.m * p.m);
+            if (p.grouped) {
+                p.DWh = cv.take<float>(mn);
+                p.DWl = cv.take<float>(mn);
+                const size_t gnn = (size_t)p.rgroups * p.n * p.n;
+                p.HGh = cv.take<float>(gnn);
+                p.HGl = cv.take<float>(gnn);
+                p.GGh = cv.take<float>(gnn);
+                p.GGl = cv.take<float>(gnn);
+            }
         } else {
             p.P = cv.take<float>(mn);
             p.G = cv.take<float>(mn);
@@ -424,12 +439,19 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
 
 realq_status_t sweep_init(cudaStream_t s, SweepPlan &p) {
     const int64_t mn = p.m * p.n;
-    {
+    // per row group: the group's dead channels (one group: dead)
+    for (int gr = 0; gr < p.rgroups; ++gr) {
+        const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+        if (rows <= 0) break;
+        const uint8_t *dd = p.grouped ? p.dead_g + (size_t)gr * p.n : p.dead;
+        const int64_t cnt = rows * p.n;
         Launch L("init_work", s);
         if (p.w_dtype == REALQ_BF16)
-            init_work_kernel<<<blocks_for(mn), 256, 0, s>>>(p.m, p.n, static_cast<const __nv_bfloat16 *>(p.W0), p.dead, p.W);
+            init_work_kernel<<<blocks_for(cnt), 256, 0, s>>>(
+                rows, p.n, static_cast<const __nv_bfloat16 *>(p.W0) + row0 * p.n, dd, p.W + row0 * p.n);
         else
-            init_work_kernel<<<blocks_for(mn), 256, 0, s>>>(p.m, p.n, static_cast<const float *>(p.W0), p.dead, p.W);
+            init_work_kernel<<<blocks_for(cnt), 256, 0, s>>>(rows, p.n, static_cast<const float *>(p.W0) + row0 * p.n,
+                                                             dd, p.W + row0 * p.n);
     }
     REALQ_TRY(check_launch("init_work"));
     if (p.bgd_steps > 0) {
@@ -544,6 +566,53 @@ static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
     return REALQ_OK;
 }
 
+// One optimizer step with a row-grouped OBS.  Rows of group g were swept
+// against H_g,d = H̄_g + lambda_g I, so the stationarity identity holds for
+// H_g,d, and P_R = ((Ŵ - W0) H̄)_R for those rows is
+//   M_g + lambda_g (A - ΔW) - ΔW (H̄_g - H̄),   M_g = A H̄_g  (rows of g),
+// which is the one-Hessian form when H̄_g = H̄.  M_g is kept current like M;
+// ΔW (H̄_g - H̄) takes the full K = n.  Then G = F_eff P and Adam for all rows.
+static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c0) {
+    const int64_t r = p.n - c0;
+    const int64_t k0 = p.step_c;
+    if (p.w_dtype == REALQ_BF16)
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const __nv_bfloat16 *>(p.W0), p.DWh, p.DWl));
+    else
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const float *>(p.W0), p.DWh, p.DWl));
+    const size_t w0sz = p.w_dtype == REALQ_BF16 ? 2 : 4;
+    for (int gr = 0; gr < p.rgroups; ++gr) {
+        const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+        if (rows <= 0) break;
+        if (k0 < p.n) {
+            TcEpi e{};
+            e.mode = TC_ACCUM;
+            e.M = p.M + row0 * p.n; e.ldw = p.n; e.col0 = c0;
+            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMg[gr], rows, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm",
+                                     (int)row0));
+        }
+        TcEpi q{};
+        q.mode = TC_BGD_PG;
+        q.Ad = p.disp + row0 * p.n; q.W = p.W + row0 * p.n;
+        q.W0 = static_cast<const char *>(p.W0) + (size_t)row0 * p.n * w0sz; q.w0_bf16 = p.w_dtype == REALQ_BF16;
+        q.dead = p.dead_g + (size_t)gr * p.n; q.lam = p.lam_g + gr; q.R0 = p.R0 ? p.R0 + row0 * p.n : nullptr;
+        q.ldw = p.n; q.col0 = c0; q.M = p.M + row0 * p.n;
+        q.Pth = p.Pth + row0; q.Ptl = p.Ptl + row0; q.ldp = p.m;
+        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsQg[gr], rows, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm", (int)row0));
+    }
+    const int64_t t = ++(*p.adam_t);
+    TcEpi g{};
+    g.mode = TC_ADAM;
+    g.ldw = p.n; g.col0 = c0;
+    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
+    g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
+    g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
+    g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
+    g.sgd = p.optimizer == REALQ_OPT_SGD;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    p.step_c = c0;
+    return REALQ_OK;
+}
+
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
     if (col_start >= p.n) return REALQ_OK;
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
@@ -567,16 +636,23 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
                                                               p.zero);
     }
     if (!params_here) REALQ_TRY(check_launch("group_params"));
-    QArgs qa{};
-    qa.m = p.m; qa.n = p.n; qa.bs = bs; qa.kb = kb;
-    qa.W = p.W; qa.U = p.U;
-    qa.g = p.group; qa.ngroups = p.ngroups; qa.bits = p.bits; qa.sym = p.sym;
-    qa.scale = p.scale; qa.zero = p.zero; qa.codes = p.codes; qa.ncb = (p.n + 1) / 2;
-    qa.Et = p.Et; qa.status = p.status;
     const int Gk = !params_here ? 0 : (p.group >= p.n ? B : p.group);
-    if (B == 128) REALQ_TRY(launch_qb_g<128>(s, qa, Gk));
-    else if (B == 64) REALQ_TRY(launch_qb_g<64>(s, qa, Gk));
-    else REALQ_TRY(launch_qb_g<32>(s, qa, Gk));
+    for (int gr = 0; gr < p.rgroups; ++gr) {
+        // row group gr against its own U (one group: all rows, U)
+        const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+        if (rows <= 0) break;
+        const int64_t ncb = (p.n + 1) / 2;
+        QArgs qa{};
+        qa.m = rows; qa.n = p.n; qa.bs = bs; qa.kb = kb;
+        qa.W = p.W + row0 * p.n; qa.U = p.Ug + (size_t)gr * p.n * p.n;
+        qa.g = p.group; qa.ngroups = p.ngroups; qa.bits = p.bits; qa.sym = p.sym;
+        qa.scale = p.scale + row0 * p.ngroups; qa.zero = p.zero + row0 * p.ngroups; qa.codes = p.codes + row0 * ncb;
+        qa.ncb = ncb;
+        qa.Et = p.Et + row0; qa.ldet = p.m; qa.status = p.status;
+        if (B == 128) REALQ_TRY(launch_qb_g<128>(s, qa, Gk));
+        else if (B == 64) REALQ_TRY(launch_qb_g<64>(s, qa, Gk));
+        else REALQ_TRY(launch_qb_g<32>(s, qa, Gk));
+    }
     if (p.W_deq) {
         Launch L("copy_deq", s);
         if (p.deq_dtype == REALQ_BF16)
@@ -587,13 +663,18 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     if (p.W_deq) REALQ_TRY(check_launch("copy_deq"));
     if (be >= p.n) return REALQ_OK;
     // lazy batch update of every later column: W[:, be:] -= E_b U[bs:be, be:]
-    GemmArgs g{};
-    g.M = p.m; g.N = p.n - be; g.K = kb;
-    g.A = p.Et; g.lda = p.m;
-    g.B = p.U + bs * p.n + be; g.ldb = p.n;
-    g.C = p.W + be; g.ldc = p.n;
-    g.alpha = 1.f;
-    REALQ_TRY(gemm_f32(s, A_KMAJOR, EPI_SUB, g, "trailing_update"));
+    // (per row group with its own U)
+    for (int gr = 0; gr < p.rgroups; ++gr) {
+        const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+        if (rows <= 0) break;
+        GemmArgs g{};
+        g.M = rows; g.N = p.n - be; g.K = kb;
+        g.A = p.Et + row0; g.lda = p.m;
+        g.B = p.Ug + (size_t)gr * p.n * p.n + bs * p.n + be; g.ldb = p.n;
+        g.C = p.W + row0 * p.n + be; g.ldc = p.n;
+        g.alpha = 1.f;
+        REALQ_TRY(gemm_f32(s, A_KMAJOR, EPI_SUB, g, "trailing_update"));
+    }
     if (p.bgd_steps <= 0) return REALQ_OK;
     const int64_t b_global = p.b_global_start + b;
     float alpha = 1.f;
@@ -607,7 +688,8 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             p.f_split_alpha_valid = 1;
             p.f_split_alpha = a_eff;
         }
-        for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one_tc(s, p, be));
+        for (int k = 0; k < p.bgd_steps; ++k)
+            REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be) : bgd_one_tc(s, p, be));
         return REALQ_OK;
     }
     const float *Fuse = nullptr;
@@ -633,14 +715,47 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
         REALQ_TRY(tc_make_maps(&p.mapsG, p.Fh, p.Fl, p.m, p.m, p.m, p.Pth, p.Ptl, p.n, p.m, p.m));
         p.f_split_alpha_valid = 0;
         p.step_c = p.n;
+        if (p.grouped) {
+            // per row group: lambda_g, planes of H̄_g and H̄_g - H̄, the maps of
+            // the M_g update and of the correction product
+            const size_t nn = (size_t)p.n * p.n;
+            p.mapsMg.assign(p.rgroups, TcMaps{});
+            p.mapsQg.assign(p.rgroups, TcMaps{});
+            for (int gr = 0; gr < p.rgroups; ++gr) {
+                {
+                    Launch L("bgd_lambda", s);
+                    lambda_kernel<<<1, 1024, 0, s>>>(p.n, p.Hbar_g + gr * nn, p.dead_g + (size_t)gr * p.n, p.damp,
+                                                     p.lam_g + gr);
+                }
+                REALQ_TRY(check_launch("bgd_lambda"));
+                REALQ_TRY(tc_split(s, (int64_t)nn, p.Hbar_g + gr * nn, nullptr, 1.f, p.HGh + gr * nn, p.HGl + gr * nn));
+                REALQ_TRY(tc_split_diff(s, (int64_t)nn, p.Hbar_g + gr * nn, p.Hbar, p.GGh + gr * nn, p.GGl + gr * nn));
+                REALQ_TRY(tc_make_maps(&p.mapsMg[gr], p.Sh, p.Sl, p.m, p.n, p.n, p.HGh + gr * nn, p.HGl + gr * nn, p.n,
+                                       p.n, p.n));
+                REALQ_TRY(tc_make_maps(&p.mapsQg[gr], p.DWh, p.DWl, p.m, p.n, p.n, p.GGh + gr * nn, p.GGl + gr * nn,
+                                       p.n, p.n, p.n));
+            }
+        }
         if (fresh) {
             REALQ_CUDA_TRY(cudaMemsetAsync(p.M, 0, (size_t)p.m * p.n * sizeof(float), s));
         } else {
             REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Sh, p.Sl));
-            TcEpi e{};
-            e.mode = TC_STORE;
-            e.C = p.M; e.ldc = p.n;
-            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm"));
+            if (p.grouped) {
+                for (int gr = 0; gr < p.rgroups; ++gr) {
+                    const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+                    if (rows <= 0) break;
+                    TcEpi e{};
+                    e.mode = TC_STORE;
+                    e.C = p.M + row0 * p.n; e.ldc = p.n;
+                    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMg[gr], rows, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm",
+                                             (int)row0));
+                }
+            } else {
+                TcEpi e{};
+                e.mode = TC_STORE;
+                e.C = p.M; e.ldc = p.n;
+                REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm"));
+            }
         }
     }
     return REALQ_OK;
