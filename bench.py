@@ -156,17 +156,22 @@ def gpu_arm(args, wl, rank, world):
     bq = BlockQuantizer([BlockInput(nm, sp.n, sp.T) for nm, sp in wl.inputs.items()],
                         [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
                         wl.steps_per_block, sliding_window=wl.sliding_window, device=dev,
-                        act_quant=(args.act_bits, args.a_clip) if args.act_bits else None)
+                        act_quant=(args.act_bits, args.a_clip) if args.act_bits else None,
+                        saliency_groups=args.saliency_groups)
+    dev_sal = None
+    if args.saliency_groups:
+        dev_sal = {mod.name: torch.from_numpy(synth.saliency(wl, mod, args.saliency_groups)).to(dev)
+                   for mod in wl.modules}
     host_out = {mod.name: {k: torch.empty_like(bq.out[mod.name][k], device="cpu").pin_memory()
                            for k in ("codes", "scale", "zero")} for mod in wl.modules}
     e2e_bytes = {"h2d": 0, "d2h": 0}
 
     def step_device():
-        bq.run(dev_x, dev_w, dev_f, dev_fn)
+        bq.run(dev_x, dev_w, dev_f, dev_fn, saliency=dev_sal)
         bq.check_status()
 
     def step_serial():
-        bq.run_serial(dev_x, dev_w, dev_f, dev_fn)
+        bq.run_serial(dev_x, dev_w, dev_f, dev_fn, saliency=dev_sal)
 
     def step_e2e():
         h2d, d2h = bq.run_host(host_x, host_w, host_f, host_out)
@@ -225,7 +230,7 @@ def gpu_arm(args, wl, rank, world):
 
     # ---- end to end through host buffers
     e2e = None
-    if not args.no_e2e and not args.act_bits:
+    if not args.no_e2e and not args.act_bits and not args.saliency_groups:
         step_e2e()
         torch.cuda.synchronize()
         barrier()
@@ -260,7 +265,9 @@ def gpu_arm(args, wl, rank, world):
                        "columns_per_step": wl.total_columns, "column_blocks_per_step": wl.total_column_blocks,
                        "quantizer": f"W{wl.bits}" + (f"A{args.act_bits} (activation-aware, a_clip {args.a_clip})"
                                                      if args.act_bits else "") +
-                                    f" {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}",
+                                    f" {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}" +
+                                    (f", saliency-weighted grouped Hessians (N_g={args.saliency_groups}, clip p99)"
+                                     if args.saliency_groups else ""),
                        "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}",
                        "parallelism": f"replicas x{world}",
                        "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
@@ -468,6 +475,8 @@ def main():
     ap.add_argument("--act-bits", type=int, default=0,
                     help="activation-aware weight-activation variant: per-token activation bits (0: weights only)")
     ap.add_argument("--a-clip", type=float, default=0.9, help="activation clipping ratio for --act-bits")
+    ap.add_argument("--saliency-groups", type=int, default=0,
+                    help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep"], default=None,

@@ -22,9 +22,11 @@ from typing import Dict, List, Optional, Sequence
 
 import torch
 
-from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_hessian_prepare,
+from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_hessian_accumulate_weighted,
+               realq_hessian_prepare, realq_hessian_prepare_scaled, realq_hessian_weighted_workspace_size,
                realq_hessian_workspace_size, realq_prepare_workspace_size, realq_quantize_activations,
-               realq_quantize_layer, realq_quantize_workspace_size, realq_scale_moment, realq_workspace_status,
+               realq_quantize_grouped_workspace_size, realq_quantize_layer, realq_quantize_layer_grouped,
+               realq_quantize_workspace_size, realq_saliency_clip, realq_scale_moment, realq_workspace_status,
                workspace)
 
 
@@ -58,11 +60,18 @@ class BlockQuantizer:
     variant (Sec. 5): each input is quantized per token first, the Hessian is
     taken over the quantized activations, and the Block-GD surrogate keeps
     the full-precision ones through the cross moment D.
+
+    saliency_groups=N_g > 0 selects the saliency-weighted grouped Hessians
+    (Sec. 3.3, Alg. 1 "for all row-groups g"): every module's rows form N_g
+    groups, run() takes a (T x N_g) saliency per module, clipped to its
+    saliency_pct percentile, and each group is swept against its own factor;
+    Block-GD keeps the input's plain H̄.
     """
 
     def __init__(self, inputs: Sequence[BlockInput], modules: Sequence[BlockModule], qcfg: QuantCfg, lr: float,
                  steps_per_block: int = 1, sliding_window: bool = False, device="cuda",
-                 host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None):
+                 host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None, saliency_groups: int = 0,
+                 saliency_pct: float = 0.99):
         self.inputs: Dict[str, BlockInput] = {i.name: i for i in inputs}
         self.modules: List[BlockModule] = list(modules)
         for md in self.modules:
@@ -74,6 +83,8 @@ class BlockQuantizer:
             self.device = torch.device(self.device.type, torch.cuda.current_device())
         self.sliding_window = sliding_window
         self.act_quant = act_quant
+        self.sgroups = saliency_groups
+        self.spct = saliency_pct
         self.mods_of = {name: [md for md in self.modules if md.input == name] for name in self.inputs}
         B = qcfg.block_size
         self.B_total = sum(-(-md.n // B) for md in self.modules)
@@ -100,14 +111,31 @@ class BlockQuantizer:
                          B_total=self.B_total if sliding_window else 1)
             bstart += -(-n // B)
             bgd = steps_per_block > 0
+            if saliency_groups:
+                ngs = saliency_groups
+                ws_q = workspace(realq_quantize_grouped_workspace_size(m, n, ngs, qcfg, bc if bgd else None,
+                                                                       sliding_window, act_quant is not None and bgd),
+                                 dev)
+                grp = dict(Sc=torch.empty(self.inputs[md.input].T, ngs, device=dev),
+                           clip=torch.empty(ngs, device=dev),
+                           Hg=torch.empty(ngs, n, n, device=dev), Ug=torch.empty(ngs, n, n, device=dev),
+                           Hbg=torch.empty(ngs, n, n, device=dev),
+                           dg=torch.empty(ngs, n, dtype=torch.uint8, device=dev),
+                           wsum=torch.empty(ngs, dtype=torch.float64, device=dev),
+                           wws=workspace(realq_hessian_weighted_workspace_size(n, self.inputs[md.input].T), dev),
+                           pws=workspace(realq_prepare_workspace_size(n), dev))
+            else:
+                ws_q = workspace(realq_quantize_workspace_size(m, n, qcfg, bc if bgd else None, sliding_window,
+                                                               act_quant is not None and bgd), dev)
+                grp = None
             self.out[md.name] = dict(
+                grp=grp,
                 W=torch.empty(m, n, device=dev),
                 codes=torch.empty(m, (n + 1) // 2, dtype=torch.uint8, device=dev),
                 scale=torch.empty(m, ng, device=dev), zero=torch.empty(m, ng, dtype=torch.uint8, device=dev),
                 am=torch.empty(m, n, device=dev) if bgd else None, av=torch.empty(m, n, device=dev) if bgd else None,
                 disp=torch.empty(m, n, device=dev) if bgd else None, bcfg=bc if bgd else None,
-                ws=workspace(realq_quantize_workspace_size(m, n, qcfg, bc if bgd else None, sliding_window,
-                                                           act_quant is not None and bgd), dev),
+                ws=ws_q,
                 adam_t=0)
         self.in_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
         self.copy_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
@@ -120,15 +148,38 @@ class BlockQuantizer:
         self._w_stage = None
 
     # ------------------------------------------------------------------ device
-    def _quantize_module(self, md: BlockModule, s_in, W0, F, F_next, stream):
+    def _quantize_module(self, md: BlockModule, s_in, W0, F, F_next, stream, X=None, sal=None):
         o = self.out[md.name]
+        if o["grp"] is not None:
+            # saliency-weighted Hessians of this module's row groups, their
+            # factors, then the grouped sweep (all on the module's stream)
+            gp, T = o["grp"], self.inputs[md.input].T
+            realq_saliency_clip(sal, self.spct, S_out=gp["Sc"], clip_out=gp["clip"], stream=stream)
+            with torch.cuda.stream(stream if stream is not None else torch.cuda.current_stream(self.device)):
+                gp["Hg"].zero_()
+                gp["wsum"].zero_()
+            realq_hessian_accumulate_weighted(s_in["Xq"] if self.act_quant is not None else X, gp["Sc"], gp["Hg"],
+                                              gp["wsum"], gp["wws"], stream=stream)
+            wsum = gp["wsum"].cpu() if stream is None else None
+            if wsum is None:
+                stream.synchronize()
+                wsum = gp["wsum"].cpu()
+            for g in range(self.sgroups):
+                realq_hessian_prepare_scaled(gp["Hg"][g], float(wsum[g]), self.qcfg.damp_frac, gp["Ug"][g],
+                                             gp["Hbg"][g], gp["dg"][g], gp["pws"], stream=stream)
+            o["adam_t"] = realq_quantize_layer_grouped(
+                W0, gp["Ug"], gp["Hbg"], gp["dg"], s_in["Hbar"], self.qcfg, o["W"], o["codes"], o["scale"],
+                o["zero"], Dbar=s_in.get("Dbar") if o["bcfg"] is not None else None, bcfg=o["bcfg"], F=F,
+                F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"], bgd_disp=o["disp"],
+                ws=o["ws"], stream=stream)
+            return
         o["adam_t"] = realq_quantize_layer(
             W0, s_in["U"], s_in["Hbar"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"],
             Dbar=s_in.get("Dbar") if o["bcfg"] is not None else None, dead=s_in["dead"],
             bcfg=o["bcfg"], F=F, F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"],
             bgd_disp=o["disp"], ws=o["ws"], stream=stream)
 
-    def _input_pipeline(self, name, start, X, W0, F, F_next):
+    def _input_pipeline(self, name, start, X, W0, F, F_next, sal=None):
         torch.cuda.set_device(self.device)
         spec, s_in, si = self.inputs[name], self.state[name], self.in_streams[name]
         si.wait_event(start)
@@ -136,7 +187,8 @@ class BlockQuantizer:
         for md in self.mods_of[name]:
             sm = self.mod_streams[md.name]
             sm.wait_stream(si)
-            self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), sm)
+            self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), sm, X=X[name],
+                                  sal=(sal or {}).get(md.name))
 
     def _hessian(self, name, X, stream):
         """H (and, activation-aware, D) of one input, then its preparation."""
@@ -145,6 +197,11 @@ class BlockQuantizer:
             s_in["H"].zero_()
             if self.act_quant is not None:
                 s_in["D"].zero_()
+        if self.act_quant is None and self.sgroups:
+            # the groups' factors come per module; the plain H̄ serves Block-GD
+            realq_hessian_accumulate(X, s_in["H"], ws=s_in["hws"], stream=stream)
+            realq_scale_moment(s_in["H"], spec.T, s_in["Hbar"], stream=stream)
+            return
         if self.act_quant is None:
             realq_hessian_accumulate(X, s_in["H"], ws=s_in["hws"], stream=stream)
         else:
@@ -164,25 +221,31 @@ class BlockQuantizer:
             start_stream.wait_stream(self.copy_streams[name])
 
     def run(self, X: Dict[str, torch.Tensor], W0: Dict[str, torch.Tensor], F: Dict[str, torch.Tensor],
-            F_next: Optional[Dict[str, torch.Tensor]] = None) -> None:
+            F_next: Optional[Dict[str, torch.Tensor]] = None,
+            saliency: Optional[Dict[str, torch.Tensor]] = None) -> None:
         """Quantize the block from device-resident inputs (X̂ per input, W0 and
-        F per module).  Work is enqueued after everything already on the
-        current stream, and the current stream waits for all of it on return."""
+        F per module, and with saliency groups a T x N_g saliency per module).
+        Work is enqueued after everything already on the current stream, and
+        the current stream waits for all of it on return."""
+        if self.sgroups and saliency is None:
+            raise ValueError("saliency_groups: run() needs a saliency per module")
         cur = torch.cuda.current_stream(self.device)
         start = torch.cuda.Event()
         start.record(cur)
-        futs = [self.pool.submit(self._input_pipeline, name, start, X, W0, F, F_next) for name in self.inputs]
+        futs = [self.pool.submit(self._input_pipeline, name, start, X, W0, F, F_next, saliency)
+                for name in self.inputs]
         for f in futs:
             f.result()
         self._join(cur)
 
-    def run_serial(self, X, W0, F, F_next=None) -> None:
+    def run_serial(self, X, W0, F, F_next=None, saliency=None) -> None:
         """The same work, one call after another on the current stream."""
         for name, spec in self.inputs.items():
             s_in = self.state[name]
             self._hessian(name, X[name], None)
             for md in self.mods_of[name]:
-                self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), None)
+                self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), None,
+                                      X=X[name], sal=(saliency or {}).get(md.name))
 
     def check_status(self) -> None:
         """Raise if any module's sweep recorded a non-finite value or a timeout."""
@@ -240,8 +303,8 @@ class BlockQuantizer:
         and F are copied per module, codes / scale / zero are copied back into
         out_host[module][...] (pinned).  Returns (h2d bytes, d2h bytes).
         The activation-aware variant is not streamed (it runs with run())."""
-        if self.act_quant is not None:
-            raise NotImplementedError("run_host: the activation-aware variant runs from device-resident inputs")
+        if self.act_quant is not None or self.sgroups:
+            raise NotImplementedError("run_host: this variant runs from device-resident inputs")
         dev = self.device
         if self._stage is None:
             self._stage = {name: [torch.empty(self.host_chunk, spec.n, dtype=X_host[name].dtype, device=dev)

@@ -58,8 +58,8 @@ __device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
 
 __global__ void __launch_bounds__(THREADS, 1)
     hess_tc_kernel(const __grid_constant__ CUtensorMap tmap, const __grid_constant__ CUtensorMap tmapB, int64_t n,
-                   int64_t T, int64_t tper, float *H, float *H2, float *part, int direct, int cross, float sign,
-                   int chunk_stages, int *err) {
+                   int64_t T, int64_t tper, float *H, float *H2, float *part, int direct, int cross, int two_maps,
+                   float sign, int chunk_stages, int *err) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -78,7 +78,10 @@ __global__ void __launch_bounds__(THREADS, 1)
     } else {
         lower_tile(blockIdx.x, ti, tj);
     }
-    const bool diag = !cross && ti == tj;
+    // cross: all tiles, no mirror; two_maps: the B operand comes from tmapB
+    // (a lower-triangle pass with two maps computes a product known to be
+    // symmetric, e.g. X̂ᵀ(s X̂), and mirrors it)
+    const bool diag = !two_maps && ti == tj;
     const int i0 = ti * TILE, j0 = tj * TILE;
     const int64_t t_begin = (int64_t)blockIdx.y * tper;
     const int64_t t_end = min(T, t_begin + tper);
@@ -97,7 +100,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         *abort_flag = 0;
         tc::fence_barrier_init();
         tc::prefetch_tmap(&tmap);
-        if (cross) tc::prefetch_tmap(&tmapB);
+        if (two_maps) tc::prefetch_tmap(&tmapB);
     }
     if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 2 * TILE);
     tc::fence_before_sync();
@@ -128,7 +131,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                 tc::tma_load_2d(a, &tmap, fb, i0, y);
                 tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
                 if (!diag) {
-                    const CUtensorMap *mb = cross ? &tmapB : &tmap;
+                    const CUtensorMap *mb = two_maps ? &tmapB : &tmap;
                     tc::tma_load_2d(a + OP_BYTES, mb, fb, j0, y);
                     tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, mb, fb, j0 + 64, y);
                 }
@@ -230,10 +233,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                     const float v = sign * acc[q];
                     if (direct) {
                         H[gi * n + gj] += v;
-                        if (!diag && !cross) H[gj * n + gi] += v;
+                        if (ti != tj && !cross) H[gj * n + gi] += v;
                         if (H2) {
                             H2[gi * n + gj] += v;
-                            if (!diag) H2[gj * n + gi] += v;
+                            if (ti != tj) H2[gj * n + gi] += v;
                         }
                     } else {
                         part[(int64_t)blockIdx.y * n * n + gi * n + gj] = v;
@@ -304,14 +307,15 @@ bool hessian_tc_eligible(int64_t n, int64_t T, const void *X) {
 // workspace partials and a fixed-order reduction.
 static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
                                      float *out2, float sign, int *err, void *ws, size_t ws_bytes, int sms,
-                                     const char *name, int chunk_stages = CHUNK_STAGES) {
+                                     const char *name, int chunk_stages = CHUNK_STAGES, bool sym_pair = false) {
     CUtensorMap mapA, mapB;
     CUresult cr = encode_tmap_2d_bf16(&mapA, XA, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
     if (cr == CUDA_SUCCESS && XB)
         cr = encode_tmap_2d_bf16(&mapB, XB, (uint64_t)n, (uint64_t)T, (uint64_t)n * 2, 64, KSTAGE, 1);
     if (cr != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled failed (%d)", (int)cr);
     if (!XB) mapB = mapA;
-    const int cross = XB != nullptr;
+    const int two_maps = XB != nullptr;
+    const int cross = two_maps && !sym_pair;
     const int nt = ceil_div(n, TILE);
     const int64_t tiles = cross ? (int64_t)nt * nt : (int64_t)nt * (nt + 1) / 2;
     int splits = cross ? hessian_splits_tiles(tiles, T, sms) : hessian_splits(n, T, sms);
@@ -330,7 +334,7 @@ static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const
     {
         Launch L(name, s);
         hess_tc_kernel<<<dim3((unsigned)tiles, (unsigned)splits), THREADS, SMEM_BYTES, s>>>(
-            mapA, mapB, n, T, tper, out, out2, part, splits == 1, cross, sign, chunk_stages, err);
+            mapA, mapB, n, T, tper, out, out2, part, splits == 1, cross, two_maps, sign, chunk_stages, err);
     }
     REALQ_TRY(check_launch(name));
     if (splits > 1) {
@@ -346,9 +350,11 @@ realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void 
 }
 
 realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
-                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages) {
-    return hess_tc_launch(s, n, T, XA, XB, out, nullptr, sign, err, ws, ws_bytes, sms, "hessian_cross_tc",
-                          chunk_stages > 0 ? chunk_stages : CHUNK_STAGES);
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages,
+                                bool symmetric) {
+    return hess_tc_launch(s, n, T, XA, XB, out, nullptr, sign, err, ws, ws_bytes, sms,
+                          symmetric ? "hessian_weighted_tc" : "hessian_cross_tc",
+                          chunk_stages > 0 ? chunk_stages : CHUNK_STAGES, symmetric);
 }
 
 }  // namespace realq

@@ -98,9 +98,12 @@ realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float
 bool hessian_tc_eligible(int64_t n, int64_t T, const void *X);
 realq_status_t hessian_syrk_tc(cudaStream_t s, int64_t n, int64_t T, const void *X, float *H, int *err, void *ws,
                                size_t ws_bytes, int sms, float *H2 = nullptr);
-// chunk_stages: 64-token stages per TMEM accumulator pass before promotion (0: default)
+// out += sign X_Aᵀ X_B.  chunk_stages: 64-token stages per TMEM accumulator
+// pass before promotion (0: default).  symmetric: the product is known to be
+// symmetric (X_B = diag(s) X_A up to rounding): lower tiles only, mirrored.
 realq_status_t hessian_cross_tc(cudaStream_t s, int64_t n, int64_t T, const void *XA, const void *XB, float *out,
-                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages = 0);
+                                float sign, int *err, void *ws, size_t ws_bytes, int sms, int chunk_stages = 0,
+                                bool symmetric = false);
 int hessian_splits_tiles(int64_t tiles, int64_t T, int sms);
 
 // --------------------------------------------------------------- prepare ---

@@ -13,7 +13,9 @@
 // y = y_hi + y_lo (16 significant bits together), and accumulated by two
 // full-tile cross passes X̂ᵀ y_hi + X̂ᵀ y_lo; x̂ is exact in bf16, so each
 // product is within 2^-17 relative of s' x_i x_j, and the accumulation is
-// promoted to fp32 registers every 128 tokens.  A single bf16 rounding
+// promoted to fp32 registers every 128 tokens.  The sum is symmetric up to
+// that rounding, so only tiles on or below the diagonal are formed, then
+// mirrored.  A single bf16 rounding
 // (2^-9) is not enough: with heavy-tailed saliency a few dozen tokens carry
 // most of the weight and the rounding does not average out.  The weight sums
 // are fixed-order fp64 reductions.
@@ -71,16 +73,27 @@ __global__ void clip_kernel(int64_t count, int ng, const float *S, const float *
     if (i < count) out[i] = fminf(S[i], c[i % ng]);
 }
 
-// y = s[t, g] x[t, :] (fp32, exact up to one rounding), split into bf16 parts
+// y = s[t, g] x[t, :] (fp32, one rounding), split into bf16 parts; 8 elements
+// (16 bytes) per thread, n a multiple of 8
 __global__ void wscale_kernel(int64_t T, int64_t n, const __nv_bfloat16 *X, const float *S, int g, int ng,
                               __nv_bfloat16 *Yhi, __nv_bfloat16 *Ylo) {
-    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
-    if (i >= T * n) return;
-    const int64_t t = i / n;
-    const float y = fmaxf(S[t * ng + g], 0.f) * __bfloat162float(X[i]);
-    const __nv_bfloat16 hi = __float2bfloat16_rn(y);
-    Yhi[i] = hi;
-    Ylo[i] = __float2bfloat16_rn(y - __bfloat162float(hi));
+    const int64_t v = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (v >= T * n / 8) return;
+    const int64_t i = v * 8;
+    const float w = fmaxf(S[(i / n) * ng + g], 0.f);
+    const uint4 xv = *reinterpret_cast<const uint4 *>(X + i);
+    const __nv_bfloat16 *xe = reinterpret_cast<const __nv_bfloat16 *>(&xv);
+    uint4 hv, lv;
+    __nv_bfloat16 *he = reinterpret_cast<__nv_bfloat16 *>(&hv);
+    __nv_bfloat16 *le = reinterpret_cast<__nv_bfloat16 *>(&lv);
+#pragma unroll
+    for (int k = 0; k < 8; ++k) {
+        const float y = w * __bfloat162float(xe[k]);
+        he[k] = __float2bfloat16_rn(y);
+        le[k] = __float2bfloat16_rn(y - __bfloat162float(he[k]));
+    }
+    *reinterpret_cast<uint4 *>(Yhi + i) = hv;
+    *reinterpret_cast<uint4 *>(Ylo + i) = lv;
 }
 
 // wsum[g] += sum_t s[t, g] in fp64, one CTA per group, fixed order
@@ -141,13 +154,13 @@ realq_status_t hessian_weighted(cudaStream_t s, int64_t n, int64_t T, const void
     for (int g = 0; g < ng; ++g) {
         {
             Launch L("saliency_scale", s);
-            wscale_kernel<<<(unsigned)((T * n + 255) / 256), 256, 0, s>>>(T, n, static_cast<const __nv_bfloat16 *>(X),
-                                                                          S, g, ng, Yhi, Ylo);
+            wscale_kernel<<<(unsigned)((T * n / 8 + 255) / 256), 256, 0, s>>>(
+                T, n, static_cast<const __nv_bfloat16 *>(X), S, g, ng, Yhi, Ylo);
         }
         REALQ_TRY(check_launch("saliency_scale"));
         float *Hout = Hg + (size_t)g * n * n;
-        REALQ_TRY(hessian_cross_tc(s, n, T, X, Yhi, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages));
-        REALQ_TRY(hessian_cross_tc(s, n, T, X, Ylo, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages));
+        REALQ_TRY(hessian_cross_tc(s, n, T, X, Yhi, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages, true));
+        REALQ_TRY(hessian_cross_tc(s, n, T, X, Ylo, Hout, 1.f, err, part, pbytes, num_sms(), kPromoteStages, true));
     }
     {
         Launch L("saliency_wsum", s);

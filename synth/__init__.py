@@ -273,6 +273,20 @@ def fisher_diag(wl: Workload, mod: ModuleSpec) -> np.ndarray:
     return np.diag(d).astype(np.float32)
 
 
+def saliency(wl: Workload, mod: ModuleSpec, n_groups: int = 4) -> np.ndarray:
+    """Synthetic per-token saliency of a module's row groups (T x n_groups fp32).
+
+    Stands in for the squared output-gradient norms of Stage 0: log-normal(0, 1)
+    per token and group, with 0.1 % of the tokens 10^6 x larger (the gradient
+    outliers the paper clips at the 99th percentile)."""
+    T = wl.inputs[mod.input].T
+    r = rng(wl.seed, "saliency", mod.name)
+    s = r.lognormal(0.0, 1.0, size=(T, n_groups))
+    hot = r.random(T) < 1e-3
+    s[hot] *= 1e6
+    return s.astype(np.float32)
+
+
 # --------------------------------------------------------------------------
 # small free-form cases for tests
 # --------------------------------------------------------------------------

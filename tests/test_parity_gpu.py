@@ -653,3 +653,51 @@ def test_grouped_sweep_exact_hessians():
         rep = compare_codes(codes_np, orc, 64, 64, lr is not None)
         print(f"\ngrouped exact-H lr={lr}: {rep}")
         assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
+
+
+def test_block_scheduler_saliency_groups():
+    # the scheduler's grouped variant on a small two-input block: every module
+    # matches the oracle's row-grouped sweep from its own clipped saliency
+    from paper_2609_00049_gb300.block import BlockInput, BlockModule, BlockQuantizer
+    r = synth.rng(60, "block-grouped")
+    T, ng = 6000, 4
+    ins = {"a": 128, "b": 256}
+    mods = [("m1", 64, "a"), ("m2", 128, "a"), ("m3", 96, "b")]
+    x_bits = {k: synth.f32_to_bf16_bits(r.standard_normal((T, n)) * (1 + 9 * (r.random(n) < 0.02)))
+              for k, n in ins.items()}
+    Wf = {nm: synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(r.standard_normal((m, ins[i])) * 0.02))
+          for nm, m, i in mods}
+    Ff, Sal = {}, {}
+    for nm, m, _ in mods:
+        z = r.standard_normal((m, 4))
+        Ff[nm] = (np.eye(m) * 0.5 + z @ z.T / 8).astype(np.float32)
+        s = np.exp(0.7 * r.standard_normal((T, ng)))
+        s[r.integers(0, T, 4)] *= 1e7
+        Sal[nm] = s.astype(np.float32)
+    qcfg = rq.quant_cfg(4, 64, 64, 0, 0.01)
+    bq = BlockQuantizer([BlockInput(k, n, T) for k, n in ins.items()],
+                        [BlockModule(nm, m, ins[i], i) for nm, m, i in mods], qcfg, 2e-4, 1, saliency_groups=ng)
+    bq.run({k: bf16_dev(v) for k, v in x_bits.items()}, {nm: dev(w) for nm, w in Wf.items()},
+           {nm: dev(f) for nm, f in Ff.items()}, saliency={nm: dev(v) for nm, v in Sal.items()})
+    torch.cuda.synchronize()
+    bq.check_status()
+    bstart = 1
+    for nm, m, i in mods:
+        x = synth.bf16_bits_to_f32(x_bits[i]).astype(np.float64)
+        Sc, _ = oracle.saliency_clip(Sal[nm].astype(np.float64), 0.99)
+        Hg, w = oracle.weighted_hessian_sum([x], [Sc])
+        Hs, _ = oracle.hessian_sum([x])
+        orc = oracle.realq_sweep(Wf[nm].astype(np.float64), Hs, T, group_size=64, block_size=64,
+                                 bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": bstart, "B_total": 1},
+                                 F=Ff[nm], obs_hessians=[(Hg[g], w[g]) for g in range(ng)])
+        bstart += ins[i] // 64
+        o = bq.out[nm]
+        codes = unpack(o["codes"].cpu().numpy(), ins[i])
+        rep = compare_codes(codes, orc, 64, 64, True)
+        qkw = dict(group_size=64, block_size=64)
+        frac, med, s_unexpl = scale_agreement(o["scale"].cpu().numpy(), orc["scale"], 64,
+                                              explained=compare_codes.last_explained,
+                                              adam_bound=_adam_scale_bound(orc, ins[i], qkw, 2e-4, 1))
+        print(f"\nblock grouped {nm}: {rep} scale_within_1e-5={frac:.5f}")
+        assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (nm, rep)
+        assert s_unexpl == 0
