@@ -254,7 +254,7 @@ def gpu_arm(args, wl, rank, world):
     result = None
     if rank == 0:
         peaks = load_peaks()
-        roof = roofline(wl, prof, args.steps, peaks)
+        roof = roofline(wl, prof, args.steps, peaks, args)
         result = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
@@ -282,7 +282,7 @@ def gpu_arm(args, wl, rank, world):
     return result
 
 
-def roofline(wl, prof, steps, peaks):
+def roofline(wl, prof, steps, peaks, args=None):
     """Roofline entry for the kernel with the largest share of device time."""
     if not prof:
         return None
@@ -292,6 +292,18 @@ def roofline(wl, prof, steps, peaks):
     hess_flops = sum(s.T * s.n * (s.n + 1) for s in wl.inputs.values())       # symmetric X^T X
     per_step["hessian_syrk_simt"] = ("tensor", hess_flops, "TFLOP/s")
     per_step["hessian_syrk_tc"] = ("tensor", hess_flops, "TFLOP/s")
+    ng = getattr(args, "saliency_groups", 0) or 0
+    if ng:
+        # per module and row group: X̂ᵀ (s X̂) as two bf16 passes (high and low
+        # part of s x) over the lower tiles
+        wflops = sum(2 * wl.inputs[md.input].T * md.n * (md.n + 1) * ng for md in wl.modules)
+        per_step["hessian_weighted_tc"] = ("tensor", wflops, "TFLOP/s")
+        per_step["saliency_scale"] = ("hbm", sum(wl.inputs[md.input].T * md.n * 6 * ng for md in wl.modules),
+                                      "GB/s")
+    if getattr(args, "act_bits", 0):
+        # D = X̂ᵀX̂ - XᵀX̂: the full non-symmetric product XᵀX̂ per input
+        per_step["hessian_cross_tc"] = ("tensor", sum(2 * s.T * s.n * s.n for s in wl.inputs.values()), "TFLOP/s")
+        per_step["act_quant"] = ("hbm", sum(s.T * s.n * 2 * 3 for s in wl.inputs.values()), "GB/s")
     bgd_p = bgd_g = trail = 0
     serial_bytes = 0
     for md in wl.modules:
