@@ -258,7 +258,13 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
       steps_per_block (1 in the paper), lr, beta1, beta2, eps,
       optimizer ("adam" | "sgd"), b_global_start (1-based cumulative block index
       of this module's first block), B_total (column-block steps in the
-      transformer block; 1 disables the sliding window).
+      transformer block; 1 disables the sliding window), and optionally
+      minibatches: a list of K pairs (H_mb_sum, T_mb), the second moments of
+      calibration mini-batches (Sec. 4.3: each Block-GD step evaluates the
+      surrogate on a calibration mini-batch; Sec. 5.1: 32 sequences).  Step s
+      (0-based) of the block with global index b_global uses mini-batch
+      ((b_global - 1) * steps_per_block + s) mod K, so consecutive steps of a
+      transformer block rotate through the calibration set.
 
     Readings: group parameters are computed at the first column of each group
     from the current (compensated, Block-GD-updated) weights; group_size 0
@@ -338,8 +344,16 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             alpha = sliding_alpha(b_global, bgd.get("B_total", 1))
             Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
             before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
-            for _ in range(bgd.get("steps_per_block", 1)):
-                G = gradient(W, W0, Hbar, Dbar, Feff)[:, be:]
+            mbs = bgd.get("minibatches")
+            steps = bgd.get("steps_per_block", 1)
+            for si in range(steps):
+                Hstep = Hbar
+                if mbs:
+                    if Dbar is not None:
+                        raise ValueError("mini-batch moments with perturbed inputs are not supported")
+                    Hk, Tk = mbs[((b_global - 1) * steps + si) % len(mbs)]
+                    Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)
+                G = gradient(W, W0, Hstep, Dbar, Feff)[:, be:]
                 if bgd.get("optimizer", "adam") == "sgd":
                     opt.t += 1
                     W[:, be:] -= bgd["lr"] * G

@@ -519,3 +519,35 @@ def test_saliency_clipping_prevents_rank_one_collapse():
     Hc, _ = oracle.weighted_hessian_sum([X], [Sc])
     ev = np.linalg.eigvalsh(Hc[0])
     assert ev[-1] / ev.sum() < 0.2
+
+
+# ------------------------------------------------- mini-batch Block-GD ---
+def test_minibatch_of_all_tokens_is_the_full_batch():
+    r, X, W0, F = _grouped_case(66)
+    H, T = oracle.hessian_sum([X])
+    base = {"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
+    a = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, bgd=base, F=F)
+    b = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, bgd={**base, "minibatches": [(H, T)]}, F=F)
+    assert np.array_equal(a["codes"], b["codes"]) and np.array_equal(a["deq"], b["deq"])
+
+
+def test_minibatch_rotation_rule():
+    # two mini-batches, the second with no second moment: steps that draw it
+    # see a zero gradient and Adam does not move (m = v = 0 there); the
+    # rotation (b_global - 1) * steps + s mod 2 decides which blocks move
+    r, X, W0, F = _grouped_case(67)
+    H, T = oracle.hessian_sum([X])
+    zero = np.zeros_like(H)
+    for start in (1, 2):
+        bgd = {"lr": 2e-4, "steps_per_block": 1, "b_global_start": start, "B_total": 1,
+               "minibatches": [(H, T), (zero, T)]}
+        res = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, bgd=bgd, F=F)
+        gptq = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16)
+        # block 0's step is the first optimizer step: it moves only if it
+        # draws mini-batch 0, i.e. when b_global_start is odd
+        moved_first = start % 2 == 1
+        assert (not np.array_equal(res["codes"][:, 16:32], gptq["codes"][:, 16:32])
+                or not np.array_equal(res["deq"][:, 16:32], gptq["deq"][:, 16:32])) == moved_first
+    # the mean of the mini-batch moments is the full-batch moment
+    Hs = [oracle.hessian_sum([X[k * 100:(k + 1) * 100]])[0] for k in range(4)]
+    np.testing.assert_allclose(sum(Hs) / T, H / T, rtol=1e-13, atol=1e-15)
