@@ -157,7 +157,7 @@ def gpu_arm(args, wl, rank, world):
                         [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
                         wl.steps_per_block, sliding_window=wl.sliding_window, device=dev,
                         act_quant=(args.act_bits, args.a_clip) if args.act_bits else None,
-                        saliency_groups=args.saliency_groups)
+                        saliency_groups=args.saliency_groups, minibatch_tokens=2048 * args.minibatch_seqs)
     dev_sal = None
     if args.saliency_groups:
         dev_sal = {mod.name: torch.from_numpy(synth.saliency(wl, mod, args.saliency_groups)).to(dev)
@@ -230,7 +230,7 @@ def gpu_arm(args, wl, rank, world):
 
     # ---- end to end through host buffers
     e2e = None
-    if not args.no_e2e and not args.act_bits and not args.saliency_groups:
+    if not args.no_e2e and not args.act_bits and not args.saliency_groups and not args.minibatch_seqs:
         step_e2e()
         torch.cuda.synchronize()
         barrier()
@@ -268,7 +268,8 @@ def gpu_arm(args, wl, rank, world):
                                     f" {'sym' if wl.symmetric else 'asym'} g{wl.group_size} B{wl.block_size}" +
                                     (f", saliency-weighted grouped Hessians (N_g={args.saliency_groups}, clip p99)"
                                      if args.saliency_groups else ""),
-                       "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}",
+                       "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}" +
+                              (f", mini-batches of {args.minibatch_seqs} x 2048 tokens" if args.minibatch_seqs else ""),
                        "parallelism": f"replicas x{world}",
                        "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
                              (sum(s.T * s.n * 2 for s in wl.inputs.values()) / 1e9),
@@ -487,6 +488,8 @@ def main():
     ap.add_argument("--act-bits", type=int, default=0,
                     help="activation-aware weight-activation variant: per-token activation bits (0: weights only)")
     ap.add_argument("--a-clip", type=float, default=0.9, help="activation clipping ratio for --act-bits")
+    ap.add_argument("--minibatch-seqs", type=int, default=0,
+                    help="mini-batch Block-GD with this many 2048-token sequences per step (0: full batch)")
     ap.add_argument("--saliency-groups", type=int, default=0,
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--no-cpu-baseline", action="store_true")

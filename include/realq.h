@@ -288,6 +288,30 @@ realq_status_t realq_quantize_layer_grouped(realq_stream_t stream, int64_t m, in
                                             int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero,
                                             void *W_deq, realq_dtype_t deq_dtype, int64_t block_begin,
                                             int64_t block_end, void *ws, size_t ws_bytes);
+
+/* The sweep with mini-batch Block-GD (Sec. 4.3: each Block-GD step evaluates
+ * the surrogate on a calibration mini-batch; Sec. 5.1: 32 sequences per
+ * step).  Hbar_mb holds n_minibatch second moments H̄_k = X̂_kᵀX̂_k / T_k
+ * (n_minibatch x n x n, one per mini-batch of the calibration set, e.g. from
+ * realq_hessian_accumulate and realq_scale_moment on each mini-batch).  Step
+ * s (0-based) of block b takes mini-batch ((b_global - 1) steps_per_block + s)
+ * mod n_minibatch, with b_global = bcfg->b_global_start + b, so the steps of a
+ * transformer block rotate through the calibration set; its gradient is
+ * F_eff ((Ŵ - W0) H̄_k) on the free columns.  The OBS part still uses U and
+ * the full Hbar.  Needs Block-GD on the tensor-core path (m, n multiples of
+ * 4, at least 32) and unperturbed inputs (no Dbar).  Everything else as
+ * realq_quantize_layer; the workspace comes from
+ * realq_quantize_minibatch_workspace_size. */
+size_t realq_quantize_minibatch_workspace_size(int64_t m, int64_t n, int n_minibatch, const realq_quant_cfg_t *qcfg,
+                                               const realq_bgd_cfg_t *bcfg, int has_F_next);
+realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                              realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                              const uint8_t *dead, int n_minibatch, const float *Hbar_mb,
+                                              const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg,
+                                              const float *F, const float *F_next, float *W_work, float *adam_m,
+                                              float *adam_v, float *bgd_disp, int64_t *adam_t, uint8_t *codes,
+                                              float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
+                                              int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes);
 size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg_t *qcfg,
                                      const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar);
 

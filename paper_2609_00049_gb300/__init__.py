@@ -22,7 +22,8 @@ __all__ = [
     "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
     "realq_quantize_activations", "realq_saliency_clip", "realq_hessian_weighted_workspace_size",
     "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled", "realq_quantize_layer_grouped",
-    "realq_quantize_grouped_workspace_size",
+    "realq_quantize_grouped_workspace_size", "realq_quantize_layer_minibatch",
+    "realq_quantize_minibatch_workspace_size",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -91,6 +92,11 @@ _SIGS = {
     "realq_quantize_layer_grouped": ([_vp, _i64, _i64, _vp, _int, _int, _vp, _vp, _vp, _vp, _vp,
                                       ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp,
                                       _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
+    "realq_quantize_minibatch_workspace_size": ([_i64, _i64, _int, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
+                                                 _int], _sz),
+    "realq_quantize_layer_minibatch": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _int, _vp,
+                                        ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp,
+                                        _vp, _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_layer": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
                               ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp, _int,
                               _i64, _i64, _vp, _sz], _int),
@@ -368,6 +374,40 @@ def realq_quantize_layer_grouped(W0: torch.Tensor, U_g: torch.Tensor, Hbar_g: Op
         _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale),
         _ptr(zero), _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end),
         wp, wb))
+    return t.value
+
+
+def realq_quantize_minibatch_workspace_size(m: int, n: int, n_minibatch: int, qcfg: QuantCfg,
+                                            bcfg: Optional[BgdCfg] = None, has_F_next: bool = False) -> int:
+    return int(lib().realq_quantize_minibatch_workspace_size(m, n, n_minibatch, ctypes.byref(qcfg),
+                                                             ctypes.byref(bcfg) if bcfg is not None else None,
+                                                             int(has_F_next)))
+
+
+def realq_quantize_layer_minibatch(W0: torch.Tensor, U: torch.Tensor, Hbar: torch.Tensor, Hbar_mb: torch.Tensor,
+                                   qcfg: QuantCfg, W_work: torch.Tensor, codes: torch.Tensor, scale: torch.Tensor,
+                                   zero: torch.Tensor, *, dead=None, bcfg: Optional[BgdCfg] = None, F=None,
+                                   F_next=None, adam_m=None, adam_v=None, bgd_disp=None, adam_t: int = 0, W_deq=None,
+                                   block_begin: int = 0, block_end: Optional[int] = None, ws=None,
+                                   stream=None) -> int:
+    """The sweep with Block-GD steps on rotating calibration mini-batches; returns the Adam step counter."""
+    m, n = W0.shape
+    nmb = Hbar_mb.shape[0]
+    if block_end is None:
+        block_end = -(-n // qcfg.block_size)
+    _need(Hbar_mb, torch.float32, (nmb, n, n), "Hbar_mb")
+    _need(U, torch.float32, (n, n), "U")
+    _need(W_work, torch.float32, (m, n), "W_work")
+    _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
+    for t_, nm in ((adam_m, "adam_m"), (adam_v, "adam_v"), (bgd_disp, "bgd_disp")):
+        _need(t_, torch.float32, (m, n), nm)
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    _check(lib().realq_quantize_layer_minibatch(
+        _stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar), _ptr(dead), nmb, _ptr(Hbar_mb),
+        ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next), _ptr(W_work),
+        _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
+        _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
     return t.value
 
 

@@ -26,8 +26,8 @@ from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_he
                realq_hessian_prepare, realq_hessian_prepare_scaled, realq_hessian_weighted_workspace_size,
                realq_hessian_workspace_size, realq_prepare_workspace_size, realq_quantize_activations,
                realq_quantize_grouped_workspace_size, realq_quantize_layer, realq_quantize_layer_grouped,
-               realq_quantize_workspace_size, realq_saliency_clip, realq_scale_moment, realq_workspace_status,
-               workspace)
+               realq_quantize_layer_minibatch, realq_quantize_minibatch_workspace_size, realq_quantize_workspace_size,
+               realq_saliency_clip, realq_scale_moment, realq_workspace_status, workspace)
 
 
 @dataclass
@@ -61,6 +61,11 @@ class BlockQuantizer:
     taken over the quantized activations, and the Block-GD surrogate keeps
     the full-precision ones through the cross moment D.
 
+    minibatch_tokens=T_mb > 0 selects mini-batch Block-GD (Sec. 4.3, 32
+    sequences per step in Sec. 5.1): every input's tokens form consecutive
+    mini-batches of T_mb tokens, whose second moments the optimizer steps
+    rotate through; the OBS keeps the full H.
+
     saliency_groups=N_g > 0 selects the saliency-weighted grouped Hessians
     (Sec. 3.3, Alg. 1 "for all row-groups g"): every module's rows form N_g
     groups, run() takes a (T x N_g) saliency per module, clipped to its
@@ -71,7 +76,7 @@ class BlockQuantizer:
     def __init__(self, inputs: Sequence[BlockInput], modules: Sequence[BlockModule], qcfg: QuantCfg, lr: float,
                  steps_per_block: int = 1, sliding_window: bool = False, device="cuda",
                  host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None, saliency_groups: int = 0,
-                 saliency_pct: float = 0.99):
+                 saliency_pct: float = 0.99, minibatch_tokens: int = 0):
         self.inputs: Dict[str, BlockInput] = {i.name: i for i in inputs}
         self.modules: List[BlockModule] = list(modules)
         for md in self.modules:
@@ -85,6 +90,9 @@ class BlockQuantizer:
         self.act_quant = act_quant
         self.sgroups = saliency_groups
         self.spct = saliency_pct
+        self.mb_tokens = minibatch_tokens
+        if minibatch_tokens and (saliency_groups or act_quant is not None):
+            raise ValueError("mini-batch Block-GD is built for the plain, unperturbed sweep")
         self.mods_of = {name: [md for md in self.modules if md.input == name] for name in self.inputs}
         B = qcfg.block_size
         self.B_total = sum(-(-md.n // B) for md in self.modules)
@@ -97,6 +105,10 @@ class BlockQuantizer:
                 dead=torch.empty(n, dtype=torch.uint8, device=dev),
                 pws=workspace(realq_prepare_workspace_size(n), dev),
                 hws=workspace(realq_hessian_workspace_size(n, spec.T, REALQ_BF16, act_quant is not None), dev))
+            if minibatch_tokens:
+                nmb = -(-spec.T // minibatch_tokens)
+                self.state[name].update(Hk=torch.empty(n, n, device=dev), Hmb=torch.empty(nmb, n, n, device=dev),
+                                        kws=workspace(realq_hessian_workspace_size(n, minibatch_tokens), dev))
             if act_quant is not None:
                 self.state[name].update(Xq=torch.empty(spec.T, n, dtype=torch.bfloat16, device=dev),
                                         D=torch.empty(n, n, device=dev), Dbar=torch.empty(n, n, device=dev))
@@ -124,6 +136,10 @@ class BlockQuantizer:
                            wsum=torch.empty(ngs, dtype=torch.float64, device=dev),
                            wws=workspace(realq_hessian_weighted_workspace_size(n, self.inputs[md.input].T), dev),
                            pws=workspace(realq_prepare_workspace_size(n), dev))
+            elif minibatch_tokens and bgd:
+                nmb = -(-self.inputs[md.input].T // minibatch_tokens)
+                ws_q = workspace(realq_quantize_minibatch_workspace_size(m, n, nmb, qcfg, bc, sliding_window), dev)
+                grp = None
             else:
                 ws_q = workspace(realq_quantize_workspace_size(m, n, qcfg, bc if bgd else None, sliding_window,
                                                                act_quant is not None and bgd), dev)
@@ -173,6 +189,12 @@ class BlockQuantizer:
                 F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"], bgd_disp=o["disp"],
                 ws=o["ws"], stream=stream)
             return
+        if self.mb_tokens and o["bcfg"] is not None:
+            o["adam_t"] = realq_quantize_layer_minibatch(
+                W0, s_in["U"], s_in["Hbar"], s_in["Hmb"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"],
+                dead=s_in["dead"], bcfg=o["bcfg"], F=F, F_next=F_next if self.sliding_window else None,
+                adam_m=o["am"], adam_v=o["av"], bgd_disp=o["disp"], ws=o["ws"], stream=stream)
+            return
         o["adam_t"] = realq_quantize_layer(
             W0, s_in["U"], s_in["Hbar"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"],
             Dbar=s_in.get("Dbar") if o["bcfg"] is not None else None, dead=s_in["dead"],
@@ -204,6 +226,15 @@ class BlockQuantizer:
             return
         if self.act_quant is None:
             realq_hessian_accumulate(X, s_in["H"], ws=s_in["hws"], stream=stream)
+            if self.mb_tokens:
+                # second moments of the consecutive mini-batches
+                C = self.mb_tokens
+                for k in range(s_in["Hmb"].shape[0]):
+                    with torch.cuda.stream(stream if stream is not None else torch.cuda.current_stream(self.device)):
+                        s_in["Hk"].zero_()
+                    rows = min(C, spec.T - k * C)
+                    realq_hessian_accumulate(X[k * C:k * C + rows], s_in["Hk"], ws=s_in["kws"], stream=stream)
+                    realq_scale_moment(s_in["Hk"], rows, s_in["Hmb"][k], stream=stream)
         else:
             bits, clip = self.act_quant
             realq_quantize_activations(X, bits, clip, X_q=s_in["Xq"], stream=stream)

@@ -314,7 +314,7 @@ size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg
 
 static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
                                     int grouped, int rgroups, const float *Ug, const float *Hbar_g,
-                                    const uint8_t *dead_g,
+                                    const uint8_t *dead_g, int nmb, const float *Hbar_mb,
                                     const float *U, const float *Hbar, const float *Dbar, const uint8_t *dead,
                                     const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg, const float *F,
                                     const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
@@ -334,7 +334,7 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
             return fail(REALQ_ERR_INVALID_ARG, "%s: Block-GD needs Hbar, F, bgd_disp and adam_t", who);
         if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
             return fail(REALQ_ERR_INVALID_ARG, "%s: Adam needs adam_m and adam_v", who);
-        if (grouped && !(qcfg->block_size > 0 && tc_gemm_eligible(m, n)))
+        if ((grouped || nmb > 0) && !(qcfg->block_size > 0 && tc_gemm_eligible(m, n)))
             return fail(REALQ_ERR_UNSUPPORTED,
                         "%s: Block-GD with row groups needs m and n multiples of 4 and at least 32", who);
     }
@@ -344,8 +344,11 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
                     (long long)block_begin, (long long)block_end, (long long)nb);
     const int has_fn = bgd && F_next != nullptr;
     const int has_db = bgd && Dbar != nullptr;
+    if (nmb > 0 && bgd && (Dbar || grouped))
+        return fail(REALQ_ERR_UNSUPPORTED, "%s: mini-batch moments with perturbed inputs or row groups", who);
     REALQ_TRY(check_ws(ws, ws_bytes,
-                       sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db, grouped ? rgroups : 0), who));
+                       sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db, grouped ? rgroups : 0,
+                                      bgd ? nmb : 0), who));
 
     SweepPlan p{};
     p.m = m; p.n = n; p.W0 = W0; p.w_dtype = w_dtype;
@@ -356,6 +359,8 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     p.Ug = grouped ? Ug : U;
     p.Hbar_g = grouped ? Hbar_g : nullptr;
     p.dead_g = grouped ? dead_g : nullptr;
+    p.nmb = bgd ? nmb : 0;
+    p.Hbar_mb = bgd ? Hbar_mb : nullptr;
     p.bits = qcfg->bits; p.block = qcfg->block_size; p.sym = qcfg->symmetric;
     p.group = effective_group(qcfg, n);
     p.ngroups = (int)((n + p.group - 1) / p.group);
@@ -384,7 +389,8 @@ realq_status_t realq_quantize_layer(realq_stream_t stream, int64_t m, int64_t n,
                                     int64_t *adam_t,
                                     uint8_t *codes, float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
                                     int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
-    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, U, Hbar, Dbar, dead, qcfg, bcfg, F,
+    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, Hbar, Dbar, dead, qcfg,
+                         bcfg, F,
                          F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq, deq_dtype,
                          block_begin, block_end, ws, ws_bytes, "quantize_layer");
 }
@@ -410,9 +416,32 @@ realq_status_t realq_quantize_layer_grouped(realq_stream_t stream, int64_t m, in
     if (!U_g || !dead_g) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_grouped: NULL U_g or dead_g");
     const int bgd = bcfg && bcfg->steps_per_block > 0;
     if (bgd && !Hbar_g) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_grouped: Block-GD needs Hbar_g");
-    return quantize_impl(stream, m, n, W0, w_dtype, 1, n_row_groups, U_g, Hbar_g, dead_g, U_g, Hbar, Dbar, dead_g, qcfg,
+    return quantize_impl(stream, m, n, W0, w_dtype, 1, n_row_groups, U_g, Hbar_g, dead_g, 0, nullptr, U_g, Hbar, Dbar,
+                         dead_g, qcfg,
                          bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq,
                          deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_grouped");
+}
+
+size_t realq_quantize_minibatch_workspace_size(int64_t m, int64_t n, int n_minibatch, const realq_quant_cfg_t *qcfg,
+                                               const realq_bgd_cfg_t *bcfg, int has_F_next) {
+    if (m <= 0 || n <= 0 || !qcfg || n_minibatch <= 0) return 0;
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, 0, 0, bgd ? n_minibatch : 0);
+}
+
+realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                              realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                              const uint8_t *dead, int n_minibatch, const float *Hbar_mb,
+                                              const realq_quant_cfg_t *qcfg, const realq_bgd_cfg_t *bcfg,
+                                              const float *F, const float *F_next, float *W_work, float *adam_m,
+                                              float *adam_v, float *bgd_disp, int64_t *adam_t, uint8_t *codes,
+                                              float *scale, uint8_t *zero, void *W_deq, realq_dtype_t deq_dtype,
+                                              int64_t block_begin, int64_t block_end, void *ws, size_t ws_bytes) {
+    if (n_minibatch <= 0 || !Hbar_mb)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_minibatch: n_minibatch >= 1 and Hbar_mb required");
+    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, n_minibatch, Hbar_mb, U, Hbar,
+                         nullptr, dead, qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale,
+                         zero, W_deq, deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_minibatch");
 }
 
 // ---------------------------------------------------------------- BGD -----

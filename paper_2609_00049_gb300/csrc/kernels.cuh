@@ -153,10 +153,17 @@ struct SweepPlan {
     float *lam_g;                               // lambda_g per group (workspace)
     float *HGh, *HGl, *GGh, *GGl, *DWh, *DWl;   // tf32 planes of H̄_g, H̄_g - H̄, W - W0
     std::vector<TcMaps> mapsMg, mapsQg;
+    // mini-batch Block-GD: step s of block b draws mini-batch
+    // ((b_global - 1) steps + s) mod nmb, with moment H̄_mb (nmb x n x n)
+    int nmb;
+    const float *Hbar_mb;
+    float *MBh, *MBl;                           // tf32 planes of H̄ - H̄_mb,k
+    std::vector<TcMaps> mapsMB;
     int f_split_alpha_valid;
     float f_split_alpha;
 };
-size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0);
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0,
+                      int nmb = 0);
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);
 realq_status_t sweep_init(cudaStream_t s, SweepPlan &p);
 realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b);

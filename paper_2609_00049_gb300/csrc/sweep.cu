@@ -377,7 +377,8 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 // and need hi / lo planes of the displacement, H̄, F and P^T; otherwise the
 // fp32 SIMT path needs P, G (and F_eff).  block = 0: Block-GD only (literal
 // gradient form, SIMT).
-size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups) {
+size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups,
+                      int nmb) {
     const size_t mn = align_up((size_t)m * n * sizeof(float));
     const size_t nn = align_up((size_t)n * n * sizeof(float));
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
@@ -386,6 +387,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
         if (block > 0 && tc_gemm_eligible(m, n)) {
             b += 5 * mn + 2 * nn + 2 * align_up((size_t)m * m * sizeof(float));
             if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
+            if (nmb > 0) b += (rgroups > 0 ? 0 : 2 * mn) + 2 * (size_t)nmb * nn;
         } else {
             b += 2 * mn;
             if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
@@ -403,7 +405,7 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
     p.Et = cv.take<float>((size_t)p.block * p.m);
     p.P = p.G = p.Feff = p.R0 = nullptr;
     p.Sh = p.Sl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = p.M = nullptr;
-    p.HGh = p.HGl = p.GGh = p.GGl = p.DWh = p.DWl = nullptr;
+    p.HGh = p.HGl = p.GGh = p.GGl = p.DWh = p.DWl = p.MBh = p.MBl = nullptr;
     p.lam_g = p.grouped ? cv.take<float>((size_t)p.rgroups) : nullptr;
     p.step_c = p.n;
     p.tc = 0;
@@ -419,6 +421,14 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
             p.Hl = cv.take<float>((size_t)p.n * p.n);
             p.Fh = cv.take<float>((size_t)p.m * p.m);
             p.Fl = cv.take<float>((size_t)p.m * p.m);
+            if (p.nmb > 0) {
+                p.MBh = cv.take<float>((size_t)p.nmb * p.n * p.n);
+                p.MBl = cv.take<float>((size_t)p.nmb * p.n * p.n);
+                if (!p.grouped) {
+                    p.DWh = cv.take<float>(mn);
+                    p.DWl = cv.take<float>(mn);
+                }
+            }
             if (p.grouped) {
                 p.DWh = cv.take<float>(mn);
                 p.DWl = cv.take<float>(mn);
@@ -613,6 +623,43 @@ static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c
     return REALQ_OK;
 }
 
+// One optimizer step on a calibration mini-batch: the gradient factor is
+// ((Ŵ - W0) H̄_mb)_R = (stationarity form with H̄)_R + (ΔW (H̄_mb - H̄))_R,
+// i.e. M + lambda (A - ΔW) - ΔW (H̄ - H̄_mb,k), with M = A H̄ kept current.
+static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, int kmb) {
+    const int64_t r = p.n - c0;
+    const int64_t k0 = p.step_c;
+    if (p.w_dtype == REALQ_BF16)
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const __nv_bfloat16 *>(p.W0), p.DWh, p.DWl));
+    else
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const float *>(p.W0), p.DWh, p.DWl));
+    if (k0 < p.n) {
+        TcEpi e{};
+        e.mode = TC_ACCUM;
+        e.M = p.M; e.ldw = p.n; e.col0 = c0;
+        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm"));
+    }
+    TcEpi q{};
+    q.mode = TC_BGD_PG;
+    q.Ad = p.disp; q.W = p.W; q.W0 = p.W0; q.w0_bf16 = p.w_dtype == REALQ_BF16;
+    q.dead = p.dead; q.lam = p.lam; q.R0 = nullptr;
+    q.ldw = p.n; q.col0 = c0; q.M = p.M;
+    q.Pth = p.Pth; q.Ptl = p.Ptl; q.ldp = p.m;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMB[kmb], p.m, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm"));
+    const int64_t t = ++(*p.adam_t);
+    TcEpi g{};
+    g.mode = TC_ADAM;
+    g.ldw = p.n; g.col0 = c0;
+    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
+    g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
+    g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
+    g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
+    g.sgd = p.optimizer == REALQ_OPT_SGD;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    p.step_c = c0;
+    return REALQ_OK;
+}
+
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
     if (col_start >= p.n) return REALQ_OK;
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
@@ -688,8 +735,12 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             p.f_split_alpha_valid = 1;
             p.f_split_alpha = a_eff;
         }
-        for (int k = 0; k < p.bgd_steps; ++k)
-            REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be) : bgd_one_tc(s, p, be));
+        for (int k = 0; k < p.bgd_steps; ++k) {
+            if (p.nmb > 0)
+                REALQ_TRY(bgd_one_tc_mb(s, p, be, (int)(((b_global - 1) * p.bgd_steps + k) % p.nmb)));
+            else
+                REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be) : bgd_one_tc(s, p, be));
+        }
         return REALQ_OK;
     }
     const float *Fuse = nullptr;
@@ -733,6 +784,16 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
                 REALQ_TRY(tc_make_maps(&p.mapsMg[gr], p.Sh, p.Sl, p.m, p.n, p.n, p.HGh + gr * nn, p.HGl + gr * nn, p.n,
                                        p.n, p.n));
                 REALQ_TRY(tc_make_maps(&p.mapsQg[gr], p.DWh, p.DWl, p.m, p.n, p.n, p.GGh + gr * nn, p.GGl + gr * nn,
+                                       p.n, p.n, p.n));
+            }
+        }
+        if (p.nmb > 0) {
+            // planes of H̄ - H̄_mb,k and the maps of the correction product
+            const size_t nn = (size_t)p.n * p.n;
+            p.mapsMB.assign(p.nmb, TcMaps{});
+            for (int k = 0; k < p.nmb; ++k) {
+                REALQ_TRY(tc_split_diff(s, (int64_t)nn, p.Hbar, p.Hbar_mb + k * nn, p.MBh + k * nn, p.MBl + k * nn));
+                REALQ_TRY(tc_make_maps(&p.mapsMB[k], p.DWh, p.DWl, p.m, p.n, p.n, p.MBh + k * nn, p.MBl + k * nn,
                                        p.n, p.n, p.n));
             }
         }

@@ -701,3 +701,43 @@ def test_block_scheduler_saliency_groups():
         print(f"\nblock grouped {nm}: {rep} scale_within_1e-5={frac:.5f}")
         assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (nm, rep)
         assert s_unexpl == 0
+
+
+# ------------------------------------------------- mini-batch Block-GD ---
+@pytest.mark.parametrize("start,steps", [(1, 1), (3, 1), (2, 2)])
+def test_minibatch_block_gd(start, steps):
+    case = synth.layer_case(61, 128, 384, 8000, bf16=True, outliers=3)
+    K, Tm = 4, 2000
+    qkw = dict(group_size=128, block_size=128)
+    mbs = [oracle.hessian_sum([case.Xhat[k * Tm:(k + 1) * Tm]]) for k in range(K)]
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1, "minibatches": mbs}
+    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd, F=case.F)
+    X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
+    H, _, _ = layer.accumulate([X], 384)
+    prep = layer.prepare(H, T)
+    Hmb = torch.empty(K, 384, 384, device="cuda")
+    for k in range(K):
+        Hk, _, _ = layer.accumulate([X[k * Tm:(k + 1) * Tm]], 384)
+        rq.realq_scale_moment(Hk, Tm, Hmb[k])
+    q = rq.quant_cfg(**qkw)
+    b = rq.bgd_cfg(2e-4, steps_per_block=steps, b_global_start=start)
+    m, n = 128, 384
+    W = torch.empty(m, n, device="cuda")
+    codes = torch.empty(m, n // 2, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(m, 3, device="cuda")
+    zero = torch.empty(m, 3, dtype=torch.uint8, device="cuda")
+    st = {k: torch.empty(m, n, device="cuda") for k in ("adam_m", "adam_v", "bgd_disp")}
+    ws = rq.workspace(rq.realq_quantize_minibatch_workspace_size(m, n, K, q, b))
+    t = rq.realq_quantize_layer_minibatch(dev(case.W0), prep.U, prep.Hbar, Hmb, q, W, codes, scale, zero,
+                                          dead=prep.dead, bcfg=b, F=dev(case.F), ws=ws, **st)
+    rq.realq_workspace_status(ws)
+    assert t == orc["adam_t"] == 2 * steps
+    c = unpack(codes.cpu().numpy(), n)
+    rep = compare_codes(c, orc, 128, 128, True)
+    frac, med, s_unexpl = scale_agreement(scale.cpu().numpy(), orc["scale"], 128,
+                                          explained=compare_codes.last_explained,
+                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, steps))
+    print(f"\nmini-batch start={start} steps={steps}: {rep} scale_within_1e-5={frac:.5f}")
+    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
+    assert s_unexpl == 0
