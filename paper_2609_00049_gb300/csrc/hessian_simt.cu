@@ -179,17 +179,33 @@ realq_status_t hessian_reduce(cudaStream_t s, int64_t n, int splits, const float
 }
 
 int hessian_splits(int64_t n, int64_t T, int sms) {
-    const int nt = ceil_div(n, TB);
-    return hessian_splits_tiles((int64_t)nt * (nt + 1) / 2, T, sms);
+    // tiles of the tensor-core symmetric product: 128-channel row blocks by
+    // 256-channel column blocks reaching the diagonal
+    const int nti = ceil_div(n, 128);
+    int64_t tiles = 0;
+    for (int r = 0; r < nti; ++r) tiles += r / 2 + 1;
+    return hessian_splits_tiles(tiles, T, sms);
 }
 
-int hessian_splits_tiles(int64_t lower, int64_t T, int sms) {
-    int64_t want = (sms + lower / 2) / lower;       // nearest whole number of waves
-    const int64_t by_tokens = T / 4096;              // at least 4096 tokens per split
-    if (want > by_tokens) want = by_tokens;
-    if (want > 16) want = 16;
-    if (want < 1) want = 1;
-    return (int)want;
+// Token splits of a tile grid: the count that minimises the rounds of waves
+// per unit of work, ceil(tiles s / sms) / s, plus a small cost per split for
+// the partial sums and their reduction; at least 4096 tokens per split and at
+// most 16 splits.
+int hessian_splits_tiles(int64_t tiles, int64_t T, int sms) {
+    int64_t max_s = T / 4096;
+    if (max_s > 16) max_s = 16;
+    if (max_s < 1) max_s = 1;
+    double best = 1e300;
+    int bs = 1;
+    for (int s2 = 1; s2 <= max_s; ++s2) {
+        const int64_t rounds = (tiles * s2 + sms - 1) / sms;
+        const double cost = (double)rounds / s2 + 0.01 * s2;
+        if (cost < best - 1e-12) {
+            best = cost;
+            bs = s2;
+        }
+    }
+    return bs;
 }
 
 size_t hessian_ws_bytes(int64_t n, int64_t T, int has_xfp) {

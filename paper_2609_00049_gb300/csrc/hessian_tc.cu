@@ -1,26 +1,30 @@
 // Step a2 (Sec. 3.2) on the 5th-generation tensor cores: H_sum += X̂^T X̂ for
 // bf16 calibration activations.
 //
-// One CTA owns one 128 x 128 tile (i-block >= j-block) of H and a contiguous
-// range of tokens.  X̂ is token-major (T x n), so both MMA operands are read
+// One CTA owns one 128 x 256 tile (128 channels i by 256 channels j, on or
+// below the diagonal at 128-channel granularity) of H and a contiguous range
+// of tokens.  X̂ is token-major (T x n), so both MMA operands are read
 // MN-major straight from the activation rows: a TMA box of 64 tokens x 64
 // channels (128-byte rows, 128-byte swizzle) is one canonical MN-major atom
-// stack; two boxes make the 128-channel operand (LBO = 8 KB between them,
-// SBO = 1 KB between 8-token groups).  Diagonal tiles load one operand.
+// stack; two boxes make the 128-channel A operand and four the 256-channel B
+// operand (LBO = 8 KB between boxes, SBO = 1 KB between 8-token groups), and
+// one tcgen05.mma of M = 128, N = 256, K = 16 covers a 16-token step.  The
+// wide tile halves the A traffic per flop and lets a 4-stage, 192 KB ring
+// cover twice the MMA time of a 128 x 128 tile's.
 //
 // Precision: the tensor core's fp32 accumulation loses about one unit in the
 // last place per accumulated MMA, in one direction, so a TMEM accumulator that
 // takes all 2^18 tokens of a calibration set (2^14 MMAs) drifts by ~1e-3 of
-// the entry.  The accumulation is therefore promoted: TMEM holds two 128 x 128
+// the entry.  The accumulation is therefore promoted: TMEM holds two 128 x 256
 // accumulators, the MMA issuer switches between them every 1024 tokens, and
-// the four drain warps add each finished chunk into fp32 registers (IEEE
+// the eight drain warps add each finished chunk into fp32 registers (IEEE
 // adds) while the other accumulator fills.
 //
-// Roles (192 threads): warp 4 lane 0 issues TMA into a STAGES-deep ring,
-// warp 5 lane 0 issues tcgen05.mma (4 x K16 per 64-token stage) and frees
-// stages with tcgen05.commit; warps 0-3 drain the accumulators (warp w owns
-// TMEM lanes 32w..32w+31, i.e. tile rows 32w..) and finally add the tile to H
-// and its mirror, or store it as a partial sum when tokens are split.
+// Roles (320 threads): warp 8 lane 0 issues TMA into a STAGES-deep ring,
+// warp 9 lane 0 issues the MMAs and frees stages with tcgen05.commit; warps
+// 0-7 drain the accumulators (warp w owns TMEM lanes 32 (w % 4).. and columns
+// 128 (w / 4)..) and finally add their piece to H (mirrored below the
+// diagonal block), or store it as a partial sum when tokens are split.
 // The cross mode computes the full (non-symmetric) product X_Aᵀ X_B of two
 // token-major inputs over all tiles, scaled by a sign and added to the output
 // without mirroring: the cross moment of the perturbed-input surrogate is
@@ -36,24 +40,38 @@
 namespace realq {
 namespace {
 
-constexpr int TILE = 128;
+constexpr int TM = 128;                          // tile rows (channels i)
+constexpr int TN = 256;                          // tile columns (channels j)
 constexpr int KSTAGE = 64;                       // tokens per pipeline stage
-constexpr int STAGES = 6;
+constexpr int STAGES = 4;
 constexpr int CHUNK_STAGES = 16;                 // default: 1024 tokens per TMEM accumulator pass
-constexpr int THREADS = 192;
-constexpr int OP_BYTES = TILE * KSTAGE * 2;      // one 128 x 64 bf16 operand tile
+constexpr int DRAIN_WARPS = 8;                   // two per TMEM lane quarter, 128 columns each
+constexpr int THREADS = (DRAIN_WARPS + 2) * 32;  // + the TMA warp and the MMA warp
 constexpr int BOX_BYTES = 64 * KSTAGE * 2;       // one TMA box (64 channels x 64 tokens)
-constexpr int STAGE_BYTES = 2 * OP_BYTES;
+constexpr int A_BYTES = TM * KSTAGE * 2;         // 2 boxes
+constexpr int B_BYTES = TN * KSTAGE * 2;         // 4 boxes
+constexpr int STAGE_BYTES = A_BYTES + B_BYTES;
 constexpr int SMEM_BYTES = STAGES * STAGE_BYTES + 1024 + 256;
-constexpr uint32_t IDESC = tc::idesc_bf16_f32(TILE, TILE, 1, 1);
+constexpr uint32_t IDESC = tc::idesc_bf16_f32(TM, TN, 1, 1);
 constexpr unsigned FULL = 0xFFFFFFFFu;
 
-__device__ __forceinline__ void lower_tile(int64_t idx, int &ti, int &tj) {
-    int r = (int)((sqrt(8.0 * (double)idx + 1.0) - 1.0) * 0.5);
-    while ((int64_t)(r + 1) * (r + 2) / 2 <= idx) ++r;
-    while ((int64_t)r * (r + 1) / 2 > idx) --r;
+// Tiles of the symmetric product: row block ti (128 channels) with every
+// 256-wide column block tj that reaches the diagonal (256 tj <= 128 ti).
+__host__ __device__ inline int64_t lower_tiles(int nti) {
+    int64_t c = 0;
+    for (int r = 0; r < nti; ++r) c += r / 2 + 1;
+    return c;
+}
+
+__device__ __forceinline__ void lower_tile(int64_t idx, int nti, int &ti, int &tj) {
+    int r = 0;
+    for (; r < nti; ++r) {
+        const int64_t c = r / 2 + 1;
+        if (idx < c) break;
+        idx -= c;
+    }
     ti = r;
-    tj = (int)(idx - (int64_t)r * (r + 1) / 2);
+    tj = (int)idx;
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
@@ -70,19 +88,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nti = (int)((n + TM - 1) / TM), ntj = (int)((n + TN - 1) / TN);
     int ti, tj;
     if (cross) {
-        const int nt = (int)((n + TILE - 1) / TILE);
-        ti = (int)(blockIdx.x / nt);
-        tj = (int)(blockIdx.x % nt);
+        ti = (int)(blockIdx.x / ntj);
+        tj = (int)(blockIdx.x % ntj);
     } else {
-        lower_tile(blockIdx.x, ti, tj);
+        lower_tile(blockIdx.x, nti, ti, tj);
     }
-    // cross: all tiles, no mirror; two_maps: the B operand comes from tmapB
-    // (a lower-triangle pass with two maps computes a product known to be
-    // symmetric, e.g. X̂ᵀ(s X̂), and mirrors it)
-    const bool diag = !two_maps && ti == tj;
-    const int i0 = ti * TILE, j0 = tj * TILE;
+    const int i0 = ti * TM, j0 = tj * TN;
     const int64_t t_begin = (int64_t)blockIdx.y * tper;
     const int64_t t_end = min(T, t_begin + tper);
     const int nk = t_end > t_begin ? (int)((t_end - t_begin + KSTAGE - 1) / KSTAGE) : 0;
@@ -95,27 +109,28 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
         for (int b = 0; b < 2; ++b) {
             tc::mbar_init(tc::smem_u32(&accf[b]), 1);
-            tc::mbar_init(tc::smem_u32(&acce[b]), 4);
+            tc::mbar_init(tc::smem_u32(&acce[b]), DRAIN_WARPS);
         }
         *abort_flag = 0;
         tc::fence_barrier_init();
         tc::prefetch_tmap(&tmap);
         if (two_maps) tc::prefetch_tmap(&tmapB);
     }
-    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 2 * TILE);
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 2 * TN);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tmem = *tslot;
 
-    float acc[TILE];
+    float acc[128];
 #pragma unroll
-    for (int c = 0; c < TILE; ++c) acc[c] = 0.f;
+    for (int c = 0; c < 128; ++c) acc[c] = 0.f;
     bool good = true;
 
-    if (warp == 4) {
+    if (warp == DRAIN_WARPS) {
         if (lane == 0) {
             // ---------------- TMA producer ----------------
+            const CUtensorMap *mb = two_maps ? &tmapB : &tmap;
             int it = 0;
             for (; it < nk; ++it) {
                 const int s = it % STAGES;
@@ -125,16 +140,13 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 const uint32_t fb = tc::smem_u32(&full[s]);
-                tc::mbar_arrive_expect_tx(fb, diag ? OP_BYTES : 2 * OP_BYTES);
+                tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
                 const int y = (int)(t_begin + (int64_t)it * KSTAGE);
                 const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
                 tc::tma_load_2d(a, &tmap, fb, i0, y);
                 tc::tma_load_2d(a + BOX_BYTES, &tmap, fb, i0 + 64, y);
-                if (!diag) {
-                    const CUtensorMap *mb = two_maps ? &tmapB : &tmap;
-                    tc::tma_load_2d(a + OP_BYTES, mb, fb, j0, y);
-                    tc::tma_load_2d(a + OP_BYTES + BOX_BYTES, mb, fb, j0 + 64, y);
-                }
+#pragma unroll
+                for (int q = 0; q < 4; ++q) tc::tma_load_2d(a + A_BYTES + q * BOX_BYTES, mb, fb, j0 + 64 * q, y);
             }
             // on abort, let the copies already issued land before the CTA exits
             if (*abort_flag) {
@@ -144,7 +156,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                                   100000000ull);
             }
         }
-    } else if (warp == 5) {
+    } else if (warp == DRAIN_WARPS + 1) {
         if (lane == 0) {
             // ---------------- MMA issuer ----------------
             for (int c = 0; c < nch && !*abort_flag; ++c) {
@@ -154,7 +166,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     break;
                 }
                 tc::fence_after_sync();
-                const uint32_t d = tmem + (uint32_t)(b * TILE);
+                const uint32_t d = tmem + (uint32_t)(b * TN);
                 const int it_end = min(nk, (c + 1) * chunk_stages);
                 for (int it = c * chunk_stages; it < it_end; ++it) {
                     const int s = it % STAGES;
@@ -165,7 +177,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     }
                     tc::fence_after_sync();
                     const uint32_t a = tc::smem_u32(smem + s * STAGE_BYTES);
-                    const uint32_t bop = diag ? a : a + OP_BYTES;
+                    const uint32_t bop = a + A_BYTES;
                     const bool first = it == c * chunk_stages;
 #pragma unroll
                     for (int k = 0; k < KSTAGE / 16; ++k) {
@@ -179,8 +191,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
         }
     } else {
-        // ---------------- drain warps: TMEM chunk -> fp32 registers ----------------
-        const uint32_t lane_base = (uint32_t)(warp * 32) << 16;
+        // ------- drain warps: TMEM chunk -> fp32 registers (lane quarter, column half) -------
+        const uint32_t lane_base = (uint32_t)((warp & 3) * 32) << 16;
+        const uint32_t col_base = (uint32_t)((warp >> 2) * 128);
         for (int c = 0; c < nch; ++c) {
             const int b = c & 1;
             const bool ok = tc::mbar_wait(tc::smem_u32(&accf[b]), (uint32_t)(c >> 1) & 1u, abort_flag);
@@ -190,9 +203,9 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             tc::fence_after_sync();
 #pragma unroll
-            for (int c0 = 0; c0 < TILE; c0 += 32) {
+            for (int c0 = 0; c0 < 128; c0 += 32) {
                 uint32_t v[32];
-                tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(b * TILE + c0), v);
+                tc::tmem_ld_32x32b_x32(tmem + lane_base + (uint32_t)(b * TN) + col_base + (uint32_t)c0, v);
 #pragma unroll
                 for (int q = 0; q < 32; ++q) acc[c0 + q] += __uint_as_float(v[q]);
             }
@@ -205,41 +218,48 @@ __global__ void __launch_bounds__(THREADS, 1)
     const bool all_good = __syncthreads_and(good && !*abort_flag) != 0;
 
     // ---------------- epilogue: registers -> global (drain warps) ----------------
-    if (warp < 4) {
-        const int row = warp * 32 + lane;
-        const int64_t gi = i0 + row;
-        if (!all_good) {
-            // poison the tile: the factorisation of H then reports a non-finite pivot
-            if (gi < n) {
-                for (int c = 0; c < TILE && j0 + c < n; ++c) {
-                    const int64_t gj = j0 + c;
+    // Each drain warp owns a 32-row x 128-column piece, in 128-column block
+    // jb of the matrix.  Symmetric product: jb < ti is added and mirrored,
+    // jb == ti (the diagonal block) is added in full, jb > ti lies above the
+    // diagonal and is left to the tile that holds its mirror image.
+    if (warp < DRAIN_WARPS) {
+        const int jb = 2 * tj + (warp >> 2);
+        const bool write = cross || jb <= ti;
+        const bool mirror = !cross && jb < ti;
+        const int64_t gi = i0 + (warp & 3) * 32 + lane;
+        const int64_t gj0 = (int64_t)jb * 128;
+        if (write && gi < n) {
+            if (!all_good) {
+                // poison: the factorisation of H then reports a non-finite pivot
+                for (int q = 0; q < 128 && gj0 + q < n; ++q) {
+                    const int64_t gj = gj0 + q;
                     if (direct) {
                         H[gi * n + gj] = __int_as_float(0x7fc00000);
-                        if (!cross) H[gj * n + gi] = __int_as_float(0x7fc00000);
+                        if (mirror) H[gj * n + gi] = __int_as_float(0x7fc00000);
                         if (H2) {
                             H2[gi * n + gj] = __int_as_float(0x7fc00000);
-                            H2[gj * n + gi] = __int_as_float(0x7fc00000);
+                            if (mirror) H2[gj * n + gi] = __int_as_float(0x7fc00000);
                         }
                     } else {
                         part[(int64_t)blockIdx.y * n * n + gi * n + gj] = __int_as_float(0x7fc00000);
                     }
                 }
-            }
-        } else if (nk > 0 && gi < n) {
+            } else if (nk > 0) {
 #pragma unroll
-            for (int q = 0; q < TILE; ++q) {
-                const int64_t gj = j0 + q;
-                if (gj < n) {
-                    const float v = sign * acc[q];
-                    if (direct) {
-                        H[gi * n + gj] += v;
-                        if (ti != tj && !cross) H[gj * n + gi] += v;
-                        if (H2) {
-                            H2[gi * n + gj] += v;
-                            if (ti != tj) H2[gj * n + gi] += v;
+                for (int q = 0; q < 128; ++q) {
+                    const int64_t gj = gj0 + q;
+                    if (gj < n) {
+                        const float v = sign * acc[q];
+                        if (direct) {
+                            H[gi * n + gj] += v;
+                            if (mirror) H[gj * n + gi] += v;
+                            if (H2) {
+                                H2[gi * n + gj] += v;
+                                if (mirror) H2[gj * n + gi] += v;
+                            }
+                        } else {
+                            part[(int64_t)blockIdx.y * n * n + gi * n + gj] = v;
                         }
-                    } else {
-                        part[(int64_t)blockIdx.y * n * n + gi * n + gj] = v;
                     }
                 }
             }
@@ -248,7 +268,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (!all_good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
     tc::fence_before_sync();
     __syncthreads();
-    if (warp == 0) tc::tmem_dealloc(tmem, 2 * TILE);
+    if (warp == 0) tc::tmem_dealloc(tmem, 2 * TN);
 }
 
 using EncodeFn = CUresult (*)(CUtensorMap *, CUtensorMapDataType, cuuint32_t, void *, const cuuint64_t *,
@@ -316,9 +336,9 @@ static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const
     if (!XB) mapB = mapA;
     const int two_maps = XB != nullptr;
     const int cross = two_maps && !sym_pair;
-    const int nt = ceil_div(n, TILE);
-    const int64_t tiles = cross ? (int64_t)nt * nt : (int64_t)nt * (nt + 1) / 2;
-    int splits = cross ? hessian_splits_tiles(tiles, T, sms) : hessian_splits(n, T, sms);
+    const int nti = ceil_div(n, TM), ntj = ceil_div(n, TN);
+    const int64_t tiles = cross ? (int64_t)nti * ntj : lower_tiles(nti);
+    int splits = hessian_splits_tiles(tiles, T, sms);
     const size_t per = (size_t)n * n * sizeof(float);
     if (splits > 1 && (ws == nullptr || ws_bytes < 2 * per)) splits = 1;
     if (splits > 1 && (size_t)splits * per > ws_bytes) splits = (int)(ws_bytes / per);
