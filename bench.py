@@ -37,6 +37,9 @@ NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
     ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
+    # the Block-GD G product with the fused Adam step: 219 launches of a
+    # Qwen3-0.6B block over 3 steps, 50.05 MB read + 1.08 MB written on average
+    ("qwen3-0.6b", "bgd_g_gemm_adam"): 51125381,
 }
 
 
