@@ -208,11 +208,13 @@ __global__ void __launch_bounds__(128) chol_diag_kernel(int64_t n, float *A, int
     }
 }
 
-// A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles).
-__global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, int64_t k0, int kb) {
+// A[i][j] -= sum_c A[i][k0+c] A[j][k0+c] for i <= j < k0 (64 x 64 upper tiles,
+// tile idx0 + blockIdx.x of the column-by-column enumeration: tile column tj
+// holds tiles (0..tj, tj)).
+__global__ void __launch_bounds__(256) chol_update_kernel(int64_t n, float *A, int64_t k0, int kb, int64_t idx0) {
     __shared__ __align__(16) float Pi[NB][NB + 4];
     __shared__ __align__(16) float Pj[NB][NB + 4];
-    const int64_t idx = blockIdx.x;
+    const int64_t idx = idx0 + blockIdx.x;
     int r = (int)((sqrt(8.0 * (double)idx + 1.0) - 1.0) * 0.5);
     while ((int64_t)(r + 1) * (r + 2) / 2 <= idx) ++r;
     while ((int64_t)r * (r + 1) / 2 > idx) --r;
@@ -316,9 +318,10 @@ realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp,
 // use and kept for the life of the thread.
 struct AuxStream {
     int device = -1, priority = 0;
-    cudaStream_t stream = nullptr;
-    cudaEvent_t ev[2] = {nullptr, nullptr};
-    std::vector<cudaEvent_t> steps;
+    cudaStream_t stream = nullptr;       // U row work
+    cudaStream_t wide = nullptr;         // the look-ahead's wide trailing updates
+    cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
+    std::vector<cudaEvent_t> steps, pdone, wdone;
 };
 static thread_local std::vector<AuxStream> g_aux;
 
@@ -332,18 +335,20 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
     if (!found) {
         AuxStream a;
         REALQ_CUDA_TRY(cudaStreamCreateWithPriority(&a.stream, cudaStreamNonBlocking, prio));
-        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[0], cudaEventDisableTiming));
-        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[1], cudaEventDisableTiming));
+        REALQ_CUDA_TRY(cudaStreamCreateWithPriority(&a.wide, cudaStreamNonBlocking, prio));
+        for (int i = 0; i < 3; ++i) REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[i], cudaEventDisableTiming));
         a.device = dev;
         a.priority = prio;
         g_aux.push_back(a);
         found = &g_aux.back();
     }
     AuxStream &a = *found;
-    while ((int64_t)a.steps.size() < nsteps) {
-        cudaEvent_t e;
-        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
-        a.steps.push_back(e);
+    for (std::vector<cudaEvent_t> *v : {&a.steps, &a.pdone, &a.wdone}) {
+        while ((int64_t)v->size() < nsteps) {
+            cudaEvent_t e;
+            REALQ_CUDA_TRY(cudaEventCreateWithFlags(&e, cudaEventDisableTiming));
+            v->push_back(e);
+        }
     }
     *out = &a;
     return REALQ_OK;
@@ -392,6 +397,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
         REALQ_CUDA_TRY(cudaEventRecord(aux->ev[0], s));
         REALQ_CUDA_TRY(cudaStreamWaitEvent(rs, aux->ev[0], 0));
     }
+    std::vector<char> wide_pending(nbk + 1, 0);
     for (int K = nbk - 1; K >= 0; --K) {
         const int64_t k0 = (int64_t)K * NB;
         const int kb = (int)std::min<int64_t>(NB, n - k0);
@@ -415,12 +421,36 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
             pg.C = U + k0; pg.ldc = n;
             pg.alpha = 1.f;
             REALQ_TRY(gemm_f32(s, A_ROW, EPI_STORE, pg, "chol_panel"));
+            // Rank-kb update of the block above.  Look-ahead: the next step
+            // needs only tile column nt0 - 1 (its diagonal block and its
+            // panel), which is updated at once; the other columns ("wide")
+            // run on a second stream, overlapped with the next diagonal
+            // factorisation and panel, and the next narrow update waits for
+            // them because it touches their last column.
             const int64_t nt0 = k0 / NB;
+            const int64_t nwide = (nt0 - 1) * nt0 / 2;
+            if (aux && nwide > 0) {
+                REALQ_CUDA_TRY(cudaEventRecord(aux->pdone[K], s));
+                REALQ_CUDA_TRY(cudaStreamWaitEvent(aux->wide, aux->pdone[K], 0));
+            }
+            if (aux && K + 1 < nbk && wide_pending[K + 1]) REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->wdone[K + 1], 0));
             {
                 Launch L("chol_update", s);
-                chol_update_kernel<<<(unsigned)(nt0 * (nt0 + 1) / 2), 256, 0, s>>>(n, U, k0, kb);
+                chol_update_kernel<<<(unsigned)nt0, 256, 0, s>>>(n, U, k0, kb, nwide);
             }
             REALQ_TRY(check_launch("chol_update"));
+            if (nwide > 0) {
+                cudaStream_t ws_ = aux ? aux->wide : s;
+                {
+                    Launch L("chol_update", ws_);
+                    chol_update_kernel<<<(unsigned)nwide, 256, 0, ws_>>>(n, U, k0, kb, 0);
+                }
+                REALQ_TRY(check_launch("chol_update"));
+                if (aux) {
+                    REALQ_CUDA_TRY(cudaEventRecord(aux->wdone[K], aux->wide));
+                    wide_pending[K] = 1;
+                }
+            }
         }
         if (k1 < n) {
             const int64_t r = n - k1;
@@ -448,6 +478,8 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
     if (aux) {
         REALQ_CUDA_TRY(cudaEventRecord(aux->ev[1], rs));
         REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[1], 0));
+        REALQ_CUDA_TRY(cudaEventRecord(aux->ev[2], aux->wide));
+        REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[2], 0));
     }
     int host_status = -1;
     REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
