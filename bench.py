@@ -169,18 +169,32 @@ def gpu_arm(args, wl, rank, world):
                            for k in ("codes", "scale", "zero")} for mod in wl.modules}
     e2e_bytes = {"h2d": 0, "d2h": 0}
 
+    # One step enqueues about a thousand small kernels over eleven streams;
+    # by default it is captured once into a CUDA graph and replayed (every
+    # kernel still runs every step, on the same resident inputs).  The
+    # saliency-grouped variant reads token weights on the host mid-step and
+    # always runs eagerly.
+    use_graph = not args.no_graph and not args.saliency_groups
+    if use_graph:
+        bq.capture(dev_x, dev_w, dev_f, dev_fn)
+
     def step_device():
-        bq.run(dev_x, dev_w, dev_f, dev_fn, saliency=dev_sal)
+        if use_graph:
+            bq.replay()
+        else:
+            bq.run(dev_x, dev_w, dev_f, dev_fn, saliency=dev_sal)
         bq.check_status()
 
     def step_serial():
         bq.run_serial(dev_x, dev_w, dev_f, dev_fn, saliency=dev_sal)
 
     def step_e2e():
-        h2d, d2h = bq.run_host(host_x, host_w, host_f, host_out)
+        if use_graph:
+            bq.replay()
+        else:
+            e2e_bytes["h2d"], e2e_bytes["d2h"] = bq.run_host(host_x, host_w, host_f, host_out)
         bq.check_status()
         torch.cuda.current_stream().synchronize()
-        e2e_bytes["h2d"], e2e_bytes["d2h"] = h2d, d2h
 
     # ---- warm-up
     for _ in range(args.warmup):
@@ -209,7 +223,7 @@ def gpu_arm(args, wl, rank, world):
     barrier()
     ms_total = t0.elapsed_time(t1)
     clk = clocks.stop()
-    launches = rq.realq_launch_count() - launches0
+    launches = rq.realq_launch_count() - launches0   # a graph launch adds the library kernels it holds
 
     # The same K steps again, serialized on one stream, with every library
     # launch bracketed by CUDA events on that stream: per-kernel device time for
@@ -234,6 +248,8 @@ def gpu_arm(args, wl, rank, world):
     # ---- end to end through host buffers
     e2e = None
     if not args.no_e2e and not args.act_bits and not args.saliency_groups and not args.minibatch_seqs:
+        if use_graph:
+            e2e_bytes["h2d"], e2e_bytes["d2h"] = bq.capture_host(host_x, host_w, host_f, host_out)
         step_e2e()
         torch.cuda.synchronize()
         barrier()
@@ -274,6 +290,8 @@ def gpu_arm(args, wl, rank, world):
                        "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}" +
                               (f", mini-batches of {args.minibatch_seqs} x 2048 tokens" if args.minibatch_seqs else ""),
                        "parallelism": f"replicas x{world}",
+                       "launch": "one CUDA graph per step (11 streams)" if use_graph else
+                                 "eager, one host thread per input",
                        "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
                              (sum(s.T * s.n * 2 for s in wl.inputs.values()) / 1e9),
                        "input_generation_s": round(t_gen, 1)},
@@ -497,6 +515,7 @@ def main():
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
+    ap.add_argument("--no-graph", action="store_true", help="launch the block step eagerly instead of as a CUDA graph")
     ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep"], default=None,
                     help="time one stage alone on a small synthetic case")
     ap.add_argument("--n", type=int, default=2048)

@@ -137,6 +137,23 @@ realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T
                                      int64_t *fail_col, void *ws, size_t ws_bytes);
 size_t realq_prepare_workspace_size(int64_t n);
 
+/* realq_hessian_prepare without the host synchronisation, for stream
+ * capture into a CUDA graph and for callers that check later: the call only
+ * enqueues work on `stream` (and on auxiliary streams of the calling thread
+ * that fork from and join back into it; make one call on a given stream
+ * before capturing it, so that they exist).  Same arguments and results as
+ * realq_hessian_prepare; the factorisation status stays in the workspace's
+ * first word (-1, or the first column whose pivot was not positive) until
+ * the next prepare call on that workspace and is read with
+ * realq_prepare_status once the work has completed. */
+realq_status_t realq_hessian_prepare_deferred(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                              const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                              void *ws, size_t ws_bytes);
+/* Status of the last prepare call on workspace ws (synchronizes `stream`,
+ * which must be ordered after that call): REALQ_ERR_NOT_SPD with *fail_col
+ * (host) = the column, else REALQ_OK with *fail_col = -1. */
+realq_status_t realq_prepare_status(realq_stream_t stream, void *ws, size_t ws_bytes, int64_t *fail_col);
+
 /* Allocation-free variant of realq_hessian_prepare.  The paper has no
  * counterpart: this exists for callers that cannot allocate device memory,
  * e.g. a plugin running inside a host application that owns every device
@@ -358,6 +375,34 @@ typedef struct {
 int64_t realq_launch_count(void);
 void realq_profile_enable(int on);
 int realq_profile_collect(realq_kernel_stat_t *out, int max_entries);
+
+
+/* CUDA graphs of whole steps.  A step of many small launches over several
+ * streams (the block scheduler's) is recorded once and relaunched whole:
+ *   realq_graph_begin(stream)   starts a thread-local stream capture of
+ *                               `stream` (not the legacy default stream);
+ *                               other streams join it by waiting on events
+ *                               recorded in it and must join back before
+ *                               the end.  Calls made meanwhile only enqueue.
+ *   realq_graph_end(stream, node_priorities, &g)
+ *                               ends the capture and instantiates the graph;
+ *                               with node_priorities != 0 each kernel keeps
+ *                               the priority of the stream it was captured
+ *                               from (the critical chain of a step can be
+ *                               favoured), else all run at the priority of
+ *                               the stream the graph is launched into.
+ *                               On failure *g = NULL.
+ *   realq_graph_launch(g, s)    launches the graph on s (asynchronous); the
+ *                               library's kernels in it count towards
+ *                               realq_launch_count().
+ *   realq_graph_kernels(g)      how many of this library's kernels g holds.
+ *   realq_graph_destroy(g)      frees it (NULL is a no-op). */
+typedef struct realq_graph_s *realq_graph_t;
+realq_status_t realq_graph_begin(realq_stream_t stream);
+realq_status_t realq_graph_end(realq_stream_t stream, int node_priorities, realq_graph_t *graph);
+realq_status_t realq_graph_launch(realq_graph_t graph, realq_stream_t stream);
+int64_t realq_graph_kernels(realq_graph_t graph);
+void realq_graph_destroy(realq_graph_t graph);
 
 #ifdef __cplusplus
 }

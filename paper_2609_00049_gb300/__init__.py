@@ -19,7 +19,8 @@ import torch
 __all__ = [
     "RealqError", "QuantCfg", "BgdCfg", "lib", "library_path", "quant_cfg", "bgd_cfg", "workspace",
     "realq_hessian_accumulate", "realq_hessian_workspace_size", "realq_hessian_prepare",
-    "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc", "realq_scale_moment", "realq_quantize_layer",
+    "realq_prepare_workspace_size", "realq_hessian_prepare_noalloc",
+    "realq_hessian_prepare_deferred", "realq_prepare_status", "Graph", "realq_graph_begin", "realq_graph_end", "realq_scale_moment", "realq_quantize_layer",
     "realq_quantize_activations", "realq_saliency_clip", "realq_hessian_weighted_workspace_size",
     "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled", "realq_quantize_layer_grouped",
     "realq_quantize_grouped_workspace_size", "realq_quantize_layer_minibatch",
@@ -81,6 +82,13 @@ _SIGS = {
     "realq_hessian_prepare": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
     "realq_prepare_workspace_size": ([_i64], _sz),
     "realq_hessian_prepare_noalloc": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _P_i64], _int),
+    "realq_hessian_prepare_deferred": ([_vp, _i64, _i64, _f32, _vp, _vp, _vp, _vp, _vp, _sz], _int),
+    "realq_prepare_status": ([_vp, _vp, _sz, _P_i64], _int),
+    "realq_graph_begin": ([_vp], _int),
+    "realq_graph_end": ([_vp, _int, ctypes.POINTER(_vp)], _int),
+    "realq_graph_launch": ([_vp, _vp], _int),
+    "realq_graph_kernels": ([_vp], _i64),
+    "realq_graph_destroy": ([_vp], None),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
     "realq_quantize_activations": ([_vp, _i64, _i64, _vp, _int, _int, _f32, _vp, _vp, _vp], _int),
     "realq_saliency_clip": ([_vp, _i64, _int, _vp, _f32, _vp, _vp], _int),
@@ -216,6 +224,62 @@ def realq_hessian_prepare(H_sum: torch.Tensor, T_total: int, damp_frac: float, U
                                      _ptr(Hbar_out), _ptr(dead_out), ctypes.byref(fc), wp, wb)
     _check(st, fail_col=fc.value)
     return fc.value
+
+
+def realq_hessian_prepare_deferred(H_sum: torch.Tensor, T_total: int, damp_frac: float, U_out: torch.Tensor,
+                                   Hbar_out: Optional[torch.Tensor], dead_out: torch.Tensor, ws: torch.Tensor,
+                                   stream=None) -> None:
+    """realq_hessian_prepare that only enqueues (capturable into a CUDA graph);
+    the factorisation status stays in ws, read with realq_prepare_status."""
+    n = H_sum.shape[0]
+    _need(U_out, torch.float32, (n, n), "U_out")
+    _need(Hbar_out, torch.float32, (n, n), "Hbar_out")
+    _need(dead_out, torch.uint8, (n,), "dead_out")
+    wp, wb = _ws(ws)
+    _check(lib().realq_hessian_prepare_deferred(_stream(stream), n, int(T_total), float(damp_frac), _ptr(H_sum),
+                                                _ptr(U_out), _ptr(Hbar_out), _ptr(dead_out), wp, wb))
+
+
+def realq_prepare_status(ws: torch.Tensor, stream=None) -> int:
+    """Synchronizes; returns -1, or raises RealqError(status=NOT_SPD, fail_col=j)
+    for the last prepare call on ws."""
+    fc = ctypes.c_int64(-1)
+    wp, wb = _ws(ws)
+    st = lib().realq_prepare_status(_stream(stream), wp, wb, ctypes.byref(fc))
+    _check(st, fail_col=fc.value)
+    return fc.value
+
+
+class Graph:
+    """A captured step (realq_graph_t), destroyed with the object."""
+
+    def __init__(self, handle: int):
+        self.handle = handle
+
+    @property
+    def kernels(self) -> int:
+        return int(lib().realq_graph_kernels(self.handle))
+
+    def launch(self, stream=None) -> None:
+        _check(lib().realq_graph_launch(self.handle, _stream(stream)))
+
+    def __del__(self):
+        if getattr(self, "handle", None) and _lib is not None:
+            _lib.realq_graph_destroy(self.handle)
+            self.handle = None
+
+
+def realq_graph_begin(stream=None) -> None:
+    """Start capturing `stream` (thread-local mode) into a graph."""
+    _check(lib().realq_graph_begin(_stream(stream)))
+
+
+def realq_graph_end(stream=None, node_priorities: bool = True) -> Graph:
+    """End the capture of `stream`; with node_priorities the graph's kernels
+    keep the priorities of the streams they were captured from."""
+    h = ctypes.c_void_p()
+    _check(lib().realq_graph_end(_stream(stream), int(bool(node_priorities)), ctypes.byref(h)))
+    return Graph(h.value)
 
 
 PREPARE_NOALLOC_MAX_N = 32768

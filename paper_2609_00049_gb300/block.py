@@ -6,11 +6,18 @@ input, o the attention output, gate/up the MLP input and down the MLP hidden
 state.  Each distinct input needs one Hessian and one preparation; each
 module then runs its own column sweep.  Those chains are independent of one
 another, so they run concurrently: one host thread per input drives the
-input's stream (accumulate, then prepare, which waits on that stream only),
-then issues every module fed by that input on a stream of its own.  The
-library calls release the interpreter lock, so the threads overlap on the
-host as well.  All state (Hessians, factors, optimizer moments, outputs,
-workspaces) is allocated once and reused across calls.
+input's stream (accumulate, then prepare), then issues every module fed by
+that input on a stream of its own.  The library calls release the
+interpreter lock, so the threads overlap on the host as well.  All state
+(Hessians, factors, optimizer moments, outputs, workspaces) is allocated once
+and reused across calls.
+
+One step enqueues about a thousand kernels, most of them small (the 64-column
+steps of the Cholesky factorisation and of the sweeps), so launching them
+costs as much host time as they take on the GPU.  capture() records the same
+multi-stream step once into a CUDA graph; replay() then launches it whole.
+The preparation's factorisation status is therefore never read mid-step:
+check_status() reads it, with the sweeps' status words, after the step.
 
 No arithmetic happens here; every step is a call through the C ABI.
 """
@@ -22,8 +29,8 @@ from typing import Dict, List, Optional, Sequence
 
 import torch
 
-from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_hessian_accumulate, realq_hessian_accumulate_weighted,
-               realq_hessian_prepare, realq_hessian_prepare_scaled, realq_hessian_weighted_workspace_size,
+from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_graph_begin, realq_graph_end, realq_hessian_accumulate, realq_hessian_accumulate_weighted,
+               realq_hessian_prepare_deferred, realq_hessian_prepare_scaled, realq_prepare_status, realq_hessian_weighted_workspace_size,
                realq_hessian_workspace_size, realq_prepare_workspace_size, realq_quantize_activations,
                realq_quantize_grouped_workspace_size, realq_quantize_layer, realq_quantize_layer_grouped,
                realq_quantize_layer_minibatch, realq_quantize_minibatch_workspace_size, realq_quantize_workspace_size,
@@ -103,7 +110,7 @@ class BlockQuantizer:
             self.state[name] = dict(
                 H=torch.empty(n, n, device=dev), U=torch.empty(n, n, device=dev), Hbar=torch.empty(n, n, device=dev),
                 dead=torch.empty(n, dtype=torch.uint8, device=dev),
-                pws=workspace(realq_prepare_workspace_size(n), dev),
+                pws=workspace(realq_prepare_workspace_size(n), dev).fill_(0xFF),  # status word -1: no failure
                 hws=workspace(realq_hessian_workspace_size(n, spec.T, REALQ_BF16, act_quant is not None), dev))
             if minibatch_tokens:
                 nmb = -(-spec.T // minibatch_tokens)
@@ -153,15 +160,32 @@ class BlockQuantizer:
                 disp=torch.empty(m, n, device=dev) if bgd else None, bcfg=bc if bgd else None,
                 ws=ws_q,
                 adam_t=0)
-        self.in_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
-        self.copy_streams = {name: torch.cuda.Stream(device=dev) for name in self.inputs}
-        self.mod_streams = {md.name: torch.cuda.Stream(device=dev) for md in self.modules}
+        # Stream priorities follow the length of each input's chain (its
+        # preparation and its modules' sweeps are sequences of 64-column
+        # steps, so the widest input's chain is the longest): the widest input
+        # and its modules get the highest priority, and kernels keep it inside
+        # a captured graph.
+        lo, hi = torch.cuda.Stream.priority_range()
+        widths = sorted({spec.n for spec in self.inputs.values()}, reverse=True)
+        self.priority = {name: max(hi, min(lo, hi + widths.index(spec.n))) for name, spec in self.inputs.items()}
+        self.in_streams = {name: torch.cuda.Stream(device=dev, priority=self.priority[name]) for name in self.inputs}
+        # one host-to-device copy stream shared by all inputs: a single stream
+        # already saturates the host link, and in a captured step the inputs
+        # arrive in chain order (the longest chain's activations first), so
+        # that chain's preparation and sweeps overlap the other copies
+        self.chain_order = sorted(self.inputs, key=lambda name: self.priority[name])
+        copy_stream = torch.cuda.Stream(device=dev)
+        self.copy_streams = {name: copy_stream for name in self.inputs}
+
+        self.mod_streams = {md.name: torch.cuda.Stream(device=dev, priority=self.priority[md.input])
+                            for md in self.modules}
         self.pool = ThreadPoolExecutor(len(self.inputs))
         # staging for inputs streamed from host memory (two chunks per input)
         self.host_chunk = host_chunk_tokens
         self._stage = None
         self._chunk_ws = None
         self._w_stage = None
+        self.graph = None
 
     # ------------------------------------------------------------------ device
     def _quantize_module(self, md: BlockModule, s_in, W0, F, F_next, stream, X=None, sal=None):
@@ -239,8 +263,8 @@ class BlockQuantizer:
             bits, clip = self.act_quant
             realq_quantize_activations(X, bits, clip, X_q=s_in["Xq"], stream=stream)
             realq_hessian_accumulate(s_in["Xq"], s_in["H"], s_in["D"], X, ws=s_in["hws"], stream=stream)
-        realq_hessian_prepare(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                              s_in["pws"], stream=stream)
+        realq_hessian_prepare_deferred(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
+                                       s_in["pws"], stream=stream)
         if self.act_quant is not None:
             realq_scale_moment(s_in["D"], spec.T, s_in["Dbar"], stream=stream)
 
@@ -278,8 +302,60 @@ class BlockQuantizer:
                 self._quantize_module(md, s_in, W0[md.name], F[md.name], (F_next or {}).get(md.name), None,
                                       X=X[name], sal=(saliency or {}).get(md.name))
 
+    def capture(self, X: Dict[str, torch.Tensor], W0: Dict[str, torch.Tensor], F: Dict[str, torch.Tensor],
+                F_next: Optional[Dict[str, torch.Tensor]] = None) -> None:
+        """Record one step of run() on these tensors into a CUDA graph (every
+        input's and module's stream forks from and joins back into the
+        capturing stream), after one eager step that creates the library's
+        auxiliary streams for the calling thread.  replay() then re-runs the
+        whole step, reading the same tensors in place: change their contents,
+        not their storage.  The saliency-grouped variant reads its groups'
+        token weights on the host mid-step and is not capturable."""
+        if self.sgroups:
+            raise NotImplementedError("capture: the saliency-grouped variant reads token weights on the host")
+        torch.cuda.set_device(self.device)
+        self._enqueue(X, W0, F, F_next)
+        torch.cuda.synchronize(self.device)
+        self.check_status()
+        self.graph = self._capture(lambda: self._enqueue(X, W0, F, F_next))
+
+    def _capture(self, enqueue, node_priorities=True):
+        cur = torch.cuda.current_stream(self.device)
+        cap = torch.cuda.Stream(device=self.device)
+        cap.wait_stream(cur)
+        with torch.cuda.stream(cap):
+            realq_graph_begin(cap)
+            try:
+                out = enqueue()
+            finally:
+                g = realq_graph_end(cap, node_priorities)
+        cur.wait_stream(cap)
+        self.graph_counts = out
+        return g
+
+    def replay(self) -> None:
+        """Launch the captured step on the current stream."""
+        if self.graph is None:
+            raise RuntimeError("replay: capture() first")
+        self.graph.launch(torch.cuda.current_stream(self.device))
+
+    def _enqueue(self, X, W0, F, F_next) -> None:
+        cur = torch.cuda.current_stream(self.device)
+        start = torch.cuda.Event()
+        start.record(cur)
+        for name in self.chain_order:
+            self._input_pipeline(name, start, X, W0, F, F_next)
+        for md in self.modules:
+            cur.wait_stream(self.mod_streams[md.name])
+        for name in self.inputs:
+            cur.wait_stream(self.in_streams[name])
+
     def check_status(self) -> None:
-        """Raise if any module's sweep recorded a non-finite value or a timeout."""
+        """Synchronizes; raises RealqError(NOT_SPD) if an input's damped Hessian
+        was not positive definite, else if any module's sweep recorded a
+        non-finite value or a timeout."""
+        for name in self.inputs:
+            realq_prepare_status(self.state[name]["pws"])
         for md in self.modules:
             realq_workspace_status(self.out[md.name]["ws"])
 
@@ -311,8 +387,8 @@ class BlockQuantizer:
             ev.record(si)
             used[c % 2] = ev
             h2d += rows * spec.n * xs.element_size()
-        realq_hessian_prepare(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
-                              s_in["pws"], stream=si)
+        realq_hessian_prepare_deferred(s_in["H"], spec.T, self.qcfg.damp_frac, s_in["U"], s_in["Hbar"], s_in["dead"],
+                                       s_in["pws"], stream=si)
         for md in self.mods_of[name]:
             sm, o, w = self.mod_streams[md.name], out_host[md.name], self._w_stage[md.name]
             sm.wait_stream(si)
@@ -334,6 +410,46 @@ class BlockQuantizer:
         and F are copied per module, codes / scale / zero are copied back into
         out_host[module][...] (pinned).  Returns (h2d bytes, d2h bytes).
         The activation-aware variant is not streamed (it runs with run())."""
+        self._host_setup(X_host, W0_host, F_host)
+        cur = torch.cuda.current_stream(self.device)
+        start = torch.cuda.Event()
+        start.record(cur)
+        counts = {}
+        futs = [self.pool.submit(self._host_pipeline, name, start, X_host, W0_host, F_host, out_host, counts)
+                for name in self.inputs]
+        for f in futs:
+            f.result()
+        self._join(cur)
+        return sum(v[0] for v in counts.values()), sum(v[1] for v in counts.values())
+
+    def capture_host(self, X_host, W0_host, F_host, out_host):
+        """capture() for run_host(): the graph holds the host-to-device copies
+        of every step's inputs and the copies of the outputs back into
+        out_host, so replay() is the whole step end to end from the same
+        pinned host buffers.  Returns (h2d bytes, d2h bytes) per step."""
+        self._host_setup(X_host, W0_host, F_host)
+        torch.cuda.set_device(self.device)
+        self._enqueue_host(X_host, W0_host, F_host, out_host)
+        torch.cuda.synchronize(self.device)
+        self.check_status()
+        # without kernel priorities: a prioritised sweep would delay another
+        # input's chunk accumulation, whose staging buffer then holds up the
+        # shared copy stream (measured: 24 ms per step without, 27 with)
+        self.graph = self._capture(lambda: self._enqueue_host(X_host, W0_host, F_host, out_host),
+                                   node_priorities=False)
+        return self.graph_counts
+
+    def _enqueue_host(self, X_host, W0_host, F_host, out_host):
+        cur = torch.cuda.current_stream(self.device)
+        start = torch.cuda.Event()
+        start.record(cur)
+        counts = {}
+        for name in self.chain_order:
+            self._host_pipeline(name, start, X_host, W0_host, F_host, out_host, counts)
+        self._join(cur)
+        return sum(v[0] for v in counts.values()), sum(v[1] for v in counts.values())
+
+    def _host_setup(self, X_host, W0_host, F_host):
         if self.act_quant is not None or self.sgroups:
             raise NotImplementedError("run_host: this variant runs from device-resident inputs")
         dev = self.device
@@ -347,13 +463,3 @@ class BlockQuantizer:
                                            F=torch.empty(F_host[md.name].shape, dtype=F_host[md.name].dtype,
                                                          device=dev))
                              for md in self.modules}
-        cur = torch.cuda.current_stream(dev)
-        start = torch.cuda.Event()
-        start.record(cur)
-        counts = {}
-        futs = [self.pool.submit(self._host_pipeline, name, start, X_host, W0_host, F_host, out_host, counts)
-                for name in self.inputs]
-        for f in futs:
-            f.result()
-        self._join(cur)
-        return sum(v[0] for v in counts.values()), sum(v[1] for v in counts.values())

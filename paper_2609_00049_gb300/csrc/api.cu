@@ -159,6 +159,58 @@ const char *realq_last_error(void) { return g_err; }
 
 int64_t realq_launch_count(void) { return g_launches.load(); }
 
+// ------------------------------------------------------------ CUDA graphs ---
+struct realq_graph_s {
+    cudaGraphExec_t exec = nullptr;
+    int64_t kernels = 0;  // this library's kernels in the graph
+};
+static thread_local int64_t g_capture_start = -1;
+
+realq_status_t realq_graph_begin(realq_stream_t stream) {
+    if (!stream) return fail(REALQ_ERR_INVALID_ARG, "graph_begin: the legacy default stream cannot be captured");
+    REALQ_CUDA_TRY(cudaStreamBeginCapture(S(stream), cudaStreamCaptureModeThreadLocal));
+    g_capture_start = g_launches.load();
+    return REALQ_OK;
+}
+
+realq_status_t realq_graph_end(realq_stream_t stream, int node_priorities, realq_graph_t *out) {
+    if (!out) return fail(REALQ_ERR_INVALID_ARG, "graph_end: NULL output");
+    *out = nullptr;
+    cudaGraph_t g = nullptr;
+    const cudaError_t e = cudaStreamEndCapture(S(stream), &g);
+    const int64_t kernels = g_capture_start >= 0 ? g_launches.load() - g_capture_start : 0;
+    g_capture_start = -1;
+    if (e != cudaSuccess) {
+        if (g) cudaGraphDestroy(g);
+        return fail(REALQ_ERR_CUDA, "cudaStreamEndCapture: %s", cudaGetErrorString(e));
+    }
+    cudaGraphExec_t x = nullptr;
+    const cudaError_t ei =
+        cudaGraphInstantiateWithFlags(&x, g, node_priorities ? cudaGraphInstantiateFlagUseNodePriority : 0);
+    cudaGraphDestroy(g);
+    if (ei != cudaSuccess) return fail(REALQ_ERR_CUDA, "cudaGraphInstantiate: %s", cudaGetErrorString(ei));
+    realq_graph_s *h = new realq_graph_s;
+    h->exec = x;
+    h->kernels = kernels;
+    *out = h;
+    return REALQ_OK;
+}
+
+realq_status_t realq_graph_launch(realq_graph_t graph, realq_stream_t stream) {
+    if (!graph || !graph->exec) return fail(REALQ_ERR_INVALID_ARG, "graph_launch: no graph");
+    REALQ_CUDA_TRY(cudaGraphLaunch(graph->exec, S(stream)));
+    g_launches.fetch_add(graph->kernels, std::memory_order_relaxed);
+    return REALQ_OK;
+}
+
+int64_t realq_graph_kernels(realq_graph_t graph) { return graph ? graph->kernels : 0; }
+
+void realq_graph_destroy(realq_graph_t graph) {
+    if (!graph) return;
+    if (graph->exec) cudaGraphExecDestroy(graph->exec);
+    delete graph;
+}
+
 void realq_profile_enable(int on) { g_prof_on.store(on ? 1 : 0); }
 
 int realq_profile_collect(realq_kernel_stat_t *out, int max_entries) {
@@ -228,6 +280,29 @@ realq_status_t realq_hessian_prepare(realq_stream_t stream, int64_t n, int64_t T
     REALQ_TRY(check_ws(ws, ws_bytes, prepare_ws_bytes(n), "hessian_prepare"));
     *fail_col = -1;
     return prepare(S(stream), n, T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, fail_col, ws, ws_bytes);
+}
+
+realq_status_t realq_hessian_prepare_deferred(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,
+                                              const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
+                                              void *ws, size_t ws_bytes) {
+    if (n <= 0 || T_total <= 0) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_deferred: n > 0, T_total > 0 required");
+    if (!H_sum || !U_out || !dead_out) return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_deferred: NULL argument");
+    if ((const void *)U_out == (const void *)H_sum)
+        return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_deferred: U_out may not alias H_sum");
+    if (!(damp_frac >= 0.f) || !std::isfinite(damp_frac))
+        return fail(REALQ_ERR_INVALID_ARG, "hessian_prepare_deferred: damp_frac >= 0");
+    REALQ_TRY(check_ws(ws, ws_bytes, prepare_ws_bytes(n), "hessian_prepare_deferred"));
+    return prepare_deferred(S(stream), n, (double)T_total, damp_frac, H_sum, U_out, Hbar_out, dead_out, ws, ws_bytes);
+}
+
+realq_status_t realq_prepare_status(realq_stream_t stream, void *ws, size_t ws_bytes, int64_t *fail_col) {
+    if (!ws || ws_bytes < sizeof(int) || !fail_col) return fail(REALQ_ERR_INVALID_ARG, "prepare_status: bad argument");
+    int st = -1;
+    REALQ_CUDA_TRY(cudaMemcpyAsync(&st, ws, sizeof(int), cudaMemcpyDeviceToHost, S(stream)));
+    REALQ_CUDA_TRY(cudaStreamSynchronize(S(stream)));
+    *fail_col = st;
+    if (st >= 0) return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", st);
+    return REALQ_OK;
 }
 
 realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, int64_t T_total, float damp_frac,

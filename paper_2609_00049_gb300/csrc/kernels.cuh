@@ -110,6 +110,8 @@ int hessian_splits_tiles(int64_t tiles, int64_t T, int sms);
 size_t prepare_ws_bytes(int64_t n);
 realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes);
+realq_status_t prepare_deferred(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U,
+                                float *Hbar, uint8_t *dead, void *ws, size_t ws_bytes);
 realq_status_t scale_copy(cudaStream_t s, int64_t count, float mul, const float *in, float *out);
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                                uint8_t *dead, int64_t *fail_col);

@@ -303,21 +303,25 @@ realq_status_t noalloc_scratch(void **out) {
 size_t prepare_ws_bytes(int64_t n) { return prepare_bytes_split(n, KSPLIT_MAX); }
 
 realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
-                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap);
+                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap, bool sync);
 
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                                uint8_t *dead, int64_t *fail_col) {
     void *scratch = nullptr;
     REALQ_TRY(noalloc_scratch(&scratch));
     // single stream: this entry point creates no stream or event
-    return prepare_impl(s, n, (double)T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes, false);
+    return prepare_impl(s, n, (double)T, damp, H, U, Hbar, dead, fail_col, scratch, kNoAllocBytes, false, true);
 }
 
-// Auxiliary stream of the calling thread (and its events) for the U row
-// work, one per (device, priority of the caller's stream), created on first
-// use and kept for the life of the thread.
+// Auxiliary streams of the calling thread (and their events) for the U row
+// work and the look-ahead, one set per (device, caller's stream, its
+// priority), created on first use and kept for the life of the thread.  Keyed
+// by the caller's stream so that calls on different streams (e.g. enqueued
+// one after another into one CUDA graph) share no stream and so no false
+// dependency.
 struct AuxStream {
     int device = -1, priority = 0;
+    cudaStream_t caller = nullptr;
     cudaStream_t stream = nullptr;       // U row work
     cudaStream_t wide = nullptr;         // the look-ahead's wide trailing updates
     cudaEvent_t ev[3] = {nullptr, nullptr, nullptr};
@@ -331,7 +335,7 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
     REALQ_CUDA_TRY(cudaStreamGetPriority(s, &prio));
     AuxStream *found = nullptr;
     for (AuxStream &x : g_aux)
-        if (x.device == dev && x.priority == prio) found = &x;
+        if (x.device == dev && x.priority == prio && x.caller == s) found = &x;
     if (!found) {
         AuxStream a;
         REALQ_CUDA_TRY(cudaStreamCreateWithPriority(&a.stream, cudaStreamNonBlocking, prio));
@@ -339,6 +343,7 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
         for (int i = 0; i < 3; ++i) REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.ev[i], cudaEventDisableTiming));
         a.device = dev;
         a.priority = prio;
+        a.caller = s;
         g_aux.push_back(a);
         found = &g_aux.back();
     }
@@ -356,11 +361,16 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
 
 realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes) {
-    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true);
+    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true, true);
+}
+
+realq_status_t prepare_deferred(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U,
+                                float *Hbar, uint8_t *dead, void *ws, size_t ws_bytes) {
+    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, nullptr, ws, ws_bytes, true, false);
 }
 
 realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
-                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap) {
+                            uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap, bool sync) {
     Carve cv(ws);
     int *status = cv.take<int>(1);
     float *lam = cv.take<float>(1);
@@ -398,6 +408,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
         REALQ_CUDA_TRY(cudaStreamWaitEvent(rs, aux->ev[0], 0));
     }
     std::vector<char> wide_pending(nbk + 1, 0);
+    bool wide_used = false;
     for (int K = nbk - 1; K >= 0; --K) {
         const int64_t k0 = (int64_t)K * NB;
         const int kb = (int)std::min<int64_t>(NB, n - k0);
@@ -449,6 +460,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
                 if (aux) {
                     REALQ_CUDA_TRY(cudaEventRecord(aux->wdone[K], aux->wide));
                     wide_pending[K] = 1;
+                    wide_used = true;
                 }
             }
         }
@@ -478,9 +490,14 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
     if (aux) {
         REALQ_CUDA_TRY(cudaEventRecord(aux->ev[1], rs));
         REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[1], 0));
-        REALQ_CUDA_TRY(cudaEventRecord(aux->ev[2], aux->wide));
-        REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[2], 0));
+        // join the wide stream only if it forked from s (under stream capture
+        // a wait on an event recorded outside the capture is an error)
+        if (wide_used) {
+            REALQ_CUDA_TRY(cudaEventRecord(aux->ev[2], aux->wide));
+            REALQ_CUDA_TRY(cudaStreamWaitEvent(s, aux->ev[2], 0));
+        }
     }
+    if (!sync) return REALQ_OK;  // the failing column stays in the workspace's first word
     int host_status = -1;
     REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
     REALQ_CUDA_TRY(cudaStreamSynchronize(s));

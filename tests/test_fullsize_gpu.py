@@ -1,7 +1,8 @@
 """Parity at the full size of the Qwen3-0.6B-shaped decoder block (4 inputs of
 262,144 tokens, 7 modules, asymmetric g128 W4, Block-GD with Adam at lr 3e-4),
 run exactly as the benchmark times it: the library's concurrent block
-scheduler, one stream per input and per module.
+scheduler, one stream per input and per module, captured into a CUDA graph
+and replayed (the outputs are cleared between the capture and the replay).
 
 The fp64 oracle computes its own Hessians of all four inputs (bf16 values and
 their products are exact in fp64), and everything else from those:
@@ -47,7 +48,11 @@ def block_run():
     bq = BlockQuantizer([BlockInput(nm, sp.n, sp.T) for nm, sp in wl.inputs.items()],
                         [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
                         wl.steps_per_block, sliding_window=wl.sliding_window, device=dev)
-    bq.run(X, W0, F)
+    bq.capture(X, W0, F)
+    for o in bq.out.values():
+        for k in ("codes", "scale", "zero", "W"):
+            o[k].fill_(0 if o[k].dtype == torch.uint8 else float("nan"))
+    bq.replay()
     torch.cuda.synchronize()
     bq.check_status()
     return wl, bq, x_bits, w_bits, F_np

@@ -741,3 +741,90 @@ def test_minibatch_block_gd(start, steps):
     print(f"\nmini-batch start={start} steps={steps}: {rep} scale_within_1e-5={frac:.5f}")
     assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
     assert s_unexpl == 0
+
+
+def test_prepare_deferred_status():
+    # the capturable prepare leaves the failing column in its workspace
+    n = 96
+    H = -torch.eye(n, device="cuda") * 10.0
+    U, Hbar = torch.empty(n, n, device="cuda"), torch.empty(n, n, device="cuda")
+    dead = torch.empty(n, dtype=torch.uint8, device="cuda")
+    ws = rq.workspace(rq.realq_prepare_workspace_size(n))
+    rq.realq_hessian_prepare_deferred(H, 10, 0.01, U, Hbar, dead, ws)
+    with pytest.raises(rq.RealqError) as ei:
+        rq.realq_prepare_status(ws)
+    assert ei.value.status == rq.REALQ_ERR_NOT_SPD and ei.value.fail_col == n - 1
+    case = synth.layer_case(23, 4, n, 4 * n, outliers=2)
+    Href, T = oracle.hessian_sum([case.Xhat])
+    rq.realq_hessian_prepare_deferred(dev(Href), T, 0.01, U, Hbar, dead, ws)
+    assert rq.realq_prepare_status(ws) == -1
+    ref = oracle.prepare(Href, T, 0.01)
+    Uref = oracle.inverse_upper_cholesky(ref["Hd"])
+    assert np.abs(U.cpu().numpy() - Uref).max() <= 2e-4 * np.abs(Uref).max()
+
+
+@pytest.mark.parametrize("variant", ["plain", "minibatch", "w4a4", "host"])
+def test_block_graph_replay_matches_eager(variant):
+    # capture() / capture_host() and replay() give the eager step's outputs
+    # bit for bit, and a replay recomputes them (outputs are cleared first)
+    from paper_2609_00049_gb300.block import BlockInput, BlockModule, BlockQuantizer
+    r = synth.rng(44, "block-graph-" + variant)
+    T = 4096 + 320
+    ins = {"a": 128, "b": 192}
+    mods = [("m1", 64, "a"), ("m2", 200, "a"), ("m3", 96, "b")]
+    x_bits = {k: synth.f32_to_bf16_bits(r.standard_normal((T, n)) * (1 + 9 * (r.random(n) < 0.02)))
+              for k, n in ins.items()}
+    Wf = {nm: synth.bf16_bits_to_f32(synth.f32_to_bf16_bits(r.standard_normal((m, ins[i])) * 0.02))
+          for nm, m, i in mods}
+    Ff = {}
+    for nm, m, _ in mods:
+        z = r.standard_normal((m, 4))
+        Ff[nm] = (np.eye(m) * 0.5 + z @ z.T / 8).astype(np.float32)
+    qcfg = rq.quant_cfg(4, 64, 64, 0, 0.01)
+    kw = dict(minibatch_tokens=1024) if variant == "minibatch" else {}
+    if variant == "w4a4":
+        kw = dict(act_quant=(4, 0.9))
+    if variant == "host":
+        kw = dict(host_chunk_tokens=1024)   # five chunks, the last one ragged
+    bq = BlockQuantizer([BlockInput(k, n, T) for k, n in ins.items()],
+                        [BlockModule(nm, m, ins[i], i) for nm, m, i in mods], qcfg, 2e-4, 1, **kw)
+    X = {k: bf16_dev(v) for k, v in x_bits.items()}
+    W0 = {nm: dev(w) for nm, w in Wf.items()}
+    F = {nm: dev(f) for nm, f in Ff.items()}
+    keys = ("codes", "scale", "zero", "W")
+    if variant == "host":
+        # chunked accumulation sums in another order than the one-shot
+        # Hessian: the eager reference is run_host itself
+        X_h = {k: v.cpu().pin_memory() for k, v in X.items()}
+        W_h = {k: v.cpu().pin_memory() for k, v in W0.items()}
+        F_h = {k: v.cpu().pin_memory() for k, v in F.items()}
+        out_h = {nm: {k: torch.empty_like(bq.out[nm][k], device="cpu").pin_memory() for k in keys[:3]}
+                 for nm, _, _ in mods}
+        bq.run_host(X_h, W_h, F_h, out_h)
+    else:
+        bq.run(X, W0, F)
+    torch.cuda.synchronize()
+    bq.check_status()
+    eager = {nm: {k: bq.out[nm][k].clone() for k in keys} for nm, _, _ in mods}
+    if variant == "host":
+        h2d, d2h = bq.capture_host(X_h, W_h, F_h, out_h)
+        assert h2d == sum(v.numel() * v.element_size() for d in (X_h, W_h, F_h) for v in d.values())
+        assert d2h == sum(v.numel() * v.element_size() for d in out_h.values() for v in d.values())
+    else:
+        bq.capture(X, W0, F)
+    for _ in range(2):
+        for nm, _, _ in mods:
+            for k in keys:
+                bq.out[nm][k].fill_(0 if bq.out[nm][k].dtype == torch.uint8 else float("nan"))
+            if variant == "host":
+                for k in keys[:3]:
+                    out_h[nm][k].fill_(0 if out_h[nm][k].dtype == torch.uint8 else float("nan"))
+        bq.replay()
+        torch.cuda.synchronize()
+        bq.check_status()
+        for nm, _, _ in mods:
+            for k in keys:
+                assert torch.equal(bq.out[nm][k], eager[nm][k]), (variant, nm, k)
+            if variant == "host":
+                for k in keys[:3]:
+                    assert torch.equal(out_h[nm][k], eager[nm][k].cpu()), (variant, nm, k)
