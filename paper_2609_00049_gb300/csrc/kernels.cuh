@@ -163,7 +163,16 @@ struct SweepPlan {
     std::vector<TcMaps> mapsMB;
     int f_split_alpha_valid;
     float f_split_alpha;
+    // The optimizer step's G product is split: the next block's columns on
+    // the sweep's stream (the next OBS block needs only those), the other
+    // free columns on a side stream, joined before anything else reads or
+    // writes them.  wide == nullptr: everything on the sweep's stream.
+    cudaStream_t wide = nullptr;
+    cudaEvent_t wide_fork = nullptr, wide_done = nullptr;
+    int wide_pending = 0;
 };
+realq_status_t sweep_side_stream(cudaStream_t s, SweepPlan &p);
+realq_status_t sweep_join_wide(cudaStream_t s, SweepPlan &p);
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0,
                       int nmb = 0);
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);

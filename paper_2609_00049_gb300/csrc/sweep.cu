@@ -553,15 +553,13 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
 // M = A H̄ up to date for them: the last step moved A only in its own free
 // columns [step_c, n), so M[:, c0:] += step[:, step_c:] H̄[step_c:, c0:]
 // (K = n - step_c instead of n), then the epilogue forms P from M.
-static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
+// G = F_eff P on the free columns c0.. and one Adam step on them (fused).
+// For the last step of a block with a side stream, the next block's columns
+// (c0 .. c0 + B) run on s and the rest on the side stream: the next OBS block
+// waits only for its own columns, and sweep_join_wide orders the rest before
+// the next trailing update (the next reader or writer of those columns).
+static realq_status_t g_adam(cudaStream_t s, SweepPlan &p, int64_t c0, bool last) {
     const int64_t r = p.n - c0;
-    const int64_t k0 = p.step_c;
-    TcEpi e{};
-    e.mode = TC_BGD_P;
-    e.Ad = p.disp; e.W = p.W; e.W0 = p.W0; e.w0_bf16 = p.w_dtype == REALQ_BF16;
-    e.dead = p.dead; e.lam = p.lam; e.R0 = p.R0; e.ldw = p.n; e.col0 = c0;
-    e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m; e.M = p.M;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
     const int64_t t = ++(*p.adam_t);
     TcEpi g{};
     g.mode = TC_ADAM;
@@ -571,7 +569,77 @@ static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
     g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
     g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
     g.sgd = p.optimizer == REALQ_OPT_SGD;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    const int64_t nb = std::min<int64_t>(p.block, r);
+    if (!last || !p.wide || r <= nb) return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
+    REALQ_CUDA_TRY(cudaEventRecord(p.wide_fork, s));
+    REALQ_CUDA_TRY(cudaStreamWaitEvent(p.wide, p.wide_fork, 0));
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, nb, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    TcEpi gw = g;
+    gw.col0 = c0 + nb;
+    REALQ_TRY(tc_gemm_tf32x3(p.wide, p.mapsG, p.m, r - nb, p.m, 0, (int)nb, gw, p.status, "bgd_g_gemm_adam"));
+    REALQ_CUDA_TRY(cudaEventRecord(p.wide_done, p.wide));
+    p.wide_pending = 1;
+    return REALQ_OK;
+}
+
+realq_status_t sweep_join_wide(cudaStream_t s, SweepPlan &p) {
+    if (!p.wide_pending) return REALQ_OK;
+    REALQ_CUDA_TRY(cudaStreamWaitEvent(s, p.wide_done, 0));
+    p.wide_pending = 0;
+    return REALQ_OK;
+}
+
+// Side stream of the calling thread for the split G product, one per
+// (device, caller's stream, its priority), created on first use and kept for
+// the life of the thread.
+namespace {
+struct SideStream {
+    int device = -1, priority = 0;
+    cudaStream_t caller = nullptr, stream = nullptr;
+    cudaEvent_t fork = nullptr, done = nullptr;
+};
+thread_local std::vector<SideStream> g_side;
+}  // namespace
+
+realq_status_t sweep_side_stream(cudaStream_t s, SweepPlan &p) {
+    int dev = 0, prio = 0;
+    REALQ_CUDA_TRY(cudaGetDevice(&dev));
+    REALQ_CUDA_TRY(cudaStreamGetPriority(s, &prio));
+    SideStream *f = nullptr;
+    for (SideStream &x : g_side)
+        if (x.device == dev && x.priority == prio && x.caller == s) f = &x;
+    if (!f) {
+        // one step below the caller's priority: when the side product's CTAs
+        // hold the SMs, the next OBS block's CTAs are placed first as they free
+        int least = 0, greatest = 0;
+        REALQ_CUDA_TRY(cudaDeviceGetStreamPriorityRange(&least, &greatest));
+        SideStream a;
+        REALQ_CUDA_TRY(cudaStreamCreateWithPriority(&a.stream, cudaStreamNonBlocking, std::min(prio + 1, least)));
+        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.fork, cudaEventDisableTiming));
+        REALQ_CUDA_TRY(cudaEventCreateWithFlags(&a.done, cudaEventDisableTiming));
+        a.device = dev;
+        a.priority = prio;
+        a.caller = s;
+        g_side.push_back(a);
+        f = &g_side.back();
+    }
+    p.wide = f->stream;
+    p.wide_fork = f->fork;
+    p.wide_done = f->done;
+    p.wide_pending = 0;
+    return REALQ_OK;
+}
+
+static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0, bool last) {
+    const int64_t r = p.n - c0;
+    const int64_t k0 = p.step_c;
+    TcEpi e{};
+    e.mode = TC_BGD_P;
+    e.Ad = p.disp; e.W = p.W; e.W0 = p.W0; e.w0_bf16 = p.w_dtype == REALQ_BF16;
+    e.dead = p.dead; e.lam = p.lam; e.R0 = p.R0; e.ldw = p.n; e.col0 = c0;
+    e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m; e.M = p.M;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
+    REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
     return REALQ_OK;
 }
@@ -582,7 +650,7 @@ static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0) {
 //   M_g + lambda_g (A - ΔW) - ΔW (H̄_g - H̄),   M_g = A H̄_g  (rows of g),
 // which is the one-Hessian form when H̄_g = H̄.  M_g is kept current like M;
 // ΔW (H̄_g - H̄) takes the full K = n.  Then G = F_eff P and Adam for all rows.
-static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c0) {
+static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c0, bool last) {
     const int64_t r = p.n - c0;
     const int64_t k0 = p.step_c;
     if (p.w_dtype == REALQ_BF16)
@@ -609,16 +677,7 @@ static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c
         q.Pth = p.Pth + row0; q.Ptl = p.Ptl + row0; q.ldp = p.m;
         REALQ_TRY(tc_gemm_tf32x3(s, p.mapsQg[gr], rows, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm", (int)row0));
     }
-    const int64_t t = ++(*p.adam_t);
-    TcEpi g{};
-    g.mode = TC_ADAM;
-    g.ldw = p.n; g.col0 = c0;
-    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
-    g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
-    g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
-    g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
-    g.sgd = p.optimizer == REALQ_OPT_SGD;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
     return REALQ_OK;
 }
@@ -626,7 +685,7 @@ static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c
 // One optimizer step on a calibration mini-batch: the gradient factor is
 // ((Ŵ - W0) H̄_mb)_R = (stationarity form with H̄)_R + (ΔW (H̄_mb - H̄))_R,
 // i.e. M + lambda (A - ΔW) - ΔW (H̄ - H̄_mb,k), with M = A H̄ kept current.
-static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, int kmb) {
+static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, int kmb, bool last) {
     const int64_t r = p.n - c0;
     const int64_t k0 = p.step_c;
     if (p.w_dtype == REALQ_BF16)
@@ -646,16 +705,7 @@ static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, in
     q.ldw = p.n; q.col0 = c0; q.M = p.M;
     q.Pth = p.Pth; q.Ptl = p.Ptl; q.ldp = p.m;
     REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMB[kmb], p.m, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm"));
-    const int64_t t = ++(*p.adam_t);
-    TcEpi g{};
-    g.mode = TC_ADAM;
-    g.ldw = p.n; g.col0 = c0;
-    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
-    g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
-    g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
-    g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
-    g.sgd = p.optimizer == REALQ_OPT_SGD;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
     return REALQ_OK;
 }
@@ -677,6 +727,8 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     // a single group no wider than a block is handled inside the block kernel
     const int params_here = p.group <= B || (p.group >= p.n && p.n <= B);
     if (!params_here && bs % p.group == 0) {
+        // a group wider than the block reads columns beyond it
+        REALQ_TRY(sweep_join_wide(s, p));
         Launch L("group_params", s);
         group_params_kernel<<<ceil_div(p.m, 8), 256, 0, s>>>(p.m, p.n, p.W, bs, std::min<int64_t>(bs + p.group, p.n),
                                                               (int)(bs / p.group), p.ngroups, p.bits, p.sym, p.scale,
@@ -708,6 +760,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             copy_cols_kernel<<<blocks_for(p.m * kb), 256, 0, s>>>(p.m, p.n, bs, be, p.W, static_cast<float *>(p.W_deq));
     }
     if (p.W_deq) REALQ_TRY(check_launch("copy_deq"));
+    REALQ_TRY(sweep_join_wide(s, p));
     if (be >= p.n) return REALQ_OK;
     // lazy batch update of every later column: W[:, be:] -= E_b U[bs:be, be:]
     // (per row group with its own U)
@@ -736,10 +789,11 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             p.f_split_alpha = a_eff;
         }
         for (int k = 0; k < p.bgd_steps; ++k) {
+            const bool last = k == p.bgd_steps - 1;
             if (p.nmb > 0)
-                REALQ_TRY(bgd_one_tc_mb(s, p, be, (int)(((b_global - 1) * p.bgd_steps + k) % p.nmb)));
+                REALQ_TRY(bgd_one_tc_mb(s, p, be, (int)(((b_global - 1) * p.bgd_steps + k) % p.nmb), last));
             else
-                REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be) : bgd_one_tc(s, p, be));
+                REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be, last) : bgd_one_tc(s, p, be, last));
         }
         return REALQ_OK;
     }
