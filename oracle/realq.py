@@ -36,6 +36,7 @@ __all__ = [
     "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
     "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
     "round_bf16", "quantize_activations", "saliency_clip", "weighted_hessian_sum",
+    "loss_clip_factors", "gradient_tokens", "surrogate_tokens_clipped",
 ]
 
 
@@ -239,6 +240,61 @@ def gradient(What, W0, Hbar, Dbar, F) -> np.ndarray:
     return np.asarray(F, dtype=np.float64) @ P
 
 
+# ---------------------------------------------------------------------------
+# Output-perturbation clipping of the Block-GD loss (App. "Activation
+# clipping (a_loss_clip) for small Qwen3 models": a_loss_clip = 0.95 on
+# Qwen3-0.6B, 1.7B and 4B).  Per token, the output channels whose |Δy| lies
+# above the 95th percentile are scaled down by a detached factor, so that a
+# few outlier channels cannot dominate the Fisher MSE while their gradient
+# stays non-zero.
+# Readings: the percentile is taken per token over its m output channels, as
+# the nearest-rank one of the saliency clip (the ceil(pct m)-th smallest
+# |Δy_t,i|, pct as a single-precision value); a channel above it is scaled by
+# kappa = q_t / |Δy_t,i| (its scaled residual has magnitude q_t), every other
+# channel by 1; kappa is a constant of the step (detached), so with
+# L = (1/2T) sum_t (kappa_t ⊙ Δy_t)^T F (kappa_t ⊙ Δy_t)
+# the gradient is dL/dŴ = (1/T) sum_t (kappa_t ⊙ F (kappa_t ⊙ Δy_t)) x̂_t^T.
+# The factors depend on the tokens, so this gradient is taken in token form
+# on the step's mini-batch.  kappa is continuous in Δy (it is 1 at the
+# threshold), so rounding differences near the threshold move it by no more
+# than they move Δy.
+# ---------------------------------------------------------------------------
+def loss_clip_factors(dY: np.ndarray, pct: float):
+    """kappa (T x m) and the per-token thresholds q (T) for residuals dY (T x m)."""
+    dY = np.asarray(dY, dtype=np.float64)
+    m = dY.shape[1]
+    p32 = float(np.float32(pct))
+    k = min(max(int(math.ceil(p32 * m)) - 1, 0), m - 1)
+    a = np.abs(dY)
+    q = np.sort(a, axis=1)[:, k]
+    kappa = np.ones_like(a)
+    over = a > q[:, None]
+    kappa[over] = (q[:, None] / np.where(over, a, 1.0))[over]
+    return kappa, q
+
+
+def gradient_tokens(What, W0, Xhat, X, F, a_loss_clip: Optional[float] = None) -> np.ndarray:
+    """dL/dŴ (m x n) on the tokens Xhat (T x n), in token form: Δy_t = Ŵ x̂_t - W0 x_t,
+    (1/T) sum_t (kappa_t ⊙ F (kappa_t ⊙ Δy_t)) x̂_t^T with kappa = 1 without clipping."""
+    What = np.asarray(What, dtype=np.float64)
+    W0 = np.asarray(W0, dtype=np.float64)
+    F = np.asarray(F, dtype=np.float64)
+    Xh = np.asarray(Xhat, dtype=np.float64)
+    Xf = Xh if X is None else np.asarray(X, dtype=np.float64)
+    dY = Xh @ What.T - Xf @ W0.T
+    kappa = np.ones_like(dY) if a_loss_clip is None else loss_clip_factors(dY, a_loss_clip)[0]
+    Z = (kappa * dY) @ F
+    return (kappa * Z).T @ Xh / float(Xh.shape[0])
+
+
+def surrogate_tokens_clipped(What, W0, Xhat, F, kappa) -> float:
+    """(1/2)(1/T) sum_t (kappa_t ⊙ Δy_t)^T F (kappa_t ⊙ Δy_t) with given factors."""
+    Xh = np.asarray(Xhat, dtype=np.float64)
+    dY = Xh @ (np.asarray(What, dtype=np.float64) - np.asarray(W0, dtype=np.float64)).T
+    Y = np.asarray(kappa, dtype=np.float64) * dY
+    return 0.5 * float(np.sum((Y @ np.asarray(F, dtype=np.float64)) * Y)) / Xh.shape[0]
+
+
 def pack_codes(codes: np.ndarray) -> np.ndarray:
     """Two int4 codes per byte, even column in the low nibble (m x ceil(n/2) uint8)."""
     m, n = codes.shape
@@ -264,7 +320,11 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
       surrogate on a calibration mini-batch; Sec. 5.1: 32 sequences).  Step s
       (0-based) of the block with global index b_global uses mini-batch
       ((b_global - 1) * steps_per_block + s) mod K, so consecutive steps of a
-      transformer block rotate through the calibration set.
+      transformer block rotate through the calibration set; or
+      minibatch_tokens: a list of K token blocks X̂_k (T_k x n) with the same
+      rotation, whose gradient is taken in token form, and then optionally
+      a_loss_clip: the per-token output clipping percentile (0.95 in the
+      paper's small-model runs; see loss_clip_factors).
 
     Readings: group parameters are computed at the first column of each group
     from the current (compensated, Block-GD-updated) weights; group_size 0
@@ -345,15 +405,22 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
             before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
             mbs = bgd.get("minibatches")
+            mbt = bgd.get("minibatch_tokens")
             steps = bgd.get("steps_per_block", 1)
             for si in range(steps):
                 Hstep = Hbar
-                if mbs:
+                if mbt:
                     if Dbar is not None:
-                        raise ValueError("mini-batch moments with perturbed inputs are not supported")
-                    Hk, Tk = mbs[((b_global - 1) * steps + si) % len(mbs)]
-                    Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)
-                G = gradient(W, W0, Hstep, Dbar, Feff)[:, be:]
+                        raise ValueError("mini-batch tokens with perturbed inputs are not supported")
+                    Xk = mbt[((b_global - 1) * steps + si) % len(mbt)]
+                    G = gradient_tokens(W, W0, Xk, None, Feff, bgd.get("a_loss_clip"))[:, be:]
+                else:
+                    if mbs:
+                        if Dbar is not None:
+                            raise ValueError("mini-batch moments with perturbed inputs are not supported")
+                        Hk, Tk = mbs[((b_global - 1) * steps + si) % len(mbs)]
+                        Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)
+                    G = gradient(W, W0, Hstep, Dbar, Feff)[:, be:]
                 if bgd.get("optimizer", "adam") == "sgd":
                     opt.t += 1
                     W[:, be:] -= bgd["lr"] * G

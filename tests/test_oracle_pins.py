@@ -551,3 +551,94 @@ def test_minibatch_rotation_rule():
     # the mean of the mini-batch moments is the full-batch moment
     Hs = [oracle.hessian_sum([X[k * 100:(k + 1) * 100]])[0] for k in range(4)]
     np.testing.assert_allclose(sum(Hs) / T, H / T, rtol=1e-13, atol=1e-15)
+
+
+# ---------------------------------------------------------------------------
+# output-perturbation clipping of the Block-GD loss (a_loss_clip) and the
+# token-form gradient it needs
+# ---------------------------------------------------------------------------
+def test_loss_clip_worked_example():
+    # one token with residuals 1..20 (shuffled, signs alternating): the 95th
+    # nearest-rank percentile of 20 channels is the 19th smallest |Δy| = 19
+    # (float32(0.95) = 0.949999988, times 20 = 18.99999976, rank 19), so only
+    # the channel with |Δy| = 20 is scaled, by 19/20
+    perm = np.random.default_rng(5).permutation(20)
+    dY = (np.arange(1, 21, dtype=np.float64) * np.where(np.arange(20) % 2, -1.0, 1.0))[perm][None, :]
+    kappa, q = oracle.loss_clip_factors(dY, 0.95)
+    assert q[0] == 19.0
+    expect = np.ones(20)
+    expect[np.abs(dY[0]) == 20.0] = 19.0 / 20.0
+    assert np.array_equal(kappa[0], expect)
+    # 0.99 of 100 channels: float32(0.99) = 0.99000001, times 100 =
+    # 99.0000009, rank 100: the threshold is the maximum and nothing is scaled;
+    # 0.98 of 100: float32(0.98) = 0.98000002, times 100 = 98.0000019, rank 99
+    dY = np.arange(1, 101, dtype=np.float64)[None, :]
+    kappa, q = oracle.loss_clip_factors(dY, 0.99)
+    assert q[0] == 100.0 and np.all(kappa == 1.0)
+    kappa, q = oracle.loss_clip_factors(dY, 0.98)
+    assert q[0] == 99.0 and np.all(kappa[0, :99] == 1.0) and kappa[0, 99] == 99.0 / 100.0
+
+
+def test_loss_clip_invariants():
+    # per token: the scaled residuals never exceed the threshold, those above
+    # it land exactly on it, and m - rank channels are scaled (distinct values)
+    r = np.random.default_rng(6)
+    dY = r.standard_t(3, size=(50, 64)) * np.exp(r.standard_normal((50, 1)))
+    kappa, q = oracle.loss_clip_factors(dY, 0.95)
+    k = math.ceil(float(np.float32(0.95)) * 64)
+    Y = np.abs(kappa * dY)
+    assert np.all(Y <= q[:, None] * (1 + 1e-15))
+    np.testing.assert_allclose(Y.max(axis=1), q, rtol=1e-15)
+    assert np.all((kappa < 1.0).sum(axis=1) == 64 - k)
+    assert np.all((kappa > 0) & (kappa <= 1.0))
+
+
+def test_token_gradient_without_clipping_is_the_moment_gradient():
+    # kappa = 1: the token form equals F (Ŵ - W0) H̄ on the same tokens
+    r, X, W0, F = _grouped_case(68)
+    What = W0 + r.standard_normal(W0.shape) * 0.003
+    H, T = oracle.hessian_sum([X])
+    Gm = oracle.gradient(What, W0, H / T, None, F)
+    Gt = oracle.gradient_tokens(What, W0, X, None, F)
+    np.testing.assert_allclose(Gt, Gm, rtol=1e-11, atol=1e-15)
+    # a percentile at the maximum scales nothing
+    Gc = oracle.gradient_tokens(What, W0, X, None, F, a_loss_clip=1.0)
+    np.testing.assert_allclose(Gc, Gm, rtol=1e-11, atol=1e-15)
+
+
+def test_clipped_gradient_is_the_gradient_of_the_detached_loss():
+    # central differences of L_kappa (kappa frozen at Ŵ) on sampled entries:
+    # the loss is quadratic in Ŵ for fixed kappa, so they are exact up to
+    # rounding
+    r, X, W0, F = _grouped_case(69, m=12, n=10, T=60)
+    X[:, 2] *= 40.0                                  # a few large residual channels
+    What = W0 + r.standard_normal(W0.shape) * 0.01
+    dY = X @ (What - W0).T
+    kappa, _ = oracle.loss_clip_factors(dY, 0.9)
+    assert (kappa < 1).any()
+    G = oracle.gradient_tokens(What, W0, X, None, F, a_loss_clip=0.9)
+    h = 1e-4
+    for i, j in [(0, 0), (3, 2), (11, 9), (5, 7)]:
+        E = np.zeros_like(What)
+        E[i, j] = h
+        fd = (oracle.surrogate_tokens_clipped(What + E, W0, X, F, kappa)
+              - oracle.surrogate_tokens_clipped(What - E, W0, X, F, kappa)) / (2 * h)
+        assert abs(fd - G[i, j]) <= 1e-8 * max(1.0, abs(G[i, j])), (i, j, fd, G[i, j])
+
+
+def test_token_minibatch_sweep_reduces_to_the_moment_minibatch_sweep():
+    # without clipping the token-form mini-batch sweep is the moment-form one
+    r, X, W0, F = _grouped_case(70)
+    H, T = oracle.hessian_sum([X])
+    parts = [X[k * 100:(k + 1) * 100] for k in range(4)]
+    base = {"lr": 2e-4, "steps_per_block": 1, "b_global_start": 2, "B_total": 1}
+    a = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, F=F,
+                           bgd={**base, "minibatches": [oracle.hessian_sum([p]) for p in parts]})
+    b = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, F=F, bgd={**base, "minibatch_tokens": parts})
+    assert np.array_equal(a["codes"], b["codes"])
+    np.testing.assert_allclose(b["deq"], a["deq"], rtol=0, atol=1e-12)
+    # with clipping the sweep differs, and only after the first block
+    c = oracle.realq_sweep(W0, H, T, group_size=16, block_size=16, F=F,
+                           bgd={**base, "minibatch_tokens": parts, "a_loss_clip": 0.95})
+    assert np.array_equal(c["codes"][:, :16], a["codes"][:, :16])
+    assert not np.allclose(c["deq"][:, 16:], a["deq"][:, 16:], rtol=0, atol=1e-9)
