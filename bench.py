@@ -160,7 +160,8 @@ def gpu_arm(args, wl, rank, world):
                         [BlockModule(md.name, md.m, md.n, md.input) for md in wl.modules], qcfg, wl.lr,
                         wl.steps_per_block, sliding_window=wl.sliding_window, device=dev,
                         act_quant=(args.act_bits, args.a_clip) if args.act_bits else None,
-                        saliency_groups=args.saliency_groups, minibatch_tokens=2048 * args.minibatch_seqs)
+                        saliency_groups=args.saliency_groups, minibatch_tokens=2048 * args.minibatch_seqs,
+                        a_loss_clip=args.a_loss_clip)
     dev_sal = None
     if args.saliency_groups:
         dev_sal = {mod.name: torch.from_numpy(synth.saliency(wl, mod, args.saliency_groups)).to(dev)
@@ -288,7 +289,9 @@ def gpu_arm(args, wl, rank, world):
                                     (f", saliency-weighted grouped Hessians (N_g={args.saliency_groups}, clip p99)"
                                      if args.saliency_groups else ""),
                        "bgd": f"Adam lr={wl.lr} steps_per_block={wl.steps_per_block}" +
-                              (f", mini-batches of {args.minibatch_seqs} x 2048 tokens" if args.minibatch_seqs else ""),
+                              (f", mini-batches of {args.minibatch_seqs} x 2048 tokens" if args.minibatch_seqs else "") +
+                              (f", token-form gradient with a_loss_clip {args.a_loss_clip}" if args.a_loss_clip
+                               else ""),
                        "parallelism": f"replicas x{world}",
                        "launch": "one CUDA graph per step (11 streams)" if use_graph else
                                  "eager, one host thread per input",
@@ -339,6 +342,27 @@ def roofline(wl, prof, steps, peaks, args=None):
             bgd_g += 2 * m * m * r
             trail += 2 * m * (be - b * B) * r
             serial_bytes += m * (be - b * B) * (4 + 4 + 4) + m * (be - b * B) // 2
+    if getattr(args, "a_loss_clip", None) and getattr(args, "minibatch_seqs", 0):
+        # token-form gradient per optimizer step (every block but the last):
+        # Δ = X̂_k ΔWᵀ, Z = (κ ⊙ Δ) F, G = gᵀ X̂_k[:, free] on T_k tokens
+        tr = tf = tg = clip_b = conv_b = gt_b = 0
+        for md in wl.modules:
+            m, n, B = md.m, md.n, wl.block_size
+            Tk = min(2048 * args.minibatch_seqs, wl.inputs[md.input].T)
+            for b in range(-(-n // B) - 1):
+                r = n - min((b + 1) * B, n)
+                tr += 2 * Tk * m * n
+                tf += 2 * Tk * m * m
+                tg += 2 * m * r * Tk
+                clip_b += Tk * m * 16          # read Δ, write κ and Y's two planes
+                conv_b += Tk * n * 10          # read bf16, write fp32 both ways
+                gt_b += Tk * m * 16            # read κ and Z, write two planes
+        per_step["tok_residual_gemm"] = ("tf32x3", tr, "TFLOP/s")
+        per_step["tok_fisher_gemm"] = ("tf32x3", tf, "TFLOP/s")
+        per_step["tok_grad_gemm"] = ("tf32x3", tg, "TFLOP/s")
+        per_step["tok_clip"] = ("hbm", clip_b, "GB/s")
+        per_step["tok_xconv"] = ("hbm", conv_b, "GB/s")
+        per_step["tok_grad_t"] = ("hbm", gt_b, "GB/s")
     per_step["bgd_p_gemm"] = ("tf32x3", bgd_p, "TFLOP/s")
     per_step["bgd_g_gemm_adam"] = ("tf32x3", bgd_g, "TFLOP/s")
     per_step["trailing_update"] = ("alu", trail, "TFLOP/s")
@@ -513,6 +537,8 @@ def main():
                     help="mini-batch Block-GD with this many 2048-token sequences per step (0: full batch)")
     ap.add_argument("--saliency-groups", type=int, default=0,
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
+    ap.add_argument("--a-loss-clip", type=float, default=None,
+                    help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--no-graph", action="store_true", help="launch the block step eagerly instead of as a CUDA graph")

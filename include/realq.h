@@ -177,6 +177,41 @@ realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, i
                                              const float *H_sum, float *U_out, float *Hbar_out, uint8_t *dead_out,
                                              int64_t *fail_col);
 
+/* Token-form mini-batch Block-GD with per-token output clipping (Sec. 4.3,
+ * "a calibration mini-batch" per step, 32 sequences in Sec. 5.1; App.
+ * "Activation clipping (a_loss_clip) for small Qwen3 models", 0.95 there).
+ * The same sweep as realq_quantize_layer_minibatch, but each optimizer step
+ * takes its gradient from the mini-batch's tokens:
+ *   Δ_t = (Ŵ - W0) x̂_t                       (m, per token of the mini-batch)
+ *   q_t = the ceil(a_loss_clip m)-th smallest |Δ_t,i| (a_loss_clip as given,
+ *         single precision; the product is taken exactly)
+ *   kappa_t,i = q_t / |Δ_t,i| if |Δ_t,i| > q_t, else 1   (held constant)
+ *   G = (1/T_k) sum_t (kappa_t ⊙ F_eff (kappa_t ⊙ Δ_t)) x̂_tᵀ, free columns
+ * and one optimizer step per G.  Mini-batch k holds tokens
+ * [k T_mb, min((k+1) T_mb, T)) of X_hat; step s of the block with global
+ * index b_global uses k = ((b_global - 1) steps_per_block + s) mod
+ * ceil(T / T_mb).  a_loss_clip = 1 scales no channel: the gradient is then
+ * the moment form on the mini-batch (F_eff (Ŵ - W0) H̄_k).
+ *   X_hat   T x n bf16, token-major, 16-byte aligned, n % 8 == 0; the
+ *           calibration tokens whose H gave U and Hbar (unperturbed: the
+ *           reference output is W0 x̂).
+ *   T_mb    tokens per mini-batch, a multiple of 4.
+ * Needs the tensor-core path (m, n multiples of 4, >= 32; block_size > 0).
+ * Everything else as realq_quantize_layer.  The products take the token
+ * axis on the tensor cores in fp32-level precision (tf32x3); the workspace
+ * holds the mini-batch twice in fp32 plus four T_mb x m buffers. */
+size_t realq_quantize_tokens_workspace_size(int64_t m, int64_t n, int64_t T_mb, const realq_quant_cfg_t *qcfg,
+                                            const realq_bgd_cfg_t *bcfg, int has_F_next);
+realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                           realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                           const uint8_t *dead, const void *X_hat, int64_t T, int64_t T_mb,
+                                           float a_loss_clip, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                           float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
+                                           size_t ws_bytes);
+
 /* Weight-activation setting (Sec. 5, "Weight-Activation Quantization";
  * W4A4 uses 4 bits and a_clip = 0.9).  Per-token symmetric quantization of
  * the calibration activations X (T x n, row-major, REALQ_BF16 or REALQ_F32):

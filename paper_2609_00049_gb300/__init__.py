@@ -24,7 +24,7 @@ __all__ = [
     "realq_quantize_activations", "realq_saliency_clip", "realq_hessian_weighted_workspace_size",
     "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled", "realq_quantize_layer_grouped",
     "realq_quantize_grouped_workspace_size", "realq_quantize_layer_minibatch",
-    "realq_quantize_minibatch_workspace_size",
+    "realq_quantize_minibatch_workspace_size", "realq_quantize_tokens_workspace_size", "realq_quantize_layer_tokens",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -102,6 +102,11 @@ _SIGS = {
                                       _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_minibatch_workspace_size": ([_i64, _i64, _int, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
                                                  _int], _sz),
+    "realq_quantize_tokens_workspace_size": ([_i64, _i64, _i64, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
+                                              _int], _sz),
+    "realq_quantize_layer_tokens": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64, _i64, _f32,
+                                     ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp,
+                                     _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_layer_minibatch": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _int, _vp,
                                         ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp,
                                         _vp, _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
@@ -472,6 +477,42 @@ def realq_quantize_layer_minibatch(W0: torch.Tensor, U: torch.Tensor, Hbar: torc
         ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next), _ptr(W_work),
         _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
         _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
+    return t.value
+
+
+def realq_quantize_tokens_workspace_size(m: int, n: int, T_mb: int, qcfg: QuantCfg, bcfg: Optional[BgdCfg] = None,
+                                         has_F_next: bool = False) -> int:
+    return int(lib().realq_quantize_tokens_workspace_size(m, n, int(T_mb), ctypes.byref(qcfg),
+                                                          ctypes.byref(bcfg) if bcfg is not None else None,
+                                                          int(has_F_next)))
+
+
+def realq_quantize_layer_tokens(W0: torch.Tensor, U: torch.Tensor, Hbar: torch.Tensor, X_hat: torch.Tensor,
+                                T_mb: int, a_loss_clip: float, qcfg: QuantCfg, W_work: torch.Tensor,
+                                codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *, dead=None,
+                                bcfg: Optional[BgdCfg] = None, F=None, F_next=None, adam_m=None, adam_v=None,
+                                bgd_disp=None, adam_t: int = 0, W_deq=None, block_begin: int = 0,
+                                block_end: Optional[int] = None, ws=None, stream=None) -> int:
+    """The sweep with Block-GD steps in token form on rotating mini-batches of
+    X_hat's tokens, with per-token output clipping; returns the Adam step counter."""
+    m, n = W0.shape
+    T = X_hat.shape[0]
+    if block_end is None:
+        block_end = -(-n // qcfg.block_size)
+    _need(X_hat, torch.bfloat16, (T, n), "X_hat")
+    _need(U, torch.float32, (n, n), "U")
+    _need(W_work, torch.float32, (m, n), "W_work")
+    _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
+    for t_, nm in ((adam_m, "adam_m"), (adam_v, "adam_v"), (bgd_disp, "bgd_disp")):
+        _need(t_, torch.float32, (m, n), nm)
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    _check(lib().realq_quantize_layer_tokens(
+        _stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar), _ptr(dead), _ptr(X_hat), T, int(T_mb),
+        float(a_loss_clip), ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F),
+        _ptr(F_next), _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes),
+        _ptr(scale), _ptr(zero), _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin),
+        int(block_end), wp, wb))
     return t.value
 
 

@@ -29,12 +29,14 @@ from typing import Dict, List, Optional, Sequence
 
 import torch
 
-from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_graph_begin, realq_graph_end, realq_hessian_accumulate, realq_hessian_accumulate_weighted,
-               realq_hessian_prepare_deferred, realq_hessian_prepare_scaled, realq_prepare_status, realq_hessian_weighted_workspace_size,
-               realq_hessian_workspace_size, realq_prepare_workspace_size, realq_quantize_activations,
-               realq_quantize_grouped_workspace_size, realq_quantize_layer, realq_quantize_layer_grouped,
-               realq_quantize_layer_minibatch, realq_quantize_minibatch_workspace_size, realq_quantize_workspace_size,
-               realq_saliency_clip, realq_scale_moment, realq_workspace_status, workspace)
+from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_graph_begin, realq_graph_end, realq_hessian_accumulate,
+               realq_hessian_accumulate_weighted, realq_hessian_prepare_deferred, realq_hessian_prepare_scaled,
+               realq_hessian_weighted_workspace_size, realq_hessian_workspace_size, realq_prepare_status,
+               realq_prepare_workspace_size, realq_quantize_activations, realq_quantize_grouped_workspace_size,
+               realq_quantize_layer, realq_quantize_layer_grouped, realq_quantize_layer_minibatch,
+               realq_quantize_layer_tokens, realq_quantize_minibatch_workspace_size,
+               realq_quantize_tokens_workspace_size, realq_quantize_workspace_size, realq_saliency_clip,
+               realq_scale_moment, realq_workspace_status, workspace)
 
 
 @dataclass
@@ -71,7 +73,9 @@ class BlockQuantizer:
     minibatch_tokens=T_mb > 0 selects mini-batch Block-GD (Sec. 4.3, 32
     sequences per step in Sec. 5.1): every input's tokens form consecutive
     mini-batches of T_mb tokens, whose second moments the optimizer steps
-    rotate through; the OBS keeps the full H.
+    rotate through; the OBS keeps the full H.  With a_loss_clip (0.95 in the
+    paper's small-model runs) each step's gradient is taken in token form on
+    its mini-batch, with the per-token output clipping.
 
     saliency_groups=N_g > 0 selects the saliency-weighted grouped Hessians
     (Sec. 3.3, Alg. 1 "for all row-groups g"): every module's rows form N_g
@@ -83,7 +87,7 @@ class BlockQuantizer:
     def __init__(self, inputs: Sequence[BlockInput], modules: Sequence[BlockModule], qcfg: QuantCfg, lr: float,
                  steps_per_block: int = 1, sliding_window: bool = False, device="cuda",
                  host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None, saliency_groups: int = 0,
-                 saliency_pct: float = 0.99, minibatch_tokens: int = 0):
+                 saliency_pct: float = 0.99, minibatch_tokens: int = 0, a_loss_clip: Optional[float] = None):
         self.inputs: Dict[str, BlockInput] = {i.name: i for i in inputs}
         self.modules: List[BlockModule] = list(modules)
         for md in self.modules:
@@ -98,6 +102,9 @@ class BlockQuantizer:
         self.sgroups = saliency_groups
         self.spct = saliency_pct
         self.mb_tokens = minibatch_tokens
+        self.a_loss_clip = a_loss_clip
+        if a_loss_clip is not None and not minibatch_tokens:
+            raise ValueError("a_loss_clip takes its gradient on mini-batches: set minibatch_tokens")
         if minibatch_tokens and (saliency_groups or act_quant is not None):
             raise ValueError("mini-batch Block-GD is built for the plain, unperturbed sweep")
         self.mods_of = {name: [md for md in self.modules if md.input == name] for name in self.inputs}
@@ -112,7 +119,7 @@ class BlockQuantizer:
                 dead=torch.empty(n, dtype=torch.uint8, device=dev),
                 pws=workspace(realq_prepare_workspace_size(n), dev).fill_(0xFF),  # status word -1: no failure
                 hws=workspace(realq_hessian_workspace_size(n, spec.T, REALQ_BF16, act_quant is not None), dev))
-            if minibatch_tokens:
+            if minibatch_tokens and a_loss_clip is None:
                 nmb = -(-spec.T // minibatch_tokens)
                 self.state[name].update(Hk=torch.empty(n, n, device=dev), Hmb=torch.empty(nmb, n, n, device=dev),
                                         kws=workspace(realq_hessian_workspace_size(n, minibatch_tokens), dev))
@@ -143,6 +150,10 @@ class BlockQuantizer:
                            wsum=torch.empty(ngs, dtype=torch.float64, device=dev),
                            wws=workspace(realq_hessian_weighted_workspace_size(n, self.inputs[md.input].T), dev),
                            pws=workspace(realq_prepare_workspace_size(n), dev))
+            elif minibatch_tokens and bgd and a_loss_clip is not None:
+                ws_q = workspace(realq_quantize_tokens_workspace_size(m, n, minibatch_tokens, qcfg, bc, sliding_window),
+                                 dev)
+                grp = None
             elif minibatch_tokens and bgd:
                 nmb = -(-self.inputs[md.input].T // minibatch_tokens)
                 ws_q = workspace(realq_quantize_minibatch_workspace_size(m, n, nmb, qcfg, bc, sliding_window), dev)
@@ -213,6 +224,13 @@ class BlockQuantizer:
                 F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"], bgd_disp=o["disp"],
                 ws=o["ws"], stream=stream)
             return
+        if self.mb_tokens and o["bcfg"] is not None and self.a_loss_clip is not None:
+            o["adam_t"] = realq_quantize_layer_tokens(
+                W0, s_in["U"], s_in["Hbar"], X, self.mb_tokens, self.a_loss_clip, self.qcfg, o["W"], o["codes"],
+                o["scale"], o["zero"], dead=s_in["dead"], bcfg=o["bcfg"], F=F,
+                F_next=F_next if self.sliding_window else None, adam_m=o["am"], adam_v=o["av"], bgd_disp=o["disp"],
+                ws=o["ws"], stream=stream)
+            return
         if self.mb_tokens and o["bcfg"] is not None:
             o["adam_t"] = realq_quantize_layer_minibatch(
                 W0, s_in["U"], s_in["Hbar"], s_in["Hmb"], self.qcfg, o["W"], o["codes"], o["scale"], o["zero"],
@@ -250,7 +268,7 @@ class BlockQuantizer:
             return
         if self.act_quant is None:
             realq_hessian_accumulate(X, s_in["H"], ws=s_in["hws"], stream=stream)
-            if self.mb_tokens:
+            if self.mb_tokens and self.a_loss_clip is None:
                 # second moments of the consecutive mini-batches
                 C = self.mb_tokens
                 for k in range(s_in["Hmb"].shape[0]):

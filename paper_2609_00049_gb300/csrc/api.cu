@@ -387,6 +387,14 @@ size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg
     return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, has_Dbar);
 }
 
+// The calibration tokens of token-form mini-batch Block-GD (nullptr: the
+// moment form).
+struct TokArgs {
+    const void *X;       // T x n bf16
+    int64_t T, tmb;      // tokens, tokens per mini-batch
+    float clip;          // per-token output clipping percentile, (0, 1]
+};
+
 static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
                                     int grouped, int rgroups, const float *Ug, const float *Hbar_g,
                                     const uint8_t *dead_g, int nmb, const float *Hbar_mb,
@@ -395,7 +403,7 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
                                     const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
                                     int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
                                     realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
-                                    size_t ws_bytes, const char *who) {
+                                    size_t ws_bytes, const char *who, const TokArgs *tok = nullptr) {
     if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n must be > 0", who);
     if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n too large", who);
     if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "%s: bad dtype", who);
@@ -409,7 +417,7 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
             return fail(REALQ_ERR_INVALID_ARG, "%s: Block-GD needs Hbar, F, bgd_disp and adam_t", who);
         if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
             return fail(REALQ_ERR_INVALID_ARG, "%s: Adam needs adam_m and adam_v", who);
-        if ((grouped || nmb > 0) && !(qcfg->block_size > 0 && tc_gemm_eligible(m, n)))
+        if ((grouped || nmb > 0 || tok) && !(qcfg->block_size > 0 && tc_gemm_eligible(m, n)))
             return fail(REALQ_ERR_UNSUPPORTED,
                         "%s: Block-GD with row groups needs m and n multiples of 4 and at least 32", who);
     }
@@ -421,9 +429,10 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     const int has_db = bgd && Dbar != nullptr;
     if (nmb > 0 && bgd && (Dbar || grouped))
         return fail(REALQ_ERR_UNSUPPORTED, "%s: mini-batch moments with perturbed inputs or row groups", who);
+    const int64_t tmb = (bgd && tok) ? tok->tmb : 0;
     REALQ_TRY(check_ws(ws, ws_bytes,
                        sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_fn, has_db, grouped ? rgroups : 0,
-                                      bgd ? nmb : 0), who));
+                                      bgd ? nmb : 0, tmb), who));
 
     SweepPlan p{};
     p.m = m; p.n = n; p.W0 = W0; p.w_dtype = w_dtype;
@@ -448,6 +457,14 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     p.W = W_work; p.adam_m = adam_m; p.adam_v = adam_v; p.disp = bgd ? bgd_disp : nullptr; p.adam_t = adam_t;
     p.damp = qcfg->damp_frac;
     p.codes = codes; p.scale = scale; p.zero = zero; p.W_deq = W_deq; p.deq_dtype = deq_dtype;
+    if (tmb > 0) {
+        p.Xtok = tok->X; p.Ttok = tok->T; p.tmb = tmb;
+        p.ntok = (int)((tok->T + tmb - 1) / tmb);
+        // nearest-rank threshold: the ceil(pct m)-th smallest |Δ| (pct the
+        // single-precision value; the product is exact in double)
+        const int64_t k = (int64_t)std::ceil((double)tok->clip * (double)m) - 1;
+        p.rank_q = std::min<int64_t>(std::max<int64_t>(k, 0), m - 1);
+    }
     sweep_carve(p, ws, bgd, has_fn, has_db);
     cudaStream_t s = S(stream);
     REALQ_CUDA_TRY(cudaMemsetAsync(p.status, 0, sizeof(int), s));
@@ -519,6 +536,37 @@ realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, 
     return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, n_minibatch, Hbar_mb, U, Hbar,
                          nullptr, dead, qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale,
                          zero, W_deq, deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_minibatch");
+}
+
+size_t realq_quantize_tokens_workspace_size(int64_t m, int64_t n, int64_t T_mb, const realq_quant_cfg_t *qcfg,
+                                            const realq_bgd_cfg_t *bcfg, int has_F_next) {
+    if (m <= 0 || n <= 0 || !qcfg || T_mb <= 0) return 0;
+    const int bgd = bcfg && bcfg->steps_per_block > 0;
+    return sweep_ws_bytes(m, n, qcfg->block_size, bgd, has_F_next, 0, 0, 0, bgd ? T_mb : 0);
+}
+
+realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                           realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                           const uint8_t *dead, const void *X_hat, int64_t T, int64_t T_mb,
+                                           float a_loss_clip, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                           float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
+                                           size_t ws_bytes) {
+    if (!X_hat || T <= 0 || T_mb <= 0)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: X_hat, T > 0 and T_mb > 0 required");
+    if (T_mb % 4 != 0) return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: T_mb must be a multiple of 4");
+    if (T_mb > ((int64_t)1 << 30) || T > ((int64_t)1 << 40))
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: T or T_mb too large");
+    if (reinterpret_cast<uintptr_t>(X_hat) % 16 != 0 || n % 8 != 0)
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: X_hat must be 16-byte aligned with n % 8 == 0");
+    if (!(a_loss_clip > 0.f && a_loss_clip <= 1.f))
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: 0 < a_loss_clip <= 1");
+    const TokArgs tok{X_hat, T, T_mb, a_loss_clip};
+    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, Hbar, nullptr, dead,
+                         qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq,
+                         deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_tokens", &tok);
 }
 
 // ---------------------------------------------------------------- BGD -----

@@ -163,6 +163,16 @@ struct SweepPlan {
     std::vector<TcMaps> mapsMB;
     int f_split_alpha_valid;
     float f_split_alpha;
+    // token-form mini-batch Block-GD with per-token output clipping: the
+    // calibration tokens X̂ (T_tok x n bf16) form ntok mini-batches of tmb
+    // tokens; rank_q = the 0-based rank of the clip threshold among m
+    // channels (m - 1: no channel scaled)
+    const void *Xtok = nullptr;
+    int64_t Ttok = 0, tmb = 0, rank_q = 0;
+    int ntok = 0;
+    float *Xf = nullptr, *XfT = nullptr, *Zero = nullptr, *Dk = nullptr, *Yh = nullptr, *Yl = nullptr,
+          *Zk = nullptr, *Gc = nullptr;
+    std::vector<TcMaps> mapsT1, mapsT2, mapsT3;
     // The optimizer step's G product is split: the next block's columns on
     // the sweep's stream (the next OBS block needs only those), the other
     // free columns on a side stream, joined before anything else reads or
@@ -174,7 +184,11 @@ struct SweepPlan {
 realq_status_t sweep_side_stream(cudaStream_t s, SweepPlan &p);
 realq_status_t sweep_join_wide(cudaStream_t s, SweepPlan &p);
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0,
-                      int nmb = 0);
+                      int nmb = 0, int64_t tmb = 0);
+realq_status_t tok_xconv(cudaStream_t s, int64_t T, int64_t n, const void *X, float *Xf, float *XfT, int64_t ldT);
+realq_status_t tok_clip(cudaStream_t s, int64_t T, int64_t m, float *D, int64_t k, float *Yh, float *Yl);
+realq_status_t tok_gt(cudaStream_t s, int64_t T, int64_t m, const float *kap, const float *Z, float inv_T, float *gTh,
+                      float *gTl, int64_t ldT);
 void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dbar);
 realq_status_t sweep_init(cudaStream_t s, SweepPlan &p);
 realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b);

@@ -378,7 +378,7 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 // fp32 SIMT path needs P, G (and F_eff).  block = 0: Block-GD only (literal
 // gradient form, SIMT).
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups,
-                      int nmb) {
+                      int nmb, int64_t tmb) {
     const size_t mn = align_up((size_t)m * n * sizeof(float));
     const size_t nn = align_up((size_t)n * n * sizeof(float));
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
@@ -388,6 +388,14 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
             b += 5 * mn + 2 * nn + 2 * align_up((size_t)m * m * sizeof(float));
             if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
             if (nmb > 0) b += (rgroups > 0 ? 0 : 2 * mn) + 2 * (size_t)nmb * nn;
+            if (tmb > 0) {
+                // ΔW planes, the mini-batch in fp32 both ways and a zero plane,
+                // Δ (then kappa), the clipped residual's planes (then the
+                // gradient factor's), Z and the gradient
+                const size_t tn = align_up((size_t)tmb * n * sizeof(float));
+                const size_t tm = align_up((size_t)tmb * m * sizeof(float));
+                b += 3 * mn + 3 * tn + 4 * tm;
+            }
         } else {
             b += 2 * mn;
             if (has_fnext) b += align_up((size_t)m * m * sizeof(float));
@@ -428,6 +436,18 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
                     p.DWh = cv.take<float>(mn);
                     p.DWl = cv.take<float>(mn);
                 }
+            }
+            if (p.tmb > 0) {
+                p.DWh = cv.take<float>(mn);
+                p.DWl = cv.take<float>(mn);
+                p.Gc = cv.take<float>(mn);
+                p.Xf = cv.take<float>((size_t)p.tmb * p.n);
+                p.XfT = cv.take<float>((size_t)p.tmb * p.n);
+                p.Zero = cv.take<float>((size_t)p.tmb * p.n);
+                p.Dk = cv.take<float>((size_t)p.tmb * p.m);
+                p.Yh = cv.take<float>((size_t)p.tmb * p.m);
+                p.Yl = cv.take<float>((size_t)p.tmb * p.m);
+                p.Zk = cv.take<float>((size_t)p.tmb * p.m);
             }
             if (p.grouped) {
                 p.DWh = cv.take<float>(mn);
@@ -710,6 +730,54 @@ static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, in
     return REALQ_OK;
 }
 
+// One optimizer step on mini-batch kmb in token form, with the per-token
+// output clipping (rank_q = m - 1 scales nothing):
+//   Δ = X̂_k (Ŵ - W0)ᵀ, kappa from the per-token threshold, Y = kappa ⊙ Δ,
+//   Z = Y F_eff, g = kappa ⊙ Z / T_k, G = gᵀ X̂_k[:, c0:], then Adam.
+// The token axis of the last product is taken in fixed-order chunks of 8192
+// (each accumulated into G in turn), so the accumulation is deterministic
+// and each chunk's tensor-core sum stays short.
+static realq_status_t bgd_one_tokens(cudaStream_t s, SweepPlan &p, int64_t c0, int kmb) {
+    const int64_t r = p.n - c0;
+    const int64_t Tk = std::min<int64_t>(p.tmb, p.Ttok - (int64_t)kmb * p.tmb);
+    const void *Xk = static_cast<const __nv_bfloat16 *>(p.Xtok) + (size_t)kmb * p.tmb * p.n;
+    REALQ_TRY(tok_xconv(s, Tk, p.n, Xk, p.Xf, p.XfT, p.tmb));
+    if (p.w_dtype == REALQ_BF16)
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const __nv_bfloat16 *>(p.W0), p.DWh, p.DWl));
+    else
+        REALQ_TRY(tc_split_diff(s, p.m * p.n, p.W, static_cast<const float *>(p.W0), p.DWh, p.DWl));
+    TcEpi e1{};
+    e1.mode = TC_STORE;
+    e1.C = p.Dk; e1.ldc = p.m;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT1[kmb], Tk, p.m, p.n, 0, 0, e1, p.status, "tok_residual_gemm"));
+    REALQ_TRY(tok_clip(s, Tk, p.m, p.Dk, p.rank_q, p.Yh, p.Yl));
+    TcEpi e2{};
+    e2.mode = TC_STORE;
+    e2.C = p.Zk; e2.ldc = p.m;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT2[kmb], Tk, p.m, p.m, 0, 0, e2, p.status, "tok_fisher_gemm"));
+    REALQ_TRY(tok_gt(s, Tk, p.m, p.Dk, p.Zk, (float)(1.0 / (double)Tk), p.Yh, p.Yl, p.tmb));
+    REALQ_CUDA_TRY(cudaMemsetAsync(p.Gc, 0, (size_t)p.m * r * sizeof(float), s));
+    TcEpi e3{};
+    e3.mode = TC_ACCUM;
+    e3.M = p.Gc; e3.ldw = r; e3.col0 = 0;
+    constexpr int64_t kChunk = 8192;
+    for (int64_t k0 = 0; k0 < Tk; k0 += kChunk)
+        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT3[kmb], p.m, r, std::min<int64_t>(kChunk, Tk - k0), (int)k0, (int)c0, e3,
+                                 p.status, "tok_grad_gemm"));
+    const int64_t t = ++(*p.adam_t);
+    const double bc1 = 1.0 - std::pow((double)p.beta1, (double)t);
+    const double bc2 = 1.0 - std::pow((double)p.beta2, (double)t);
+    {
+        Launch L("bgd_adam", s);
+        adam_kernel<<<blocks_for(p.m * r), 256, 0, s>>>(p.m, r, p.n, c0, p.Gc, p.W, p.adam_m, p.adam_v, p.disp, p.lr,
+                                                         p.beta1, p.beta2, p.eps, (float)bc1, (float)bc2,
+                                                         p.optimizer == REALQ_OPT_SGD);
+    }
+    REALQ_TRY(check_launch("bgd_adam"));
+    p.step_c = c0;
+    return REALQ_OK;
+}
+
 realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float alpha) {
     if (col_start >= p.n) return REALQ_OK;
     if (p.Dbar) REALQ_TRY(compute_r0(s, p));
@@ -790,7 +858,9 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
         }
         for (int k = 0; k < p.bgd_steps; ++k) {
             const bool last = k == p.bgd_steps - 1;
-            if (p.nmb > 0)
+            if (p.tmb > 0)
+                REALQ_TRY(bgd_one_tokens(s, p, be, (int)(((b_global - 1) * p.bgd_steps + k) % p.ntok)));
+            else if (p.nmb > 0)
                 REALQ_TRY(bgd_one_tc_mb(s, p, be, (int)(((b_global - 1) * p.bgd_steps + k) % p.nmb), last));
             else
                 REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be, last) : bgd_one_tc(s, p, be, last));
@@ -849,6 +919,21 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
                 REALQ_TRY(tc_split_diff(s, (int64_t)nn, p.Hbar, p.Hbar_mb + k * nn, p.MBh + k * nn, p.MBl + k * nn));
                 REALQ_TRY(tc_make_maps(&p.mapsMB[k], p.DWh, p.DWl, p.m, p.n, p.n, p.MBh + k * nn, p.MBl + k * nn,
                                        p.n, p.n, p.n));
+            }
+        }
+        if (p.tmb > 0) {
+            // per mini-batch (the last may be short, and the products must
+            // see zeros past its tokens): Δ = X̂_k ΔWᵀ, Z = Y F_eff and
+            // G = gᵀ X̂_k with the token axis as K
+            REALQ_CUDA_TRY(cudaMemsetAsync(p.Zero, 0, (size_t)p.tmb * p.n * sizeof(float), s));
+            p.mapsT1.assign(p.ntok, TcMaps{});
+            p.mapsT2.assign(p.ntok, TcMaps{});
+            p.mapsT3.assign(p.ntok, TcMaps{});
+            for (int k = 0; k < p.ntok; ++k) {
+                const int64_t Tk = std::min<int64_t>(p.tmb, p.Ttok - (int64_t)k * p.tmb);
+                REALQ_TRY(tc_make_maps(&p.mapsT1[k], p.Xf, p.Zero, Tk, p.n, p.n, p.DWh, p.DWl, p.m, p.n, p.n));
+                REALQ_TRY(tc_make_maps(&p.mapsT2[k], p.Yh, p.Yl, Tk, p.m, p.m, p.Fh, p.Fl, p.m, p.m, p.m));
+                REALQ_TRY(tc_make_maps(&p.mapsT3[k], p.Yh, p.Yl, p.m, Tk, p.tmb, p.XfT, p.Zero, p.n, Tk, p.tmb));
             }
         }
         if (fresh) {

@@ -828,3 +828,45 @@ def test_block_graph_replay_matches_eager(variant):
             if variant == "host":
                 for k in keys[:3]:
                     assert torch.equal(out_h[nm][k], eager[nm][k].cpu()), (variant, nm, k)
+
+
+@pytest.mark.parametrize("clip,start,steps", [(0.95, 1, 1), (0.95, 2, 2), (0.9, 3, 1), (1.0, 1, 1)])
+def test_token_block_gd_with_output_clipping(clip, start, steps):
+    # token-form mini-batch Block-GD with per-token output clipping against
+    # the oracle's token-form sweep; 8000 tokens in mini-batches of 2048 (the
+    # last one 1856 tokens); clip = 1 scales nothing (the moment form)
+    case = synth.layer_case(62, 128, 384, 8000, bf16=True, outliers=3)
+    Tm = 2048
+    parts = [case.Xhat[k * Tm:(k + 1) * Tm] for k in range(-(-8000 // Tm))]
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1,
+           "minibatch_tokens": parts, "a_loss_clip": clip}
+    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd, F=case.F)
+    qkw = dict(group_size=128, block_size=128)
+    X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
+    H, _, _ = layer.accumulate([X], 384)
+    prep = layer.prepare(H, T)
+    q = rq.quant_cfg(**qkw)
+    b = rq.bgd_cfg(2e-4, steps_per_block=steps, b_global_start=start)
+    m, n = 128, 384
+    W = torch.empty(m, n, device="cuda")
+    codes = torch.empty(m, n // 2, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(m, 3, device="cuda")
+    zero = torch.empty(m, 3, dtype=torch.uint8, device="cuda")
+    st = {k: torch.empty(m, n, device="cuda") for k in ("adam_m", "adam_v", "bgd_disp")}
+    ws = rq.workspace(rq.realq_quantize_tokens_workspace_size(m, n, Tm, q, b))
+    t = rq.realq_quantize_layer_tokens(dev(case.W0), prep.U, prep.Hbar, X, Tm, clip, q, W, codes, scale, zero,
+                                       dead=prep.dead, bcfg=b, F=dev(case.F), ws=ws, **st)
+    rq.realq_workspace_status(ws)
+    assert t == orc["adam_t"] == 2 * steps
+    c = unpack(codes.cpu().numpy(), n)
+    rep = compare_codes(c, orc, 128, 128, True)
+    frac, med, s_unexpl = scale_agreement(scale.cpu().numpy(), orc["scale"], 128,
+                                          explained=compare_codes.last_explained,
+                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, steps))
+    dev_deq = np.abs(W.cpu().numpy() - orc["deq"]).max()
+    print(f"\ntoken form clip={clip} start={start} steps={steps}: {rep} scale_within_1e-5={frac:.5f} "
+          f"max|deq - oracle|={dev_deq:.2e}")
+    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
+    assert s_unexpl == 0
+
