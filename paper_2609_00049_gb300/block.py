@@ -184,7 +184,10 @@ class BlockQuantizer:
         # already saturates the host link, and in a captured step the inputs
         # arrive in chain order (the longest chain's activations first), so
         # that chain's preparation and sweeps overlap the other copies
-        self.chain_order = sorted(self.inputs, key=lambda name: self.priority[name])
+        # (equal widths: the input feeding more weights first, so the input
+        # whose copy ends the stream has the shortest chain after it)
+        load = {name: sum(md.m * md.n for md in self.modules if md.input == name) for name in self.inputs}
+        self.chain_order = sorted(self.inputs, key=lambda name: (self.priority[name], -load[name]))
         copy_stream = torch.cuda.Stream(device=dev)
         self.copy_streams = {name: copy_stream for name in self.inputs}
 

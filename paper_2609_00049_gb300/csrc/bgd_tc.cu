@@ -230,7 +230,7 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
 
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
-                       int a_row0, const TcEpi e, int *err) {
+                       int a_row0, const TcEpi e, int *err, int kchunk) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -241,7 +241,10 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TB;
-    const int nk = (int)((K + KS - 1) / KS);
+    // K split over blockIdx.z: this CTA takes K range [kz0, kz0 + Kz)
+    const int64_t kz0 = kchunk > 0 ? (int64_t)blockIdx.z * kchunk : 0;
+    const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+    const int nk = (int)((Kz + KS - 1) / KS);
 
     if (threadIdx.x == 0) {
         for (int s = 0; s < STAGES; ++s) {
@@ -274,7 +277,7 @@ __global__ void __launch_bounds__(THREADS, 1)
             }
             const uint32_t fb = tc::smem_u32(&full[s]);
             tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
-            const int x = k_off + it * KS;
+            const int x = k_off + (int)kz0 + it * KS;
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
             tc::tma_load_2d(base, &maps.a_hi, fb, x, a_row0 + (int)i0);
             tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, a_row0 + (int)i0);
@@ -366,7 +369,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int q = 0; q < 4; ++q) {
                         if (gj + q >= N) break;
                         float &t = T[rr * TP + cc + q];
-                        if (e.mode == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
+                        if (e.mode == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
+                        else if (e.mode == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
                         else if (e.mode == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
                         else epi_apply(e, gi, gj + q, t);
                     }
@@ -395,6 +399,28 @@ __global__ void __launch_bounds__(THREADS, 1)
     tc::fence_before_sync();
     __syncthreads();
     if (warp == 0) tc::tmem_dealloc(tmem, TB);
+}
+
+// g = sum over the K splits (z = 0, 1, ... in order), then the TC_ADAM
+// epilogue on element (i, j) of the m x N block at column e.col0
+__global__ void gsum_adam_kernel(int64_t m, int64_t N, int nz, const float *part, const TcEpi e) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * N) return;
+    const int64_t i = idx / N, j = idx % N;
+    float g = 0.f;
+    for (int z = 0; z < nz; ++z) g += part[(int64_t)z * m * N + idx];
+    const int64_t w = i * e.ldw + e.col0 + j;
+    float mv = e.sgd ? 0.f : e.mA[w], vv = e.sgd ? 0.f : e.vA[w];
+    const float st = adam_step(e, g, mv, vv);
+    if (!e.sgd) {
+        e.mA[w] = mv;
+        e.vA[w] = vv;
+    }
+    e.Wm[w] -= st;
+    e.D[w] -= st;
+    const float sh = tc::tf32_hi(-st);
+    e.Sh[w] = sh;
+    e.Sl[w] = -st - sh;
 }
 
 // hi / lo planes of x (or of alpha x + (1 - alpha) y when y is given)
@@ -447,6 +473,15 @@ realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const flo
     return check_launch("tf32_split");
 }
 
+realq_status_t tc_gsum_adam(cudaStream_t s, int64_t m, int64_t N, int nz, const float *part, const TcEpi &e) {
+    if (m <= 0 || N <= 0) return REALQ_OK;
+    {
+        Launch L("bgd_g_gsum_adam", s);
+        gsum_adam_kernel<<<(unsigned)ceil_div(m * N, 256), 256, 0, s>>>(m, N, nz, part, e);
+    }
+    return check_launch("bgd_g_gsum_adam");
+}
+
 realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb) {
@@ -464,9 +499,11 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
 }
 
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0) {
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk) {
     if (M <= 0 || N <= 0) return REALQ_OK;
     if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
+    if (kchunk < 0 || (kchunk % KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name, KS);
     static bool configured = false;
     if (!configured) {
         REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM));
@@ -475,8 +512,9 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
     {
         Launch L(name, s);
-        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB)), THREADS, SMEM, s>>>(
-            m, M, N, K, k_off, b_row0, a_row0, e, err);
+        const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
+        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB), nz), THREADS, SMEM, s>>>(
+            m, M, N, K, k_off, b_row0, a_row0, e, err, kchunk);
     }
     return check_launch(name);
 }

@@ -61,6 +61,7 @@ struct TcEpi {
     float *M;                                                // running A H̄ (acc += M, M = acc)
     float *Wm; float *mA; float *vA; float *D; float *Sh; float *Sl;  // TC_ADAM (ldw, col0 shared)
     float lr, b1, b2, eps, bc1, bc2; int sgd;
+    int64_t czs;                                             // TC_STORE with a K split: C of split z at C + z czs
 };
 struct TcMaps {
     alignas(64) unsigned char storage[4 * 128];
@@ -72,7 +73,10 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb);
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0);
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0, int kchunk = 0);
+// g = sum_z part[z] (fixed order) and one optimizer step on the m x N block at
+// column e.col0 (the TC_ADAM epilogue as a separate pass)
+realq_status_t tc_gsum_adam(cudaStream_t s, int64_t m, int64_t N, int nz, const float *part, const TcEpi &e);
 template <typename TY>
 realq_status_t tc_split_diff(cudaStream_t s, int64_t count, const float *x, const TY *y, float *hi, float *lo);
 
@@ -177,6 +181,7 @@ struct SweepPlan {
     // the sweep's stream (the next OBS block needs only those), the other
     // free columns on a side stream, joined before anything else reads or
     // writes them.  wide == nullptr: everything on the sweep's stream.
+    float *Gpart = nullptr;                  // K-split partials of the next block's G (8 x m x B)
     cudaStream_t wide = nullptr;
     cudaEvent_t wide_fork = nullptr, wide_done = nullptr;
     int wide_pending = 0;

@@ -92,6 +92,9 @@ struct QArgs {
 // of the group's sub-blocks gathered through shared memory; G = 0: they were
 // computed before the block.
 constexpr int QB_ROWS = 32;
+}  // namespace
+constexpr int kGSplit = 8;   // K slices of the next block's G product
+namespace {
 
 template <int B, int G>
 __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
@@ -191,6 +194,14 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
         }
         if (warp == s) {
             uint32_t packed[4] = {0u, 0u, 0u, 0u};
+            // rint(w / sc) through the reciprocal: x = w * rn(1/sc) is within
+            // 3 * 2^-24 |w / sc| of the quotient and of its IEEE rounding, so
+            // where x is farther than 4 * 2^-24 |x| from every half-integer
+            // both round to the same integer; nearer (and for non-finite
+            // values) the IEEE division decides, so the code is the one of
+            // rint(w / sc) in every case and the chain from one column's
+            // error to the next column's code avoids the division
+            const float rcp = __frcp_rn(sc);
 #pragma unroll
             for (int jj = 0; jj < 32; ++jj) {
                 const int j = c0 + jj;
@@ -199,7 +210,11 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
                 if (j < kb) {
                     const float w = r[jj];
                     bad |= !isfinite(w);
-                    float q = rintf(w / sc) + zr;
+                    const float x = __fmul_rn(w, rcp);
+                    float qx = rintf(x);
+                    const float gap = 0.5f - fabsf(x - qx);
+                    if (!(gap > 2.4e-7f * fabsf(x) + 1e-30f)) qx = rintf(w / sc);
+                    float q = qx + zr;
                     q = fminf(fmaxf(q, 0.f), maxq);
                     const float dq = sc * (q - zr);
                     err = (w - dq) * invd[j];
@@ -386,6 +401,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
     if (has_bgd) {
         if (block > 0 && tc_gemm_eligible(m, n)) {
             b += 5 * mn + 2 * nn + 2 * align_up((size_t)m * m * sizeof(float));
+            b += align_up((size_t)kGSplit * m * block * sizeof(float));
             if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
             if (nmb > 0) b += (rgroups > 0 ? 0 : 2 * mn) + 2 * (size_t)nmb * nn;
             if (tmb > 0) {
@@ -429,6 +445,7 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
             p.Hl = cv.take<float>((size_t)p.n * p.n);
             p.Fh = cv.take<float>((size_t)p.m * p.m);
             p.Fl = cv.take<float>((size_t)p.m * p.m);
+            p.Gpart = cv.take<float>((size_t)kGSplit * p.m * p.block);
             if (p.nmb > 0) {
                 p.MBh = cv.take<float>((size_t)p.nmb * p.n * p.n);
                 p.MBl = cv.take<float>((size_t)p.nmb * p.n * p.n);
@@ -573,9 +590,10 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
 // M = A H̄ up to date for them: the last step moved A only in its own free
 // columns [step_c, n), so M[:, c0:] += step[:, step_c:] H̄[step_c:, c0:]
 // (K = n - step_c instead of n), then the epilogue forms P from M.
-// G = F_eff P on the free columns c0.. and one Adam step on them (fused).
-// For the last step of a block with a side stream, the next block's columns
-// (c0 .. c0 + B) run on s and the rest on the side stream: the next OBS block
+// G = F_eff P on the free columns c0.. and one Adam step on them.  On the
+// last step of a block the next block's columns (c0 .. c0 + B) run first, K
+// split into slices whose fixed-order sum takes the step, and the rest (fused
+// Adam epilogue) on the side stream when there is one: the next OBS block
 // waits only for its own columns, and sweep_join_wide orders the rest before
 // the next trailing update (the next reader or writer of those columns).
 static realq_status_t g_adam(cudaStream_t s, SweepPlan &p, int64_t c0, bool last) {
@@ -590,15 +608,32 @@ static realq_status_t g_adam(cudaStream_t s, SweepPlan &p, int64_t c0, bool last
     g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
     g.sgd = p.optimizer == REALQ_OPT_SGD;
     const int64_t nb = std::min<int64_t>(p.block, r);
-    if (!last || !p.wide || r <= nb) return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
-    REALQ_CUDA_TRY(cudaEventRecord(p.wide_fork, s));
-    REALQ_CUDA_TRY(cudaStreamWaitEvent(p.wide, p.wide_fork, 0));
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, nb, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam"));
+    if (!last) return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
+    // (the split below is the same arithmetic with or without the side
+    // stream, so a sweep resumed at any block gives the same bits)
+    cudaStream_t ws = (p.wide && r > nb) ? p.wide : s;
+    if (ws != s) {
+        REALQ_CUDA_TRY(cudaEventRecord(p.wide_fork, s));
+        REALQ_CUDA_TRY(cudaStreamWaitEvent(p.wide, p.wide_fork, 0));
+    }
+    // the next block's columns: few tiles with K = m, so K is split into
+    // kGSplit slices (more CTAs, shorter chains), summed in a fixed order by
+    // the pass that takes the optimizer step
+    const int kchunk = (int)((ceil_div(p.m, kGSplit) + 31) / 32 * 32);
+    const int nz = ceil_div(p.m, kchunk);
+    TcEpi st{};
+    st.mode = TC_STORE;
+    st.C = p.Gpart; st.ldc = nb; st.czs = p.m * nb;
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, nb, p.m, 0, 0, st, p.status, "bgd_g_gemm_adam", 0, kchunk));
+    REALQ_TRY(tc_gsum_adam(s, p.m, nb, nz, p.Gpart, g));
+    if (r <= nb) return REALQ_OK;
     TcEpi gw = g;
     gw.col0 = c0 + nb;
-    REALQ_TRY(tc_gemm_tf32x3(p.wide, p.mapsG, p.m, r - nb, p.m, 0, (int)nb, gw, p.status, "bgd_g_gemm_adam"));
-    REALQ_CUDA_TRY(cudaEventRecord(p.wide_done, p.wide));
-    p.wide_pending = 1;
+    REALQ_TRY(tc_gemm_tf32x3(ws, p.mapsG, p.m, r - nb, p.m, 0, (int)nb, gw, p.status, "bgd_g_gemm_adam"));
+    if (ws != s) {
+        REALQ_CUDA_TRY(cudaEventRecord(p.wide_done, p.wide));
+        p.wide_pending = 1;
+    }
     return REALQ_OK;
 }
 
