@@ -230,7 +230,7 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
 
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
-                       int a_row0, const TcEpi e, int *err, int kchunk) {
+                       int a_row0, const TcEpi e, int *err, int kchunk, int exact) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -276,13 +276,15 @@ __global__ void __launch_bounds__(THREADS, 1)
                 break;
             }
             const uint32_t fb = tc::smem_u32(&full[s]);
-            tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+            // an operand exact in tf32 (exact & 1: A, exact & 2: B) has no
+            // low plane to load or multiply
+            tc::mbar_arrive_expect_tx(fb, STAGE_BYTES - ((exact & 1) ? PLANE : 0) - ((exact & 2) ? PLANE : 0));
             const int x = k_off + (int)kz0 + it * KS;
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
             tc::tma_load_2d(base, &maps.a_hi, fb, x, a_row0 + (int)i0);
-            tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, a_row0 + (int)i0);
+            if (!(exact & 1)) tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, a_row0 + (int)i0);
             tc::tma_load_2d(base + 2 * PLANE, &maps.b_hi, fb, x, b_row0 + (int)j0);
-            tc::tma_load_2d(base + 3 * PLANE, &maps.b_lo, fb, x, b_row0 + (int)j0);
+            if (!(exact & 2)) tc::tma_load_2d(base + 3 * PLANE, &maps.b_lo, fb, x, b_row0 + (int)j0);
         }
         if (*abort_flag) {
             int never = 0;
@@ -307,8 +309,8 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const uint64_t bh = tc::smem_desc(base + 2 * PLANE + k * 32, 16, 1024, tc::SW_128B);
                 const uint64_t bl = tc::smem_desc(base + 3 * PLANE + k * 32, 16, 1024, tc::SW_128B);
                 tc::mma_tf32_ss(tmem, ah, bh, IDESC, (it > 0 || k > 0) ? 1u : 0u);
-                tc::mma_tf32_ss(tmem, ah, bl, IDESC, 1u);
-                tc::mma_tf32_ss(tmem, al, bh, IDESC, 1u);
+                if (!(exact & 2)) tc::mma_tf32_ss(tmem, ah, bl, IDESC, 1u);
+                if (!(exact & 1)) tc::mma_tf32_ss(tmem, al, bh, IDESC, 1u);
             }
             tc::mma_commit(tc::smem_u32(&empty[s]));
         }
@@ -499,7 +501,8 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
 }
 
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk) {
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk,
+                              int exact) {
     if (M <= 0 || N <= 0) return REALQ_OK;
     if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
     if (kchunk < 0 || (kchunk % KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
@@ -514,7 +517,7 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
         Launch L(name, s);
         const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
         gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB), nz), THREADS, SMEM, s>>>(
-            m, M, N, K, k_off, b_row0, a_row0, e, err, kchunk);
+            m, M, N, K, k_off, b_row0, a_row0, e, err, kchunk, exact);
     }
     return check_launch(name);
 }

@@ -73,7 +73,8 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb);
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
-                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0, int kchunk = 0);
+                              int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0, int kchunk = 0,
+                              int exact = 0);   // exact & 1: A exact in tf32 (no low plane), & 2: B
 // g = sum_z part[z] (fixed order) and one optimizer step on the m x N block at
 // column e.col0 (the TC_ADAM epilogue as a separate pass)
 realq_status_t tc_gsum_adam(cudaStream_t s, int64_t m, int64_t N, int nz, const float *part, const TcEpi &e);
@@ -174,7 +175,7 @@ struct SweepPlan {
     const void *Xtok = nullptr;
     int64_t Ttok = 0, tmb = 0, rank_q = 0;
     int ntok = 0;
-    float *Xf = nullptr, *XfT = nullptr, *Zero = nullptr, *Dk = nullptr, *Yh = nullptr, *Yl = nullptr,
+    float *Xf = nullptr, *XfT = nullptr, *Dk = nullptr, *Yh = nullptr, *Yl = nullptr,
           *Zk = nullptr, *Gc = nullptr;
     std::vector<TcMaps> mapsT1, mapsT2, mapsT3;
     // The optimizer step's G product is split: the next block's columns on

@@ -43,14 +43,26 @@ __global__ void __launch_bounds__(256) xconv_kernel(int64_t T, int64_t n, const 
 }
 
 // One warp per token: q = the (k+1)-th smallest |D[t, :]| (k 0-based), then
-// kappa into D and the tf32 planes of kappa * D into Yh / Yl.
-__global__ void __launch_bounds__(256) clip_kernel(int64_t T, int64_t m, float *D, int64_t k, float *Yh,
-                                                   float *Yl) {
-    __shared__ unsigned int hist[8][256];
+// kappa into D and the tf32 planes of kappa * D into Yh / Yl.  With STAGE the
+// token's row is read from global memory once and kept in shared memory for
+// the four select passes and the final one (CLIP_WARPS rows per CTA).
+constexpr int CLIP_WARPS = 4;
+
+template <bool STAGE>
+__global__ void __launch_bounds__(CLIP_WARPS * 32) clip_kernel(int64_t T, int64_t m, float *D, int64_t k, float *Yh,
+                                                               float *Yl) {
+    __shared__ unsigned int hist[CLIP_WARPS][256];
+    extern __shared__ float rowbuf[];
     const int w = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t t = (int64_t)blockIdx.x * 8 + w;
+    const int64_t t = (int64_t)blockIdx.x * CLIP_WARPS + w;
     if (t >= T) return;
-    float *row = D + t * m;
+    float *grow = D + t * m;
+    float *row = grow;
+    if (STAGE) {
+        row = rowbuf + (int64_t)w * m;
+        for (int64_t i = lane; i < m; i += 32) row[i] = grow[i];
+        __syncwarp();
+    }
     unsigned int *h = hist[w];
     uint32_t prefix = 0u, mask = 0u;
     int64_t kr = k;
@@ -103,7 +115,7 @@ __global__ void __launch_bounds__(256) clip_kernel(int64_t T, int64_t m, float *
         const float hi = tc::tf32_hi(y);
         Yh[t * m + i] = hi;
         Yl[t * m + i] = y - hi;
-        row[i] = kap;
+        grow[i] = kap;
     }
 }
 
@@ -143,9 +155,20 @@ realq_status_t tok_xconv(cudaStream_t s, int64_t T, int64_t n, const void *X, fl
 
 realq_status_t tok_clip(cudaStream_t s, int64_t T, int64_t m, float *D, int64_t k, float *Yh, float *Yl) {
     if (T <= 0) return REALQ_OK;
+    const size_t stage = (size_t)CLIP_WARPS * m * sizeof(float);
+    constexpr size_t kMaxStage = 160 * 1024;
+    static bool configured = false;
+    if (!configured) {
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(clip_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                            (int)kMaxStage));
+        configured = true;
+    }
     {
         Launch L("tok_clip", s);
-        clip_kernel<<<(unsigned)ceil_div(T, 8), 256, 0, s>>>(T, m, D, k, Yh, Yl);
+        if (stage <= kMaxStage)
+            clip_kernel<true><<<(unsigned)ceil_div(T, CLIP_WARPS), CLIP_WARPS * 32, stage, s>>>(T, m, D, k, Yh, Yl);
+        else
+            clip_kernel<false><<<(unsigned)ceil_div(T, CLIP_WARPS), CLIP_WARPS * 32, 0, s>>>(T, m, D, k, Yh, Yl);
     }
     return check_launch("tok_clip");
 }

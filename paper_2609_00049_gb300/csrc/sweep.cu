@@ -405,12 +405,12 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
             if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
             if (nmb > 0) b += (rgroups > 0 ? 0 : 2 * mn) + 2 * (size_t)nmb * nn;
             if (tmb > 0) {
-                // ΔW planes, the mini-batch in fp32 both ways and a zero plane,
-                // Δ (then kappa), the clipped residual's planes (then the
-                // gradient factor's), Z and the gradient
+                // ΔW planes, the mini-batch in fp32 both ways (exact in tf32:
+                // no low plane), Δ (then kappa), the clipped residual's planes
+                // (then the gradient factor's), Z and the gradient
                 const size_t tn = align_up((size_t)tmb * n * sizeof(float));
                 const size_t tm = align_up((size_t)tmb * m * sizeof(float));
-                b += 3 * mn + 3 * tn + 4 * tm;
+                b += 3 * mn + 2 * tn + 4 * tm;
             }
         } else {
             b += 2 * mn;
@@ -460,7 +460,6 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
                 p.Gc = cv.take<float>(mn);
                 p.Xf = cv.take<float>((size_t)p.tmb * p.n);
                 p.XfT = cv.take<float>((size_t)p.tmb * p.n);
-                p.Zero = cv.take<float>((size_t)p.tmb * p.n);
                 p.Dk = cv.take<float>((size_t)p.tmb * p.m);
                 p.Yh = cv.take<float>((size_t)p.tmb * p.m);
                 p.Yl = cv.take<float>((size_t)p.tmb * p.m);
@@ -784,7 +783,7 @@ static realq_status_t bgd_one_tokens(cudaStream_t s, SweepPlan &p, int64_t c0, i
     TcEpi e1{};
     e1.mode = TC_STORE;
     e1.C = p.Dk; e1.ldc = p.m;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT1[kmb], Tk, p.m, p.n, 0, 0, e1, p.status, "tok_residual_gemm"));
+    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT1[kmb], Tk, p.m, p.n, 0, 0, e1, p.status, "tok_residual_gemm", 0, 0, 1));
     REALQ_TRY(tok_clip(s, Tk, p.m, p.Dk, p.rank_q, p.Yh, p.Yl));
     TcEpi e2{};
     e2.mode = TC_STORE;
@@ -798,7 +797,7 @@ static realq_status_t bgd_one_tokens(cudaStream_t s, SweepPlan &p, int64_t c0, i
     constexpr int64_t kChunk = 8192;
     for (int64_t k0 = 0; k0 < Tk; k0 += kChunk)
         REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT3[kmb], p.m, r, std::min<int64_t>(kChunk, Tk - k0), (int)k0, (int)c0, e3,
-                                 p.status, "tok_grad_gemm"));
+                                 p.status, "tok_grad_gemm", 0, 0, 2));
     const int64_t t = ++(*p.adam_t);
     const double bc1 = 1.0 - std::pow((double)p.beta1, (double)t);
     const double bc2 = 1.0 - std::pow((double)p.beta2, (double)t);
@@ -959,16 +958,16 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
         if (p.tmb > 0) {
             // per mini-batch (the last may be short, and the products must
             // see zeros past its tokens): Δ = X̂_k ΔWᵀ, Z = Y F_eff and
-            // G = gᵀ X̂_k with the token axis as K
-            REALQ_CUDA_TRY(cudaMemsetAsync(p.Zero, 0, (size_t)p.tmb * p.n * sizeof(float), s));
+            // G = gᵀ X̂_k with the token axis as K (X̂_k is exact in tf32: its
+            // low plane is never loaded, the map's second plane is a stand-in)
             p.mapsT1.assign(p.ntok, TcMaps{});
             p.mapsT2.assign(p.ntok, TcMaps{});
             p.mapsT3.assign(p.ntok, TcMaps{});
             for (int k = 0; k < p.ntok; ++k) {
                 const int64_t Tk = std::min<int64_t>(p.tmb, p.Ttok - (int64_t)k * p.tmb);
-                REALQ_TRY(tc_make_maps(&p.mapsT1[k], p.Xf, p.Zero, Tk, p.n, p.n, p.DWh, p.DWl, p.m, p.n, p.n));
+                REALQ_TRY(tc_make_maps(&p.mapsT1[k], p.Xf, p.Xf, Tk, p.n, p.n, p.DWh, p.DWl, p.m, p.n, p.n));
                 REALQ_TRY(tc_make_maps(&p.mapsT2[k], p.Yh, p.Yl, Tk, p.m, p.m, p.Fh, p.Fl, p.m, p.m, p.m));
-                REALQ_TRY(tc_make_maps(&p.mapsT3[k], p.Yh, p.Yl, p.m, Tk, p.tmb, p.XfT, p.Zero, p.n, Tk, p.tmb));
+                REALQ_TRY(tc_make_maps(&p.mapsT3[k], p.Yh, p.Yl, p.m, Tk, p.tmb, p.XfT, p.XfT, p.n, Tk, p.tmb));
             }
         }
         if (fresh) {
