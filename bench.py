@@ -37,9 +37,11 @@ NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
     ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
-    # the Block-GD G product with the fused Adam step: 219 launches of a
-    # Qwen3-0.6B block over 3 steps, 50.05 MB read + 1.08 MB written on average
-    ("qwen3-0.6b", "bgd_g_gemm_adam"): 51125381,
+    # the Block-GD G product: per block the next block's columns as a K split
+    # (store epilogue) and the other free columns with the fused Adam step;
+    # 695 launches of a Qwen3-0.6B block over 5 steps, 37.46 MB of DRAM
+    # traffic per launch on average
+    ("qwen3-0.6b", "bgd_g_gemm_adam"): 37455628,
 }
 
 
@@ -268,8 +270,19 @@ def gpu_arm(args, wl, rank, world):
             tt = torch.tensor([e_ms], device=dev)
             dist.all_reduce(tt, op=dist.ReduceOp.MAX)
             e_ms = float(tt.item())
+        # the host link's rate right after the timed steps (one pinned copy of
+        # the largest input): the end-to-end step is bound by it, and the
+        # link is shared with the host's other GPUs
+        big = max(host_x.values(), key=lambda t: t.numel())
+        dst = dev_x[max(dev_x, key=lambda k: dev_x[k].numel())]
+        torch.cuda.synchronize()
+        l0 = time.perf_counter()
+        dst.copy_(big, non_blocking=True)
+        torch.cuda.synchronize()
+        link_gbs = big.numel() * big.element_size() / (time.perf_counter() - l0) / 1e9
         e2e = {"value": cols / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": e2e_bytes["h2d"],
-               "d2h_bytes_per_step": e2e_bytes["d2h"], "ms_per_step": e_ms / args.steps}
+               "d2h_bytes_per_step": e2e_bytes["d2h"], "ms_per_step": e_ms / args.steps,
+               "h2d_link_gbs": round(link_gbs, 1)}
 
     result = None
     if rank == 0:

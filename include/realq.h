@@ -400,8 +400,10 @@ const char *realq_last_error(void);
 /* Launch accounting and per-kernel timing.
  * realq_launch_count(): number of kernels this library has launched since load.
  * With profiling on, every launch is bracketed by CUDA events recorded on its
- * own stream; realq_profile_collect synchronizes those events, writes up to
- * max_entries per-kernel totals and clears them. */
+ * own stream, and calls keep all of their work on the caller's stream (no
+ * auxiliary streams, same arithmetic), so that with one caller stream each
+ * interval is the kernel's own time; realq_profile_collect synchronizes those
+ * events, writes up to max_entries per-kernel totals and clears them. */
 typedef struct {
     char name[48];
     int64_t launches;

@@ -42,6 +42,7 @@ realq_status_t check_launch(const char *what) {
 // ------------------------------------------------------ launch accounting ---
 static std::atomic<int64_t> g_launches{0};
 static std::atomic<int> g_prof_on{0};
+bool profiling() { return g_prof_on.load(std::memory_order_relaxed) != 0; }
 struct ProfRec {
     const char *name;
     cudaEvent_t a, b;
@@ -470,7 +471,9 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     REALQ_CUDA_TRY(cudaMemsetAsync(p.status, 0, sizeof(int), s));
     if (block_begin == 0) REALQ_TRY(sweep_init(s, p));
     REALQ_TRY(sweep_prologue_r0(s, p, block_begin == 0));
-    if (p.tc && p.bgd_steps > 0 && block_end - block_begin > 1) REALQ_TRY(sweep_side_stream(s, p));
+    // (while profiling, everything stays on the caller's stream, so that each
+    // launch's event interval is its own time; the arithmetic is the same)
+    if (p.tc && p.bgd_steps > 0 && block_end - block_begin > 1 && !profiling()) REALQ_TRY(sweep_side_stream(s, p));
     for (int64_t b = block_begin; b < block_end; ++b) REALQ_TRY(sweep_block(s, p, b));
     REALQ_TRY(sweep_join_wide(s, p));
     return REALQ_OK;

@@ -228,6 +228,9 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
     e.Sl[w] = -step - sh;
 }
 
+// MODE = e.mode, fixed at compile time: one kernel per epilogue (and so one
+// name per role in a profiler's launch list)
+template <int MODE>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
                        int a_row0, const TcEpi e, int *err, int kchunk, int exact) {
@@ -353,15 +356,15 @@ __global__ void __launch_bounds__(THREADS, 1)
         constexpr int RPW = TB / (THREADS / 32);   // tile rows per warp
         const int cc = lane * 4;
         const int64_t gj = j0 + cc;
-        const bool vec = e.mode != TC_STORE && gj + 3 < N;
+        const bool vec = MODE != TC_STORE && gj + 3 < N;
         for (int rb = warp * RPW; rb < warp * RPW + RPW; rb += 4) {
             if (i0 + rb >= M) break;
             // a batch of 4 rows runs vectorized when all 4 exist (M need not be
             // a multiple of 4 for a row group)
             if (vec && i0 + rb + 3 < M) {
-                if (e.mode == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
-                else if (e.mode == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
-                else if (e.mode == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
+                if (MODE == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                else if (MODE == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                else if (MODE == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
                 else accum_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
             } else {
                 for (int u = 0; u < 4; ++u) {
@@ -371,9 +374,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                     for (int q = 0; q < 4; ++q) {
                         if (gj + q >= N) break;
                         float &t = T[rr * TP + cc + q];
-                        if (e.mode == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
-                        else if (e.mode == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
-                        else if (e.mode == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
+                        if (MODE == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
+                        else if (MODE == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
+                        else if (MODE == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
                         else epi_apply(e, gi, gj + q, t);
                     }
                 }
@@ -381,7 +384,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         }
     }
     __syncthreads();
-    if (good && (e.mode == TC_BGD_P || e.mode == TC_BGD_PG)) {
+    if (good && (MODE == TC_BGD_P || MODE == TC_BGD_PG)) {
         // columns of the tile, lanes over rows: P^T rows are contiguous
         constexpr int CPW = TB / (THREADS / 32);   // tile columns per warp
         for (int cc = warp * CPW; cc < warp * CPW + CPW; ++cc) {
@@ -507,17 +510,44 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
     if (kchunk < 0 || (kchunk % KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
         return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name, KS);
+    if (e.mode < TC_STORE || e.mode > TC_BGD_PG) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
     static bool configured = false;
     if (!configured) {
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM));
+        constexpr cudaFuncAttribute kSmem = cudaFuncAttributeMaxDynamicSharedMemorySize;
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_STORE>, kSmem, SMEM));
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_BGD_P>, kSmem, SMEM));
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_ADAM>, kSmem, SMEM));
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_ACCUM>, kSmem, SMEM));
+        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_BGD_PG>, kSmem, SMEM));
         configured = true;
     }
     const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
     {
         Launch L(name, s);
         const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
-        gemm_tf32x3_kernel<<<dim3((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB), nz), THREADS, SMEM, s>>>(
-            m, M, N, K, k_off, b_row0, a_row0, e, err, kchunk, exact);
+        const dim3 grid((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB), nz);
+        switch (e.mode) {
+            case TC_STORE:
+                gemm_tf32x3_kernel<TC_STORE><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                         kchunk, exact);
+                break;
+            case TC_BGD_P:
+                gemm_tf32x3_kernel<TC_BGD_P><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                         kchunk, exact);
+                break;
+            case TC_ADAM:
+                gemm_tf32x3_kernel<TC_ADAM><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                        kchunk, exact);
+                break;
+            case TC_ACCUM:
+                gemm_tf32x3_kernel<TC_ACCUM><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                         kchunk, exact);
+                break;
+            default:
+                gemm_tf32x3_kernel<TC_BGD_PG><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                          kchunk, exact);
+                break;
+        }
     }
     return check_launch(name);
 }

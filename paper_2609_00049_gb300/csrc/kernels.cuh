@@ -188,6 +188,7 @@ struct SweepPlan {
     int wide_pending = 0;
 };
 realq_status_t sweep_side_stream(cudaStream_t s, SweepPlan &p);
+bool profiling();   // per-launch event profiling on (work then stays on the caller's stream)
 realq_status_t sweep_join_wide(cudaStream_t s, SweepPlan &p);
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups = 0,
                       int nmb = 0, int64_t tmb = 0);

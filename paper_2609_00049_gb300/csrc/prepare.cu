@@ -361,12 +361,12 @@ realq_status_t aux_for(cudaStream_t s, int64_t nsteps, AuxStream **out) {
 
 realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                        uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes) {
-    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, true, true);
+    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, fail_col, ws, ws_bytes, !profiling(), true);
 }
 
 realq_status_t prepare_deferred(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U,
                                 float *Hbar, uint8_t *dead, void *ws, size_t ws_bytes) {
-    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, nullptr, ws, ws_bytes, true, false);
+    return prepare_impl(s, n, norm, damp, H, U, Hbar, dead, nullptr, ws, ws_bytes, !profiling(), false);
 }
 
 realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,

@@ -30,6 +30,14 @@ def test_exports_every_declared_symbol(L):
         assert hasattr(L, n), n
 
 
+def test_every_symbol_resolves_at_load(L):
+    # immediate binding: a symbol the library uses but does not define (e.g.
+    # a helper declared in one namespace and defined in another) fails here
+    # instead of at its first call on a GPU
+    from paper_2609_00049_gb300 import library_path
+    ctypes.CDLL(library_path, mode=os.RTLD_NOW)
+
+
 def test_status_strings(L):
     import paper_2609_00049_gb300 as rq
     for s in range(8):
