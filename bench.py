@@ -114,6 +114,22 @@ class ClockSampler:
 # --------------------------------------------------------------------------
 # the GPU arm
 # --------------------------------------------------------------------------
+def max_over_ranks(x: float, dist=None, device="cpu") -> float:
+    """The largest of every rank's x (each rank's replica timed on its own
+    clock; the job takes as long as its slowest rank); x itself on one rank."""
+    if dist is None:
+        return x
+    import torch
+    t = torch.tensor([float(x)], device=device, dtype=torch.float64)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(columns_per_step: int, steps: int, world: int, ms: float) -> float:
+    """Whole-job columns/s: every rank quantizes its own replica of the block."""
+    return columns_per_step * steps * world / (ms / 1e3)
+
+
 def gpu_arm(args, wl, rank, world):
     import torch
     import paper_2609_00049_gb300 as rq
@@ -241,12 +257,9 @@ def gpu_arm(args, wl, rank, world):
         torch.cuda.synchronize()
         rq.realq_profile_enable(False)
         prof = rq.realq_profile_collect(256)
-    if dist is not None:
-        tt = torch.tensor([ms_total], device=dev)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        ms_total = float(tt.item())
+    ms_total = max_over_ranks(ms_total, dist, dev)
     cols = wl.total_columns * args.steps * world
-    value = cols / (ms_total / 1e3)
+    value = job_throughput(wl.total_columns, args.steps, world, ms_total)
 
     # ---- end to end through host buffers
     e2e = None
@@ -266,10 +279,7 @@ def gpu_arm(args, wl, rank, world):
         torch.cuda.synchronize()
         barrier()
         e_ms = (time.perf_counter() - e0) * 1e3
-        if dist is not None:
-            tt = torch.tensor([e_ms], device=dev)
-            dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-            e_ms = float(tt.item())
+        e_ms = max_over_ranks(e_ms, dist, dev)
         # the host link's rate right after the timed steps (one pinned copy of
         # the largest input): the end-to-end step is bound by it, and the
         # link is shared with the host's other GPUs
