@@ -367,6 +367,30 @@ realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, 
 size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg_t *qcfg,
                                      const realq_bgd_cfg_t *bcfg, int has_F_next, int has_Dbar);
 
+/* realq_quantize_layer with a trace of the surrogate (Eq. fisher_loss, moment
+ * form at the layer level, L = 1/2 tr(F_eff ΔW H̄ ΔWᵀ), ΔW = Ŵ - W0 with the
+ * quantized columns dequantized and the rest as they stand): for every block
+ * b of the range that takes Block-GD steps (all but the layer's last),
+ *   block_loss[2 b]     = L before the block's steps (after its OBS and lazy
+ *                         update),
+ *   block_loss[2 b + 1] = L after them,
+ * with the block's F_eff (the sliding window's blend).  block_loss: device,
+ * nb x 2 floats (the last block's pair is not written); trace_ws: device,
+ * realq_quantize_trace_workspace_size(m, n) bytes.  Unperturbed inputs only
+ * (no Dbar).  Each value is a full surrogate evaluation (about 2 m n^2 +
+ * 2 m^2 n flops), and the block's optimizer step completes before the second
+ * one, so tracing slows the sweep. */
+realq_status_t realq_quantize_layer_traced(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                           realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                           const uint8_t *dead, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                           float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
+                                           size_t ws_bytes, float *block_loss, void *trace_ws,
+                                           size_t trace_ws_bytes);
+size_t realq_quantize_trace_workspace_size(int64_t m, int64_t n);
+
 /* Step 4 alone: bcfg->steps_per_block optimizer steps of Eq. block_gd_update
  * on the columns col_start..n-1 of W (columns < col_start are locked; they
  * hold dequantized values).  alpha blends F and F_next (ignored when F_next is

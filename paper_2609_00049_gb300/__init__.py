@@ -25,6 +25,7 @@ __all__ = [
     "realq_hessian_accumulate_weighted", "realq_hessian_prepare_scaled", "realq_quantize_layer_grouped",
     "realq_quantize_grouped_workspace_size", "realq_quantize_layer_minibatch",
     "realq_quantize_minibatch_workspace_size", "realq_quantize_tokens_workspace_size", "realq_quantize_layer_tokens",
+    "realq_quantize_trace_workspace_size",
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
@@ -102,6 +103,10 @@ _SIGS = {
                                       _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_minibatch_workspace_size": ([_i64, _i64, _int, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
                                                  _int], _sz),
+    "realq_quantize_layer_traced": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, ctypes.POINTER(QuantCfg),
+                                     ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp, _P_i64, _vp, _vp, _vp, _vp,
+                                     _int, _i64, _i64, _vp, _sz, _vp, _vp, _sz], _int),
+    "realq_quantize_trace_workspace_size": ([_i64, _i64], _sz),
     "realq_quantize_tokens_workspace_size": ([_i64, _i64, _i64, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
                                               _int], _sz),
     "realq_quantize_layer_tokens": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64, _i64, _f32,
@@ -381,12 +386,19 @@ def realq_quantize_workspace_size(m: int, n: int, qcfg: QuantCfg, bcfg: Optional
                                                    int(has_F_next), int(has_Dbar)))
 
 
+def realq_quantize_trace_workspace_size(m: int, n: int) -> int:
+    return int(lib().realq_quantize_trace_workspace_size(m, n))
+
+
 def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch.Tensor], qcfg: QuantCfg,
                          W_work: torch.Tensor, codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *,
                          Dbar=None, dead=None, bcfg: Optional[BgdCfg] = None, F=None, F_next=None,
                          adam_m=None, adam_v=None, bgd_disp=None, adam_t: int = 0, W_deq=None,
-                         block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None) -> int:
-    """Runs blocks [block_begin, block_end) of the sweep; returns the Adam step counter."""
+                         block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None,
+                         block_loss: Optional[torch.Tensor] = None, trace_ws=None) -> int:
+    """Runs blocks [block_begin, block_end) of the sweep; returns the Adam step counter.
+    With block_loss (nb x 2 fp32, device) the surrogate before and after every
+    block's Block-GD steps is written there (realq_quantize_layer_traced)."""
     m, n = W0.shape
     nb = -(-n // qcfg.block_size)
     if block_end is None:
@@ -399,11 +411,17 @@ def realq_quantize_layer(W0: torch.Tensor, U: torch.Tensor, Hbar: Optional[torch
     _need(bgd_disp, torch.float32, (m, n), "bgd_disp")
     t = ctypes.c_int64(adam_t)
     wp, wb = _ws(ws)
-    _check(lib().realq_quantize_layer(
-        _stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar), _ptr(Dbar), _ptr(dead),
-        ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
-        _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero),
-        _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin), int(block_end), wp, wb))
+    common = (_stream(stream), m, n, _ptr(W0), _dtype(W0), _ptr(U), _ptr(Hbar))
+    tail = (ctypes.byref(qcfg), ctypes.byref(bcfg) if bcfg is not None else None, _ptr(F), _ptr(F_next),
+            _ptr(W_work), _ptr(adam_m), _ptr(adam_v), _ptr(bgd_disp), ctypes.byref(t), _ptr(codes), _ptr(scale),
+            _ptr(zero), _ptr(W_deq), _dtype(W_deq) if W_deq is not None else REALQ_F32, int(block_begin),
+            int(block_end), wp, wb)
+    if block_loss is None:
+        _check(lib().realq_quantize_layer(*common, _ptr(Dbar), _ptr(dead), *tail))
+    else:
+        _need(block_loss, torch.float32, (nb, 2), "block_loss")
+        tp, tb = _ws(trace_ws)
+        _check(lib().realq_quantize_layer_traced(*common, _ptr(dead), *tail, _ptr(block_loss), tp, tb))
     return t.value
 
 

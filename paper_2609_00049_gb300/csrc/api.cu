@@ -396,6 +396,13 @@ struct TokArgs {
     float clip;          // per-token output clipping percentile, (0, 1]
 };
 
+// Per-block surrogate values (nullptr: not traced).
+struct TraceArgs {
+    float *block_loss;   // device, nb x 2
+    void *ws;
+    size_t ws_bytes;
+};
+
 static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
                                     int grouped, int rgroups, const float *Ug, const float *Hbar_g,
                                     const uint8_t *dead_g, int nmb, const float *Hbar_mb,
@@ -404,7 +411,8 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
                                     const float *F_next, float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
                                     int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
                                     realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
-                                    size_t ws_bytes, const char *who, const TokArgs *tok = nullptr) {
+                                    size_t ws_bytes, const char *who, const TokArgs *tok = nullptr,
+                                    const TraceArgs *trace = nullptr) {
     if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n must be > 0", who);
     if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n too large", who);
     if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "%s: bad dtype", who);
@@ -465,6 +473,15 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
         // single-precision value; the product is exact in double)
         const int64_t k = (int64_t)std::ceil((double)tok->clip * (double)m) - 1;
         p.rank_q = std::min<int64_t>(std::max<int64_t>(k, 0), m - 1);
+    }
+    if (trace) {
+        if (!trace->block_loss) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL block_loss", who);
+        if (has_db) return fail(REALQ_ERR_UNSUPPORTED, "%s: the trace takes unperturbed inputs (Dbar = NULL)", who);
+        REALQ_TRY(check_ws(trace->ws, trace->ws_bytes, surrogate_ws_bytes(m, n) + 256, who));
+        if (bgd) {
+            p.block_loss = trace->block_loss;
+            p.trace_ws = trace->ws;
+        }
     }
     sweep_carve(p, ws, bgd, has_fn, has_db);
     cudaStream_t s = S(stream);
@@ -570,6 +587,25 @@ realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int
     return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, Hbar, nullptr, dead,
                          qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq,
                          deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_tokens", &tok);
+}
+
+size_t realq_quantize_trace_workspace_size(int64_t m, int64_t n) {
+    return (m > 0 && n > 0) ? surrogate_ws_bytes(m, n) + 256 : 0;
+}
+
+realq_status_t realq_quantize_layer_traced(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
+                                           realq_dtype_t w_dtype, const float *U, const float *Hbar,
+                                           const uint8_t *dead, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
+                                           float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
+                                           size_t ws_bytes, float *block_loss, void *trace_ws,
+                                           size_t trace_ws_bytes) {
+    const TraceArgs tr{block_loss, trace_ws, trace_ws_bytes};
+    return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, Hbar, nullptr, dead,
+                         qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale, zero, W_deq,
+                         deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_traced", nullptr, &tr);
 }
 
 // ---------------------------------------------------------------- BGD -----

@@ -183,6 +183,10 @@ struct SweepPlan {
     // free columns on a side stream, joined before anything else reads or
     // writes them.  wide == nullptr: everything on the sweep's stream.
     float *Gpart = nullptr;                  // K-split partials of the next block's G (8 x m x B)
+    // tracing: the surrogate with the block's F_eff before and after its
+    // Block-GD steps, into block_loss[2 b], block_loss[2 b + 1] (device)
+    float *block_loss = nullptr;
+    void *trace_ws = nullptr;
     cudaStream_t wide = nullptr;
     cudaEvent_t wide_fork = nullptr, wide_done = nullptr;
     int wide_pending = 0;

@@ -821,6 +821,28 @@ realq_status_t bgd_step(cudaStream_t s, SweepPlan &p, int64_t col_start, float a
     return REALQ_OK;
 }
 
+namespace {
+__global__ void blend_kernel(float alpha, const float *a, const float *b, float *out) {
+    out[0] = alpha * a[0] + (1.f - alpha) * b[0];
+}
+}  // namespace
+
+// The surrogate of the current weights (quantized columns dequantized, the
+// rest as they stand) with F_eff = alpha F + (1 - alpha) F_next, which is
+// linear in F: alpha L(F) + (1 - alpha) L(F_next).
+static realq_status_t trace_loss(cudaStream_t s, SweepPlan &p, float alpha, float *out) {
+    const size_t sb = surrogate_ws_bytes(p.m, p.n);
+    float *tmp = reinterpret_cast<float *>(static_cast<char *>(p.trace_ws) + sb);
+    REALQ_TRY(surrogate(s, p.m, p.n, p.W, p.W0, p.w_dtype, p.Hbar, p.F, p.F_next ? tmp : out, p.trace_ws));
+    if (!p.F_next) return REALQ_OK;
+    REALQ_TRY(surrogate(s, p.m, p.n, p.W, p.W0, p.w_dtype, p.Hbar, p.F_next, tmp + 1, p.trace_ws));
+    {
+        Launch L("trace_blend", s);
+        blend_kernel<<<1, 1, 0, s>>>(alpha, tmp, tmp + 1, out);
+    }
+    return check_launch("trace_blend");
+}
+
 realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     const int B = p.block;
     const int64_t bs = b * B;
@@ -890,6 +912,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             p.f_split_alpha_valid = 1;
             p.f_split_alpha = a_eff;
         }
+        if (p.block_loss) REALQ_TRY(trace_loss(s, p, p.F_next ? alpha : 1.f, p.block_loss + 2 * b));
         for (int k = 0; k < p.bgd_steps; ++k) {
             const bool last = k == p.bgd_steps - 1;
             if (p.tmb > 0)
@@ -899,11 +922,17 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             else
                 REALQ_TRY(p.grouped ? bgd_one_tc_grouped(s, p, be, last) : bgd_one_tc(s, p, be, last));
         }
+        if (p.block_loss) {
+            REALQ_TRY(sweep_join_wide(s, p));
+            REALQ_TRY(trace_loss(s, p, p.F_next ? alpha : 1.f, p.block_loss + 2 * b + 1));
+        }
         return REALQ_OK;
     }
     const float *Fuse = nullptr;
     REALQ_TRY(fisher_for(s, p, alpha, &Fuse));
+    if (p.block_loss) REALQ_TRY(trace_loss(s, p, p.F_next ? alpha : 1.f, p.block_loss + 2 * b));
     for (int k = 0; k < p.bgd_steps; ++k) REALQ_TRY(bgd_one(s, p, be, Fuse, 1));
+    if (p.block_loss) REALQ_TRY(trace_loss(s, p, p.F_next ? alpha : 1.f, p.block_loss + 2 * b + 1));
     return REALQ_OK;
 }
 

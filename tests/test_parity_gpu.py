@@ -870,3 +870,43 @@ def test_token_block_gd_with_output_clipping(clip, start, steps):
     assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
     assert s_unexpl == 0
 
+
+
+@pytest.mark.parametrize("with_next", [False, True])
+def test_traced_block_losses(with_next):
+    # the surrogate before and after every block's Block-GD step against the
+    # oracle's record of the same values (1e-3 relative, the loss tolerance);
+    # with the sliding window the trace uses each block's blended F_eff
+    case = synth.layer_case(28, 96, 320, 1200, with_next=True)
+    qkw = dict(group_size=64, block_size=64)
+    kw = dict(b_global_start=3, B_total=9) if with_next else {}
+    Hs, T = oracle.hessian_sum([case.Xhat])
+    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=64, block_size=64,
+                             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": kw.get("b_global_start", 1),
+                                  "B_total": kw.get("B_total", 1)},
+                             F=case.F, F_next=case.F_next if with_next else None)
+    H, _, T_ = layer.accumulate([dev(case.Xhat)], 320)
+    prep = layer.prepare(H, T_)
+    q = rq.quant_cfg(**qkw)
+    b = rq.bgd_cfg(2e-4, **kw)
+    m, n = 96, 320
+    nb = n // 64
+    W = torch.empty(m, n, device="cuda")
+    codes = torch.empty(m, n // 2, dtype=torch.uint8, device="cuda")
+    scale = torch.empty(m, n // 64, device="cuda")
+    zero = torch.empty(m, n // 64, dtype=torch.uint8, device="cuda")
+    st = {k: torch.empty(m, n, device="cuda") for k in ("adam_m", "adam_v", "bgd_disp")}
+    ws = rq.workspace(rq.realq_quantize_workspace_size(m, n, q, b, with_next))
+    bl = torch.full((nb, 2), float("nan"), device="cuda")
+    tws = rq.workspace(rq.realq_quantize_trace_workspace_size(m, n))
+    rq.realq_quantize_layer(dev(case.W0), prep.U, prep.Hbar, q, W, codes, scale, zero, dead=prep.dead, bcfg=b,
+                            F=dev(case.F), F_next=dev(case.F_next) if with_next else None, ws=ws,
+                            block_loss=bl, trace_ws=tws, **st)
+    rq.realq_workspace_status(ws)
+    got = bl.cpu().numpy()
+    assert np.isnan(got[nb - 1]).all()          # the last block takes no step
+    for blk, alpha, before, after in orc["block_loss"]:
+        print(f"\nblock {blk} alpha {alpha:.3f}: before {got[blk, 0]:.6e} / {before:.6e}, "
+              f"after {got[blk, 1]:.6e} / {after:.6e}")
+        assert abs(got[blk, 0] - before) <= 1e-3 * abs(before)
+        assert abs(got[blk, 1] - after) <= 1e-3 * abs(after)
