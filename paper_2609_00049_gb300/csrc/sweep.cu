@@ -108,6 +108,8 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int kb = a.kb;
     if ((a.n & 3) == 0 && kb == B) {
+        // (unrolled so that several loads are in flight per thread)
+#pragma unroll 8
         for (int idx = threadIdx.x; idx < B * B / 4; idx += blockDim.x) {
             const int j = (idx * 4) / B, k = (idx * 4) % B;
             const float4 v = *reinterpret_cast<const float4 *>(a.U + (a.bs + j) * a.n + a.bs + k);
@@ -239,20 +241,20 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
         }
         __syncthreads();
         if (warp > s) {
-            // the 32 errors of sub-block s, column by column in order
-            float e[32];
-#pragma unroll
-            for (int jj = 0; jj < 32; ++jj) e[jj] = Es[lane * 33 + jj];
-#pragma unroll
+            // the 32 errors of sub-block s, column by column in order (the
+            // column loop stays rolled: the kernel's code then fits the
+            // instruction cache)
+#pragma unroll 1
             for (int jj = 0; jj < 32; ++jj) {
+                const float ej = Es[lane * 33 + jj];
                 const float *urow = Us + (s * 32 + jj) * UP + c0;
 #pragma unroll
                 for (int c = 0; c < 32; c += 4) {
                     const float4 u = *reinterpret_cast<const float4 *>(urow + c);
-                    r[c] = fmaf(-e[jj], u.x, r[c]);
-                    r[c + 1] = fmaf(-e[jj], u.y, r[c + 1]);
-                    r[c + 2] = fmaf(-e[jj], u.z, r[c + 2]);
-                    r[c + 3] = fmaf(-e[jj], u.w, r[c + 3]);
+                    r[c] = fmaf(-ej, u.x, r[c]);
+                    r[c + 1] = fmaf(-ej, u.y, r[c + 1]);
+                    r[c + 2] = fmaf(-ej, u.z, r[c + 2]);
+                    r[c + 3] = fmaf(-ej, u.w, r[c + 3]);
                 }
             }
         }
