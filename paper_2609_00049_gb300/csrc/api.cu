@@ -10,6 +10,8 @@
 #include <cstring>
 #include <map>
 #include <mutex>
+#include <set>
+#include <tuple>
 #include <string>
 #include <vector>
 
@@ -36,6 +38,19 @@ realq_status_t fail(realq_status_t s, const char *fmt, ...) {
 realq_status_t check_launch(const char *what) {
     cudaError_t e = cudaGetLastError();
     if (e != cudaSuccess) return fail(REALQ_ERR_CUDA, "%s: %s", what, cudaGetErrorString(e));
+    return REALQ_OK;
+}
+
+realq_status_t set_smem_limit(const void *kernel, int bytes) {
+    int dev = 0;
+    REALQ_CUDA_TRY(cudaGetDevice(&dev));
+    static std::mutex mu;
+    static std::set<std::tuple<const void *, int, int>> done;
+    std::lock_guard<std::mutex> lk(mu);
+    const auto key = std::make_tuple(kernel, dev, bytes);
+    if (done.count(key)) return REALQ_OK;
+    REALQ_CUDA_TRY(cudaFuncSetAttribute(kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, bytes));
+    done.insert(key);
     return REALQ_OK;
 }
 

@@ -511,16 +511,11 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     if (kchunk < 0 || (kchunk % KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
         return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name, KS);
     if (e.mode < TC_STORE || e.mode > TC_BGD_PG) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
-    static bool configured = false;
-    if (!configured) {
-        constexpr cudaFuncAttribute kSmem = cudaFuncAttributeMaxDynamicSharedMemorySize;
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_STORE>, kSmem, SMEM));
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_BGD_P>, kSmem, SMEM));
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_ADAM>, kSmem, SMEM));
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_ACCUM>, kSmem, SMEM));
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(gemm_tf32x3_kernel<TC_BGD_PG>, kSmem, SMEM));
-        configured = true;
-    }
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_STORE>), SMEM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_P>), SMEM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ADAM>), SMEM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ACCUM>), SMEM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_PG>), SMEM));
     const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
     {
         Launch L(name, s);

@@ -27,6 +27,9 @@ struct Launch {
 
 // cudaGetLastError after a launch, as a library status
 realq_status_t check_launch(const char *what);
+// The dynamic shared-memory limit of a kernel, set once per (kernel, device,
+// size); safe to call from several host threads.
+realq_status_t set_smem_limit(const void *kernel, int bytes);
 
 // Device status word layout (int32) kept at the start of workspaces.
 enum : int {

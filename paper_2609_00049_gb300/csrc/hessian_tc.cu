@@ -345,11 +345,7 @@ static realq_status_t hess_tc_launch(cudaStream_t s, int64_t n, int64_t T, const
     int64_t tper = (T + splits - 1) / splits;
     tper = (tper + KSTAGE - 1) / KSTAGE * KSTAGE;
     splits = (int)((T + tper - 1) / tper);
-    static bool configured = false;
-    if (!configured) {
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(hess_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, SMEM_BYTES));
-        configured = true;
-    }
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(hess_tc_kernel), SMEM_BYTES));
     float *part = static_cast<float *>(ws);
     {
         Launch L(name, s);

@@ -157,12 +157,7 @@ realq_status_t tok_clip(cudaStream_t s, int64_t T, int64_t m, float *D, int64_t 
     if (T <= 0) return REALQ_OK;
     const size_t stage = (size_t)CLIP_WARPS * m * sizeof(float);
     constexpr size_t kMaxStage = 160 * 1024;
-    static bool configured = false;
-    if (!configured) {
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(clip_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                            (int)kMaxStage));
-        configured = true;
-    }
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(clip_kernel<true>), (int)kMaxStage));
     {
         Launch L("tok_clip", s);
         if (stage <= kMaxStage)

@@ -366,11 +366,7 @@ inline unsigned blocks_for(int64_t count, int threads = 256) { return (unsigned)
 template <int B, int G>
 realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
     const size_t smem = (size_t)(B * (B + 4) + B + QB_ROWS * 33 + 2 * (B / 32) * QB_ROWS) * sizeof(float);
-    static bool configured = false;
-    if (!configured) {
-        REALQ_CUDA_TRY(cudaFuncSetAttribute(quant_block_kernel<B, G>, cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem));
-        configured = true;
-    }
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(quant_block_kernel<B, G>), (int)smem));
     {
         Launch L("quant_block", s);
         quant_block_kernel<B, G><<<ceil_div(qa.m, QB_ROWS), B, smem, s>>>(qa);
