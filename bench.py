@@ -19,6 +19,7 @@ import os
 import statistics
 import subprocess
 import sys
+import tempfile
 import time
 
 import numpy as np
@@ -66,17 +67,17 @@ class ClockSampler:
               "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
               "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
 
-    def __init__(self, uuid):
+    def __init__(self, uuid, log_dir=None):
         self.uuid = uuid
         self.proc = None
-        self.path = os.path.join(ROOT, "gpurun_out", f"clocks_{os.getpid()}.csv")
+        self.path = os.path.join(log_dir or tempfile.gettempdir(), f"clocks_{os.getpid()}.csv")
 
     def start(self):
         try:
             os.makedirs(os.path.dirname(self.path), exist_ok=True)
             self.f = open(self.path, "w")
             self.proc = subprocess.Popen(["nvidia-smi", f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits",
-                                          "-lms", "200"], stdout=self.f, stderr=subprocess.DEVNULL)
+                                          "-lms", "100"], stdout=self.f, stderr=subprocess.DEVNULL)
         except Exception:
             self.proc = None
 
@@ -227,7 +228,7 @@ def gpu_arm(args, wl, rank, world):
         uuid = str(torch.cuda.get_device_properties(dev).uuid)
     except Exception:
         pass
-    clocks = ClockSampler(uuid)
+    clocks = ClockSampler(uuid, args.clock_log)
     launches0 = rq.realq_launch_count()
     clocks.start()
     torch.cuda.synchronize()
@@ -562,6 +563,7 @@ def main():
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--a-loss-clip", type=float, default=None,
                     help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
+    ap.add_argument("--clock-log", default=None, help="directory for the raw clock samples (default: temp dir)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--no-graph", action="store_true", help="launch the block step eagerly instead of as a CUDA graph")
