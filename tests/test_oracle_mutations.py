@@ -1,0 +1,83 @@
+"""The pins must catch plausible mistakes in the oracle.
+
+Each case plants one mistake in a copy of the oracle (a flipped sign, a
+dropped term, a transposed operand, an off-by-one rank, a missing factor)
+and runs the pin suite against the copy: it must fail.  The copy lives in a
+temporary directory; nothing here touches the CUDA path."""
+import os
+import shutil
+import subprocess
+import sys
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+MUTATIONS = {
+    # OBS compensation of Eq. (gptq_update): its sign, its columns shifted by one
+    "compensation_sign": ("W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])",
+                          "W[rows, j + 1:] += np.outer(e[rows] / d, Hinv[j, j + 1:])"),
+    "compensation_shift": ("W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])",
+                           "W[rows, j + 1:] -= np.outer(e[rows] / d, np.roll(Hinv[j, j + 1:], 1))"),
+    # the Schur-complement downdate dropped
+    "no_downdate": ("Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d",
+                    "Hinv[j + 1:, j + 1:] -= 0.0 * np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d"),
+    # the residual of the quantizer halved
+    "residual": ("e = W[:, j] - dq ", "e = W[:, j] - 0.5 * dq "),
+    # the cross-moment term transposed
+    "dbar_transposed": ("P = P + W0 @ np.asarray(Dbar, dtype=np.float64)",
+                        "P = P + W0 @ np.asarray(Dbar, dtype=np.float64).T"),
+    # the 1/2 of the surrogate
+    "surrogate_half": ("return 0.5 * acc / T", "return acc / T"),
+    # Adam's second bias correction
+    "adam_bias": ("vhat = v / (1.0 - self.beta2 ** self.t)", "vhat = v"),
+    # the damping 1.5 times too large
+    "damping_mean": ("lam = damp_frac * float(np.mean(np.diag(Hd)))",
+                     "lam = damp_frac * float(np.mean(np.diag(Hd))) * 1.5"),
+    # the sliding-window weight off by one block
+    "alpha_index": ("return 1.0 - (b_global - 1) / (B_total - 1)", "return 1.0 - b_global / (B_total - 1)"),
+    # the output clipping: rank off by one, the factor inverted, a missing
+    # factor in the gradient
+    "clip_rank": ("k = min(max(int(math.ceil(p32 * m)) - 1, 0), m - 1)",
+                  "k = min(max(int(math.ceil(p32 * m)), 0), m - 1)"),
+    "clip_factor": ("kappa[over] = (q[:, None] / np.where(over, a, 1.0))[over]",
+                    "kappa[over] = (np.where(over, a, 1.0) / q[:, None])[over]"),
+    "clip_gradient": ("return (kappa * Z).T @ Xh / float(Xh.shape[0])", "return Z.T @ Xh / float(Xh.shape[0])"),
+    # the mini-batch moment not normalised by its own token count
+    "minibatch_norm": ("Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)",
+                       "Hstep = np.asarray(Hk, dtype=np.float64) / float(T)"),
+    # the saliency percentile rank off by one
+    "saliency_rank": ("k = min(max(int(math.ceil(p32 * T)) - 1, 0), T - 1)",
+                      "k = min(max(int(math.ceil(p32 * T)), 0), T - 1)"),
+    # the weighted Hessian without the weights
+    "weighted_hessian": ("H[g] += (c * sc[:, g:g + 1]).T @ c", "H[g] += c.T @ c"),
+    # the activation grid without its clipping ratio
+    "act_clip": ("xmax = (np.float32(a_clip) * np.abs(x).max(axis=1)).astype(np.float32)",
+                 "xmax = (np.abs(x).max(axis=1)).astype(np.float32)"),
+}
+
+
+def _pins_on_copy(tmp_path, old=None, new=None):
+    for d in ("oracle", "synth", "tests"):
+        shutil.copytree(os.path.join(ROOT, d), tmp_path / d, ignore=shutil.ignore_patterns("__pycache__"))
+    if old is not None:
+        src = (tmp_path / "oracle" / "realq.py").read_text()
+        assert src.count(old) == 1, f"mutation anchor not found once: {old}"
+        (tmp_path / "oracle" / "realq.py").write_text(src.replace(old, new))
+    env = dict(os.environ, PYTHONPATH=str(tmp_path))
+    return subprocess.run([sys.executable, "-m", "pytest", "tests/test_oracle_pins.py", "-x", "-q", "-p",
+                           "no:cacheprovider", "-m", "not gpu"], cwd=tmp_path, env=env, capture_output=True,
+                          text=True, timeout=600)
+
+
+def test_unchanged_copy_passes(tmp_path):
+    # the control: the copy itself passes, so a failure below is the mistake's
+    r = _pins_on_copy(tmp_path)
+    assert r.returncode == 0, r.stdout[-2000:]
+
+
+@pytest.mark.parametrize("name", sorted(MUTATIONS))
+def test_pins_catch_the_mistake(name, tmp_path):
+    r = _pins_on_copy(tmp_path, *MUTATIONS[name])
+    assert r.returncode != 0, f"the pins did not catch '{name}':\n{r.stdout[-2000:]}"
+    assert " failed" in r.stdout, r.stdout[-2000:]     # a failing pin, not a crash
