@@ -195,7 +195,7 @@ realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, i
  *   X_hat   T x n bf16, token-major, 16-byte aligned, n % 8 == 0; the
  *           calibration tokens whose H gave U and Hbar (unperturbed: the
  *           reference output is W0 x̂).
- *   T_mb    tokens per mini-batch, a multiple of 4.
+ *   T_mb    tokens per mini-batch, a multiple of 4, at most 2,097,120.
  * Needs the tensor-core path (m, n multiples of 4, >= 32; block_size > 0).
  * Everything else as realq_quantize_layer.  The products take the token
  * axis on the tensor cores in fp32-level precision (tf32x3); the workspace

@@ -113,3 +113,54 @@ def test_binding_fails_loudly_without_library(tmp_path, monkeypatch):
     monkeypatch.setattr(rq, "library_path", str(tmp_path / "missing.so"))
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         rq.lib()
+
+
+def _qt(L, T=8000, T_mb=2048, clip=0.95, X=FAKE, n=512):
+    import paper_2609_00049_gb300 as rq
+    q = rq.quant_cfg()
+    b = rq.bgd_cfg(1e-4)
+    t = ctypes.c_int64(0)
+    return L.realq_quantize_layer_tokens(None, 256, n, FAKE, 0, FAKE, FAKE, None, X, T, T_mb, clip, ctypes.byref(q),
+                                         ctypes.byref(b), FAKE, None, FAKE, FAKE, FAKE, FAKE, ctypes.byref(t), FAKE,
+                                         FAKE, FAKE, None, 0, 0, 4, FAKE, 1 << 40)
+
+
+def test_token_path_argument_validation(L):
+    import paper_2609_00049_gb300 as rq
+    assert _qt(L, T_mb=2046) == rq.REALQ_ERR_INVALID_ARG                 # not a multiple of 4
+    assert _qt(L, T_mb=65535 * 32 + 4) == rq.REALQ_ERR_INVALID_ARG       # beyond the layout kernels' grid
+    assert _qt(L, T=0) == rq.REALQ_ERR_INVALID_ARG
+    assert _qt(L, clip=0.0) == rq.REALQ_ERR_INVALID_ARG
+    assert _qt(L, clip=1.5) == rq.REALQ_ERR_INVALID_ARG
+    assert _qt(L, clip=float("nan")) == rq.REALQ_ERR_INVALID_ARG
+    assert _qt(L, X=ctypes.c_void_p(0x10008)) == rq.REALQ_ERR_INVALID_ARG  # not 16-byte aligned
+    assert _qt(L, X=None) == rq.REALQ_ERR_INVALID_ARG
+    assert rq.realq_quantize_tokens_workspace_size(256, 512, 2048, rq.quant_cfg(), rq.bgd_cfg(1e-4)) > \
+        rq.realq_quantize_workspace_size(256, 512, rq.quant_cfg(), rq.bgd_cfg(1e-4))
+
+
+def test_trace_and_graph_argument_validation(L):
+    import paper_2609_00049_gb300 as rq
+    q = rq.quant_cfg()
+    b = rq.bgd_cfg(1e-4)
+    t = ctypes.c_int64(0)
+    # a NULL block_loss, and a trace workspace too small
+    assert L.realq_quantize_layer_traced(None, 256, 512, FAKE, 0, FAKE, FAKE, None, ctypes.byref(q), ctypes.byref(b),
+                                         FAKE, None, FAKE, FAKE, FAKE, FAKE, ctypes.byref(t), FAKE, FAKE, FAKE, None,
+                                         0, 0, 4, FAKE, 1 << 40, None, FAKE, 1 << 30) == rq.REALQ_ERR_INVALID_ARG
+    assert L.realq_quantize_layer_traced(None, 256, 512, FAKE, 0, FAKE, FAKE, None, ctypes.byref(q), ctypes.byref(b),
+                                         FAKE, None, FAKE, FAKE, FAKE, FAKE, ctypes.byref(t), FAKE, FAKE, FAKE, None,
+                                         0, 0, 4, FAKE, 1 << 40, FAKE, FAKE, 16) == rq.REALQ_ERR_WORKSPACE
+    assert rq.realq_quantize_trace_workspace_size(256, 512) > 3 * 256 * 512 * 4
+    # graphs: the legacy default stream cannot be captured; no graph to launch
+    assert L.realq_graph_begin(None) == rq.REALQ_ERR_INVALID_ARG
+    assert L.realq_graph_launch(None, None) == rq.REALQ_ERR_INVALID_ARG
+    assert L.realq_graph_kernels(None) == 0
+    L.realq_graph_destroy(None)                                          # a no-op
+    # the deferred preparation and its status
+    fc = ctypes.c_int64(7)
+    assert L.realq_hessian_prepare_deferred(None, 0, 10, 0.01, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20) == 1
+    assert L.realq_hessian_prepare_deferred(None, 64, 10, 0.01, FAKE, FAKE, FAKE, FAKE, FAKE, 1 << 20) == 1  # U == H
+    assert L.realq_hessian_prepare_deferred(None, 64, 10, 0.01, FAKE, ctypes.c_void_p(0x20000), FAKE, FAKE, None,
+                                            0) == rq.REALQ_ERR_WORKSPACE
+    assert L.realq_prepare_status(None, None, 0, ctypes.byref(fc)) == rq.REALQ_ERR_INVALID_ARG
