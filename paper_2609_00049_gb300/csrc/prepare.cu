@@ -54,75 +54,77 @@ __global__ void prep_damp_kernel(int64_t n, float *A, float damp, float *lam_out
     if (threadIdx.x == 0) *lam_out = lam;
 }
 
-// One warp, a 32 x 32 block As (pitch 33, upper triangle): reverse-order
-// Cholesky As = R R^T (R upper) fused with the back substitution V = R^-1,
-// written to Vs (row-major, zeros below the diagonal).  Lane j keeps column j
-// of the block and row j of V in registers.  Pivot k needs only column k of R
-// and row k of V: lane k publishes both (unscaled) through a double-buffered
-// 64-float slot bf[(k & 1) * 64 ..] in shared memory, every lane reads them
-// back with 16-byte broadcast loads and applies
+// A 32 x 32 block As (pitch 33, upper triangle): reverse-order Cholesky
+// As = R R^T (R upper) fused with the back substitution V = R^-1, written to
+// Vs (row-major, zeros below the diagonal), by the 128 threads of the CTA.
+// Lane j owns column j of the block and row j of V; warp w keeps entries
+// 8w .. 8w + 7 of both in registers.  Pivot k needs only column k of R and
+// row k of V: lane k of every warp publishes its eight entries of both
+// (unscaled) into a double-buffered 64-float slot bf[(k & 1) * 64 ..] with
+// one CTA barrier per pivot (the slot of pivot k is next written at pivot
+// k - 2, after the barrier of pivot k - 1, which every warp reaches only after
+// its reads of pivot k); every thread then applies
 //   a_ij -= r_ik r_jk (i <= j < k),   V[j] -= r_jk V[k] (j < k),
-// with r_ik = a_ik / sqrt(a_kk).  Row k of V is scaled by its own 1 / r_kk
-// once, at the end (no later pivot reads it).  A pivot that is not positive
-// (or not finite) is recorded (the first one wins; columns >= valid are
-// padding) and replaced by 1 to keep going.  Single-warp code issues slowly,
-// so the pivot step avoids shuffles and keeps to ~100 instructions.
-__device__ __forceinline__ void warp_rchol_inv32(const float (*As)[33], float (*Vs)[33], float *bf, int lane,
-                                                 int *status, int64_t col0, int valid) {
-    float c[32], v[32];
+// with r_ik = a_ik / sqrt(a_kk), to its entries.  Row k of V is scaled by its
+// own 1 / r_kk once, at the end (no later pivot reads it).  A pivot that is
+// not positive (or not finite) is recorded (the first one wins; columns >=
+// valid are padding) and replaced by 1 to keep going.  (One warp doing all 32
+// entries issues a ~100-instruction pivot at about seven cycles each; split
+// four ways with a barrier the pivot is about three times shorter.)
+__device__ __forceinline__ void cta_rchol_inv32(const float (*As)[33], float (*Vs)[33], float *bf, int warp,
+                                                int lane, int *status, int64_t col0, int valid) {
+    const int q0 = warp * 8;
+    float c[8], v[8];
 #pragma unroll
-    for (int i = 0; i < 32; ++i) {
-        c[i] = As[i][lane];
-        v[i] = (i == lane) ? 1.f : 0.f;
+    for (int i = 0; i < 8; ++i) {
+        c[i] = As[q0 + i][lane];
+        v[i] = (q0 + i == lane) ? 1.f : 0.f;
     }
     float rown = 1.f;
 #pragma unroll 1
     for (int k = 31; k >= 0; --k) {
         float *b = bf + (k & 1) * 64;
         if (lane == k) {
-#pragma unroll
-            for (int q = 0; q < 32; q += 4) {
-                *reinterpret_cast<float4 *>(b + q) = make_float4(c[q], c[q + 1], c[q + 2], c[q + 3]);
-                *reinterpret_cast<float4 *>(b + 32 + q) = make_float4(v[q], v[q + 1], v[q + 2], v[q + 3]);
-            }
+            *reinterpret_cast<float4 *>(b + q0) = make_float4(c[0], c[1], c[2], c[3]);
+            *reinterpret_cast<float4 *>(b + q0 + 4) = make_float4(c[4], c[5], c[6], c[7]);
+            *reinterpret_cast<float4 *>(b + 32 + q0) = make_float4(v[0], v[1], v[2], v[3]);
+            *reinterpret_cast<float4 *>(b + 32 + q0 + 4) = make_float4(v[4], v[5], v[6], v[7]);
         }
-        __syncwarp();
+        __syncthreads();
         float d = b[k];
         if (!(d > 0.f) || !isfinite(d)) {
-            if (lane == 0 && k < valid) atomicCAS(status, -1, (int)(col0 + k));
+            if (warp == 0 && lane == 0 && k < valid) atomicCAS(status, -1, (int)(col0 + k));
             d = 1.f;
         }
         const float rinv = rsqrtf(d);
         if (lane == k) rown = rinv;
-        const float rjk = lane < k ? b[lane] * rinv : 0.f;   // r_jk on lanes j < k
-        const float cf = -rjk * rinv;                          // r_ik = b[i] rinv
+        const float rjk = lane < k ? b[lane] * rinv : 0.f;
+        const float cf = -rjk * rinv;
+        const float4 bc0 = *reinterpret_cast<const float4 *>(b + q0);
+        const float4 bc1 = *reinterpret_cast<const float4 *>(b + q0 + 4);
+        const float4 bv0 = *reinterpret_cast<const float4 *>(b + 32 + q0);
+        const float4 bv1 = *reinterpret_cast<const float4 *>(b + 32 + q0 + 4);
+        const float bc[8] = {bc0.x, bc0.y, bc0.z, bc0.w, bc1.x, bc1.y, bc1.z, bc1.w};
+        const float bv[8] = {bv0.x, bv0.y, bv0.z, bv0.w, bv1.x, bv1.y, bv1.z, bv1.w};
 #pragma unroll
-        for (int q = 0; q < 32; q += 4) {
-            const float4 bc = *reinterpret_cast<const float4 *>(b + q);
-            const float4 bv = *reinterpret_cast<const float4 *>(b + 32 + q);
-            if (q + 0 <= lane) c[q + 0] = fmaf(bc.x, cf, c[q + 0]);
-            if (q + 1 <= lane) c[q + 1] = fmaf(bc.y, cf, c[q + 1]);
-            if (q + 2 <= lane) c[q + 2] = fmaf(bc.z, cf, c[q + 2]);
-            if (q + 3 <= lane) c[q + 3] = fmaf(bc.w, cf, c[q + 3]);
-            v[q + 0] = fmaf(bv.x, cf, v[q + 0]);
-            v[q + 1] = fmaf(bv.y, cf, v[q + 1]);
-            v[q + 2] = fmaf(bv.z, cf, v[q + 2]);
-            v[q + 3] = fmaf(bv.w, cf, v[q + 3]);
+        for (int q = 0; q < 8; ++q) {
+            if (q0 + q <= lane) c[q] = fmaf(bc[q], cf, c[q]);
+            v[q] = fmaf(bv[q], cf, v[q]);
         }
     }
 #pragma unroll
-    for (int q = 0; q < 32; ++q) Vs[lane][q] = v[q] * rown;
+    for (int q = 0; q < 8; ++q) Vs[lane][q0 + q] = v[q] * rown;
 }
 
 // Diagonal block [k0, k0 + kb) of the reverse-order blocked Cholesky, 128
 // threads.  With the block split 2 x 2 into 32 x 32 pieces,
 //   A22 = R22 R22^T,  R12 = A12 R22^-T,  A11 - R12 R12^T = R11 R11^T,
 //   V = R^-1 = [[V11, -V11 R12 V22], [0, V22]].
-// Warp 0 factors and inverts the two diagonal pieces, all four warps form the
-// 32 x 32 products (warps 1-3 form R12 V22 while warp 0 works on the second
-// piece).  Out: U_KK = V into A[K, K] (upper, in place of the block) and
-// Vt = V^T (dense 64 x 64, row-major) for the panel solve.  Rows / columns
-// >= kb are padded with the identity.
+// All four warps factor and invert the two diagonal pieces together
+// (cta_rchol_inv32) and form the 32 x 32 products.  Out: U_KK = V into
+// A[K, K] (upper, in place of the block) and Vt = V^T (dense 64 x 64,
+// row-major) for the panel solve.  Rows / columns >= kb are padded with the
+// identity.
 __global__ void __launch_bounds__(128) chol_diag_kernel(int64_t n, float *A, int64_t k0, int kb, int *status,
                                                         float *Vt) {
     __shared__ float S11[32][33], S22[32][33], A12[32][33];
@@ -151,7 +153,7 @@ __global__ void __launch_bounds__(128) chol_diag_kernel(int64_t n, float *A, int
         }
     }
     __syncthreads();
-    if (warp == 0) warp_rchol_inv32(S22, V22, bf, lane, status, k0 + 32, kb - 32);
+    cta_rchol_inv32(S22, V22, bf, warp, lane, status, k0 + 32, kb - 32);
     __syncthreads();
     // R12[i][j] = sum_l A12[i][l] V22[j][l]   (V22 upper, zeros below)
 #pragma unroll 1
@@ -163,29 +165,21 @@ __global__ void __launch_bounds__(128) chol_diag_kernel(int64_t n, float *A, int
         R12[i][j] = acc;
     }
     __syncthreads();
-    // A11 -= R12 R12^T
+    // A11 -= R12 R12^T and X = R12 V22
 #pragma unroll 1
     for (int e = tid; e < 32 * 32; e += 128) {
         const int i = e >> 5, j = e & 31;
-        float acc = 0.f;
+        float acc = 0.f, accx = 0.f;
 #pragma unroll 8
-        for (int l = 0; l < 32; ++l) acc = fmaf(R12[i][l], R12[j][l], acc);
+        for (int l = 0; l < 32; ++l) {
+            acc = fmaf(R12[i][l], R12[j][l], acc);
+            accx = fmaf(R12[i][l], V22[l][j], accx);
+        }
         S11[i][j] -= acc;
+        X[i][j] = accx;
     }
     __syncthreads();
-    if (warp == 0) {
-        warp_rchol_inv32(S11, V11, bf, lane, status, k0, kb);
-    } else {
-        // X = R12 V22
-#pragma unroll 1
-        for (int e = tid - 32; e < 32 * 32; e += 96) {
-            const int i = e >> 5, j = e & 31;
-            float acc = 0.f;
-#pragma unroll 8
-            for (int l = 0; l < 32; ++l) acc = fmaf(R12[i][l], V22[l][j], acc);
-            X[i][j] = acc;
-        }
-    }
+    cta_rchol_inv32(S11, V11, bf, warp, lane, status, k0, kb);
     __syncthreads();
     // V12 = -V11 X   (V11 upper, zeros below)
 #pragma unroll 1
