@@ -12,6 +12,10 @@ Sections cited:
   Algorithm 1 "REAL-Q Quantization"
   App. "Reconstruction error of GPTQ" theorem and the Schur-complement proof
   App. "Full Setup": Adam hyper-parameters, Eq. (reverse_cosine)
+  Sec. 3.3 Eq. (saliency_hessian) and App. "Hessian-side saliency clipping"
+  Sec. 4.3 / Sec. 5.1 mini-batches and App. "Activation clipping
+    (a_loss_clip) for small Qwen3 models"
+  Sec. 5 "Weight-Activation Quantization" (per-token activation grid)
 
 Everything is fp64 except the integer decisions of the quantizer (the code and
 the zero point), which are taken in fp32 arithmetic: the paper does not fix the
