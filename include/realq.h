@@ -29,9 +29,20 @@
  *     leave every buffer untouched: REALQ_ERR_INVALID_ARG /
  *     REALQ_ERR_WORKSPACE / REALQ_ERR_UNSUPPORTED.  realq_last_error() gives a
  *     thread-local description of the last failure.
- *   - No exception crosses the ABI.  The library keeps no per-call state
- *     besides the thread-local error string and the optional profiling
- *     counters.
+ *   - No exception crosses the ABI.  Besides the thread-local error string
+ *     and the optional profiling counters, the library keeps only reusable
+ *     helpers: for each (calling thread, caller's stream, its priority) a few
+ *     auxiliary streams and events, created on the first call that wants
+ *     them (prepare's triangular-inverse work and look-ahead, the sweep's
+ *     side product) and kept for the life of the thread.  Work on them forks
+ *     from the caller's stream and joins back into it inside the call, so
+ *     every call stays ordered on the caller's stream; make one call on a
+ *     stream before capturing that stream into a CUDA graph.  While
+ *     profiling is on they are not used.
+ *   - Device-side conditions (a non-positive pivot, a non-finite weight, a
+ *     bounded wait that gave up) are recorded in the workspace's status word
+ *     and read by the calls documented to synchronize (realq_hessian_prepare,
+ *     realq_prepare_status, realq_workspace_status).
  */
 #ifndef REALQ_H
 #define REALQ_H
