@@ -580,13 +580,6 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
     return check_launch("bgd_adam");
 }
 
-// One Block-GD step on columns c0..n-1 on the tensor cores (identity form):
-// P^T planes from the displacement planes and H̄ planes, then G = F_eff P with
-// the optimizer step fused into the epilogue.
-// One optimizer step on the free columns [c0, n).  The first product brings
-// M = A H̄ up to date for them: the last step moved A only in its own free
-// columns [step_c, n), so M[:, c0:] += step[:, step_c:] H̄[step_c:, c0:]
-// (K = n - step_c instead of n), then the epilogue forms P from M.
 // G = F_eff P on the free columns c0.. and one Adam step on them.  On the
 // last step of a block the next block's columns (c0 .. c0 + B) run first, K
 // split into slices whose fixed-order sum takes the step, and the rest (fused
@@ -682,6 +675,12 @@ realq_status_t sweep_side_stream(cudaStream_t s, SweepPlan &p) {
     return REALQ_OK;
 }
 
+// One Block-GD step on the free columns [c0, n) on the tensor cores
+// (identity form).  The first product brings M = A H̄ up to date for them:
+// the last step moved A only in its own free columns [step_c, n), so
+// M[:, c0:] += step[:, step_c:] H̄[step_c:, c0:] (K = n - step_c instead of
+// n), and its epilogue forms P from M and writes Pᵀ's tf32 planes; then
+// G = F_eff P with the optimizer step (g_adam).
 static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0, bool last) {
     const int64_t r = p.n - c0;
     const int64_t k0 = p.step_c;
