@@ -10,7 +10,9 @@
 // Both factorizations are blocked with 64-wide blocks: a one-CTA kernel
 // factors / inverts the diagonal block in shared memory, the off-diagonal work
 // runs as fp32 GEMMs.  A pivot that is not positive (or not finite) records its
-// column in the workspace status word; the host reads it once at the end.
+// column in the workspace status word; prepare reads it once at the end, the
+// deferred variant leaves it for realq_prepare_status (a captured step reads
+// no host memory).
 #include "kernels.cuh"
 
 #include <mutex>
