@@ -28,7 +28,11 @@
 //             H̄_g:  p = M + lambda_g (A_disp - (W - W0)) - acc (+ W0 Dbar),
 //             acc = ΔW (H̄_g - H̄); written like TC_BGD_P
 // The A operand starts at row a_row0 of its planes (a row group), and the
-// epilogue pointers are offset to that row by the caller.
+// epilogue pointers are offset to that row by the caller.  The epilogue is a
+// template parameter (one kernel per mode).  With TC_STORE, K may be split
+// over grid z (slice z writes its partial tile at C + z czs; a separate
+// pass sums the slices in order), and an operand exact in tf32 (a bf16 input
+// widened to fp32) skips its low plane: neither loaded nor multiplied.
 #include "kernels.cuh"
 #include "tc.cuh"
 
