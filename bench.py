@@ -322,7 +322,9 @@ def gpu_arm(args, wl, rank, world):
                        "l2": "inputs larger than L2: %.2f GB of calibration activations streamed per step" %
                              (sum(s.T * s.n * 2 for s in wl.inputs.values()) / 1e9),
                        "input_generation_s": round(t_gen, 1)},
-            "roofline": roof, "kernels": {k: {"launches": v[0], "ms": round(v[1], 3)} for k, v in
+            "roofline": roof,
+            "roofline_by_kernel": roofline_table(wl, prof, args.steps, peaks, args),
+            "kernels": {k: {"launches": v[0], "ms": round(v[1], 3)} for k, v in
                                            sorted(prof.items(), key=lambda kv: -kv[1][1])},
             "gpu_launches": int(launches), "clocks": clk, "e2e": e2e,
         }
@@ -331,11 +333,8 @@ def gpu_arm(args, wl, rank, world):
     return result
 
 
-def roofline(wl, prof, steps, peaks, args=None):
-    """Roofline entry for the kernel with the largest share of device time."""
-    if not prof:
-        return None
-    name, (launches, ms) = max(prof.items(), key=lambda kv: kv[1][1])
+def work_models(wl, args=None):
+    """Algorithmic work per step of each kernel family: (bound, work, unit)."""
     per_step = {}
     # algorithmic work per step of each kernel family
     hess_flops = sum(s.T * s.n * (s.n + 1) for s in wl.inputs.values())       # symmetric X^T X
@@ -395,6 +394,11 @@ def roofline(wl, prof, steps, peaks, args=None):
     per_step["chol_diag"] = ("alu", sum(s.n * 64 * 64 for s in wl.inputs.values()), "TFLOP/s")
     per_step["trtri_trmm"] = ("alu", prep_flops // 2, "TFLOP/s")
     per_step["chol_update"] = ("alu", prep_flops // 2, "TFLOP/s")
+    return per_step
+
+
+def roofline_entry(wl, name, launches, ms, steps, peaks, per_step):
+    """Achieved against peak for one kernel family from its summed event time."""
     if name not in per_step:
         return {"kernel": name, "bound": None, "achieved": None, "peak": None, "unit": None, "frac": None,
                 "traffic": None, "note": "no algorithmic model for this kernel"}
@@ -426,6 +430,28 @@ def roofline(wl, prof, steps, peaks, args=None):
             "frac": achieved / peak, "traffic": traffic, "peak_source": peak_note,
             "launches": launches, "avg_launch_ms": ms / launches,
             "work_per_step": work}
+
+
+def roofline(wl, prof, steps, peaks, args=None):
+    """Roofline entry for the kernel with the largest share of device time."""
+    if not prof:
+        return None
+    name, (launches, ms) = max(prof.items(), key=lambda kv: kv[1][1])
+    return roofline_entry(wl, name, launches, ms, steps, peaks, work_models(wl, args))
+
+
+def roofline_table(wl, prof, steps, peaks, args=None, top=8):
+    """The same entry for every kernel family with a work model, by device time."""
+    if not prof:
+        return []
+    models = work_models(wl, args)
+    rows = sorted(((n, v) for n, v in prof.items() if n in models and v[1] > 0 and v[0] > 0),
+                  key=lambda kv: -kv[1][1])[:top]
+    out = []
+    for n, (launches, ms) in rows:
+        e = roofline_entry(wl, n, launches, ms, steps, peaks, models)
+        out.append({k: e[k] for k in ("kernel", "bound", "achieved", "peak", "unit", "frac")})
+    return out
 
 
 # --------------------------------------------------------------------------
