@@ -1,0 +1,192 @@
+"""fp64 statement of one synthetic decoder block and of the exact two-block
+sliding-window loss (test infrastructure only; no CUDA counterpart yet).
+
+Sec. 4.4, Eq. (slide_window): while quantizing block l the surrogate blends
+this block's Fisher loss with the next block's, L = alpha L(l) + (1 - alpha)
+L(l+1), and the gradient of L(l+1) is taken by back-propagating from the
+output of block l+1 into block l.  The layer-level sweep replaces L(l+1) by
+a linearised pull-back F' of the next block's Fisher; this module states the
+exact form for the module whose output is block l's residual increment
+(down_proj: h = r + W x, so the block output's perturbation is
+Δh_t = (Ŵ - W0) x_t exactly).
+
+Readings (the paper names the modules q, k, v, o, gate, up, down and a SwiGLU
+MLP, Sec. 3.1 and App. "cosine alignment"; the rest is the common structure
+of the LLaMA-3.1 and Qwen3 blocks it evaluates):
+  pre-norm block   a = RMSNorm(x; g1),  h = x + Attn(a),
+                   b = RMSNorm(h; g2),  y = h + W_d (silu(W_g b) * (W_u b))
+  RMSNorm          x / sqrt(mean(x^2) + eps) * g, eps = 1e-6
+  attention        H query heads of width dh, H_kv key/value heads (query
+                   head i reads key/value head i // (H / H_kv)), rotary
+                   position embedding on q and k (pairs (j, j + dh/2), angle
+                   pos * base^(-2j/dh), base 10000), causal softmax over each
+                   sequence with scale 1/sqrt(dh), output projection W_o
+  tokens           S sequences of L tokens, (S, L, d); the Fisher losses
+                   average over the S L tokens.
+The backward pass is written out by hand (no autograd) and pinned by central
+finite differences.
+"""
+from __future__ import annotations
+
+from typing import Dict, Tuple
+
+import numpy as np
+
+__all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down"]
+
+EPS = 1e-6
+
+
+def block_params(rng: np.random.Generator, d: int, n_heads: int, n_kv: int, dh: int, f: int,
+                 scale: float = 0.2) -> Dict[str, np.ndarray]:
+    """Random fp64 parameters of one block (weights ~ N(0, scale^2 / fan_in))."""
+    def w(rows, cols):
+        return rng.standard_normal((rows, cols)) * scale / np.sqrt(cols)
+    return {"g1": 1.0 + 0.1 * rng.standard_normal(d), "Wq": w(n_heads * dh, d), "Wk": w(n_kv * dh, d),
+            "Wv": w(n_kv * dh, d), "Wo": w(d, n_heads * dh), "g2": 1.0 + 0.1 * rng.standard_normal(d),
+            "Wg": w(f, d), "Wu": w(f, d), "Wd": w(d, f), "n_heads": n_heads, "n_kv": n_kv, "dh": dh}
+
+
+def _rms(x, g):
+    r = 1.0 / np.sqrt(np.mean(x * x, axis=-1, keepdims=True) + EPS)
+    return x * r * g, r
+
+
+def _rms_vjp(x, g, r, gy):
+    # y = x r g, r = (mean(x^2) + eps)^-1/2;  dr/dx = -r^3 x / d
+    d = x.shape[-1]
+    gxr = gy * g
+    return gxr * r - x * (r ** 3) * np.sum(gxr * x, axis=-1, keepdims=True) / d, np.sum(gy * x * r, axis=(0, 1))
+
+
+def _rope_tables(L, dh, base=10000.0):
+    half = dh // 2
+    inv = base ** (-np.arange(half) * 2.0 / dh)
+    ang = np.arange(L)[:, None] * inv[None, :]
+    return np.cos(ang), np.sin(ang)
+
+
+def _rope(x, cos, sin):
+    # x: (S, L, heads, dh); pairs (j, j + dh/2) rotated by the position's angle
+    half = x.shape[-1] // 2
+    x1, x2 = x[..., :half], x[..., half:]
+    c, s = cos[None, :, None, :], sin[None, :, None, :]
+    return np.concatenate([x1 * c - x2 * s, x1 * s + x2 * c], axis=-1)
+
+
+def _rope_t(gy, cos, sin):
+    # the transpose (inverse) rotation
+    half = gy.shape[-1] // 2
+    g1, g2 = gy[..., :half], gy[..., half:]
+    c, s = cos[None, :, None, :], sin[None, :, None, :]
+    return np.concatenate([g1 * c + g2 * s, -g1 * s + g2 * c], axis=-1)
+
+
+def _silu(z):
+    return z / (1.0 + np.exp(-z))
+
+
+def block_forward(x: np.ndarray, P: Dict) -> Tuple[np.ndarray, Dict]:
+    """y = block(x) for x of shape (S, L, d); returns (y, cache for block_vjp)."""
+    S, L, d = x.shape
+    H, Hkv, dh = P["n_heads"], P["n_kv"], P["dh"]
+    rep = H // Hkv
+    a, r1 = _rms(x, P["g1"])
+    q = (a @ P["Wq"].T).reshape(S, L, H, dh)
+    k = (a @ P["Wk"].T).reshape(S, L, Hkv, dh)
+    v = (a @ P["Wv"].T).reshape(S, L, Hkv, dh)
+    cos, sin = _rope_tables(L, dh)
+    qr, kr = _rope(q, cos, sin), _rope(k, cos, sin)
+    kr_h = np.repeat(kr, rep, axis=2)                      # (S, L, H, dh)
+    v_h = np.repeat(v, rep, axis=2)
+    sc = np.einsum("sthe,suhe->shtu", qr, kr_h) / np.sqrt(dh)
+    mask = np.triu(np.ones((L, L), dtype=bool), 1)
+    sc = np.where(mask[None, None], -np.inf, sc)
+    sc = sc - sc.max(axis=-1, keepdims=True)
+    p = np.exp(sc)
+    p = p / p.sum(axis=-1, keepdims=True)                  # (S, H, L, L)
+    o = np.einsum("shtu,suhe->sthe", p, v_h).reshape(S, L, H * dh)
+    h = x + o @ P["Wo"].T
+    b, r2 = _rms(h, P["g2"])
+    zg, zu = b @ P["Wg"].T, b @ P["Wu"].T
+    m = _silu(zg) * zu
+    y = h + m @ P["Wd"].T
+    cache = dict(x=x, a=a, r1=r1, q=q, k=k, v=v, qr=qr, kr_h=kr_h, v_h=v_h, p=p, o=o, h=h, b=b, r2=r2, zg=zg,
+                 zu=zu, m=m, cos=cos, sin=sin, P=P)
+    return y, cache
+
+
+def block_vjp(cache: Dict, gy: np.ndarray) -> Tuple[np.ndarray, Dict[str, np.ndarray]]:
+    """(dL/dx, {dL/dparam}) for an upstream gradient gy = dL/dy."""
+    P = cache["P"]
+    S, L, d = cache["x"].shape
+    H, Hkv, dh = P["n_heads"], P["n_kv"], P["dh"]
+    rep = H // Hkv
+    g = {}
+    # MLP: y = h + m Wd^T, m = silu(zg) * zu
+    g["Wd"] = np.einsum("sti,stj->ij", gy, cache["m"])
+    gm = gy @ P["Wd"]
+    zg, zu = cache["zg"], cache["zu"]
+    sg = 1.0 / (1.0 + np.exp(-zg))
+    gzu = gm * _silu(zg)
+    gzg = gm * zu * (sg * (1.0 + zg * (1.0 - sg)))
+    g["Wg"] = np.einsum("sti,stj->ij", gzg, cache["b"])
+    g["Wu"] = np.einsum("sti,stj->ij", gzu, cache["b"])
+    gb = gzg @ P["Wg"] + gzu @ P["Wu"]
+    gh_n, g["g2"] = _rms_vjp(cache["h"], P["g2"], cache["r2"], gb)
+    gh = gy + gh_n
+    # attention: h = x + o Wo^T
+    g["Wo"] = np.einsum("sti,stj->ij", gh, cache["o"])
+    go = (gh @ P["Wo"]).reshape(S, L, H, dh)
+    p, v_h = cache["p"], cache["v_h"]
+    gp = np.einsum("sthe,suhe->shtu", go, v_h)
+    gv_h = np.einsum("shtu,sthe->suhe", p, go)
+    gsc = p * (gp - np.sum(gp * p, axis=-1, keepdims=True)) / np.sqrt(dh)
+    gqr = np.einsum("shtu,suhe->sthe", gsc, cache["kr_h"])
+    gkr_h = np.einsum("shtu,sthe->suhe", gsc, cache["qr"])
+    gkr = gkr_h.reshape(S, L, Hkv, rep, dh).sum(axis=3)
+    gv = gv_h.reshape(S, L, Hkv, rep, dh).sum(axis=3)
+    gq = _rope_t(gqr, cache["cos"], cache["sin"]).reshape(S, L, H * dh)
+    gk = _rope_t(gkr, cache["cos"], cache["sin"]).reshape(S, L, Hkv * dh)
+    gv = gv.reshape(S, L, Hkv * dh)
+    a = cache["a"]
+    g["Wq"] = np.einsum("sti,stj->ij", gq, a)
+    g["Wk"] = np.einsum("sti,stj->ij", gk, a)
+    g["Wv"] = np.einsum("sti,stj->ij", gv, a)
+    ga = gq @ P["Wq"] + gk @ P["Wk"] + gv @ P["Wv"]
+    gx_n, g["g1"] = _rms_vjp(cache["x"], P["g1"], cache["r1"], ga)
+    return gh + gx_n, g
+
+
+def next_block_loss(h: np.ndarray, dh_: np.ndarray, P_next: Dict, F_next: np.ndarray):
+    """L(l+1) = (1/2T) sum_t Δz_t^T F Δz_t with Δz = B(h + Δh) - B(h), and its
+    gradient with respect to Δh (T = S L tokens)."""
+    z0, _ = block_forward(h, P_next)
+    z1, cache = block_forward(h + dh_, P_next)
+    dz = z1 - z0
+    T = h.shape[0] * h.shape[1]
+    w = dz @ F_next
+    loss = 0.5 * float(np.sum(w * dz)) / T
+    g, _ = block_vjp(cache, w / T)
+    return loss, g
+
+
+def sliding_window_down(W: np.ndarray, W0: np.ndarray, X: np.ndarray, R: np.ndarray, alpha: float,
+                        F_this: np.ndarray, F_next: np.ndarray, P_next: Dict):
+    """The exact two-block sliding-window loss of a down_proj-type module and
+    its gradient with respect to W (d x n).
+
+    X: the module's inputs (S, L, n); R: block l's output without this
+    module's contribution (S, L, d), so h = R + X W0^T is the reference output
+    and R + X W^T the current one.  Block l's own Fisher loss is exact at the
+    module level here: Δh_t = (W - W0) x_t."""
+    S, L, n = X.shape
+    T = S * L
+    dW = np.asarray(W, dtype=np.float64) - np.asarray(W0, dtype=np.float64)
+    dh_ = X @ dW.T
+    h = R + X @ np.asarray(W0, dtype=np.float64).T
+    l_this = 0.5 * float(np.sum((dh_ @ F_this) * dh_)) / T
+    l_next, g_next = next_block_loss(h, dh_, P_next, F_next)
+    g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next
+    grad = np.einsum("sti,stj->ij", g_h, X)
+    return alpha * l_this + (1.0 - alpha) * l_next, grad

@@ -1,0 +1,130 @@
+"""Pins of the fp64 decoder block and of the exact two-block sliding window
+(oracle/block.py): central finite differences of every hand-written
+derivative, structural invariants of the attention, and the reduction of the
+exact window to the layer-level one when the next block is the identity."""
+import numpy as np
+import pytest
+
+import oracle
+from oracle import block as ob
+
+
+def _tiny(seed=0, d=16, H=4, Hkv=2, dh=4, f=24, S=2, L=5):
+    r = np.random.default_rng(seed)
+    P = ob.block_params(r, d, H, Hkv, dh, f, scale=0.8)
+    x = r.standard_normal((S, L, d))
+    return r, P, x
+
+
+def test_block_vjp_matches_finite_differences():
+    r, P, x = _tiny(1)
+    y, cache = ob.block_forward(x, P)
+    c = r.standard_normal(y.shape)
+    gx, gp = ob.block_vjp(cache, c)
+
+    def loss(xx, PP):
+        return float(np.sum(ob.block_forward(xx, PP)[0] * c))
+
+    h = 1e-6
+    for idx in [(0, 0, 0), (1, 4, 7), (0, 2, 15), (1, 0, 3)]:
+        e = np.zeros_like(x)
+        e[idx] = h
+        fd = (loss(x + e, P) - loss(x - e, P)) / (2 * h)
+        assert abs(fd - gx[idx]) <= 1e-6 * max(1.0, abs(fd)), (idx, fd, gx[idx])
+    for name in ("Wq", "Wk", "Wv", "Wo", "Wg", "Wu", "Wd", "g1", "g2"):
+        for k in range(3):
+            idx = tuple(int(r.integers(0, s)) for s in P[name].shape)
+            Pp = dict(P)
+            Pm = dict(P)
+            Pp[name] = P[name].copy()
+            Pm[name] = P[name].copy()
+            Pp[name][idx] += h
+            Pm[name][idx] -= h
+            fd = (loss(x, Pp) - loss(x, Pm)) / (2 * h)
+            assert abs(fd - gp[name][idx]) <= 1e-6 * max(1.0, abs(fd)), (name, idx, fd, gp[name][idx])
+
+
+def test_attention_is_causal_within_each_sequence():
+    r, P, x = _tiny(2)
+    y0, _ = ob.block_forward(x, P)
+    x1 = x.copy()
+    x1[1, 2] += r.standard_normal(x.shape[2])
+    y1, _ = ob.block_forward(x1, P)
+    changed = np.abs(y1 - y0).max(axis=2) > 0
+    assert not changed[0].any()                      # the other sequence
+    assert not changed[1, :2].any()                  # earlier positions
+    assert changed[1, 2:].all()                      # the token and every later one
+
+
+def test_rotary_scores_depend_on_the_position_difference():
+    r = np.random.default_rng(3)
+    dh, L = 8, 12
+    q = r.standard_normal((1, L, 1, dh))
+    k = r.standard_normal((1, L, 1, dh))
+    cos, sin = ob._rope_tables(L, dh)
+    # the same two vectors placed at (i, j) and at (i + 4, j + 4)
+    qs = np.repeat(q[:, :1], L, axis=1)
+    ks = np.repeat(k[:, :1], L, axis=1)
+    qr, kr = ob._rope(qs, cos, sin), ob._rope(ks, cos, sin)
+    s1 = float(np.sum(qr[0, 5, 0] * kr[0, 2, 0]))
+    s2 = float(np.sum(qr[0, 9, 0] * kr[0, 6, 0]))
+    assert abs(s1 - s2) <= 1e-12 * max(1.0, abs(s1))
+    # and the rotation is orthogonal (its transpose undoes it)
+    assert np.allclose(ob._rope_t(ob._rope(q, cos, sin), cos, sin), q, atol=1e-14)
+
+
+def _down_case(seed, zero_next):
+    r = np.random.default_rng(seed)
+    S, L, n, d = 2, 6, 12, 16
+    P = ob.block_params(r, d, 4, 2, 4, 24, scale=0.8)
+    if zero_next:
+        P["Wo"] = np.zeros_like(P["Wo"])
+        P["Wd"] = np.zeros_like(P["Wd"])
+    X = r.standard_normal((S, L, n))
+    R = r.standard_normal((S, L, d))
+    W0 = r.standard_normal((d, n)) * 0.1
+    W = W0 + r.standard_normal((d, n)) * 0.02
+    Z = r.standard_normal((d, 3))
+    F = 0.5 * np.eye(d) + Z @ Z.T / 6
+    Z2 = r.standard_normal((d, 3))
+    Fn = 0.5 * np.eye(d) + Z2 @ Z2.T / 6
+    return X, R, W0, W, F, Fn, P
+
+
+def test_identity_next_block_reduces_to_the_layer_level_window():
+    # with its output projections zero the next block is the identity, so its
+    # Fisher loss is the layer-level one with F' = F_next
+    X, R, W0, W, F, Fn, P = _down_case(4, True)
+    alpha = 0.3
+    loss, grad = ob.sliding_window_down(W, W0, X, R, alpha, F, Fn, P)
+    Xf = X.reshape(-1, X.shape[2])
+    Hbar = Xf.T @ Xf / Xf.shape[0]
+    Feff = alpha * F + (1 - alpha) * Fn
+    np.testing.assert_allclose(grad, oracle.gradient(W, W0, Hbar, None, Feff), rtol=1e-11, atol=1e-14)
+    assert abs(loss - oracle.surrogate_moment(W, W0, Hbar, Feff)) <= 1e-12 * abs(loss)
+
+
+@pytest.mark.parametrize("alpha", [1.0, 0.4, 0.0])
+def test_sliding_window_gradient_matches_finite_differences(alpha):
+    X, R, W0, W, F, Fn, P = _down_case(5, False)
+    _, grad = ob.sliding_window_down(W, W0, X, R, alpha, F, Fn, P)
+    h = 1e-6
+    r = np.random.default_rng(6)
+    for _ in range(6):
+        i, j = int(r.integers(0, W.shape[0])), int(r.integers(0, W.shape[1]))
+        E = np.zeros_like(W)
+        E[i, j] = h
+        lp, _ = ob.sliding_window_down(W + E, W0, X, R, alpha, F, Fn, P)
+        lm, _ = ob.sliding_window_down(W - E, W0, X, R, alpha, F, Fn, P)
+        fd = (lp - lm) / (2 * h)
+        assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-3, abs(fd)), (i, j, fd, grad[i, j])
+
+
+def test_next_block_loss_is_second_order_in_the_perturbation():
+    # B(h + e u) - B(h) = e J u + O(e^2): the loss scales as e^2 for small e
+    X, R, W0, W, F, Fn, P = _down_case(7, False)
+    h = R + X @ W0.T
+    u = np.random.default_rng(8).standard_normal(h.shape)
+    l1, _ = ob.next_block_loss(h, 1e-3 * u, P, Fn)
+    l2, _ = ob.next_block_loss(h, 2e-3 * u, P, Fn)
+    assert abs(l2 / l1 - 4.0) < 1e-2

@@ -57,15 +57,30 @@ MUTATIONS = {
 }
 
 
-def _pins_on_copy(tmp_path, old=None, new=None):
+# the decoder block of the exact sliding window (oracle/block.py)
+BLOCK_MUTATIONS = {
+    "silu_derivative": ("gzg = gm * zu * (sg * (1.0 + zg * (1.0 - sg)))", "gzg = gm * zu * sg"),
+    "softmax_backward": ("gsc = p * (gp - np.sum(gp * p, axis=-1, keepdims=True)) / np.sqrt(dh)",
+                         "gsc = p * gp / np.sqrt(dh)"),
+    "rope_transpose": ("return np.concatenate([g1 * c + g2 * s, -g1 * s + g2 * c], axis=-1)",
+                       "return np.concatenate([g1 * c - g2 * s, g1 * s + g2 * c], axis=-1)"),
+    "rms_backward": ("return gxr * r - x * (r ** 3) * np.sum(gxr * x, axis=-1, keepdims=True) / d,",
+                     "return gxr * r,"),
+    "causal_mask": ("mask = np.triu(np.ones((L, L), dtype=bool), 1)", "mask = np.zeros((L, L), dtype=bool)"),
+    "window_blend": ("g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next",
+                     "g_h = alpha * (dh_ @ F_this) / T + alpha * g_next"),
+}
+
+
+def _pins_on_copy(tmp_path, old=None, new=None, target="realq.py", pins="tests/test_oracle_pins.py"):
     for d in ("oracle", "synth", "tests"):
         shutil.copytree(os.path.join(ROOT, d), tmp_path / d, ignore=shutil.ignore_patterns("__pycache__"))
     if old is not None:
-        src = (tmp_path / "oracle" / "realq.py").read_text()
+        src = (tmp_path / "oracle" / target).read_text()
         assert src.count(old) == 1, f"mutation anchor not found once: {old}"
-        (tmp_path / "oracle" / "realq.py").write_text(src.replace(old, new))
+        (tmp_path / "oracle" / target).write_text(src.replace(old, new))
     env = dict(os.environ, PYTHONPATH=str(tmp_path))
-    return subprocess.run([sys.executable, "-m", "pytest", "tests/test_oracle_pins.py", "-x", "-q", "-p",
+    return subprocess.run([sys.executable, "-m", "pytest", pins, "-x", "-q", "-p",
                            "no:cacheprovider", "-m", "not gpu"], cwd=tmp_path, env=env, capture_output=True,
                           text=True, timeout=600)
 
@@ -81,3 +96,16 @@ def test_pins_catch_the_mistake(name, tmp_path):
     r = _pins_on_copy(tmp_path, *MUTATIONS[name])
     assert r.returncode != 0, f"the pins did not catch '{name}':\n{r.stdout[-2000:]}"
     assert " failed" in r.stdout, r.stdout[-2000:]     # a failing pin, not a crash
+
+
+def test_unchanged_block_copy_passes(tmp_path):
+    r = _pins_on_copy(tmp_path, pins="tests/test_oracle_block_pins.py")
+    assert r.returncode == 0, r.stdout[-2000:]
+
+
+@pytest.mark.parametrize("name", sorted(BLOCK_MUTATIONS))
+def test_block_pins_catch_the_mistake(name, tmp_path):
+    old, new = BLOCK_MUTATIONS[name]
+    r = _pins_on_copy(tmp_path, old, new, target="block.py", pins="tests/test_oracle_block_pins.py")
+    assert r.returncode != 0, f"the pins did not catch '{name}':\n{r.stdout[-2000:]}"
+    assert " failed" in r.stdout, r.stdout[-2000:]
