@@ -6,8 +6,9 @@ this block's Fisher loss with the next block's, L = alpha L(l) + (1 - alpha)
 L(l+1), and the gradient of L(l+1) is taken by back-propagating from the
 output of block l+1 into block l.  The layer-level sweep replaces L(l+1) by
 a linearised pull-back F' of the next block's Fisher; this module states the
-exact form for the module whose output is block l's residual increment
-(down_proj: h = r + W x, so the block output's perturbation is
+exact form: for any linear module of block l (sliding_window_module, through
+block l's own backward), and the direct form for the module whose output is
+block l's residual increment (sliding_window_down: h = r + W x, so
 Δh_t = (Ŵ - W0) x_t exactly).
 
 Readings (the paper names the modules q, k, v, o, gate, up, down and a SwiGLU
@@ -32,7 +33,8 @@ from typing import Dict, Tuple
 
 import numpy as np
 
-__all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down"]
+__all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down",
+           "sliding_window_module"]
 
 EPS = 1e-6
 
@@ -190,3 +192,32 @@ def sliding_window_down(W: np.ndarray, W0: np.ndarray, X: np.ndarray, R: np.ndar
     g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next
     grad = np.einsum("sti,stj->ij", g_h, X)
     return alpha * l_this + (1.0 - alpha) * l_next, grad
+
+
+_MODULE_WEIGHT = {"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg",
+                  "up_proj": "Wu", "down_proj": "Wd"}
+
+
+def sliding_window_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, P_next: Dict, alpha: float,
+                          F_this: np.ndarray, F_next: np.ndarray):
+    """The exact two-block sliding-window loss of any linear module of block l
+    and its gradient with respect to that module's weight.
+
+    x: block l's input (S, L, d); P_this: block l with its reference (full
+    precision) weights; W replaces the module's weight.  Block l's output is
+    h = B_l(x; W) and its reference h* = B_l(x; W0); the loss is
+      alpha (1/2T) sum_t Δh_t^T F_this Δh_t
+        + (1 - alpha) (1/2T) sum_t (B_{l+1}(h)_t - B_{l+1}(h*)_t)^T F_next (...),
+    Δh = h - h*, both terms back-propagated through block l to W."""
+    name = _MODULE_WEIGHT[module]
+    P_cur = dict(P_this)
+    P_cur[name] = np.asarray(W, dtype=np.float64)
+    h_ref, _ = block_forward(x, P_this)
+    h, cache = block_forward(x, P_cur)
+    dh_ = h - h_ref
+    T = x.shape[0] * x.shape[1]
+    l_this = 0.5 * float(np.sum((dh_ @ F_this) * dh_)) / T
+    l_next, g_next = next_block_loss(h_ref, dh_, P_next, F_next)
+    g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next
+    _, grads = block_vjp(cache, g_h)
+    return alpha * l_this + (1.0 - alpha) * l_next, grads[name]

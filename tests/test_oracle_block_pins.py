@@ -128,3 +128,48 @@ def test_next_block_loss_is_second_order_in_the_perturbation():
     l1, _ = ob.next_block_loss(h, 1e-3 * u, P, Fn)
     l2, _ = ob.next_block_loss(h, 2e-3 * u, P, Fn)
     assert abs(l2 / l1 - 4.0) < 1e-2
+
+
+def _module_case(seed):
+    r = np.random.default_rng(seed)
+    d = 16
+    P = ob.block_params(r, d, 4, 2, 4, 24, scale=0.8)
+    Pn = ob.block_params(r, d, 4, 2, 4, 24, scale=0.8)
+    x = r.standard_normal((2, 5, d))
+    Z = r.standard_normal((d, 3))
+    F = 0.5 * np.eye(d) + Z @ Z.T / 6
+    Z2 = r.standard_normal((d, 3))
+    Fn = 0.5 * np.eye(d) + Z2 @ Z2.T / 6
+    return r, P, Pn, x, F, Fn
+
+
+@pytest.mark.parametrize("module", ["q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj"])
+def test_every_module_window_gradient_matches_finite_differences(module):
+    r, P, Pn, x, F, Fn = _module_case(9)
+    name = ob._MODULE_WEIGHT[module]
+    W = P[name] + r.standard_normal(P[name].shape) * 0.05
+    loss, grad = ob.sliding_window_module(module, W, x, P, Pn, 0.6, F, Fn)
+    assert loss > 0
+    h = 1e-6
+    for _ in range(4):
+        i, j = int(r.integers(0, W.shape[0])), int(r.integers(0, W.shape[1]))
+        E = np.zeros_like(W)
+        E[i, j] = h
+        lp, _ = ob.sliding_window_module(module, W + E, x, P, Pn, 0.6, F, Fn)
+        lm, _ = ob.sliding_window_module(module, W - E, x, P, Pn, 0.6, F, Fn)
+        fd = (lp - lm) / (2 * h)
+        assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-3, abs(fd)), (module, i, j, fd, grad[i, j])
+
+
+def test_module_window_agrees_with_the_down_proj_form():
+    # for down_proj the block-level statement equals the module-level one
+    # (h = r + W_d m, with m the SwiGLU product and r the rest of the block)
+    r, P, Pn, x, F, Fn = _module_case(10)
+    W = P["Wd"] + r.standard_normal(P["Wd"].shape) * 0.05
+    loss, grad = ob.sliding_window_module("down_proj", W, x, P, Pn, 0.35, F, Fn)
+    y, cache = ob.block_forward(x, P)
+    m = cache["m"]
+    R = y - m @ P["Wd"].T
+    loss2, grad2 = ob.sliding_window_down(W, P["Wd"], m, R, 0.35, F, Fn, Pn)
+    assert abs(loss - loss2) <= 1e-12 * abs(loss)
+    np.testing.assert_allclose(grad, grad2, rtol=1e-10, atol=1e-15)
