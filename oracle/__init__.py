@@ -13,8 +13,9 @@ realq.py   the sweep in the paper's order and notation, fp64 throughout except
            the zero point), which is taken in fp32 on both sides.
 brute.c    exhaustive search over all int4 codes of a tiny layer (the
            brute-force pin of the quantizer + surrogate), built by build.py.
-block.py   one synthetic decoder block in fp64 with its backward, and the
-           exact two-block sliding-window loss (Sec. 4.4) of a down_proj-type
-           module; imported as ``oracle.block``.
+block.py   one synthetic decoder block in fp64 with its backward, the
+           exact two-block sliding-window loss (Sec. 4.4) of any linear
+           module of the block, and the final block's true KL at the LM head
+           with the Fisher of Eq. (fisher_full); imported as ``oracle.block``.
 """
 from .realq import *  # noqa: F401,F403

@@ -26,6 +26,19 @@ of the LLaMA-3.1 and Qwen3 blocks it evaluates):
                    average over the S L tokens.
 The backward pass is written out by hand (no autograd) and pinned by central
 finite differences.
+
+The final block has no next block: it takes the true KL against the LM head
+(Eq. kl_loss; App. "Pre-computation of the aggregated Fisher and
+last-transformer-block handling").  Readings for that part:
+  head             z = RMSNorm(h; g_f) W_h^T (a final norm, then the head,
+                   as in the evaluated model families), V logits per token
+  KL               (1/T) sum_t KL(p_t || q_t), p_t = softmax of the reference
+                   logits, q_t = softmax of the perturbed ones (Eq. kl_loss's
+                   direction: full precision first)
+  Fisher           Eq. fisher_full with g_t the gradient of the NLL of a label
+                   drawn from p_t (the draw is an input, fisher_sampled); its
+                   exact expectation over the label is fisher_tokens, which is
+                   the per-token Hessian H_t of Eq. taylor_expansion.
 """
 from __future__ import annotations
 
@@ -34,7 +47,8 @@ from typing import Dict, Tuple
 import numpy as np
 
 __all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down",
-           "sliding_window_module"]
+           "sliding_window_module", "head_params", "head_logits", "kl_logits", "kl_head_loss", "nll_scores",
+           "fisher_sampled", "fisher_tokens", "kl_final_module"]
 
 EPS = 1e-6
 
@@ -221,3 +235,93 @@ def sliding_window_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dic
     g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next
     _, grads = block_vjp(cache, g_h)
     return alpha * l_this + (1.0 - alpha) * l_next, grads[name]
+
+
+# ---------------------------------------------------------------------------
+# The final block: the true KL divergence against the LM head.
+
+
+def head_params(rng: np.random.Generator, d: int, V: int, scale: float = 1.0) -> Dict[str, np.ndarray]:
+    """Random fp64 final norm and LM head (W_h ~ N(0, scale^2 / d), V x d)."""
+    return {"gf": 1.0 + 0.1 * rng.standard_normal(d), "Wh": rng.standard_normal((V, d)) * scale / np.sqrt(d)}
+
+
+def head_logits(h: np.ndarray, head: Dict):
+    """z = RMSNorm(h; g_f) W_h^T for h of shape (S, L, d); returns (z, cache)."""
+    u, r = _rms(h, head["gf"])
+    return u @ head["Wh"].T, (h, r)
+
+
+def _head_vjp(hc, head, gz):
+    h, r = hc
+    gh, _ = _rms_vjp(h, head["gf"], r, gz @ head["Wh"])
+    return gh
+
+
+def _log_softmax(z):
+    z = z - z.max(axis=-1, keepdims=True)
+    return z - np.log(np.sum(np.exp(z), axis=-1, keepdims=True))
+
+
+def kl_logits(z_ref: np.ndarray, z: np.ndarray) -> np.ndarray:
+    """KL(softmax(z_ref) || softmax(z)) over the last axis, one value per token."""
+    lp, lq = _log_softmax(z_ref), _log_softmax(z)
+    return np.sum(np.exp(lp) * (lp - lq), axis=-1)
+
+
+def kl_head_loss(h_ref: np.ndarray, dh_: np.ndarray, head: Dict):
+    """L = (1/T) sum_t KL(p_t || q_t) with p from the reference block output
+    h* and q from h* + Δh, and its gradient with respect to Δh.  The gradient
+    of KL(p || softmax(z)) in z is softmax(z) - p."""
+    z0, _ = head_logits(h_ref, head)
+    z1, hc = head_logits(h_ref + dh_, head)
+    T = h_ref.shape[0] * h_ref.shape[1]
+    loss = float(np.sum(kl_logits(z0, z1))) / T
+    gz = (np.exp(_log_softmax(z1)) - np.exp(_log_softmax(z0))) / T
+    return loss, _head_vjp(hc, head, gz)
+
+
+def nll_scores(h_ref: np.ndarray, head: Dict, labels: np.ndarray) -> np.ndarray:
+    """g_t = the gradient in y_t of -log p(label_t | y_t) at the reference
+    output (S, L, d); labels (S, L) are integers in [0, V)."""
+    z, hc = head_logits(h_ref, head)
+    p = np.exp(_log_softmax(z))
+    onehot = np.zeros_like(p)
+    np.put_along_axis(onehot, np.asarray(labels)[..., None], 1.0, axis=-1)
+    return _head_vjp(hc, head, p - onehot)
+
+
+def fisher_sampled(h_ref: np.ndarray, head: Dict, labels: np.ndarray) -> np.ndarray:
+    """Eq. fisher_full: F = (1/T) sum_t g_t g_t^T with one label per token
+    drawn from the reference distribution p_t (the draw is passed in)."""
+    g = nll_scores(h_ref, head, labels)
+    g = g.reshape(-1, g.shape[-1])
+    return g.T @ g / g.shape[0]
+
+
+def fisher_tokens(h_ref: np.ndarray, head: Dict) -> np.ndarray:
+    """The per-token Fisher as the exact expectation over the label:
+    F_t = sum_v p_t(v) g_t(v) g_t(v)^T, shape (S, L, d, d).  Its token mean is
+    the expectation of fisher_sampled over the draw."""
+    z, _ = head_logits(h_ref, head)
+    p = np.exp(_log_softmax(z))
+    S, L, d = h_ref.shape
+    F = np.zeros((S, L, d, d))
+    for v in range(p.shape[-1]):
+        g = nll_scores(h_ref, head, np.full((S, L), v))
+        F += p[..., v, None, None] * g[..., :, None] * g[..., None, :]
+    return F
+
+
+def kl_final_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, head: Dict):
+    """The final block's loss for any linear module: the true KL at the LM
+    head between the reference block output and the one with W in place of
+    the module's weight, and its gradient with respect to W."""
+    name = _MODULE_WEIGHT[module]
+    P_cur = dict(P_this)
+    P_cur[name] = np.asarray(W, dtype=np.float64)
+    h_ref, _ = block_forward(x, P_this)
+    h, cache = block_forward(x, P_cur)
+    loss, g_h = kl_head_loss(h_ref, h - h_ref, head)
+    _, grads = block_vjp(cache, g_h)
+    return loss, grads[name]

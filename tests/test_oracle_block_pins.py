@@ -173,3 +173,114 @@ def test_module_window_agrees_with_the_down_proj_form():
     loss2, grad2 = ob.sliding_window_down(W, P["Wd"], m, R, 0.35, F, Fn, Pn)
     assert abs(loss - loss2) <= 1e-12 * abs(loss)
     np.testing.assert_allclose(grad, grad2, rtol=1e-10, atol=1e-15)
+
+
+# --- the final block: the true KL at the LM head ---------------------------
+
+def _head_case(seed, d=6, V=7, S=2, L=3):
+    r = np.random.default_rng(seed)
+    head = ob.head_params(r, d, V, scale=1.5)
+    h = r.standard_normal((S, L, d))
+    return r, head, h
+
+
+def test_kl_of_two_hand_computed_distributions():
+    # p = softmax(0, ln 3) = (1/4, 3/4), q = softmax(0, 0) = (1/2, 1/2)
+    z_ref = np.array([[0.0, np.log(3.0)]])
+    z = np.zeros((1, 2))
+    want = 0.25 * np.log(0.5) + 0.75 * np.log(1.5)
+    assert abs(ob.kl_logits(z_ref, z)[0] - want) <= 1e-15
+    # a constant shift of either side's logits changes neither distribution
+    assert abs(ob.kl_logits(z_ref + 7.0, z - 3.0)[0] - want) <= 1e-14
+    assert ob.kl_logits(z_ref, z_ref)[0] == 0.0
+
+
+def test_kl_head_loss_is_zero_with_a_zero_gradient_at_the_reference():
+    r, head, h = _head_case(11)
+    loss, g = ob.kl_head_loss(h, np.zeros_like(h), head)
+    assert loss == 0.0 and np.abs(g).max() == 0.0
+    loss, _ = ob.kl_head_loss(h, 0.3 * r.standard_normal(h.shape), head)
+    assert loss > 0.0
+
+
+def test_kl_head_gradient_matches_finite_differences():
+    r, head, h = _head_case(12)
+    dh0 = 0.4 * r.standard_normal(h.shape)
+    _, g = ob.kl_head_loss(h, dh0, head)
+    e = 1e-6
+    for idx in [(0, 0, 0), (1, 2, 5), (0, 1, 3), (1, 0, 1)]:
+        E = np.zeros_like(h)
+        E[idx] = e
+        fd = (ob.kl_head_loss(h, dh0 + E, head)[0] - ob.kl_head_loss(h, dh0 - E, head)[0]) / (2 * e)
+        assert abs(fd - g[idx]) <= 1e-7 * max(1e-3, abs(fd)), (idx, fd, g[idx])
+
+
+def test_fisher_is_the_kl_hessian_at_the_reference_output():
+    # at h* the first-order term of KL vanishes and its Hessian in y_t is the
+    # expected outer product of the NLL score (Eq. taylor_expansion and the
+    # Fisher-Hessian identity); per token, (1/T) F_t u_t is the derivative of
+    # the KL gradient along u
+    r, head, h = _head_case(13)
+    S, L, d = h.shape
+    F = ob.fisher_tokens(h, head)
+    u = r.standard_normal(h.shape)
+    e = 1e-5
+    gp = ob.kl_head_loss(h, e * u, head)[1]
+    gm = ob.kl_head_loss(h, -e * u, head)[1]
+    hv = (gp - gm) / (2 * e)
+    want = np.einsum("stij,stj->sti", F, u) / (S * L)
+    np.testing.assert_allclose(hv, want, rtol=1e-6, atol=1e-9 * np.abs(want).max())
+    # and the loss itself: KL(h* + e u) / e^2 -> (1/2T) sum_t u_t^T F_t u_t
+    quad = 0.5 * float(np.einsum("sti,stij,stj->", u, F, u)) / (S * L)
+    r1 = ob.kl_head_loss(h, 2e-3 * u, head)[0] / 4e-6
+    r2 = ob.kl_head_loss(h, 1e-3 * u, head)[0] / 1e-6
+    assert abs((2 * r2 - r1) - quad) <= 1e-5 * quad        # Richardson: O(e^2) left
+    # each F_t is symmetric positive semidefinite with the head's null
+    # direction: the score is orthogonal to h_t (RMSNorm is scale-free up to eps)
+    assert np.allclose(F, np.swapaxes(F, -1, -2), atol=1e-15)
+    assert np.linalg.eigvalsh(F).min() > -1e-12
+    assert np.abs(np.einsum("stij,stj->sti", F, h)).max() <= 1e-5 * np.abs(F).max() * np.abs(h).max()
+
+
+def test_sampled_fisher_averages_to_the_exact_expectation():
+    # Eq. fisher_full with labels drawn from p_t: its mean over many draws is
+    # the token mean of the per-token expectation (fixed seed: deterministic)
+    r, head, h = _head_case(14, d=4, V=5)
+    z, _ = ob.head_logits(h, head)
+    p = np.exp(z - z.max(axis=-1, keepdims=True))
+    p /= p.sum(axis=-1, keepdims=True)
+    want = ob.fisher_tokens(h, head).mean(axis=(0, 1))
+    K = 4000
+    cdf = np.cumsum(p, axis=-1)
+    draws = []
+    for _ in range(K):
+        lab = (r.random(p.shape[:-1])[..., None] > cdf).sum(axis=-1)
+        draws.append(ob.fisher_sampled(h, head, np.minimum(lab, p.shape[-1] - 1)))
+    draws = np.array(draws)
+    se = draws.std(axis=0) / np.sqrt(K)
+    assert np.all(np.abs(draws.mean(axis=0) - want) <= 5 * se + 1e-12)
+    # the test has the power to see a wrong expectation: labels drawn
+    # uniformly instead of from p_t fall outside the bound
+    V = p.shape[-1]
+    gs = [ob.nll_scores(h, head, np.full(h.shape[:2], v)) for v in range(V)]
+    uniform = sum(np.einsum("sti,stj->ij", g, g) for g in gs) / (V * h.shape[0] * h.shape[1])
+    assert not np.all(np.abs(draws.mean(axis=0) - uniform) <= 5 * se + 1e-12)
+
+
+@pytest.mark.parametrize("module", ["q_proj", "v_proj", "gate_proj", "down_proj"])
+def test_final_block_kl_gradient_matches_finite_differences(module):
+    r, P, _, x, _, _ = _module_case(15)
+    head = ob.head_params(r, x.shape[2], 11, scale=1.5)
+    name = ob._MODULE_WEIGHT[module]
+    l0, g0 = ob.kl_final_module(module, P[name], x, P, head)
+    assert l0 == 0.0 and np.abs(g0).max() == 0.0
+    W = P[name] + r.standard_normal(P[name].shape) * 0.05
+    loss, grad = ob.kl_final_module(module, W, x, P, head)
+    assert loss > 0
+    e = 1e-6
+    for _ in range(4):
+        i, j = int(r.integers(0, W.shape[0])), int(r.integers(0, W.shape[1]))
+        E = np.zeros_like(W)
+        E[i, j] = e
+        fd = (ob.kl_final_module(module, W + E, x, P, head)[0] - ob.kl_final_module(module, W - E, x, P, head)[0]) / (2 * e)
+        assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-4, abs(fd)), (module, i, j, fd, grad[i, j])

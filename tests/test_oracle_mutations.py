@@ -67,8 +67,21 @@ BLOCK_MUTATIONS = {
     "rms_backward": ("return gxr * r - x * (r ** 3) * np.sum(gxr * x, axis=-1, keepdims=True) / d,",
                      "return gxr * r,"),
     "causal_mask": ("mask = np.triu(np.ones((L, L), dtype=bool), 1)", "mask = np.zeros((L, L), dtype=bool)"),
-    "window_blend": ("g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next",
-                     "g_h = alpha * (dh_ @ F_this) / T + alpha * g_next"),
+    "window_blend": ("g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next\n    grad =",
+                     "g_h = alpha * (dh_ @ F_this) / T + alpha * g_next\n    grad ="),
+    # the module-level window with the current weights as its reference
+    "module_reference": ("h_ref, _ = block_forward(x, P_this)\n    h, cache = block_forward(x, P_cur)\n    dh_",
+                         "h_ref, _ = block_forward(x, P_cur)\n    h, cache = block_forward(x, P_cur)\n    dh_"),
+    # the KL head: the gradient's sign, the head's norm left out of the
+    # backward, the Fisher's label weights dropped, the KL's direction swapped
+    "kl_gradient_sign": ("gz = (np.exp(_log_softmax(z1)) - np.exp(_log_softmax(z0))) / T",
+                         "gz = (np.exp(_log_softmax(z0)) - np.exp(_log_softmax(z1))) / T"),
+    "head_norm_backward": ("gh, _ = _rms_vjp(h, head[\"gf\"], r, gz @ head[\"Wh\"])",
+                           "gh = (gz @ head[\"Wh\"]) * head[\"gf\"] * r"),
+    "fisher_weights": ("F += p[..., v, None, None] * g[..., :, None] * g[..., None, :]",
+                       "F += g[..., :, None] * g[..., None, :] / p.shape[-1]"),
+    "kl_direction": ("return np.sum(np.exp(lp) * (lp - lq), axis=-1)",
+                     "return np.sum(np.exp(lq) * (lq - lp), axis=-1)"),
 }
 
 
