@@ -48,7 +48,8 @@ import numpy as np
 
 __all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down",
            "sliding_window_module", "head_params", "head_logits", "kl_logits", "kl_head_loss", "nll_scores",
-           "fisher_sampled", "fisher_tokens", "kl_final_module"]
+           "fisher_sampled", "fisher_tokens", "kl_final_module", "module_inputs", "window_gradient_fn",
+           "kl_gradient_fn"]
 
 EPS = 1e-6
 
@@ -325,3 +326,35 @@ def kl_final_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, hea
     loss, g_h = kl_head_loss(h_ref, h - h_ref, head)
     _, grads = block_vjp(cache, g_h)
     return loss, grads[name]
+
+
+# ---------------------------------------------------------------------------
+# The sweep's Block-GD step on these losses (realq_sweep's gradient_fn).
+
+_MODULE_INPUT = {"q_proj": "a", "k_proj": "a", "v_proj": "a", "o_proj": "o", "gate_proj": "b", "up_proj": "b",
+                 "down_proj": "m"}
+
+
+def module_inputs(module: str, x: np.ndarray, P: Dict) -> np.ndarray:
+    """The inputs of a module of block l at its reference weights, as the
+    (S L) x n token matrix whose second moment is the module's OBS Hessian."""
+    _, cache = block_forward(x, P)
+    a = cache[_MODULE_INPUT[module]]
+    return a.reshape(-1, a.shape[-1])
+
+
+def window_gradient_fn(module: str, x: np.ndarray, P_this: Dict, P_next: Dict, F_this: np.ndarray,
+                       F_next: np.ndarray):
+    """(W, alpha) -> (loss, gradient) of the exact two-block window for the
+    Block-GD step of the module's sweep (alpha is the step's blend weight)."""
+    def fn(W, alpha):
+        return sliding_window_module(module, W, x, P_this, P_next, alpha, F_this, F_next)
+    return fn
+
+
+def kl_gradient_fn(module: str, x: np.ndarray, P_this: Dict, head: Dict):
+    """(W, alpha) -> (loss, gradient) of the final block's KL at the LM head
+    (no window: alpha is not used)."""
+    def fn(W, alpha):
+        return kl_final_module(module, W, x, P_this, head)
+    return fn

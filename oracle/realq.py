@@ -328,7 +328,14 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
       minibatch_tokens: a list of K token blocks X̂_k (T_k x n) with the same
       rotation, whose gradient is taken in token form, and then optionally
       a_loss_clip: the per-token output clipping percentile (0.95 in the
-      paper's small-model runs; see loss_clip_factors).
+      paper's small-model runs; see loss_clip_factors); or
+      gradient_fn: a callable (W, alpha) -> (loss, G) that gives the
+      surrogate and its gradient in W (m x n) at the current weights, in
+      place of the layer-level surrogate: the exact two-block window of
+      Sec. 4.4 and the final block's KL at the LM head (App. "Pre-computation
+      of the aggregated Fisher and last-transformer-block handling"), both
+      stated in oracle.block.  The per-block values it records are its own
+      loss before and after the block's steps.
 
     Readings: group parameters are computed at the first column of each group
     from the current (compensated, Block-GD-updated) weights; group_size 0
@@ -406,14 +413,21 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             b = j // B
             b_global = bgd.get("b_global_start", 1) + b
             alpha = sliding_alpha(b_global, bgd.get("B_total", 1))
-            Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
-            before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
+            gfn = bgd.get("gradient_fn")
+            if gfn is not None:
+                Feff = None
+                before = gfn(W, alpha)[0] if record else None
+            else:
+                Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
+                before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
             mbs = bgd.get("minibatches")
             mbt = bgd.get("minibatch_tokens")
             steps = bgd.get("steps_per_block", 1)
             for si in range(steps):
                 Hstep = Hbar
-                if mbt:
+                if gfn is not None:
+                    G = gfn(W, alpha)[1][:, be:]
+                elif mbt:
                     if Dbar is not None:
                         raise ValueError("mini-batch tokens with perturbed inputs are not supported")
                     Xk = mbt[((b_global - 1) * steps + si) % len(mbt)]
@@ -430,7 +444,10 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
                     W[:, be:] -= bgd["lr"] * G
                 else:
                     W[:, be:] -= opt.direction(G, slice(be, n))
-            after = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
+            if gfn is not None:
+                after = gfn(W, alpha)[0] if record else None
+            else:
+                after = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
             block_loss.append((b, alpha, before, after))
 
     return {

@@ -284,3 +284,77 @@ def test_final_block_kl_gradient_matches_finite_differences(module):
         E[i, j] = e
         fd = (ob.kl_final_module(module, W + E, x, P, head)[0] - ob.kl_final_module(module, W - E, x, P, head)[0]) / (2 * e)
         assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-4, abs(fd)), (module, i, j, fd, grad[i, j])
+
+
+# --- the sweep's Block-GD step on the exact losses ---------------------------
+
+def _spd(r, d, k=3):
+    Z = r.standard_normal((d, k))
+    return 0.5 * np.eye(d) + Z @ Z.T / (2 * k)
+
+
+def test_exact_window_sweep_reduces_to_the_layer_level_sweep():
+    # down_proj with an identity next block: the exact window's gradient is
+    # F_eff ΔW H̄ and its loss the layer-level surrogate, so the whole sweep
+    # (codes, weights, per-block losses) is the layer-level one
+    r = np.random.default_rng(20)
+    d, f = 16, 64
+    P = ob.block_params(r, d, 4, 2, 4, f, scale=0.8)
+    Pn = ob.block_params(r, d, 4, 2, 4, f, scale=0.8)
+    Pn["Wo"] = np.zeros_like(Pn["Wo"])
+    Pn["Wd"] = np.zeros_like(Pn["Wd"])
+    x = r.standard_normal((4, 8, d))
+    F, Fn = _spd(r, d), _spd(r, d)
+    Xm = ob.module_inputs("down_proj", x, P)
+    H_sum, T = Xm.T @ Xm, Xm.shape[0]
+    bgd = dict(lr=1e-3, steps_per_block=1, b_global_start=2, B_total=6)
+    kw = dict(block_size=16, group_size=16)
+    ref = oracle.realq_sweep(P["Wd"], H_sum, T, bgd=bgd, F=F, F_next=Fn, **kw)
+    ex = oracle.realq_sweep(P["Wd"], H_sum, T, bgd=dict(bgd, gradient_fn=ob.window_gradient_fn("down_proj", x, P, Pn, F, Fn)),
+                            **kw)
+    assert np.array_equal(ref["codes"], ex["codes"])
+    np.testing.assert_allclose(ex["deq"], ref["deq"], rtol=1e-9, atol=1e-12)
+    assert len(ex["block_loss"]) == 3 and ex["adam_t"] == ref["adam_t"] == 3
+    for (b1, a1, bf1, af1), (b2, a2, bf2, af2) in zip(ref["block_loss"], ex["block_loss"]):
+        assert (b1, a1) == (b2, a2)
+        assert abs(bf1 - bf2) <= 1e-10 * bf1 and abs(af1 - af2) <= 1e-10 * af1
+
+
+@pytest.mark.parametrize("module", ["q_proj", "v_proj", "gate_proj"])
+def test_exact_window_sweep_descends_with_small_sgd_steps(module):
+    # a small enough gradient step lowers a smooth loss: every block's loss
+    # after its Block-GD step is below the loss before it
+    r = np.random.default_rng(21)
+    d, f = 32, 48
+    P = ob.block_params(r, d, 4, 2, 8, f, scale=0.8)
+    Pn = ob.block_params(r, d, 4, 2, 8, f, scale=0.8)
+    x = r.standard_normal((2, 8, d))
+    F, Fn = _spd(r, d), _spd(r, d)
+    name = ob._MODULE_WEIGHT[module]
+    Xm = ob.module_inputs(module, x, P)
+    bgd = dict(optimizer="sgd", lr=1e-2, steps_per_block=1, b_global_start=1, B_total=4,
+               gradient_fn=ob.window_gradient_fn(module, x, P, Pn, F, Fn))
+    out = oracle.realq_sweep(P[name], Xm.T @ Xm, Xm.shape[0], block_size=8, group_size=8, bgd=bgd)
+    assert len(out["block_loss"]) == P[name].shape[1] // 8 - 1
+    for b, alpha, before, after in out["block_loss"]:
+        assert abs(alpha - (1.0 - b / 3.0)) <= 1e-15
+        assert 0.0 < after < before, (module, b, before, after)
+
+
+def test_final_block_kl_sweep_descends_with_small_sgd_steps():
+    r = np.random.default_rng(22)
+    d, f = 32, 48
+    P = ob.block_params(r, d, 4, 2, 8, f, scale=0.8)
+    head = ob.head_params(r, d, 40, scale=2.0)
+    x = r.standard_normal((2, 8, d))
+    Xm = ob.module_inputs("up_proj", x, P)
+    bgd = dict(optimizer="sgd", lr=1e-1, steps_per_block=1, b_global_start=1, B_total=1,
+               gradient_fn=ob.kl_gradient_fn("up_proj", x, P, head))
+    out = oracle.realq_sweep(P["Wu"], Xm.T @ Xm, Xm.shape[0], block_size=8, group_size=8, bgd=bgd)
+    assert len(out["block_loss"]) == 3
+    for b, alpha, before, after in out["block_loss"]:
+        assert 0.0 < after < before, (b, before, after)
+    # the Block-GD steps moved the weights: the sweep differs from the plain
+    # column sweep on the same Hessian
+    plain = oracle.realq_sweep(P["Wu"], Xm.T @ Xm, Xm.shape[0], block_size=8, group_size=8)
+    assert np.abs(out["deq"] - plain["deq"]).max() > 0.0

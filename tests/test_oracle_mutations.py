@@ -85,6 +85,15 @@ BLOCK_MUTATIONS = {
 }
 
 
+# the sweep's hook for the exact losses (oracle/realq.py), caught by the
+# block pins: the gradient's columns shifted to the quantized side
+SWEEP_HOOK_MUTATIONS = {
+    "hook_columns": ("G = gfn(W, alpha)[1][:, be:]", "G = gfn(W, alpha)[1][:, :n - be]"),
+    "hook_blend": ("before = gfn(W, alpha)[0] if record else None",
+                   "before = gfn(W, 1.0)[0] if record else None"),
+}
+
+
 def _pins_on_copy(tmp_path, old=None, new=None, target="realq.py", pins="tests/test_oracle_pins.py"):
     for d in ("oracle", "synth", "tests"):
         shutil.copytree(os.path.join(ROOT, d), tmp_path / d, ignore=shutil.ignore_patterns("__pycache__"))
@@ -120,5 +129,13 @@ def test_unchanged_block_copy_passes(tmp_path):
 def test_block_pins_catch_the_mistake(name, tmp_path):
     old, new = BLOCK_MUTATIONS[name]
     r = _pins_on_copy(tmp_path, old, new, target="block.py", pins="tests/test_oracle_block_pins.py")
+    assert r.returncode != 0, f"the pins did not catch '{name}':\n{r.stdout[-2000:]}"
+    assert " failed" in r.stdout, r.stdout[-2000:]
+
+
+@pytest.mark.parametrize("name", sorted(SWEEP_HOOK_MUTATIONS))
+def test_block_pins_catch_the_sweep_hook_mistake(name, tmp_path):
+    old, new = SWEEP_HOOK_MUTATIONS[name]
+    r = _pins_on_copy(tmp_path, old, new, target="realq.py", pins="tests/test_oracle_block_pins.py")
     assert r.returncode != 0, f"the pins did not catch '{name}':\n{r.stdout[-2000:]}"
     assert " failed" in r.stdout, r.stdout[-2000:]
