@@ -22,7 +22,7 @@ LIBDIR = os.path.join(HERE, "_lib")
 LIB = os.path.join(LIBDIR, "librealq.so")
 
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
-CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-I", INCLUDE, "-I", CSRC,
+CFLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC,-Wformat,-Werror=format", "-I", INCLUDE, "-I", CSRC,
           "--expt-relaxed-constexpr", "-Xptxas", "-warn-spills"]
 
 

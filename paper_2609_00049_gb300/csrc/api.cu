@@ -596,7 +596,7 @@ realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int
     if (T_mb > (int64_t)65535 * 32 || T > ((int64_t)1 << 40))
         return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: T_mb <= 2097120 and T <= 2^40 required");
     if (reinterpret_cast<uintptr_t>(X_hat) % 16 != 0 || n % 8 != 0)
-        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: X_hat must be 16-byte aligned with n % 8 == 0");
+        return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: X_hat must be 16-byte aligned with n %% 8 == 0");
     if (!(a_loss_clip > 0.f && a_loss_clip <= 1.f))
         return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: 0 < a_loss_clip <= 1");
     const TokArgs tok{X_hat, T, T_mb, a_loss_clip};

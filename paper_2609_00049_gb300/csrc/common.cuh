@@ -11,8 +11,9 @@
 namespace realq {
 
 // ---------------------------------------------------------------- errors ---
-void set_error(const char *fmt, ...);
-realq_status_t fail(realq_status_t s, const char *fmt, ...);
+// (printf-style: the compiler checks each format against its arguments)
+void set_error(const char *fmt, ...) __attribute__((format(printf, 1, 2)));
+realq_status_t fail(realq_status_t s, const char *fmt, ...) __attribute__((format(printf, 2, 3)));
 
 // Launch bookkeeping: every kernel launch of the library goes through
 // Launch, which counts it and, when profiling is on, brackets it with CUDA
