@@ -476,6 +476,52 @@ realq_status_t realq_graph_launch(realq_graph_t graph, realq_stream_t stream);
 int64_t realq_graph_kernels(realq_graph_t graph);
 void realq_graph_destroy(realq_graph_t graph);
 
+/* ---- The next decoder block of the exact two-block sliding window ----
+ * Sec. 4.4, Eq. (slide_window): while block l is quantized, the loss blends
+ * block l's Fisher loss with block l+1's, and the latter is back-propagated
+ * from block l+1's output.  These entry points compute that block: its
+ * forward pass, and the next block's Fisher loss
+ *   L(l+1) = (1/2T) sum_t dz_t^T F' dz_t,  dz = B(h + dh) - B(h),
+ * with its gradient g_h = dL(l+1)/d(dh) (T = S L tokens).
+ * The block is the pre-norm LLaMA-3.1 / Qwen3 structure:
+ *   a = RMSNorm(x; g1), h = x + Attn(a) Wo^T, b = RMSNorm(h; g2),
+ *   y = h + (silu(b Wg^T) * (b Wu^T)) Wd^T,
+ * RMSNorm(x; g) = x g / sqrt(mean(x^2) + rms_eps); causal grouped-query
+ * attention (query head i reads key/value head i / (n_heads / n_kv)) with
+ * rotary embedding on the pairs (j, j + head_dim/2) at angle
+ * pos * rope_base^(-2j/head_dim), pos the token's place in its sequence, and
+ * scale 1/sqrt(head_dim).
+ *   dims      n_heads % n_kv == 0, head_dim even and <= 256.
+ *   weights   device fp32, row-major (out x in): Wq (n_heads head_dim) x d,
+ *             Wk, Wv (n_kv head_dim) x d, Wo d x (n_heads head_dim),
+ *             Wg, Wu ffn x d, Wd d x ffn; gains g1, g2 of length d.
+ *   x, y, h_ref, dh, g_h
+ *             device fp32, S L x d row-major, token (s, t) at row s L + t
+ *             (S sequences of L tokens).
+ *   F_next    device fp32 d x d (the next block's Fisher).
+ *   loss      device fp32 scalar, or NULL.
+ *   ws        device workspace of realq_block_workspace_size(dims, S, L)
+ *             bytes, 256-byte aligned; it holds the forward caches.
+ * Computed in fp32 with fp32 accumulation (the loss summed in double).
+ * Asynchronous on `stream`; argument errors are returned before any launch.
+ * S L is at most 4194240 tokens.  Outputs may not alias inputs. */
+typedef struct {
+    int64_t d, n_heads, n_kv, head_dim, ffn;
+    float rms_eps;    /* 1e-6 */
+    float rope_base;  /* 10000 */
+} realq_block_dims_t;
+typedef struct {
+    const float *g1, *Wq, *Wk, *Wv, *Wo, *g2, *Wg, *Wu, *Wd;
+} realq_block_weights_t;
+size_t realq_block_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L);
+realq_status_t realq_block_forward(realq_stream_t stream, const realq_block_dims_t *dims,
+                                   const realq_block_weights_t *weights, int64_t S, int64_t L, const float *x,
+                                   float *y, void *ws, size_t ws_bytes);
+realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_t *dims,
+                                  const realq_block_weights_t *weights, int64_t S, int64_t L, const float *h_ref,
+                                  const float *dh, const float *F_next, float *g_h, float *loss, void *ws,
+                                  size_t ws_bytes);
+
 #ifdef __cplusplus
 }
 #endif

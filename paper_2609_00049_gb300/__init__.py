@@ -29,7 +29,8 @@ __all__ = [
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
-    "realq_profile_collect",
+    "realq_profile_collect", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
+    "realq_block_window",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -59,6 +60,16 @@ class BgdCfg(ctypes.Structure):
     _fields_ = [("steps_per_block", ctypes.c_int), ("optimizer", ctypes.c_int), ("lr", ctypes.c_float),
                 ("beta1", ctypes.c_float), ("beta2", ctypes.c_float), ("eps", ctypes.c_float),
                 ("b_global_start", ctypes.c_int), ("B_total", ctypes.c_int)]
+
+
+class BlockDims(ctypes.Structure):
+    _fields_ = [("d", ctypes.c_int64), ("n_heads", ctypes.c_int64), ("n_kv", ctypes.c_int64),
+                ("head_dim", ctypes.c_int64), ("ffn", ctypes.c_int64), ("rms_eps", ctypes.c_float),
+                ("rope_base", ctypes.c_float)]
+
+
+class BlockWeights(ctypes.Structure):
+    _fields_ = [(k, ctypes.c_void_p) for k in ("g1", "Wq", "Wk", "Wv", "Wo", "g2", "Wg", "Wu", "Wd")]
 
 
 class KernelStat(ctypes.Structure):
@@ -126,6 +137,11 @@ _SIGS = {
     "realq_surrogate_loss": ([_vp, _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _vp, _sz], _int),
     "realq_surrogate_workspace_size": ([_i64, _i64], _sz),
     "realq_workspace_status": ([_vp, _vp, _sz], _int),
+    "realq_block_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64], _sz),
+    "realq_block_forward": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
+                             _vp, _sz], _int),
+    "realq_block_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp, _vp,
+                            _vp, _vp, _vp, _sz], _int),
     "realq_status_string": ([_int], ctypes.c_char_p),
     "realq_last_error": ([], ctypes.c_char_p),
     "realq_launch_count": ([], _i64),
@@ -560,6 +576,55 @@ def realq_surrogate_loss(W_hat: torch.Tensor, W0: torch.Tensor, Hbar: torch.Tens
     wp, wb = _ws(ws)
     _check(lib().realq_surrogate_loss(_stream(stream), m, n, _ptr(W_hat), _ptr(W0), _dtype(W0), _ptr(Hbar), _ptr(F),
                                       _ptr(loss_out), wp, wb))
+
+
+_BLOCK_KEYS = ("g1", "Wq", "Wk", "Wv", "Wo", "g2", "Wg", "Wu", "Wd")
+
+
+def block_dims(d: int, n_heads: int, n_kv: int, head_dim: int, ffn: int, rms_eps: float = 1e-6,
+               rope_base: float = 10000.0) -> BlockDims:
+    return BlockDims(d, n_heads, n_kv, head_dim, ffn, rms_eps, rope_base)
+
+
+def _block_weights(w: dict) -> BlockWeights:
+    out = BlockWeights()
+    for k in _BLOCK_KEYS:
+        t = w[k]
+        if t.dtype != torch.float32:
+            raise ValueError(f"block weight {k}: expected float32, got {t.dtype}")
+        setattr(out, k, _ptr(t).value)
+    return out
+
+
+def realq_block_workspace_size(dims: BlockDims, S: int, L: int) -> int:
+    return int(lib().realq_block_workspace_size(ctypes.byref(dims), int(S), int(L)))
+
+
+def realq_block_forward(dims: BlockDims, weights: dict, x: torch.Tensor, y: torch.Tensor, ws: torch.Tensor,
+                        stream=None):
+    """y = block(x) for x, y of shape (S, L, d), fp32 (the decoder block of
+    the exact sliding window)."""
+    S, L, d = x.shape
+    _need(y, torch.float32, (S, L, d), "y")
+    wp, wb = _ws(ws)
+    w = _block_weights(weights)
+    _check(lib().realq_block_forward(_stream(stream), ctypes.byref(dims), ctypes.byref(w), S, L, _ptr(x), _ptr(y),
+                                     wp, wb))
+
+
+def realq_block_window(dims: BlockDims, weights: dict, h_ref: torch.Tensor, dh: torch.Tensor, F_next: torch.Tensor,
+                       g_h: torch.Tensor, ws: torch.Tensor, loss: Optional[torch.Tensor] = None, stream=None):
+    """The next block's Fisher loss (1/2T) sum_t dz_t^T F_next dz_t with
+    dz = B(h_ref + dh) - B(h_ref), into loss (a 1-element fp32 tensor, or
+    None), and its gradient in dh into g_h; all (S, L, d) fp32."""
+    S, L, d = h_ref.shape
+    for t, name in ((dh, "dh"), (g_h, "g_h")):
+        _need(t, torch.float32, (S, L, d), name)
+    _need(F_next, torch.float32, (d, d), "F_next")
+    wp, wb = _ws(ws)
+    w = _block_weights(weights)
+    _check(lib().realq_block_window(_stream(stream), ctypes.byref(dims), ctypes.byref(w), S, L, _ptr(h_ref), _ptr(dh),
+                                    _ptr(F_next), _ptr(g_h), _ptr(loss), wp, wb))
 
 
 def realq_workspace_status(ws: torch.Tensor, stream=None) -> int:

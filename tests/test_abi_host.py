@@ -134,6 +134,7 @@ def test_token_path_argument_validation(L):
     assert _qt(L, clip=1.5) == rq.REALQ_ERR_INVALID_ARG
     assert _qt(L, clip=float("nan")) == rq.REALQ_ERR_INVALID_ARG
     assert _qt(L, X=ctypes.c_void_p(0x10008)) == rq.REALQ_ERR_INVALID_ARG  # not 16-byte aligned
+    assert rq.realq_last_error().endswith("16-byte aligned with n % 8 == 0")
     assert _qt(L, X=None) == rq.REALQ_ERR_INVALID_ARG
     assert rq.realq_quantize_tokens_workspace_size(256, 512, 2048, rq.quant_cfg(), rq.bgd_cfg(1e-4)) > \
         rq.realq_quantize_workspace_size(256, 512, rq.quant_cfg(), rq.bgd_cfg(1e-4))
@@ -164,3 +165,35 @@ def test_trace_and_graph_argument_validation(L):
     assert L.realq_hessian_prepare_deferred(None, 64, 10, 0.01, FAKE, ctypes.c_void_p(0x20000), FAKE, FAKE, None,
                                             0) == rq.REALQ_ERR_WORKSPACE
     assert L.realq_prepare_status(None, None, 0, ctypes.byref(fc)) == rq.REALQ_ERR_INVALID_ARG
+
+
+def test_block_entry_points_reject_bad_arguments(L):
+    # the decoder block of the exact sliding window: every check is on the
+    # host, before any launch (fake device addresses are never dereferenced)
+    import paper_2609_00049_gb300 as rq
+    fake = ctypes.c_void_p(1 << 20)
+    w = rq.BlockWeights(*([fake.value] * 9))
+
+    def fwd(dims, S=2, L=8, ws=fake, nbytes=1 << 40):
+        return L_.realq_block_forward(None, ctypes.byref(dims), ctypes.byref(w), S, L, fake, fake, ws, nbytes)
+
+    L_ = L
+    ok = rq.block_dims(64, 4, 2, 16, 96)
+    assert rq.realq_block_workspace_size(ok, 2, 8) > (2 * 8) * (8 * 64 + 3 * 96) * 4
+    assert fwd(rq.block_dims(64, 4, 3, 16, 96)) == rq.REALQ_ERR_INVALID_ARG      # n_heads % n_kv
+    assert rq.realq_last_error() == "block_forward: n_heads % n_kv != 0"
+    assert fwd(rq.block_dims(64, 4, 2, 15, 96)) == rq.REALQ_ERR_INVALID_ARG      # odd head_dim
+    assert fwd(rq.block_dims(64, 4, 2, 512, 96)) == rq.REALQ_ERR_INVALID_ARG     # head_dim > 256
+    assert fwd(rq.block_dims(64, 4, 2, 16, 96, rms_eps=0.0)) == rq.REALQ_ERR_INVALID_ARG
+    assert fwd(rq.block_dims(64, 4, 2, 16, 96, rope_base=1.0)) == rq.REALQ_ERR_INVALID_ARG
+    assert fwd(ok, S=0) == rq.REALQ_ERR_INVALID_ARG
+    assert fwd(ok, S=4096, L=4096) == rq.REALQ_ERR_UNSUPPORTED                   # over 4194240 tokens
+    assert fwd(ok, nbytes=16) == rq.REALQ_ERR_WORKSPACE
+    assert fwd(ok, ws=ctypes.c_void_p((1 << 20) + 4)) == rq.REALQ_ERR_WORKSPACE  # misaligned
+    w.Wd = None
+    assert fwd(ok) == rq.REALQ_ERR_INVALID_ARG
+    w.Wd = fake.value
+    # the window: a NULL F_next
+    assert L_.realq_block_window(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, fake, None, fake, None, fake,
+                                 1 << 40) == rq.REALQ_ERR_INVALID_ARG
+    assert "block_window" in rq.realq_last_error()

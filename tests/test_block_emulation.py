@@ -1,0 +1,171 @@
+"""The decoder block's launch sequence (csrc/block_ops.cuh) run on the host
+against the fp64 oracle (oracle/block.py).
+
+The header's per-thread bodies and the order and arguments of its launches
+and GEMMs are compiled with g++ into a test-only library whose executor calls
+each body for every index of its launch and does each GEMM as a plain loop
+(tests/emu/block_emu.cpp).  The fp32 results must match the oracle within a
+tolerance derived below; this checks the index arithmetic and the argument
+of every step before the CUDA build of the same header runs on a GPU."""
+import ctypes
+import os
+import shutil
+import subprocess
+
+import numpy as np
+import pytest
+
+from oracle import block as ob
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+CSRC = os.path.join(ROOT, "paper_2609_00049_gb300", "csrc")
+SRC = os.path.join(ROOT, "tests", "emu", "block_emu.cpp")
+
+
+@pytest.fixture(scope="module")
+def emu(tmp_path_factory):
+    cxx = shutil.which("g++") or shutil.which("c++")
+    if cxx is None:
+        pytest.skip("no C++ compiler")
+    out = str(tmp_path_factory.mktemp("emu") / "libblock_emu.so")
+    subprocess.run([cxx, "-O2", "-std=c++17", "-shared", "-fPIC", "-Wall", "-Wextra", "-Werror", "-I", CSRC, SRC,
+                    "-o", out], check=True, capture_output=True, text=True)
+    lib = ctypes.CDLL(out)
+    lib.emu_block_workspace.restype = ctypes.c_size_t
+    lib.emu_block_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    lib.emu_block_forward.restype = ctypes.c_int
+    lib.emu_block_window.restype = ctypes.c_int
+    return lib
+
+
+_ORDER = ("g1", "Wq", "Wk", "Wv", "Wo", "g2", "Wg", "Wu", "Wd")
+
+
+class _Block:
+    def __init__(self, lib, P, S, L):
+        self.lib = lib
+        d = P["g1"].shape[0]
+        self.iv = np.array([S, L, d, P["n_heads"], P["n_kv"], P["dh"], P["Wg"].shape[0]], dtype=np.int64)
+        self.fv = np.array([1e-6, 10000.0], dtype=np.float32)
+        self.w32 = [np.ascontiguousarray(P[k], dtype=np.float32) for k in _ORDER]
+        self.wptr = (ctypes.c_void_p * 9)(*[a.ctypes.data for a in self.w32])
+        n = lib.emu_block_workspace(self.iv.ctypes.data, self.fv.ctypes.data)
+        self.ws = np.zeros(n // 4 + 64, dtype=np.float32)
+        self.shape = (S, L, d)
+
+    def forward(self, x):
+        x32 = np.ascontiguousarray(x, dtype=np.float32)
+        y = np.zeros(self.shape, dtype=np.float32)
+        rc = self.lib.emu_block_forward(ctypes.c_void_p(self.iv.ctypes.data), ctypes.c_void_p(self.fv.ctypes.data),
+                                        self.wptr, ctypes.c_void_p(x32.ctypes.data), ctypes.c_void_p(y.ctypes.data),
+                                        ctypes.c_void_p(self.ws.ctypes.data))
+        assert rc == 0
+        return y
+
+    def window(self, h, dh_, F):
+        h32, d32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (h, dh_))
+        F32 = np.ascontiguousarray(F, dtype=np.float32)
+        g = np.zeros(self.shape, dtype=np.float32)
+        loss = np.zeros(1, dtype=np.float32)
+        rc = self.lib.emu_block_window(ctypes.c_void_p(self.iv.ctypes.data), ctypes.c_void_p(self.fv.ctypes.data),
+                                       self.wptr, *(ctypes.c_void_p(a.ctypes.data) for a in (h32, d32, F32, g, loss)),
+                                       ctypes.c_void_p(self.ws.ctypes.data))
+        assert rc == 0
+        return float(loss[0]), g
+
+
+CASES = [
+    # (S, L, d, H, Hkv, dh, f): grouped queries over a ragged length; one
+    # key/value head per query head; a single token per sequence; wide heads
+    (2, 7, 16, 4, 2, 4, 24),
+    (3, 5, 24, 3, 3, 8, 40),
+    (2, 1, 16, 4, 1, 4, 20),
+    (1, 9, 32, 2, 1, 16, 48),
+    (4, 96, 256, 8, 2, 32, 704),
+]
+
+
+def _case(seed, S, L, d, H, Hkv, dh, f):
+    r = np.random.default_rng(seed)
+    P = ob.block_params(r, d, H, Hkv, dh, f, scale=0.8)
+    # round the parameters to fp32 so that both sides see the same block
+    for k in _ORDER:
+        P[k] = P[k].astype(np.float32).astype(np.float64)
+    return r, P
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_forward_matches_the_oracle(emu, case):
+    S, L, d, H, Hkv, dh, f = case
+    r, P = _case(1, *case)
+    x = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    want, _ = ob.block_forward(x, P)
+    got = _Block(emu, P, S, L).forward(x)
+    # fp32 arithmetic with fp32 accumulation over at most max(d, f, L) terms
+    # of unit size: a few 1e-7 relative per operation, well inside 1e-5 of
+    # the output's scale
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-5 * np.abs(want).max())
+
+
+@pytest.mark.parametrize("case", CASES)
+def test_window_loss_and_gradient_match_the_oracle(emu, case):
+    S, L, d, H, Hkv, dh, f = case
+    r, P = _case(2, *case)
+    h = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    dh_ = (0.1 * r.standard_normal((S, L, d))).astype(np.float32).astype(np.float64)
+    Z = r.standard_normal((d, 3))
+    F = (0.5 * np.eye(d) + Z @ Z.T / 6).astype(np.float32).astype(np.float64)
+    want_loss, want_g = ob.next_block_loss(h, dh_, P, F)
+    loss, g = _Block(emu, P, S, L).window(h, dh_, F)
+    # Δz is the difference of two fp32 forward passes whose outputs are about
+    # |h| / |Δh| = 10 times larger than Δz, so its relative error is ~10x the
+    # forward's (1e-5 of scale): 1e-4 of the gradient's and the loss's scale
+    assert abs(loss - want_loss) <= 1e-4 * abs(want_loss), (loss, want_loss)
+    np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
+def test_window_of_a_zero_perturbation_is_zero(emu):
+    S, L, d, H, Hkv, dh, f = CASES[0]
+    r, P = _case(3, *CASES[0])
+    h = r.standard_normal((S, L, d))
+    F = np.eye(d)
+    loss, g = _Block(emu, P, S, L).window(h, np.zeros_like(h), F)
+    assert loss == 0.0 and np.abs(g).max() == 0.0
+
+
+# Plausible mistakes planted in a copy of the header must fail the check:
+# the transpose rotation's sign, the softmax backward's row term, the
+# RMSNorm backward's correction, the key/value head of a query head, the
+# SiLU derivative, and a GEMM fed the untransposed weight.
+PLANTED = {
+    "rope_inverse": ("p[j] = x1 * c + x2 * s;", "p[j] = x1 * c - x2 * s;"),
+    "softmax_row_term": ("const float ds = p * (dp - Dt);", "const float ds = p * dp;"),
+    "rms_correction": ("const float v = gr[k] * g[k] * rr - xr[k] * c;", "const float v = gr[k] * g[k] * rr;"),
+    "kv_head": ("const int64_t kvh = h / a.rep();\n        const int64_t off",
+                "const int64_t kvh = h % a.Hkv;\n        const int64_t off"),
+    "silu_derivative": ("zg[i] = c * u * (sg * (1.f + g * (1.f - sg)));", "zg[i] = c * u * sg;"),
+    "untransposed_weight": ("gemm_rr(T, d, qw, B.o, B.WoT, B.h, B.x)", "gemm_rr(T, d, qw, B.o, W.Wo, B.h, B.x)"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PLANTED))
+def test_the_check_catches_a_planted_mistake(name, tmp_path):
+    old, new = PLANTED[name]
+    src = open(os.path.join(CSRC, "block_ops.cuh")).read()
+    assert src.count(old) == 1, f"anchor not found once: {old}"
+    (tmp_path / "block_ops.cuh").write_text(src.replace(old, new))
+    out = str(tmp_path / "libmut.so")
+    subprocess.run([shutil.which("g++") or "c++", "-O2", "-std=c++17", "-shared", "-fPIC", "-I", str(tmp_path), SRC,
+                    "-o", out], check=True, capture_output=True, text=True)
+    lib = ctypes.CDLL(out)
+    lib.emu_block_workspace.restype = ctypes.c_size_t
+    lib.emu_block_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    S, L, d, H, Hkv, dh, f = CASES[0]
+    r, P = _case(2, *CASES[0])
+    h = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    dh_ = (0.1 * r.standard_normal((S, L, d))).astype(np.float32).astype(np.float64)
+    F = np.eye(d)
+    want_loss, want_g = ob.next_block_loss(h, dh_, P, F)
+    loss, g = _Block(lib, P, S, L).window(h, dh_, F)
+    bad = abs(loss - want_loss) > 1e-4 * abs(want_loss) or np.abs(g - want_g).max() > 1e-4 * np.abs(want_g).max()
+    assert bad, f"the planted mistake '{name}' went unnoticed"
