@@ -522,6 +522,47 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
                                   const float *dh, const float *F_next, float *g_h, float *loss, void *ws,
                                   size_t ws_bytes);
 
+/* Module level (any linear module of block l, Eq. slide_window): block l is
+ * run at its reference weights (h*) and with the module's weight replaced
+ * by W_module (h), dh = h - h*, and
+ *   loss = alpha (1/2T) sum_t dh_t^T F_this dh_t + (1 - alpha) L(l+1)(h*, dh),
+ *   grad = d loss / d W_module, back-propagated through block l's own
+ *          backward (grad has W_module's shape).
+ *   module    0..6 = q_proj, k_proj, v_proj, o_proj, gate_proj, up_proj,
+ *             down_proj; W_module has that weight's shape (out x in).
+ *   this_block, next_block
+ *             both blocks' weights (same dims); this_block holds the
+ *             reference weight of the module.
+ *   x         block l's input, S L x d.
+ *   alpha     the window's weight in [0, 1].
+ *   ws        realq_block_module_workspace_size(dims, S, L, 0) bytes.
+ * The final block (App. "Pre-computation of the aggregated Fisher and
+ * last-transformer-block handling") has no next block; its loss is the true
+ * KL at the LM head, Eq. (kl_loss):
+ *   z = RMSNorm(h; gf) Wh^T (Wh vocab x d, gf length d),
+ *   realq_block_head_kl:  loss = (1/T) sum_t KL(softmax z(h*_t) || softmax
+ *             z(h*_t + dh_t)) and g_h = d loss / d dh, for given h* and dh
+ *             (ws: realq_block_head_workspace_size(d, S, L, vocab) bytes);
+ *   realq_block_module_kl: the same loss with h* and dh from block l as
+ *             above, and grad = d loss / d W_module
+ *             (ws: realq_block_module_workspace_size(dims, S, L, vocab)).
+ * Same conventions as above (fp32 device buffers, 256-byte aligned
+ * workspace, asynchronous on `stream`, host-side argument checks). */
+size_t realq_block_module_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L, int64_t vocab);
+size_t realq_block_head_workspace_size(int64_t d, int64_t S, int64_t L, int64_t vocab);
+realq_status_t realq_block_module_window(realq_stream_t stream, const realq_block_dims_t *dims,
+                                         const realq_block_weights_t *this_block,
+                                         const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
+                                         int module, const float *W_module, float alpha, const float *F_this,
+                                         const float *F_next, float *grad, float *loss, void *ws, size_t ws_bytes);
+realq_status_t realq_block_head_kl(realq_stream_t stream, int64_t d, int64_t S, int64_t L, const float *gf,
+                                   const float *Wh, int64_t vocab, float rms_eps, const float *h_ref, const float *dh,
+                                   float *g_h, float *loss, void *ws, size_t ws_bytes);
+realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_dims_t *dims,
+                                     const realq_block_weights_t *this_block, int64_t S, int64_t L, const float *x,
+                                     int module, const float *W_module, const float *gf, const float *Wh,
+                                     int64_t vocab, float *grad, float *loss, void *ws, size_t ws_bytes);
+
 #ifdef __cplusplus
 }
 #endif

@@ -30,7 +30,8 @@ __all__ = [
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
     "realq_profile_collect", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
-    "realq_block_window",
+    "realq_block_window", "BLOCK_MODULES", "realq_block_module_workspace_size", "realq_block_head_workspace_size",
+    "realq_block_module_window", "realq_block_head_kl", "realq_block_module_kl",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -142,6 +143,14 @@ _SIGS = {
                              _vp, _sz], _int),
     "realq_block_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp, _vp,
                             _vp, _vp, _vp, _sz], _int),
+    "realq_block_module_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _i64], _sz),
+    "realq_block_head_workspace_size": ([_i64, _i64, _i64, _i64], _sz),
+    "realq_block_module_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
+                                   ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int, _vp, _f32, _vp, _vp, _vp, _vp,
+                                   _vp, _sz], _int),
+    "realq_block_head_kl": ([_vp, _i64, _i64, _i64, _vp, _vp, _i64, _f32, _vp, _vp, _vp, _vp, _vp, _sz], _int),
+    "realq_block_module_kl": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int,
+                               _vp, _vp, _vp, _i64, _vp, _vp, _vp, _sz], _int),
     "realq_status_string": ([_int], ctypes.c_char_p),
     "realq_last_error": ([], ctypes.c_char_p),
     "realq_launch_count": ([], _i64),
@@ -625,6 +634,58 @@ def realq_block_window(dims: BlockDims, weights: dict, h_ref: torch.Tensor, dh: 
     w = _block_weights(weights)
     _check(lib().realq_block_window(_stream(stream), ctypes.byref(dims), ctypes.byref(w), S, L, _ptr(h_ref), _ptr(dh),
                                     _ptr(F_next), _ptr(g_h), _ptr(loss), wp, wb))
+
+
+BLOCK_MODULES = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def realq_block_module_workspace_size(dims: BlockDims, S: int, L: int, vocab: int = 0) -> int:
+    return int(lib().realq_block_module_workspace_size(ctypes.byref(dims), int(S), int(L), int(vocab)))
+
+
+def realq_block_head_workspace_size(d: int, S: int, L: int, vocab: int) -> int:
+    return int(lib().realq_block_head_workspace_size(int(d), int(S), int(L), int(vocab)))
+
+
+def realq_block_module_window(dims: BlockDims, this_block: dict, next_block: dict, x: torch.Tensor, module: str,
+                              W_module: torch.Tensor, alpha: float, F_this: torch.Tensor, F_next: torch.Tensor,
+                              grad: torch.Tensor, ws: torch.Tensor, loss: Optional[torch.Tensor] = None,
+                              stream=None):
+    """The exact two-block window of one module of block l: its loss into
+    loss (or None) and its gradient in W_module into grad (W_module's shape)."""
+    S, L, d = x.shape
+    _need(grad, torch.float32, tuple(W_module.shape), "grad")
+    wp, wb = _ws(ws)
+    a, b = _block_weights(this_block), _block_weights(next_block)
+    _check(lib().realq_block_module_window(_stream(stream), ctypes.byref(dims), ctypes.byref(a), ctypes.byref(b), S, L,
+                                           _ptr(x), BLOCK_MODULES.index(module), _ptr(W_module), float(alpha),
+                                           _ptr(F_this), _ptr(F_next), _ptr(grad), _ptr(loss), wp, wb))
+
+
+def realq_block_head_kl(gf: torch.Tensor, Wh: torch.Tensor, h_ref: torch.Tensor, dh: torch.Tensor,
+                        g_h: torch.Tensor, ws: torch.Tensor, loss: Optional[torch.Tensor] = None,
+                        rms_eps: float = 1e-6, stream=None):
+    """The final block's KL at the LM head between the outputs h_ref and
+    h_ref + dh, and its gradient in dh; h_ref, dh, g_h (S, L, d) fp32."""
+    S, L, d = h_ref.shape
+    V = Wh.shape[0]
+    _need(g_h, torch.float32, (S, L, d), "g_h")
+    wp, wb = _ws(ws)
+    _check(lib().realq_block_head_kl(_stream(stream), d, S, L, _ptr(gf), _ptr(Wh), V, float(rms_eps), _ptr(h_ref),
+                                     _ptr(dh), _ptr(g_h), _ptr(loss), wp, wb))
+
+
+def realq_block_module_kl(dims: BlockDims, this_block: dict, x: torch.Tensor, module: str, W_module: torch.Tensor,
+                          gf: torch.Tensor, Wh: torch.Tensor, grad: torch.Tensor, ws: torch.Tensor,
+                          loss: Optional[torch.Tensor] = None, stream=None):
+    """The final block's KL for one module's weight, and its gradient."""
+    S, L, d = x.shape
+    _need(grad, torch.float32, tuple(W_module.shape), "grad")
+    wp, wb = _ws(ws)
+    a = _block_weights(this_block)
+    _check(lib().realq_block_module_kl(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
+                                       BLOCK_MODULES.index(module), _ptr(W_module), _ptr(gf), _ptr(Wh), Wh.shape[0],
+                                       _ptr(grad), _ptr(loss), wp, wb))
 
 
 def realq_workspace_status(ws: torch.Tensor, stream=None) -> int:

@@ -1,7 +1,8 @@
 // The decoder block of the exact two-block sliding window on the GPU: the
 // launch executor of block_ops.cuh (one thread per flat index, the fp32 SIMT
-// GEMM for the projections) and the C ABI entry points realq_block_forward
-// and realq_block_window (include/realq.h).
+// GEMM for the projections) and the C ABI entry points realq_block_* of
+// include/realq.h (the block's forward, the next block's window, the
+// module-level window, the final block's KL head).
 #include "kernels.cuh"
 #include "block_ops.cuh"
 
@@ -42,7 +43,7 @@ struct DevExec {
         a.R = g.R; a.ldr = g.ldr;
         a.alpha = g.alpha;
         a.nsum = 1; a.nsum_b = 1; a.ksplit = 1;
-        st = gemm_f32(s, A_ROW, g.R ? EPI_BIAS : EPI_STORE, a, name);
+        st = gemm_f32(s, g.a_kmajor ? A_KMAJOR : A_ROW, g.R ? EPI_BIAS : EPI_STORE, a, name);
         return st != REALQ_OK;
     }
 };
@@ -73,6 +74,33 @@ realq_status_t check_block(const realq_block_dims_t *dims, const realq_block_wei
 
 blk::Weights weights_of(const realq_block_weights_t *w) {
     return blk::Weights{w->g1, w->Wq, w->Wk, w->Wv, w->Wo, w->g2, w->Wg, w->Wu, w->Wd};
+}
+
+realq_status_t check_ws_block(void *ws, size_t have, size_t need, const char *who) {
+    if (!ws || have < need || reinterpret_cast<uintptr_t>(ws) % kAlign)
+        return fail(REALQ_ERR_WORKSPACE, "%s: workspace of %zu bytes (%zu-byte aligned) required", who, need, kAlign);
+    return REALQ_OK;
+}
+
+realq_status_t check_module(int module, const float *Wm, const float *grad, const char *who) {
+    if (module < blk::M_Q || module > blk::M_DOWN)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: module must be 0..6 (q, k, v, o, gate, up, down)", who);
+    if (!Wm || !grad) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL module weight or gradient", who);
+    return REALQ_OK;
+}
+
+realq_status_t check_head(const float *gf, const float *Wh, int64_t vocab, const blk::Dims &dm, const char *who) {
+    if (!gf || !Wh) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL head gain or weight", who);
+    if (vocab <= 0 || vocab > ((int64_t)1 << 38) / dm.T())
+        return fail(REALQ_ERR_INVALID_ARG, "%s: 0 < vocab and S L vocab < 2^38 required", who);
+    return REALQ_OK;
+}
+
+size_t module_ws(const blk::Dims &dm, int64_t vocab) {
+    if (vocab > 0)
+        return blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr) +
+               blk::carve_head(dm, vocab, nullptr, nullptr);
+    return 2 * blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr);
 }
 
 }  // namespace
@@ -125,6 +153,88 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
     const blk::Weights W = weights_of(weights);
     blk::setup(X, dm, W, B);
     blk::window(X, dm, W, B, h_ref, dh, F_next, g_h, loss);
+    return X.st;
+}
+
+size_t realq_block_module_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L, int64_t vocab) {
+    if (!dims || S <= 0 || L <= 0 || dims->head_dim <= 0 || vocab < 0) return 0;
+    const blk::Dims dm{S, L, dims->d, dims->n_heads, dims->n_kv, dims->head_dim, dims->ffn, dims->rms_eps,
+                       dims->rope_base};
+    return module_ws(dm, vocab);
+}
+
+size_t realq_block_head_workspace_size(int64_t d, int64_t S, int64_t L, int64_t vocab) {
+    if (d <= 0 || S <= 0 || L <= 0 || vocab <= 0) return 0;
+    const blk::Dims dm{S, L, d, 1, 1, 2, 1, 1e-6f, 10000.f};
+    return blk::carve_head(dm, vocab, nullptr, nullptr);
+}
+
+realq_status_t realq_block_module_window(realq_stream_t stream, const realq_block_dims_t *dims,
+                                         const realq_block_weights_t *this_block,
+                                         const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
+                                         int module, const float *W_module, float alpha, const float *F_this,
+                                         const float *F_next, float *grad, float *loss, void *ws, size_t ws_bytes) {
+    const char *who = "block_module_window";
+    blk::Dims dm{};
+    REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    REALQ_TRY(check_block(dims, next_block, S, L, who, &dm));
+    REALQ_TRY(check_module(module, W_module, grad, who));
+    if (!x || !F_this || !F_next) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x, F_this or F_next", who);
+    if (!(alpha >= 0.f && alpha <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "%s: alpha must be in [0, 1]", who);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, module_ws(dm, 0), who));
+    blk::Buffers Bl{}, Bn{};
+    blk::ModuleBuffers M{};
+    char *p = static_cast<char *>(ws);
+    p += blk::carve(dm, p, &Bl);
+    p += blk::carve(dm, p, &Bn);
+    blk::carve_module(dm, p, &M);
+    DevExec X{static_cast<cudaStream_t>(stream)};
+    const blk::Weights Wref = weights_of(this_block);
+    blk::module_window(X, dm, Wref, blk::with_module(Wref, module, W_module), weights_of(next_block), Bl, Bn, M, x,
+                       module, alpha, F_this, F_next, grad, loss);
+    return X.st;
+}
+
+realq_status_t realq_block_head_kl(realq_stream_t stream, int64_t d, int64_t S, int64_t L, const float *gf,
+                                   const float *Wh, int64_t vocab, float rms_eps, const float *h_ref, const float *dh,
+                                   float *g_h, float *loss, void *ws, size_t ws_bytes) {
+    const char *who = "block_head_kl";
+    if (d <= 0 || S <= 0 || L <= 0 || S * L > 64LL * 65535LL || d > ((int64_t)1 << 38) / (S * L))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: d, S, L > 0 and S L <= 4194240 required", who);
+    if (!(rms_eps > 0.f) || !std::isfinite(rms_eps)) return fail(REALQ_ERR_INVALID_ARG, "%s: rms_eps > 0", who);
+    const blk::Dims dm{S, L, d, 1, 1, 2, 1, rms_eps, 10000.f};
+    REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
+    if (!h_ref || !dh || !g_h) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL h_ref, dh or g_h", who);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, blk::carve_head(dm, vocab, nullptr, nullptr), who));
+    blk::HeadBuffers H{};
+    blk::carve_head(dm, vocab, ws, &H);
+    DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::kl_head(X, dm, blk::Head{gf, Wh, vocab}, H, h_ref, dh, g_h, loss);
+    return X.st;
+}
+
+realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_dims_t *dims,
+                                     const realq_block_weights_t *this_block, int64_t S, int64_t L, const float *x,
+                                     int module, const float *W_module, const float *gf, const float *Wh,
+                                     int64_t vocab, float *grad, float *loss, void *ws, size_t ws_bytes) {
+    const char *who = "block_module_kl";
+    blk::Dims dm{};
+    REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    REALQ_TRY(check_module(module, W_module, grad, who));
+    REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
+    if (!x) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x", who);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, module_ws(dm, vocab), who));
+    blk::Buffers Bl{};
+    blk::ModuleBuffers M{};
+    blk::HeadBuffers H{};
+    char *p = static_cast<char *>(ws);
+    p += blk::carve(dm, p, &Bl);
+    p += blk::carve_module(dm, p, &M);
+    blk::carve_head(dm, vocab, p, &H);
+    DevExec X{static_cast<cudaStream_t>(stream)};
+    const blk::Weights Wref = weights_of(this_block);
+    blk::module_kl(X, dm, Wref, blk::with_module(Wref, module, W_module), Bl, M, blk::Head{gf, Wh, vocab}, H, x,
+                   module, grad, loss);
     return X.st;
 }
 

@@ -56,7 +56,9 @@ struct Weights {             // row-major (out x in), fp32
 };
 
 // C = alpha A B (+ R): A M x K (lda), B K x N (ldb), C and R M x N (ldc, ldr);
-// R may be C itself (each element is read before it is written).
+// R may be C itself (each element is read before it is written).  With
+// a_kmajor, A(i, k) = A[k * lda + i] (A stored K x M: a weight gradient
+// A^T B over the token axis).
 struct Gemm {
     int64_t M, N, K;
     const float *A; int64_t lda;
@@ -64,6 +66,7 @@ struct Gemm {
     float *C; int64_t ldc;
     const float *R; int64_t ldr;
     float alpha;
+    int a_kmajor;
 };
 
 // ------------------------------------------------------------ bodies ---
@@ -321,12 +324,48 @@ struct ChunkSum {
         part[c] = acc;
     }
 };
-struct HalfSum {
-    const double *part; float *out; int64_t nparts;
+struct ScaledSum {
+    const double *part; float *out; int64_t nparts; double scale;
     RQ_HD void operator()(int64_t) const {
         double acc = 0.0;
         for (int64_t c = 0; c < nparts; ++c) acc += part[c];
-        *out = (float)(0.5 * acc);
+        *out = (float)(scale * acc);
+    }
+};
+
+// out = alpha a + (1 - alpha) b for two device scalars
+struct Blend {
+    const float *a; const float *b; float *out; float alpha;
+    RQ_HD void operator()(int64_t) const { *out = alpha * *a + (1.f - alpha) * *b; }
+};
+
+// The KL head of the final block, one token row of V logits:
+//   kl_t = sum_v p_v (log p_v - log q_v),  p = softmax(z0_t), q = softmax(z1_t),
+// and z1_t is overwritten by (q - p) / T, the gradient of (1/T) sum_t kl_t.
+struct KlRow {
+    const float *z0; float *z1; float *kl; int64_t V; float inv_T;
+    RQ_HD void operator()(int64_t t) const {
+        const float *a = z0 + t * V;
+        float *b = z1 + t * V;
+        float ma = a[0], mb = b[0];
+        for (int64_t v = 1; v < V; ++v) {
+            ma = a[v] > ma ? a[v] : ma;
+            mb = b[v] > mb ? b[v] : mb;
+        }
+        float sa = 0.f, sb = 0.f;
+        for (int64_t v = 0; v < V; ++v) {
+            sa += expf(a[v] - ma);
+            sb += expf(b[v] - mb);
+        }
+        const float la = ma + logf(sa), lb = mb + logf(sb);   // log-partition functions
+        float acc = 0.f;
+        for (int64_t v = 0; v < V; ++v) {
+            const float lp = a[v] - la, lq = b[v] - lb;
+            const float p = expf(lp), q = expf(lq);
+            acc += p * (lp - lq);
+            b[v] = (q - p) * inv_T;
+        }
+        kl[t] = acc;
     }
 };
 
@@ -380,8 +419,17 @@ inline size_t carve(const Dims &dm, void *base, Buffers *bf) {
 inline Gemm gemm_rr(int64_t M, int64_t N, int64_t K, const float *A, const float *B, float *C, const float *R = nullptr,
                     float alpha = 1.f) {
     // A M x K, B K x N, C (and R) M x N, all dense row-major
-    return Gemm{M, N, K, A, K, B, N, C, N, R, N, alpha};
+    return Gemm{M, N, K, A, K, B, N, C, N, R, N, alpha, 0};
 }
+
+// the weight gradient gW (out x in) = gout^T in over T tokens: gout T x out,
+// in T x in, both row-major
+inline Gemm gemm_wgrad(int64_t T, int64_t out, int64_t in, const float *gout, const float *xin, float *gW) {
+    return Gemm{out, in, T, gout, out, xin, in, gW, in, nullptr, in, 1.f, 1};
+}
+
+// the modules of the block, in the paper's order (q, k, v, o, gate, up, down)
+enum Module : int { M_Q = 0, M_K = 1, M_V = 2, M_O = 3, M_GATE = 4, M_UP = 5, M_DOWN = 6 };
 
 // the weight transposes and the rotary tables (once per call)
 template <class X>
@@ -423,22 +471,31 @@ int forward(X &x, const Dims &dm, const Weights &W, const Buffers &B, const floa
     return e;
 }
 
-// gx = (d y / d x)^T gy for the caches of the last forward pass; gy is
-// read only; gx may not alias any buffer of B except B.y
+// gx = (d y / d x)^T gy for the caches of the last forward pass, and, for
+// module >= 0, that module's weight gradient gW (out x in) = gout^T in,
+// taken where both factors are still in the buffers.  gy is read only; gx
+// (null: not computed) may not alias any buffer of B except B.y.
 template <class X>
-int backward(X &x, const Dims &dm, const Weights &W, const Buffers &B, const float *gy, float *gx) {
+int backward(X &x, const Dims &dm, const Weights &W, const Buffers &B, const float *gy, float *gx, int module = -1,
+             float *gW = nullptr) {
     const int64_t T = dm.T(), d = dm.d, f = dm.f, qw = dm.qw(), kw = dm.kw();
     const AttnShape as{dm.L, dm.H, dm.Hkv, dm.dh};
     const int64_t rows = dm.S * dm.H * dm.L;
     int e = 0;
-    // MLP: gm = gy Wd (into m), then the SwiGLU backward over zg / zu
+    // MLP: W_d's gradient gy^T m, then gm = gy Wd (into m) and the SwiGLU
+    // backward over zg / zu
+    if (module == M_DOWN) e |= x.gemm(gemm_wgrad(T, d, f, gy, B.m, gW), "blk_wgrad");
     e |= x.gemm(gemm_rr(T, f, d, gy, W.Wd, B.m), "blk_proj_bwd");
     e |= x.map(T * f, SwigluBwd{B.m, B.zg, B.zu}, "blk_swiglu_bwd");
+    if (module == M_GATE) e |= x.gemm(gemm_wgrad(T, f, d, B.zg, B.b, gW), "blk_wgrad");
+    if (module == M_UP) e |= x.gemm(gemm_wgrad(T, f, d, B.zu, B.b, gW), "blk_wgrad");
+    if (module == M_DOWN || module == M_GATE || module == M_UP) return e;
     // gb = gzg Wg + gzu Wu (into b)
     e |= x.gemm(gemm_rr(T, d, f, B.zg, W.Wg, B.b), "blk_proj_bwd");
     e |= x.gemm(gemm_rr(T, d, f, B.zu, W.Wu, B.b, B.b), "blk_proj_bwd");
     // gh = gy + RMSNorm2 backward (into y)
     e |= x.map(T, RmsBwd{B.h, W.g2, B.r2, B.b, gy, B.y, d}, "blk_rms_bwd");
+    if (module == M_O) return e | x.gemm(gemm_wgrad(T, d, qw, B.y, B.o, gW), "blk_wgrad");
     // attention: go = gh Wo, the row terms, dq (into o), dk, dv
     e |= x.gemm(gemm_rr(T, qw, d, B.y, W.Wo, B.go), "blk_proj_bwd");
     e |= x.map(rows, AttnRowDot{B.go, B.o, B.D, as}, "blk_attn_rowdot");
@@ -446,6 +503,10 @@ int backward(X &x, const Dims &dm, const Weights &W, const Buffers &B, const flo
     e |= x.map(dm.S * dm.Hkv * dm.L, AttnBwdKV{B.q, B.k, B.v, B.go, B.lse, B.D, B.gk, B.gv, as}, "blk_attn_bwd_kv");
     e |= x.map(T * dm.H * (dm.dh / 2), Rope{B.o, qw, dm.H, dm.dh / 2, dm.dh, dm.L, B.cs, B.sn, 1}, "blk_rope");
     e |= x.map(T * dm.Hkv * (dm.dh / 2), Rope{B.gk, kw, dm.Hkv, dm.dh / 2, dm.dh, dm.L, B.cs, B.sn, 1}, "blk_rope");
+    if (module == M_Q) return e | x.gemm(gemm_wgrad(T, qw, d, B.o, B.a, gW), "blk_wgrad");
+    if (module == M_K) return e | x.gemm(gemm_wgrad(T, kw, d, B.gk, B.a, gW), "blk_wgrad");
+    if (module == M_V) return e | x.gemm(gemm_wgrad(T, kw, d, B.gv, B.a, gW), "blk_wgrad");
+    if (!gx) return e;
     // ga = gq Wq + gk Wk + gv Wv (into a)
     e |= x.gemm(gemm_rr(T, d, qw, B.o, W.Wq, B.a), "blk_proj_bwd");
     e |= x.gemm(gemm_rr(T, d, kw, B.gk, W.Wk, B.a, B.a), "blk_proj_bwd");
@@ -472,10 +533,158 @@ int window(X &x, const Dims &dm, const Weights &W, const Buffers &B, const float
         const int64_t np = (T + kChunk - 1) / kChunk;
         e |= x.map(T, RowDot{B.w, B.z0, B.rows, d}, "blk_rowdot");
         e |= x.map(np, ChunkSum{B.rows, B.part, T}, "blk_chunksum");
-        e |= x.map(1, HalfSum{B.part, loss, np}, "blk_halfsum");
+        e |= x.map(1, ScaledSum{B.part, loss, np, 0.5}, "blk_sum");
     }
     e |= backward(x, dm, W, B, B.w, g);
     return e;
+}
+
+// ------------------------------------------------- module-level losses ---
+
+// block l's side of the module-level losses: the reference and perturbed
+// outputs, the upstream gradient, this block's Fisher term, scalars
+struct ModuleBuffers {
+    float *href, *dh, *gnext, *tmp, *gh, *wthis, *rows;
+    double *part;
+    float *lthis, *lnext;
+};
+
+inline size_t carve_module(const Dims &dm, void *base, ModuleBuffers *mb) {
+    const size_t T = (size_t)dm.T(), d = (size_t)dm.d;
+    size_t off = 0;
+    char *p = static_cast<char *>(base);
+    auto take = [&](size_t count) -> float * {
+        float *r = p ? reinterpret_cast<float *>(p + off) : nullptr;
+        off += rnd(count * sizeof(float));
+        return r;
+    };
+    ModuleBuffers M{};
+    M.href = take(T * d); M.dh = take(T * d); M.gnext = take(T * d); M.tmp = take(T * d); M.gh = take(T * d);
+    M.wthis = take(T * d); M.rows = take(T);
+    M.part = reinterpret_cast<double *>(take(2 * ((T + kChunk - 1) / kChunk)));
+    M.lthis = take(1); M.lnext = take(1);
+    if (mb) *mb = M;
+    return off;
+}
+
+// the final norm and LM head: z = RMSNorm(h; gf) Wh^T, Wh V x d
+struct Head {
+    const float *gf; const float *Wh; int64_t V;
+};
+struct HeadBuffers {
+    float *WhT, *u, *r, *z0, *z1, *x1, *kl, *gu;
+    double *part;
+};
+
+inline size_t carve_head(const Dims &dm, int64_t V, void *base, HeadBuffers *hb) {
+    const size_t T = (size_t)dm.T(), d = (size_t)dm.d, v = (size_t)V;
+    size_t off = 0;
+    char *p = static_cast<char *>(base);
+    auto take = [&](size_t count) -> float * {
+        float *r = p ? reinterpret_cast<float *>(p + off) : nullptr;
+        off += rnd(count * sizeof(float));
+        return r;
+    };
+    HeadBuffers H{};
+    H.WhT = take(d * v); H.u = take(T * d); H.r = take(T); H.z0 = take(T * v); H.z1 = take(T * v);
+    H.x1 = take(T * d); H.kl = take(T); H.gu = take(T * d);
+    H.part = reinterpret_cast<double *>(take(2 * ((T + kChunk - 1) / kChunk)));
+    if (hb) *hb = H;
+    return off;
+}
+
+// The final block's loss, the true KL at the LM head (Eq. kl_loss):
+//   z0 = RMSNorm(h*; gf) Wh^T,  z1 = RMSNorm(h* + Δh; gf) Wh^T,
+//   loss = (1/T) sum_t KL(softmax z0_t || softmax z1_t),
+//   g = d loss / d Δh = RMSNorm backward of ((softmax z1 - softmax z0) Wh / T)
+template <class X>
+int kl_head(X &x, const Dims &dm, const Head &hd, const HeadBuffers &H, const float *h_ref, const float *dh_,
+            float *g, float *loss) {
+    const int64_t T = dm.T(), d = dm.d, V = hd.V;
+    int e = 0;
+    e |= x.map(V * d, Transpose{hd.Wh, H.WhT, V, d}, "blk_transpose");
+    e |= x.map(T, RmsFwd{h_ref, hd.gf, H.u, H.r, d, dm.eps}, "blk_rms_fwd");
+    e |= x.gemm(gemm_rr(T, V, d, H.u, H.WhT, H.z0), "blk_head");
+    e |= x.map(T * d, Axpy{h_ref, dh_, H.x1, 1.f}, "blk_axpy");
+    e |= x.map(T, RmsFwd{H.x1, hd.gf, H.u, H.r, d, dm.eps}, "blk_rms_fwd");
+    e |= x.gemm(gemm_rr(T, V, d, H.u, H.WhT, H.z1), "blk_head");
+    e |= x.map(T, KlRow{H.z0, H.z1, H.kl, V, 1.f / (float)T}, "blk_kl_row");
+    e |= x.gemm(gemm_rr(T, d, V, H.z1, hd.Wh, H.gu), "blk_head_bwd");
+    e |= x.map(T, RmsBwd{H.x1, hd.gf, H.r, H.gu, nullptr, g, d}, "blk_rms_bwd");
+    if (loss) {
+        const int64_t np = (T + kChunk - 1) / kChunk;
+        e |= x.map(np, ChunkSum{H.kl, H.part, T}, "blk_chunksum");
+        e |= x.map(1, ScaledSum{H.part, loss, np, 1.0 / (double)T}, "blk_sum");
+    }
+    return e;
+}
+
+// block l at its reference weights and with one module's weight replaced:
+// h* into M.href, Δh = h - h* into M.dh, and block l's caches (of the
+// perturbed pass) left in Bl for the module's backward
+template <class X>
+int module_delta(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Buffers &Bl,
+                 const ModuleBuffers &M, const float *xin) {
+    const int64_t T = dm.T(), d = dm.d;
+    int e = 0;
+    e |= setup(x, dm, Wref, Bl);
+    e |= forward(x, dm, Wref, Bl, xin, M.href);
+    e |= setup(x, dm, Wcur, Bl);
+    e |= forward(x, dm, Wcur, Bl, xin, M.dh);
+    e |= x.map(T * d, Axpy{M.dh, M.href, M.dh, -1.f}, "blk_axpy");
+    return e;
+}
+
+// The exact two-block sliding window of one module of block l (Eq.
+// slide_window), its loss and the gradient in the module's weight:
+//   loss = alpha (1/2T) sum_t Δh_t^T F Δh_t + (1 - alpha) L(l+1)(h*, Δh),
+//   g_h = alpha Δh F / T + (1 - alpha) dL(l+1)/dΔh, back through block l.
+// Wcur is Wref with the module's weight replaced; Wn the next block's.
+template <class X>
+int module_window(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Weights &Wn, const Buffers &Bl,
+                  const Buffers &Bn, const ModuleBuffers &M, const float *xin, int module, float alpha,
+                  const float *F_this, const float *F_next, float *gW, float *loss) {
+    const int64_t T = dm.T(), d = dm.d;
+    const int64_t np = (T + kChunk - 1) / kChunk;
+    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin);
+    e |= setup(x, dm, Wn, Bn);
+    e |= window(x, dm, Wn, Bn, M.href, M.dh, F_next, M.gnext, M.lnext);
+    e |= x.gemm(gemm_rr(T, d, d, M.dh, F_this, M.wthis, nullptr, 1.f / (float)T), "blk_fisher");
+    e |= x.map(T, RowDot{M.wthis, M.dh, M.rows, d}, "blk_rowdot");
+    e |= x.map(np, ChunkSum{M.rows, M.part, T}, "blk_chunksum");
+    e |= x.map(1, ScaledSum{M.part, M.lthis, np, 0.5}, "blk_sum");
+    e |= x.map(T * d, Axpy{M.gnext, M.gnext, M.tmp, -alpha}, "blk_axpy");   // (1 - alpha) g_next
+    e |= x.map(T * d, Axpy{M.tmp, M.wthis, M.gh, alpha}, "blk_axpy");       // + alpha Δh F / T
+    if (loss) e |= x.map(1, Blend{M.lthis, M.lnext, loss, alpha}, "blk_blend");
+    e |= backward(x, dm, Wcur, Bl, M.gh, nullptr, module, gW);
+    return e;
+}
+
+// The final block's loss of one module: the KL at the LM head between the
+// reference output and the one with the module's weight replaced, and the
+// gradient in that weight.
+template <class X>
+int module_kl(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Buffers &Bl,
+              const ModuleBuffers &M, const Head &hd, const HeadBuffers &H, const float *xin, int module, float *gW,
+              float *loss) {
+    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin);
+    e |= kl_head(x, dm, hd, H, M.href, M.dh, M.gh, loss);
+    e |= backward(x, dm, Wcur, Bl, M.gh, nullptr, module, gW);
+    return e;
+}
+
+// the block weights with one module's weight replaced
+inline Weights with_module(Weights w, int module, const float *Wm) {
+    switch (module) {
+        case M_Q: w.Wq = Wm; break;
+        case M_K: w.Wk = Wm; break;
+        case M_V: w.Wv = Wm; break;
+        case M_O: w.Wo = Wm; break;
+        case M_GATE: w.Wg = Wm; break;
+        case M_UP: w.Wu = Wm; break;
+        default: w.Wd = Wm; break;
+    }
+    return w;
 }
 
 }  // namespace blk

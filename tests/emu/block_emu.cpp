@@ -21,7 +21,8 @@ struct HostExec {
         for (int64_t i = 0; i < g.M; ++i)
             for (int64_t j = 0; j < g.N; ++j) {
                 float acc = 0.f;
-                for (int64_t k = 0; k < g.K; ++k) acc += g.A[i * g.lda + k] * g.B[k * g.ldb + j];
+                for (int64_t k = 0; k < g.K; ++k)
+                    acc += (g.a_kmajor ? g.A[k * g.lda + i] : g.A[i * g.lda + k]) * g.B[k * g.ldb + j];
                 const float r = g.R ? g.R[i * g.ldr + j] : 0.f;
                 g.C[i * g.ldc + j] = g.alpha * acc + r;
             }
@@ -67,4 +68,57 @@ extern "C" int emu_block_window(const int64_t *iv, const float *fv, const float 
     int e = realq::blk::setup(X, dm, W, B);
     e |= realq::blk::window(X, dm, W, B, h_ref, dh, F_next, g, loss);
     return e;
+}
+
+// the exact window of one module of block l: wl = block l, wn = next block,
+// Wm = the module's weight (module 0..6 = q, k, v, o, gate, up, down)
+extern "C" size_t emu_module_workspace(const int64_t *iv, const float *fv, int64_t V) {
+    const realq::blk::Dims dm = dims_of(iv, fv);
+    size_t b = 2 * realq::blk::carve(dm, nullptr, nullptr) + realq::blk::carve_module(dm, nullptr, nullptr);
+    if (V > 0) b += realq::blk::carve_head(dm, V, nullptr, nullptr);
+    return b;
+}
+
+extern "C" int emu_module_window(const int64_t *iv, const float *fv, const float *const *wl, const float *const *wn,
+                                 const float *x, int module, const float *Wm, float alpha, const float *F_this,
+                                 const float *F_next, float *gW, float *loss, void *ws) {
+    using namespace realq::blk;
+    const Dims dm = dims_of(iv, fv);
+    Buffers Bl{}, Bn{};
+    ModuleBuffers M{};
+    char *p = static_cast<char *>(ws);
+    p += carve(dm, p, &Bl);
+    p += carve(dm, p, &Bn);
+    carve_module(dm, p, &M);
+    HostExec X;
+    const Weights Wref = weights_of(wl);
+    return module_window(X, dm, Wref, with_module(Wref, module, Wm), weights_of(wn), Bl, Bn, M, x, module, alpha,
+                         F_this, F_next, gW, loss);
+}
+
+extern "C" int emu_head_kl(const int64_t *iv, const float *fv, const float *gf, const float *Wh, int64_t V,
+                           const float *h_ref, const float *dh, float *g, float *loss, void *ws) {
+    using namespace realq::blk;
+    const Dims dm = dims_of(iv, fv);
+    HeadBuffers H{};
+    carve_head(dm, V, ws, &H);
+    HostExec X;
+    return kl_head(X, dm, Head{gf, Wh, V}, H, h_ref, dh, g, loss);
+}
+
+extern "C" int emu_module_kl(const int64_t *iv, const float *fv, const float *const *wl, const float *x, int module,
+                             const float *Wm, const float *gf, const float *Wh, int64_t V, float *gW, float *loss,
+                             void *ws) {
+    using namespace realq::blk;
+    const Dims dm = dims_of(iv, fv);
+    Buffers Bl{};
+    ModuleBuffers M{};
+    HeadBuffers H{};
+    char *p = static_cast<char *>(ws);
+    p += carve(dm, p, &Bl);
+    p += carve_module(dm, p, &M);
+    carve_head(dm, V, p, &H);
+    HostExec X;
+    const Weights Wref = weights_of(wl);
+    return module_kl(X, dm, Wref, with_module(Wref, module, Wm), Bl, M, Head{gf, Wh, V}, H, x, module, gW, loss);
 }

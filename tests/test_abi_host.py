@@ -197,3 +197,34 @@ def test_block_entry_points_reject_bad_arguments(L):
     assert L_.realq_block_window(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, fake, None, fake, None, fake,
                                  1 << 40) == rq.REALQ_ERR_INVALID_ARG
     assert "block_window" in rq.realq_last_error()
+
+
+def test_block_module_and_head_entry_points_reject_bad_arguments(L):
+    import paper_2609_00049_gb300 as rq
+    fake = ctypes.c_void_p(1 << 20)
+    w = rq.BlockWeights(*([fake.value] * 9))
+    ok = rq.block_dims(64, 4, 2, 16, 96)
+    big = 1 << 40
+
+    def win(module=0, alpha=0.5, F=fake, nbytes=big):
+        return L.realq_block_module_window(None, ctypes.byref(ok), ctypes.byref(w), ctypes.byref(w), 2, 8, fake,
+                                           module, fake, alpha, F, fake, fake, None, fake, nbytes)
+
+    assert rq.realq_block_module_workspace_size(ok, 2, 8) > 2 * rq.realq_block_workspace_size(ok, 2, 8)
+    assert rq.realq_block_module_workspace_size(ok, 2, 8, 1000) > 2 * 8 * 1000 * 8
+    assert rq.realq_block_head_workspace_size(64, 2, 8, 1000) > 2 * 8 * 1000 * 8
+    assert win(module=7) == rq.REALQ_ERR_INVALID_ARG
+    assert win(module=-1) == rq.REALQ_ERR_INVALID_ARG
+    assert win(alpha=1.5) == rq.REALQ_ERR_INVALID_ARG
+    assert win(F=None) == rq.REALQ_ERR_INVALID_ARG
+    assert win(nbytes=1024) == rq.REALQ_ERR_WORKSPACE
+    assert "block_module_window" in rq.realq_last_error()
+    # the head: vocab, eps and the token limit
+    kl = L.realq_block_head_kl
+    assert kl(None, 64, 2, 8, fake, fake, 0, 1e-6, fake, fake, fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG
+    assert kl(None, 64, 2, 8, fake, fake, 100, 0.0, fake, fake, fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG
+    assert kl(None, 64, 4096, 4096, fake, fake, 100, 1e-6, fake, fake, fake, None, fake, big) == \
+        rq.REALQ_ERR_INVALID_ARG
+    assert kl(None, 64, 2, 8, fake, fake, 100, 1e-6, fake, fake, fake, None, fake, 64) == rq.REALQ_ERR_WORKSPACE
+    assert L.realq_block_module_kl(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, 3, fake, fake, None, 100,
+                                   fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG     # NULL Wh

@@ -133,6 +133,115 @@ def test_window_of_a_zero_perturbation_is_zero(emu):
     assert loss == 0.0 and np.abs(g).max() == 0.0
 
 
+MODULES = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def _ptrs(P):
+    arrs = [np.ascontiguousarray(P[k], dtype=np.float32) for k in _ORDER]
+    return arrs, (ctypes.c_void_p * 9)(*[a.ctypes.data for a in arrs])
+
+
+def _c(a):
+    return ctypes.c_void_p(a.ctypes.data)
+
+
+def _spd32(r, d):
+    Z = r.standard_normal((d, 3))
+    return (0.5 * np.eye(d) + Z @ Z.T / 6).astype(np.float32).astype(np.float64)
+
+
+def _module_case(seed, case, module):
+    S, L, d, H, Hkv, dh, f = case
+    r, P = _case(seed, *case)
+    _, Pn = _case(seed + 100, *case)
+    name = ob._MODULE_WEIGHT[module]
+    Wm = (P[name] + 0.05 * r.standard_normal(P[name].shape)).astype(np.float32).astype(np.float64)
+    x = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    return r, P, Pn, name, Wm, x
+
+
+def _iv(P, S, L):
+    d = P["g1"].shape[0]
+    return (np.array([S, L, d, P["n_heads"], P["n_kv"], P["dh"], P["Wg"].shape[0]], dtype=np.int64),
+            np.array([1e-6, 10000.0], dtype=np.float32))
+
+
+def _ws(emu, iv, fv, V=0):
+    emu.emu_module_workspace.restype = ctypes.c_size_t
+    emu.emu_module_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p, ctypes.c_int64]
+    return np.zeros(emu.emu_module_workspace(iv.ctypes.data, fv.ctypes.data, V) // 4 + 64, dtype=np.float32)
+
+
+@pytest.mark.parametrize("module", MODULES)
+def test_module_window_matches_the_oracle(emu, module):
+    # block l's own backward to each module's weight, with the next block's
+    # window (Eq. slide_window); the case with grouped queries and a ragged
+    # length
+    case = CASES[0]
+    S, L, d = case[0], case[1], case[2]
+    r, P, Pn, name, Wm, x = _module_case(4, case, module)
+    F, Fn = _spd32(r, d), _spd32(r, d)
+    alpha = 0.6
+    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, alpha, F, Fn)
+    iv, fv = _iv(P, S, L)
+    al, pl = _ptrs(P)
+    an, pn = _ptrs(Pn)
+    x32, W32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, F, Fn))
+    g = np.zeros(Wm.shape, dtype=np.float32)
+    loss = np.zeros(1, dtype=np.float32)
+    ws = _ws(emu, iv, fv)
+    rc = emu.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(MODULES.index(module)), _c(W32),
+                               ctypes.c_float(alpha), _c(F32), _c(Fn32), _c(g), _c(loss), _c(ws))
+    assert rc == 0
+    # Δh is a difference of two fp32 forward passes, as in the window
+    assert abs(float(loss[0]) - want_loss) <= 1e-4 * abs(want_loss), (float(loss[0]), want_loss)
+    np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
+def test_kl_head_matches_the_oracle(emu):
+    r = np.random.default_rng(5)
+    S, L, d, V = 3, 5, 16, 37
+    head = ob.head_params(r, d, V, scale=1.5)
+    head = {k: v.astype(np.float32).astype(np.float64) for k, v in head.items()}
+    h = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    dh_ = (0.1 * r.standard_normal((S, L, d))).astype(np.float32).astype(np.float64)
+    want_loss, want_g = ob.kl_head_loss(h, dh_, head)
+    iv = np.array([S, L, d, 1, 1, 2, 1], dtype=np.int64)
+    fv = np.array([1e-6, 10000.0], dtype=np.float32)
+    gf, Wh, h32, d32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (head["gf"], head["Wh"], h, dh_))
+    g = np.zeros((S, L, d), dtype=np.float32)
+    loss = np.zeros(1, dtype=np.float32)
+    ws = _ws(emu, iv, fv, V)
+    rc = emu.emu_head_kl(_c(iv), _c(fv), _c(gf), _c(Wh), ctypes.c_int64(V), _c(h32), _c(d32), _c(g), _c(loss),
+                         _c(ws))
+    assert rc == 0
+    # the KL of distributions 1e-1 apart is second order: its fp32 value is
+    # a sum of p (log p - log q) terms 10x larger than the result
+    assert abs(float(loss[0]) - want_loss) <= 1e-4 * abs(want_loss), (float(loss[0]), want_loss)
+    np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
+@pytest.mark.parametrize("module", ("k_proj", "o_proj", "up_proj", "down_proj"))
+def test_final_block_module_kl_matches_the_oracle(emu, module):
+    case = CASES[1]
+    S, L, d = case[0], case[1], case[2]
+    r, P, _, name, Wm, x = _module_case(6, case, module)
+    V = 29
+    head = {k: v.astype(np.float32).astype(np.float64) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
+    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head)
+    iv, fv = _iv(P, S, L)
+    al, pl = _ptrs(P)
+    x32, W32, gf, Wh = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, head["gf"], head["Wh"]))
+    g = np.zeros(Wm.shape, dtype=np.float32)
+    loss = np.zeros(1, dtype=np.float32)
+    ws = _ws(emu, iv, fv, V)
+    rc = emu.emu_module_kl(_c(iv), _c(fv), pl, _c(x32), ctypes.c_int(MODULES.index(module)), _c(W32), _c(gf),
+                           _c(Wh), ctypes.c_int64(V), _c(g), _c(loss), _c(ws))
+    assert rc == 0
+    assert abs(float(loss[0]) - want_loss) <= 1e-4 * abs(want_loss), (float(loss[0]), want_loss)
+    np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
 # Plausible mistakes planted in a copy of the header must fail the check:
 # the transpose rotation's sign, the softmax backward's row term, the
 # RMSNorm backward's correction, the key/value head of a query head, the
@@ -145,7 +254,15 @@ PLANTED = {
                 "const int64_t kvh = h % a.Hkv;\n        const int64_t off"),
     "silu_derivative": ("zg[i] = c * u * (sg * (1.f + g * (1.f - sg)));", "zg[i] = c * u * sg;"),
     "untransposed_weight": ("gemm_rr(T, d, qw, B.o, B.WoT, B.h, B.x)", "gemm_rr(T, d, qw, B.o, W.Wo, B.h, B.x)"),
+    # module-level: q_proj's gradient taken before the transpose rotation,
+    # the blend of the two blocks' gradients, the KL gradient's sign
+    "wgrad_before_rope": ("if (module == M_Q) return e | x.gemm(gemm_wgrad(T, qw, d, B.o, B.a, gW), \"blk_wgrad\");\n",
+                          ""),
+    "module_blend": ("Axpy{M.tmp, M.wthis, M.gh, alpha}", "Axpy{M.tmp, M.wthis, M.gh, 1.f - alpha}"),
+    "kl_sign": ("b[v] = (q - p) * inv_T;", "b[v] = (p - q) * inv_T;"),
 }
+# the check each planted mistake is run against
+_PLANTED_CHECK = {"wgrad_before_rope": "module_q", "module_blend": "module_q", "kl_sign": "kl"}
 
 
 @pytest.mark.parametrize("name", sorted(PLANTED))
@@ -153,6 +270,14 @@ def test_the_check_catches_a_planted_mistake(name, tmp_path):
     old, new = PLANTED[name]
     src = open(os.path.join(CSRC, "block_ops.cuh")).read()
     assert src.count(old) == 1, f"anchor not found once: {old}"
+    if name == "wgrad_before_rope":
+        # move q_proj's weight gradient ahead of the transpose rotation
+        new = old
+        src = src.replace(old, "")
+        anchor = '    e |= x.map(T * dm.H * (dm.dh / 2), Rope{B.o, qw'
+        assert src.count(anchor) == 1
+        src = src.replace(anchor, old + anchor)
+        old = new
     (tmp_path / "block_ops.cuh").write_text(src.replace(old, new))
     out = str(tmp_path / "libmut.so")
     subprocess.run([shutil.which("g++") or "c++", "-O2", "-std=c++17", "-shared", "-fPIC", "-I", str(tmp_path), SRC,
@@ -160,6 +285,10 @@ def test_the_check_catches_a_planted_mistake(name, tmp_path):
     lib = ctypes.CDLL(out)
     lib.emu_block_workspace.restype = ctypes.c_size_t
     lib.emu_block_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    check = _PLANTED_CHECK.get(name, "window")
+    if check != "window":
+        assert _planted_module_or_kl_differs(lib, check), f"the planted mistake '{name}' went unnoticed"
+        return
     S, L, d, H, Hkv, dh, f = CASES[0]
     r, P = _case(2, *CASES[0])
     h = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
@@ -169,3 +298,38 @@ def test_the_check_catches_a_planted_mistake(name, tmp_path):
     loss, g = _Block(lib, P, S, L).window(h, dh_, F)
     bad = abs(loss - want_loss) > 1e-4 * abs(want_loss) or np.abs(g - want_g).max() > 1e-4 * np.abs(want_g).max()
     assert bad, f"the planted mistake '{name}' went unnoticed"
+
+
+def _planted_module_or_kl_differs(lib, check):
+    case = CASES[0]
+    S, L, d = case[0], case[1], case[2]
+    if check == "kl":
+        r = np.random.default_rng(5)
+        V = 37
+        head = {k: v.astype(np.float32).astype(np.float64) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
+        h = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+        dh_ = (0.1 * r.standard_normal((S, L, d))).astype(np.float32).astype(np.float64)
+        want_loss, want_g = ob.kl_head_loss(h, dh_, head)
+        iv = np.array([S, L, d, 1, 1, 2, 1], dtype=np.int64)
+        fv = np.array([1e-6, 10000.0], dtype=np.float32)
+        gf, Wh, h32, d32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (head["gf"], head["Wh"], h, dh_))
+        g = np.zeros((S, L, d), dtype=np.float32)
+        loss = np.zeros(1, dtype=np.float32)
+        ws = _ws(lib, iv, fv, V)
+        assert lib.emu_head_kl(_c(iv), _c(fv), _c(gf), _c(Wh), ctypes.c_int64(V), _c(h32), _c(d32), _c(g), _c(loss),
+                               _c(ws)) == 0
+    else:
+        r, P, Pn, name, Wm, x = _module_case(4, case, "q_proj")
+        F, Fn = _spd32(r, d), _spd32(r, d)
+        want_loss, want_g = ob.sliding_window_module("q_proj", Wm, x, P, Pn, 0.6, F, Fn)
+        iv, fv = _iv(P, S, L)
+        al, pl = _ptrs(P)
+        an, pn = _ptrs(Pn)
+        x32, W32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, F, Fn))
+        g = np.zeros(Wm.shape, dtype=np.float32)
+        loss = np.zeros(1, dtype=np.float32)
+        ws = _ws(lib, iv, fv)
+        assert lib.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(0), _c(W32), ctypes.c_float(0.6),
+                                     _c(F32), _c(Fn32), _c(g), _c(loss), _c(ws)) == 0
+    return (abs(float(loss[0]) - want_loss) > 1e-4 * abs(want_loss)
+            or np.abs(g - want_g).max() > 1e-4 * np.abs(want_g).max())

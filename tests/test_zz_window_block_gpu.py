@@ -104,3 +104,72 @@ def test_block_window_is_deterministic_and_zero_at_zero():
     loss = torch.ones(1, dtype=torch.float32, device="cuda")
     rq.realq_block_window(dims, W, h, torch.zeros_like(h), F, g, ws, loss=loss)
     assert loss.item() == 0.0 and g.abs().max().item() == 0.0
+
+
+MODULES = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def _spd(r, d):
+    Z = r.standard_normal((d, 3))
+    return _f32(0.5 * np.eye(d) + Z @ Z.T / 6)
+
+
+def _weights(P):
+    return {k: torch.from_numpy(P[k].astype(np.float32)).cuda() for k in _KEYS}
+
+
+@pytest.mark.parametrize("case", [CASES[0], CASES[4]])
+@pytest.mark.parametrize("module", MODULES)
+def test_module_window_matches_the_oracle(case, module):
+    # block l's own backward to the module's weight with the next block's
+    # window (Eq. slide_window), against oracle.block.sliding_window_module
+    S, L, d, H, Hkv, dh, f = case
+    r, P, W, dims, _ = _case(4, *case)
+    _, Pn, Wn, _, _ = _case(104, *case)
+    name = ob._MODULE_WEIGHT[module]
+    Wm = _f32(P[name] + 0.05 * r.standard_normal(P[name].shape))
+    x = _f32(r.standard_normal((S, L, d)))
+    F, Fn = _spd(r, d), _spd(r, d)
+    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, 0.6, F, Fn)
+    grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float32, device="cuda")
+    ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L))
+    rq.realq_block_module_window(dims, W, Wn, _dev(x), module, _dev(Wm), 0.6, _dev(F), _dev(Fn), grad, ws, loss=loss)
+    got = grad.cpu().numpy()
+    assert abs(loss.item() - want_loss) <= 1e-4 * abs(want_loss), (loss.item(), want_loss)
+    np.testing.assert_allclose(got, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
+def test_head_kl_matches_the_oracle():
+    r = np.random.default_rng(5)
+    S, L, d, V = 4, 33, 64, 1000
+    head = {k: _f32(v) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
+    h = _f32(r.standard_normal((S, L, d)))
+    dh_ = _f32(0.1 * r.standard_normal((S, L, d)))
+    want_loss, want_g = ob.kl_head_loss(h, dh_, head)
+    g = torch.empty((S, L, d), dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float32, device="cuda")
+    ws = rq.workspace(rq.realq_block_head_workspace_size(d, S, L, V))
+    rq.realq_block_head_kl(_dev(head["gf"]), _dev(head["Wh"]), _dev(h), _dev(dh_), g, ws, loss=loss)
+    assert abs(loss.item() - want_loss) <= 1e-4 * abs(want_loss), (loss.item(), want_loss)
+    np.testing.assert_allclose(g.cpu().numpy(), want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+
+
+@pytest.mark.parametrize("module", ("k_proj", "o_proj", "up_proj", "down_proj"))
+def test_final_block_module_kl_matches_the_oracle(module):
+    case = CASES[1]
+    S, L, d, H, Hkv, dh, f = case
+    r, P, W, dims, _ = _case(6, *case)
+    name = ob._MODULE_WEIGHT[module]
+    Wm = _f32(P[name] + 0.05 * r.standard_normal(P[name].shape))
+    x = _f32(r.standard_normal((S, L, d)))
+    V = 29
+    head = {k: _f32(v) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
+    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head)
+    grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
+    loss = torch.zeros(1, dtype=torch.float32, device="cuda")
+    ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L, V))
+    rq.realq_block_module_kl(dims, W, _dev(x), module, _dev(Wm), _dev(head["gf"]), _dev(head["Wh"]), grad, ws,
+                             loss=loss)
+    assert abs(loss.item() - want_loss) <= 1e-4 * abs(want_loss), (loss.item(), want_loss)
+    np.testing.assert_allclose(grad.cpu().numpy(), want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
