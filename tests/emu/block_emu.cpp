@@ -11,13 +11,35 @@
 
 namespace {
 
+// 0: each launch's indices in increasing order; 1: in decreasing order.  A
+// launch whose result depends on the order has indices that read what
+// another index of the same launch writes, which the GPU does not order.
+int g_order = 0;
+
+bool overlaps(const void *a, size_t an, const void *b, size_t bn) {
+    const char *p = static_cast<const char *>(a), *q = static_cast<const char *>(b);
+    return p < q + bn && q < p + an;
+}
+
 struct HostExec {
     template <class Fn>
     int map(int64_t count, const Fn &fn, const char *) {
-        for (int64_t i = 0; i < count; ++i) fn(i);
+        if (g_order == 0)
+            for (int64_t i = 0; i < count; ++i) fn(i);
+        else
+            for (int64_t i = count - 1; i >= 0; --i) fn(i);
         return 0;
     }
+    // The GPU GEMM's CTAs read A and B while others write C, so C may share
+    // no byte with A or B; R may be C itself (each element is read by the
+    // thread that writes it) but not overlap it otherwise.  Returns 2 when an
+    // operand breaks that.
     int gemm(const realq::blk::Gemm &g, const char *) {
+        const size_t cb = (size_t)((g.M - 1) * g.ldc + g.N) * sizeof(float);
+        const size_t ab = (size_t)(g.a_kmajor ? (g.K - 1) * g.lda + g.M : (g.M - 1) * g.lda + g.K) * sizeof(float);
+        const size_t bb = (size_t)((g.K - 1) * g.ldb + g.N) * sizeof(float);
+        if (overlaps(g.C, cb, g.A, ab) || overlaps(g.C, cb, g.B, bb)) return 2;
+        if (g.R && g.R != g.C && overlaps(g.C, cb, g.R, (size_t)((g.M - 1) * g.ldr + g.N) * sizeof(float))) return 2;
         for (int64_t i = 0; i < g.M; ++i)
             for (int64_t j = 0; j < g.N; ++j) {
                 float acc = 0.f;
@@ -39,6 +61,8 @@ realq::blk::Weights weights_of(const float *const *w) {
 }
 
 }  // namespace
+
+extern "C" void emu_set_order(int order) { g_order = order; }
 
 // iv = {S, L, d, H, Hkv, dh, f}, fv = {eps, rope_base},
 // w = {g1, Wq, Wk, Wv, Wo, g2, Wg, Wu, Wd}

@@ -6,7 +6,10 @@ and GEMMs are compiled with g++ into a test-only library whose executor calls
 each body for every index of its launch and does each GEMM as a plain loop
 (tests/emu/block_emu.cpp).  The fp32 results must match the oracle within a
 tolerance derived below; this checks the index arithmetic and the argument
-of every step before the CUDA build of the same header runs on a GPU."""
+of every step before the CUDA build of the same header runs on a GPU.  Each
+launch also runs with its indices reversed (the result must not change: the
+GPU orders no index before another), and every GEMM is checked for an output
+that overlaps its operands."""
 import ctypes
 import os
 import shutil
@@ -35,6 +38,8 @@ def emu(tmp_path_factory):
     lib.emu_block_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
     lib.emu_block_forward.restype = ctypes.c_int
     lib.emu_block_window.restype = ctypes.c_int
+    lib.emu_set_order.argtypes = [ctypes.c_int]
+    lib.emu_set_order(0)
     return lib
 
 
@@ -53,16 +58,19 @@ class _Block:
         self.ws = np.zeros(n // 4 + 64, dtype=np.float32)
         self.shape = (S, L, d)
 
-    def forward(self, x):
+    def forward(self, x, rcs=None):
         x32 = np.ascontiguousarray(x, dtype=np.float32)
         y = np.zeros(self.shape, dtype=np.float32)
         rc = self.lib.emu_block_forward(ctypes.c_void_p(self.iv.ctypes.data), ctypes.c_void_p(self.fv.ctypes.data),
                                         self.wptr, ctypes.c_void_p(x32.ctypes.data), ctypes.c_void_p(y.ctypes.data),
                                         ctypes.c_void_p(self.ws.ctypes.data))
-        assert rc == 0
+        if rcs is None:
+            assert rc == 0
+        else:
+            rcs.append(rc)
         return y
 
-    def window(self, h, dh_, F):
+    def window(self, h, dh_, F, rcs=None):
         h32, d32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (h, dh_))
         F32 = np.ascontiguousarray(F, dtype=np.float32)
         g = np.zeros(self.shape, dtype=np.float32)
@@ -70,7 +78,10 @@ class _Block:
         rc = self.lib.emu_block_window(ctypes.c_void_p(self.iv.ctypes.data), ctypes.c_void_p(self.fv.ctypes.data),
                                        self.wptr, *(ctypes.c_void_p(a.ctypes.data) for a in (h32, d32, F32, g, loss)),
                                        ctypes.c_void_p(self.ws.ctypes.data))
-        assert rc == 0
+        if rcs is None:
+            assert rc == 0
+        else:
+            rcs.append(rc)
         return float(loss[0]), g
 
 
@@ -333,3 +344,104 @@ def _planted_module_or_kl_differs(lib, check):
                                      _c(F32), _c(Fn32), _c(g), _c(loss), _c(ws)) == 0
     return (abs(float(loss[0]) - want_loss) > 1e-4 * abs(want_loss)
             or np.abs(g - want_g).max() > 1e-4 * np.abs(want_g).max())
+
+
+def _all_ops(lib, case, V=23):
+    """Every op of the header on one case (forward, window, the module
+    window and the final block's KL for all seven modules, the KL head), as
+    one flat fp32 vector, with the return codes."""
+    S, L, d, H, Hkv, dh, f = case
+    r, P = _case(7, *case)
+    _, Pn = _case(107, *case)
+    out, rcs = [], []
+    blk = _Block(lib, P, S, L)
+    x = r.standard_normal((S, L, d))
+    dh_ = 0.1 * r.standard_normal((S, L, d))
+    F, Fn = _spd32(r, d), _spd32(r, d)
+    out.append(blk.forward(x, rcs).ravel())
+    loss, g = blk.window(x, dh_, F, rcs)
+    out += [g.ravel(), np.float32([loss])]
+    iv, fv = _iv(P, S, L)
+    al, pl = _ptrs(P)
+    an, pn = _ptrs(Pn)
+    head = {k: np.ascontiguousarray(v, dtype=np.float32) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
+    x32, d32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, dh_, F, Fn))
+    for i, module in enumerate(MODULES):
+        W32 = np.ascontiguousarray(P[ob._MODULE_WEIGHT[module]] + 0.05 * r.standard_normal(
+            P[ob._MODULE_WEIGHT[module]].shape), dtype=np.float32)
+        for kind in ("window", "kl"):
+            gW = np.zeros(W32.shape, dtype=np.float32)
+            lo = np.zeros(1, dtype=np.float32)
+            if kind == "window":
+                ws = _ws(lib, iv, fv)
+                rcs.append(lib.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(i), _c(W32),
+                                                 ctypes.c_float(0.6), _c(F32), _c(Fn32), _c(gW), _c(lo), _c(ws)))
+            else:
+                ws = _ws(lib, iv, fv, V)
+                rcs.append(lib.emu_module_kl(_c(iv), _c(fv), pl, _c(x32), ctypes.c_int(i), _c(W32), _c(head["gf"]),
+                                             _c(head["Wh"]), ctypes.c_int64(V), _c(gW), _c(lo), _c(ws)))
+            out += [gW.ravel(), lo]
+    g = np.zeros((S, L, d), dtype=np.float32)
+    lo = np.zeros(1, dtype=np.float32)
+    ws = _ws(lib, iv, fv, V)
+    rcs.append(lib.emu_head_kl(_c(iv), _c(fv), _c(head["gf"]), _c(head["Wh"]), ctypes.c_int64(V), _c(x32), _c(d32),
+                               _c(g), _c(lo), _c(ws)))
+    out += [g.ravel(), lo]
+    return np.concatenate(out), rcs
+
+
+# grouped queries over a ragged length, one key/value head per query head,
+# and more than one 1024-token chunk of the fixed-order loss sum
+ORDER_CASES = [CASES[0], CASES[1], (1, 1100, 8, 2, 1, 4, 12)]
+
+
+@pytest.mark.parametrize("case", ORDER_CASES)
+def test_launches_do_not_depend_on_the_order_of_their_indices(emu, case):
+    # The GPU runs the indices of one launch in no fixed order, so no index
+    # may read what another index of the same launch writes: every op run
+    # with each launch's indices reversed gives the same bits.  Every GEMM's
+    # output also shares no memory with its A and B operands (the host
+    # executor returns an error code if one does).
+    try:
+        emu.emu_set_order(0)
+        a, rca = _all_ops(emu, case)
+        emu.emu_set_order(1)
+        b, rcb = _all_ops(emu, case)
+    finally:
+        emu.emu_set_order(0)
+    assert rca == [0] * len(rca) and rcb == [0] * len(rcb)
+    assert np.isfinite(a).all()
+    assert a.tobytes() == b.tobytes()
+
+
+# A launch whose indices depend on each other, and a GEMM that overwrites
+# its own operand, planted in a copy of the header, must each be caught.
+PLANTED_ORDER = {
+    # the attention output written over the values that later queries read
+    "attn_output_over_values": ("AttnFwd{B.q, B.k, B.v, B.o, B.lse, as}", "AttnFwd{B.q, B.k, B.v, B.v, B.lse, as}"),
+    # the gate's input gradient written over the gate gradient it reads
+    "gemm_over_its_operand": ("e |= x.gemm(gemm_rr(T, d, f, B.zg, W.Wg, B.b), \"blk_proj_bwd\");",
+                              "e |= x.gemm(gemm_rr(T, d, f, B.zg, W.Wg, B.zg), \"blk_proj_bwd\");"),
+}
+
+
+@pytest.mark.parametrize("name", sorted(PLANTED_ORDER))
+def test_the_order_check_catches_a_planted_dependence(name, tmp_path):
+    old, new = PLANTED_ORDER[name]
+    src = open(os.path.join(CSRC, "block_ops.cuh")).read()
+    assert src.count(old) == 1, f"anchor not found once: {old}"
+    (tmp_path / "block_ops.cuh").write_text(src.replace(old, new))
+    out = str(tmp_path / "libmut.so")
+    subprocess.run([shutil.which("g++") or "c++", "-O2", "-std=c++17", "-shared", "-fPIC", "-I", str(tmp_path), SRC,
+                    "-o", out], check=True, capture_output=True, text=True)
+    lib = ctypes.CDLL(out)
+    lib.emu_block_workspace.restype = ctypes.c_size_t
+    lib.emu_block_workspace.argtypes = [ctypes.c_void_p, ctypes.c_void_p]
+    lib.emu_set_order.argtypes = [ctypes.c_int]
+    case = CASES[1]     # H = H_kv, so that the attention output and the values have one width
+    lib.emu_set_order(0)
+    a, rca = _all_ops(lib, case)
+    lib.emu_set_order(1)
+    b, rcb = _all_ops(lib, case)
+    caught = any(rca) or any(rcb) or a.tobytes() != b.tobytes()
+    assert caught, f"the planted dependence '{name}' went unnoticed"

@@ -7,7 +7,8 @@ unit-scale terms): the forward within 1e-5 of the output's scale; the
 window's Δz is the difference of two forward passes about |h|/|Δh| = 10
 times larger than it, so the loss and the gradient within 1e-4 of their
 scale.  Inputs and parameters are rounded to fp32 first, so that both sides
-see the same block.  Collected after the other GPU files."""
+see the same block.  Collected after the other parity files and before the
+no-allocation entry point's test, which runs last."""
 import numpy as np
 import pytest
 import torch
