@@ -563,6 +563,54 @@ realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_di
                                      int module, const float *W_module, const float *gf, const float *Wh,
                                      int64_t vocab, float *grad, float *loss, void *ws, size_t ws_bytes);
 
+/* ---- The sweep with Block-GD on the block ops' loss ----
+ * Alg. 1's column sweep for one linear module of decoder block l (Eq.
+ * gptq_update inside each block, the lazy batch update after it) with each
+ * Block-GD step (Eq. block_gd_update) descending the exact two-block window
+ * of Sec. 4.4, Eq. (slide_window) (next_block given) or, for the last
+ * decoder block, the true KL at the LM head of Eq. (kl_loss) (next_block
+ * NULL; App. "Pre-computation of the aggregated Fisher and
+ * last-transformer-block handling") in place of the layer-level surrogate.
+ * After block b (columns < b_end quantized; b_end < n), steps_per_block
+ * times: G = d loss / d W at W = W_work (the dequantized columns and the
+ * free ones), through block l's own backward (realq_block_module_window with
+ * alpha = 1 - (b_global - 1)/(B_total - 1), 1 when B_total = 1, b_global =
+ * b_global_start + b; or realq_block_module_kl), then one Adam (or SGD) step
+ * on the columns >= b_end of W_work with those columns of G.
+ *   dims, this_block, next_block, S, L, x, module, F_this, F_next
+ *             as realq_block_module_window.  The module's weight in
+ *             this_block (fp32) is both the loss's reference and the sweep's
+ *             W0; m x n is its shape (out x in).
+ *   head_gf, head_Wh, vocab   the final norm and LM head (next_block NULL);
+ *             ignored otherwise.
+ *   U, dead   realq_hessian_prepare of the module's input second moment
+ *             (its calibration inputs at block l's reference weights).
+ *   bcfg      steps_per_block >= 1; optimizer, lr, betas, eps,
+ *             b_global_start and B_total as for realq_quantize_layer.
+ *   W_work, adam_m, adam_v, adam_t, codes, scale, zero, W_deq, deq_dtype,
+ *   block_begin, block_end    as realq_quantize_layer (adam_m, adam_v and
+ *             adam_t are zeroed at block 0).
+ *   block_loss  NULL, or 2 device floats per column block: the loss before
+ *             and after the block's steps (blocks with no free columns after
+ *             them are left untouched; asking for them costs one more
+ *             evaluation of the loss per block).
+ *   ws        realq_quantize_window_workspace_size(dims, S, L, module, vocab,
+ *             qcfg) bytes (vocab 0 for the window), 256-byte aligned; its
+ *             first word is the sweep's status word (realq_workspace_status).
+ * Asynchronous on `stream`; argument errors are returned before any launch. */
+size_t realq_quantize_window_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L, int module,
+                                            int64_t vocab, const realq_quant_cfg_t *qcfg);
+realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_block_dims_t *dims,
+                                           const realq_block_weights_t *this_block,
+                                           const realq_block_weights_t *next_block, int64_t S, int64_t L,
+                                           const float *x, int module, const float *F_this, const float *F_next,
+                                           const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
+                                           const uint8_t *dead, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, float *block_loss, int64_t block_begin,
+                                           int64_t block_end, void *ws, size_t ws_bytes);
+
 #ifdef __cplusplus
 }
 #endif

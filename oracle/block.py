@@ -1,5 +1,6 @@
 """fp64 statement of one synthetic decoder block and of the exact two-block
-sliding-window loss (test infrastructure only; no CUDA counterpart yet).
+sliding-window loss (test infrastructure only: the CUDA path never imports
+it).
 
 Sec. 4.4, Eq. (slide_window): while quantizing block l the surrogate blends
 this block's Fisher loss with the next block's, L = alpha L(l) + (1 - alpha)

@@ -32,6 +32,7 @@ __all__ = [
     "realq_profile_collect", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
     "realq_block_window", "BLOCK_MODULES", "realq_block_module_workspace_size", "realq_block_head_workspace_size",
     "realq_block_module_window", "realq_block_head_kl", "realq_block_module_kl",
+    "realq_quantize_window_workspace_size", "realq_quantize_layer_window",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -151,6 +152,12 @@ _SIGS = {
     "realq_block_head_kl": ([_vp, _i64, _i64, _i64, _vp, _vp, _i64, _f32, _vp, _vp, _vp, _vp, _vp, _sz], _int),
     "realq_block_module_kl": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int,
                                _vp, _vp, _vp, _i64, _vp, _vp, _vp, _sz], _int),
+    "realq_quantize_window_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _int, _i64,
+                                              ctypes.POINTER(QuantCfg)], _sz),
+    "realq_quantize_layer_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
+                                     ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64,
+                                     _vp, _vp, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _P_i64,
+                                     _vp, _vp, _vp, _vp, _int, _vp, _i64, _i64, _vp, _sz], _int),
     "realq_status_string": ([_int], ctypes.c_char_p),
     "realq_last_error": ([], ctypes.c_char_p),
     "realq_launch_count": ([], _i64),
@@ -686,6 +693,55 @@ def realq_block_module_kl(dims: BlockDims, this_block: dict, x: torch.Tensor, mo
     _check(lib().realq_block_module_kl(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
                                        BLOCK_MODULES.index(module), _ptr(W_module), _ptr(gf), _ptr(Wh), Wh.shape[0],
                                        _ptr(grad), _ptr(loss), wp, wb))
+
+
+def realq_quantize_window_workspace_size(dims: BlockDims, S: int, L: int, module: str, qcfg: QuantCfg,
+                                         vocab: int = 0) -> int:
+    """Workspace bytes of realq_quantize_layer_window (vocab 0: the exact
+    window; the LM head's vocabulary: the final block's KL)."""
+    return int(lib().realq_quantize_window_workspace_size(ctypes.byref(dims), int(S), int(L),
+                                                          BLOCK_MODULES.index(module), int(vocab),
+                                                          ctypes.byref(qcfg)))
+
+
+def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: Optional[dict], x: torch.Tensor,
+                                module: str, U: torch.Tensor, qcfg: QuantCfg, bcfg: BgdCfg, W_work: torch.Tensor,
+                                codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *, F_this=None,
+                                F_next=None, head_gf=None, head_Wh=None, dead=None, adam_m=None, adam_v=None,
+                                adam_t: int = 0, W_deq=None, block_loss: Optional[torch.Tensor] = None,
+                                block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None) -> int:
+    """The column sweep of one module of decoder block l with Block-GD on the
+    exact two-block window (next_block given, with F_this and F_next) or on
+    the final block's KL at the LM head (next_block None, with head_gf and
+    head_Wh); x (S, L, d) is block l's input.  The module's weight in
+    this_block is the reference and the sweep's W0.  Runs blocks
+    [block_begin, block_end); returns the optimizer step counter."""
+    S, L, d = x.shape
+    Wref = this_block[{"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg",
+                       "up_proj": "Wu", "down_proj": "Wd"}[module]]
+    m, n = Wref.shape
+    nb = -(-n // qcfg.block_size)
+    if block_end is None:
+        block_end = nb
+    _need(W_work, torch.float32, (m, n), "W_work")
+    _need(U, torch.float32, (n, n), "U")
+    _need(codes, torch.uint8, (m, (n + 1) // 2), "codes")
+    _need(adam_m, torch.float32, (m, n), "adam_m")
+    _need(adam_v, torch.float32, (m, n), "adam_v")
+    _need(block_loss, torch.float32, (nb, 2), "block_loss")
+    t = ctypes.c_int64(adam_t)
+    wp, wb = _ws(ws)
+    a = _block_weights(this_block)
+    b = _block_weights(next_block) if next_block is not None else None
+    V = int(head_Wh.shape[0]) if head_Wh is not None else 0
+    _check(lib().realq_quantize_layer_window(
+        _stream(stream), ctypes.byref(dims), ctypes.byref(a), ctypes.byref(b) if b is not None else None, S, L,
+        _ptr(x), BLOCK_MODULES.index(module), _ptr(F_this), _ptr(F_next), _ptr(head_gf), _ptr(head_Wh), V,
+        _ptr(U), _ptr(dead), ctypes.byref(qcfg), ctypes.byref(bcfg), _ptr(W_work), _ptr(adam_m), _ptr(adam_v),
+        ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero), _ptr(W_deq),
+        _dtype(W_deq) if W_deq is not None else REALQ_F32, _ptr(block_loss), int(block_begin), int(block_end), wp,
+        wb))
+    return t.value
 
 
 def realq_workspace_status(ws: torch.Tensor, stream=None) -> int:

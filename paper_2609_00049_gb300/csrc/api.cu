@@ -3,6 +3,7 @@
 // accounting and optional per-kernel event timing.
 #include "kernels.cuh"
 
+#include <algorithm>
 #include <atomic>
 #include <cmath>
 #include <cstdarg>
@@ -418,6 +419,14 @@ struct TraceArgs {
     size_t ws_bytes;
 };
 
+// Called after each column block of the sweep (the OBS step and the lazy
+// batch update enqueued), on the sweep's stream: an optimizer step whose
+// gradient the sweep does not form itself.
+struct BlockHook {
+    realq_status_t (*fn)(cudaStream_t s, SweepPlan &p, int64_t b, void *ctx);
+    void *ctx;
+};
+
 static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n, const void *W0, realq_dtype_t w_dtype,
                                     int grouped, int rgroups, const float *Ug, const float *Hbar_g,
                                     const uint8_t *dead_g, int nmb, const float *Hbar_mb,
@@ -427,7 +436,7 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
                                     int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
                                     realq_dtype_t deq_dtype, int64_t block_begin, int64_t block_end, void *ws,
                                     size_t ws_bytes, const char *who, const TokArgs *tok = nullptr,
-                                    const TraceArgs *trace = nullptr) {
+                                    const TraceArgs *trace = nullptr, const BlockHook *hook = nullptr) {
     if (m <= 0 || n <= 0) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n must be > 0", who);
     if (m > (int64_t)1 << 30 || n > (int64_t)1 << 30) return fail(REALQ_ERR_INVALID_ARG, "%s: m, n too large", who);
     if (!valid_dtype(w_dtype) || !valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "%s: bad dtype", who);
@@ -506,7 +515,10 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     // (while profiling, everything stays on the caller's stream, so that each
     // launch's event interval is its own time; the arithmetic is the same)
     if (p.tc && p.bgd_steps > 0 && block_end - block_begin > 1 && !profiling()) REALQ_TRY(sweep_side_stream(s, p));
-    for (int64_t b = block_begin; b < block_end; ++b) REALQ_TRY(sweep_block(s, p, b));
+    for (int64_t b = block_begin; b < block_end; ++b) {
+        REALQ_TRY(sweep_block(s, p, b));
+        if (hook) REALQ_TRY(hook->fn(s, p, b, hook->ctx));
+    }
     REALQ_TRY(sweep_join_wide(s, p));
     return REALQ_OK;
 }
@@ -571,6 +583,131 @@ realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, 
     return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, n_minibatch, Hbar_mb, U, Hbar,
                          nullptr, dead, qcfg, bcfg, F, F_next, W_work, adam_m, adam_v, bgd_disp, adam_t, codes, scale,
                          zero, W_deq, deq_dtype, block_begin, block_end, ws, ws_bytes, "quantize_layer_minibatch");
+}
+
+// Block-GD on the block ops' loss (the exact window of Eq. slide_window or
+// the final block's KL of Eq. kl_loss): the after-block step of
+// realq_quantize_layer_window.
+struct WindowStep {
+    realq_stream_t stream;
+    const realq_block_dims_t *dims;
+    const realq_block_weights_t *this_block, *next_block;
+    int64_t S, L;
+    const float *x;
+    int module;
+    const float *F_this, *F_next, *gf, *Wh;
+    int64_t vocab;
+    realq_bgd_cfg_t cfg;
+    float *adam_m, *adam_v;
+    int64_t *adam_t;
+    float *grad, *block_loss;
+    void *mws;
+    size_t mws_bytes;
+};
+
+static realq_status_t window_loss(const WindowStep &w, const float *W, float alpha, float *loss) {
+    if (w.next_block)
+        return realq_block_module_window(w.stream, w.dims, w.this_block, w.next_block, w.S, w.L, w.x, w.module, W,
+                                         alpha, w.F_this, w.F_next, w.grad, loss, w.mws, w.mws_bytes);
+    return realq_block_module_kl(w.stream, w.dims, w.this_block, w.S, w.L, w.x, w.module, W, w.gf, w.Wh, w.vocab,
+                                 w.grad, loss, w.mws, w.mws_bytes);
+}
+
+static realq_status_t window_step(cudaStream_t s, SweepPlan &p, int64_t b, void *ctx) {
+    const WindowStep &w = *static_cast<const WindowStep *>(ctx);
+    const int64_t be = std::min<int64_t>((b + 1) * p.block, p.n);
+    if (be >= p.n) return REALQ_OK;   // no free columns after the last block
+    const int64_t b_global = w.cfg.b_global_start + b;
+    float alpha = 1.f;
+    if (w.cfg.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(w.cfg.B_total - 1));
+    float *bl = w.block_loss ? w.block_loss + 2 * b : nullptr;
+    for (int k = 0; k < w.cfg.steps_per_block; ++k) {
+        // the loss and its gradient at the current weights: the dequantized
+        // columns < be and the free ones
+        REALQ_TRY(window_loss(w, p.W, alpha, k == 0 ? bl : nullptr));
+        const int64_t t = ++(*w.adam_t);
+        REALQ_TRY(adam_cols(s, p.m, p.n, be, w.grad, p.W, w.adam_m, w.adam_v, w.cfg.lr, w.cfg.beta1, w.cfg.beta2,
+                            w.cfg.eps, t, w.cfg.optimizer == REALQ_OPT_SGD));
+    }
+    if (bl) REALQ_TRY(window_loss(w, p.W, alpha, bl + 1));
+    return REALQ_OK;
+}
+
+size_t realq_quantize_window_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L, int module,
+                                            int64_t vocab, const realq_quant_cfg_t *qcfg) {
+    if (!dims || !qcfg || module < 0 || module > 6 || vocab < 0) return 0;
+    const int64_t qw = dims->n_heads * dims->head_dim, kw = dims->n_kv * dims->head_dim;
+    const int64_t shape[7][2] = {{qw, dims->d}, {kw, dims->d}, {kw, dims->d}, {dims->d, qw},
+                                 {dims->ffn, dims->d}, {dims->ffn, dims->d}, {dims->d, dims->ffn}};
+    const int64_t m = shape[module][0], n = shape[module][1];
+    if (m <= 0 || n <= 0 || qcfg->block_size <= 0) return 0;
+    const size_t mod = realq_block_module_workspace_size(dims, S, L, vocab);
+    if (mod == 0) return 0;
+    return sweep_ws_bytes(m, n, qcfg->block_size, 0, 0, 0) + align_up((size_t)m * n * sizeof(float)) + mod;
+}
+
+realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_block_dims_t *dims,
+                                           const realq_block_weights_t *this_block,
+                                           const realq_block_weights_t *next_block, int64_t S, int64_t L,
+                                           const float *x, int module, const float *F_this, const float *F_next,
+                                           const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
+                                           const uint8_t *dead, const realq_quant_cfg_t *qcfg,
+                                           const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,
+                                           int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
+                                           realq_dtype_t deq_dtype, float *block_loss, int64_t block_begin,
+                                           int64_t block_end, void *ws, size_t ws_bytes) {
+    const char *who = "quantize_layer_window";
+    int64_t m = 0, n = 0;
+    size_t mws = 0;
+    REALQ_TRY(block_loss_check(dims, this_block, next_block, S, L, x, module, F_this, F_next, head_gf, head_Wh,
+                               next_block ? 0 : vocab, who, &m, &n, &mws));
+    if (m * n > ((int64_t)1 << 38)) return fail(REALQ_ERR_UNSUPPORTED, "%s: m n must be below 2^38", who);
+    REALQ_TRY(check_qcfg(qcfg, n));
+    REALQ_TRY(check_bcfg(bcfg));
+    if (!bcfg || bcfg->steps_per_block < 1)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: a Block-GD configuration with steps_per_block >= 1 required", who);
+    if (!adam_t) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL adam_t", who);
+    if (bcfg->optimizer == REALQ_OPT_ADAM && (!adam_m || !adam_v))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: Adam needs adam_m and adam_v", who);
+    if (!U || !W_work || !codes || !scale || !zero)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: NULL U, W_work, codes, scale or zero", who);
+    if (!valid_dtype(deq_dtype)) return fail(REALQ_ERR_INVALID_ARG, "%s: bad dtype", who);
+    const int64_t nb = (n + qcfg->block_size - 1) / qcfg->block_size;
+    if (block_begin < 0 || block_end > nb || block_begin > block_end)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: block range [%lld, %lld) outside [0, %lld)", who,
+                    (long long)block_begin, (long long)block_end, (long long)nb);
+    const size_t sw = sweep_ws_bytes(m, n, qcfg->block_size, 0, 0, 0);
+    const size_t gb = align_up((size_t)m * n * sizeof(float));
+    REALQ_TRY(check_ws(ws, ws_bytes, sw + gb + mws, who));
+    const float *W0 = nullptr;
+    switch (module) {
+        case 0: W0 = this_block->Wq; break;
+        case 1: W0 = this_block->Wk; break;
+        case 2: W0 = this_block->Wv; break;
+        case 3: W0 = this_block->Wo; break;
+        case 4: W0 = this_block->Wg; break;
+        case 5: W0 = this_block->Wu; break;
+        default: W0 = this_block->Wd; break;
+    }
+    char *base = static_cast<char *>(ws);
+    WindowStep w{stream, dims, this_block, next_block, S, L, x, module, F_this, F_next, head_gf, head_Wh, vocab,
+                 *bcfg, adam_m, adam_v, adam_t, reinterpret_cast<float *>(base + sw), block_loss, base + sw + gb,
+                 mws};
+    if (block_begin == 0) {
+        // (S is the sequence count here; the stream is cast directly)
+        cudaStream_t cs = static_cast<cudaStream_t>(stream);
+        *adam_t = 0;
+        if (bcfg->optimizer == REALQ_OPT_ADAM) {
+            REALQ_CUDA_TRY(cudaMemsetAsync(adam_m, 0, (size_t)m * n * sizeof(float), cs));
+            REALQ_CUDA_TRY(cudaMemsetAsync(adam_v, 0, (size_t)m * n * sizeof(float), cs));
+        }
+    }
+    const BlockHook hook{window_step, &w};
+    // the column sweep itself is the plain one (no layer-level Block-GD); the
+    // hook takes each block's optimizer steps
+    return quantize_impl(stream, m, n, W0, REALQ_F32, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, nullptr, nullptr,
+                         dead, qcfg, nullptr, nullptr, nullptr, W_work, nullptr, nullptr, nullptr, nullptr, codes,
+                         scale, zero, W_deq, deq_dtype, block_begin, block_end, ws, sw, who, nullptr, nullptr, &hook);
 }
 
 size_t realq_quantize_tokens_workspace_size(int64_t m, int64_t n, int64_t T_mb, const realq_quant_cfg_t *qcfg,

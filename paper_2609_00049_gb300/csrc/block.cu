@@ -2,7 +2,8 @@
 // launch executor of block_ops.cuh (one thread per flat index, the fp32 SIMT
 // GEMM for the projections) and the C ABI entry points realq_block_* of
 // include/realq.h (the block's forward, the next block's window, the
-// module-level window, the final block's KL head).
+// module-level window, the final block's KL head), and the optimizer step of
+// the sweep whose Block-GD gradient comes from those ops.
 #include "kernels.cuh"
 #include "block_ops.cuh"
 
@@ -47,6 +48,26 @@ struct DevExec {
         return st != REALQ_OK;
     }
 };
+
+__global__ void __launch_bounds__(256) adam_cols_kernel(int64_t m, int64_t r, int64_t n, int64_t c0, const float *G,
+                                                        float *W, float *mA, float *vA, float lr, float b1, float b2,
+                                                        float eps, float bc1, float bc2, int sgd) {
+    const int64_t idx = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (idx >= m * r) return;
+    const int64_t w = (idx / r) * n + c0 + idx % r;
+    const float g = G[w];
+    float step;
+    if (sgd) {
+        step = lr * g;
+    } else {
+        const float mv = b1 * mA[w] + (1.f - b1) * g;
+        const float vv = b2 * vA[w] + (1.f - b2) * g * g;
+        mA[w] = mv;
+        vA[w] = vv;
+        step = lr * (mv / bc1) / (sqrtf(vv / bc2) + eps);
+    }
+    W[w] -= step;
+}
 
 realq_status_t check_block(const realq_block_dims_t *dims, const realq_block_weights_t *w, int64_t S, int64_t L,
                            const char *who, blk::Dims *out) {
@@ -104,6 +125,49 @@ size_t module_ws(const blk::Dims &dm, int64_t vocab) {
 }
 
 }  // namespace
+
+realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_block_weights_t *this_block,
+                                const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
+                                int module, const float *F_this, const float *F_next, const float *gf, const float *Wh,
+                                int64_t vocab, const char *who, int64_t *m, int64_t *n, size_t *ws_bytes) {
+    blk::Dims dm{};
+    REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    if (module < blk::M_Q || module > blk::M_DOWN)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: module must be 0..6 (q, k, v, o, gate, up, down)", who);
+    if (!x) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x", who);
+    if (next_block) {
+        REALQ_TRY(check_block(dims, next_block, S, L, who, &dm));
+        if (!F_this || !F_next) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL F_this or F_next", who);
+        *ws_bytes = module_ws(dm, 0);
+    } else {
+        REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
+        *ws_bytes = module_ws(dm, vocab);
+    }
+    const int64_t qw = dm.qw(), kw = dm.kw();
+    switch (module) {
+        case blk::M_Q: *m = qw; *n = dm.d; break;
+        case blk::M_K: case blk::M_V: *m = kw; *n = dm.d; break;
+        case blk::M_O: *m = dm.d; *n = qw; break;
+        case blk::M_GATE: case blk::M_UP: *m = dm.f; *n = dm.d; break;
+        default: *m = dm.d; *n = dm.f; break;
+    }
+    return REALQ_OK;
+}
+
+realq_status_t adam_cols(cudaStream_t s, int64_t m, int64_t n, int64_t c0, const float *G, float *W, float *mA,
+                         float *vA, float lr, float b1, float b2, float eps, int64_t t, int sgd) {
+    const int64_t r = n - c0;
+    if (m <= 0 || r <= 0) return REALQ_OK;
+    const float bc1 = (float)(1.0 - std::pow((double)b1, (double)t));
+    const float bc2 = (float)(1.0 - std::pow((double)b2, (double)t));
+    {
+        Launch L("window_adam", s);
+        adam_cols_kernel<<<(unsigned)ceil_div(m * r, 256), 256, 0, s>>>(m, r, n, c0, G, W, mA, vA, lr, b1, b2, eps,
+                                                                        bc1, bc2, sgd);
+    }
+    return check_launch("window_adam");
+}
+
 }  // namespace realq
 
 using namespace realq;

@@ -118,6 +118,19 @@ realq_status_t prepare(cudaStream_t s, int64_t n, double norm, float damp, const
 realq_status_t prepare_deferred(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U,
                                 float *Hbar, uint8_t *dead, void *ws, size_t ws_bytes);
 realq_status_t scale_copy(cudaStream_t s, int64_t count, float mul, const float *in, float *out);
+// Host-side checks of the block ops' arguments for one module (the exact
+// window when next_block is given, else the final block's KL at the LM head
+// gf, Wh of vocab rows): the module's weight shape m x n and the block ops'
+// workspace bytes.  Launches nothing.
+realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_block_weights_t *this_block,
+                                const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
+                                int module, const float *F_this, const float *F_next, const float *gf, const float *Wh,
+                                int64_t vocab, const char *who, int64_t *m, int64_t *n, size_t *ws_bytes);
+// One Adam (or SGD) step of Eq. block_gd_update on the columns c0.. of the
+// m x n weights W with a full-width m x n gradient G (the block ops' module
+// gradient): PyTorch-form Adam with bias corrections for step t >= 1.
+realq_status_t adam_cols(cudaStream_t s, int64_t m, int64_t n, int64_t c0, const float *G, float *W, float *mA,
+                         float *vA, float lr, float b1, float b2, float eps, int64_t t, int sgd);
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,
                                uint8_t *dead, int64_t *fail_col);
 

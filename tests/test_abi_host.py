@@ -228,3 +228,44 @@ def test_block_module_and_head_entry_points_reject_bad_arguments(L):
     assert kl(None, 64, 2, 8, fake, fake, 100, 1e-6, fake, fake, fake, None, fake, 64) == rq.REALQ_ERR_WORKSPACE
     assert L.realq_block_module_kl(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, 3, fake, fake, None, 100,
                                    fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG     # NULL Wh
+
+
+def test_window_sweep_entry_point_rejects_bad_arguments(L):
+    # the sweep with Block-GD on the block ops' loss: every check is on the
+    # host, before any launch or memset
+    import paper_2609_00049_gb300 as rq
+    fake = ctypes.c_void_p(1 << 20)
+    w = rq.BlockWeights(*([fake.value] * 9))
+    ok = rq.block_dims(64, 4, 2, 16, 96)
+    q = rq.quant_cfg(group_size=64, block_size=64)
+    big = 1 << 40
+    t = ctypes.c_int64(0)
+
+    def sweep(module=6, nxt=True, F=fake, vocab=0, head=fake, bcfg=None, qcfg=q, blocks=(0, 2), nbytes=big,
+              deq_dtype=0, adam=fake):
+        b = bcfg if bcfg is not None else rq.bgd_cfg(1e-3)
+        return L.realq_quantize_layer_window(None, ctypes.byref(ok), ctypes.byref(w),
+                                             ctypes.byref(w) if nxt else None, 2, 8, fake, module, F, fake, head, head,
+                                             vocab, fake, None, ctypes.byref(qcfg), ctypes.byref(b), fake, adam, adam,
+                                             ctypes.byref(t), fake, fake, fake, None, deq_dtype, None, blocks[0],
+                                             blocks[1], fake, nbytes)
+
+    n_win = rq.realq_quantize_window_workspace_size(ok, 2, 8, "down_proj", q)
+    n_kl = rq.realq_quantize_window_workspace_size(ok, 2, 8, "down_proj", q, vocab=1000)
+    assert n_win > rq.realq_block_module_workspace_size(ok, 2, 8) + 64 * 96 * 4
+    assert n_kl > rq.realq_block_module_workspace_size(ok, 2, 8, 1000)
+    assert rq.realq_quantize_window_workspace_size(ok, 2, 8, "q_proj", q) < n_win   # 64 x 64 against 64 x 96
+    assert sweep(module=7) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(F=None) == rq.REALQ_ERR_INVALID_ARG                               # the window needs F, F'
+    assert sweep(nxt=False, vocab=0) == rq.REALQ_ERR_INVALID_ARG                   # the final block needs a head
+    assert sweep(nxt=False, vocab=100, head=None) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(bcfg=rq.bgd_cfg(1e-3, steps_per_block=0)) == rq.REALQ_ERR_INVALID_ARG
+    assert "steps_per_block >= 1" in rq.realq_last_error()
+    assert sweep(bcfg=rq.bgd_cfg(-1.0)) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(adam=None) == rq.REALQ_ERR_INVALID_ARG                             # Adam needs its moments
+    assert sweep(qcfg=rq.quant_cfg(block_size=96)) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(blocks=(0, 3)) == rq.REALQ_ERR_INVALID_ARG                         # down_proj: 96 columns, 2 blocks
+    assert sweep(deq_dtype=5) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(nbytes=n_win - 1) == rq.REALQ_ERR_WORKSPACE
+    assert "quantize_layer_window" in rq.realq_last_error()
+    assert t.value == 0
