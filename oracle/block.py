@@ -190,23 +190,30 @@ def next_block_loss(h: np.ndarray, dh_: np.ndarray, P_next: Dict, F_next: np.nda
 
 
 def sliding_window_down(W: np.ndarray, W0: np.ndarray, X: np.ndarray, R: np.ndarray, alpha: float,
-                        F_this: np.ndarray, F_next: np.ndarray, P_next: Dict):
+                        F_this: np.ndarray, F_next: np.ndarray, P_next: Dict, X_hat=None, R_hat=None):
     """The exact two-block sliding-window loss of a down_proj-type module and
     its gradient with respect to W (d x n).
 
     X: the module's inputs (S, L, n); R: block l's output without this
     module's contribution (S, L, d), so h = R + X W0^T is the reference output
     and R + X W^T the current one.  Block l's own Fisher loss is exact at the
-    module level here: Δh_t = (W - W0) x_t."""
+    module level here: Δh_t = (W - W0) x_t.  With the current pass's X_hat
+    and R_hat (the model quantized so far), the current output is
+    R_hat + X_hat W^T and Δh its difference from the reference."""
     S, L, n = X.shape
     T = S * L
-    dW = np.asarray(W, dtype=np.float64) - np.asarray(W0, dtype=np.float64)
-    dh_ = X @ dW.T
-    h = R + X @ np.asarray(W0, dtype=np.float64).T
+    W0 = np.asarray(W0, dtype=np.float64)
+    h = R + X @ W0.T
+    if X_hat is None and R_hat is None:
+        dh_ = X @ (np.asarray(W, dtype=np.float64) - W0).T
+        X_hat = X
+    else:
+        X_hat = X if X_hat is None else X_hat
+        dh_ = (R if R_hat is None else R_hat) + X_hat @ np.asarray(W, dtype=np.float64).T - h
     l_this = 0.5 * float(np.sum((dh_ @ F_this) * dh_)) / T
     l_next, g_next = next_block_loss(h, dh_, P_next, F_next)
     g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next
-    grad = np.einsum("sti,stj->ij", g_h, X)
+    grad = np.einsum("sti,stj->ij", g_h, X_hat)
     return alpha * l_this + (1.0 - alpha) * l_next, grad
 
 
@@ -214,22 +221,34 @@ _MODULE_WEIGHT = {"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo"
                   "up_proj": "Wu", "down_proj": "Wd"}
 
 
+def _current(module: str, W: np.ndarray, P_this: Dict, P_hat) -> Tuple[str, Dict]:
+    name = _MODULE_WEIGHT[module]
+    P_cur = dict(P_this if P_hat is None else P_hat)
+    P_cur[name] = np.asarray(W, dtype=np.float64)
+    return name, P_cur
+
+
 def sliding_window_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, P_next: Dict, alpha: float,
-                          F_this: np.ndarray, F_next: np.ndarray):
+                          F_this: np.ndarray, F_next: np.ndarray, x_hat=None, P_hat=None):
     """The exact two-block sliding-window loss of any linear module of block l
     and its gradient with respect to that module's weight.
 
     x: block l's input (S, L, d); P_this: block l with its reference (full
     precision) weights; W replaces the module's weight.  Block l's output is
-    h = B_l(x; W) and its reference h* = B_l(x; W0); the loss is
+    h = B_l(x̂; Ŵ) and its reference h* = B_l(x; W0); the loss is
       alpha (1/2T) sum_t Δh_t^T F_this Δh_t
         + (1 - alpha) (1/2T) sum_t (B_{l+1}(h)_t - B_{l+1}(h*)_t)^T F_next (...),
-    Δh = h - h*, both terms back-propagated through block l to W."""
-    name = _MODULE_WEIGHT[module]
-    P_cur = dict(P_this)
-    P_cur[name] = np.asarray(W, dtype=np.float64)
+    Δh = h - h*, both terms back-propagated through block l to W.
+
+    The current pass (Sec. 4.3: the surrogate is evaluated by a forward pass
+    through the current transformer block; Eq. fisher_loss: Δy_t = y_t - y*_t)
+    takes x_hat, block l's input in the model quantized so far (the
+    perturbed x̂ of Sec. 1), and P_hat, block l's weights with the modules
+    quantized so far; both default to the reference (x, P_this).  W
+    replaces the module's weight in P_hat."""
+    name, P_cur = _current(module, W, P_this, P_hat)
     h_ref, _ = block_forward(x, P_this)
-    h, cache = block_forward(x, P_cur)
+    h, cache = block_forward(x if x_hat is None else x_hat, P_cur)
     dh_ = h - h_ref
     T = x.shape[0] * x.shape[1]
     l_this = 0.5 * float(np.sum((dh_ @ F_this) * dh_)) / T
@@ -315,15 +334,15 @@ def fisher_tokens(h_ref: np.ndarray, head: Dict) -> np.ndarray:
     return F
 
 
-def kl_final_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, head: Dict):
+def kl_final_module(module: str, W: np.ndarray, x: np.ndarray, P_this: Dict, head: Dict, x_hat=None, P_hat=None):
     """The final block's loss for any linear module: the true KL at the LM
-    head between the reference block output and the one with W in place of
-    the module's weight, and its gradient with respect to W."""
-    name = _MODULE_WEIGHT[module]
-    P_cur = dict(P_this)
-    P_cur[name] = np.asarray(W, dtype=np.float64)
+    head between the reference block output and the current one (input
+    x_hat, weights P_hat with W in place of the module's weight; both default
+    to the reference, as in sliding_window_module), and its gradient with
+    respect to W."""
+    name, P_cur = _current(module, W, P_this, P_hat)
     h_ref, _ = block_forward(x, P_this)
-    h, cache = block_forward(x, P_cur)
+    h, cache = block_forward(x if x_hat is None else x_hat, P_cur)
     loss, g_h = kl_head_loss(h_ref, h - h_ref, head)
     _, grads = block_vjp(cache, g_h)
     return loss, grads[name]
@@ -337,25 +356,26 @@ _MODULE_INPUT = {"q_proj": "a", "k_proj": "a", "v_proj": "a", "o_proj": "o", "ga
 
 
 def module_inputs(module: str, x: np.ndarray, P: Dict) -> np.ndarray:
-    """The inputs of a module of block l at its reference weights, as the
-    (S L) x n token matrix whose second moment is the module's OBS Hessian."""
+    """The inputs of a module of block l with input x and weights P, as the
+    (S L) x n token matrix whose second moment is the module's OBS Hessian
+    (in the sequential pipeline: the current pass's x̂ and weights)."""
     _, cache = block_forward(x, P)
     a = cache[_MODULE_INPUT[module]]
     return a.reshape(-1, a.shape[-1])
 
 
 def window_gradient_fn(module: str, x: np.ndarray, P_this: Dict, P_next: Dict, F_this: np.ndarray,
-                       F_next: np.ndarray):
+                       F_next: np.ndarray, x_hat=None, P_hat=None):
     """(W, alpha) -> (loss, gradient) of the exact two-block window for the
     Block-GD step of the module's sweep (alpha is the step's blend weight)."""
     def fn(W, alpha):
-        return sliding_window_module(module, W, x, P_this, P_next, alpha, F_this, F_next)
+        return sliding_window_module(module, W, x, P_this, P_next, alpha, F_this, F_next, x_hat, P_hat)
     return fn
 
 
-def kl_gradient_fn(module: str, x: np.ndarray, P_this: Dict, head: Dict):
+def kl_gradient_fn(module: str, x: np.ndarray, P_this: Dict, head: Dict, x_hat=None, P_hat=None):
     """(W, alpha) -> (loss, gradient) of the final block's KL at the LM head
     (no window: alpha is not used)."""
     def fn(W, alpha):
-        return kl_final_module(module, W, x, P_this, head)
+        return kl_final_module(module, W, x, P_this, head, x_hat, P_hat)
     return fn

@@ -175,6 +175,93 @@ def test_module_window_agrees_with_the_down_proj_form():
     np.testing.assert_allclose(grad, grad2, rtol=1e-10, atol=1e-15)
 
 
+# --- the current pass: perturbed input, modules quantized so far -----------
+
+def _current_pass(r, P, x, skip):
+    # block l's input in the model quantized so far, and its weights with
+    # every other module moved off the reference
+    x_hat = x + 0.1 * r.standard_normal(x.shape)
+    P_hat = dict(P)
+    for k in ("Wq", "Wk", "Wv", "Wo", "Wg", "Wu", "Wd"):
+        if k != skip:
+            P_hat[k] = P[k] + 0.03 * r.standard_normal(P[k].shape)
+    return x_hat, P_hat
+
+
+@pytest.mark.parametrize("module", ["q_proj", "o_proj", "up_proj", "down_proj"])
+def test_current_pass_window_gradient_matches_finite_differences(module):
+    r, P, Pn, x, F, Fn = _module_case(21)
+    name = ob._MODULE_WEIGHT[module]
+    x_hat, P_hat = _current_pass(r, P, x, name)
+    W = P[name] + r.standard_normal(P[name].shape) * 0.05
+    args = (x, P, Pn, 0.6, F, Fn, x_hat, P_hat)
+    loss, grad = ob.sliding_window_module(module, W, *args)
+    # at the module's reference weight the loss is still positive: the input
+    # and the other modules differ from the reference
+    assert ob.sliding_window_module(module, P[name], *args)[0] > 0
+    e = 1e-6
+    for _ in range(4):
+        i, j = int(r.integers(0, W.shape[0])), int(r.integers(0, W.shape[1]))
+        E = np.zeros_like(W)
+        E[i, j] = e
+        fd = (ob.sliding_window_module(module, W + E, *args)[0] -
+              ob.sliding_window_module(module, W - E, *args)[0]) / (2 * e)
+        assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-3, abs(fd)), (module, i, j, fd, grad[i, j])
+
+
+def test_current_pass_agrees_with_the_down_proj_form():
+    # Δh = (R̂ + X̂ Wᵀ) - (R + X W0ᵀ): the down_proj form from the two passes'
+    # cached SwiGLU products and residuals against the block-level statement
+    r, P, Pn, x, F, Fn = _module_case(22)
+    x_hat, P_hat = _current_pass(r, P, x, "Wd")
+    W = P["Wd"] + r.standard_normal(P["Wd"].shape) * 0.05
+    loss, grad = ob.sliding_window_module("down_proj", W, x, P, Pn, 0.35, F, Fn, x_hat, P_hat)
+    y, cache = ob.block_forward(x, P)
+    y_hat, cache_hat = ob.block_forward(x_hat, P_hat)
+    R = y - cache["m"] @ P["Wd"].T
+    R_hat = y_hat - cache_hat["m"] @ P_hat["Wd"].T
+    loss2, grad2 = ob.sliding_window_down(W, P["Wd"], cache["m"], R, 0.35, F, Fn, Pn, cache_hat["m"], R_hat)
+    assert abs(loss - loss2) <= 1e-10 * abs(loss)
+    np.testing.assert_allclose(grad, grad2, rtol=1e-8, atol=1e-12 * np.abs(grad).max())
+
+
+@pytest.mark.parametrize("module", ["k_proj", "gate_proj"])
+def test_current_pass_kl_gradient_matches_finite_differences(module):
+    r, P, _, x, _, _ = _module_case(23)
+    head = ob.head_params(r, x.shape[2], 11, scale=1.5)
+    name = ob._MODULE_WEIGHT[module]
+    x_hat, P_hat = _current_pass(r, P, x, name)
+    W = P[name] + r.standard_normal(P[name].shape) * 0.05
+    loss, grad = ob.kl_final_module(module, W, x, P, head, x_hat, P_hat)
+    assert loss > 0
+    e = 1e-6
+    for _ in range(4):
+        i, j = int(r.integers(0, W.shape[0])), int(r.integers(0, W.shape[1]))
+        E = np.zeros_like(W)
+        E[i, j] = e
+        fd = (ob.kl_final_module(module, W + E, x, P, head, x_hat, P_hat)[0] -
+              ob.kl_final_module(module, W - E, x, P, head, x_hat, P_hat)[0]) / (2 * e)
+        assert abs(fd - grad[i, j]) <= 1e-6 * max(1e-4, abs(fd)), (module, i, j, fd, grad[i, j])
+
+
+def test_current_pass_kl_agrees_with_the_down_proj_form():
+    # down_proj's KL gradient is the head's gradient in Δh times the current
+    # pass's SwiGLU product, Σ_t g_t m̂_tᵀ, with no backward through block l
+    r, P, _, x, _, _ = _module_case(24)
+    head = ob.head_params(r, x.shape[2], 11, scale=1.5)
+    x_hat, P_hat = _current_pass(r, P, x, "Wd")
+    W = P["Wd"] + r.standard_normal(P["Wd"].shape) * 0.05
+    loss, grad = ob.kl_final_module("down_proj", W, x, P, head, x_hat, P_hat)
+    y, _ = ob.block_forward(x, P)
+    y_hat, cache_hat = ob.block_forward(x_hat, P_hat)
+    m_hat = cache_hat["m"]
+    h = y_hat + m_hat @ (W - P_hat["Wd"]).T
+    loss2, g_h = ob.kl_head_loss(y, h - y, head)
+    assert abs(loss - loss2) <= 1e-10 * abs(loss)
+    np.testing.assert_allclose(grad, np.einsum("sti,stj->ij", g_h, m_hat), rtol=1e-8,
+                               atol=1e-12 * np.abs(grad).max())
+
+
 # --- the final block: the true KL at the LM head ---------------------------
 
 def _head_case(seed, d=6, V=7, S=2, L=3):

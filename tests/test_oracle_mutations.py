@@ -70,8 +70,15 @@ BLOCK_MUTATIONS = {
     "window_blend": ("g_h = alpha * (dh_ @ F_this) / T + (1.0 - alpha) * g_next\n    grad =",
                      "g_h = alpha * (dh_ @ F_this) / T + alpha * g_next\n    grad ="),
     # the module-level window with the current weights as its reference
-    "module_reference": ("h_ref, _ = block_forward(x, P_this)\n    h, cache = block_forward(x, P_cur)\n    dh_",
-                         "h_ref, _ = block_forward(x, P_cur)\n    h, cache = block_forward(x, P_cur)\n    dh_"),
+    "module_reference": ("h_ref, _ = block_forward(x, P_this)\n    h, cache = block_forward(x if x_hat is None else "
+                         "x_hat, P_cur)\n    dh_",
+                         "h_ref, _ = block_forward(x, P_cur)\n    h, cache = block_forward(x if x_hat is None else "
+                         "x_hat, P_cur)\n    dh_"),
+    # the current pass run on the reference input instead of the perturbed one
+    "current_input": ("h, cache = block_forward(x if x_hat is None else x_hat, P_cur)\n    dh_",
+                      "h, cache = block_forward(x, P_cur)\n    dh_"),
+    "kl_current_input": ("h, cache = block_forward(x if x_hat is None else x_hat, P_cur)\n    loss, g_h",
+                         "h, cache = block_forward(x, P_cur)\n    loss, g_h"),
     # the KL head: the gradient's sign, the head's norm left out of the
     # backward, the Fisher's label weights dropped, the KL's direction swapped
     "kl_gradient_sign": ("gz = (np.exp(_log_softmax(z1)) - np.exp(_log_softmax(z0))) / T",
