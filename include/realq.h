@@ -523,17 +523,24 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
                                   size_t ws_bytes);
 
 /* Module level (any linear module of block l, Eq. slide_window): block l is
- * run at its reference weights (h*) and with the module's weight replaced
- * by W_module (h), dh = h - h*, and
+ * run at its reference weights on its reference input (h*, the full-precision
+ * model) and as the current block (h: Sec. 4.3 evaluates the surrogate by a
+ * forward pass through the current transformer block, on the perturbed
+ * inputs that the quantized earlier blocks produce), dh = h - h*, and
  *   loss = alpha (1/2T) sum_t dh_t^T F_this dh_t + (1 - alpha) L(l+1)(h*, dh),
  *   grad = d loss / d W_module, back-propagated through block l's own
  *          backward (grad has W_module's shape).
  *   module    0..6 = q_proj, k_proj, v_proj, o_proj, gate_proj, up_proj,
  *             down_proj; W_module has that weight's shape (out x in).
  *   this_block, next_block
- *             both blocks' weights (same dims); this_block holds the
- *             reference weight of the module.
- *   x         block l's input, S L x d.
+ *             both blocks' weights (same dims), at full precision;
+ *             this_block holds the reference weight of the module.
+ *   this_block_hat
+ *             block l's weights in the current pass (the modules quantized
+ *             so far), or NULL (= this_block); the module's own entry is
+ *             replaced by W_module either way.
+ *   x, x_hat  block l's reference input and its input in the current pass
+ *             (the model quantized so far), S L x d; x_hat NULL (= x).
  *   alpha     the window's weight in [0, 1].
  *   ws        realq_block_module_workspace_size(dims, S, L, 0) bytes.
  * The final block (App. "Pre-computation of the aggregated Fisher and
@@ -552,16 +559,20 @@ size_t realq_block_module_workspace_size(const realq_block_dims_t *dims, int64_t
 size_t realq_block_head_workspace_size(int64_t d, int64_t S, int64_t L, int64_t vocab);
 realq_status_t realq_block_module_window(realq_stream_t stream, const realq_block_dims_t *dims,
                                          const realq_block_weights_t *this_block,
+                                         const realq_block_weights_t *this_block_hat,
                                          const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
-                                         int module, const float *W_module, float alpha, const float *F_this,
-                                         const float *F_next, float *grad, float *loss, void *ws, size_t ws_bytes);
+                                         const float *x_hat, int module, const float *W_module, float alpha,
+                                         const float *F_this, const float *F_next, float *grad, float *loss, void *ws,
+                                         size_t ws_bytes);
 realq_status_t realq_block_head_kl(realq_stream_t stream, int64_t d, int64_t S, int64_t L, const float *gf,
                                    const float *Wh, int64_t vocab, float rms_eps, const float *h_ref, const float *dh,
                                    float *g_h, float *loss, void *ws, size_t ws_bytes);
 realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_dims_t *dims,
-                                     const realq_block_weights_t *this_block, int64_t S, int64_t L, const float *x,
-                                     int module, const float *W_module, const float *gf, const float *Wh,
-                                     int64_t vocab, float *grad, float *loss, void *ws, size_t ws_bytes);
+                                     const realq_block_weights_t *this_block,
+                                     const realq_block_weights_t *this_block_hat, int64_t S, int64_t L,
+                                     const float *x, const float *x_hat, int module, const float *W_module,
+                                     const float *gf, const float *Wh, int64_t vocab, float *grad, float *loss,
+                                     void *ws, size_t ws_bytes);
 
 /* ---- The sweep with Block-GD on the block ops' loss ----
  * Alg. 1's column sweep for one linear module of decoder block l (Eq.
@@ -577,14 +588,15 @@ realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_di
  * alpha = 1 - (b_global - 1)/(B_total - 1), 1 when B_total = 1, b_global =
  * b_global_start + b; or realq_block_module_kl), then one Adam (or SGD) step
  * on the columns >= b_end of W_work with those columns of G.
- *   dims, this_block, next_block, S, L, x, module, F_this, F_next
+ *   dims, this_block, this_block_hat, next_block, S, L, x, x_hat, module,
+ *   F_this, F_next
  *             as realq_block_module_window.  The module's weight in
  *             this_block (fp32) is both the loss's reference and the sweep's
  *             W0; m x n is its shape (out x in).
  *   head_gf, head_Wh, vocab   the final norm and LM head (next_block NULL);
  *             ignored otherwise.
  *   U, dead   realq_hessian_prepare of the module's input second moment
- *             (its calibration inputs at block l's reference weights).
+ *             (its calibration inputs in the current pass).
  *   bcfg      steps_per_block >= 1; optimizer, lr, betas, eps,
  *             b_global_start and B_total as for realq_quantize_layer.
  *   W_work, adam_m, adam_v, adam_t, codes, scale, zero, W_deq, deq_dtype,
@@ -602,8 +614,10 @@ size_t realq_quantize_window_workspace_size(const realq_block_dims_t *dims, int6
                                             int64_t vocab, const realq_quant_cfg_t *qcfg);
 realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_block_dims_t *dims,
                                            const realq_block_weights_t *this_block,
+                                           const realq_block_weights_t *this_block_hat,
                                            const realq_block_weights_t *next_block, int64_t S, int64_t L,
-                                           const float *x, int module, const float *F_this, const float *F_next,
+                                           const float *x, const float *x_hat, int module, const float *F_this,
+                                           const float *F_next,
                                            const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
                                            const uint8_t *dead, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,

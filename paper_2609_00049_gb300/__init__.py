@@ -147,15 +147,17 @@ _SIGS = {
     "realq_block_module_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _i64], _sz),
     "realq_block_head_workspace_size": ([_i64, _i64, _i64, _i64], _sz),
     "realq_block_module_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
-                                   ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int, _vp, _f32, _vp, _vp, _vp, _vp,
-                                   _vp, _sz], _int),
+                                   ctypes.POINTER(BlockWeights), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
+                                   _int, _vp, _f32, _vp, _vp, _vp, _vp, _vp, _sz], _int),
     "realq_block_head_kl": ([_vp, _i64, _i64, _i64, _vp, _vp, _i64, _f32, _vp, _vp, _vp, _vp, _vp, _sz], _int),
-    "realq_block_module_kl": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int,
-                               _vp, _vp, _vp, _i64, _vp, _vp, _vp, _sz], _int),
+    "realq_block_module_kl": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
+                               ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _i64, _vp, _vp,
+                               _vp, _sz], _int),
     "realq_quantize_window_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _int, _i64,
                                               ctypes.POINTER(QuantCfg)], _sz),
     "realq_quantize_layer_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
-                                     ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64,
+                                     ctypes.POINTER(BlockWeights), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
+                                     _int, _vp, _vp, _vp, _vp, _i64,
                                      _vp, _vp, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _P_i64,
                                      _vp, _vp, _vp, _vp, _int, _vp, _i64, _i64, _vp, _sz], _int),
     "realq_status_string": ([_int], ctypes.c_char_p),
@@ -654,19 +656,27 @@ def realq_block_head_workspace_size(d: int, S: int, L: int, vocab: int) -> int:
     return int(lib().realq_block_head_workspace_size(int(d), int(S), int(L), int(vocab)))
 
 
+def _opt_weights(w: Optional[dict]):
+    return ctypes.byref(_block_weights(w)) if w is not None else None
+
+
 def realq_block_module_window(dims: BlockDims, this_block: dict, next_block: dict, x: torch.Tensor, module: str,
                               W_module: torch.Tensor, alpha: float, F_this: torch.Tensor, F_next: torch.Tensor,
                               grad: torch.Tensor, ws: torch.Tensor, loss: Optional[torch.Tensor] = None,
+                              this_block_hat: Optional[dict] = None, x_hat: Optional[torch.Tensor] = None,
                               stream=None):
     """The exact two-block window of one module of block l: its loss into
-    loss (or None) and its gradient in W_module into grad (W_module's shape)."""
+    loss (or None) and its gradient in W_module into grad (W_module's shape).
+    this_block_hat / x_hat: block l's weights and input in the current pass
+    (the model quantized so far); None: the reference ones."""
     S, L, d = x.shape
     _need(grad, torch.float32, tuple(W_module.shape), "grad")
     wp, wb = _ws(ws)
     a, b = _block_weights(this_block), _block_weights(next_block)
-    _check(lib().realq_block_module_window(_stream(stream), ctypes.byref(dims), ctypes.byref(a), ctypes.byref(b), S, L,
-                                           _ptr(x), BLOCK_MODULES.index(module), _ptr(W_module), float(alpha),
-                                           _ptr(F_this), _ptr(F_next), _ptr(grad), _ptr(loss), wp, wb))
+    _check(lib().realq_block_module_window(_stream(stream), ctypes.byref(dims), ctypes.byref(a),
+                                           _opt_weights(this_block_hat), ctypes.byref(b), S, L, _ptr(x), _ptr(x_hat),
+                                           BLOCK_MODULES.index(module), _ptr(W_module), float(alpha), _ptr(F_this),
+                                           _ptr(F_next), _ptr(grad), _ptr(loss), wp, wb))
 
 
 def realq_block_head_kl(gf: torch.Tensor, Wh: torch.Tensor, h_ref: torch.Tensor, dh: torch.Tensor,
@@ -684,13 +694,16 @@ def realq_block_head_kl(gf: torch.Tensor, Wh: torch.Tensor, h_ref: torch.Tensor,
 
 def realq_block_module_kl(dims: BlockDims, this_block: dict, x: torch.Tensor, module: str, W_module: torch.Tensor,
                           gf: torch.Tensor, Wh: torch.Tensor, grad: torch.Tensor, ws: torch.Tensor,
-                          loss: Optional[torch.Tensor] = None, stream=None):
-    """The final block's KL for one module's weight, and its gradient."""
+                          loss: Optional[torch.Tensor] = None, this_block_hat: Optional[dict] = None,
+                          x_hat: Optional[torch.Tensor] = None, stream=None):
+    """The final block's KL for one module's weight, and its gradient
+    (this_block_hat / x_hat as for realq_block_module_window)."""
     S, L, d = x.shape
     _need(grad, torch.float32, tuple(W_module.shape), "grad")
     wp, wb = _ws(ws)
     a = _block_weights(this_block)
-    _check(lib().realq_block_module_kl(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
+    _check(lib().realq_block_module_kl(_stream(stream), ctypes.byref(dims), ctypes.byref(a),
+                                       _opt_weights(this_block_hat), S, L, _ptr(x), _ptr(x_hat),
                                        BLOCK_MODULES.index(module), _ptr(W_module), _ptr(gf), _ptr(Wh), Wh.shape[0],
                                        _ptr(grad), _ptr(loss), wp, wb))
 
@@ -709,13 +722,17 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
                                 codes: torch.Tensor, scale: torch.Tensor, zero: torch.Tensor, *, F_this=None,
                                 F_next=None, head_gf=None, head_Wh=None, dead=None, adam_m=None, adam_v=None,
                                 adam_t: int = 0, W_deq=None, block_loss: Optional[torch.Tensor] = None,
-                                block_begin: int = 0, block_end: Optional[int] = None, ws=None, stream=None) -> int:
+                                block_begin: int = 0, block_end: Optional[int] = None, ws=None,
+                                this_block_hat: Optional[dict] = None, x_hat: Optional[torch.Tensor] = None,
+                                stream=None) -> int:
     """The column sweep of one module of decoder block l with Block-GD on the
     exact two-block window (next_block given, with F_this and F_next) or on
     the final block's KL at the LM head (next_block None, with head_gf and
     head_Wh); x (S, L, d) is block l's input.  The module's weight in
-    this_block is the reference and the sweep's W0.  Runs blocks
-    [block_begin, block_end); returns the optimizer step counter."""
+    this_block is the reference and the sweep's W0; this_block_hat / x_hat
+    are block l's weights and input in the current pass (the model quantized
+    so far; None: the reference ones).  Runs blocks [block_begin, block_end);
+    returns the optimizer step counter."""
     S, L, d = x.shape
     Wref = this_block[{"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg",
                        "up_proj": "Wu", "down_proj": "Wd"}[module]]
@@ -735,8 +752,9 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
     b = _block_weights(next_block) if next_block is not None else None
     V = int(head_Wh.shape[0]) if head_Wh is not None else 0
     _check(lib().realq_quantize_layer_window(
-        _stream(stream), ctypes.byref(dims), ctypes.byref(a), ctypes.byref(b) if b is not None else None, S, L,
-        _ptr(x), BLOCK_MODULES.index(module), _ptr(F_this), _ptr(F_next), _ptr(head_gf), _ptr(head_Wh), V,
+        _stream(stream), ctypes.byref(dims), ctypes.byref(a), _opt_weights(this_block_hat),
+        ctypes.byref(b) if b is not None else None, S, L, _ptr(x), _ptr(x_hat), BLOCK_MODULES.index(module),
+        _ptr(F_this), _ptr(F_next), _ptr(head_gf), _ptr(head_Wh), V,
         _ptr(U), _ptr(dead), ctypes.byref(qcfg), ctypes.byref(bcfg), _ptr(W_work), _ptr(adam_m), _ptr(adam_v),
         ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero), _ptr(W_deq),
         _dtype(W_deq) if W_deq is not None else REALQ_F32, _ptr(block_loss), int(block_begin), int(block_end), wp,

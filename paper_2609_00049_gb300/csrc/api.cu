@@ -591,9 +591,9 @@ realq_status_t realq_quantize_layer_minibatch(realq_stream_t stream, int64_t m, 
 struct WindowStep {
     realq_stream_t stream;
     const realq_block_dims_t *dims;
-    const realq_block_weights_t *this_block, *next_block;
+    const realq_block_weights_t *this_block, *this_block_hat, *next_block;
     int64_t S, L;
-    const float *x;
+    const float *x, *x_hat;
     int module;
     const float *F_this, *F_next, *gf, *Wh;
     int64_t vocab;
@@ -607,10 +607,11 @@ struct WindowStep {
 
 static realq_status_t window_loss(const WindowStep &w, const float *W, float alpha, float *loss) {
     if (w.next_block)
-        return realq_block_module_window(w.stream, w.dims, w.this_block, w.next_block, w.S, w.L, w.x, w.module, W,
-                                         alpha, w.F_this, w.F_next, w.grad, loss, w.mws, w.mws_bytes);
-    return realq_block_module_kl(w.stream, w.dims, w.this_block, w.S, w.L, w.x, w.module, W, w.gf, w.Wh, w.vocab,
-                                 w.grad, loss, w.mws, w.mws_bytes);
+        return realq_block_module_window(w.stream, w.dims, w.this_block, w.this_block_hat, w.next_block, w.S, w.L,
+                                         w.x, w.x_hat, w.module, W, alpha, w.F_this, w.F_next, w.grad, loss, w.mws,
+                                         w.mws_bytes);
+    return realq_block_module_kl(w.stream, w.dims, w.this_block, w.this_block_hat, w.S, w.L, w.x, w.x_hat, w.module,
+                                 W, w.gf, w.Wh, w.vocab, w.grad, loss, w.mws, w.mws_bytes);
 }
 
 static realq_status_t window_step(cudaStream_t s, SweepPlan &p, int64_t b, void *ctx) {
@@ -648,8 +649,10 @@ size_t realq_quantize_window_workspace_size(const realq_block_dims_t *dims, int6
 
 realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_block_dims_t *dims,
                                            const realq_block_weights_t *this_block,
+                                           const realq_block_weights_t *this_block_hat,
                                            const realq_block_weights_t *next_block, int64_t S, int64_t L,
-                                           const float *x, int module, const float *F_this, const float *F_next,
+                                           const float *x, const float *x_hat, int module, const float *F_this,
+                                           const float *F_next,
                                            const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
                                            const uint8_t *dead, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,
@@ -659,8 +662,8 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
     const char *who = "quantize_layer_window";
     int64_t m = 0, n = 0;
     size_t mws = 0;
-    REALQ_TRY(block_loss_check(dims, this_block, next_block, S, L, x, module, F_this, F_next, head_gf, head_Wh,
-                               next_block ? 0 : vocab, who, &m, &n, &mws));
+    REALQ_TRY(block_loss_check(dims, this_block, this_block_hat, next_block, S, L, x, module, F_this, F_next, head_gf,
+                               head_Wh, next_block ? 0 : vocab, who, &m, &n, &mws));
     if (m * n > ((int64_t)1 << 38)) return fail(REALQ_ERR_UNSUPPORTED, "%s: m n must be below 2^38", who);
     REALQ_TRY(check_qcfg(qcfg, n));
     REALQ_TRY(check_bcfg(bcfg));
@@ -690,9 +693,9 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
         default: W0 = this_block->Wd; break;
     }
     char *base = static_cast<char *>(ws);
-    WindowStep w{stream, dims, this_block, next_block, S, L, x, module, F_this, F_next, head_gf, head_Wh, vocab,
-                 *bcfg, adam_m, adam_v, adam_t, reinterpret_cast<float *>(base + sw), block_loss, base + sw + gb,
-                 mws};
+    WindowStep w{stream, dims, this_block, this_block_hat, next_block, S, L, x, x_hat, module, F_this, F_next,
+                 head_gf, head_Wh, vocab, *bcfg, adam_m, adam_v, adam_t, reinterpret_cast<float *>(base + sw),
+                 block_loss, base + sw + gb, mws};
     if (block_begin == 0) {
         // (S is the sequence count here; the stream is cast directly)
         cudaStream_t cs = static_cast<cudaStream_t>(stream);

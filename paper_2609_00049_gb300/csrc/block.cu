@@ -127,11 +127,13 @@ size_t module_ws(const blk::Dims &dm, int64_t vocab) {
 }  // namespace
 
 realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_block_weights_t *this_block,
-                                const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
-                                int module, const float *F_this, const float *F_next, const float *gf, const float *Wh,
-                                int64_t vocab, const char *who, int64_t *m, int64_t *n, size_t *ws_bytes) {
+                                const realq_block_weights_t *this_block_hat, const realq_block_weights_t *next_block,
+                                int64_t S, int64_t L, const float *x, int module, const float *F_this,
+                                const float *F_next, const float *gf, const float *Wh, int64_t vocab, const char *who,
+                                int64_t *m, int64_t *n, size_t *ws_bytes) {
     blk::Dims dm{};
     REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    if (this_block_hat) REALQ_TRY(check_block(dims, this_block_hat, S, L, who, &dm));
     if (module < blk::M_Q || module > blk::M_DOWN)
         return fail(REALQ_ERR_INVALID_ARG, "%s: module must be 0..6 (q, k, v, o, gate, up, down)", who);
     if (!x) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x", who);
@@ -235,12 +237,15 @@ size_t realq_block_head_workspace_size(int64_t d, int64_t S, int64_t L, int64_t 
 
 realq_status_t realq_block_module_window(realq_stream_t stream, const realq_block_dims_t *dims,
                                          const realq_block_weights_t *this_block,
+                                         const realq_block_weights_t *this_block_hat,
                                          const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
-                                         int module, const float *W_module, float alpha, const float *F_this,
-                                         const float *F_next, float *grad, float *loss, void *ws, size_t ws_bytes) {
+                                         const float *x_hat, int module, const float *W_module, float alpha,
+                                         const float *F_this, const float *F_next, float *grad, float *loss, void *ws,
+                                         size_t ws_bytes) {
     const char *who = "block_module_window";
     blk::Dims dm{};
     REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    if (this_block_hat) REALQ_TRY(check_block(dims, this_block_hat, S, L, who, &dm));
     REALQ_TRY(check_block(dims, next_block, S, L, who, &dm));
     REALQ_TRY(check_module(module, W_module, grad, who));
     if (!x || !F_this || !F_next) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x, F_this or F_next", who);
@@ -254,8 +259,9 @@ realq_status_t realq_block_module_window(realq_stream_t stream, const realq_bloc
     blk::carve_module(dm, p, &M);
     DevExec X{static_cast<cudaStream_t>(stream)};
     const blk::Weights Wref = weights_of(this_block);
-    blk::module_window(X, dm, Wref, blk::with_module(Wref, module, W_module), weights_of(next_block), Bl, Bn, M, x,
-                       module, alpha, F_this, F_next, grad, loss);
+    const blk::Weights Wcur = weights_of(this_block_hat ? this_block_hat : this_block);
+    blk::module_window(X, dm, Wref, blk::with_module(Wcur, module, W_module), weights_of(next_block), Bl, Bn, M, x,
+                       x_hat ? x_hat : x, module, alpha, F_this, F_next, grad, loss);
     return X.st;
 }
 
@@ -278,12 +284,15 @@ realq_status_t realq_block_head_kl(realq_stream_t stream, int64_t d, int64_t S, 
 }
 
 realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_dims_t *dims,
-                                     const realq_block_weights_t *this_block, int64_t S, int64_t L, const float *x,
-                                     int module, const float *W_module, const float *gf, const float *Wh,
-                                     int64_t vocab, float *grad, float *loss, void *ws, size_t ws_bytes) {
+                                     const realq_block_weights_t *this_block,
+                                     const realq_block_weights_t *this_block_hat, int64_t S, int64_t L,
+                                     const float *x, const float *x_hat, int module, const float *W_module,
+                                     const float *gf, const float *Wh, int64_t vocab, float *grad, float *loss,
+                                     void *ws, size_t ws_bytes) {
     const char *who = "block_module_kl";
     blk::Dims dm{};
     REALQ_TRY(check_block(dims, this_block, S, L, who, &dm));
+    if (this_block_hat) REALQ_TRY(check_block(dims, this_block_hat, S, L, who, &dm));
     REALQ_TRY(check_module(module, W_module, grad, who));
     REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
     if (!x) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x", who);
@@ -297,8 +306,9 @@ realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_di
     blk::carve_head(dm, vocab, p, &H);
     DevExec X{static_cast<cudaStream_t>(stream)};
     const blk::Weights Wref = weights_of(this_block);
-    blk::module_kl(X, dm, Wref, blk::with_module(Wref, module, W_module), Bl, M, blk::Head{gf, Wh, vocab}, H, x,
-                   module, grad, loss);
+    const blk::Weights Wcur = weights_of(this_block_hat ? this_block_hat : this_block);
+    blk::module_kl(X, dm, Wref, blk::with_module(Wcur, module, W_module), Bl, M, blk::Head{gf, Wh, vocab}, H, x,
+                   x_hat ? x_hat : x, module, grad, loss);
     return X.st;
 }
 

@@ -619,18 +619,20 @@ int kl_head(X &x, const Dims &dm, const Head &hd, const HeadBuffers &H, const fl
     return e;
 }
 
-// block l at its reference weights and with one module's weight replaced:
-// h* into M.href, Δh = h - h* into M.dh, and block l's caches (of the
-// perturbed pass) left in Bl for the module's backward
+// block l's reference pass (full-precision weights Wref on the reference
+// input xin) and its current pass (Wcur, the weights quantized so far with
+// the module's weight replaced, on the perturbed input xhat; Sec. 4.3): h*
+// into M.href, Δh = h - h* into M.dh, and the current pass's caches left in
+// Bl for the module's backward
 template <class X>
 int module_delta(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Buffers &Bl,
-                 const ModuleBuffers &M, const float *xin) {
+                 const ModuleBuffers &M, const float *xin, const float *xhat) {
     const int64_t T = dm.T(), d = dm.d;
     int e = 0;
     e |= setup(x, dm, Wref, Bl);
     e |= forward(x, dm, Wref, Bl, xin, M.href);
     e |= setup(x, dm, Wcur, Bl);
-    e |= forward(x, dm, Wcur, Bl, xin, M.dh);
+    e |= forward(x, dm, Wcur, Bl, xhat, M.dh);
     e |= x.map(T * d, Axpy{M.dh, M.href, M.dh, -1.f}, "blk_axpy");
     return e;
 }
@@ -639,14 +641,15 @@ int module_delta(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur,
 // slide_window), its loss and the gradient in the module's weight:
 //   loss = alpha (1/2T) sum_t Δh_t^T F Δh_t + (1 - alpha) L(l+1)(h*, Δh),
 //   g_h = alpha Δh F / T + (1 - alpha) dL(l+1)/dΔh, back through block l.
-// Wcur is Wref with the module's weight replaced; Wn the next block's.
+// Wcur is the current pass's weights with the module's weight replaced
+// (module_delta); Wn the next block's.
 template <class X>
 int module_window(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Weights &Wn, const Buffers &Bl,
-                  const Buffers &Bn, const ModuleBuffers &M, const float *xin, int module, float alpha,
-                  const float *F_this, const float *F_next, float *gW, float *loss) {
+                  const Buffers &Bn, const ModuleBuffers &M, const float *xin, const float *xhat, int module,
+                  float alpha, const float *F_this, const float *F_next, float *gW, float *loss) {
     const int64_t T = dm.T(), d = dm.d;
     const int64_t np = (T + kChunk - 1) / kChunk;
-    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin);
+    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin, xhat);
     e |= setup(x, dm, Wn, Bn);
     e |= window(x, dm, Wn, Bn, M.href, M.dh, F_next, M.gnext, M.lnext);
     e |= x.gemm(gemm_rr(T, d, d, M.dh, F_this, M.wthis, nullptr, 1.f / (float)T), "blk_fisher");
@@ -661,13 +664,13 @@ int module_window(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur
 }
 
 // The final block's loss of one module: the KL at the LM head between the
-// reference output and the one with the module's weight replaced, and the
-// gradient in that weight.
+// reference output and the current pass's (module_delta), and the gradient
+// in the module's weight.
 template <class X>
 int module_kl(X &x, const Dims &dm, const Weights &Wref, const Weights &Wcur, const Buffers &Bl,
-              const ModuleBuffers &M, const Head &hd, const HeadBuffers &H, const float *xin, int module, float *gW,
-              float *loss) {
-    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin);
+              const ModuleBuffers &M, const Head &hd, const HeadBuffers &H, const float *xin, const float *xhat,
+              int module, float *gW, float *loss) {
+    int e = module_delta(x, dm, Wref, Wcur, Bl, M, xin, xhat);
     e |= kl_head(x, dm, hd, H, M.href, M.dh, M.gh, loss);
     e |= backward(x, dm, Wcur, Bl, M.gh, nullptr, module, gW);
     return e;

@@ -120,12 +120,13 @@ realq_status_t prepare_deferred(cudaStream_t s, int64_t n, double norm, float da
 realq_status_t scale_copy(cudaStream_t s, int64_t count, float mul, const float *in, float *out);
 // Host-side checks of the block ops' arguments for one module (the exact
 // window when next_block is given, else the final block's KL at the LM head
-// gf, Wh of vocab rows): the module's weight shape m x n and the block ops'
-// workspace bytes.  Launches nothing.
+// gf, Wh of vocab rows; this_block_hat may be NULL): the module's weight
+// shape m x n and the block ops' workspace bytes.  Launches nothing.
 realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_block_weights_t *this_block,
-                                const realq_block_weights_t *next_block, int64_t S, int64_t L, const float *x,
-                                int module, const float *F_this, const float *F_next, const float *gf, const float *Wh,
-                                int64_t vocab, const char *who, int64_t *m, int64_t *n, size_t *ws_bytes);
+                                const realq_block_weights_t *this_block_hat, const realq_block_weights_t *next_block,
+                                int64_t S, int64_t L, const float *x, int module, const float *F_this,
+                                const float *F_next, const float *gf, const float *Wh, int64_t vocab, const char *who,
+                                int64_t *m, int64_t *n, size_t *ws_bytes);
 // One Adam (or SGD) step of Eq. block_gd_update on the columns c0.. of the
 // m x n weights W with a full-width m x n gradient G (the block ops' module
 // gradient): PyTorch-form Adam with bias corrections for step t >= 1.

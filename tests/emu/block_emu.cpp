@@ -94,8 +94,10 @@ extern "C" int emu_block_window(const int64_t *iv, const float *fv, const float 
     return e;
 }
 
-// the exact window of one module of block l: wl = block l, wn = next block,
-// Wm = the module's weight (module 0..6 = q, k, v, o, gate, up, down)
+// the exact window of one module of block l: wl = block l, wh = block l's
+// weights in the current pass (NULL: wl), wn = next block, x / x_hat = block
+// l's reference and current inputs (x_hat NULL: x), Wm = the module's weight
+// (module 0..6 = q, k, v, o, gate, up, down)
 extern "C" size_t emu_module_workspace(const int64_t *iv, const float *fv, int64_t V) {
     const realq::blk::Dims dm = dims_of(iv, fv);
     size_t b = 2 * realq::blk::carve(dm, nullptr, nullptr) + realq::blk::carve_module(dm, nullptr, nullptr);
@@ -103,9 +105,10 @@ extern "C" size_t emu_module_workspace(const int64_t *iv, const float *fv, int64
     return b;
 }
 
-extern "C" int emu_module_window(const int64_t *iv, const float *fv, const float *const *wl, const float *const *wn,
-                                 const float *x, int module, const float *Wm, float alpha, const float *F_this,
-                                 const float *F_next, float *gW, float *loss, void *ws) {
+extern "C" int emu_module_window(const int64_t *iv, const float *fv, const float *const *wl, const float *const *wh,
+                                 const float *const *wn, const float *x, const float *x_hat, int module,
+                                 const float *Wm, float alpha, const float *F_this, const float *F_next, float *gW,
+                                 float *loss, void *ws) {
     using namespace realq::blk;
     const Dims dm = dims_of(iv, fv);
     Buffers Bl{}, Bn{};
@@ -116,8 +119,8 @@ extern "C" int emu_module_window(const int64_t *iv, const float *fv, const float
     carve_module(dm, p, &M);
     HostExec X;
     const Weights Wref = weights_of(wl);
-    return module_window(X, dm, Wref, with_module(Wref, module, Wm), weights_of(wn), Bl, Bn, M, x, module, alpha,
-                         F_this, F_next, gW, loss);
+    return module_window(X, dm, Wref, with_module(weights_of(wh ? wh : wl), module, Wm), weights_of(wn), Bl, Bn, M, x,
+                         x_hat ? x_hat : x, module, alpha, F_this, F_next, gW, loss);
 }
 
 extern "C" int emu_head_kl(const int64_t *iv, const float *fv, const float *gf, const float *Wh, int64_t V,
@@ -130,9 +133,9 @@ extern "C" int emu_head_kl(const int64_t *iv, const float *fv, const float *gf, 
     return kl_head(X, dm, Head{gf, Wh, V}, H, h_ref, dh, g, loss);
 }
 
-extern "C" int emu_module_kl(const int64_t *iv, const float *fv, const float *const *wl, const float *x, int module,
-                             const float *Wm, const float *gf, const float *Wh, int64_t V, float *gW, float *loss,
-                             void *ws) {
+extern "C" int emu_module_kl(const int64_t *iv, const float *fv, const float *const *wl, const float *const *wh,
+                             const float *x, const float *x_hat, int module, const float *Wm, const float *gf,
+                             const float *Wh, int64_t V, float *gW, float *loss, void *ws) {
     using namespace realq::blk;
     const Dims dm = dims_of(iv, fv);
     Buffers Bl{};
@@ -144,5 +147,6 @@ extern "C" int emu_module_kl(const int64_t *iv, const float *fv, const float *co
     carve_head(dm, V, p, &H);
     HostExec X;
     const Weights Wref = weights_of(wl);
-    return module_kl(X, dm, Wref, with_module(Wref, module, Wm), Bl, M, Head{gf, Wh, V}, H, x, module, gW, loss);
+    return module_kl(X, dm, Wref, with_module(weights_of(wh ? wh : wl), module, Wm), Bl, M, Head{gf, Wh, V}, H, x,
+                     x_hat ? x_hat : x, module, gW, loss);
 }

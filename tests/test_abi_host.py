@@ -206,9 +206,9 @@ def test_block_module_and_head_entry_points_reject_bad_arguments(L):
     ok = rq.block_dims(64, 4, 2, 16, 96)
     big = 1 << 40
 
-    def win(module=0, alpha=0.5, F=fake, nbytes=big):
-        return L.realq_block_module_window(None, ctypes.byref(ok), ctypes.byref(w), ctypes.byref(w), 2, 8, fake,
-                                           module, fake, alpha, F, fake, fake, None, fake, nbytes)
+    def win(module=0, alpha=0.5, F=fake, nbytes=big, hat=None):
+        return L.realq_block_module_window(None, ctypes.byref(ok), ctypes.byref(w), hat, ctypes.byref(w), 2, 8, fake,
+                                           None, module, fake, alpha, F, fake, fake, None, fake, nbytes)
 
     assert rq.realq_block_module_workspace_size(ok, 2, 8) > 2 * rq.realq_block_workspace_size(ok, 2, 8)
     assert rq.realq_block_module_workspace_size(ok, 2, 8, 1000) > 2 * 8 * 1000 * 8
@@ -219,6 +219,8 @@ def test_block_module_and_head_entry_points_reject_bad_arguments(L):
     assert win(F=None) == rq.REALQ_ERR_INVALID_ARG
     assert win(nbytes=1024) == rq.REALQ_ERR_WORKSPACE
     assert "block_module_window" in rq.realq_last_error()
+    bad = rq.BlockWeights(*([fake.value] * 8 + [None]))                 # the current pass's weights are checked too
+    assert win(hat=ctypes.byref(bad)) == rq.REALQ_ERR_INVALID_ARG
     # the head: vocab, eps and the token limit
     kl = L.realq_block_head_kl
     assert kl(None, 64, 2, 8, fake, fake, 0, 1e-6, fake, fake, fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG
@@ -226,8 +228,8 @@ def test_block_module_and_head_entry_points_reject_bad_arguments(L):
     assert kl(None, 64, 4096, 4096, fake, fake, 100, 1e-6, fake, fake, fake, None, fake, big) == \
         rq.REALQ_ERR_INVALID_ARG
     assert kl(None, 64, 2, 8, fake, fake, 100, 1e-6, fake, fake, fake, None, fake, 64) == rq.REALQ_ERR_WORKSPACE
-    assert L.realq_block_module_kl(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, 3, fake, fake, None, 100,
-                                   fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG     # NULL Wh
+    assert L.realq_block_module_kl(None, ctypes.byref(ok), ctypes.byref(w), None, 2, 8, fake, None, 3, fake, fake,
+                                   None, 100, fake, None, fake, big) == rq.REALQ_ERR_INVALID_ARG     # NULL Wh
 
 
 def test_window_sweep_entry_point_rejects_bad_arguments(L):
@@ -244,8 +246,9 @@ def test_window_sweep_entry_point_rejects_bad_arguments(L):
     def sweep(module=6, nxt=True, F=fake, vocab=0, head=fake, bcfg=None, qcfg=q, blocks=(0, 2), nbytes=big,
               deq_dtype=0, adam=fake):
         b = bcfg if bcfg is not None else rq.bgd_cfg(1e-3)
-        return L.realq_quantize_layer_window(None, ctypes.byref(ok), ctypes.byref(w),
-                                             ctypes.byref(w) if nxt else None, 2, 8, fake, module, F, fake, head, head,
+        return L.realq_quantize_layer_window(None, ctypes.byref(ok), ctypes.byref(w), None,
+                                             ctypes.byref(w) if nxt else None, 2, 8, fake, None, module, F, fake, head,
+                                             head,
                                              vocab, fake, None, ctypes.byref(qcfg), ctypes.byref(b), fake, adam, adam,
                                              ctypes.byref(t), fake, fake, fake, None, deq_dtype, None, blocks[0],
                                              blocks[1], fake, nbytes)

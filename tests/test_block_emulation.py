@@ -183,26 +183,43 @@ def _ws(emu, iv, fv, V=0):
     return np.zeros(emu.emu_module_workspace(iv.ctypes.data, fv.ctypes.data, V) // 4 + 64, dtype=np.float32)
 
 
+def _current_pass32(r, P, x, name):
+    # block l's input and weights in the model quantized so far (the other
+    # modules moved off the reference), rounded to fp32
+    x_hat = (x + 0.1 * r.standard_normal(x.shape)).astype(np.float32).astype(np.float64)
+    P_hat = dict(P)
+    for k in ("Wq", "Wk", "Wv", "Wo", "Wg", "Wu", "Wd"):
+        if k != name:
+            P_hat[k] = (P[k] + 0.03 * r.standard_normal(P[k].shape)).astype(np.float32).astype(np.float64)
+    return x_hat, P_hat
+
+
+@pytest.mark.parametrize("current", [False, True])
 @pytest.mark.parametrize("module", MODULES)
-def test_module_window_matches_the_oracle(emu, module):
+def test_module_window_matches_the_oracle(emu, module, current):
     # block l's own backward to each module's weight, with the next block's
     # window (Eq. slide_window); the case with grouped queries and a ragged
-    # length
+    # length; with current, block l's current pass takes a perturbed input
+    # and other weights than the reference
     case = CASES[0]
     S, L, d = case[0], case[1], case[2]
     r, P, Pn, name, Wm, x = _module_case(4, case, module)
     F, Fn = _spd32(r, d), _spd32(r, d)
     alpha = 0.6
-    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, alpha, F, Fn)
+    x_hat, P_hat = _current_pass32(r, P, x, name) if current else (None, None)
+    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, alpha, F, Fn, x_hat, P_hat)
     iv, fv = _iv(P, S, L)
     al, pl = _ptrs(P)
     an, pn = _ptrs(Pn)
+    ah, ph = _ptrs(P_hat) if current else (None, None)
+    xh32 = np.ascontiguousarray(x_hat, dtype=np.float32) if current else None
     x32, W32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, F, Fn))
     g = np.zeros(Wm.shape, dtype=np.float32)
     loss = np.zeros(1, dtype=np.float32)
     ws = _ws(emu, iv, fv)
-    rc = emu.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(MODULES.index(module)), _c(W32),
-                               ctypes.c_float(alpha), _c(F32), _c(Fn32), _c(g), _c(loss), _c(ws))
+    rc = emu.emu_module_window(_c(iv), _c(fv), pl, ph, pn, _c(x32), _c(xh32) if current else None,
+                               ctypes.c_int(MODULES.index(module)), _c(W32), ctypes.c_float(alpha), _c(F32), _c(Fn32),
+                               _c(g), _c(loss), _c(ws))
     assert rc == 0
     # Δh is a difference of two fp32 forward passes, as in the window
     assert abs(float(loss[0]) - want_loss) <= 1e-4 * abs(want_loss), (float(loss[0]), want_loss)
@@ -232,22 +249,27 @@ def test_kl_head_matches_the_oracle(emu):
     np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
 
 
+@pytest.mark.parametrize("current", [False, True])
 @pytest.mark.parametrize("module", ("k_proj", "o_proj", "up_proj", "down_proj"))
-def test_final_block_module_kl_matches_the_oracle(emu, module):
+def test_final_block_module_kl_matches_the_oracle(emu, module, current):
     case = CASES[1]
     S, L, d = case[0], case[1], case[2]
     r, P, _, name, Wm, x = _module_case(6, case, module)
     V = 29
     head = {k: v.astype(np.float32).astype(np.float64) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
-    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head)
+    x_hat, P_hat = _current_pass32(r, P, x, name) if current else (None, None)
+    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head, x_hat, P_hat)
     iv, fv = _iv(P, S, L)
     al, pl = _ptrs(P)
+    ah, ph = _ptrs(P_hat) if current else (None, None)
+    xh32 = np.ascontiguousarray(x_hat, dtype=np.float32) if current else None
     x32, W32, gf, Wh = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, head["gf"], head["Wh"]))
     g = np.zeros(Wm.shape, dtype=np.float32)
     loss = np.zeros(1, dtype=np.float32)
     ws = _ws(emu, iv, fv, V)
-    rc = emu.emu_module_kl(_c(iv), _c(fv), pl, _c(x32), ctypes.c_int(MODULES.index(module)), _c(W32), _c(gf),
-                           _c(Wh), ctypes.c_int64(V), _c(g), _c(loss), _c(ws))
+    rc = emu.emu_module_kl(_c(iv), _c(fv), pl, ph, _c(x32), _c(xh32) if current else None,
+                           ctypes.c_int(MODULES.index(module)), _c(W32), _c(gf), _c(Wh), ctypes.c_int64(V), _c(g),
+                           _c(loss), _c(ws))
     assert rc == 0
     assert abs(float(loss[0]) - want_loss) <= 1e-4 * abs(want_loss), (float(loss[0]), want_loss)
     np.testing.assert_allclose(g, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
@@ -271,9 +293,12 @@ PLANTED = {
                           ""),
     "module_blend": ("Axpy{M.tmp, M.wthis, M.gh, alpha}", "Axpy{M.tmp, M.wthis, M.gh, 1.f - alpha}"),
     "kl_sign": ("b[v] = (q - p) * inv_T;", "b[v] = (p - q) * inv_T;"),
+    # the current pass run on the reference input
+    "current_input": ("e |= forward(x, dm, Wcur, Bl, xhat, M.dh);", "e |= forward(x, dm, Wcur, Bl, xin, M.dh);"),
 }
 # the check each planted mistake is run against
-_PLANTED_CHECK = {"wgrad_before_rope": "module_q", "module_blend": "module_q", "kl_sign": "kl"}
+_PLANTED_CHECK = {"wgrad_before_rope": "module_q", "module_blend": "module_q", "kl_sign": "kl",
+                  "current_input": "module_q_current"}
 
 
 @pytest.mark.parametrize("name", sorted(PLANTED))
@@ -332,24 +357,30 @@ def _planted_module_or_kl_differs(lib, check):
     else:
         r, P, Pn, name, Wm, x = _module_case(4, case, "q_proj")
         F, Fn = _spd32(r, d), _spd32(r, d)
-        want_loss, want_g = ob.sliding_window_module("q_proj", Wm, x, P, Pn, 0.6, F, Fn)
+        current = check == "module_q_current"
+        x_hat, P_hat = _current_pass32(r, P, x, name) if current else (None, None)
+        want_loss, want_g = ob.sliding_window_module("q_proj", Wm, x, P, Pn, 0.6, F, Fn, x_hat, P_hat)
         iv, fv = _iv(P, S, L)
         al, pl = _ptrs(P)
         an, pn = _ptrs(Pn)
+        ah, ph = _ptrs(P_hat) if current else (None, None)
+        xh32 = np.ascontiguousarray(x_hat, dtype=np.float32) if current else None
         x32, W32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, Wm, F, Fn))
         g = np.zeros(Wm.shape, dtype=np.float32)
         loss = np.zeros(1, dtype=np.float32)
         ws = _ws(lib, iv, fv)
-        assert lib.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(0), _c(W32), ctypes.c_float(0.6),
-                                     _c(F32), _c(Fn32), _c(g), _c(loss), _c(ws)) == 0
+        assert lib.emu_module_window(_c(iv), _c(fv), pl, ph, pn, _c(x32), _c(xh32) if current else None,
+                                     ctypes.c_int(0), _c(W32), ctypes.c_float(0.6), _c(F32), _c(Fn32), _c(g),
+                                     _c(loss), _c(ws)) == 0
     return (abs(float(loss[0]) - want_loss) > 1e-4 * abs(want_loss)
             or np.abs(g - want_g).max() > 1e-4 * np.abs(want_g).max())
 
 
 def _all_ops(lib, case, V=23):
     """Every op of the header on one case (forward, window, the module
-    window and the final block's KL for all seven modules, the KL head), as
-    one flat fp32 vector, with the return codes."""
+    window and the final block's KL for all seven modules with a current
+    pass off the reference, the KL head), as one flat fp32 vector, with the
+    return codes."""
     S, L, d, H, Hkv, dh, f = case
     r, P = _case(7, *case)
     _, Pn = _case(107, *case)
@@ -366,6 +397,9 @@ def _all_ops(lib, case, V=23):
     an, pn = _ptrs(Pn)
     head = {k: np.ascontiguousarray(v, dtype=np.float32) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
     x32, d32, F32, Fn32 = (np.ascontiguousarray(a, dtype=np.float32) for a in (x, dh_, F, Fn))
+    x_hat, P_hat = _current_pass32(r, P, x, None)
+    xh32 = np.ascontiguousarray(x_hat, dtype=np.float32)
+    ah, ph = _ptrs(P_hat)
     for i, module in enumerate(MODULES):
         W32 = np.ascontiguousarray(P[ob._MODULE_WEIGHT[module]] + 0.05 * r.standard_normal(
             P[ob._MODULE_WEIGHT[module]].shape), dtype=np.float32)
@@ -374,12 +408,14 @@ def _all_ops(lib, case, V=23):
             lo = np.zeros(1, dtype=np.float32)
             if kind == "window":
                 ws = _ws(lib, iv, fv)
-                rcs.append(lib.emu_module_window(_c(iv), _c(fv), pl, pn, _c(x32), ctypes.c_int(i), _c(W32),
-                                                 ctypes.c_float(0.6), _c(F32), _c(Fn32), _c(gW), _c(lo), _c(ws)))
+                rcs.append(lib.emu_module_window(_c(iv), _c(fv), pl, ph, pn, _c(x32), _c(xh32), ctypes.c_int(i),
+                                                 _c(W32), ctypes.c_float(0.6), _c(F32), _c(Fn32), _c(gW), _c(lo),
+                                                 _c(ws)))
             else:
                 ws = _ws(lib, iv, fv, V)
-                rcs.append(lib.emu_module_kl(_c(iv), _c(fv), pl, _c(x32), ctypes.c_int(i), _c(W32), _c(head["gf"]),
-                                             _c(head["Wh"]), ctypes.c_int64(V), _c(gW), _c(lo), _c(ws)))
+                rcs.append(lib.emu_module_kl(_c(iv), _c(fv), pl, ph, _c(x32), _c(xh32), ctypes.c_int(i), _c(W32),
+                                             _c(head["gf"]), _c(head["Wh"]), ctypes.c_int64(V), _c(gW), _c(lo),
+                                             _c(ws)))
             out += [gW.ravel(), lo]
     g = np.zeros((S, L, d), dtype=np.float32)
     lo = np.zeros(1, dtype=np.float32)

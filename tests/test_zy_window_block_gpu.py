@@ -119,11 +119,25 @@ def _weights(P):
     return {k: torch.from_numpy(P[k].astype(np.float32)).cuda() for k in _KEYS}
 
 
-@pytest.mark.parametrize("case", [CASES[0], CASES[4]])
+def _current_pass(r, P, x, name):
+    # block l's input and weights in the model quantized so far: a perturbed
+    # input and every other module moved off the reference (fp32-rounded)
+    x_hat = _f32(x + 0.1 * r.standard_normal(x.shape))
+    P_hat = dict(P)
+    for k in ("Wq", "Wk", "Wv", "Wo", "Wg", "Wu", "Wd"):
+        if k != name:
+            P_hat[k] = _f32(P[k] + 0.03 * r.standard_normal(P[k].shape))
+    W_hat = {k: torch.from_numpy(np.asarray(P_hat[k], dtype=np.float32)).cuda() for k in _KEYS}
+    return x_hat, P_hat, W_hat
+
+
+@pytest.mark.parametrize("case,current", [(CASES[0], False), (CASES[4], False), (CASES[4], True)])
 @pytest.mark.parametrize("module", MODULES)
-def test_module_window_matches_the_oracle(case, module):
+def test_module_window_matches_the_oracle(case, current, module):
     # block l's own backward to the module's weight with the next block's
-    # window (Eq. slide_window), against oracle.block.sliding_window_module
+    # window (Eq. slide_window), against oracle.block.sliding_window_module;
+    # with current, block l's current pass runs on a perturbed input with
+    # the other modules off the reference
     S, L, d, H, Hkv, dh, f = case
     r, P, W, dims, _ = _case(4, *case)
     _, Pn, Wn, _, _ = _case(104, *case)
@@ -131,11 +145,13 @@ def test_module_window_matches_the_oracle(case, module):
     Wm = _f32(P[name] + 0.05 * r.standard_normal(P[name].shape))
     x = _f32(r.standard_normal((S, L, d)))
     F, Fn = _spd(r, d), _spd(r, d)
-    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, 0.6, F, Fn)
+    x_hat, P_hat, W_hat = _current_pass(r, P, x, name) if current else (None, None, None)
+    want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, 0.6, F, Fn, x_hat, P_hat)
     grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
     loss = torch.zeros(1, dtype=torch.float32, device="cuda")
     ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L))
-    rq.realq_block_module_window(dims, W, Wn, _dev(x), module, _dev(Wm), 0.6, _dev(F), _dev(Fn), grad, ws, loss=loss)
+    rq.realq_block_module_window(dims, W, Wn, _dev(x), module, _dev(Wm), 0.6, _dev(F), _dev(Fn), grad, ws, loss=loss,
+                                 this_block_hat=W_hat, x_hat=_dev(x_hat) if current else None)
     got = grad.cpu().numpy()
     assert abs(loss.item() - want_loss) <= 1e-4 * abs(want_loss), (loss.item(), want_loss)
     np.testing.assert_allclose(got, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
@@ -156,8 +172,9 @@ def test_head_kl_matches_the_oracle():
     np.testing.assert_allclose(g.cpu().numpy(), want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
 
 
+@pytest.mark.parametrize("current", [False, True])
 @pytest.mark.parametrize("module", ("k_proj", "o_proj", "up_proj", "down_proj"))
-def test_final_block_module_kl_matches_the_oracle(module):
+def test_final_block_module_kl_matches_the_oracle(module, current):
     case = CASES[1]
     S, L, d, H, Hkv, dh, f = case
     r, P, W, dims, _ = _case(6, *case)
@@ -166,12 +183,13 @@ def test_final_block_module_kl_matches_the_oracle(module):
     x = _f32(r.standard_normal((S, L, d)))
     V = 29
     head = {k: _f32(v) for k, v in ob.head_params(r, d, V, scale=1.5).items()}
-    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head)
+    x_hat, P_hat, W_hat = _current_pass(r, P, x, name) if current else (None, None, None)
+    want_loss, want_g = ob.kl_final_module(module, Wm, x, P, head, x_hat, P_hat)
     grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
     loss = torch.zeros(1, dtype=torch.float32, device="cuda")
     ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L, V))
     rq.realq_block_module_kl(dims, W, _dev(x), module, _dev(Wm), _dev(head["gf"]), _dev(head["Wh"]), grad, ws,
-                             loss=loss)
+                             loss=loss, this_block_hat=W_hat, x_hat=_dev(x_hat) if current else None)
     assert abs(loss.item() - want_loss) <= 1e-4 * abs(want_loss), (loss.item(), want_loss)
     np.testing.assert_allclose(grad.cpu().numpy(), want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
 
@@ -197,22 +215,26 @@ SWEEP_CASE = (4, 96, 128, 4, 2, 32, 256)   # m x n from 64 x 128 up to 128 x 256
 QKW = dict(bits=4, group_size=64, block_size=64)
 
 
-def _sweep_inputs(seed, module, kl):
+def _sweep_inputs(seed, module, kl, current=False):
     S, L, d, H, Hkv, dh, f = SWEEP_CASE
     r, P, W, dims, _ = _case(seed, *SWEEP_CASE)
     _, Pn, Wn, _, _ = _case(seed + 100, *SWEEP_CASE)
     x = _f32(r.standard_normal((S, L, d)))
     F, Fn = _spd(r, d), _spd(r, d)
     head = {k: _f32(v) for k, v in ob.head_params(r, d, 50, scale=1.5).items()} if kl else None
-    X = _f32(ob.module_inputs(module, x, P))
-    return dict(P=P, W=W, Pn=Pn, Wn=Wn, dims=dims, x=x, F=F, Fn=Fn, head=head, X=X)
+    name = ob._MODULE_WEIGHT[module]
+    x_hat, P_hat, W_hat = _current_pass(r, P, x, name) if current else (None, None, None)
+    # the module's OBS Hessian comes from its inputs in the current pass
+    X = _f32(ob.module_inputs(module, x, P) if not current else ob.module_inputs(module, x_hat, P_hat))
+    return dict(P=P, W=W, Pn=Pn, Wn=Wn, dims=dims, x=x, F=F, Fn=Fn, head=head, X=X, x_hat=x_hat, P_hat=P_hat,
+                W_hat=W_hat)
 
 
 def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None):
     if c["head"] is not None:
-        fn = ob.kl_gradient_fn(module, c["x"], c["P"], c["head"])
+        fn = ob.kl_gradient_fn(module, c["x"], c["P"], c["head"], c["x_hat"], c["P_hat"])
     else:
-        fn = ob.window_gradient_fn(module, c["x"], c["P"], c["Pn"], c["F"], c["Fn"])
+        fn = ob.window_gradient_fn(module, c["x"], c["P"], c["Pn"], c["F"], c["Fn"], c["x_hat"], c["P_hat"])
     if capture is not None:
         inner = fn
 
@@ -253,7 +275,8 @@ def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=N
     state["t"] = rq.realq_quantize_layer_window(
         c["dims"], c["W"], c["Wn"] if c["head"] is None else None, _dev(c["x"]), module, prep.U, q, b, state["W"],
         state["codes"], state["scale"], state["zero"], dead=prep.dead, adam_m=state["am"], adam_v=state["av"],
-        adam_t=state["t"], block_loss=state["loss"], block_begin=b0, block_end=b1, ws=state["ws"], **kw)
+        adam_t=state["t"], block_loss=state["loss"], block_begin=b0, block_end=b1, ws=state["ws"],
+        this_block_hat=c["W_hat"], x_hat=_dev(c["x_hat"]) if c["x_hat"] is not None else None, **kw)
     rq.realq_workspace_status(state["ws"])
     torch.cuda.synchronize()
     return state
@@ -285,11 +308,14 @@ def _check_sweep(orc, st, n, lr, loss_rtol):
 # fp32 rounding of each token's log-partition functions (about 2.4e-7,
 # random in sign) leaves about 5e-4 of the KL after the mean over the 384
 # tokens: 3e-3.
-@pytest.mark.parametrize("module,kl,lr,steps", [
-    ("q_proj", False, 1.0, 1), ("o_proj", False, 1.0, 1), ("down_proj", False, 1.0, 1),
-    ("down_proj", False, 0.3, 2), ("k_proj", True, 10.0, 1), ("down_proj", True, 10.0, 1)])
-def test_window_sweep_with_gradient_steps_matches_the_oracle(module, kl, lr, steps):
-    c = _sweep_inputs(7, module, kl)
+@pytest.mark.parametrize("module,kl,lr,steps,current", [
+    ("q_proj", False, 1.0, 1, False), ("o_proj", False, 1.0, 1, False), ("down_proj", False, 1.0, 1, False),
+    ("down_proj", False, 0.3, 2, False), ("k_proj", True, 10.0, 1, False), ("down_proj", True, 10.0, 1, False),
+    ("q_proj", False, 1.0, 1, True), ("down_proj", True, 10.0, 1, True)])
+def test_window_sweep_with_gradient_steps_matches_the_oracle(module, kl, lr, steps, current):
+    # current: block l's current pass runs on a perturbed input with the
+    # other modules off the reference (the sequential pipeline's state)
+    c = _sweep_inputs(7, module, kl, current)
     orc = _oracle_sweep(c, module, "sgd", lr, steps, 3, 10)
     st = _gpu_sweep(c, module, "sgd", lr, steps, 3, 10)
     n = c["W"][ob._MODULE_WEIGHT[module]].shape[1]
