@@ -522,6 +522,17 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
                                   const float *dh, const float *F_next, float *g_h, float *loss, void *ws,
                                   size_t ws_bytes);
 
+/* realq_block_module_inputs: the calibration inputs of one module of the
+ * block in a forward pass with `weights` on input x (S L x d), written to
+ * X_out (S L x n, n the module's in-dimension): q/k/v read RMSNorm(x; g1),
+ * o_proj the attention output (S L x n_heads head_dim), gate/up RMSNorm(h;
+ * g2), down_proj the SwiGLU product (S L x ffn).  Their second moment is the
+ * module's OBS Hessian (Sec. 3.2; in the sequential pipeline, the current
+ * pass's inputs).  module 0..6 as below; ws as realq_block_forward. */
+realq_status_t realq_block_module_inputs(realq_stream_t stream, const realq_block_dims_t *dims,
+                                         const realq_block_weights_t *weights, int64_t S, int64_t L, const float *x,
+                                         int module, float *X_out, void *ws, size_t ws_bytes);
+
 /* Module level (any linear module of block l, Eq. slide_window): block l is
  * run at its reference weights on its reference input (h*, the full-precision
  * model) and as the current block (h: Sec. 4.3 evaluates the surrogate by a

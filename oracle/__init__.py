@@ -16,6 +16,7 @@ brute.c    exhaustive search over all int4 codes of a tiny layer (the
 block.py   one synthetic decoder block in fp64 with its backward, the
            exact two-block sliding-window loss (Sec. 4.4) of any linear
            module of the block, and the final block's true KL at the LM head
-           with the Fisher of Eq. (fisher_full); imported as ``oracle.block``.
+           with the Fisher of Eq. (fisher_full), and Alg. 1's loop over the
+           block's modules with those losses; imported as ``oracle.block``.
 """
 from .realq import *  # noqa: F401,F403

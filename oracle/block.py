@@ -43,14 +43,16 @@ last-transformer-block handling").  Readings for that part:
 """
 from __future__ import annotations
 
-from typing import Dict, Tuple
+from typing import Dict, Optional, Sequence, Tuple
 
 import numpy as np
+
+from . import realq as _sweep
 
 __all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down",
            "sliding_window_module", "head_params", "head_logits", "kl_logits", "kl_head_loss", "nll_scores",
            "fisher_sampled", "fisher_tokens", "kl_final_module", "module_inputs", "window_gradient_fn",
-           "kl_gradient_fn"]
+           "kl_gradient_fn", "MODULES", "quantize_block"]
 
 EPS = 1e-6
 
@@ -379,3 +381,57 @@ def kl_gradient_fn(module: str, x: np.ndarray, P_this: Dict, head: Dict, x_hat=N
     def fn(W, alpha):
         return kl_final_module(module, W, x, P_this, head, x_hat, P_hat)
     return fn
+
+
+# ---------------------------------------------------------------------------
+# Alg. 1's loop over the linear modules of one decoder block with the exact
+# losses.
+
+MODULES = ("q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj")
+
+
+def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] = None, P_next: Optional[Dict] = None,
+                   F_this: Optional[np.ndarray] = None, F_next: Optional[np.ndarray] = None,
+                   head: Optional[Dict] = None, lr: float, steps_per_block: int = 1, optimizer: str = "adam",
+                   bits: int = 4, group_size: int = 128, block_size: int = 128, damp_frac: float = 0.01,
+                   modules: Sequence[str] = MODULES):
+    """Quantize the linear modules of block l one after another (Alg. 1: for
+    each linear module, the column sweep with a Block-GD step after every
+    column block), each against the exact two-block window (P_next, F_this,
+    F_next given) or, for the last block, the true KL at the LM head (head
+    given).
+
+    x: block l's full-precision input; x_hat: its input in the model
+    quantized so far (default x).  The current weights start at P_this; as
+    each module finishes, its dequantized weights replace it there, so the
+    next module's current pass, OBS Hessian (the second moment of its inputs
+    in that pass) and loss see every module quantized before it.  b_global
+    runs over the column blocks of all the block's modules, B_total being
+    their sum (Eq. slide_window; Alg. 1's note on b_global).  Returns the
+    sweep result of every module and the final current weights."""
+    x_hat = x if x_hat is None else x_hat
+    P_hat = dict(P_this)
+    nbs = {}
+    for module in modules:
+        n = P_this[_MODULE_WEIGHT[module]].shape[1]
+        nbs[module] = -(-n // block_size)
+    B_total = sum(nbs.values())
+    b_start = 1
+    out = {}
+    for module in modules:
+        name = _MODULE_WEIGHT[module]
+        X = module_inputs(module, x_hat, P_hat)
+        H_sum, T = _sweep.hessian_sum([X])
+        cur = dict(P_hat)
+        if head is not None:
+            fn = kl_gradient_fn(module, x, P_this, head, x_hat, cur)
+        else:
+            fn = window_gradient_fn(module, x, P_this, P_next, F_this, F_next, x_hat, cur)
+        bgd = {"lr": lr, "steps_per_block": steps_per_block, "optimizer": optimizer, "b_global_start": b_start,
+               "B_total": B_total, "gradient_fn": fn}
+        res = _sweep.realq_sweep(P_this[name], H_sum, T, bits=bits, group_size=group_size, block_size=block_size,
+                                 damp_frac=damp_frac, bgd=bgd)
+        P_hat[name] = res["deq"]
+        out[module] = res
+        b_start += nbs[module]
+    return out, P_hat

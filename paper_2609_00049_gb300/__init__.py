@@ -32,7 +32,7 @@ __all__ = [
     "realq_profile_collect", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
     "realq_block_window", "BLOCK_MODULES", "realq_block_module_workspace_size", "realq_block_head_workspace_size",
     "realq_block_module_window", "realq_block_head_kl", "realq_block_module_kl",
-    "realq_quantize_window_workspace_size", "realq_quantize_layer_window",
+    "realq_quantize_window_workspace_size", "realq_quantize_layer_window", "realq_block_module_inputs",
 ]
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
@@ -153,6 +153,8 @@ _SIGS = {
     "realq_block_module_kl": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
                                ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _i64, _vp, _vp,
                                _vp, _sz], _int),
+    "realq_block_module_inputs": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp,
+                                   _int, _vp, _vp, _sz], _int),
     "realq_quantize_window_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _int, _i64,
                                               ctypes.POINTER(QuantCfg)], _sz),
     "realq_quantize_layer_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
@@ -654,6 +656,17 @@ def realq_block_module_workspace_size(dims: BlockDims, S: int, L: int, vocab: in
 
 def realq_block_head_workspace_size(d: int, S: int, L: int, vocab: int) -> int:
     return int(lib().realq_block_head_workspace_size(int(d), int(S), int(L), int(vocab)))
+
+
+def realq_block_module_inputs(dims: BlockDims, weights: dict, x: torch.Tensor, module: str, X_out: torch.Tensor,
+                              ws: torch.Tensor, stream=None):
+    """The module's calibration inputs (S L x n) in a forward pass of the
+    block with `weights` on x (S, L, d); ws as realq_block_forward."""
+    S, L, d = x.shape
+    wp, wb = _ws(ws)
+    a = _block_weights(weights)
+    _check(lib().realq_block_module_inputs(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
+                                           BLOCK_MODULES.index(module), _ptr(X_out), wp, wb))
 
 
 def _opt_weights(w: Optional[dict]):

@@ -19,6 +19,11 @@ multi-stream step once into a CUDA graph; replay() then launches it whole.
 The preparation's factorisation status is therefore never read mid-step:
 check_status() reads it, with the sweeps' status words, after the step.
 
+quantize_block_exact runs a block with the exact losses of Sec. 4.4 (the
+two-block window, or the KL at the LM head for the last block) instead:
+there each module's loss and OBS Hessian depend on the modules quantized
+before it, so the modules run one after another on the caller's stream.
+
 No arithmetic happens here; every step is a call through the C ABI.
 """
 from __future__ import annotations
@@ -29,13 +34,16 @@ from typing import Dict, List, Optional, Sequence
 
 import torch
 
-from . import (REALQ_BF16, QuantCfg, bgd_cfg, realq_graph_begin, realq_graph_end, realq_hessian_accumulate,
+from . import layer
+from . import (BLOCK_MODULES, REALQ_BF16, REALQ_OPT_ADAM, QuantCfg, bgd_cfg, realq_block_module_inputs,
+               realq_block_workspace_size, realq_graph_begin, realq_graph_end, realq_hessian_accumulate,
                realq_hessian_accumulate_weighted, realq_hessian_prepare_deferred, realq_hessian_prepare_scaled,
                realq_hessian_weighted_workspace_size, realq_hessian_workspace_size, realq_prepare_status,
                realq_prepare_workspace_size, realq_quantize_activations, realq_quantize_grouped_workspace_size,
                realq_quantize_layer, realq_quantize_layer_grouped, realq_quantize_layer_minibatch,
                realq_quantize_layer_tokens, realq_quantize_minibatch_workspace_size,
-               realq_quantize_tokens_workspace_size, realq_quantize_workspace_size, realq_saliency_clip,
+               realq_quantize_layer_window, realq_quantize_tokens_workspace_size,
+               realq_quantize_window_workspace_size, realq_quantize_workspace_size, realq_saliency_clip,
                realq_scale_moment, realq_workspace_status, workspace)
 
 
@@ -484,3 +492,83 @@ class BlockQuantizer:
                                            F=torch.empty(F_host[md.name].shape, dtype=F_host[md.name].dtype,
                                                          device=dev))
                              for md in self.modules}
+
+
+# ---------------------------------------------------------------------------
+# The block with the exact losses (Sec. 4.4 Eq. slide_window; Eq. kl_loss for
+# the last block): Alg. 1's loop over the linear modules, one after another,
+# each module's current pass seeing the modules quantized before it.
+
+_MODULE_KEY = {"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg", "up_proj": "Wu",
+               "down_proj": "Wd"}
+
+
+@dataclass
+class ExactModule:
+    """One module's result: packed codes, scale, zero, the dequantized fp32
+    weights, the optimizer step count and the per-block losses (before and
+    after each block's steps; -1 where a block took none)."""
+    codes: torch.Tensor
+    scale: torch.Tensor
+    zero: torch.Tensor
+    W: torch.Tensor
+    adam_t: int
+    block_loss: torch.Tensor
+
+
+def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor, qcfg: QuantCfg, lr: float, *,
+                         x_hat: Optional[torch.Tensor] = None, W_next: Optional[Dict[str, torch.Tensor]] = None,
+                         F_this: Optional[torch.Tensor] = None, F_next: Optional[torch.Tensor] = None,
+                         head_gf: Optional[torch.Tensor] = None, head_Wh: Optional[torch.Tensor] = None,
+                         steps_per_block: int = 1, optimizer: int = REALQ_OPT_ADAM,
+                         modules: Sequence[str] = BLOCK_MODULES, stream=None):
+    """Quantizes the linear modules of decoder block l in order, each with
+    Block-GD on the exact two-block window (W_next, F_this, F_next given) or,
+    for the last block, on the KL at the LM head (head_gf, head_Wh given).
+
+    W_this: block l's full-precision weights (the reference); x its
+    full-precision input (S, L, d) and x_hat its input in the model quantized
+    so far (default x).  For each module: its inputs in the current pass
+    (realq_block_module_inputs with the weights quantized so far, on x_hat),
+    their Hessian and factor, then realq_quantize_layer_window with b_global
+    running over the column blocks of all the modules; its dequantized
+    weights then replace it in the current weights.  Returns each module's
+    ExactModule and the final current weights."""
+    S, L, d = x.shape
+    dev = x.device
+    nb = {md: -(-W_this[_MODULE_KEY[md]].shape[1] // qcfg.block_size) for md in modules}
+    B_total = sum(nb.values())
+    vocab = int(head_Wh.shape[0]) if head_Wh is not None else 0
+    W_hat = dict(W_this)
+    bws = workspace(realq_block_workspace_size(dims, S, L), dev)
+    g = qcfg.group_size
+    out = {}
+    b_start = 1
+    for md in modules:
+        key = _MODULE_KEY[md]
+        m, n = W_this[key].shape
+        X = torch.empty((S * L, n), dtype=torch.float32, device=dev)
+        realq_block_module_inputs(dims, W_hat, x if x_hat is None else x_hat, md, X, bws, stream=stream)
+        H, _, T = layer.accumulate([X], n, device=dev, stream=stream)
+        prep = layer.prepare(H, T, qcfg.damp_frac, stream=stream)
+        ngroups = -(-n // g) if g > 0 else 1
+        W = torch.empty((m, n), dtype=torch.float32, device=dev)
+        codes = torch.empty((m, (n + 1) // 2), dtype=torch.uint8, device=dev)
+        scale = torch.empty((m, ngroups), dtype=torch.float32, device=dev)
+        zero = torch.empty((m, ngroups), dtype=torch.uint8, device=dev)
+        am = torch.empty((m, n), dtype=torch.float32, device=dev)
+        av = torch.empty((m, n), dtype=torch.float32, device=dev)
+        loss = torch.full((nb[md], 2), -1.0, dtype=torch.float32, device=dev)
+        ws = workspace(realq_quantize_window_workspace_size(dims, S, L, md, qcfg, vocab), dev)
+        b = bgd_cfg(lr, steps_per_block=steps_per_block, optimizer=optimizer, b_global_start=b_start,
+                    B_total=B_total)
+        t = realq_quantize_layer_window(dims, W_this, W_next if head_Wh is None else None, x, md, prep.U, qcfg, b,
+                                        W, codes, scale, zero, F_this=F_this, F_next=F_next, head_gf=head_gf,
+                                        head_Wh=head_Wh, dead=prep.dead, adam_m=am, adam_v=av, block_loss=loss,
+                                        ws=ws, this_block_hat=W_hat, x_hat=x_hat, stream=stream)
+        realq_workspace_status(ws, stream=stream)
+        W_hat = dict(W_hat)
+        W_hat[key] = W
+        out[md] = ExactModule(codes, scale, zero, W, t, loss)
+        b_start += nb[md]
+    return out, W_hat

@@ -222,6 +222,23 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
     return X.st;
 }
 
+realq_status_t realq_block_module_inputs(realq_stream_t stream, const realq_block_dims_t *dims,
+                                         const realq_block_weights_t *weights, int64_t S, int64_t L, const float *x,
+                                         int module, float *X_out, void *ws, size_t ws_bytes) {
+    const char *who = "block_module_inputs";
+    blk::Dims dm{};
+    REALQ_TRY(check_block(dims, weights, S, L, who, &dm));
+    if (module < blk::M_Q || module > blk::M_DOWN)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: module must be 0..6 (q, k, v, o, gate, up, down)", who);
+    if (!x || !X_out) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x or X_out", who);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, blk::carve(dm, nullptr, nullptr), who));
+    blk::Buffers B{};
+    blk::carve(dm, ws, &B);
+    DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::module_input(X, dm, weights_of(weights), B, x, module, X_out);
+    return X.st;
+}
+
 size_t realq_block_module_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L, int64_t vocab) {
     if (!dims || S <= 0 || L <= 0 || dims->head_dim <= 0 || vocab < 0) return 0;
     const blk::Dims dm{S, L, dims->d, dims->n_heads, dims->n_kv, dims->head_dim, dims->ffn, dims->rms_eps,

@@ -539,6 +539,26 @@ int window(X &x, const Dims &dm, const Weights &W, const Buffers &B, const float
     return e;
 }
 
+// The input of one module in a forward pass of the block (weights W, input
+// xin), copied to Xout (T x n, the module's in-dimension n): q/k/v read the
+// attention norm's output a, o_proj the attention output o, gate/up the MLP
+// norm's output b, down_proj the SwiGLU product m.  Its second moment is the
+// module's OBS Hessian.
+template <class X>
+int module_input(X &x, const Dims &dm, const Weights &W, const Buffers &B, const float *xin, int module,
+                 float *Xout) {
+    const int64_t T = dm.T();
+    int e = setup(x, dm, W, B);
+    e |= forward(x, dm, W, B, xin, B.y);
+    const float *src = B.a;
+    int64_t n = dm.d;
+    if (module == M_O) { src = B.o; n = dm.qw(); }
+    else if (module == M_GATE || module == M_UP) { src = B.b; n = dm.d; }
+    else if (module == M_DOWN) { src = B.m; n = dm.f; }
+    e |= x.map(T * n, Axpy{src, src, Xout, 0.f}, "blk_copy");
+    return e;
+}
+
 // ------------------------------------------------- module-level losses ---
 
 // block l's side of the module-level losses: the reference and perturbed

@@ -94,6 +94,16 @@ extern "C" int emu_block_window(const int64_t *iv, const float *fv, const float 
     return e;
 }
 
+// the input of module (0..6) in a forward pass with weights w on x, into X
+extern "C" int emu_module_inputs(const int64_t *iv, const float *fv, const float *const *w, const float *x,
+                                 int module, float *X, void *ws) {
+    const realq::blk::Dims dm = dims_of(iv, fv);
+    realq::blk::Buffers B{};
+    realq::blk::carve(dm, ws, &B);
+    HostExec E;
+    return realq::blk::module_input(E, dm, weights_of(w), B, x, module, X);
+}
+
 // the exact window of one module of block l: wl = block l, wh = block l's
 // weights in the current pass (NULL: wl), wn = next block, x / x_hat = block
 // l's reference and current inputs (x_hat NULL: x), Wm = the module's weight

@@ -272,3 +272,19 @@ def test_window_sweep_entry_point_rejects_bad_arguments(L):
     assert sweep(nbytes=n_win - 1) == rq.REALQ_ERR_WORKSPACE
     assert "quantize_layer_window" in rq.realq_last_error()
     assert t.value == 0
+
+
+def test_module_inputs_entry_point_rejects_bad_arguments(L):
+    import paper_2609_00049_gb300 as rq
+    fake = ctypes.c_void_p(1 << 20)
+    w = rq.BlockWeights(*([fake.value] * 9))
+    ok = rq.block_dims(64, 4, 2, 16, 96)
+
+    def mi(module=0, X=fake, nbytes=1 << 40):
+        return L.realq_block_module_inputs(None, ctypes.byref(ok), ctypes.byref(w), 2, 8, fake, module, X, fake,
+                                           nbytes)
+
+    assert mi(module=7) == rq.REALQ_ERR_INVALID_ARG
+    assert mi(X=None) == rq.REALQ_ERR_INVALID_ARG
+    assert mi(nbytes=rq.realq_block_workspace_size(ok, 2, 8) - 1) == rq.REALQ_ERR_WORKSPACE
+    assert "block_module_inputs" in rq.realq_last_error()

@@ -183,6 +183,26 @@ def _ws(emu, iv, fv, V=0):
     return np.zeros(emu.emu_module_workspace(iv.ctypes.data, fv.ctypes.data, V) // 4 + 64, dtype=np.float32)
 
 
+@pytest.mark.parametrize("module", MODULES)
+def test_module_inputs_match_the_oracle(emu, module):
+    # the module's calibration inputs from a forward pass (its OBS Hessian's
+    # tokens): the attention norm's output, the attention output, the MLP
+    # norm's output or the SwiGLU product
+    case = CASES[0]
+    S, L, d = case[0], case[1], case[2]
+    r, P = _case(8, *case)
+    x = r.standard_normal((S, L, d)).astype(np.float32).astype(np.float64)
+    want = ob.module_inputs(module, x, P)
+    iv, fv = _iv(P, S, L)
+    al, pl = _ptrs(P)
+    x32 = np.ascontiguousarray(x, dtype=np.float32)
+    got = np.zeros(want.shape, dtype=np.float32)
+    ws = np.zeros(emu.emu_block_workspace(iv.ctypes.data, fv.ctypes.data) // 4 + 64, dtype=np.float32)
+    assert emu.emu_module_inputs(_c(iv), _c(fv), pl, _c(x32), ctypes.c_int(MODULES.index(module)), _c(got),
+                                 _c(ws)) == 0
+    np.testing.assert_allclose(got, want, rtol=0, atol=1e-5 * np.abs(want).max())
+
+
 def _current_pass32(r, P, x, name):
     # block l's input and weights in the model quantized so far (the other
     # modules moved off the reference), rounded to fp32

@@ -445,3 +445,74 @@ def test_final_block_kl_sweep_descends_with_small_sgd_steps():
     # column sweep on the same Hessian
     plain = oracle.realq_sweep(P["Wu"], Xm.T @ Xm, Xm.shape[0], block_size=8, group_size=8)
     assert np.abs(out["deq"] - plain["deq"]).max() > 0.0
+
+
+# --- Alg. 1's loop over the block's modules with the exact losses ------------
+
+def _driver_case(seed=31):
+    r = np.random.default_rng(seed)
+    d, H, Hkv, dh, f, S, L = 32, 4, 2, 8, 48, 2, 24
+    P = ob.block_params(r, d, H, Hkv, dh, f, scale=0.8)
+    Pn = ob.block_params(r, d, H, Hkv, dh, f, scale=0.8)
+    x = r.standard_normal((S, L, d))
+    x_hat = x + 0.05 * r.standard_normal(x.shape)
+    F, Fn = _spd(r, d), _spd(r, d)
+    return r, P, Pn, x, x_hat, F, Fn
+
+
+def test_block_driver_runs_the_global_block_index_over_all_modules():
+    # Eq. slide_window: b_global counts the column blocks of every module of
+    # the block in order, B_total is their sum; each recorded step's alpha is
+    # 1 - (b_global - 1)/(B_total - 1) (a module's last block takes no step)
+    r, P, Pn, x, x_hat, F, Fn = _driver_case()
+    out, _ = ob.quantize_block(x, P, x_hat=x_hat, P_next=Pn, F_this=F, F_next=Fn, lr=1e-3, group_size=16,
+                               block_size=16)
+    widths = {"q_proj": 32, "k_proj": 32, "v_proj": 32, "o_proj": 32, "gate_proj": 32, "up_proj": 32,
+              "down_proj": 48}
+    B_total = sum(w // 16 for w in widths.values())
+    assert B_total == 15
+    b_global = 1
+    for module in ob.MODULES:
+        nb = widths[module] // 16
+        got = [a for _, a, _, _ in out[module]["block_loss"]]
+        assert got == pytest.approx([1.0 - (b_global + b - 1) / (B_total - 1) for b in range(nb - 1)], abs=1e-15)
+        assert out[module]["adam_t"] == nb - 1
+        b_global += nb
+    assert out["q_proj"]["block_loss"][0][1] == 1.0
+
+
+def test_block_driver_threads_the_modules_quantized_so_far():
+    # o_proj's OBS Hessian and current pass see q, k, v quantized: the
+    # driver's o_proj sweep equals one run from those weights by hand
+    r, P, Pn, x, x_hat, F, Fn = _driver_case(32)
+    kw = dict(lr=1e-3, group_size=16, block_size=16)
+    out, P_hat = ob.quantize_block(x, P, x_hat=x_hat, P_next=Pn, F_this=F, F_next=Fn, **kw)
+    cur = dict(P)
+    for module in ("q_proj", "k_proj", "v_proj"):
+        cur[ob._MODULE_WEIGHT[module]] = out[module]["deq"]
+        assert not np.allclose(out[module]["deq"], P[ob._MODULE_WEIGHT[module]])
+    X = ob.module_inputs("o_proj", x_hat, cur)
+    H_sum, T = oracle.hessian_sum([X])
+    fn = ob.window_gradient_fn("o_proj", x, P, Pn, F, Fn, x_hat, cur)
+    bgd = {"lr": 1e-3, "b_global_start": 7, "B_total": 15, "gradient_fn": fn}
+    want = oracle.realq_sweep(P["Wo"], H_sum, T, group_size=16, block_size=16, bgd=bgd)
+    assert np.array_equal(out["o_proj"]["codes"], want["codes"])
+    np.testing.assert_allclose(out["o_proj"]["deq"], want["deq"], rtol=0, atol=1e-15)
+    # and the final current weights are every module's dequantized weights
+    for module in ob.MODULES:
+        assert P_hat[ob._MODULE_WEIGHT[module]] is out[module]["deq"]
+
+
+def test_block_driver_with_small_sgd_steps_lowers_every_modules_loss():
+    # with small plain gradient steps each block step lowers the exact
+    # window's loss (the descent lemma of Sec. 4.3's analysis), module after
+    # module through the whole block, and the final block's KL likewise
+    r, P, Pn, x, x_hat, F, Fn = _driver_case(33)
+    out, _ = ob.quantize_block(x, P, x_hat=x_hat, P_next=Pn, F_this=F, F_next=Fn, lr=0.5, optimizer="sgd",
+                               group_size=16, block_size=16)
+    head = ob.head_params(r, x.shape[2], 13, scale=1.5)
+    out_kl, _ = ob.quantize_block(x, P, x_hat=x_hat, head=head, lr=2.0, optimizer="sgd", group_size=16,
+                                  block_size=16)
+    for res in list(out.values()) + list(out_kl.values()):
+        for _, _, before, after in res["block_loss"]:
+            assert after < before, (before, after)
