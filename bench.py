@@ -525,6 +525,8 @@ def kernel_bench(args):
     rq.lib()
     from paper_2609_00049_gb300 import layer
     peaks = load_peaks()
+    if args.kernel == "window":
+        return window_bench(args, peaks)
     n, T = args.n, args.tokens
     wl = synth.Workload("kernel", {"x": synth.InputSpec("x", n, T, "gauss", outlier_frac=0.01, outlier_scale=20.0)},
                         [synth.ModuleSpec("w", args.m, n, "x")], seed=1, lr=3e-4)
@@ -572,6 +574,65 @@ def kernel_bench(args):
                       "input_bytes": T * n * 2}))
 
 
+def window_bench(args, peaks):
+    """Times one Block-GD gradient of the exact two-block window
+    (realq_block_module_window for down_proj: block l's reference and
+    current passes, the next block's two passes and its backward, block l's
+    backward to the module) on one decoder-block shape, with seeded random
+    weights and inputs.  Prints one JSON line."""
+    import torch
+    import paper_2609_00049_gb300 as rq
+    d, H, Hkv, dh, f = args.d, args.heads, args.kv_heads, args.head_dim, args.ffn
+    S, L = args.seqs, args.seq_len
+    T = S * L
+    g = torch.Generator().manual_seed(5)
+
+    def w(rows, cols):
+        return (torch.randn(rows, cols, generator=g) * 0.8 / cols ** 0.5).cuda()
+
+    def block():
+        return {"g1": (1 + 0.1 * torch.randn(d, generator=g)).cuda(), "Wq": w(H * dh, d), "Wk": w(Hkv * dh, d),
+                "Wv": w(Hkv * dh, d), "Wo": w(d, H * dh), "g2": (1 + 0.1 * torch.randn(d, generator=g)).cuda(),
+                "Wg": w(f, d), "Wu": w(f, d), "Wd": w(d, f)}
+
+    Wl, Wn = block(), block()
+    x = torch.randn(S, L, d, generator=g).cuda()
+    x_hat = x + 0.05 * torch.randn(S, L, d, generator=g).cuda()
+    Z = torch.randn(d, 16, generator=g)
+    F = (0.5 * torch.eye(d) + Z @ Z.T / 32).cuda()
+    Wm = Wl["Wd"] + 0.01 * torch.randn(d, f, generator=g).cuda()
+    dims = rq.block_dims(d, H, Hkv, dh, f)
+    ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L))
+    grad = torch.empty(d, f, device="cuda")
+    loss = torch.zeros(1, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    def run():
+        rq.realq_block_module_window(dims, Wl, Wn, x, "down_proj", Wm, 0.5, F, F, grad, ws, loss=loss,
+                                     x_hat=x_hat)
+    for _ in range(args.warmup):
+        run()
+    torch.cuda.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(args.steps):
+        run()
+    e1.record(stream)
+    torch.cuda.synchronize()
+    ms = e0.elapsed_time(e1) / args.steps
+    # one forward pass: the seven projections and the causal attention
+    # (q.k and p.v over half the sequence on average); a backward is about
+    # two forwards; a call runs four forwards and two backwards
+    fwd = 2 * T * (2 * d * H * dh + 2 * d * Hkv * dh + 3 * d * f) + 2 * T * L * H * dh
+    flop = 8 * fwd
+    alu = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+    tf = flop / (ms / 1e3) / 1e12
+    print(json.dumps({"kernel": "block_module_window", "d": d, "heads": H, "kv_heads": Hkv, "head_dim": dh,
+                      "ffn": f, "seqs": S, "seq_len": L, "ms_per_call": ms, "achieved": tf, "unit": "TFLOP/s",
+                      "peak": alu, "frac": tf / alu, "peak_source": "fp32 ALU: 152 SMs x 128 lanes x 2 x max clock",
+                      "bound": "alu"}))
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -593,8 +654,16 @@ def main():
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--no-graph", action="store_true", help="launch the block step eagerly instead of as a CUDA graph")
-    ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep"], default=None,
-                    help="time one stage alone on a small synthetic case")
+    ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep", "window"], default=None,
+                    help="time one stage alone on a small synthetic case (window: the exact two-block window's "
+                         "gradient on the decoder-block shape below)")
+    ap.add_argument("--d", type=int, default=1024)
+    ap.add_argument("--heads", type=int, default=16)
+    ap.add_argument("--kv-heads", type=int, default=8)
+    ap.add_argument("--head-dim", type=int, default=128)
+    ap.add_argument("--ffn", type=int, default=3072)
+    ap.add_argument("--seqs", type=int, default=2)
+    ap.add_argument("--seq-len", type=int, default=2048)
     ap.add_argument("--n", type=int, default=2048)
     ap.add_argument("--m", type=int, default=1024)
     ap.add_argument("--tokens", type=int, default=65536)
