@@ -1,0 +1,91 @@
+"""Host logic of the block-level driver with the exact losses
+(paper_2609_00049_gb300.block.quantize_block_exact), with the library's
+device calls replaced by recorders: the modules run in the paper's order,
+b_global runs over the column blocks of all of them with B_total their sum,
+each module sees the modules quantized before it (the current weights and
+the perturbed input), and the final current weights are every module's
+dequantized weights.  No GPU is used."""
+import pytest
+import torch
+
+import paper_2609_00049_gb300 as rq
+from paper_2609_00049_gb300 import block as pb
+from paper_2609_00049_gb300 import layer
+
+KEYS = ("g1", "Wq", "Wk", "Wv", "Wo", "g2", "Wg", "Wu", "Wd")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _built():
+    from paper_2609_00049_gb300 import build as b
+    b.build()
+    rq.lib()
+
+
+def _weights(d, H, Hkv, dh, f):
+    shapes = {"g1": (d,), "Wq": (H * dh, d), "Wk": (Hkv * dh, d), "Wv": (Hkv * dh, d), "Wo": (d, H * dh),
+              "g2": (d,), "Wg": (f, d), "Wu": (f, d), "Wd": (d, f)}
+    return {k: torch.zeros(shapes[k]) for k in KEYS}
+
+
+@pytest.mark.parametrize("kl", [False, True])
+def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl):
+    d, H, Hkv, dh, f, S, L = 128, 4, 2, 32, 320, 2, 8
+    dims = rq.block_dims(d, H, Hkv, dh, f)
+    W_this, W_next = _weights(d, H, Hkv, dh, f), _weights(d, H, Hkv, dh, f)
+    x, x_hat = torch.zeros(S, L, d), torch.ones(S, L, d)
+    calls = []
+
+    def module_inputs(dims_, weights, xin, module, X_out, ws, stream=None):
+        calls.append(("inputs", module, dict(weights), xin))
+
+    def accumulate(chunks, n, x_fp_chunks=None, device="cuda", stream=None):
+        (X,) = list(chunks)
+        assert X.shape == (S * L, n)
+        return torch.zeros(n, n), None, X.shape[0]
+
+    def prepare(H_, T, damp_frac=0.01, D_sum=None, stream=None):
+        n = H_.shape[0]
+        return layer.Prepared(torch.zeros(n, n), torch.zeros(n, n), torch.zeros(n, dtype=torch.uint8), T)
+
+    def sweep(dims_, this_block, next_block, xin, module, U, qcfg, bcfg, W, codes, scale, zero, **kw):
+        calls.append(("sweep", module, bcfg.b_global_start, bcfg.B_total, dict(kw["this_block_hat"]), kw["x_hat"],
+                      next_block is None, kw["head_Wh"] is not None))
+        assert this_block is W_this and xin is x
+        W.fill_(float(len(calls)))
+        return 7
+
+    monkeypatch.setattr(pb, "realq_block_module_inputs", module_inputs)
+    monkeypatch.setattr(pb.layer, "accumulate", accumulate)
+    monkeypatch.setattr(pb.layer, "prepare", prepare)
+    monkeypatch.setattr(pb, "realq_quantize_layer_window", sweep)
+    monkeypatch.setattr(pb, "realq_workspace_status", lambda ws, stream=None: 0)
+    monkeypatch.setattr(pb, "workspace", lambda nbytes, device=None: torch.zeros(8, dtype=torch.uint8))
+    q = rq.quant_cfg(group_size=64, block_size=64)
+    if kl:
+        out, W_hat = pb.quantize_block_exact(dims, W_this, x, q, 1e-3, x_hat=x_hat, head_gf=torch.zeros(d),
+                                             head_Wh=torch.zeros(50, d))
+    else:
+        out, W_hat = pb.quantize_block_exact(dims, W_this, x, q, 1e-3, x_hat=x_hat, W_next=W_next,
+                                             F_this=torch.zeros(d, d), F_next=torch.zeros(d, d))
+    sweeps = [c for c in calls if c[0] == "sweep"]
+    inputs = [c for c in calls if c[0] == "inputs"]
+    order = ["q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj"]
+    assert [c[1] for c in sweeps] == order and [c[1] for c in inputs] == order
+    # column blocks: six modules of 128 inputs (2 blocks each), o_proj 128, down 320 (5 blocks)
+    nb = [2, 2, 2, 2, 2, 2, 5]
+    starts = [1 + sum(nb[:i]) for i in range(7)]
+    assert [c[2] for c in sweeps] == starts
+    assert all(c[3] == sum(nb) for c in sweeps)
+    key = {"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg", "up_proj": "Wu",
+           "down_proj": "Wd"}
+    for i, (inp, sw) in enumerate(zip(inputs, sweeps)):
+        assert inp[3] is x_hat and sw[5] is x_hat                  # the current pass runs on x̂
+        for j, prev in enumerate(order):
+            # modules before this one are their dequantized weights; the rest the reference
+            want = out[prev].W if j < i else W_this[key[prev]]
+            assert inp[2][key[prev]] is want and sw[4][key[prev]] is want
+        assert sw[6] == kl and sw[7] == kl                          # the next block or the LM head
+    for md in order:
+        assert W_hat[key[md]] is out[md].W and out[md].adam_t == 7
+        assert out[md].block_loss.shape == (nb[order.index(md)], 2)
