@@ -366,20 +366,32 @@ def module_inputs(module: str, x: np.ndarray, P: Dict) -> np.ndarray:
     return a.reshape(-1, a.shape[-1])
 
 
-def window_gradient_fn(module: str, x: np.ndarray, P_this: Dict, P_next: Dict, F_this: np.ndarray,
-                       F_next: np.ndarray, x_hat=None, P_hat=None):
-    """(W, alpha) -> (loss, gradient) of the exact two-block window for the
-    Block-GD step of the module's sweep (alpha is the step's blend weight)."""
-    def fn(W, alpha):
-        return sliding_window_module(module, W, x, P_this, P_next, alpha, F_this, F_next, x_hat, P_hat)
+def _minibatch(x, k):
+    """Mini-batch k of a rotation: x itself when it is one array, else
+    x[k mod len(x)]."""
+    if x is None or isinstance(x, np.ndarray):
+        return x
+    return x[k % len(x)]
+
+
+def window_gradient_fn(module: str, x, P_this: Dict, P_next: Dict, F_this: np.ndarray, F_next: np.ndarray,
+                       x_hat=None, P_hat=None):
+    """(W, alpha, k) -> (loss, gradient) of the exact two-block window for
+    the Block-GD step of the module's sweep (alpha is the step's blend
+    weight).  x (and x_hat) are block l's inputs, or a list of calibration
+    mini-batches of them, step k taking mini-batch k mod their number."""
+    def fn(W, alpha, k=0):
+        return sliding_window_module(module, W, _minibatch(x, k), P_this, P_next, alpha, F_this, F_next,
+                                     _minibatch(x_hat, k), P_hat)
     return fn
 
 
-def kl_gradient_fn(module: str, x: np.ndarray, P_this: Dict, head: Dict, x_hat=None, P_hat=None):
-    """(W, alpha) -> (loss, gradient) of the final block's KL at the LM head
-    (no window: alpha is not used)."""
-    def fn(W, alpha):
-        return kl_final_module(module, W, x, P_this, head, x_hat, P_hat)
+def kl_gradient_fn(module: str, x, P_this: Dict, head: Dict, x_hat=None, P_hat=None):
+    """(W, alpha, k) -> (loss, gradient) of the final block's KL at the LM
+    head (no window: alpha is not used; x, x_hat and k as in
+    window_gradient_fn)."""
+    def fn(W, alpha, k=0):
+        return kl_final_module(module, W, _minibatch(x, k), P_this, head, _minibatch(x_hat, k), P_hat)
     return fn
 
 

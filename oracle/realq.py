@@ -329,13 +329,17 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
       rotation, whose gradient is taken in token form, and then optionally
       a_loss_clip: the per-token output clipping percentile (0.95 in the
       paper's small-model runs; see loss_clip_factors); or
-      gradient_fn: a callable (W, alpha) -> (loss, G) that gives the
+      gradient_fn: a callable (W, alpha, k) -> (loss, G) that gives the
       surrogate and its gradient in W (m x n) at the current weights, in
       place of the layer-level surrogate: the exact two-block window of
       Sec. 4.4 and the final block's KL at the LM head (App. "Pre-computation
       of the aggregated Fisher and last-transformer-block handling"), both
-      stated in oracle.block.  The per-block values it records are its own
-      loss before and after the block's steps.
+      stated in oracle.block.  k = (b_global - 1) * steps_per_block + s is
+      the step's place in the rotation over calibration mini-batches (Sec.
+      4.3: each step's forward pass uses a calibration mini-batch), the same
+      rotation as minibatches above.  The per-block values it records are its
+      own loss before the block's steps (on the first step's mini-batch) and
+      after them (on the last step's).
 
     Readings: group parameters are computed at the first column of each group
     from the current (compensated, Block-GD-updated) weights; group_size 0
@@ -416,7 +420,8 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             gfn = bgd.get("gradient_fn")
             if gfn is not None:
                 Feff = None
-                before = gfn(W, alpha)[0] if record else None
+                k0 = (b_global - 1) * bgd.get("steps_per_block", 1)
+                before = gfn(W, alpha, k0)[0] if record else None
             else:
                 Feff = Fm if Fn is None else alpha * Fm + (1.0 - alpha) * Fn
                 before = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
@@ -426,7 +431,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             for si in range(steps):
                 Hstep = Hbar
                 if gfn is not None:
-                    G = gfn(W, alpha)[1][:, be:]
+                    G = gfn(W, alpha, (b_global - 1) * steps + si)[1][:, be:]
                 elif mbt:
                     if Dbar is not None:
                         raise ValueError("mini-batch tokens with perturbed inputs are not supported")
@@ -445,7 +450,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
                 else:
                     W[:, be:] -= opt.direction(G, slice(be, n))
             if gfn is not None:
-                after = gfn(W, alpha)[0] if record else None
+                after = gfn(W, alpha, (b_global - 1) * steps + steps - 1)[0] if record else None
             else:
                 after = surrogate_moment(W, W0, Hbar, Feff) if (record and Dbar is None) else None
             block_loss.append((b, alpha, before, after))

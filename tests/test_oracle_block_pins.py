@@ -516,3 +516,58 @@ def test_block_driver_with_small_sgd_steps_lowers_every_modules_loss():
     for res in list(out.values()) + list(out_kl.values()):
         for _, _, before, after in res["block_loss"]:
             assert after < before, (before, after)
+
+
+# --- calibration mini-batches of the exact losses (Sec. 4.3) ---------------
+
+def test_minibatch_losses_average_to_the_full_batch_loss():
+    # the losses are means over tokens and attention stays within a
+    # sequence, so over mini-batches of whole sequences of equal size the
+    # mean of the mini-batch losses and gradients is the full batch's
+    r, P, Pn, x, x_hat, F, Fn = _driver_case(34)
+    x = np.concatenate([x, r.standard_normal(x.shape)], axis=0)            # 4 sequences
+    x_hat = x + 0.05 * r.standard_normal(x.shape)
+    head = ob.head_params(r, x.shape[2], 13, scale=1.5)
+    W = P["Wg"] + 0.05 * r.standard_normal(P["Wg"].shape)
+    mb = [x[i:i + 2] for i in (0, 2)]
+    mbh = [x_hat[i:i + 2] for i in (0, 2)]
+    for full, part in ((ob.window_gradient_fn("gate_proj", x, P, Pn, F, Fn, x_hat),
+                        ob.window_gradient_fn("gate_proj", mb, P, Pn, F, Fn, mbh)),
+                       (ob.kl_gradient_fn("gate_proj", x, P, head, x_hat),
+                        ob.kl_gradient_fn("gate_proj", mb, P, head, mbh))):
+        lf, gf = full(W, 0.4)
+        parts = [part(W, 0.4, k) for k in range(2)]
+        assert parts[0][0] != parts[1][0]
+        assert abs(np.mean([p[0] for p in parts]) - lf) <= 1e-12 * abs(lf)
+        np.testing.assert_allclose(np.mean([p[1] for p in parts], axis=0), gf, rtol=0,
+                                   atol=1e-12 * np.abs(gf).max())
+
+
+def test_sweep_rotation_over_minibatches_is_a_full_batch_step_to_first_order():
+    # K plain gradient steps per block over K mini-batches (the rotation
+    # starting at mini-batch 0 for every block when steps_per_block = K) sum
+    # to K lr times the full-batch gradient up to O(lr^2): with a small lr the
+    # sweep equals the full-batch one with a single step of K lr
+    r, P, Pn, x, x_hat, F, Fn = _driver_case(35)
+    x = np.concatenate([x, r.standard_normal(x.shape)], axis=0)
+    x_hat = x + 0.05 * r.standard_normal(x.shape)
+    mb, mbh = [x[i:i + 2] for i in (0, 2)], [x_hat[i:i + 2] for i in (0, 2)]
+    X = ob.module_inputs("up_proj", x_hat, P)
+    H_sum, T = oracle.hessian_sum([X])
+    lr = 1e-3
+    kw = dict(group_size=16, block_size=16)
+    rot = oracle.realq_sweep(P["Wu"], H_sum, T, bgd={
+        "lr": lr, "optimizer": "sgd", "steps_per_block": 2, "B_total": 1,
+        "gradient_fn": ob.window_gradient_fn("up_proj", mb, P, Pn, F, Fn, mbh)}, **kw)
+    full = oracle.realq_sweep(P["Wu"], H_sum, T, bgd={
+        "lr": 2 * lr, "optimizer": "sgd", "steps_per_block": 1, "B_total": 1,
+        "gradient_fn": ob.window_gradient_fn("up_proj", x, P, Pn, F, Fn, x_hat)}, **kw)
+    first = oracle.realq_sweep(P["Wu"], H_sum, T, bgd={
+        "lr": 2 * lr, "optimizer": "sgd", "steps_per_block": 1, "B_total": 1,
+        "gradient_fn": ob.window_gradient_fn("up_proj", mb[:1], P, Pn, F, Fn, mbh[:1])}, **kw)
+    assert np.array_equal(rot["codes"], full["codes"])
+    d_rot = np.abs(rot["deq"] - full["deq"]).max()
+    d_first = np.abs(first["deq"] - full["deq"]).max()
+    # (the scales are fp32, so an O(lr^2) change of a group's extreme weight
+    # can move its scale, and every weight of the group, by one fp32 step)
+    assert d_rot <= 1e-6 and d_rot <= 1e-2 * d_first, (d_rot, d_first)

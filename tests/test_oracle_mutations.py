@@ -95,9 +95,13 @@ BLOCK_MUTATIONS = {
 # the sweep's hook for the exact losses (oracle/realq.py), caught by the
 # block pins: the gradient's columns shifted to the quantized side
 SWEEP_HOOK_MUTATIONS = {
-    "hook_columns": ("G = gfn(W, alpha)[1][:, be:]", "G = gfn(W, alpha)[1][:, :n - be]"),
-    "hook_blend": ("before = gfn(W, alpha)[0] if record else None",
-                   "before = gfn(W, 1.0)[0] if record else None"),
+    "hook_columns": ("G = gfn(W, alpha, (b_global - 1) * steps + si)[1][:, be:]",
+                     "G = gfn(W, alpha, (b_global - 1) * steps + si)[1][:, :n - be]"),
+    "hook_blend": ("before = gfn(W, alpha, k0)[0] if record else None",
+                   "before = gfn(W, 1.0, k0)[0] if record else None"),
+    # the rotation over calibration mini-batches stuck at the first one
+    "hook_rotation": ("G = gfn(W, alpha, (b_global - 1) * steps + si)[1][:, be:]",
+                      "G = gfn(W, alpha, 0)[1][:, be:]"),
 }
 
 

@@ -238,8 +238,8 @@ def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None):
     if capture is not None:
         inner = fn
 
-        def fn(W, alpha):
-            out = inner(W, alpha)
+        def fn(W, alpha, k=0):
+            out = inner(W, alpha, k)
             capture.append((W.copy(), out[1]))
             return out
     Hs, T = orq.hessian_sum([c["X"]])
