@@ -599,11 +599,19 @@ realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_di
  * alpha = 1 - (b_global - 1)/(B_total - 1), 1 when B_total = 1, b_global =
  * b_global_start + b; or realq_block_module_kl), then one Adam (or SGD) step
  * on the columns >= b_end of W_work with those columns of G.
- *   dims, this_block, this_block_hat, next_block, S, L, x, x_hat, module,
- *   F_this, F_next
- *             as realq_block_module_window.  The module's weight in
+ *   dims, this_block, this_block_hat, next_block, S, L, module, F_this,
+ *   F_next    as realq_block_module_window.  The module's weight in
  *             this_block (fp32) is both the loss's reference and the sweep's
  *             W0; m x n is its shape (out x in).
+ *   n_minibatch, x, x_hat
+ *             the calibration mini-batches (Sec. 4.3: each step's forward
+ *             pass uses a calibration mini-batch): x and x_hat (NULL: x) hold
+ *             n_minibatch S sequences of L tokens (n_minibatch S L x d), and
+ *             step s of column block b takes mini-batch
+ *             ((b_global - 1) steps_per_block + s) mod n_minibatch, the
+ *             sequences k S .. k S + S - 1.  The losses before and after a
+ *             block's steps are those of its first and last step's
+ *             mini-batch.
  *   head_gf, head_Wh, vocab   the final norm and LM head (next_block NULL);
  *             ignored otherwise.
  *   U, dead   realq_hessian_prepare of the module's input second moment
@@ -627,8 +635,8 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
                                            const realq_block_weights_t *this_block,
                                            const realq_block_weights_t *this_block_hat,
                                            const realq_block_weights_t *next_block, int64_t S, int64_t L,
-                                           const float *x, const float *x_hat, int module, const float *F_this,
-                                           const float *F_next,
+                                           int64_t n_minibatch, const float *x, const float *x_hat, int module,
+                                           const float *F_this, const float *F_next,
                                            const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
                                            const uint8_t *dead, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,

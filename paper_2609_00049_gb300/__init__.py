@@ -158,7 +158,8 @@ _SIGS = {
     "realq_quantize_window_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64, _int, _i64,
                                               ctypes.POINTER(QuantCfg)], _sz),
     "realq_quantize_layer_window": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights),
-                                     ctypes.POINTER(BlockWeights), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
+                                     ctypes.POINTER(BlockWeights), ctypes.POINTER(BlockWeights), _i64, _i64, _i64,
+                                     _vp, _vp,
                                      _int, _vp, _vp, _vp, _vp, _i64,
                                      _vp, _vp, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _P_i64,
                                      _vp, _vp, _vp, _vp, _int, _vp, _i64, _i64, _vp, _sz], _int),
@@ -737,16 +738,21 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
                                 adam_t: int = 0, W_deq=None, block_loss: Optional[torch.Tensor] = None,
                                 block_begin: int = 0, block_end: Optional[int] = None, ws=None,
                                 this_block_hat: Optional[dict] = None, x_hat: Optional[torch.Tensor] = None,
-                                stream=None) -> int:
+                                n_minibatch: int = 1, stream=None) -> int:
     """The column sweep of one module of decoder block l with Block-GD on the
     exact two-block window (next_block given, with F_this and F_next) or on
     the final block's KL at the LM head (next_block None, with head_gf and
     head_Wh); x (S, L, d) is block l's input.  The module's weight in
     this_block is the reference and the sweep's W0; this_block_hat / x_hat
     are block l's weights and input in the current pass (the model quantized
-    so far; None: the reference ones).  Runs blocks [block_begin, block_end);
-    returns the optimizer step counter."""
-    S, L, d = x.shape
+    so far; None: the reference ones).  With n_minibatch > 1, x and x_hat
+    hold that many calibration mini-batches of whole sequences, and each
+    Block-GD step takes one in rotation.  Runs blocks [block_begin,
+    block_end); returns the optimizer step counter."""
+    S_all, L, d = x.shape
+    if n_minibatch < 1 or S_all % n_minibatch:
+        raise ValueError(f"{S_all} sequences do not split into {n_minibatch} mini-batches")
+    S = S_all // n_minibatch
     Wref = this_block[{"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg",
                        "up_proj": "Wu", "down_proj": "Wd"}[module]]
     m, n = Wref.shape
@@ -766,7 +772,8 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
     V = int(head_Wh.shape[0]) if head_Wh is not None else 0
     _check(lib().realq_quantize_layer_window(
         _stream(stream), ctypes.byref(dims), ctypes.byref(a), _opt_weights(this_block_hat),
-        ctypes.byref(b) if b is not None else None, S, L, _ptr(x), _ptr(x_hat), BLOCK_MODULES.index(module),
+        ctypes.byref(b) if b is not None else None, S, L, int(n_minibatch), _ptr(x), _ptr(x_hat),
+        BLOCK_MODULES.index(module),
         _ptr(F_this), _ptr(F_next), _ptr(head_gf), _ptr(head_Wh), V,
         _ptr(U), _ptr(dead), ctypes.byref(qcfg), ctypes.byref(bcfg), _ptr(W_work), _ptr(adam_m), _ptr(adam_v),
         ctypes.byref(t), _ptr(codes), _ptr(scale), _ptr(zero), _ptr(W_deq),

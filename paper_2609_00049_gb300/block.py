@@ -521,7 +521,7 @@ def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor,
                          F_this: Optional[torch.Tensor] = None, F_next: Optional[torch.Tensor] = None,
                          head_gf: Optional[torch.Tensor] = None, head_Wh: Optional[torch.Tensor] = None,
                          steps_per_block: int = 1, optimizer: int = REALQ_OPT_ADAM,
-                         modules: Sequence[str] = BLOCK_MODULES, stream=None):
+                         modules: Sequence[str] = BLOCK_MODULES, n_minibatch: int = 1, stream=None):
     """Quantizes the linear modules of decoder block l in order, each with
     Block-GD on the exact two-block window (W_next, F_this, F_next given) or,
     for the last block, on the KL at the LM head (head_gf, head_Wh given).
@@ -532,22 +532,25 @@ def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor,
     (realq_block_module_inputs with the weights quantized so far, on x_hat),
     their Hessian and factor, then realq_quantize_layer_window with b_global
     running over the column blocks of all the modules; its dequantized
-    weights then replace it in the current weights.  Returns each module's
-    ExactModule and the final current weights."""
-    S, L, d = x.shape
+    weights then replace it in the current weights.  With n_minibatch > 1
+    the sequences of x form that many calibration mini-batches: the Hessians
+    take all of them, each Block-GD step one in rotation.  Returns each
+    module's ExactModule and the final current weights."""
+    S_all, L, d = x.shape
+    S = S_all // n_minibatch
     dev = x.device
     nb = {md: -(-W_this[_MODULE_KEY[md]].shape[1] // qcfg.block_size) for md in modules}
     B_total = sum(nb.values())
     vocab = int(head_Wh.shape[0]) if head_Wh is not None else 0
     W_hat = dict(W_this)
-    bws = workspace(realq_block_workspace_size(dims, S, L), dev)
+    bws = workspace(realq_block_workspace_size(dims, S_all, L), dev)
     g = qcfg.group_size
     out = {}
     b_start = 1
     for md in modules:
         key = _MODULE_KEY[md]
         m, n = W_this[key].shape
-        X = torch.empty((S * L, n), dtype=torch.float32, device=dev)
+        X = torch.empty((S_all * L, n), dtype=torch.float32, device=dev)
         realq_block_module_inputs(dims, W_hat, x if x_hat is None else x_hat, md, X, bws, stream=stream)
         H, _, T = layer.accumulate([X], n, device=dev, stream=stream)
         prep = layer.prepare(H, T, qcfg.damp_frac, stream=stream)
@@ -565,7 +568,8 @@ def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor,
         t = realq_quantize_layer_window(dims, W_this, W_next if head_Wh is None else None, x, md, prep.U, qcfg, b,
                                         W, codes, scale, zero, F_this=F_this, F_next=F_next, head_gf=head_gf,
                                         head_Wh=head_Wh, dead=prep.dead, adam_m=am, adam_v=av, block_loss=loss,
-                                        ws=ws, this_block_hat=W_hat, x_hat=x_hat, stream=stream)
+                                        ws=ws, this_block_hat=W_hat, x_hat=x_hat, n_minibatch=n_minibatch,
+                                        stream=stream)
         realq_workspace_status(ws, stream=stream)
         W_hat = dict(W_hat)
         W_hat[key] = W

@@ -592,7 +592,7 @@ struct WindowStep {
     realq_stream_t stream;
     const realq_block_dims_t *dims;
     const realq_block_weights_t *this_block, *this_block_hat, *next_block;
-    int64_t S, L;
+    int64_t S, L, n_minibatch;
     const float *x, *x_hat;
     int module;
     const float *F_this, *F_next, *gf, *Wh;
@@ -605,13 +605,17 @@ struct WindowStep {
     size_t mws_bytes;
 };
 
-static realq_status_t window_loss(const WindowStep &w, const float *W, float alpha, float *loss) {
+// the loss and gradient on calibration mini-batch k of the rotation
+// (sequences (k mod n_minibatch) S .. + S of x and x_hat)
+static realq_status_t window_loss(const WindowStep &w, const float *W, float alpha, int64_t k, float *loss) {
+    const int64_t off = (k % w.n_minibatch) * w.S * w.L * w.dims->d;
+    const float *x = w.x + off, *xh = w.x_hat ? w.x_hat + off : nullptr;
     if (w.next_block)
-        return realq_block_module_window(w.stream, w.dims, w.this_block, w.this_block_hat, w.next_block, w.S, w.L,
-                                         w.x, w.x_hat, w.module, W, alpha, w.F_this, w.F_next, w.grad, loss, w.mws,
+        return realq_block_module_window(w.stream, w.dims, w.this_block, w.this_block_hat, w.next_block, w.S, w.L, x,
+                                         xh, w.module, W, alpha, w.F_this, w.F_next, w.grad, loss, w.mws,
                                          w.mws_bytes);
-    return realq_block_module_kl(w.stream, w.dims, w.this_block, w.this_block_hat, w.S, w.L, w.x, w.x_hat, w.module,
-                                 W, w.gf, w.Wh, w.vocab, w.grad, loss, w.mws, w.mws_bytes);
+    return realq_block_module_kl(w.stream, w.dims, w.this_block, w.this_block_hat, w.S, w.L, x, xh, w.module, W,
+                                 w.gf, w.Wh, w.vocab, w.grad, loss, w.mws, w.mws_bytes);
 }
 
 static realq_status_t window_step(cudaStream_t s, SweepPlan &p, int64_t b, void *ctx) {
@@ -622,15 +626,16 @@ static realq_status_t window_step(cudaStream_t s, SweepPlan &p, int64_t b, void 
     float alpha = 1.f;
     if (w.cfg.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(w.cfg.B_total - 1));
     float *bl = w.block_loss ? w.block_loss + 2 * b : nullptr;
-    for (int k = 0; k < w.cfg.steps_per_block; ++k) {
-        // the loss and its gradient at the current weights: the dequantized
-        // columns < be and the free ones
-        REALQ_TRY(window_loss(w, p.W, alpha, k == 0 ? bl : nullptr));
+    const int64_t steps = w.cfg.steps_per_block, k0 = (b_global - 1) * steps;
+    for (int64_t k = 0; k < steps; ++k) {
+        // the loss and its gradient at the current weights (the dequantized
+        // columns < be and the free ones) on the step's mini-batch
+        REALQ_TRY(window_loss(w, p.W, alpha, k0 + k, k == 0 ? bl : nullptr));
         const int64_t t = ++(*w.adam_t);
         REALQ_TRY(adam_cols(s, p.m, p.n, be, w.grad, p.W, w.adam_m, w.adam_v, w.cfg.lr, w.cfg.beta1, w.cfg.beta2,
                             w.cfg.eps, t, w.cfg.optimizer == REALQ_OPT_SGD));
     }
-    if (bl) REALQ_TRY(window_loss(w, p.W, alpha, bl + 1));
+    if (bl) REALQ_TRY(window_loss(w, p.W, alpha, k0 + steps - 1, bl + 1));
     return REALQ_OK;
 }
 
@@ -651,8 +656,8 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
                                            const realq_block_weights_t *this_block,
                                            const realq_block_weights_t *this_block_hat,
                                            const realq_block_weights_t *next_block, int64_t S, int64_t L,
-                                           const float *x, const float *x_hat, int module, const float *F_this,
-                                           const float *F_next,
+                                           int64_t n_minibatch, const float *x, const float *x_hat, int module,
+                                           const float *F_this, const float *F_next,
                                            const float *head_gf, const float *head_Wh, int64_t vocab, const float *U,
                                            const uint8_t *dead, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, float *W_work, float *adam_m, float *adam_v,
@@ -665,6 +670,8 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
     REALQ_TRY(block_loss_check(dims, this_block, this_block_hat, next_block, S, L, x, module, F_this, F_next, head_gf,
                                head_Wh, next_block ? 0 : vocab, who, &m, &n, &mws));
     if (m * n > ((int64_t)1 << 38)) return fail(REALQ_ERR_UNSUPPORTED, "%s: m n must be below 2^38", who);
+    if (n_minibatch < 1 || n_minibatch > ((int64_t)1 << 38) / (S * L * dims->d))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: n_minibatch >= 1 and n_minibatch S L d < 2^38 required", who);
     REALQ_TRY(check_qcfg(qcfg, n));
     REALQ_TRY(check_bcfg(bcfg));
     if (!bcfg || bcfg->steps_per_block < 1)
@@ -693,8 +700,8 @@ realq_status_t realq_quantize_layer_window(realq_stream_t stream, const realq_bl
         default: W0 = this_block->Wd; break;
     }
     char *base = static_cast<char *>(ws);
-    WindowStep w{stream, dims, this_block, this_block_hat, next_block, S, L, x, x_hat, module, F_this, F_next,
-                 head_gf, head_Wh, vocab, *bcfg, adam_m, adam_v, adam_t, reinterpret_cast<float *>(base + sw),
+    WindowStep w{stream, dims, this_block, this_block_hat, next_block, S, L, n_minibatch, x, x_hat, module, F_this,
+                 F_next, head_gf, head_Wh, vocab, *bcfg, adam_m, adam_v, adam_t, reinterpret_cast<float *>(base + sw),
                  block_loss, base + sw + gb, mws};
     if (block_begin == 0) {
         // (S is the sequence count here; the stream is cast directly)

@@ -244,11 +244,11 @@ def test_window_sweep_entry_point_rejects_bad_arguments(L):
     t = ctypes.c_int64(0)
 
     def sweep(module=6, nxt=True, F=fake, vocab=0, head=fake, bcfg=None, qcfg=q, blocks=(0, 2), nbytes=big,
-              deq_dtype=0, adam=fake):
+              deq_dtype=0, adam=fake, nmb=1):
         b = bcfg if bcfg is not None else rq.bgd_cfg(1e-3)
         return L.realq_quantize_layer_window(None, ctypes.byref(ok), ctypes.byref(w), None,
-                                             ctypes.byref(w) if nxt else None, 2, 8, fake, None, module, F, fake, head,
-                                             head,
+                                             ctypes.byref(w) if nxt else None, 2, 8, nmb, fake, None, module, F, fake,
+                                             head, head,
                                              vocab, fake, None, ctypes.byref(qcfg), ctypes.byref(b), fake, adam, adam,
                                              ctypes.byref(t), fake, fake, fake, None, deq_dtype, None, blocks[0],
                                              blocks[1], fake, nbytes)
@@ -269,6 +269,8 @@ def test_window_sweep_entry_point_rejects_bad_arguments(L):
     assert sweep(qcfg=rq.quant_cfg(block_size=96)) == rq.REALQ_ERR_INVALID_ARG
     assert sweep(blocks=(0, 3)) == rq.REALQ_ERR_INVALID_ARG                         # down_proj: 96 columns, 2 blocks
     assert sweep(deq_dtype=5) == rq.REALQ_ERR_INVALID_ARG
+    assert sweep(nmb=0) == rq.REALQ_ERR_INVALID_ARG
+    assert "n_minibatch" in rq.realq_last_error()
     assert sweep(nbytes=n_win - 1) == rq.REALQ_ERR_WORKSPACE
     assert "quantize_layer_window" in rq.realq_last_error()
     assert t.value == 0

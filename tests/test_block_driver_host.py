@@ -28,8 +28,8 @@ def _weights(d, H, Hkv, dh, f):
     return {k: torch.zeros(shapes[k]) for k in KEYS}
 
 
-@pytest.mark.parametrize("kl", [False, True])
-def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl):
+@pytest.mark.parametrize("kl,nmb", [(False, 1), (True, 1), (False, 2)])
+def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl, nmb):
     d, H, Hkv, dh, f, S, L = 128, 4, 2, 32, 320, 2, 8
     dims = rq.block_dims(d, H, Hkv, dh, f)
     W_this, W_next = _weights(d, H, Hkv, dh, f), _weights(d, H, Hkv, dh, f)
@@ -41,7 +41,7 @@ def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl):
 
     def accumulate(chunks, n, x_fp_chunks=None, device="cuda", stream=None):
         (X,) = list(chunks)
-        assert X.shape == (S * L, n)
+        assert X.shape == (S * L, n)                                   # the Hessian takes every mini-batch
         return torch.zeros(n, n), None, X.shape[0]
 
     def prepare(H_, T, damp_frac=0.01, D_sum=None, stream=None):
@@ -51,6 +51,7 @@ def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl):
     def sweep(dims_, this_block, next_block, xin, module, U, qcfg, bcfg, W, codes, scale, zero, **kw):
         calls.append(("sweep", module, bcfg.b_global_start, bcfg.B_total, dict(kw["this_block_hat"]), kw["x_hat"],
                       next_block is None, kw["head_Wh"] is not None))
+        assert kw["n_minibatch"] == nmb
         assert this_block is W_this and xin is x
         W.fill_(float(len(calls)))
         return 7
@@ -64,10 +65,10 @@ def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl):
     q = rq.quant_cfg(group_size=64, block_size=64)
     if kl:
         out, W_hat = pb.quantize_block_exact(dims, W_this, x, q, 1e-3, x_hat=x_hat, head_gf=torch.zeros(d),
-                                             head_Wh=torch.zeros(50, d))
+                                             head_Wh=torch.zeros(50, d), n_minibatch=nmb)
     else:
         out, W_hat = pb.quantize_block_exact(dims, W_this, x, q, 1e-3, x_hat=x_hat, W_next=W_next,
-                                             F_this=torch.zeros(d, d), F_next=torch.zeros(d, d))
+                                             F_this=torch.zeros(d, d), F_next=torch.zeros(d, d), n_minibatch=nmb)
     sweeps = [c for c in calls if c[0] == "sweep"]
     inputs = [c for c in calls if c[0] == "inputs"]
     order = ["q_proj", "k_proj", "v_proj", "o_proj", "gate_proj", "up_proj", "down_proj"]

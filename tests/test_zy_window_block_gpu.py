@@ -230,11 +230,20 @@ def _sweep_inputs(seed, module, kl, current=False):
                 W_hat=W_hat)
 
 
-def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None):
+def _split(a, nmb):
+    # nmb calibration mini-batches of whole sequences
+    if a is None or nmb == 1:
+        return a
+    s = a.shape[0] // nmb
+    return [a[i * s:(i + 1) * s] for i in range(nmb)]
+
+
+def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None, nmb=1):
+    x, xh = _split(c["x"], nmb), _split(c["x_hat"], nmb)
     if c["head"] is not None:
-        fn = ob.kl_gradient_fn(module, c["x"], c["P"], c["head"], c["x_hat"], c["P_hat"])
+        fn = ob.kl_gradient_fn(module, x, c["P"], c["head"], xh, c["P_hat"])
     else:
-        fn = ob.window_gradient_fn(module, c["x"], c["P"], c["Pn"], c["F"], c["Fn"], c["x_hat"], c["P_hat"])
+        fn = ob.window_gradient_fn(module, x, c["P"], c["Pn"], c["F"], c["Fn"], xh, c["P_hat"])
     if capture is not None:
         inner = fn
 
@@ -248,7 +257,7 @@ def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None):
     return orq.realq_sweep(c["P"][ob._MODULE_WEIGHT[module]], Hs, T, bgd=bgd, **QKW)
 
 
-def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=None):
+def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=None, nmb=1):
     W0 = c["W"][ob._MODULE_WEIGHT[module]]
     m, n = W0.shape
     H, _, T = layer.accumulate([_dev(c["X"])], n)
@@ -267,7 +276,7 @@ def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=N
                      av=torch.empty((m, n), dtype=torch.float32, device="cuda"),
                      loss=torch.full((nb, 2), -1.0, dtype=torch.float32, device="cuda"), t=0,
                      ws=rq.workspace(rq.realq_quantize_window_workspace_size(
-                         c["dims"], c["x"].shape[0], c["x"].shape[1], module, q,
+                         c["dims"], c["x"].shape[0] // nmb, c["x"].shape[1], module, q,
                          vocab=0 if c["head"] is None else c["head"]["Wh"].shape[0])))
     b0, b1 = blocks or (0, nb)
     kw = dict(F_this=_dev(c["F"]), F_next=_dev(c["Fn"])) if c["head"] is None else dict(
@@ -276,7 +285,8 @@ def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=N
         c["dims"], c["W"], c["Wn"] if c["head"] is None else None, _dev(c["x"]), module, prep.U, q, b, state["W"],
         state["codes"], state["scale"], state["zero"], dead=prep.dead, adam_m=state["am"], adam_v=state["av"],
         adam_t=state["t"], block_loss=state["loss"], block_begin=b0, block_end=b1, ws=state["ws"],
-        this_block_hat=c["W_hat"], x_hat=_dev(c["x_hat"]) if c["x_hat"] is not None else None, **kw)
+        this_block_hat=c["W_hat"], x_hat=_dev(c["x_hat"]) if c["x_hat"] is not None else None, n_minibatch=nmb,
+        **kw)
     rq.realq_workspace_status(state["ws"])
     torch.cuda.synchronize()
     return state
@@ -320,6 +330,20 @@ def test_window_sweep_with_gradient_steps_matches_the_oracle(module, kl, lr, ste
     st = _gpu_sweep(c, module, "sgd", lr, steps, 3, 10)
     n = c["W"][ob._MODULE_WEIGHT[module]].shape[1]
     assert st["t"] == orc["adam_t"] == steps * len(orc["block_loss"])
+    _check_sweep(orc, st, n, lr, 3e-3 if kl else 1e-3)
+
+
+@pytest.mark.parametrize("module,kl,steps,nmb", [("down_proj", False, 2, 2), ("o_proj", False, 1, 4),
+                                                 ("up_proj", True, 1, 2)])
+def test_window_sweep_over_minibatches_matches_the_oracle(module, kl, steps, nmb):
+    # each Block-GD step on one calibration mini-batch of whole sequences, in
+    # rotation (Sec. 4.3), with a perturbed current pass
+    lr = 10.0 if kl else 0.3
+    c = _sweep_inputs(12, module, kl, current=True)
+    orc = _oracle_sweep(c, module, "sgd", lr, steps, 3, 10, nmb=nmb)
+    st = _gpu_sweep(c, module, "sgd", lr, steps, 3, 10, nmb=nmb)
+    n = c["W"][ob._MODULE_WEIGHT[module]].shape[1]
+    assert st["t"] == orc["adam_t"]
     _check_sweep(orc, st, n, lr, 3e-3 if kl else 1e-3)
 
 
