@@ -1,6 +1,11 @@
-"""Parity of the decoder block of the exact two-block sliding window
-(realq_block_forward, realq_block_window) with the fp64 oracle
-(oracle/block.py: block_forward, next_block_loss), through the C ABI.
+"""Parity of the exact losses of Sec. 4.4 with the fp64 oracle
+(oracle/block.py), through the C ABI: the decoder block's forward and the
+next block's window (realq_block_forward, realq_block_window), a module's
+window and final-block KL with their weight gradients
+(realq_block_module_window, realq_block_module_kl), the final block's KL
+head, a module's calibration inputs (realq_block_module_inputs), the sweep
+with Block-GD on these losses (realq_quantize_layer_window) and the
+block-level loop over the seven modules (block.quantize_block_exact).
 
 Tolerances (fp32 arithmetic, fp32 accumulation over at most max(d, f, L)
 unit-scale terms): the forward within 1e-5 of the output's scale; the
