@@ -52,7 +52,7 @@ from . import realq as _sweep
 __all__ = ["block_params", "block_forward", "block_vjp", "next_block_loss", "sliding_window_down",
            "sliding_window_module", "head_params", "head_logits", "kl_logits", "kl_head_loss", "nll_scores",
            "fisher_sampled", "fisher_tokens", "kl_final_module", "module_inputs", "window_gradient_fn",
-           "kl_gradient_fn", "MODULES", "quantize_block"]
+           "kl_gradient_fn", "MODULES", "quantize_block", "quantize_model"]
 
 EPS = 1e-6
 
@@ -447,3 +447,29 @@ def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] =
         out[module] = res
         b_start += nbs[module]
     return out, P_hat
+
+
+def quantize_model(x: np.ndarray, blocks: Sequence[Dict], fishers: Sequence[np.ndarray], head: Dict, *,
+                   lr_final: float, **kw):
+    """Alg. 1's outer loop (Stage 1) over a stack of L decoder blocks: block
+    l is quantized with quantize_block against the exact two-block window
+    with block l+1 (F^(l), F^(l+1) its aggregated Fishers) or, for the last
+    block, the KL at the LM head, at the learning rate of the reverse-cosine
+    schedule over blocks (eta_l from 0.01 eta_final up to eta_final).  The
+    full-precision input of block l+1 is block l's full-precision output; its
+    input in the model quantized so far is block l's output with its
+    quantized weights on its own such input.  kw go to quantize_block.
+    Returns each block's module results and its quantized weights."""
+    L = len(blocks)
+    x_ref, x_hat = x, x
+    out = []
+    for l, P in enumerate(blocks):
+        last = l == L - 1
+        lr = _sweep.reverse_cosine_lr(l + 1, L, lr_final)
+        res, P_hat = quantize_block(x_ref, P, x_hat=x_hat, P_next=None if last else blocks[l + 1],
+                                    F_this=fishers[l], F_next=None if last else fishers[l + 1],
+                                    head=head if last else None, lr=lr, **kw)
+        out.append((res, P_hat))
+        x_ref = block_forward(x_ref, P)[0]
+        x_hat = block_forward(x_hat, P_hat)[0]
+    return out

@@ -28,6 +28,7 @@ No arithmetic happens here; every step is a call through the C ABI.
 """
 from __future__ import annotations
 
+import math
 from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass
 from typing import Dict, List, Optional, Sequence
@@ -35,7 +36,8 @@ from typing import Dict, List, Optional, Sequence
 import torch
 
 from . import layer
-from . import (BLOCK_MODULES, REALQ_BF16, REALQ_OPT_ADAM, QuantCfg, bgd_cfg, realq_block_module_inputs,
+from . import (BLOCK_MODULES, REALQ_BF16, REALQ_OPT_ADAM, QuantCfg, bgd_cfg, realq_block_forward,
+               realq_block_module_inputs,
                realq_block_workspace_size, realq_graph_begin, realq_graph_end, realq_hessian_accumulate,
                realq_hessian_accumulate_weighted, realq_hessian_prepare_deferred, realq_hessian_prepare_scaled,
                realq_hessian_weighted_workspace_size, realq_hessian_workspace_size, realq_prepare_status,
@@ -576,3 +578,47 @@ def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor,
         out[md] = ExactModule(codes, scale, zero, W, t, loss)
         b_start += nb[md]
     return out, W_hat
+
+
+def reverse_cosine_lr(i: int, L: int, lr_final: float) -> float:
+    """The learning rate of decoder block i (1-based) of L: a reverse-cosine
+    ramp from 0.01 lr_final at the first block to lr_final at the last."""
+    base = 0.01 * lr_final
+    if L <= 1:
+        return lr_final
+    return base + (lr_final - base) * math.sin(0.5 * math.pi * (i - 1) / (L - 1))
+
+
+def quantize_model_exact(dims, blocks: Sequence[Dict[str, torch.Tensor]], x: torch.Tensor,
+                         fishers: Sequence[torch.Tensor], head_gf: torch.Tensor, head_Wh: torch.Tensor,
+                         qcfg: QuantCfg, lr_final: float, **kw):
+    """Alg. 1's outer loop over a stack of decoder blocks with the exact
+    losses: block l with quantize_block_exact against the two-block window
+    with block l+1 (fishers[l], fishers[l+1]: the blocks' aggregated
+    Fishers, d x d) or, for the last block, the KL at the LM head (head_gf,
+    head_Wh), at the reverse-cosine learning rate of block l.  Block l+1's
+    full-precision input is block l's full-precision output, and its input in
+    the quantized model is block l's output with its quantized weights on its
+    own such input (realq_block_forward).  kw go to quantize_block_exact.
+    Returns [(modules, quantized weights)] per block."""
+    Lb = len(blocks)
+    S, L, d = x.shape
+    ws = workspace(realq_block_workspace_size(dims, S, L), x.device)
+    stream = kw.get("stream")
+    x_ref, x_hat = x, x
+    out = []
+    for l, W in enumerate(blocks):
+        last = l == Lb - 1
+        lr = reverse_cosine_lr(l + 1, Lb, lr_final)
+        if last:
+            res, W_hat = quantize_block_exact(dims, W, x_ref, qcfg, lr, x_hat=x_hat, head_gf=head_gf,
+                                              head_Wh=head_Wh, **kw)
+        else:
+            res, W_hat = quantize_block_exact(dims, W, x_ref, qcfg, lr, x_hat=x_hat, W_next=blocks[l + 1],
+                                              F_this=fishers[l], F_next=fishers[l + 1], **kw)
+        out.append((res, W_hat))
+        y_ref, y_hat = torch.empty_like(x), torch.empty_like(x)
+        realq_block_forward(dims, W, x_ref, y_ref, ws, stream=stream)
+        realq_block_forward(dims, W_hat, x_hat, y_hat, ws, stream=stream)
+        x_ref, x_hat = y_ref, y_hat
+    return out

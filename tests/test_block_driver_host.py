@@ -90,3 +90,48 @@ def test_driver_order_global_block_index_and_current_weights(monkeypatch, kl, nm
     for md in order:
         assert W_hat[key[md]] is out[md].W and out[md].adam_t == 7
         assert out[md].block_loss.shape == (nb[order.index(md)], 2)
+
+
+def test_model_loop_schedule_windows_and_inputs(monkeypatch):
+    # Alg. 1's outer loop: the reverse-cosine rate per block, the window to
+    # the next block (the KL head for the last), and each block's inputs are
+    # the previous block's outputs (full precision and quantized)
+    import oracle
+    d, H, Hkv, dh, f, S, L = 64, 4, 2, 16, 96, 2, 8
+    dims = rq.block_dims(d, H, Hkv, dh, f)
+    blocks = [_weights(d, H, Hkv, dh, f) for _ in range(4)]
+    fishers = [torch.zeros(d, d) for _ in range(4)]
+    gf, Wh = torch.zeros(d), torch.zeros(30, d)
+    x = torch.zeros(S, L, d)
+    calls, fwd = [], []
+
+    def block_exact(dims_, W, x_ref, qcfg, lr, x_hat=None, W_next=None, F_this=None, F_next=None, head_gf=None,
+                    head_Wh=None, **kw):
+        calls.append((W, x_ref, x_hat, lr, W_next, F_this, F_next, head_gf, head_Wh))
+        return {}, {"hat": len(calls)}
+
+    def forward(dims_, weights, xin, y, ws, stream=None):
+        fwd.append((weights, xin, y))
+
+    monkeypatch.setattr(pb, "quantize_block_exact", block_exact)
+    monkeypatch.setattr(pb, "realq_block_forward", forward)
+    monkeypatch.setattr(pb, "workspace", lambda nbytes, device=None: torch.zeros(8, dtype=torch.uint8))
+    out = pb.quantize_model_exact(dims, blocks, x, fishers, gf, Wh, rq.quant_cfg(), 1e-3)
+    assert len(out) == 4 and [o[1]["hat"] for o in out] == [1, 2, 3, 4]
+    for l, c in enumerate(calls):
+        W, x_ref, x_hat, lr, W_next, F_this, F_next, hgf, hWh = c
+        assert W is blocks[l]
+        assert lr == pytest.approx(oracle.reverse_cosine_lr(l + 1, 4, 1e-3), rel=1e-15)
+        if l < 3:
+            assert W_next is blocks[l + 1] and F_this is fishers[l] and F_next is fishers[l + 1] and hWh is None
+        else:
+            assert W_next is None and hgf is gf and hWh is Wh
+        if l == 0:
+            assert x_ref is x and x_hat is x
+        else:
+            # block l-1's two forward passes: reference weights on the
+            # reference input, quantized weights on the quantized input
+            (w_ref, in_ref, y_ref), (w_hat, in_hat, y_hat) = fwd[2 * (l - 1)], fwd[2 * (l - 1) + 1]
+            assert w_ref is blocks[l - 1] and w_hat == {"hat": l}
+            assert in_ref is calls[l - 1][1] and in_hat is calls[l - 1][2]
+            assert x_ref is y_ref and x_hat is y_hat

@@ -571,3 +571,34 @@ def test_sweep_rotation_over_minibatches_is_a_full_batch_step_to_first_order():
     # (the scales are fp32, so an O(lr^2) change of a group's extreme weight
     # can move its scale, and every weight of the group, by one fp32 step)
     assert d_rot <= 1e-6 and d_rot <= 1e-2 * d_first, (d_rot, d_first)
+
+
+def test_model_loop_feeds_each_block_the_quantized_stack_and_its_schedule():
+    # Alg. 1's outer loop: block l+1's perturbed input is the quantized
+    # block l's output on its own perturbed input, its reference input the
+    # full-precision output; the learning rate follows the reverse-cosine
+    # schedule over blocks; the last block takes the KL at the LM head
+    r = np.random.default_rng(36)
+    d, H, Hkv, dh, f, S, L = 32, 4, 2, 8, 48, 2, 12
+    blocks = [ob.block_params(r, d, H, Hkv, dh, f, scale=0.8) for _ in range(3)]
+    fishers = [_spd(r, d) for _ in range(3)]
+    head = ob.head_params(r, d, 13, scale=1.5)
+    x = r.standard_normal((S, L, d))
+    kw = dict(group_size=16, block_size=16, optimizer="sgd")
+    out = ob.quantize_model(x, blocks, fishers, head, lr_final=0.3, **kw)
+    assert len(out) == 3
+    # block 2 by hand: its inputs from blocks 0 and 1 as the loop left them
+    x1 = ob.block_forward(ob.block_forward(x, blocks[0])[0], blocks[1])[0]
+    x1_hat = ob.block_forward(ob.block_forward(x, out[0][1])[0], out[1][1])[0]
+    res, _ = ob.quantize_block(x1, blocks[2], x_hat=x1_hat, head=head, lr=0.3, **kw)
+    for module in ob.MODULES:
+        assert np.array_equal(res[module]["codes"], out[2][0][module]["codes"])
+        np.testing.assert_allclose(res[module]["deq"], out[2][0][module]["deq"], rtol=0, atol=1e-15)
+    # block 0 at the first rate of the schedule (0.01 lr_final), with the
+    # window to block 1
+    res0, _ = ob.quantize_block(x, blocks[0], P_next=blocks[1], F_this=fishers[0], F_next=fishers[1], lr=0.003,
+                                **kw)
+    for module in ob.MODULES:
+        np.testing.assert_allclose(res0[module]["deq"], out[0][0][module]["deq"], rtol=0, atol=1e-15)
+    # the quantized stack's output is off the reference, and block 1 saw it
+    assert not np.allclose(x1, x1_hat)

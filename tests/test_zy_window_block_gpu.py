@@ -461,3 +461,39 @@ def test_block_driver_matches_the_oracle(kl):
         z = out.zero.cpu().numpy()[:, np.arange(n) // 32].astype(np.float32)
         assert np.array_equal((s * (codes.astype(np.float32) - z)).astype(np.float32), out.W.cpu().numpy())
         upstream_exact = upstream_exact and rep["n_mismatch"] == 0
+
+
+def test_model_loop_matches_the_oracle():
+    # Alg. 1's outer loop over three blocks (windows to the next block, the
+    # KL head for the last; reverse-cosine rates), plain gradient steps,
+    # against oracle.block.quantize_model, with the same upstream rule as
+    # the block driver's test over the whole stack
+    from paper_2609_00049_gb300 import block as pb
+    S, L, d, H, Hkv, dh, f = (4, 80, 128, 4, 2, 32, 256)
+    blocks, Ws = [], []
+    for i in range(3):
+        _, P, W, dims, _ = _case(20 + i, S, L, d, H, Hkv, dh, f)
+        blocks.append(P)
+        Ws.append(W)
+    r = np.random.default_rng(23)
+    fishers = [_spd(r, d) for _ in range(3)]
+    head = {k: _f32(v) for k, v in ob.head_params(r, d, 40, scale=1.5).items()}
+    x = _f32(r.standard_normal((S, L, d)))
+    want = ob.quantize_model(x, blocks, fishers, head, lr_final=1.0, optimizer="sgd", group_size=32, block_size=64)
+    got = pb.quantize_model_exact(dims, Ws, _dev(x), [_dev(F) for F in fishers], _dev(head["gf"]),
+                                  _dev(head["Wh"]), rq.quant_cfg(group_size=32, block_size=64), 1.0,
+                                  optimizer=rq.REALQ_OPT_SGD)
+    torch.cuda.synchronize()
+    upstream_exact = True
+    for l in range(3):
+        for module in ob.MODULES:
+            orc, out = want[l][0][module], got[l][0][module]
+            n = orc["codes"].shape[1]
+            codes = unpack(out.codes.cpu().numpy(), n)
+            rep = compare_codes(codes, orc, 64, 32, True)
+            print(f"\nblock {l} {module}: {rep}")
+            if upstream_exact:
+                assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (l, module, rep)
+            else:
+                assert rep["frac_equal"] >= 0.99, (l, module, rep)
+            upstream_exact = upstream_exact and rep["n_mismatch"] == 0
