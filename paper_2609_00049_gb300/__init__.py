@@ -664,6 +664,9 @@ def realq_block_module_inputs(dims: BlockDims, weights: dict, x: torch.Tensor, m
     """The module's calibration inputs (S L x n) in a forward pass of the
     block with `weights` on x (S, L, d); ws as realq_block_forward."""
     S, L, d = x.shape
+    n = {"q_proj": d, "k_proj": d, "v_proj": d, "o_proj": dims.n_heads * dims.head_dim, "gate_proj": d,
+         "up_proj": d, "down_proj": dims.ffn}[module]
+    _need(X_out, torch.float32, (S * L, n), "X_out")
     wp, wb = _ws(ws)
     a = _block_weights(weights)
     _check(lib().realq_block_module_inputs(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
