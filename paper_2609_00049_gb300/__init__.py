@@ -607,14 +607,35 @@ def block_dims(d: int, n_heads: int, n_kv: int, head_dim: int, ffn: int, rms_eps
     return BlockDims(d, n_heads, n_kv, head_dim, ffn, rms_eps, rope_base)
 
 
-def _block_weights(w: dict) -> BlockWeights:
-    out = BlockWeights()
+def _block_shapes(dims: BlockDims) -> dict:
+    d, qw, kw, f = dims.d, dims.n_heads * dims.head_dim, dims.n_kv * dims.head_dim, dims.ffn
+    return {"g1": (d,), "Wq": (qw, d), "Wk": (kw, d), "Wv": (kw, d), "Wo": (d, qw), "g2": (d,), "Wg": (f, d),
+            "Wu": (f, d), "Wd": (d, f)}
+
+
+def _block_weights(w: dict, dims: Optional[BlockDims] = None) -> BlockWeights:
+    """The C struct of a block's weights; with dims, every shape is checked
+    (the library reads them at the sizes dims implies)."""
+    shapes = _block_shapes(dims) if dims is not None else None
     for k in _BLOCK_KEYS:
         t = w[k]
         if t.dtype != torch.float32:
             raise ValueError(f"block weight {k}: expected float32, got {t.dtype}")
-        setattr(out, k, _ptr(t).value)
+        if shapes is not None and tuple(t.shape) != shapes[k]:
+            raise ValueError(f"block weight {k}: expected shape {shapes[k]}, got {tuple(t.shape)}")
+    out = BlockWeights()
+    for k in _BLOCK_KEYS:
+        setattr(out, k, _ptr(w[k]).value)
     return out
+
+
+def _need_tokens(x: Optional[torch.Tensor], dims: BlockDims, name: str, like: Optional[torch.Tensor] = None):
+    if x is None:
+        return
+    if x.dim() != 3 or x.shape[2] != dims.d or x.dtype != torch.float32:
+        raise ValueError(f"{name}: expected float32 (S, L, {dims.d}), got {x.dtype} {tuple(x.shape)}")
+    if like is not None and x.shape != like.shape:
+        raise ValueError(f"{name}: expected shape {tuple(like.shape)}, got {tuple(x.shape)}")
 
 
 def realq_block_workspace_size(dims: BlockDims, S: int, L: int) -> int:
@@ -625,10 +646,11 @@ def realq_block_forward(dims: BlockDims, weights: dict, x: torch.Tensor, y: torc
                         stream=None):
     """y = block(x) for x, y of shape (S, L, d), fp32 (the decoder block of
     the exact sliding window)."""
+    _need_tokens(x, dims, "x")
     S, L, d = x.shape
     _need(y, torch.float32, (S, L, d), "y")
     wp, wb = _ws(ws)
-    w = _block_weights(weights)
+    w = _block_weights(weights, dims)
     _check(lib().realq_block_forward(_stream(stream), ctypes.byref(dims), ctypes.byref(w), S, L, _ptr(x), _ptr(y),
                                      wp, wb))
 
@@ -638,12 +660,13 @@ def realq_block_window(dims: BlockDims, weights: dict, h_ref: torch.Tensor, dh: 
     """The next block's Fisher loss (1/2T) sum_t dz_t^T F_next dz_t with
     dz = B(h_ref + dh) - B(h_ref), into loss (a 1-element fp32 tensor, or
     None), and its gradient in dh into g_h; all (S, L, d) fp32."""
+    _need_tokens(h_ref, dims, "h_ref")
     S, L, d = h_ref.shape
     for t, name in ((dh, "dh"), (g_h, "g_h")):
         _need(t, torch.float32, (S, L, d), name)
     _need(F_next, torch.float32, (d, d), "F_next")
     wp, wb = _ws(ws)
-    w = _block_weights(weights)
+    w = _block_weights(weights, dims)
     _check(lib().realq_block_window(_stream(stream), ctypes.byref(dims), ctypes.byref(w), S, L, _ptr(h_ref), _ptr(dh),
                                     _ptr(F_next), _ptr(g_h), _ptr(loss), wp, wb))
 
@@ -663,18 +686,34 @@ def realq_block_module_inputs(dims: BlockDims, weights: dict, x: torch.Tensor, m
                               ws: torch.Tensor, stream=None):
     """The module's calibration inputs (S L x n) in a forward pass of the
     block with `weights` on x (S, L, d); ws as realq_block_forward."""
+    _need_tokens(x, dims, "x")
     S, L, d = x.shape
     n = {"q_proj": d, "k_proj": d, "v_proj": d, "o_proj": dims.n_heads * dims.head_dim, "gate_proj": d,
          "up_proj": d, "down_proj": dims.ffn}[module]
     _need(X_out, torch.float32, (S * L, n), "X_out")
     wp, wb = _ws(ws)
-    a = _block_weights(weights)
+    a = _block_weights(weights, dims)
     _check(lib().realq_block_module_inputs(_stream(stream), ctypes.byref(dims), ctypes.byref(a), S, L, _ptr(x),
                                            BLOCK_MODULES.index(module), _ptr(X_out), wp, wb))
 
 
-def _opt_weights(w: Optional[dict]):
-    return ctypes.byref(_block_weights(w)) if w is not None else None
+def _opt_weights(w: Optional[dict], dims: Optional[BlockDims] = None):
+    return ctypes.byref(_block_weights(w, dims)) if w is not None else None
+
+
+_MODULE_KEY = {"q_proj": "Wq", "k_proj": "Wk", "v_proj": "Wv", "o_proj": "Wo", "gate_proj": "Wg", "up_proj": "Wu",
+               "down_proj": "Wd"}
+
+
+def _need_module(dims: BlockDims, module: str, x: torch.Tensor, x_hat: Optional[torch.Tensor],
+                 W_module: Optional[torch.Tensor], Fs=()):
+    # the shapes the library reads: tokens (S, L, d), x_hat like x, the
+    # module's weight as dims implies, d x d Fishers
+    _need_tokens(x, dims, "x")
+    _need_tokens(x_hat, dims, "x_hat", like=x)
+    _need(W_module, torch.float32, _block_shapes(dims)[_MODULE_KEY[module]], "W_module")
+    for F, name in Fs:
+        _need(F, torch.float32, (dims.d, dims.d), name)
 
 
 def realq_block_module_window(dims: BlockDims, this_block: dict, next_block: dict, x: torch.Tensor, module: str,
@@ -686,12 +725,14 @@ def realq_block_module_window(dims: BlockDims, this_block: dict, next_block: dic
     loss (or None) and its gradient in W_module into grad (W_module's shape).
     this_block_hat / x_hat: block l's weights and input in the current pass
     (the model quantized so far); None: the reference ones."""
+    _need_module(dims, module, x, x_hat, W_module, ((F_this, "F_this"), (F_next, "F_next")))
     S, L, d = x.shape
     _need(grad, torch.float32, tuple(W_module.shape), "grad")
     wp, wb = _ws(ws)
-    a, b = _block_weights(this_block), _block_weights(next_block)
+    a, b = _block_weights(this_block, dims), _block_weights(next_block, dims)
     _check(lib().realq_block_module_window(_stream(stream), ctypes.byref(dims), ctypes.byref(a),
-                                           _opt_weights(this_block_hat), ctypes.byref(b), S, L, _ptr(x), _ptr(x_hat),
+                                           _opt_weights(this_block_hat, dims), ctypes.byref(b), S, L, _ptr(x),
+                                           _ptr(x_hat),
                                            BLOCK_MODULES.index(module), _ptr(W_module), float(alpha), _ptr(F_this),
                                            _ptr(F_next), _ptr(grad), _ptr(loss), wp, wb))
 
@@ -715,12 +756,15 @@ def realq_block_module_kl(dims: BlockDims, this_block: dict, x: torch.Tensor, mo
                           x_hat: Optional[torch.Tensor] = None, stream=None):
     """The final block's KL for one module's weight, and its gradient
     (this_block_hat / x_hat as for realq_block_module_window)."""
+    _need_module(dims, module, x, x_hat, W_module)
+    _need(Wh, torch.float32, (Wh.shape[0], dims.d), "Wh")
+    _need(gf, torch.float32, (dims.d,), "gf")
     S, L, d = x.shape
     _need(grad, torch.float32, tuple(W_module.shape), "grad")
     wp, wb = _ws(ws)
-    a = _block_weights(this_block)
+    a = _block_weights(this_block, dims)
     _check(lib().realq_block_module_kl(_stream(stream), ctypes.byref(dims), ctypes.byref(a),
-                                       _opt_weights(this_block_hat), S, L, _ptr(x), _ptr(x_hat),
+                                       _opt_weights(this_block_hat, dims), S, L, _ptr(x), _ptr(x_hat),
                                        BLOCK_MODULES.index(module), _ptr(W_module), _ptr(gf), _ptr(Wh), Wh.shape[0],
                                        _ptr(grad), _ptr(loss), wp, wb))
 
@@ -752,6 +796,10 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
     hold that many calibration mini-batches of whole sequences, and each
     Block-GD step takes one in rotation.  Runs blocks [block_begin,
     block_end); returns the optimizer step counter."""
+    _need_module(dims, module, x, x_hat, None, ((F_this, "F_this"), (F_next, "F_next")))
+    if head_Wh is not None:
+        _need(head_Wh, torch.float32, (head_Wh.shape[0], dims.d), "head_Wh")
+        _need(head_gf, torch.float32, (dims.d,), "head_gf")
     S_all, L, d = x.shape
     if n_minibatch < 1 or S_all % n_minibatch:
         raise ValueError(f"{S_all} sequences do not split into {n_minibatch} mini-batches")
@@ -770,11 +818,11 @@ def realq_quantize_layer_window(dims: BlockDims, this_block: dict, next_block: O
     _need(block_loss, torch.float32, (nb, 2), "block_loss")
     t = ctypes.c_int64(adam_t)
     wp, wb = _ws(ws)
-    a = _block_weights(this_block)
-    b = _block_weights(next_block) if next_block is not None else None
+    a = _block_weights(this_block, dims)
+    b = _block_weights(next_block, dims) if next_block is not None else None
     V = int(head_Wh.shape[0]) if head_Wh is not None else 0
     _check(lib().realq_quantize_layer_window(
-        _stream(stream), ctypes.byref(dims), ctypes.byref(a), _opt_weights(this_block_hat),
+        _stream(stream), ctypes.byref(dims), ctypes.byref(a), _opt_weights(this_block_hat, dims),
         ctypes.byref(b) if b is not None else None, S, L, int(n_minibatch), _ptr(x), _ptr(x_hat),
         BLOCK_MODULES.index(module),
         _ptr(F_this), _ptr(F_next), _ptr(head_gf), _ptr(head_Wh), V,

@@ -290,3 +290,33 @@ def test_module_inputs_entry_point_rejects_bad_arguments(L):
     assert mi(X=None) == rq.REALQ_ERR_INVALID_ARG
     assert mi(nbytes=rq.realq_block_workspace_size(ok, 2, 8) - 1) == rq.REALQ_ERR_WORKSPACE
     assert "block_module_inputs" in rq.realq_last_error()
+
+
+def test_block_bindings_check_shapes_before_any_call(L):
+    # the binding checks every shape the library will read against dims
+    # (the C ABI takes plain pointers and cannot)
+    import torch
+    import paper_2609_00049_gb300 as rq
+    d, H, Hkv, dh, f = 64, 4, 2, 16, 96
+    dims = rq.block_dims(d, H, Hkv, dh, f)
+    shapes = {"g1": (d,), "Wq": (H * dh, d), "Wk": (Hkv * dh, d), "Wv": (Hkv * dh, d), "Wo": (d, H * dh),
+              "g2": (d,), "Wg": (f, d), "Wu": (f, d), "Wd": (d, f)}
+    W = {k: torch.zeros(v) for k, v in shapes.items()}
+    x, F = torch.zeros(2, 8, d), torch.zeros(d, d)
+    grad = torch.zeros(d, f)
+    with pytest.raises(ValueError, match="x"):
+        rq.realq_block_module_window(dims, W, W, torch.zeros(2, 8, d + 1), "down_proj", W["Wd"], 0.5, F, F, grad,
+                                     None)
+    with pytest.raises(ValueError, match="x_hat"):
+        rq.realq_block_module_window(dims, W, W, x, "down_proj", W["Wd"], 0.5, F, F, grad, None,
+                                     x_hat=torch.zeros(3, 8, d))
+    with pytest.raises(ValueError, match="W_module"):
+        rq.realq_block_module_window(dims, W, W, x, "down_proj", torch.zeros(f, d), 0.5, F, F, torch.zeros(f, d),
+                                     None)
+    with pytest.raises(ValueError, match="F_next"):
+        rq.realq_block_module_window(dims, W, W, x, "down_proj", W["Wd"], 0.5, F, torch.zeros(d, d + 1), grad, None)
+    bad = dict(W, Wk=torch.zeros(H * dh, d))                     # n_kv heads' worth of rows expected
+    with pytest.raises(ValueError, match="Wk"):
+        rq.realq_block_forward(dims, bad, x, torch.zeros_like(x), None)
+    with pytest.raises(ValueError, match="X_out"):
+        rq.realq_block_module_inputs(dims, W, x, "o_proj", torch.zeros(16, d + 1), None)
