@@ -406,7 +406,7 @@ def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] =
                    F_this: Optional[np.ndarray] = None, F_next: Optional[np.ndarray] = None,
                    head: Optional[Dict] = None, lr: float, steps_per_block: int = 1, optimizer: str = "adam",
                    bits: int = 4, group_size: int = 128, block_size: int = 128, damp_frac: float = 0.01,
-                   modules: Sequence[str] = MODULES):
+                   modules: Sequence[str] = MODULES, follow: Optional[Dict[str, Dict]] = None):
     """Quantize the linear modules of block l one after another (Alg. 1: for
     each linear module, the column sweep with a Block-GD step after every
     column block), each against the exact two-block window (P_next, F_this,
@@ -419,8 +419,10 @@ def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] =
     next module's current pass, OBS Hessian (the second moment of its inputs
     in that pass) and loss see every module quantized before it.  b_global
     runs over the column blocks of all the block's modules, B_total being
-    their sum (Eq. slide_window; Alg. 1's note on b_global).  Returns the
-    sweep result of every module and the final current weights."""
+    their sum (Eq. slide_window; Alg. 1's note on b_global).  follow maps a
+    module to the rounding decisions of another run that its sweep takes at
+    rounding ties (realq_sweep's follow).  Returns the sweep result of every
+    module and the final current weights."""
     x_hat = x if x_hat is None else x_hat
     P_hat = dict(P_this)
     nbs = {}
@@ -442,7 +444,7 @@ def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] =
         bgd = {"lr": lr, "steps_per_block": steps_per_block, "optimizer": optimizer, "b_global_start": b_start,
                "B_total": B_total, "gradient_fn": fn}
         res = _sweep.realq_sweep(P_this[name], H_sum, T, bits=bits, group_size=group_size, block_size=block_size,
-                                 damp_frac=damp_frac, bgd=bgd)
+                                 damp_frac=damp_frac, bgd=bgd, follow=(follow or {}).get(module))
         P_hat[name] = res["deq"]
         out[module] = res
         b_start += nbs[module]
@@ -450,7 +452,7 @@ def quantize_block(x: np.ndarray, P_this: Dict, *, x_hat: Optional[np.ndarray] =
 
 
 def quantize_model(x: np.ndarray, blocks: Sequence[Dict], fishers: Sequence[np.ndarray], head: Dict, *,
-                   lr_final: float, **kw):
+                   lr_final: float, follow: Optional[Sequence[Dict[str, Dict]]] = None, **kw):
     """Alg. 1's outer loop (Stage 1) over a stack of L decoder blocks: block
     l is quantized with quantize_block against the exact two-block window
     with block l+1 (F^(l), F^(l+1) its aggregated Fishers) or, for the last
@@ -458,8 +460,9 @@ def quantize_model(x: np.ndarray, blocks: Sequence[Dict], fishers: Sequence[np.n
     schedule over blocks (eta_l from 0.01 eta_final up to eta_final).  The
     full-precision input of block l+1 is block l's full-precision output; its
     input in the model quantized so far is block l's output with its
-    quantized weights on its own such input.  kw go to quantize_block.
-    Returns each block's module results and its quantized weights."""
+    quantized weights on its own such input.  follow: per block, the
+    quantize_block follow of that block.  kw go to quantize_block.  Returns
+    each block's module results and its quantized weights."""
     L = len(blocks)
     x_ref, x_hat = x, x
     out = []
@@ -468,7 +471,8 @@ def quantize_model(x: np.ndarray, blocks: Sequence[Dict], fishers: Sequence[np.n
         lr = _sweep.reverse_cosine_lr(l + 1, L, lr_final)
         res, P_hat = quantize_block(x_ref, P, x_hat=x_hat, P_next=None if last else blocks[l + 1],
                                     F_this=fishers[l], F_next=None if last else fishers[l + 1],
-                                    head=head if last else None, lr=lr, **kw)
+                                    head=head if last else None, lr=lr,
+                                    follow=None if follow is None else follow[l], **kw)
         out.append((res, P_hat))
         x_ref = block_forward(x_ref, P)[0]
         x_hat = block_forward(x_hat, P_hat)[0]

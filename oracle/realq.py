@@ -31,16 +31,19 @@ the Schur-complement downdate named in the theorem's proof.
 from __future__ import annotations
 
 import math
+from fractions import Fraction
 from typing import Iterable, Optional
 
 import numpy as np
+
+from . import native
 
 __all__ = [
     "hessian_sum", "cross_moment_sum", "prepare", "inverse_upper_cholesky",
     "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
     "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
     "round_bf16", "quantize_activations", "saliency_clip", "weighted_hessian_sum",
-    "loss_clip_factors", "gradient_tokens", "surrogate_tokens_clipped",
+    "loss_clip_factors", "gradient_tokens", "surrogate_tokens_clipped", "nearest_rank",
 ]
 
 
@@ -109,8 +112,8 @@ def inverse_upper_cholesky(Hd: np.ndarray) -> np.ndarray:
 # variant: xmax = max(|xmin|, xmax), xmin = -xmax, zero = 2^(b-1).  Rounding is
 # round-half-to-even.  Decisions in fp32 (module docstring).
 # ---------------------------------------------------------------------------
-def quant_params(w_rows: np.ndarray, bits: int = 4, symmetric: bool = False):
-    """Per-row (scale fp32, zero int) for a group of columns w_rows (m x g)."""
+def _grid(w_rows: np.ndarray, bits: int, symmetric: bool):
+    """quant(.)'s per-row grid of a group: (scale fp32, zero int, zero margin, zero before rounding)."""
     w = np.asarray(w_rows, dtype=np.float64).astype(np.float32)
     maxq = np.float32(2 ** bits - 1)
     xmin = np.minimum(w.min(axis=1), np.float32(0.0))
@@ -125,11 +128,34 @@ def quant_params(w_rows: np.ndarray, bits: int = 4, symmetric: bool = False):
     if symmetric:
         zero = np.full(w.shape[0], 2 ** (bits - 1), dtype=np.int64)
         zmargin = np.full(w.shape[0], 0.5)
+        zf = zero.astype(np.float64)
     else:
         zf = (-xmin / scale).astype(np.float32)
         zero = np.rint(zf).astype(np.int64)
-        zmargin = np.abs(np.abs(zf.astype(np.float64) - np.floor(zf)) - 0.5)
+        zf = zf.astype(np.float64)
+        zmargin = np.abs(np.abs(zf - np.floor(zf)) - 0.5)
+    return scale, zero, zmargin, zf
+
+
+def quant_params(w_rows: np.ndarray, bits: int = 4, symmetric: bool = False):
+    """Per-row (scale fp32, zero int) for a group of columns w_rows (m x g)."""
+    scale, zero, zmargin, _ = _grid(w_rows, bits, symmetric)
     return scale, zero, zmargin
+
+
+def _round(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int):
+    """(q, w/scale in fp32 as fp64, margin) of quant(.) on one column."""
+    maxq = 2 ** bits - 1
+    x = (np.asarray(w, dtype=np.float64).astype(np.float32) / scale.astype(np.float32)).astype(np.float32)
+    r = np.rint(x)
+    q = np.clip(r.astype(np.int64) + zero, 0, maxq)
+    x64 = x.astype(np.float64)
+    margin = np.abs(np.abs(x64 - np.floor(x64)) - 0.5)
+    return q, x64, margin
+
+
+def _dequant(q: np.ndarray, scale: np.ndarray, zero: np.ndarray) -> np.ndarray:
+    return (scale.astype(np.float32) * (q.astype(np.float32) - zero.astype(np.float32))).astype(np.float32)
 
 
 def quantize(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int = 4):
@@ -138,14 +164,21 @@ def quantize(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int = 4):
     Returns (q int64, deq as fp64 of the fp32 value, margin) where margin is the
     distance of w/scale from the nearest rounding boundary, in grid steps.
     """
-    maxq = 2 ** bits - 1
-    x = (np.asarray(w, dtype=np.float64).astype(np.float32) / scale.astype(np.float32)).astype(np.float32)
-    r = np.rint(x)
-    q = np.clip(r.astype(np.int64) + zero, 0, maxq)
-    deq = (scale.astype(np.float32) * (q.astype(np.float32) - zero.astype(np.float32))).astype(np.float32)
-    x64 = x.astype(np.float64)
-    margin = np.abs(np.abs(x64 - np.floor(x64)) - 0.5)
-    return q, deq.astype(np.float64), margin
+    q, _, margin = _round(w, scale, zero, bits)
+    return q, _dequant(q, scale, zero).astype(np.float64), margin
+
+
+def _follow_tie(mine: np.ndarray, value: np.ndarray, margin: np.ndarray, other: np.ndarray, tau: float,
+                offset, lo: int, hi: int):
+    """Where this run's rounding of `value` is a tie (margin < tau) and another
+    run of the sweep took the other neighbour, take that one.  The two
+    neighbours are clamp(floor(value) + offset) and clamp(ceil(value) +
+    offset).  Returns (decisions, mask of those taken from `other`)."""
+    other = np.asarray(other, dtype=np.int64)
+    down = np.clip(np.floor(value).astype(np.int64) + offset, lo, hi)
+    up = np.clip(np.ceil(value).astype(np.int64) + offset, lo, hi)
+    take = (margin < tau) & (other != mine) & ((other == down) | (other == up))
+    return np.where(take, other, mine), take
 
 
 def rtn(W: np.ndarray, bits: int = 4, group_size: int = 128, symmetric: bool = False):
@@ -245,6 +278,21 @@ def gradient(What, W0, Hbar, Dbar, F) -> np.ndarray:
 
 
 # ---------------------------------------------------------------------------
+# Nearest-rank percentile, the rule of both clipping steps of the paper (App.
+# "Hessian-side saliency clipping": the 99th percentile of the per-token
+# saliency; App. "Activation clipping (a_loss_clip)": the 95th percentile of
+# the output perturbation).  Reading: the pct-percentile of `count` values is
+# the smallest of them with at least pct * count values at or below it, i.e.
+# the ceil(pct * count)-th smallest.  pct is the number as written (0.99 is
+# 99/100) and the product is exact, so 0.99 of 8000 values is the 7920th.
+# ---------------------------------------------------------------------------
+def nearest_rank(pct: float, count: int) -> int:
+    """0-based position of the nearest-rank pct-percentile in `count` sorted values."""
+    r = math.ceil(Fraction(repr(float(pct))) * count)
+    return min(max(r - 1, 0), count - 1)
+
+
+# ---------------------------------------------------------------------------
 # Output-perturbation clipping of the Block-GD loss (App. "Activation
 # clipping (a_loss_clip) for small Qwen3 models": a_loss_clip = 0.95 on
 # Qwen3-0.6B, 1.7B and 4B).  Per token, the output channels whose |Δy| lies
@@ -253,7 +301,7 @@ def gradient(What, W0, Hbar, Dbar, F) -> np.ndarray:
 # stays non-zero.
 # Readings: the percentile is taken per token over its m output channels, as
 # the nearest-rank one of the saliency clip (the ceil(pct m)-th smallest
-# |Δy_t,i|, pct as a single-precision value); a channel above it is scaled by
+# |Δy_t,i|, see nearest_rank); a channel above it is scaled by
 # kappa = q_t / |Δy_t,i| (its scaled residual has magnitude q_t), every other
 # channel by 1; kappa is a constant of the step (detached), so with
 # L = (1/2T) sum_t (kappa_t ⊙ Δy_t)^T F (kappa_t ⊙ Δy_t)
@@ -267,8 +315,7 @@ def loss_clip_factors(dY: np.ndarray, pct: float):
     """kappa (T x m) and the per-token thresholds q (T) for residuals dY (T x m)."""
     dY = np.asarray(dY, dtype=np.float64)
     m = dY.shape[1]
-    p32 = float(np.float32(pct))
-    k = min(max(int(math.ceil(p32 * m)) - 1, 0), m - 1)
+    k = nearest_rank(pct, m)
     a = np.abs(dY)
     q = np.sort(a, axis=1)[:, k]
     kappa = np.ones_like(a)
@@ -311,7 +358,8 @@ def pack_codes(codes: np.ndarray) -> np.ndarray:
 # The sweep: Algorithm 1, inner loops for one linear module.
 # ---------------------------------------------------------------------------
 def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetric=False,
-                damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True, obs_hessians=None):
+                damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True, obs_hessians=None,
+                follow=None, columns=None):
     """Quantize W0 column by column with OBS feedback and Block-GD after each block.
 
     bgd: None for the plain column sweep (GPTQ), else a dict with keys
@@ -355,6 +403,20 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     g's OBS step and lazy update use H̄_g = H_g_sum / norm_g (damped and with
     its own dead channels, as in prepare), while Block-GD keeps the
     surrogate's plain H̄ = H_sum / T.
+
+    follow: None, or the rounding decisions of another run of the same sweep
+    as a dict with "codes" (m x n ints), optionally "zero" (m x ngroups ints)
+    and "tau" (grid steps, default 1e-3).  quant(.) rounds to the nearest
+    grid point, and where w / scale (or -xmin / scale for the zero point)
+    lies within tau of a rounding boundary both neighbours are the correctly
+    rounded result up to the rounding of the operands (reading C3 of the
+    rounding that Sec. 3.2's quant(.) leaves open).  At every such tie where
+    the other run took the other neighbour, this run takes it too and
+    carries it forward through the compensation and Block-GD; every other
+    decision is this sweep's own.  n_followed counts the decisions taken.
+
+    columns: None for the whole sweep, or stop after that many columns (a
+    bounded sample of the work, for timing).
     """
     W0 = np.asarray(W0, dtype=np.float64)
     m, n = W0.shape
@@ -393,12 +455,23 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     Fm = None if F is None else np.asarray(F, dtype=np.float64)
     Fn = None if F_next is None else np.asarray(F_next, dtype=np.float64)
 
-    for j in range(n):
+    maxq = 2 ** bits - 1
+    tau = 1e-3 if follow is None else follow.get("tau", 1e-3)
+    n_followed = n_followed_zero = 0
+    for j in range(n if columns is None else min(int(columns), n)):
         if j % g == 0:
             gi = j // g
-            scale[:, gi], zero[:, gi], zmargin[:, gi] = quant_params(W[:, j:j + g], bits, symmetric)
+            scale[:, gi], zero[:, gi], zmargin[:, gi], zf = _grid(W[:, j:j + g], bits, symmetric)
+            if follow is not None and follow.get("zero") is not None and not symmetric:
+                zero[:, gi], took = _follow_tie(zero[:, gi], zf, zmargin[:, gi], follow["zero"][:, gi], tau, 0,
+                                                0, maxq)
+                n_followed_zero += int(took.sum())
         gi = j // g
-        q, dq, mg = quantize(W[:, j], scale[:, gi], zero[:, gi], bits)
+        q, x, mg = _round(W[:, j], scale[:, gi], zero[:, gi], bits)
+        if follow is not None:
+            q, took = _follow_tie(q, x, mg, follow["codes"][:, j], tau, zero[:, gi], 0, maxq)
+            n_followed += int(took.sum())
+        dq = _dequant(q, scale[:, gi], zero[:, gi]).astype(np.float64)
         e = W[:, j] - dq                       # residual delta_j of Eq. (gptq_update)
         codes[:, j] = q
         margin[:, j] = mg
@@ -407,9 +480,9 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             d = Hinv[j, j]
             hinv_diag[k, j] = d
             # Eq. (gptq_update): W[:, j+1:] -= delta_j H^-1[j, j+1:] / [H^-1]_jj
-            W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])
+            native.outer_sub(W[rows, j + 1:], e[rows] / d, Hinv[j, j + 1:])
             # remove j from the free set: Schur-complement downdate of H^-1
-            Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d
+            native.outer_sub(Hinv[j + 1:, j + 1:], Hinv[j + 1:, j], Hinv[j, j + 1:], d)
         W[:, j] = dq
 
         be = j + 1
@@ -460,6 +533,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         "margin": margin, "zero_margin": zmargin, "eps": eps_cols,
         "hinv_diag": hinv_diag[0] if obs_hessians is None else hinv_diag,
         "block_loss": block_loss, "adam_t": 0 if opt is None else opt.t,
+        "n_followed": n_followed, "n_followed_zero": n_followed_zero,
         "Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": prep["lam"], "Dbar": Dbar,
     }
 
@@ -509,18 +583,16 @@ def quantize_activations(X: np.ndarray, bits: int = 4, a_clip: float = 0.9, out_
 # clipping": per-token saliency clipped to the 99th percentile first).
 # Readings: the rows of W form N_g contiguous groups, s[t, g] >= 0 is token
 # t's saliency for group g; the percentile is the nearest-rank one (the
-# smallest saliency value with at least pct of the tokens at or below it,
-# pct as a single-precision value), taken per group over the T tokens; H̄_g = H_g / sum_t s'[t, g] (the
+# smallest saliency value with at least pct of the tokens at or below it, see
+# nearest_rank), taken per group over the T tokens; H̄_g = H_g / sum_t s'[t, g] (the
 # saliency-weighted mean of x x^T; the OBS step does not depend on the scale).
 # ---------------------------------------------------------------------------
 def saliency_clip(S: np.ndarray, pct: float = 0.99):
-    """Returns (S clipped, per-group thresholds).  pct is the single-precision
-    value the interface carries (0.99 -> 0.99000000953...); the rank
-    ceil(pct T) - 1 is evaluated exactly from it."""
+    """Returns (S clipped, per-group thresholds): the threshold of group g is
+    the ceil(pct T)-th smallest saliency of its column (nearest_rank)."""
     S = np.asarray(S, dtype=np.float64)
     T = S.shape[0]
-    p32 = float(np.float32(pct))
-    k = min(max(int(math.ceil(p32 * T)) - 1, 0), T - 1)
+    k = nearest_rank(pct, T)
     c = np.sort(S, axis=0)[k]
     return np.minimum(S, c[None, :]), c
 

@@ -15,13 +15,13 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 MUTATIONS = {
     # OBS compensation of Eq. (gptq_update): its sign, its columns shifted by one
-    "compensation_sign": ("W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])",
-                          "W[rows, j + 1:] += np.outer(e[rows] / d, Hinv[j, j + 1:])"),
-    "compensation_shift": ("W[rows, j + 1:] -= np.outer(e[rows] / d, Hinv[j, j + 1:])",
-                           "W[rows, j + 1:] -= np.outer(e[rows] / d, np.roll(Hinv[j, j + 1:], 1))"),
+    "compensation_sign": ("native.outer_sub(W[rows, j + 1:], e[rows] / d, Hinv[j, j + 1:])",
+                          "native.outer_sub(W[rows, j + 1:], -e[rows] / d, Hinv[j, j + 1:])"),
+    "compensation_shift": ("native.outer_sub(W[rows, j + 1:], e[rows] / d, Hinv[j, j + 1:])",
+                           "native.outer_sub(W[rows, j + 1:], e[rows] / d, np.roll(Hinv[j, j + 1:], 1))"),
     # the Schur-complement downdate dropped
-    "no_downdate": ("Hinv[j + 1:, j + 1:] -= np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d",
-                    "Hinv[j + 1:, j + 1:] -= 0.0 * np.outer(Hinv[j + 1:, j], Hinv[j, j + 1:]) / d"),
+    "no_downdate": ("native.outer_sub(Hinv[j + 1:, j + 1:], Hinv[j + 1:, j], Hinv[j, j + 1:], d)",
+                    "native.outer_sub(Hinv[j + 1:, j + 1:], 0.0 * Hinv[j + 1:, j], Hinv[j, j + 1:], d)"),
     # the residual of the quantizer halved
     "residual": ("e = W[:, j] - dq ", "e = W[:, j] - 0.5 * dq "),
     # the cross-moment term transposed
@@ -38,17 +38,19 @@ MUTATIONS = {
     "alpha_index": ("return 1.0 - (b_global - 1) / (B_total - 1)", "return 1.0 - b_global / (B_total - 1)"),
     # the output clipping: rank off by one, the factor inverted, a missing
     # factor in the gradient
-    "clip_rank": ("k = min(max(int(math.ceil(p32 * m)) - 1, 0), m - 1)",
-                  "k = min(max(int(math.ceil(p32 * m)), 0), m - 1)"),
     "clip_factor": ("kappa[over] = (q[:, None] / np.where(over, a, 1.0))[over]",
                     "kappa[over] = (np.where(over, a, 1.0) / q[:, None])[over]"),
     "clip_gradient": ("return (kappa * Z).T @ Xh / float(Xh.shape[0])", "return Z.T @ Xh / float(Xh.shape[0])"),
     # the mini-batch moment not normalised by its own token count
     "minibatch_norm": ("Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)",
                        "Hstep = np.asarray(Hk, dtype=np.float64) / float(T)"),
-    # the saliency percentile rank off by one
-    "saliency_rank": ("k = min(max(int(math.ceil(p32 * T)) - 1, 0), T - 1)",
-                      "k = min(max(int(math.ceil(p32 * T)), 0), T - 1)"),
+    # the nearest-rank percentile of both clipping steps off by one, or
+    # taken from the single-precision value of pct
+    "percentile_rank": ("return min(max(r - 1, 0), count - 1)", "return min(max(r, 0), count - 1)"),
+    "percentile_single": ("r = math.ceil(Fraction(repr(float(pct))) * count)",
+                          "r = math.ceil(Fraction(float(np.float32(pct))) * count)"),
+    # the tie following of another run's rounding: taken off the ties too
+    "follow_off_ties": ("take = (margin < tau) & (other != mine)", "take = (other != mine)"),
     # the weighted Hessian without the weights
     "weighted_hessian": ("H[g] += (c * sc[:, g:g + 1]).T @ c", "H[g] += c.T @ c"),
     # the activation grid without its clipping ratio

@@ -5,6 +5,7 @@ form, a brute-force search, a special case that reduces to a textbook routine,
 an independent route to the same quantity, or a library implementation.
 """
 import math
+from fractions import Fraction
 
 import numpy as np
 import pytest
@@ -333,6 +334,99 @@ def test_sweep_output_invariants():
 
 
 # ---------------------------------------------------------------------------
+# The rank-one updates in C are numpy's outer-product updates, bit for bit.
+# ---------------------------------------------------------------------------
+def test_native_rank_one_updates_are_numpys():
+    from oracle import native
+    r = np.random.default_rng(7)
+    A = r.standard_normal((70, 90))
+    for d in (None, 0.37):
+        B, C = A.copy(), A.copy()
+        u, v = B[5:, 3], B[2, 11:]            # a strided column and a row, outside the updated block
+        native.outer_sub(B[5:, 11:], u, v, d)
+        if d is None:
+            C[5:, 11:] -= np.outer(C[5:, 3], C[2, 11:])
+        else:
+            C[5:, 11:] -= np.outer(C[5:, 3], C[2, 11:]) / d
+        assert np.array_equal(B, C)
+        assert not np.array_equal(B, A)
+
+
+# ---------------------------------------------------------------------------
+# Following another run's decisions at rounding ties (reading C3).  With
+# H = I there is no compensation and the sweep is round-to-nearest (P1).  Row
+# 0's group spans [-7, 8]: scale 1 and zero point 7 exactly, so w = 2.5 is an
+# exact tie (rint gives 2, code 9; the other neighbour is code 10).  Row 1's
+# spans [-7.5, 7.5]: scale 1 and -xmin/scale = 7.5, a zero-point tie (rint
+# gives 8; the other neighbour is 7).
+# ---------------------------------------------------------------------------
+def _tie_case():
+    r = np.random.default_rng(8)
+    W0 = r.uniform(-3.0, 3.0, (4, 8))
+    W0[0, :3] = (-7.0, 8.0, 2.5)
+    W0[1, :2] = (-7.5, 7.5)
+    T = 10
+    return W0, T * np.eye(8), T
+
+
+def test_following_own_decisions_changes_nothing():
+    W0, H, T = _tie_case()
+    a = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8)
+    assert a["codes"][0, 2] == 9 and a["zero"][0, 0] == 7 and a["zero"][1, 0] == 8
+    assert a["margin"][0, 2] == 0.0 and a["zero_margin"][1, 0] == 0.0
+    b = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": a["codes"], "zero": a["zero"]})
+    assert b["n_followed"] == 0 and b["n_followed_zero"] == 0
+    for k in ("codes", "zero", "scale", "deq"):
+        assert np.array_equal(a[k], b[k]), k
+
+
+def test_following_takes_the_other_neighbour_only_at_ties():
+    W0, H, T = _tie_case()
+    a = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8)
+    # the other neighbour at the code tie and at the zero-point tie: taken
+    other = a["codes"].copy()
+    other[0, 2] = 10
+    zo = a["zero"].copy()
+    zo[1, 0] = 7
+    b = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": other, "zero": zo})
+    assert b["n_followed"] == 1 and b["n_followed_zero"] == 1
+    assert b["codes"][0, 2] == 10 and b["deq"][0, 2] == 3.0
+    assert b["zero"][1, 0] == 7
+    assert np.array_equal(b["deq"][1], b["scale"][1, 0] * (b["codes"][1] - 7.0))
+    assert np.array_equal(b["codes"][2:], a["codes"][2:])
+    # a code two levels away at the tie is not a rounding of w: ignored
+    other[0, 2] = 11
+    c = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": other})
+    assert c["n_followed"] == 0 and c["codes"][0, 2] == 9
+    # every code moved up by one: only decisions at a tie follow
+    up = np.minimum(a["codes"] + 1, 15)
+    d = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": up})
+    changed = d["codes"] != a["codes"]
+    assert changed[0, 2] and np.all(a["margin"][changed] < 1e-3)
+    assert d["n_followed"] == int(changed.sum())
+
+
+def test_following_a_decision_changes_only_its_row_from_there_on():
+    # compensation on (a correlated H), no Block-GD: rows are independent, so
+    # a decision taken from the other run (a wide tau makes every decision
+    # eligible) leaves every other row and the row's earlier columns alone
+    W0, X = _correlated_case(9, 6, 40, 200)
+    H, T = oracle.hessian_sum([X])
+    a = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8)
+    i0, j0 = 3, 17
+    other = a["codes"].copy()                   # a code next to the oracle's at (i0, j0)
+    other[i0, j0] = a["codes"][i0, j0] + (1 if a["codes"][i0, j0] < 15 else -1)
+    b = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": other, "tau": 0.5})
+    # (later decisions of row i0, taken from the changed state, may follow
+    # the other run back to its codes: those count too)
+    assert b["codes"][i0, j0] == other[i0, j0] and b["n_followed"] >= 1
+    keep = np.ones_like(a["codes"], dtype=bool)
+    keep[i0, j0:] = False
+    assert np.array_equal(a["codes"][keep], b["codes"][keep])
+    assert not np.array_equal(a["deq"][i0, j0:], b["deq"][i0, j0:])
+
+
+# ---------------------------------------------------------------------------
 # Brute force over all int4 codes of a 4 x 8 layer (diagonal Fisher: rows
 # decouple).  The surrogate evaluator agrees with the independent C evaluator;
 # no code vector beats the global minimum; the sweep does not lose to RTN; with
@@ -490,18 +584,21 @@ def test_saliency_clip_is_the_nearest_rank_percentile():
     S = np.exp(3.0 * r.standard_normal((1000, 4)))
     S[r.integers(0, 1000, 50), 1] = 7.0                 # ties
     S[5, 2] = 1e15                                       # an extreme outlier
-    for pct in (0.99, 0.5, 1.0, 1e-9):
+    for pct in (0.99, 0.5, 1.0, 1e-9, 0.973):
         Sc, c = oracle.saliency_clip(S, pct)
-        p32 = float(np.float32(pct))
+        frac = Fraction(repr(pct))
         for g in range(4):
             v = S[:, g]
-            cand = [x for x in np.unique(v) if (v <= x).sum() >= p32 * len(v)]
+            # brute-force counting with the exact product pct * T
+            cand = [x for x in np.unique(v) if (v <= x).sum() >= frac * len(v)]
             assert c[g] == min(cand)
             assert np.array_equal(Sc[:, g], np.minimum(v, c[g]))
     Sc, c = oracle.saliency_clip(S, 0.99)
     assert c[2] < 1e15 and Sc[5, 2] == c[2]
-    # the rank comes from the single-precision pct: 0.99f * 8000 = 7920.00008
-    assert oracle.saliency_clip(np.arange(8000.0)[:, None], 0.99)[1][0] == 7920.0
+    # the 99th percentile of 8000 values is the 7920th smallest (0.99 * 8000 is
+    # exactly 7920, so its ceiling is 7920 and not 7921)
+    assert oracle.saliency_clip(np.arange(8000.0)[:, None], 0.99)[1][0] == 7919.0
+    assert oracle.saliency_clip(np.arange(8001.0)[:, None], 0.99)[1][0] == 7920.0   # 7920.99 -> 7921st
 
 
 def test_saliency_clipping_prevents_rank_one_collapse():
@@ -560,8 +657,8 @@ def test_minibatch_rotation_rule():
 def test_loss_clip_worked_example():
     # one token with residuals 1..20 (shuffled, signs alternating): the 95th
     # nearest-rank percentile of 20 channels is the 19th smallest |Δy| = 19
-    # (float32(0.95) = 0.949999988, times 20 = 18.99999976, rank 19), so only
-    # the channel with |Δy| = 20 is scaled, by 19/20
+    # (0.95 * 20 = 19 exactly), so only the channel with |Δy| = 20 is
+    # scaled, by 19/20
     perm = np.random.default_rng(5).permutation(20)
     dY = (np.arange(1, 21, dtype=np.float64) * np.where(np.arange(20) % 2, -1.0, 1.0))[perm][None, :]
     kappa, q = oracle.loss_clip_factors(dY, 0.95)
@@ -569,14 +666,17 @@ def test_loss_clip_worked_example():
     expect = np.ones(20)
     expect[np.abs(dY[0]) == 20.0] = 19.0 / 20.0
     assert np.array_equal(kappa[0], expect)
-    # 0.99 of 100 channels: float32(0.99) = 0.99000001, times 100 =
-    # 99.0000009, rank 100: the threshold is the maximum and nothing is scaled;
-    # 0.98 of 100: float32(0.98) = 0.98000002, times 100 = 98.0000019, rank 99
+    # 0.99 of 100 channels: rank 99 exactly, so the threshold is 99 and the
+    # largest channel is scaled by 99/100; 0.98 of 100: rank 98, threshold
+    # 98, the two largest scaled; 0.995 of 100: 99.5 -> rank 100, nothing
     dY = np.arange(1, 101, dtype=np.float64)[None, :]
     kappa, q = oracle.loss_clip_factors(dY, 0.99)
-    assert q[0] == 100.0 and np.all(kappa == 1.0)
-    kappa, q = oracle.loss_clip_factors(dY, 0.98)
     assert q[0] == 99.0 and np.all(kappa[0, :99] == 1.0) and kappa[0, 99] == 99.0 / 100.0
+    kappa, q = oracle.loss_clip_factors(dY, 0.98)
+    assert q[0] == 98.0 and np.all(kappa[0, :98] == 1.0)
+    assert kappa[0, 98] == 98.0 / 99.0 and kappa[0, 99] == 98.0 / 100.0
+    kappa, q = oracle.loss_clip_factors(dY, 0.995)
+    assert q[0] == 100.0 and np.all(kappa == 1.0)
 
 
 def test_loss_clip_invariants():
@@ -585,7 +685,7 @@ def test_loss_clip_invariants():
     r = np.random.default_rng(6)
     dY = r.standard_t(3, size=(50, 64)) * np.exp(r.standard_normal((50, 1)))
     kappa, q = oracle.loss_clip_factors(dY, 0.95)
-    k = math.ceil(float(np.float32(0.95)) * 64)
+    k = math.ceil(Fraction(95, 100) * 64)
     Y = np.abs(kappa * dY)
     assert np.all(Y <= q[:, None] * (1 + 1e-15))
     np.testing.assert_allclose(Y.max(axis=1), q, rtol=1e-15)
