@@ -177,9 +177,10 @@ realq_status_t realq_prepare_status(realq_stream_t stream, void *ws, size_t ws_b
  * (about 8.4 MB, held by every GPU that loads the library until the process
  * exits).  Larger n returns REALQ_ERR_INVALID_ARG before any work is queued.
  * The call allocates nothing (no cudaMalloc / cudaFree, no allocating library
- * routine).  The first call on a device, with that device current, looks up
- * the array's device address once; make that first call before any stream
- * capture.  All calls share the one array, which keeps the last call's
+ * routine).  Every call looks up the array's device address on the current
+ * device; the first call on a device may load the library's device code
+ * there, so make that first call before any stream capture.  All calls
+ * share the one array, which keeps the last call's
  * contents (the status word is cleared at the start of each call, the rest is
  * overwritten before it is read), so calls that overlap on the GPU race: do
  * not run two of them concurrently on one device. */
@@ -194,8 +195,10 @@ realq_status_t realq_hessian_prepare_noalloc(realq_stream_t stream, int64_t n, i
  * The same sweep as realq_quantize_layer_minibatch, but each optimizer step
  * takes its gradient from the mini-batch's tokens:
  *   Δ_t = (Ŵ - W0) x̂_t                       (m, per token of the mini-batch)
- *   q_t = the ceil(a_loss_clip m)-th smallest |Δ_t,i| (a_loss_clip as given,
- *         single precision; the product is taken exactly)
+ *   q_t = the ceil(a_loss_clip m)-th smallest |Δ_t,i| (a_loss_clip in
+ *         double precision, the product and its ceiling in double: for a
+ *         percentile written with a few decimals, 0.95 or 0.99, that is the
+ *         exact rank, e.g. 0.99 of 8000 values is the 7920th)
  *   kappa_t,i = q_t / |Δ_t,i| if |Δ_t,i| > q_t, else 1   (held constant)
  *   G = (1/T_k) sum_t (kappa_t ⊙ F_eff (kappa_t ⊙ Δ_t)) x̂_tᵀ, free columns
  * and one optimizer step per G.  Mini-batch k holds tokens
@@ -216,7 +219,7 @@ size_t realq_quantize_tokens_workspace_size(int64_t m, int64_t n, int64_t T_mb, 
 realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
                                            realq_dtype_t w_dtype, const float *U, const float *Hbar,
                                            const uint8_t *dead, const void *X_hat, int64_t T, int64_t T_mb,
-                                           float a_loss_clip, const realq_quant_cfg_t *qcfg,
+                                           double a_loss_clip, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
                                            float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
                                            int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
@@ -251,10 +254,13 @@ realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int6
  * realq_saliency_clip: S is T x n_groups fp32 (row-major: S[t * n_groups + g]
  * is token t's saliency for row group g, >= 0 and finite).  clip_out[g] is the
  * nearest-rank pct-percentile of column g over the T tokens (the smallest
- * value with at least pct * T values at or below it: an input value, bit for
- * bit); S_out = min(S, clip_out[g]) elementwise (may alias S, may be NULL to
- * get the thresholds only).  0 < pct <= 1.  Asynchronous; allocates nothing. */
-realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *S, float pct,
+ * value with at least pct * T values at or below it, i.e. the ceil(pct T)-th
+ * smallest: an input value, bit for bit); S_out = min(S, clip_out[g])
+ * elementwise (may alias S, may be NULL to get the thresholds only).
+ * 0 < pct <= 1, in double precision, the rank ceil(pct T) taken in double
+ * (exact for a percentile written with a few decimals: 0.99 of 8000 tokens
+ * is the 7920th smallest).  Asynchronous; allocates nothing. */
+realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *S, double pct,
                                    float *S_out, float *clip_out);
 
 /* H_g += sum_t S[t, g] x̂_t x̂_t^T for every group g (H_g: n_groups x n x n

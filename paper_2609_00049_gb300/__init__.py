@@ -89,6 +89,7 @@ def bgd_cfg(lr, steps_per_block=1, optimizer=REALQ_OPT_ADAM, beta1=0.9, beta2=0.
 
 _lib = None
 _vp, _i64, _sz, _int, _f32 = ctypes.c_void_p, ctypes.c_int64, ctypes.c_size_t, ctypes.c_int, ctypes.c_float
+_f64 = ctypes.c_double
 _P_i64 = ctypes.POINTER(ctypes.c_int64)
 _SIGS = {
     "realq_hessian_accumulate": ([_vp, _i64, _i64, _vp, _vp, _int, _vp, _vp, _vp, _sz], _int),
@@ -105,7 +106,7 @@ _SIGS = {
     "realq_graph_destroy": ([_vp], None),
     "realq_scale_moment": ([_vp, _i64, _i64, _vp, _vp], _int),
     "realq_quantize_activations": ([_vp, _i64, _i64, _vp, _int, _int, _f32, _vp, _vp, _vp], _int),
-    "realq_saliency_clip": ([_vp, _i64, _int, _vp, _f32, _vp, _vp], _int),
+    "realq_saliency_clip": ([_vp, _i64, _int, _vp, _f64, _vp, _vp], _int),
     "realq_hessian_weighted_workspace_size": ([_i64, _i64], _sz),
     "realq_hessian_accumulate_weighted": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _sz], _int),
     "realq_hessian_prepare_scaled": ([_vp, _i64, ctypes.c_double, _f32, _vp, _vp, _vp, _vp, _P_i64, _vp, _sz], _int),
@@ -122,7 +123,7 @@ _SIGS = {
     "realq_quantize_trace_workspace_size": ([_i64, _i64], _sz),
     "realq_quantize_tokens_workspace_size": ([_i64, _i64, _i64, ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg),
                                               _int], _sz),
-    "realq_quantize_layer_tokens": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64, _i64, _f32,
+    "realq_quantize_layer_tokens": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _vp, _i64, _i64, _f64,
                                      ctypes.POINTER(QuantCfg), ctypes.POINTER(BgdCfg), _vp, _vp, _vp, _vp, _vp, _vp,
                                      _P_i64, _vp, _vp, _vp, _vp, _int, _i64, _i64, _vp, _sz], _int),
     "realq_quantize_layer_minibatch": ([_vp, _i64, _i64, _vp, _int, _vp, _vp, _vp, _int, _vp,

@@ -353,10 +353,10 @@ realq_status_t realq_quantize_activations(realq_stream_t stream, int64_t T, int6
     return act_quant(S(stream), T, n, X, x_dtype, bits, a_clip, X_q, codes, scale);
 }
 
-realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *sal, float pct,
+realq_status_t realq_saliency_clip(realq_stream_t stream, int64_t T, int n_groups, const float *sal, double pct,
                                    float *sal_out, float *clip_out) {
     if (T <= 0 || n_groups <= 0 || !sal || !clip_out) return fail(REALQ_ERR_INVALID_ARG, "saliency_clip: bad argument");
-    if (!(pct > 0.f && pct <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "saliency_clip: 0 < pct <= 1");
+    if (!(pct > 0.0 && pct <= 1.0)) return fail(REALQ_ERR_INVALID_ARG, "saliency_clip: 0 < pct <= 1");
     return saliency_clip(S(stream), T, n_groups, sal, pct, sal_out, clip_out);
 }
 
@@ -409,7 +409,7 @@ size_t realq_quantize_workspace_size(int64_t m, int64_t n, const realq_quant_cfg
 struct TokArgs {
     const void *X;       // T x n bf16
     int64_t T, tmb;      // tokens, tokens per mini-batch
-    float clip;          // per-token output clipping percentile, (0, 1]
+    double clip;         // per-token output clipping percentile, (0, 1]
 };
 
 // Per-block surrogate values (nullptr: not traced).
@@ -493,9 +493,9 @@ static realq_status_t quantize_impl(realq_stream_t stream, int64_t m, int64_t n,
     if (tmb > 0) {
         p.Xtok = tok->X; p.Ttok = tok->T; p.tmb = tmb;
         p.ntok = (int)((tok->T + tmb - 1) / tmb);
-        // nearest-rank threshold: the ceil(pct m)-th smallest |Δ| (pct the
-        // single-precision value; the product is exact in double)
-        const int64_t k = (int64_t)std::ceil((double)tok->clip * (double)m) - 1;
+        // nearest-rank threshold: the ceil(pct m)-th smallest |Δ| (pct and
+        // the product in double: the exact rank for a percentile such as 0.95)
+        const int64_t k = (int64_t)std::ceil(tok->clip * (double)m) - 1;
         p.rank_q = std::min<int64_t>(std::max<int64_t>(k, 0), m - 1);
     }
     if (trace) {
@@ -730,7 +730,7 @@ size_t realq_quantize_tokens_workspace_size(int64_t m, int64_t n, int64_t T_mb, 
 realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int64_t n, const void *W0,
                                            realq_dtype_t w_dtype, const float *U, const float *Hbar,
                                            const uint8_t *dead, const void *X_hat, int64_t T, int64_t T_mb,
-                                           float a_loss_clip, const realq_quant_cfg_t *qcfg,
+                                           double a_loss_clip, const realq_quant_cfg_t *qcfg,
                                            const realq_bgd_cfg_t *bcfg, const float *F, const float *F_next,
                                            float *W_work, float *adam_m, float *adam_v, float *bgd_disp,
                                            int64_t *adam_t, uint8_t *codes, float *scale, uint8_t *zero, void *W_deq,
@@ -744,7 +744,7 @@ realq_status_t realq_quantize_layer_tokens(realq_stream_t stream, int64_t m, int
         return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: T_mb <= 2097120 and T <= 2^40 required");
     if (reinterpret_cast<uintptr_t>(X_hat) % 16 != 0 || n % 8 != 0)
         return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: X_hat must be 16-byte aligned with n %% 8 == 0");
-    if (!(a_loss_clip > 0.f && a_loss_clip <= 1.f))
+    if (!(a_loss_clip > 0.0 && a_loss_clip <= 1.0))
         return fail(REALQ_ERR_INVALID_ARG, "quantize_layer_tokens: 0 < a_loss_clip <= 1");
     const TokArgs tok{X_hat, T, T_mb, a_loss_clip};
     return quantize_impl(stream, m, n, W0, w_dtype, 0, 1, nullptr, nullptr, nullptr, 0, nullptr, U, Hbar, nullptr, dead,

@@ -87,7 +87,7 @@ realq_status_t act_quant(cudaStream_t s, int64_t T, int64_t n, const void *X, re
 
 // ------------------------------------------- saliency-weighted Hessians ---
 size_t saliency_clip_ws_bytes();
-realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, float pct, float *S_out,
+realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, double pct, float *S_out,
                              float *clip_out);
 size_t weighted_ws_bytes(int64_t n, int64_t T);
 realq_status_t hessian_weighted(cudaStream_t s, int64_t n, int64_t T, const void *X, int ng, const float *S,

@@ -115,10 +115,10 @@ __global__ void __launch_bounds__(1024) wsum_kernel(int64_t T, int ng, const flo
 
 size_t saliency_clip_ws_bytes() { return 0; }
 
-realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, float pct, float *S_out,
+realq_status_t saliency_clip(cudaStream_t s, int64_t T, int ng, const float *S, double pct, float *S_out,
                              float *clip_out) {
     if (T <= 0) return REALQ_OK;
-    int64_t k = (int64_t)std::ceil((double)pct * (double)T) - 1;
+    int64_t k = (int64_t)std::ceil(pct * (double)T) - 1;
     if (k < 0) k = 0;
     if (k > T - 1) k = T - 1;
     {
