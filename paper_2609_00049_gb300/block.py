@@ -87,6 +87,10 @@ class BlockQuantizer:
     paper's small-model runs) each step's gradient is taken in token form on
     its mini-batch, with the per-token output clipping.
 
+    b_global_start (module name -> 1-based global index of its first column
+    block) and B_total override the numbering above, so that a subset of a
+    block's modules can run with the indices they have in the whole block.
+
     saliency_groups=N_g > 0 selects the saliency-weighted grouped Hessians
     (Sec. 3.3, Alg. 1 "for all row-groups g"): every module's rows form N_g
     groups, run() takes a (T x N_g) saliency per module, clipped to its
@@ -97,7 +101,8 @@ class BlockQuantizer:
     def __init__(self, inputs: Sequence[BlockInput], modules: Sequence[BlockModule], qcfg: QuantCfg, lr: float,
                  steps_per_block: int = 1, sliding_window: bool = False, device="cuda",
                  host_chunk_tokens: int = 32768, act_quant: Optional[tuple] = None, saliency_groups: int = 0,
-                 saliency_pct: float = 0.99, minibatch_tokens: int = 0, a_loss_clip: Optional[float] = None):
+                 saliency_pct: float = 0.99, minibatch_tokens: int = 0, a_loss_clip: Optional[float] = None,
+                 b_global_start: Optional[Dict[str, int]] = None, B_total: Optional[int] = None):
         self.inputs: Dict[str, BlockInput] = {i.name: i for i in inputs}
         self.modules: List[BlockModule] = list(modules)
         for md in self.modules:
@@ -119,7 +124,7 @@ class BlockQuantizer:
             raise ValueError("mini-batch Block-GD is built for the plain, unperturbed sweep")
         self.mods_of = {name: [md for md in self.modules if md.input == name] for name in self.inputs}
         B = qcfg.block_size
-        self.B_total = sum(-(-md.n // B) for md in self.modules)
+        self.B_total = sum(-(-md.n // B) for md in self.modules) if B_total is None else int(B_total)
         dev = self.device
         self.state = {}
         for name, spec in self.inputs.items():
@@ -143,6 +148,8 @@ class BlockQuantizer:
             m, n = md.m, md.n
             g = g_eff or n
             ng = -(-n // g)
+            if b_global_start is not None:
+                bstart = int(b_global_start[md.name])
             bc = bgd_cfg(lr, steps_per_block, b_global_start=bstart,
                          B_total=self.B_total if sliding_window else 1)
             bstart += -(-n // B)

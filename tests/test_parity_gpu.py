@@ -17,7 +17,7 @@ import oracle
 import synth
 import paper_2609_00049_gb300 as rq
 from paper_2609_00049_gb300 import layer
-from parity import compare_codes, scale_agreement, unpack
+from parity import OracleSweep, check_codes_and_scales, follow_ties, unpack
 
 pytestmark = pytest.mark.gpu
 
@@ -116,9 +116,10 @@ def _oracle_and_gpu(case, qkw, bgd=None, steps=1, with_next=False, b_global_star
     Ds = oracle.cross_moment_sum([case.Xhat], [case.X]) if use_dbar else None
     obgd = None if bgd is None else {"lr": bgd, "steps_per_block": steps, "b_global_start": b_global_start,
                                      "B_total": B_total}
-    orc = oracle.realq_sweep(case.W0, Hs, T, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
-                             block_size=qkw.get("block_size", 128), symmetric=bool(qkw.get("symmetric", 0)),
-                             bgd=obgd, F=case.F, F_next=case.F_next if with_next else None, D_sum=Ds)
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        case.W0, Hs, T, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
+        block_size=qkw.get("block_size", 128), symmetric=bool(qkw.get("symmetric", 0)), bgd=obgd, F=case.F,
+        F_next=case.F_next if with_next else None, D_sum=Ds, follow=follow))
     Xh = dev(case.Xhat)
     Xf = dev(case.X) if use_dbar else None
     H, D, T_ = layer.accumulate([Xh], case.Xhat.shape[1], [Xf] if use_dbar else None)
@@ -134,30 +135,11 @@ def _oracle_and_gpu(case, qkw, bgd=None, steps=1, with_next=False, b_global_star
     return orc, out, prep, W0
 
 
-def _adam_scale_bound(orc, n, qkw, lr, steps):
-    # per group: optimizer steps applied to its columns before its parameters
-    B = qkw.get("block_size", 128)
-    g = qkw.get("group_size", 128) or n
-    maxq = 2 ** qkw.get("bits", 4) - 1
-    first_cols = np.arange(orc["scale"].shape[1]) * g
-    taken = np.minimum(first_cols // B, max(0, -(-n // B) - 1)) * steps
-    return np.broadcast_to(4.0 * lr * taken / maxq + 1e-12, orc["scale"].shape)
-
-
 def _check(orc, out, case, qkw, bgd, loss_tol=1e-3, prep=None, W0=None, lr=0.0, steps=1):
     n = case.W0.shape[1]
     codes = unpack(out.codes.cpu().numpy(), n)
-    rep = compare_codes(codes, orc, qkw.get("block_size", 128), qkw.get("group_size", 128), bgd)
-    frac, med, s_unexpl = scale_agreement(out.scale.cpu().numpy(), orc["scale"], qkw.get("group_size", 128),
-                                          explained=compare_codes.last_explained,
-                                          adam_bound=_adam_scale_bound(orc, n, qkw, lr, steps) if bgd else None)
-    print(f"\nparity {qkw} bgd={bgd}: {rep} scale_within_1e-5={frac:.5f} median_rel={med:.2e} "
-          f"scale_unexplained={s_unexpl}")
-    assert rep["frac_equal"] >= 0.999, rep
-    assert rep["n_unexplained"] == 0, rep
-    assert s_unexpl == 0 and frac >= 0.99, (frac, med, s_unexpl)
-    zero_eq = (out.zero.cpu().numpy().astype(np.int64) == orc["zero"]).mean()
-    assert zero_eq >= 0.999
+    _, _, rep = check_codes_and_scales(orc, codes, out.zero.cpu().numpy(), out.scale.cpu().numpy(), n, qkw, bgd,
+                                       lr, steps)
     # dequantized values are the grid points of the returned codes
     g = qkw.get("group_size", 128) or n
     s = out.scale.cpu().numpy()[:, np.arange(n) // g]
@@ -375,22 +357,18 @@ def test_activation_aware_sweep():
     qkw = dict(group_size=128, block_size=128)
     Hs, T = oracle.hessian_sum([xhat])
     Ds = oracle.cross_moment_sum([xhat], [case.Xhat])
-    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128,
-                             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}, F=case.F,
-                             D_sum=Ds)
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        case.W0, Hs, T, group_size=128, block_size=128,
+        bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}, F=case.F, D_sum=Ds,
+        follow=follow))
     H, D, T_ = layer.accumulate([Xq], 256, [X])
     prep = layer.prepare(H, T_, 0.01, D_sum=D)
     out = layer.quantize(dev(case.W0), prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4), F=dev(case.F), use_dbar=True)
     torch.cuda.synchronize()
     n = 256
     codes = unpack(out.codes.cpu().numpy(), n)
-    rep = compare_codes(codes, orc, 128, 128, True)
-    frac, med, s_unexpl = scale_agreement(out.scale.cpu().numpy(), orc["scale"], 128,
-                                          explained=compare_codes.last_explained,
-                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, 1))
-    print(f"\nactivation-aware: {rep} scale_within_1e-5={frac:.5f}")
-    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
-    assert s_unexpl == 0
+    check_codes_and_scales(orc, codes, out.zero.cpu().numpy(), out.scale.cpu().numpy(), n, qkw, True, 2e-4, 1,
+                           "activation-aware ")
 
 
 def test_block_scheduler_activation_aware():
@@ -422,20 +400,16 @@ def test_block_scheduler_activation_aware():
         _, _, xhat = oracle.quantize_activations(x, 4, 0.9)
         Hs, _ = oracle.hessian_sum([xhat])
         Ds = oracle.cross_moment_sum([xhat], [x])
-        orc = oracle.realq_sweep(Wf[nm].astype(np.float64), Hs, T, group_size=64, block_size=64,
-                                 bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": bstart, "B_total": 1},
-                                 F=Ff[nm], D_sum=Ds)
+        orc = OracleSweep(lambda follow, W=Wf[nm], F=Ff[nm], Hs=Hs, Ds=Ds, b0=bstart: oracle.realq_sweep(
+            W.astype(np.float64), Hs, T, group_size=64, block_size=64,
+            bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": b0, "B_total": 1}, F=F, D_sum=Ds,
+            follow=follow))
         bstart += ins[i] // 64
         o = bq.out[nm]
         codes = unpack(o["codes"].cpu().numpy(), ins[i])
-        rep = compare_codes(codes, orc, 64, 64, True)
         qkw = dict(group_size=64, block_size=64)
-        frac, med, s_unexpl = scale_agreement(o["scale"].cpu().numpy(), orc["scale"], 64,
-                                              explained=compare_codes.last_explained,
-                                              adam_bound=_adam_scale_bound(orc, ins[i], qkw, 2e-4, 1))
-        print(f"\nblock W4A4 {nm}: {rep} scale_within_1e-5={frac:.5f}")
-        assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (nm, rep)
-        assert s_unexpl == 0
+        check_codes_and_scales(orc, codes, o["zero"].cpu().numpy(), o["scale"].cpu().numpy(), ins[i], qkw, True,
+                               2e-4, 1, f"block W4A4 {nm} ")
 
 
 # ------------------------------------------ saliency-weighted Hessians ---
@@ -548,9 +522,10 @@ def _grouped_run(seed, m, n, T, ng, qkw, lr=None, correlated=False):
     H_or, T_ = oracle.hessian_sum([case.Xhat])
     bgd = None if lr is None else {"lr": lr, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
     kappa = max(np.linalg.cond(oracle.prepare(Hg_or[g], w_or[g])["Hd"]) for g in range(ng))
-    orc = oracle.realq_sweep(case.W0, H_or, T_, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
-                             block_size=qkw.get("block_size", 128), bgd=bgd, F=case.F,
-                             obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)])
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        case.W0, H_or, T_, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
+        block_size=qkw.get("block_size", 128), bgd=bgd, F=case.F,
+        obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow))
     # GPU path
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     Sc, _ = rq.realq_saliency_clip(dev(S), 0.99)
@@ -578,15 +553,9 @@ def _grouped_run(seed, m, n, T, ng, qkw, lr=None, correlated=False):
                                         F=dev(case.F) if lr is not None else None, ws=wsq, **st)
     rq.realq_workspace_status(wsq)
     codes_np = unpack(codes.cpu().numpy(), n)
-    B = qkw.get("block_size", 128)
-    rep = compare_codes(codes_np, orc, B, qkw.get("group_size", 128), lr is not None)
-    frac, med, s_unexpl = scale_agreement(scale.cpu().numpy(), orc["scale"], qkw.get("group_size", 128),
-                                          explained=compare_codes.last_explained,
-                                          adam_bound=_adam_scale_bound(orc, n, qkw, lr, 1) if lr else None)
-    print(f"\ngrouped ng={ng} {qkw} lr={lr} max cond(H_g,d)={kappa:.1f}: {rep} scale_within_1e-5={frac:.5f} "
-          f"median_rel={med:.2e}")
-    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
-    assert s_unexpl == 0 and frac >= 0.99
+    _, _, rep = check_codes_and_scales(orc, codes_np, zero.cpu().numpy(), scale.cpu().numpy(), n, qkw,
+                                       lr is not None, lr or 0.0, 1,
+                                       f"grouped ng={ng} max cond(H_g,d)={kappa:.1f} ")
     if lr is not None:
         assert t == orc["adam_t"]
     g_ = qkw.get("group_size", 128) or n
@@ -637,8 +606,9 @@ def test_grouped_sweep_exact_hessians():
     for lr in (None, 2e-4):
         qkw = dict(group_size=64, block_size=64)
         bgd = None if lr is None else {"lr": lr, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
-        orc = oracle.realq_sweep(W0, H_or, T, group_size=64, block_size=64, bgd=bgd, F=F,
-                                 obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)])
+        orc = OracleSweep(lambda follow, bgd=bgd: oracle.realq_sweep(
+            W0, H_or, T, group_size=64, block_size=64, bgd=bgd, F=F,
+            obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow))
         q = rq.quant_cfg(**qkw)
         b = None if lr is None else rq.bgd_cfg(lr)
         W = torch.empty(m, n, device="cuda")
@@ -650,9 +620,8 @@ def test_grouped_sweep_exact_hessians():
         rq.realq_quantize_layer_grouped(dev(W0), Ug, Hbg, dg, prep.Hbar, q, W, codes, scale, zero, bcfg=b,
                                         F=dev(F) if lr else None, ws=wsq, **st)
         codes_np = unpack(codes.cpu().numpy(), n)
-        rep = compare_codes(codes_np, orc, 64, 64, lr is not None)
-        print(f"\ngrouped exact-H lr={lr}: {rep}")
-        assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
+        check_codes_and_scales(orc, codes_np, zero.cpu().numpy(), scale.cpu().numpy(), n, qkw, lr is not None,
+                               lr or 0.0, 1, "grouped exact-H ")
 
 
 def test_block_scheduler_saliency_groups():
@@ -687,20 +656,16 @@ def test_block_scheduler_saliency_groups():
         Sc, _ = oracle.saliency_clip(Sal[nm].astype(np.float64), 0.99)
         Hg, w = oracle.weighted_hessian_sum([x], [Sc])
         Hs, _ = oracle.hessian_sum([x])
-        orc = oracle.realq_sweep(Wf[nm].astype(np.float64), Hs, T, group_size=64, block_size=64,
-                                 bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": bstart, "B_total": 1},
-                                 F=Ff[nm], obs_hessians=[(Hg[g], w[g]) for g in range(ng)])
+        orc = OracleSweep(lambda follow, W=Wf[nm], F=Ff[nm], Hs=Hs, Hg=Hg, w=w, b0=bstart: oracle.realq_sweep(
+            W.astype(np.float64), Hs, T, group_size=64, block_size=64,
+            bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": b0, "B_total": 1}, F=F,
+            obs_hessians=[(Hg[g], w[g]) for g in range(ng)], follow=follow))
         bstart += ins[i] // 64
         o = bq.out[nm]
         codes = unpack(o["codes"].cpu().numpy(), ins[i])
-        rep = compare_codes(codes, orc, 64, 64, True)
         qkw = dict(group_size=64, block_size=64)
-        frac, med, s_unexpl = scale_agreement(o["scale"].cpu().numpy(), orc["scale"], 64,
-                                              explained=compare_codes.last_explained,
-                                              adam_bound=_adam_scale_bound(orc, ins[i], qkw, 2e-4, 1))
-        print(f"\nblock grouped {nm}: {rep} scale_within_1e-5={frac:.5f}")
-        assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, (nm, rep)
-        assert s_unexpl == 0
+        check_codes_and_scales(orc, codes, o["zero"].cpu().numpy(), o["scale"].cpu().numpy(), ins[i], qkw, True,
+                               2e-4, 1, f"block grouped {nm} ")
 
 
 # ------------------------------------------------- mini-batch Block-GD ---
@@ -712,7 +677,8 @@ def test_minibatch_block_gd(start, steps):
     mbs = [oracle.hessian_sum([case.Xhat[k * Tm:(k + 1) * Tm]]) for k in range(K)]
     Hs, T = oracle.hessian_sum([case.Xhat])
     bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1, "minibatches": mbs}
-    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd, F=case.F)
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
+                                                        F=case.F, follow=follow))
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     H, _, _ = layer.accumulate([X], 384)
     prep = layer.prepare(H, T)
@@ -734,13 +700,8 @@ def test_minibatch_block_gd(start, steps):
     rq.realq_workspace_status(ws)
     assert t == orc["adam_t"] == 2 * steps
     c = unpack(codes.cpu().numpy(), n)
-    rep = compare_codes(c, orc, 128, 128, True)
-    frac, med, s_unexpl = scale_agreement(scale.cpu().numpy(), orc["scale"], 128,
-                                          explained=compare_codes.last_explained,
-                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, steps))
-    print(f"\nmini-batch start={start} steps={steps}: {rep} scale_within_1e-5={frac:.5f}")
-    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
-    assert s_unexpl == 0
+    check_codes_and_scales(orc, c, zero.cpu().numpy(), scale.cpu().numpy(), n, qkw, True, 2e-4, steps,
+                           f"mini-batch start={start} steps={steps} ")
 
 
 def test_prepare_deferred_status():
@@ -841,7 +802,8 @@ def test_token_block_gd_with_output_clipping(clip, start, steps):
     Hs, T = oracle.hessian_sum([case.Xhat])
     bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1,
            "minibatch_tokens": parts, "a_loss_clip": clip}
-    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd, F=case.F)
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
+                                                        F=case.F, follow=follow))
     qkw = dict(group_size=128, block_size=128)
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     H, _, _ = layer.accumulate([X], 384)
@@ -860,15 +822,9 @@ def test_token_block_gd_with_output_clipping(clip, start, steps):
     rq.realq_workspace_status(ws)
     assert t == orc["adam_t"] == 2 * steps
     c = unpack(codes.cpu().numpy(), n)
-    rep = compare_codes(c, orc, 128, 128, True)
-    frac, med, s_unexpl = scale_agreement(scale.cpu().numpy(), orc["scale"], 128,
-                                          explained=compare_codes.last_explained,
-                                          adam_bound=_adam_scale_bound(orc, n, qkw, 2e-4, steps))
-    dev_deq = np.abs(W.cpu().numpy() - orc["deq"]).max()
-    print(f"\ntoken form clip={clip} start={start} steps={steps}: {rep} scale_within_1e-5={frac:.5f} "
-          f"max|deq - oracle|={dev_deq:.2e}")
-    assert rep["frac_equal"] >= 0.999 and rep["n_unexplained"] == 0, rep
-    assert s_unexpl == 0
+    _, fol, _ = check_codes_and_scales(orc, c, zero.cpu().numpy(), scale.cpu().numpy(), n, qkw, True, 2e-4, steps,
+                                       f"token form clip={clip} start={start} steps={steps} ")
+    print(f"max|deq - oracle|={np.abs(W.cpu().numpy() - fol['deq']).max():.2e}")
 
 
 
@@ -881,10 +837,11 @@ def test_traced_block_losses(with_next):
     qkw = dict(group_size=64, block_size=64)
     kw = dict(b_global_start=3, B_total=9) if with_next else {}
     Hs, T = oracle.hessian_sum([case.Xhat])
-    orc = oracle.realq_sweep(case.W0, Hs, T, group_size=64, block_size=64,
-                             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": kw.get("b_global_start", 1),
-                                  "B_total": kw.get("B_total", 1)},
-                             F=case.F, F_next=case.F_next if with_next else None)
+    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        case.W0, Hs, T, group_size=64, block_size=64,
+        bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": kw.get("b_global_start", 1),
+             "B_total": kw.get("B_total", 1)},
+        F=case.F, F_next=case.F_next if with_next else None, follow=follow))
     H, _, T_ = layer.accumulate([dev(case.Xhat)], 320)
     prep = layer.prepare(H, T_)
     q = rq.quant_cfg(**qkw)
@@ -905,7 +862,10 @@ def test_traced_block_losses(with_next):
     rq.realq_workspace_status(ws)
     got = bl.cpu().numpy()
     assert np.isnan(got[nb - 1]).all()          # the last block takes no step
-    for blk, alpha, before, after in orc["block_loss"]:
+    # on the CUDA path's branch at rounding ties (tests/parity.py)
+    _, fol, _ = check_codes_and_scales(orc, unpack(codes.cpu().numpy(), n), zero.cpu().numpy(),
+                                       scale.cpu().numpy(), n, qkw, True, 2e-4, 1, "traced ")
+    for blk, alpha, before, after in fol["block_loss"]:
         print(f"\nblock {blk} alpha {alpha:.3f}: before {got[blk, 0]:.6e} / {before:.6e}, "
               f"after {got[blk, 1]:.6e} / {after:.6e}")
         assert abs(got[blk, 0] - before) <= 1e-3 * abs(before)
