@@ -15,7 +15,6 @@
 // no host memory).
 #include "kernels.cuh"
 
-#include <mutex>
 #include <vector>
 
 namespace realq {
@@ -274,23 +273,16 @@ constexpr size_t prepare_bytes(int64_t n) { return prepare_bytes_split(n, 1); }
 constexpr size_t kNoAllocBytes = prepare_bytes(REALQ_PREPARE_NOALLOC_MAX_N);
 static __device__ __align__(256) unsigned char g_prepare_scratch[kNoAllocBytes];
 
-std::mutex g_noalloc_mu;
-void *g_noalloc_ptr[256] = {};
-
-// Device address of g_prepare_scratch on the current device (looked up once per device).
+// Device address of g_prepare_scratch on the current device, looked up on
+// every call (it allocates nothing): a cached address would outlive a reset
+// device or a recreated primary context, after which the module is loaded
+// again at another address.
 realq_status_t noalloc_scratch(void **out) {
-    int dev = 0;
-    REALQ_CUDA_TRY(cudaGetDevice(&dev));
-    if (dev < 0 || dev >= 256) return fail(REALQ_ERR_UNSUPPORTED, "device ordinal %d out of range", dev);
-    std::lock_guard<std::mutex> lk(g_noalloc_mu);
-    if (g_noalloc_ptr[dev] == nullptr) {
-        void *p = nullptr;
-        const cudaError_t e = cudaGetSymbolAddress(&p, g_prepare_scratch);
-        if (e != cudaSuccess || p == nullptr)
-            return fail(REALQ_ERR_CUDA, "cudaGetSymbolAddress(prepare scratch): %s", cudaGetErrorString(e));
-        g_noalloc_ptr[dev] = p;
-    }
-    *out = g_noalloc_ptr[dev];
+    void *p = nullptr;
+    const cudaError_t e = cudaGetSymbolAddress(&p, g_prepare_scratch);
+    if (e != cudaSuccess || p == nullptr)
+        return fail(REALQ_ERR_CUDA, "cudaGetSymbolAddress(prepare scratch): %s", cudaGetErrorString(e));
+    *out = p;
     return REALQ_OK;
 }
 
