@@ -1,10 +1,12 @@
 """Throughput of the REAL-Q per-layer quantization sweep on GB300.
 
 One step = the whole sweep of one synthetic decoder block (default: the
-Qwen3-0.6B-shaped block, 128 x 2048 calibration tokens): for each of its four
-distinct inputs the Hessian over all tokens and its preparation, then the
-column sweep with Block-GD of its seven linear modules.  Metric: quantized
-weight-columns per second (whole job; N GPUs run N independent replicas).
+LLaMA-3.1-70B-shaped block, 256 x 2048 calibration tokens, the largest
+block shape; --workload qwen3-0.6b | llama3.1-8b | qwen3-32b for the others):
+for each of its four distinct inputs the Hessian over all tokens and its
+preparation, then the column sweep with Block-GD of its seven linear modules.
+Metric: quantized weight-columns per second (whole job; N GPUs run N
+independent replicas).
 
   python bench.py [--gpus N] [--steps K] [--warmup W] [--impl gpu|reference]
 
@@ -152,11 +154,13 @@ def gpu_arm(args, wl, rank, world):
             dist.barrier()
 
     t_gen = time.time()
-    # ---- inputs: generated on the host (seeded), pinned, then resident on the device
+    # ---- inputs: generated on the host (seeded) straight into page-locked
+    # memory, then resident on the device
     host_x, dev_x = {}, {}
     for name, spec in wl.inputs.items():
-        bits = synth.xhat_full(wl, name, as_bits=True)
-        t = torch.from_numpy(bits.view(np.int16)).view(torch.bfloat16).pin_memory()
+        t = torch.empty((spec.T, spec.n), dtype=torch.int16, pin_memory=True)
+        synth.xhat_full(wl, name, as_bits=True, threads=os.cpu_count() or 8, out=t.numpy())
+        t = t.view(torch.bfloat16)
         host_x[name] = t
         dev_x[name] = t.to(dev, non_blocking=True)
     host_w, dev_w, host_f, dev_f = {}, {}, {}, {}
@@ -249,11 +253,13 @@ def gpu_arm(args, wl, rank, world):
     # launch bracketed by CUDA events on that stream: per-kernel device time for
     # the breakdown and the roofline (in the concurrent timed run the event
     # intervals of overlapping kernels would include each other's time).
+    # (at most two steps: the per-launch averages settle after one)
     prof = {}
+    prof_steps = min(args.steps, 2)
     if not args.no_profile:
         rq.realq_profile_collect()          # drop anything pending
         rq.realq_profile_enable(True)
-        for _ in range(args.steps):
+        for _ in range(prof_steps):
             step_serial()
         torch.cuda.synchronize()
         rq.realq_profile_enable(False)
@@ -262,8 +268,10 @@ def gpu_arm(args, wl, rank, world):
     cols = wl.total_columns * args.steps * world
     value = job_throughput(wl.total_columns, args.steps, world, ms_total)
 
-    # ---- end to end through host buffers
+    # ---- end to end through host buffers (at most three steps: each moves
+    # every input across the host link again)
     e2e = None
+    e_steps = min(args.steps, 3)
     if not args.no_e2e and not args.act_bits and not args.saliency_groups and not args.minibatch_seqs:
         if use_graph:
             e2e_bytes["h2d"], e2e_bytes["d2h"] = bq.capture_host(host_x, host_w, host_f, host_out)
@@ -274,13 +282,14 @@ def gpu_arm(args, wl, rank, world):
         a0 = torch.cuda.Event(enable_timing=True)
         a1 = torch.cuda.Event(enable_timing=True)
         a0.record(stream)
-        for _ in range(args.steps):
+        for _ in range(e_steps):
             step_e2e()
         a1.record(stream)
         torch.cuda.synchronize()
         barrier()
         e_ms = (time.perf_counter() - e0) * 1e3
         e_ms = max_over_ranks(e_ms, dist, dev)
+        e_cols = wl.total_columns * e_steps * world
         # the host link's rate right after the timed steps (one pinned copy of
         # the largest input): the end-to-end step is bound by it, and the
         # link is shared with the host's other GPUs
@@ -291,19 +300,19 @@ def gpu_arm(args, wl, rank, world):
         dst.copy_(big, non_blocking=True)
         torch.cuda.synchronize()
         link_gbs = big.numel() * big.element_size() / (time.perf_counter() - l0) / 1e9
-        e2e = {"value": cols / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": e2e_bytes["h2d"],
-               "d2h_bytes_per_step": e2e_bytes["d2h"], "ms_per_step": e_ms / args.steps,
+        e2e = {"value": e_cols / (e_ms / 1e3), "unit": UNIT, "h2d_bytes_per_step": e2e_bytes["h2d"],
+               "d2h_bytes_per_step": e2e_bytes["d2h"], "ms_per_step": e_ms / e_steps, "steps": e_steps,
                "h2d_link_gbs": round(link_gbs, 1)}
 
     result = None
     if rank == 0:
         peaks = load_peaks()
-        roof = roofline(wl, prof, args.steps, peaks, args)
+        roof = roofline(wl, prof, prof_steps, peaks, args)
         result = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f32",
-            "data": "synthetic (seeded; bf16 weights ~N(0,0.02^2), Gaussian activations with 1% outlier channels x20)",
+            "data": f"synthetic (seeded; {wl.description}; bf16 weights, random init)",
             "config": {"workload": wl.name, "description": wl.description, "modules": len(wl.modules),
                        "calibration_tokens": wl.inputs[wl.modules[0].input].T,
                        "columns_per_step": wl.total_columns, "column_blocks_per_step": wl.total_column_blocks,
@@ -323,7 +332,8 @@ def gpu_arm(args, wl, rank, world):
                              (sum(s.T * s.n * 2 for s in wl.inputs.values()) / 1e9),
                        "input_generation_s": round(t_gen, 1)},
             "roofline": roof,
-            "roofline_by_kernel": roofline_table(wl, prof, args.steps, peaks, args),
+            "roofline_by_kernel": roofline_table(wl, prof, prof_steps, peaks, args),
+            "profile_steps": prof_steps if prof else 0,
             "kernels": {k: {"launches": v[0], "ms": round(v[1], 3)} for k, v in
                                            sorted(prof.items(), key=lambda kv: -kv[1][1])},
             "gpu_launches": int(launches), "clocks": clk, "e2e": e2e,
@@ -457,29 +467,39 @@ def roofline_table(wl, prof, steps, peaks, args=None, top=8):
 # --------------------------------------------------------------------------
 # the CPU oracle (cpu_baseline leg and the reference arm)
 # --------------------------------------------------------------------------
-def oracle_sample(wl, token_sample=8192):
-    """Times the fp64 oracle on module k_proj (or the first module) end to end;
-    the Hessian is accumulated over token_sample tokens and its time scaled to
-    the full token count.  Returns (columns/s, description)."""
+def oracle_sample(wl, token_sample=4096, max_columns=128):
+    """Times the fp64 oracle, as it stands, on one bounded sample of the
+    workload: the k_proj module (or the first), its Hessian over the first
+    token_sample calibration tokens, then preparation (H̄, damping, the
+    inverse) and the literal column sweep with Block-GD over the module's
+    first max_columns columns (the whole module when n <= 2048), each
+    column's compensation and Schur downdate applied to every remaining
+    column of the full n x n inverse.  Returns (columns swept per second of
+    the whole sample, description, seconds).  Nothing is extrapolated: the
+    sample's Hessian is cheaper than the full one (fewer tokens) and its
+    preparation is whole, so the rate is of this sample, not of the module."""
     import oracle
     mod = next((md for md in wl.modules if md.name == "k_proj"), wl.modules[0])
     spec = wl.inputs[mod.input]
+    cols = mod.n if mod.n <= 2048 else min(max_columns, mod.n)
     X = synth.xhat_full(wl, mod.input, as_bits=False, max_tokens=min(token_sample, spec.T))
     W0 = synth.weights(wl, mod, as_bits=False)
     F = synth.fisher(wl, mod)
+    Fn = synth.fisher(wl, mod, "F_next") if wl.sliding_window else None
     t0 = time.perf_counter()
     Hs, T = oracle.hessian_sum([X])
     t_h = time.perf_counter() - t0
-    scale = spec.T / T
     t1 = time.perf_counter()
-    oracle.realq_sweep(W0, Hs * scale, spec.T, bits=wl.bits, group_size=wl.group_size, block_size=wl.block_size,
+    oracle.realq_sweep(W0, Hs, T, bits=wl.bits, group_size=wl.group_size, block_size=wl.block_size,
                        symmetric=bool(wl.symmetric), damp_frac=wl.damp_frac,
-                       bgd={"lr": wl.lr, "steps_per_block": wl.steps_per_block}, F=F, record=False)
+                       bgd={"lr": wl.lr, "steps_per_block": wl.steps_per_block}, F=F, F_next=Fn, record=False,
+                       columns=cols)
     t_s = time.perf_counter() - t1
-    total = t_h * scale + t_s
-    desc = (f"{mod.name} ({mod.n}->{mod.m}) of {wl.name}: Hessian over {T} of {spec.T} tokens "
-            f"({t_h:.2f} s, scaled x{scale:g}), prepare + sweep with Block-GD {t_s:.2f} s")
-    return mod.n / total, desc, total
+    total = t_h + t_s
+    desc = (f"{mod.name} ({mod.n}->{mod.m}) of {wl.name}: Hessian over the first {T} of {spec.T} tokens "
+            f"({t_h:.2f} s), prepare + literal sweep with Block-GD of columns 0..{cols - 1} of {mod.n} "
+            f"({t_s:.2f} s); rate = {cols} columns / {total:.2f} s")
+    return cols / total, desc, total
 
 
 def cpu_cores():
@@ -497,10 +517,12 @@ def cpu_cores():
 
 
 def reference_arm(args, wl, rank, world):
+    """The fp64 oracle on the host cores, one bounded sample per step
+    (oracle_sample), rank 0 only."""
     if rank != 0:
         return None
     vals, descs, secs = [], None, []
-    for _ in range(max(0, min(args.warmup, 1))):
+    for _ in range(args.warmup):
         oracle_sample(wl)
     for _ in range(args.steps):
         v, descs, s = oracle_sample(wl)
@@ -510,8 +532,9 @@ def reference_arm(args, wl, rank, world):
     cb = {"value": value, "unit": UNIT, "cores": cpu_cores(), "kind": "oracle", "sample": descs}
     return {"impl": "reference", "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(secs),
-            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": {"workload": wl.name, "description": wl.description}, "cpu_baseline": cb,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": f"synthetic (seeded; {wl.description})",
+            "config": {"workload": wl.name, "description": wl.description, "sample": descs}, "cpu_baseline": cb,
             "e2e": {"value": value, "unit": UNIT, "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
 
 
@@ -636,10 +659,10 @@ def window_bench(args, peaks):
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
-    ap.add_argument("--steps", type=int, default=40)
+    ap.add_argument("--steps", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=3)
     ap.add_argument("--impl", default="gpu", choices=["gpu", "reference"])
-    ap.add_argument("--workload", default="qwen3-0.6b")
+    ap.add_argument("--workload", default="llama3.1-70b")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--act-bits", type=int, default=0,
                     help="activation-aware weight-activation variant: per-token activation bits (0: weights only)")

@@ -216,13 +216,20 @@ def xhat_chunk(wl: Workload, input_name: str, chunk: int, chunk_tokens: int = CH
 
 
 def xhat_full(wl: Workload, input_name: str, as_bits: bool = True, max_tokens: Optional[int] = None,
-              threads: int = 8) -> np.ndarray:
-    """All (or the first max_tokens) calibration tokens of an input, generated in parallel."""
+              threads: int = 8, out: Optional[np.ndarray] = None) -> np.ndarray:
+    """All (or the first max_tokens) calibration tokens of an input, generated in
+    parallel, into `out` if given (T x n, uint16 for bf16 bits, else fp32;
+    e.g. a view of page-locked memory)."""
     spec = wl.inputs[input_name]
     T = spec.T if max_tokens is None else min(spec.T, max_tokens)
     nch = -(-T // CHUNK_TOKENS)
     dt = np.uint16 if (spec.dtype == "bf16" and as_bits) else np.float32
-    out = np.empty((T, spec.n), dtype=dt)
+    if out is None:
+        out = np.empty((T, spec.n), dtype=dt)
+    elif out.shape != (T, spec.n) or out.dtype.itemsize != np.dtype(dt).itemsize:
+        raise ValueError(f"out must be {T} x {spec.n} of {np.dtype(dt).itemsize}-byte elements")
+    else:
+        out = out.view(dt)
 
     def work(c):
         a = xhat_chunk(wl, input_name, c, CHUNK_TOKENS, as_bits)
