@@ -511,6 +511,16 @@ void realq_graph_destroy(realq_graph_t graph);
  * Computed in fp32 with fp32 accumulation (the loss summed in double).
  * Asynchronous on `stream`; argument errors are returned before any launch.
  * S L is at most 4194240 tokens.  Outputs may not alias inputs. */
+/* The learning rate of decoder block i (1-based) of L under the paper's
+ * reverse-cosine schedule over transformer blocks (App. "Full Setup",
+ * Eq. reverse_cosine; the first block's rate is 0.01 of the final one, App.
+ * "REAL-Q Learning Rates"):
+ *   eta_i = eta_base + (eta_final - eta_base) sin(pi/2 (i - 1) / (L - 1)),
+ *   eta_base = 0.01 eta_final;  eta_final when L = 1.
+ * Host arithmetic in double; *lr_out (host) receives it.  1 <= i <= L and a
+ * finite lr_final required, else REALQ_ERR_INVALID_ARG. */
+realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out);
+
 typedef struct {
     int64_t d, n_heads, n_kv, head_dim, ffn;
     float rms_eps;    /* 1e-6 */

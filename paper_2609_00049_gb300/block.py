@@ -28,7 +28,6 @@ No arithmetic happens here; every step is a call through the C ABI.
 """
 from __future__ import annotations
 
-import math
 from concurrent.futures import ThreadPoolExecutor
 from dataclasses import dataclass
 from typing import Dict, List, Optional, Sequence
@@ -37,7 +36,7 @@ import torch
 
 from . import layer
 from . import (BLOCK_MODULES, REALQ_BF16, REALQ_OPT_ADAM, QuantCfg, bgd_cfg, realq_block_forward,
-               realq_block_module_inputs,
+               realq_block_module_inputs, realq_reverse_cosine_lr,
                realq_block_workspace_size, realq_graph_begin, realq_graph_end, realq_hessian_accumulate,
                realq_hessian_accumulate_weighted, realq_hessian_prepare_deferred, realq_hessian_prepare_scaled,
                realq_hessian_weighted_workspace_size, realq_hessian_workspace_size, realq_prepare_status,
@@ -587,15 +586,6 @@ def quantize_block_exact(dims, W_this: Dict[str, torch.Tensor], x: torch.Tensor,
     return out, W_hat
 
 
-def reverse_cosine_lr(i: int, L: int, lr_final: float) -> float:
-    """The learning rate of decoder block i (1-based) of L: a reverse-cosine
-    ramp from 0.01 lr_final at the first block to lr_final at the last."""
-    base = 0.01 * lr_final
-    if L <= 1:
-        return lr_final
-    return base + (lr_final - base) * math.sin(0.5 * math.pi * (i - 1) / (L - 1))
-
-
 def quantize_model_exact(dims, blocks: Sequence[Dict[str, torch.Tensor]], x: torch.Tensor,
                          fishers: Sequence[torch.Tensor], head_gf: torch.Tensor, head_Wh: torch.Tensor,
                          qcfg: QuantCfg, lr_final: float, **kw):
@@ -616,7 +606,7 @@ def quantize_model_exact(dims, blocks: Sequence[Dict[str, torch.Tensor]], x: tor
     out = []
     for l, W in enumerate(blocks):
         last = l == Lb - 1
-        lr = reverse_cosine_lr(l + 1, Lb, lr_final)
+        lr = realq_reverse_cosine_lr(l + 1, Lb, lr_final)
         if last:
             res, W_hat = quantize_block_exact(dims, W, x_ref, qcfg, lr, x_hat=x_hat, head_gf=head_gf,
                                               head_Wh=head_Wh, **kw)

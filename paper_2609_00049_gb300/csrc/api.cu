@@ -799,6 +799,20 @@ realq_status_t realq_bgd_refine(realq_stream_t stream, int64_t m, int64_t n, int
     return bgd_step(S(stream), p, col_start, alpha);
 }
 
+// ------------------------------------------------------------ schedules ---
+realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out) {
+    if (!lr_out || L < 1 || i < 1 || i > L || !std::isfinite(lr_final))
+        return fail(REALQ_ERR_INVALID_ARG, "reverse_cosine_lr: need 1 <= i <= L and a finite rate");
+    if (L == 1) {
+        *lr_out = lr_final;
+        return REALQ_OK;
+    }
+    const double base = 0.01 * lr_final;
+    const double half_pi = 1.5707963267948966;
+    *lr_out = base + (lr_final - base) * std::sin(half_pi * (double)(i - 1) / (double)(L - 1));
+    return REALQ_OK;
+}
+
 // ------------------------------------------------------------ surrogate ---
 size_t realq_surrogate_workspace_size(int64_t m, int64_t n) { return (m > 0 && n > 0) ? surrogate_ws_bytes(m, n) : 0; }
 

@@ -320,3 +320,17 @@ def test_block_bindings_check_shapes_before_any_call(L):
         rq.realq_block_forward(dims, bad, x, torch.zeros_like(x), None)
     with pytest.raises(ValueError, match="X_out"):
         rq.realq_block_module_inputs(dims, W, x, "o_proj", torch.zeros(16, d + 1), None)
+
+
+def test_reverse_cosine_schedule_is_the_oracles(L):
+    # host arithmetic behind the ABI (Eq. reverse_cosine): the same rates as
+    # the oracle's schedule, and invalid indices refused
+    import oracle
+    import paper_2609_00049_gb300 as rq
+    for Lb in (1, 2, 28, 80):
+        for i in range(1, Lb + 1):
+            got = rq.realq_reverse_cosine_lr(i, Lb, 3e-6)
+            assert abs(got - oracle.reverse_cosine_lr(i, Lb, 3e-6)) <= 1e-15 * 3e-6
+    out = ctypes.c_double(0.0)
+    for i, Lb in ((0, 4), (5, 4), (1, 0)):
+        assert L.realq_reverse_cosine_lr(i, Lb, ctypes.c_double(1e-3), ctypes.byref(out)) == 1
