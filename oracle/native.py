@@ -13,6 +13,7 @@ from __future__ import annotations
 import ctypes
 import os
 import subprocess
+from concurrent.futures import ThreadPoolExecutor
 
 import numpy as np
 
@@ -83,3 +84,23 @@ def outer_sub(A: np.ndarray, u: np.ndarray, v: np.ndarray, d: float = None) -> N
         lib.realq_oracle_outer_sub(rows, cols, av[0], av[1], uv[0], uv[1], vp)
     else:
         lib.realq_oracle_outer_sub_div(rows, cols, av[0], av[1], uv[0], uv[1], vp, float(d))
+
+
+_pool = None
+
+
+def row_chunks(rows: int, size: int, fn, min_size: int = 1 << 20) -> None:
+    """fn(r0, r1) over row ranges covering [0, rows): in one call for small
+    work, else split among threads (numpy releases the interpreter lock in
+    its elementwise loops).  The ranges do not overlap."""
+    global _pool
+    nt = os.cpu_count() or 1
+    if size < min_size or nt == 1 or rows < 2:
+        fn(0, rows)
+        return
+    if _pool is None:
+        _pool = ThreadPoolExecutor(nt)
+    step = -(-rows // nt)
+    futs = [_pool.submit(fn, r0, min(rows, r0 + step)) for r0 in range(0, rows, step)]
+    for f in futs:
+        f.result()

@@ -41,7 +41,7 @@ from . import native
 __all__ = [
     "hessian_sum", "cross_moment_sum", "prepare", "inverse_upper_cholesky",
     "quant_params", "quantize", "rtn", "sliding_alpha", "reverse_cosine_lr", "Adam",
-    "surrogate_tokens", "surrogate_moment", "gradient", "realq_sweep", "pack_codes",
+    "surrogate_tokens", "surrogate_moment", "gradient", "gradient_error_scale", "realq_sweep", "pack_codes",
     "round_bf16", "quantize_activations", "saliency_clip", "weighted_hessian_sum",
     "loss_clip_factors", "gradient_tokens", "surrogate_tokens_clipped", "nearest_rank",
 ]
@@ -230,15 +230,24 @@ class Adam:
         self.lr, self.beta1, self.beta2, self.eps = lr, beta1, beta2, eps
 
     def direction(self, g: np.ndarray, cols: slice) -> np.ndarray:
-        """Advance the moments of columns `cols` with gradient g; return the step."""
+        """Advance the moments of columns `cols` with gradient g; return the step.
+        (Every entry is independent: large updates are shared among threads
+        by rows, with the same operations on every entry.)"""
         self.t += 1
-        m = self.m[:, cols]
-        v = self.v[:, cols]
-        m[...] = self.beta1 * m + (1.0 - self.beta1) * g
-        v[...] = self.beta2 * v + (1.0 - self.beta2) * g * g
-        mhat = m / (1.0 - self.beta1 ** self.t)
-        vhat = v / (1.0 - self.beta2 ** self.t)
-        return self.lr * mhat / (np.sqrt(vhat) + self.eps)
+        step = np.empty_like(g)
+
+        def rows(r0, r1):
+            m = self.m[r0:r1, cols]
+            v = self.v[r0:r1, cols]
+            gr = g[r0:r1]
+            m[...] = self.beta1 * m + (1.0 - self.beta1) * gr
+            v[...] = self.beta2 * v + (1.0 - self.beta2) * gr * gr
+            mhat = m / (1.0 - self.beta1 ** self.t)
+            vhat = v / (1.0 - self.beta2 ** self.t)
+            step[r0:r1] = self.lr * mhat / (np.sqrt(vhat) + self.eps)
+
+        native.row_chunks(g.shape[0], g.size, rows)
+        return step
 
 
 # ---------------------------------------------------------------------------
@@ -268,13 +277,26 @@ def surrogate_moment(What, W0, Hbar, F) -> float:
     return 0.5 * float(np.sum((np.asarray(F, dtype=np.float64) @ dW) * (dW @ np.asarray(Hbar, dtype=np.float64))))
 
 
-def gradient(What, W0, Hbar, Dbar, F) -> np.ndarray:
-    """dL/dŴ = F P with P = (1/T) sum_t Δy_t x̂_t^T = (Ŵ - W0) H̄ + W0 D̄ (m x n)."""
+def _gradient_factor(What, W0, Hbar, Dbar, cols: slice) -> np.ndarray:
+    """P = (1/T) sum_t Δy_t x̂_t^T = (Ŵ - W0) H̄ + W0 D̄, columns `cols`."""
     W0 = np.asarray(W0, dtype=np.float64)
-    P = (np.asarray(What, dtype=np.float64) - W0) @ np.asarray(Hbar, dtype=np.float64)
+    P = (np.asarray(What, dtype=np.float64) - W0) @ np.asarray(Hbar, dtype=np.float64)[:, cols]
     if Dbar is not None:
-        P = P + W0 @ np.asarray(Dbar, dtype=np.float64)
-    return np.asarray(F, dtype=np.float64) @ P
+        P = P + W0 @ np.asarray(Dbar, dtype=np.float64)[:, cols]
+    return P
+
+
+def gradient(What, W0, Hbar, Dbar, F, cols: slice = slice(None)) -> np.ndarray:
+    """dL/dŴ = F P for the columns `cols` of Ŵ (m x |cols|; every column of P
+    is its own product)."""
+    return np.asarray(F, dtype=np.float64) @ _gradient_factor(What, W0, Hbar, Dbar, cols)
+
+
+def gradient_error_scale(What, W0, Hbar, Dbar, F, cols: slice = slice(None)) -> np.ndarray:
+    """|F| |P| for the columns `cols`: the sum of the magnitudes of the terms
+    of each gradient entry, the scale of its rounding error in any
+    floating-point evaluation (a sensitivity probe; not part of the method)."""
+    return np.abs(np.asarray(F, dtype=np.float64)) @ np.abs(_gradient_factor(What, W0, Hbar, Dbar, cols))
 
 
 # ---------------------------------------------------------------------------
@@ -359,7 +381,7 @@ def pack_codes(codes: np.ndarray) -> np.ndarray:
 # ---------------------------------------------------------------------------
 def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetric=False,
                 damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True, obs_hessians=None,
-                follow=None, columns=None):
+                follow=None, columns=None, grad_noise=None):
     """Quantize W0 column by column with OBS feedback and Block-GD after each block.
 
     bgd: None for the plain column sweep (GPTQ), else a dict with keys
@@ -417,6 +439,15 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
 
     columns: None for the whole sweep, or stop after that many columns (a
     bounded sample of the work, for timing).
+
+    grad_noise: None, or a sensitivity probe {"seed", "eta"}: every moment-form
+    Block-GD gradient entry moves by eta times the magnitude of its terms
+    (gradient_error_scale) times a seeded standard normal, the size of the
+    rounding differences that any floating-point evaluation of the gradient
+    may show.  Comparing a probed run with the plain one shows which
+    decisions the sweep's arithmetic does not determine at that precision.
+    The returned "x" holds every column's w / scale before rounding, "zf"
+    every group's -xmin / scale.
     """
     W0 = np.asarray(W0, dtype=np.float64)
     m, n = W0.shape
@@ -446,7 +477,9 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     zero = np.zeros((m, ngroups), dtype=np.int64)
     margin = np.zeros((m, n))
     zmargin = np.zeros((m, ngroups))
+    zfval = np.zeros((m, ngroups))
     eps_cols = np.zeros((m, n))
+    xval = np.zeros((m, n))
     hinv_diag = np.zeros((len(groups), n))
     block_loss = []
     opt = None
@@ -462,6 +495,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         if j % g == 0:
             gi = j // g
             scale[:, gi], zero[:, gi], zmargin[:, gi], zf = _grid(W[:, j:j + g], bits, symmetric)
+            zfval[:, gi] = zf
             if follow is not None and follow.get("zero") is not None and not symmetric:
                 zero[:, gi], took = _follow_tie(zero[:, gi], zf, zmargin[:, gi], follow["zero"][:, gi], tau, 0,
                                                 0, maxq)
@@ -475,6 +509,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         e = W[:, j] - dq                       # residual delta_j of Eq. (gptq_update)
         codes[:, j] = q
         margin[:, j] = mg
+        xval[:, j] = x
         eps_cols[:, j] = e
         for k, ((rows, _, _), Hinv) in enumerate(zip(groups, Hinvs)):
             d = Hinv[j, j]
@@ -516,7 +551,14 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
                             raise ValueError("mini-batch moments with perturbed inputs are not supported")
                         Hk, Tk = mbs[((b_global - 1) * steps + si) % len(mbs)]
                         Hstep = np.asarray(Hk, dtype=np.float64) / float(Tk)
-                    G = gradient(W, W0, Hstep, Dbar, Feff)[:, be:]
+                    G = gradient(W, W0, Hstep, Dbar, Feff, slice(be, n))
+                    if grad_noise is not None:
+                        # sensitivity probe: each entry moved by a random
+                        # multiple of its terms' magnitude (eta ~ the
+                        # relative rounding of one floating-point product)
+                        gen = np.random.default_rng([int(grad_noise["seed"]), int(opt.t)])
+                        G = G + grad_noise["eta"] * gradient_error_scale(W, W0, Hstep, Dbar, Feff, slice(be, n)) \
+                            * gen.standard_normal(G.shape)
                 if bgd.get("optimizer", "adam") == "sgd":
                     opt.t += 1
                     W[:, be:] -= bgd["lr"] * G
@@ -533,7 +575,7 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
         "margin": margin, "zero_margin": zmargin, "eps": eps_cols,
         "hinv_diag": hinv_diag[0] if obs_hessians is None else hinv_diag,
         "block_loss": block_loss, "adam_t": 0 if opt is None else opt.t,
-        "n_followed": n_followed, "n_followed_zero": n_followed_zero,
+        "n_followed": n_followed, "n_followed_zero": n_followed_zero, "x": xval, "zf": zfval,
         "Hbar": Hbar, "Hd": Hd, "dead": dead, "lam": prep["lam"], "Dbar": Dbar,
     }
 

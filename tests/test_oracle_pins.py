@@ -742,3 +742,39 @@ def test_token_minibatch_sweep_reduces_to_the_moment_minibatch_sweep():
                            bgd={**base, "minibatch_tokens": parts, "a_loss_clip": 0.95})
     assert np.array_equal(c["codes"][:, :16], a["codes"][:, :16])
     assert not np.allclose(c["deq"][:, 16:], a["deq"][:, 16:], rtol=0, atol=1e-9)
+
+
+# ---------------------------------------------------------------------------
+# The gradient of a column range is those columns of the full gradient; its
+# error scale |F| |P| bounds it (triangle inequality) and equals it when no
+# term cancels; the sensitivity probe with eta = 0 is the plain sweep, and
+# the sweep's pre-rounding values give its codes and zero points.
+# ---------------------------------------------------------------------------
+def test_gradient_columns_error_scale_and_probe():
+    case = synth.layer_case(16, 24, 96, 500, outliers=2, perturbed=True)
+    H, T = oracle.hessian_sum([case.Xhat])
+    D = oracle.cross_moment_sum([case.Xhat], [case.X])
+    r = np.random.default_rng(17)
+    What = case.W0 + r.standard_normal(case.W0.shape) * 0.003
+    full = oracle.gradient(What, case.W0, H / T, D / T, case.F)
+    part = oracle.gradient(What, case.W0, H / T, D / T, case.F, slice(40, 96))
+    np.testing.assert_allclose(part, full[:, 40:], rtol=1e-12, atol=1e-15 * np.abs(full).max())
+    scale = oracle.gradient_error_scale(What, case.W0, H / T, D / T, case.F, slice(40, 96))
+    assert np.all(np.abs(part) <= scale * (1 + 1e-12))
+    pos = oracle.gradient_error_scale(np.abs(What) + 1.0, np.zeros_like(What), np.abs(H) / T, None,
+                                      np.abs(case.F))
+    np.testing.assert_allclose(pos, oracle.gradient(np.abs(What) + 1.0, np.zeros_like(What), np.abs(H) / T, None,
+                                                    np.abs(case.F)), rtol=1e-12)
+    c2 = synth.layer_case(18, 20, 256, 600, outliers=2)
+    H2, T2 = oracle.hessian_sum([c2.Xhat])
+    kw = dict(group_size=64, block_size=64, bgd={"lr": 1e-4}, F=c2.F)
+    a = oracle.realq_sweep(c2.W0, H2, T2, **kw)
+    b = oracle.realq_sweep(c2.W0, H2, T2, grad_noise={"seed": 3, "eta": 0.0}, **kw)
+    for k in ("codes", "scale", "zero", "deq", "x"):
+        assert np.array_equal(a[k], b[k]), k
+    p = oracle.realq_sweep(c2.W0, H2, T2, grad_noise={"seed": 3, "eta": 1e-6}, **kw)
+    assert not np.array_equal(a["x"][:, 64:], p["x"][:, 64:])     # the probe moves the later blocks
+    assert np.array_equal(a["x"][:, :64], p["x"][:, :64])         # and nothing before the first step
+    g = np.arange(256) // 64
+    assert np.array_equal(a["codes"], np.clip(np.rint(a["x"]).astype(np.int64) + a["zero"][:, g], 0, 15))
+    assert np.array_equal(a["zero"], np.rint(a["zf"]).astype(np.int64))
