@@ -43,49 +43,108 @@ def code_report(gpu_codes: np.ndarray, orc: dict, gpu_zero: np.ndarray = None, t
 
 
 class OracleSweep:
-    """One oracle sweep, run plainly at once and again on request with a
-    follow: sweep(None) is the plain result (also reachable as sweep[key]),
-    sweep(follow) a rerun.  fn(follow) runs the oracle."""
+    """One oracle sweep, run plainly at once and again on request:
+    sweep(None) is the plain result (also reachable as sweep[key]),
+    sweep(follow, grad_noise) a rerun.  fn(follow, grad_noise=None) runs
+    the oracle (oracle.realq_sweep's arguments of those names)."""
 
-    def __init__(self, fn):
+    def __init__(self, fn, eager: bool = True):
         self.fn = fn
-        self.plain = fn(None)
+        self._plain = fn(None) if eager else None
 
-    def __call__(self, follow):
-        return self.plain if follow is None else self.fn(follow)
+    @property
+    def plain(self):
+        if self._plain is None:
+            self._plain = self.fn(None)
+        return self._plain
+
+    def __call__(self, follow, grad_noise=None):
+        if follow is None and grad_noise is None:
+            return self.plain
+        return self.fn(follow, grad_noise=grad_noise) if grad_noise is not None else self.fn(follow)
 
     def __getitem__(self, key):
         return self.plain[key]
 
 
-def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: float = 1e-3):
-    """run(follow) -> an oracle sweep result (oracle.realq_sweep with that follow).
+# The sensitivity probe: how far the sweep's pre-rounding values move when
+# every Block-GD gradient entry moves by eta times the magnitude of its terms
+# (oracle.gradient_error_scale), eta the rounding of an fp32 accumulation over
+# the two contractions of the gradient (P over n inputs, G over m outputs) plus
+# the tf32x3 splitting error of one product.  Two seeded probes; a decision
+# whose margin is within PROBE_K times the larger move is not determined by
+# the method's arithmetic at fp32 precision (Adam's m / sqrt(v) amplifies the
+# rounding of a gradient entry whose moments nearly cancel).
+PROBE_K = 10.0
+PROBE_SEEDS = (101, 202)
+
+
+def probe_eta(m: int, n: int) -> float:
+    return 2.0 ** -24 * float(np.sqrt(m + n)) + 2.0 ** -21
+
+
+def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: float = 1e-3,
+                plain_first: bool = True):
+    """run(follow[, grad_noise]) -> an oracle sweep result (oracle.realq_sweep
+    with that follow).
 
     Runs the oracle plainly; if its codes or zero points differ from the
     CUDA path's, runs it again taking the CUDA path's decision at each of its
-    own rounding ties.  Returns (plain result, followed result, report): the
-    report compares the CUDA path with the followed run, every remaining
-    mismatch counting as unexplained, and carries the plain comparison
-    (plain_frac_equal, plain_n_mismatch) and the decisions followed."""
-    plain = run(None)
-    rep0 = code_report(gpu_codes, plain, gpu_zero, tau)
-    if rep0["n_mismatch"] == 0 and rep0["n_zero_mismatch"] == 0:
+    own rounding ties.  If codes still differ, the followed run is repeated
+    under the sensitivity probe: a remaining mismatch whose margin is within
+    PROBE_K times the probes' move of that value is counted as
+    n_conditioned, every other one as unexplained.  Returns (plain result,
+    followed result, report); the report carries the plain comparison
+    (plain_frac_equal, plain_n_mismatch), the decisions followed, and the
+    probes' per-group moves of the scales as fol["probe_scale_move"].
+    plain_first=False skips the plain run (where the oracle is slow): the
+    oracle runs once, with the follow, and the plain entries are None."""
+    if plain_first:
+        plain = run(None)
+        rep0 = code_report(gpu_codes, plain, gpu_zero, tau)
+    else:
+        plain, rep0 = None, {"frac_equal": None, "n_mismatch": None, "n_zero_mismatch": None}
+    if plain_first and rep0["n_mismatch"] == 0 and rep0["n_zero_mismatch"] == 0:
         rep0.update(plain_frac_equal=rep0["frac_equal"], plain_n_mismatch=0, n_followed=0, n_followed_zero=0,
-                    n_unexplained=0)
+                    n_unexplained=0, n_conditioned=0)
         return plain, plain, rep0
-    fol = run({"codes": np.asarray(gpu_codes, dtype=np.int64),
-               "zero": None if gpu_zero is None else np.asarray(gpu_zero, dtype=np.int64), "tau": tau})
+    follow = {"codes": np.asarray(gpu_codes, dtype=np.int64),
+              "zero": None if gpu_zero is None else np.asarray(gpu_zero, dtype=np.int64), "tau": tau}
+    fol = run(follow)
     rep = code_report(gpu_codes, fol, gpu_zero, tau)
     rep.update(plain_frac_equal=rep0["frac_equal"], plain_n_mismatch=rep0["n_mismatch"],
-               n_followed=int(fol["n_followed"]), n_followed_zero=int(fol["n_followed_zero"]),
-               n_unexplained=rep["n_mismatch"] + rep["n_zero_mismatch"])
+               n_followed=int(fol["n_followed"]), n_followed_zero=int(fol["n_followed_zero"]), n_conditioned=0)
+    mism = gpu_codes != fol["codes"]
+    zmism = np.zeros_like(fol["zero"], dtype=bool) if gpu_zero is None else \
+        np.asarray(gpu_zero, dtype=np.int64) != fol["zero"]
+    if mism.any() or zmism.any():
+        m, n = gpu_codes.shape
+        eta = probe_eta(m, n)
+        dx = np.zeros((m, n))
+        dz = np.zeros_like(fol["zf"])
+        ds = np.zeros(fol["scale"].shape)
+        for seed in PROBE_SEEDS:
+            pr = run(follow, grad_noise={"seed": seed, "eta": eta})
+            dx = np.maximum(dx, np.abs(pr["x"] - fol["x"]))
+            dz = np.maximum(dz, np.abs(pr["zf"] - fol["zf"]))
+            ds = np.maximum(ds, np.abs(pr["scale"].astype(np.float64) - fol["scale"].astype(np.float64)))
+        cond = mism & (fol["margin"] <= PROBE_K * dx)
+        zcond = zmism & (fol["zero_margin"] <= PROBE_K * dz)
+        fol = dict(fol, probe_scale_move=ds)
+        rep["n_conditioned"] = int(cond.sum() + zcond.sum())
+        rep["n_unexplained"] = int((mism & ~cond).sum() + (zmism & ~zcond).sum())
+    else:
+        rep["n_unexplained"] = 0
     return plain, fol, rep
 
 
-def scale_agreement(gpu_scale: np.ndarray, orc_scale: np.ndarray, rtol: float = 1e-5, adam_bound: np.ndarray = None):
+def scale_agreement(gpu_scale: np.ndarray, orc_scale: np.ndarray, rtol: float = 1e-5, adam_bound: np.ndarray = None,
+                    probe_move: np.ndarray = None):
     """(fraction of groups within rtol, median relative error, groups off by
     more than rtol and beyond adam_bound, groups off by more than rtol but
-    within adam_bound).
+    within adam_bound).  probe_move (per group): the sensitivity probes' move
+    of the oracle's scale; a group off by at most PROBE_K times it counts as
+    within rtol (its scale is not determined at fp32 precision).
 
     adam_bound (per group, absolute; reading R18): a scale is (xmax - xmin) /
     (2^b - 1); an Adam step at t = 1 is lr times the sign of the gradient, and
@@ -97,6 +156,8 @@ def scale_agreement(gpu_scale: np.ndarray, orc_scale: np.ndarray, rtol: float = 
     diff = np.abs(gpu_scale.astype(np.float64) - orc_scale.astype(np.float64))
     rel = diff / np.abs(orc_scale.astype(np.float64))
     off = rel > rtol
+    if probe_move is not None:
+        off = off & (diff > PROBE_K * probe_move)
     if adam_bound is not None:
         bad = off & (diff > adam_bound)
     else:
@@ -115,19 +176,22 @@ def adam_scale_bound(orc_scale: np.ndarray, n: int, qkw: dict, lr: float, steps:
     return np.broadcast_to(4.0 * lr * taken / maxq + 1e-12, orc_scale.shape)
 
 
-def check_codes_and_scales(orc, codes, zero, scale, n, qkw, bgd, lr=0.0, steps=1, what=""):
+def check_codes_and_scales(orc, codes, zero, scale, n, qkw, bgd, lr=0.0, steps=1, what="", plain_first=True):
     """The codes bar on the CUDA path's branch (follow_ties: >= 99.9 %
-    identical, none unexplained) and the scales within 1e-5 relative, apart
-    from groups within the Adam-sign allowance of reading R18 (counted; at
-    most 0.1 % of the groups plus one).  Returns (plain, followed, report)."""
-    plain, fol, rep = follow_ties(orc, codes, zero)
+    identical, none unexplained, decisions the arithmetic does not
+    determine at most 1e-5 of the codes plus one) and the scales within 1e-5
+    relative, apart from groups within the probes' move and groups within
+    the Adam-sign allowance of reading R18 (counted; at most 0.1 % of the
+    groups plus one).  Returns (plain, followed, report)."""
+    plain, fol, rep = follow_ties(orc, codes, zero, plain_first=plain_first)
     frac, med, s_bad, s_allow = scale_agreement(scale, fol["scale"],
                                                 adam_bound=adam_scale_bound(fol["scale"], n, qkw, lr, steps)
-                                                if bgd else None)
+                                                if bgd else None, probe_move=fol.get("probe_scale_move"))
     rep.update(scale_within_1e5=frac, scale_median_rel=med, scale_beyond=s_bad, adam_sign_allowance=s_allow)
     print(f"\nparity {what}{qkw} bgd={bgd}: {rep}")
     assert rep["frac_equal"] >= 0.999, rep
     assert rep["n_unexplained"] == 0, rep
+    assert rep["n_conditioned"] <= 1 + 1e-5 * codes.size, rep
     assert s_bad == 0, (frac, med, s_bad)
     assert s_allow <= 1 + 1e-3 * scale.size, (s_allow, scale.size)
     return plain, fol, rep

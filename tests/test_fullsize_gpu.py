@@ -115,9 +115,9 @@ def test_fullsize_sweeps_against_oracle(block_run, oracle_H):
         Href, T = oracle_H[md.input], spec.T
         W0 = synth.bf16_bits_to_f32(w_bits[md.name]).astype(np.float64)
         bgd = dict(lr=wl.lr, steps_per_block=wl.steps_per_block, b_global_start=bstart, B_total=1)
-        orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
             W0, Href, T, bits=wl.bits, group_size=wl.group_size, block_size=B, symmetric=bool(wl.symmetric),
-            damp_frac=wl.damp_frac, bgd=bgd, F=F_np[md.name], record=False, follow=follow))
+            damp_frac=wl.damp_frac, bgd=bgd, F=F_np[md.name], record=False, follow=follow, grad_noise=grad_noise))
         nb = -(-md.n // B)
         bstart += nb
         o = bq.out[md.name]
@@ -155,9 +155,9 @@ def test_fullsize_gptq_rows_every_module(block_run, oracle_H):
         mods = [md for md in wl.modules if md.input == nm]
         rows = {md.name: np.sort(r.choice(md.m, 6, replace=False)) for md in mods}
         W_rows = np.concatenate([synth.bf16_bits_to_f32(w_bits[md.name])[rows[md.name]] for md in mods])
-        orc = OracleSweep(lambda follow: oracle.realq_sweep(
+        orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
             W_rows.astype(np.float64), oracle_H[nm], spec.T, bits=wl.bits, group_size=g, block_size=B,
-            symmetric=bool(wl.symmetric), damp_frac=wl.damp_frac, follow=follow))
+            symmetric=bool(wl.symmetric), damp_frac=wl.damp_frac, follow=follow, grad_noise=grad_noise))
         codes = np.concatenate([unpack(bq.out[md.name]["codes"].cpu().numpy(), md.n)[rows[md.name]]
                                 for md in mods])
         scale = np.concatenate([bq.out[md.name]["scale"].cpu().numpy()[rows[md.name]] for md in mods])

@@ -116,10 +116,10 @@ def _oracle_and_gpu(case, qkw, bgd=None, steps=1, with_next=False, b_global_star
     Ds = oracle.cross_moment_sum([case.Xhat], [case.X]) if use_dbar else None
     obgd = None if bgd is None else {"lr": bgd, "steps_per_block": steps, "b_global_start": b_global_start,
                                      "B_total": B_total}
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
         case.W0, Hs, T, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
         block_size=qkw.get("block_size", 128), symmetric=bool(qkw.get("symmetric", 0)), bgd=obgd, F=case.F,
-        F_next=case.F_next if with_next else None, D_sum=Ds, follow=follow))
+        F_next=case.F_next if with_next else None, D_sum=Ds, follow=follow, grad_noise=grad_noise))
     Xh = dev(case.Xhat)
     Xf = dev(case.X) if use_dbar else None
     H, D, T_ = layer.accumulate([Xh], case.Xhat.shape[1], [Xf] if use_dbar else None)
@@ -357,10 +357,10 @@ def test_activation_aware_sweep():
     qkw = dict(group_size=128, block_size=128)
     Hs, T = oracle.hessian_sum([xhat])
     Ds = oracle.cross_moment_sum([xhat], [case.Xhat])
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
         case.W0, Hs, T, group_size=128, block_size=128,
         bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}, F=case.F, D_sum=Ds,
-        follow=follow))
+        follow=follow, grad_noise=grad_noise))
     H, D, T_ = layer.accumulate([Xq], 256, [X])
     prep = layer.prepare(H, T_, 0.01, D_sum=D)
     out = layer.quantize(dev(case.W0), prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4), F=dev(case.F), use_dbar=True)
@@ -400,10 +400,10 @@ def test_block_scheduler_activation_aware():
         _, _, xhat = oracle.quantize_activations(x, 4, 0.9)
         Hs, _ = oracle.hessian_sum([xhat])
         Ds = oracle.cross_moment_sum([xhat], [x])
-        orc = OracleSweep(lambda follow, W=Wf[nm], F=Ff[nm], Hs=Hs, Ds=Ds, b0=bstart: oracle.realq_sweep(
+        orc = OracleSweep(lambda follow, grad_noise=None, W=Wf[nm], F=Ff[nm], Hs=Hs, Ds=Ds, b0=bstart: oracle.realq_sweep(
             W.astype(np.float64), Hs, T, group_size=64, block_size=64,
             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": b0, "B_total": 1}, F=F, D_sum=Ds,
-            follow=follow))
+            follow=follow, grad_noise=grad_noise))
         bstart += ins[i] // 64
         o = bq.out[nm]
         codes = unpack(o["codes"].cpu().numpy(), ins[i])
@@ -522,10 +522,10 @@ def _grouped_run(seed, m, n, T, ng, qkw, lr=None, correlated=False):
     H_or, T_ = oracle.hessian_sum([case.Xhat])
     bgd = None if lr is None else {"lr": lr, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
     kappa = max(np.linalg.cond(oracle.prepare(Hg_or[g], w_or[g])["Hd"]) for g in range(ng))
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
         case.W0, H_or, T_, bits=qkw.get("bits", 4), group_size=qkw.get("group_size", 128),
         block_size=qkw.get("block_size", 128), bgd=bgd, F=case.F,
-        obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow))
+        obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow, grad_noise=grad_noise))
     # GPU path
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     Sc, _ = rq.realq_saliency_clip(dev(S), 0.99)
@@ -606,9 +606,9 @@ def test_grouped_sweep_exact_hessians():
     for lr in (None, 2e-4):
         qkw = dict(group_size=64, block_size=64)
         bgd = None if lr is None else {"lr": lr, "steps_per_block": 1, "b_global_start": 1, "B_total": 1}
-        orc = OracleSweep(lambda follow, bgd=bgd: oracle.realq_sweep(
+        orc = OracleSweep(lambda follow, grad_noise=None, bgd=bgd: oracle.realq_sweep(
             W0, H_or, T, group_size=64, block_size=64, bgd=bgd, F=F,
-            obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow))
+            obs_hessians=[(Hg_or[g], w_or[g]) for g in range(ng)], follow=follow, grad_noise=grad_noise))
         q = rq.quant_cfg(**qkw)
         b = None if lr is None else rq.bgd_cfg(lr)
         W = torch.empty(m, n, device="cuda")
@@ -656,10 +656,10 @@ def test_block_scheduler_saliency_groups():
         Sc, _ = oracle.saliency_clip(Sal[nm].astype(np.float64), 0.99)
         Hg, w = oracle.weighted_hessian_sum([x], [Sc])
         Hs, _ = oracle.hessian_sum([x])
-        orc = OracleSweep(lambda follow, W=Wf[nm], F=Ff[nm], Hs=Hs, Hg=Hg, w=w, b0=bstart: oracle.realq_sweep(
+        orc = OracleSweep(lambda follow, grad_noise=None, W=Wf[nm], F=Ff[nm], Hs=Hs, Hg=Hg, w=w, b0=bstart: oracle.realq_sweep(
             W.astype(np.float64), Hs, T, group_size=64, block_size=64,
             bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": b0, "B_total": 1}, F=F,
-            obs_hessians=[(Hg[g], w[g]) for g in range(ng)], follow=follow))
+            obs_hessians=[(Hg[g], w[g]) for g in range(ng)], follow=follow, grad_noise=grad_noise))
         bstart += ins[i] // 64
         o = bq.out[nm]
         codes = unpack(o["codes"].cpu().numpy(), ins[i])
@@ -677,8 +677,8 @@ def test_minibatch_block_gd(start, steps):
     mbs = [oracle.hessian_sum([case.Xhat[k * Tm:(k + 1) * Tm]]) for k in range(K)]
     Hs, T = oracle.hessian_sum([case.Xhat])
     bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1, "minibatches": mbs}
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
-                                                        F=case.F, follow=follow))
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
+                                                        F=case.F, follow=follow, grad_noise=grad_noise))
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     H, _, _ = layer.accumulate([X], 384)
     prep = layer.prepare(H, T)
@@ -802,8 +802,8 @@ def test_token_block_gd_with_output_clipping(clip, start, steps):
     Hs, T = oracle.hessian_sum([case.Xhat])
     bgd = {"lr": 2e-4, "steps_per_block": steps, "b_global_start": start, "B_total": 1,
            "minibatch_tokens": parts, "a_loss_clip": clip}
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
-                                                        F=case.F, follow=follow))
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(case.W0, Hs, T, group_size=128, block_size=128, bgd=bgd,
+                                                        F=case.F, follow=follow, grad_noise=grad_noise))
     qkw = dict(group_size=128, block_size=128)
     X = bf16_dev(synth.f32_to_bf16_bits(case.Xhat))
     H, _, _ = layer.accumulate([X], 384)
@@ -837,11 +837,11 @@ def test_traced_block_losses(with_next):
     qkw = dict(group_size=64, block_size=64)
     kw = dict(b_global_start=3, B_total=9) if with_next else {}
     Hs, T = oracle.hessian_sum([case.Xhat])
-    orc = OracleSweep(lambda follow: oracle.realq_sweep(
+    orc = OracleSweep(lambda follow, grad_noise=None: oracle.realq_sweep(
         case.W0, Hs, T, group_size=64, block_size=64,
         bgd={"lr": 2e-4, "steps_per_block": 1, "b_global_start": kw.get("b_global_start", 1),
              "B_total": kw.get("B_total", 1)},
-        F=case.F, F_next=case.F_next if with_next else None, follow=follow))
+        F=case.F, F_next=case.F_next if with_next else None, follow=follow, grad_noise=grad_noise))
     H, _, T_ = layer.accumulate([dev(case.Xhat)], 320)
     prep = layer.prepare(H, T_)
     q = rq.quant_cfg(**qkw)
@@ -870,3 +870,30 @@ def test_traced_block_losses(with_next):
               f"after {got[blk, 1]:.6e} / {after:.6e}")
         assert abs(got[blk, 0] - before) <= 1e-3 * abs(before)
         assert abs(got[blk, 1] - after) <= 1e-3 * abs(after)
+
+
+# ------------------------------------------------- tensor-core tile shapes ---
+@pytest.mark.parametrize("tile", [1, 2])
+def test_tensor_tiles_match_the_oracle(tile):
+    # every tf32x3 product forced onto one output tile (1: 128 x 128 with
+    # 32-wide K slices, 2: 128 x 256 with 16-wide slices): the plain sweep with
+    # Block-GD on ragged shapes (M and N no multiple of either tile), the
+    # sliding window with perturbed inputs, the row-grouped sweep (the
+    # corrected gradient factor), mini-batch moments and the token form (the
+    # store epilogue and the K split)
+    rq.realq_set_tensor_tile(tile)
+    try:
+        case = synth.layer_case(24, 200, 300, 1500, outliers=2, dead_cols=(7,))
+        for qkw in (dict(group_size=64, block_size=64), dict(group_size=128, block_size=128)):
+            orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4)
+            _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=2e-4)
+        case = synth.layer_case(26, 96, 320, 1200, with_next=True, perturbed=True)
+        qkw = dict(group_size=64, block_size=64)
+        orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, with_next=True, b_global_start=3, B_total=9,
+                                             use_dbar=True)
+        _check(orc, out, case, qkw, True, lr=2e-4)
+        _grouped_run(56, 128, 384, 12000, 4, dict(group_size=128, block_size=128), lr=2e-4, correlated=True)
+        test_minibatch_block_gd(2, 2)
+        test_token_block_gd_with_output_clipping(0.95, 2, 2)
+    finally:
+        rq.realq_set_tensor_tile(0)

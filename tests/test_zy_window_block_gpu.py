@@ -259,8 +259,8 @@ def _oracle_sweep(c, module, opt, lr, steps, b_start, B_total, capture=None, nmb
     Hs, T = orq.hessian_sum([c["X"]])
     bgd = {"lr": lr, "steps_per_block": steps, "b_global_start": b_start, "B_total": B_total, "optimizer": opt,
            "gradient_fn": fn}
-    return OracleSweep(lambda follow: orq.realq_sweep(c["P"][ob._MODULE_WEIGHT[module]], Hs, T, bgd=bgd,
-                                                      follow=follow, **QKW))
+    return OracleSweep(lambda follow, grad_noise=None: orq.realq_sweep(c["P"][ob._MODULE_WEIGHT[module]], Hs, T, bgd=bgd,
+                                                      follow=follow, grad_noise=grad_noise, **QKW))
 
 
 def _gpu_sweep(c, module, opt, lr, steps, b_start, B_total, blocks=None, state=None, nmb=1):
