@@ -362,7 +362,7 @@ def work_models(wl, args=None):
         # D = X̂ᵀX̂ - XᵀX̂: the full non-symmetric product XᵀX̂ per input
         per_step["hessian_cross_tc"] = ("tensor", sum(2 * s.T * s.n * s.n for s in wl.inputs.values()), "TFLOP/s")
         per_step["act_quant"] = ("hbm", sum(s.T * s.n * 2 * 3 for s in wl.inputs.values()), "GB/s")
-    bgd_p = bgd_g = trail = 0
+    bgd_p = bgd_g = trail = trail_planes = 0
     serial_bytes = 0
     for md in wl.modules:
         m, n, B = md.m, md.n, wl.block_size
@@ -374,6 +374,10 @@ def work_models(wl, args=None):
             bgd_p += 2 * m * (n - b * B) * r if b > 0 else 0
             bgd_g += 2 * m * m * r
             trail += 2 * m * (be - b * B) * r
+            if r > 0:
+                # the update's operands as tf32 planes: read E_b and the U
+                # panel once, write both planes of each
+                trail_planes += 12 * (be - b * B) * (m + r)
             serial_bytes += m * (be - b * B) * (4 + 4 + 4) + m * (be - b * B) // 2
     if getattr(args, "a_loss_clip", None) and getattr(args, "minibatch_seqs", 0):
         # token-form gradient per optimizer step (every block but the last):
@@ -398,7 +402,8 @@ def work_models(wl, args=None):
         per_step["tok_grad_t"] = ("hbm", gt_b, "GB/s")
     per_step["bgd_p_gemm"] = ("tf32x3", bgd_p, "TFLOP/s")
     per_step["bgd_g_gemm_adam"] = ("tf32x3", bgd_g, "TFLOP/s")
-    per_step["trailing_update"] = ("alu", trail, "TFLOP/s")
+    per_step["trailing_update"] = ("tf32x3", trail, "TFLOP/s")
+    per_step["trailing_planes"] = ("hbm", trail_planes, "GB/s")
     per_step["quant_block"] = ("hbm", serial_bytes, "GB/s")
     prep_flops = sum(2 * s.n ** 3 // 3 for s in wl.inputs.values())
     per_step["chol_diag"] = ("alu", sum(s.n * 64 * 64 for s in wl.inputs.values()), "TFLOP/s")

@@ -511,6 +511,15 @@ void realq_graph_destroy(realq_graph_t graph);
  * Computed in fp32 with fp32 accumulation (the loss summed in double).
  * Asynchronous on `stream`; argument errors are returned before any launch.
  * S L is at most 4194240 tokens.  Outputs may not alias inputs. */
+/* Tuning: the output tile of the fp32-accurate (tf32x3) tensor-core
+ * products of Block-GD and the lazy batch update.  0 (default): chosen per
+ * launch from its grid (128 x 256 when its waves on the SMs take less time
+ * than 128 x 128's), 1: always 128 x 128, 2: always 128 x 256.  Results do
+ * not depend on it beyond the fp32 accumulation order of the tensor pipe.
+ * Process-wide; not for use while other threads launch.  REALQ_ERR_INVALID_ARG
+ * for other values.  No counterpart in the paper. */
+realq_status_t realq_set_tensor_tile(int mode);
+
 /* The learning rate of decoder block i (1-based) of L under the paper's
  * reverse-cosine schedule over transformer blocks (App. "Full Setup",
  * Eq. reverse_cosine; the first block's rate is 0.01 of the final one, App.

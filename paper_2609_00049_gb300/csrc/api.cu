@@ -799,6 +799,12 @@ realq_status_t realq_bgd_refine(realq_stream_t stream, int64_t m, int64_t n, int
     return bgd_step(S(stream), p, col_start, alpha);
 }
 
+realq_status_t realq_set_tensor_tile(int mode) {
+    if (mode < 0 || mode > 2) return fail(REALQ_ERR_INVALID_ARG, "set_tensor_tile: mode 0, 1 or 2");
+    tc_set_tile_mode(mode);
+    return REALQ_OK;
+}
+
 // ------------------------------------------------------------ schedules ---
 realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out) {
     if (!lr_out || L < 1 || i < 1 || i > L || !std::isfinite(lr_final))

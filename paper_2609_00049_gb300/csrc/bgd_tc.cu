@@ -39,17 +39,37 @@
 namespace realq {
 namespace {
 
-constexpr int TB = 128;                       // tile rows (M) and columns (N)
-constexpr int KS = 32;                        // fp32 elements per K slice (128 bytes)
-constexpr int STAGES = 3;
+constexpr int TB = 128;                       // tile rows (M)
 constexpr int THREADS = 256;                  // 8 warps; warp 0 lane 0 loads, warp 1 lane 0 issues MMAs
-constexpr int PLANE = TB * KS * 4;            // 16 KB
-constexpr int STAGE_BYTES = 4 * PLANE;        // A hi, A lo, B hi, B lo
-constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
-constexpr uint32_t IDESC = tc::idesc_tf32_f32(TB, TB);
+
+// Two tile shapes.  Each tcgen05.mma reads both operands from shared memory,
+// and the three products of a K step read A twice and B twice; with the TMA
+// writes of the ring that is about 190 bytes of shared-memory traffic per
+// cycle for a 128 x 128 tile at the tensor pipe's tf32 rate, above the
+// 128 bytes per cycle an SM serves, so that tile tops out near two thirds of
+// the pipe.  A 128 x 256 tile reuses each A row for twice the columns
+// (about 145 bytes per cycle): it takes 16-wide K slices (64-byte rows,
+// 64-byte swizzle) so that a 4-deep ring of both planes still fits.
+template <int TN>
+struct Tile {
+    static constexpr int KS = TN == 256 ? 16 : 32;            // fp32 per K slice
+    static constexpr int STAGES = TN == 256 ? 4 : 3;
+    static constexpr uint32_t SWZ = TN == 256 ? tc::SW_64B : tc::SW_128B;
+    static constexpr uint32_t SBO = TN == 256 ? 512 : 1024;   // 8 rows of one swizzle atom
+    static constexpr int PLANE_A = TB * KS * 4;
+    static constexpr int PLANE_B = TN * KS * 4;
+    static constexpr int STAGE_BYTES = 2 * PLANE_A + 2 * PLANE_B;   // A hi, A lo, B hi, B lo
+    static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
+    static constexpr uint32_t IDESC = tc::idesc_tf32_f32(TB, TN);
+    static_assert(STAGES * STAGE_BYTES >= TB * (TN + 1) * 4, "epilogue tile must fit the ring");
+};
 
 struct Maps {
     CUtensorMap a_hi, a_lo, b_hi, b_lo;
+};
+// (narrow: the 128 x 128 tile's boxes; wide: the 128 x 256 tile's)
+struct MapPair {
+    Maps narrow, wide;
 };
 
 // M += acc; p = M + lambda (A_disp - (W - W0)) (+ W0 Dbar), 0 on dead channels
@@ -233,11 +253,14 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
 }
 
 // MODE = e.mode, fixed at compile time: one kernel per epilogue (and so one
-// name per role in a profiler's launch list)
-template <int MODE>
+// name per role in a profiler's launch list); TN = the tile's width.
+template <int MODE, int TN>
 __global__ void __launch_bounds__(THREADS, 1)
     gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
                        int a_row0, const TcEpi e, int *err, int kchunk, int exact) {
+    using TL = Tile<TN>;
+    constexpr int KS = TL::KS, STAGES = TL::STAGES, PLANE_A = TL::PLANE_A, PLANE_B = TL::PLANE_B;
+    constexpr int STAGE_BYTES = TL::STAGE_BYTES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
@@ -247,7 +270,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TB;
+    const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TN;
     // K split over blockIdx.z: this CTA takes K range [kz0, kz0 + Kz)
     const int64_t kz0 = kchunk > 0 ? (int64_t)blockIdx.z * kchunk : 0;
     const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
@@ -266,7 +289,7 @@ __global__ void __launch_bounds__(THREADS, 1)
         tc::prefetch_tmap(&maps.b_hi);
         tc::prefetch_tmap(&maps.b_lo);
     }
-    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), TB);
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), TN);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
@@ -285,13 +308,13 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t fb = tc::smem_u32(&full[s]);
             // an operand exact in tf32 (exact & 1: A, exact & 2: B) has no
             // low plane to load or multiply
-            tc::mbar_arrive_expect_tx(fb, STAGE_BYTES - ((exact & 1) ? PLANE : 0) - ((exact & 2) ? PLANE : 0));
+            tc::mbar_arrive_expect_tx(fb, STAGE_BYTES - ((exact & 1) ? PLANE_A : 0) - ((exact & 2) ? PLANE_B : 0));
             const int x = k_off + (int)kz0 + it * KS;
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
             tc::tma_load_2d(base, &maps.a_hi, fb, x, a_row0 + (int)i0);
-            if (!(exact & 1)) tc::tma_load_2d(base + PLANE, &maps.a_lo, fb, x, a_row0 + (int)i0);
-            tc::tma_load_2d(base + 2 * PLANE, &maps.b_hi, fb, x, b_row0 + (int)j0);
-            if (!(exact & 2)) tc::tma_load_2d(base + 3 * PLANE, &maps.b_lo, fb, x, b_row0 + (int)j0);
+            if (!(exact & 1)) tc::tma_load_2d(base + PLANE_A, &maps.a_lo, fb, x, a_row0 + (int)i0);
+            tc::tma_load_2d(base + 2 * PLANE_A, &maps.b_hi, fb, x, b_row0 + (int)j0);
+            if (!(exact & 2)) tc::tma_load_2d(base + 2 * PLANE_A + PLANE_B, &maps.b_lo, fb, x, b_row0 + (int)j0);
         }
         if (*abort_flag) {
             int never = 0;
@@ -311,13 +334,14 @@ __global__ void __launch_bounds__(THREADS, 1)
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
 #pragma unroll
             for (int k = 0; k < KS / 8; ++k) {
-                const uint64_t ah = tc::smem_desc(base + k * 32, 16, 1024, tc::SW_128B);
-                const uint64_t al = tc::smem_desc(base + PLANE + k * 32, 16, 1024, tc::SW_128B);
-                const uint64_t bh = tc::smem_desc(base + 2 * PLANE + k * 32, 16, 1024, tc::SW_128B);
-                const uint64_t bl = tc::smem_desc(base + 3 * PLANE + k * 32, 16, 1024, tc::SW_128B);
-                tc::mma_tf32_ss(tmem, ah, bh, IDESC, (it > 0 || k > 0) ? 1u : 0u);
-                if (!(exact & 2)) tc::mma_tf32_ss(tmem, ah, bl, IDESC, 1u);
-                if (!(exact & 1)) tc::mma_tf32_ss(tmem, al, bh, IDESC, 1u);
+                // K step k: 8 fp32 = 32 bytes into every row of the swizzle atom
+                const uint64_t ah = tc::smem_desc(base + k * 32, 16, TL::SBO, TL::SWZ);
+                const uint64_t al = tc::smem_desc(base + PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
+                const uint64_t bh = tc::smem_desc(base + 2 * PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
+                const uint64_t bl = tc::smem_desc(base + 2 * PLANE_A + PLANE_B + k * 32, 16, TL::SBO, TL::SWZ);
+                tc::mma_tf32_ss(tmem, ah, bh, TL::IDESC, (it > 0 || k > 0) ? 1u : 0u);
+                if (!(exact & 2)) tc::mma_tf32_ss(tmem, ah, bl, TL::IDESC, 1u);
+                if (!(exact & 1)) tc::mma_tf32_ss(tmem, al, bh, TL::IDESC, 1u);
             }
             tc::mma_commit(tc::smem_u32(&empty[s]));
         }
@@ -333,15 +357,15 @@ __global__ void __launch_bounds__(THREADS, 1)
     const bool ok = nk == 0 || tc::mbar_wait(tc::smem_u32(accb), 0, abort_flag);
     tc::fence_after_sync();
     const bool good = __syncthreads_and(ok && !*abort_flag) != 0;
-    constexpr int TP = TB + 1;
+    constexpr int TP = TN + 1;
     float *T = reinterpret_cast<float *>(smem);
     if (good) {
         // warp w reads TMEM lanes 32 (w % 4) .. (its lane quarter), columns
-        // 64 (w / 4) ..
+        // TN/2 (w / 4) ..
         const int quarter = warp & 3, half = warp >> 2;
         const int row = quarter * 32 + lane;
 #pragma unroll 1
-        for (int c0 = half * (TB / 2); c0 < (half + 1) * (TB / 2); c0 += 32) {
+        for (int c0 = half * (TN / 2); c0 < (half + 1) * (TN / 2); c0 += 32) {
             uint32_t v[32];
             if (nk > 0) {
                 tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)c0, v);
@@ -355,33 +379,37 @@ __global__ void __launch_bounds__(THREADS, 1)
     }
     __syncthreads();
     if (good) {
-        // rows of the tile, each lane on 4 consecutive columns; the loads of
-        // 4 rows are issued before any store so they overlap
+        // rows of the tile, each lane on 4 consecutive columns of a 128-wide
+        // column half; the loads of 4 rows are issued before any store so
+        // they overlap
         constexpr int RPW = TB / (THREADS / 32);   // tile rows per warp
-        const int cc = lane * 4;
-        const int64_t gj = j0 + cc;
-        const bool vec = MODE != TC_STORE && gj + 3 < N;
-        for (int rb = warp * RPW; rb < warp * RPW + RPW; rb += 4) {
-            if (i0 + rb >= M) break;
-            // a batch of 4 rows runs vectorized when all 4 exist (M need not be
-            // a multiple of 4 for a row group)
-            if (vec && i0 + rb + 3 < M) {
-                if (MODE == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
-                else if (MODE == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
-                else if (MODE == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
-                else accum_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
-            } else {
-                for (int u = 0; u < 4; ++u) {
-                    const int rr = rb + u;
-                    const int64_t gi = i0 + rr;
-                    if (gi >= M) break;
-                    for (int q = 0; q < 4; ++q) {
-                        if (gj + q >= N) break;
-                        float &t = T[rr * TP + cc + q];
-                        if (MODE == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
-                        else if (MODE == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
-                        else if (MODE == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
-                        else epi_apply(e, gi, gj + q, t);
+#pragma unroll 1
+        for (int ch = 0; ch < TN; ch += 128) {
+            const int cc = ch + lane * 4;
+            const int64_t gj = j0 + cc;
+            const bool vec = MODE != TC_STORE && gj + 3 < N;
+            for (int rb = warp * RPW; rb < warp * RPW + RPW; rb += 4) {
+                if (i0 + rb >= M) break;
+                // a batch of 4 rows runs vectorized when all 4 exist (M need
+                // not be a multiple of 4 for a row group)
+                if (vec && i0 + rb + 3 < M) {
+                    if (MODE == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                    else if (MODE == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
+                    else if (MODE == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
+                    else accum_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
+                } else {
+                    for (int u = 0; u < 4; ++u) {
+                        const int rr = rb + u;
+                        const int64_t gi = i0 + rr;
+                        if (gi >= M) break;
+                        for (int q = 0; q < 4; ++q) {
+                            if (gj + q >= N) break;
+                            float &t = T[rr * TP + cc + q];
+                            if (MODE == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
+                            else if (MODE == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
+                            else if (MODE == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
+                            else epi_apply(e, gi, gj + q, t);
+                        }
                     }
                 }
             }
@@ -390,7 +418,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     __syncthreads();
     if (good && (MODE == TC_BGD_P || MODE == TC_BGD_PG)) {
         // columns of the tile, lanes over rows: P^T rows are contiguous
-        constexpr int CPW = TB / (THREADS / 32);   // tile columns per warp
+        constexpr int CPW = TN / (THREADS / 32);   // tile columns per warp
         for (int cc = warp * CPW; cc < warp * CPW + CPW; ++cc) {
             const int64_t gj = j0 + cc;
             if (gj >= N) break;
@@ -407,7 +435,7 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (!good && threadIdx.x == 0 && err) atomicOr(err, ST_TIMEOUT);
     tc::fence_before_sync();
     __syncthreads();
-    if (warp == 0) tc::tmem_dealloc(tmem, TB);
+    if (warp == 0) tc::tmem_dealloc(tmem, TN);
 }
 
 // g = sum over the K splits (z = 0, 1, ... in order), then the TC_ADAM
@@ -440,6 +468,55 @@ __global__ void split_kernel(int64_t count, const float *x, const float *y, floa
     const float h = tc::tf32_hi(v);
     hi[i] = h;
     lo[i] = v - h;
+}
+
+// The lazy batch update's operands as K-major planes (tc_trail_planes): tile
+// t < te of a 32 x 32 tiling transposes E (Et[k][i] -> -E[i][k]), the others
+// the U panel (U[bs + k][be + j] -> P[j][k]); kt = kb / 32 tiles along k.
+__global__ void trail_planes_kernel(int64_t m, int64_t ldet, const float *Et, int64_t n, const float *U, int64_t bs,
+                                    int64_t be, int kt, int B, int64_t te, float *Eh, float *El, float *Ph,
+                                    float *Pl) {
+    __shared__ float tile[32][33];
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    int64_t t = blockIdx.x;
+    if (t < te) {
+        const int64_t ti = t / kt;
+        const int tk = (int)(t % kt);
+        const int64_t i = ti * 32 + tx;
+#pragma unroll
+        for (int q = 0; q < 32; q += 8) tile[ty + q][tx] = i < m ? Et[(int64_t)(tk * 32 + ty + q) * ldet + i] : 0.f;
+        __syncthreads();
+#pragma unroll
+        for (int q = 0; q < 32; q += 8) {
+            const int64_t r = ti * 32 + ty + q;
+            if (r < m) {
+                const float v = -tile[tx][ty + q];
+                const float h = tc::tf32_hi(v);
+                Eh[r * B + tk * 32 + tx] = h;
+                El[r * B + tk * 32 + tx] = v - h;
+            }
+        }
+        return;
+    }
+    t -= te;
+    const int64_t rcols = n - be;
+    const int64_t tj = t / kt;
+    const int tk = (int)(t % kt);
+    const int64_t j = tj * 32 + tx;
+#pragma unroll
+    for (int q = 0; q < 32; q += 8)
+        tile[ty + q][tx] = j < rcols ? U[(bs + tk * 32 + ty + q) * n + be + j] : 0.f;
+    __syncthreads();
+#pragma unroll
+    for (int q = 0; q < 32; q += 8) {
+        const int64_t c = tj * 32 + ty + q;
+        if (c < rcols) {
+            const float v = tile[tx][ty + q];
+            const float h = tc::tf32_hi(v);
+            Ph[c * B + tk * 32 + tx] = h;
+            Pl[c * B + tk * 32 + tx] = v - h;
+        }
+    }
 }
 
 // hi / lo planes of x - y (y fp32 or bf16)
@@ -482,6 +559,22 @@ realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const flo
     return check_launch("tf32_split");
 }
 
+realq_status_t tc_trail_planes(cudaStream_t s, int64_t m, const float *Et, int64_t ldet, int64_t n, const float *U,
+                               int64_t bs, int64_t be, int kb, int B, float *Eh, float *El, float *Ph, float *Pl) {
+    if (kb <= 0 || kb % 32 != 0 || kb > B || be > n || bs + kb > n)
+        return fail(REALQ_ERR_INVALID_ARG, "trailing planes: bad block (%d of %d at %lld)", kb, B, (long long)bs);
+    const int kt = kb / 32;
+    const int64_t te = Et ? ceil_div(m, 32) * kt : 0;
+    const int64_t tp = ceil_div(n - be, 32) * kt;
+    if (te + tp <= 0) return REALQ_OK;
+    {
+        Launch L("trailing_planes", s);
+        trail_planes_kernel<<<(unsigned)(te + tp), dim3(32, 8), 0, s>>>(m, ldet, Et, n, U, bs, be, kt, B, te, Eh, El,
+                                                                         Ph, Pl);
+    }
+    return check_launch("trailing_planes");
+}
+
 realq_status_t tc_gsum_adam(cudaStream_t s, int64_t m, int64_t N, int nz, const float *part, const TcEpi &e) {
     if (m <= 0 || N <= 0) return REALQ_OK;
     {
@@ -494,59 +587,104 @@ realq_status_t tc_gsum_adam(cudaStream_t s, int64_t m, int64_t N, int nz, const 
 realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb) {
-    static_assert(sizeof(Maps) <= sizeof(TcMaps), "map storage");
-    Maps *m = reinterpret_cast<Maps *>(out->storage);
-    CUresult r = encode_tmap_2d_f32(&m->a_hi, a_hi, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, KS, TB, 1);
-    if (r == CUDA_SUCCESS)
-        r = encode_tmap_2d_f32(&m->a_lo, a_lo, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, KS, TB, 1);
-    if (r == CUDA_SUCCESS)
-        r = encode_tmap_2d_f32(&m->b_hi, b_hi, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, KS, TB, 1);
-    if (r == CUDA_SUCCESS)
-        r = encode_tmap_2d_f32(&m->b_lo, b_lo, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, KS, TB, 1);
+    static_assert(sizeof(MapPair) <= sizeof(TcMaps), "map storage");
+    MapPair *mp = reinterpret_cast<MapPair *>(out->storage);
+    CUresult r = CUDA_SUCCESS;
+    // narrow: 32-wide K slices with 128-byte swizzle, 128-row boxes;
+    // wide: 16-wide slices with 64-byte swizzle, B boxes of 256 rows
+    for (int w = 0; w < 2 && r == CUDA_SUCCESS; ++w) {
+        Maps *m = w ? &mp->wide : &mp->narrow;
+        const uint32_t ks = w ? Tile<256>::KS : Tile<128>::KS, bn = w ? 256 : 128;
+        const int swz = w ? 2 : 1;
+        r = encode_tmap_2d_f32(&m->a_hi, a_hi, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, ks, TB, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f32(&m->a_lo, a_lo, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 4, ks, TB, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f32(&m->b_hi, b_hi, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, ks, bn, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f32(&m->b_lo, b_lo, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, ks, bn, swz);
+    }
     if (r != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled (tf32 planes) failed (%d)", (int)r);
     return REALQ_OK;
 }
+
+namespace {
+template <int TN>
+realq_status_t launch_tf32x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
+                             const TcEpi &e, int *err, int a_row0, int kchunk, int exact) {
+    constexpr int SM = Tile<TN>::SMEM;
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_STORE, TN>), SM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_P, TN>), SM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ADAM, TN>), SM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ACCUM, TN>), SM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_PG, TN>), SM));
+    const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
+    const dim3 grid((unsigned)ceil_div(N, TN), (unsigned)ceil_div(M, TB), nz);
+    switch (e.mode) {
+        case TC_STORE:
+            gemm_tf32x3_kernel<TC_STORE, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                       kchunk, exact);
+            break;
+        case TC_BGD_P:
+            gemm_tf32x3_kernel<TC_BGD_P, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                       kchunk, exact);
+            break;
+        case TC_ADAM:
+            gemm_tf32x3_kernel<TC_ADAM, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                      kchunk, exact);
+            break;
+        case TC_ACCUM:
+            gemm_tf32x3_kernel<TC_ACCUM, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                       kchunk, exact);
+            break;
+        default:
+            gemm_tf32x3_kernel<TC_BGD_PG, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                        kchunk, exact);
+            break;
+    }
+    return REALQ_OK;
+}
+
+int g_tile_mode = 0;   // 0: by the grid (wide_tiles_pay), 1: always 128 x 128, 2: always 128 x 256
+
+// The 128 x 256 tile does twice a narrow tile's work in about 1.55 narrow
+// tile times (its measured rate over the narrow one's, at the shared-memory
+// bound above); it pays when that beats the narrow grid's waves on the SMs.
+bool wide_tiles_pay(int64_t M, int64_t N, unsigned nz) {
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0, c = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && c > 0)
+            sms = c;
+        else
+            return false;
+    }
+    const int64_t rows = ceil_div(M, TB) * (int64_t)nz;
+    const int64_t waves_n = ceil_div(rows * ceil_div(N, 128), sms);
+    const int64_t waves_w = ceil_div(rows * ceil_div(N, 256), sms);
+    return 155 * waves_w < 100 * waves_n;
+}
+}  // namespace
+
+void tc_set_tile_mode(int mode) { g_tile_mode = mode; }
 
 realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
                               int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk,
                               int exact) {
     if (M <= 0 || N <= 0) return REALQ_OK;
     if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
-    if (kchunk < 0 || (kchunk % KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
-        return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name, KS);
+    if (kchunk < 0 || (kchunk % Tile<128>::KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name,
+                    Tile<128>::KS);
     if (e.mode < TC_STORE || e.mode > TC_BGD_PG) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_STORE>), SMEM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_P>), SMEM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ADAM>), SMEM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ACCUM>), SMEM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_PG>), SMEM));
-    const Maps &m = *reinterpret_cast<const Maps *>(maps.storage);
+    const MapPair &mp = *reinterpret_cast<const MapPair *>(maps.storage);
+    const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
+    const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));
     {
         Launch L(name, s);
-        const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
-        const dim3 grid((unsigned)ceil_div(N, TB), (unsigned)ceil_div(M, TB), nz);
-        switch (e.mode) {
-            case TC_STORE:
-                gemm_tf32x3_kernel<TC_STORE><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                         kchunk, exact);
-                break;
-            case TC_BGD_P:
-                gemm_tf32x3_kernel<TC_BGD_P><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                         kchunk, exact);
-                break;
-            case TC_ADAM:
-                gemm_tf32x3_kernel<TC_ADAM><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                        kchunk, exact);
-                break;
-            case TC_ACCUM:
-                gemm_tf32x3_kernel<TC_ACCUM><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                         kchunk, exact);
-                break;
-            default:
-                gemm_tf32x3_kernel<TC_BGD_PG><<<grid, THREADS, SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                          kchunk, exact);
-                break;
-        }
+        if (wide) REALQ_TRY(launch_tf32x3<256>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact));
+        else REALQ_TRY(launch_tf32x3<128>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact));
     }
     return check_launch(name);
 }

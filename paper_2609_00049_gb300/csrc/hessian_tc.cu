@@ -313,7 +313,8 @@ static CUresult encode_tmap_2d(CUtensorMapDataType dt, CUtensorMap *map, const v
     cuuint32_t estr[2] = {1, 1};
     return g_encode(map, dt, 2, const_cast<void *>(base), dims, strides, box, estr,
                     CU_TENSOR_MAP_INTERLEAVE_NONE,
-                    swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE,
+                    swizzle128 == 2 ? CU_TENSOR_MAP_SWIZZLE_64B
+                                    : (swizzle128 ? CU_TENSOR_MAP_SWIZZLE_128B : CU_TENSOR_MAP_SWIZZLE_NONE),
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 

@@ -63,10 +63,21 @@ struct TcEpi {
     float lr, b1, b2, eps, bc1, bc2; int sgd;
     int64_t czs;                                             // TC_STORE with a K split: C of split z at C + z czs
 };
+// The operand maps of one product, for both tile shapes of the kernel
+// (128 x 128 outputs with 32-wide K slices, 128 x 256 with 16-wide slices).
 struct TcMaps {
-    alignas(64) unsigned char storage[4 * 128];
+    alignas(64) unsigned char storage[8 * 128];
 };
 bool tc_gemm_eligible(int64_t m, int64_t n);
+// Tile shape of the tf32x3 products: 0 chosen per launch by its grid, 1 always
+// 128 x 128, 2 always 128 x 256 (process-wide).
+void tc_set_tile_mode(int mode);
+// The operands of the lazy batch update W[:, be:] -= E_b U[bs:be, be:] as
+// K-major tf32 planes: Eh/El = hi/lo of -E_b (m x B, from Et, kb x m with
+// leading dimension ldet; skipped when Et is NULL), Ph/Pl = hi/lo of
+// U[bs + k, be + j] (r x B, r = n - be).  kb a multiple of 32, <= B.
+realq_status_t tc_trail_planes(cudaStream_t s, int64_t m, const float *Et, int64_t ldet, int64_t n, const float *U,
+                               int64_t bs, int64_t be, int kb, int B, float *Eh, float *El, float *Ph, float *Pl);
 realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const float *y, float alpha, float *hi,
                         float *lo);
 realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
@@ -157,6 +168,11 @@ struct SweepPlan {
     int *status;
     float *lam;
     float *Et, *P, *G, *Feff, *R0;
+    // the lazy batch update on the tensor cores (tf32x3): planes of -E_b
+    // (m x block) and of the block's U panel transposed (n x block)
+    int trail_tc = 0, trail_maps = 0;
+    float *Eh = nullptr, *El = nullptr, *UPh = nullptr, *UPl = nullptr;
+    TcMaps mapsTr;
     // tensor-core path: hi / lo planes and tensor maps
     int tc;
     float *Sh, *Sl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;

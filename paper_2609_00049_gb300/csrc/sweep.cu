@@ -390,11 +390,20 @@ realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
 // and need hi / lo planes of the displacement, H̄, F and P^T; otherwise the
 // fp32 SIMT path needs P, G (and F_eff).  block = 0: Block-GD only (literal
 // gradient form, SIMT).
+// The lazy batch update runs on the tensor cores (tf32x3) when both GEMM
+// operands take the tensor-core path's shapes and the block is a whole
+// number of 32-wide K slices.
+static bool trail_tc_eligible(int64_t m, int64_t n, int block) {
+    return (block == 32 || block == 64 || block == 128) && tc_gemm_eligible(m, n);
+}
+
 size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnext, int has_dbar, int rgroups,
                       int nmb, int64_t tmb) {
     const size_t mn = align_up((size_t)m * n * sizeof(float));
     const size_t nn = align_up((size_t)n * n * sizeof(float));
     size_t b = align_up(sizeof(int)) + align_up(sizeof(float)) + align_up((size_t)block * m * sizeof(float));
+    if (trail_tc_eligible(m, n, block))
+        b += 2 * align_up((size_t)block * m * sizeof(float)) + 2 * align_up((size_t)block * n * sizeof(float));
     if (rgroups > 0) b += align_up((size_t)rgroups * sizeof(float));
     if (has_bgd) {
         if (block > 0 && tc_gemm_eligible(m, n)) {
@@ -425,6 +434,15 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
     p.status = cv.take<int>(1);
     p.lam = cv.take<float>(1);
     p.Et = cv.take<float>((size_t)p.block * p.m);
+    p.trail_tc = trail_tc_eligible(p.m, p.n, p.block) ? 1 : 0;
+    p.trail_maps = 0;
+    p.Eh = p.El = p.UPh = p.UPl = nullptr;
+    if (p.trail_tc) {
+        p.Eh = cv.take<float>((size_t)p.block * p.m);
+        p.El = cv.take<float>((size_t)p.block * p.m);
+        p.UPh = cv.take<float>((size_t)p.block * p.n);
+        p.UPl = cv.take<float>((size_t)p.block * p.n);
+    }
     p.P = p.G = p.Feff = p.R0 = nullptr;
     p.Sh = p.Sl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = p.M = nullptr;
     p.HGh = p.HGl = p.GGh = p.GGl = p.DWh = p.DWl = p.MBh = p.MBl = nullptr;
@@ -884,8 +902,29 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
     REALQ_TRY(sweep_join_wide(s, p));
     if (be >= p.n) return REALQ_OK;
     // lazy batch update of every later column: W[:, be:] -= E_b U[bs:be, be:]
-    // (per row group with its own U)
-    for (int gr = 0; gr < p.rgroups; ++gr) {
+    // (per row group with its own U).  On the tensor cores: the planes of -E_b
+    // and of the U panel, then W[:, be:] += (-E_b) U[bs:be, be:] as a tf32x3
+    // product accumulated into W.
+    if (p.trail_tc) {
+        if (!p.trail_maps) {
+            REALQ_TRY(tc_make_maps(&p.mapsTr, p.Eh, p.El, p.m, B, B, p.UPh, p.UPl, p.n, B, B));
+            p.trail_maps = 1;
+        }
+        for (int gr = 0; gr < p.rgroups; ++gr) {
+            const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
+            if (rows <= 0) break;
+            REALQ_TRY(tc_trail_planes(s, p.m, gr == 0 ? p.Et : nullptr, p.m, p.n, p.Ug + (size_t)gr * p.n * p.n, bs,
+                                      be, kb, B, p.Eh, p.El, p.UPh, p.UPl));
+            TcEpi e{};
+            e.mode = TC_ACCUM;
+            e.M = p.W + row0 * p.n;
+            e.ldw = p.n;
+            e.col0 = be;
+            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsTr, rows, p.n - be, kb, 0, 0, e, p.status, "trailing_update",
+                                     (int)row0));
+        }
+    }
+    for (int gr = 0; gr < p.rgroups && !p.trail_tc; ++gr) {
         const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
         if (rows <= 0) break;
         GemmArgs g{};

@@ -92,7 +92,7 @@ __device__ __forceinline__ void fence_before_sync() { asm volatile("tcgen05.fenc
 __device__ __forceinline__ void fence_after_sync() { asm volatile("tcgen05.fence::after_thread_sync;" ::: "memory"); }
 
 // ---- descriptors ----
-enum : uint32_t { SW_NONE = 0, SW_128B = 2 };
+enum : uint32_t { SW_NONE = 0, SW_128B = 2, SW_64B = 4 };
 
 // Shared-memory matrix descriptor: start address, leading / stride byte
 // offsets (the two strides of the canonical layout), version 1, swizzle mode.
@@ -115,7 +115,8 @@ __host__ __device__ constexpr uint32_t idesc_bf16_f32(uint32_t M, uint32_t N, ui
            | (a_mn << 15) | (b_mn << 16) | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
-// kind::tf32 with fp32 accumulation, both operands K-major.
+// kind::tf32 with fp32 accumulation, both operands K-major (M = 128,
+// N a multiple of 16 up to 256).
 __host__ __device__ constexpr uint32_t idesc_tf32_f32(uint32_t M, uint32_t N) {
     return (1u << 4)            // D format: f32
            | (2u << 7)          // A format: tf32
@@ -181,7 +182,8 @@ __device__ __forceinline__ void tmem_ld_32x32b_x32(uint32_t taddr, uint32_t (&r)
 // Host: tensor-map encoders from the driver (no link-time libcuda dependency).
 CUresult encode_tmap_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
                              uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128);
+// swizzle: 0 none, 1 128-byte, 2 64-byte
 CUresult encode_tmap_2d_f32(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
-                            uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128);
+                            uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle);
 
 }  // namespace realq
