@@ -84,7 +84,7 @@ def probe_eta(m: int, n: int) -> float:
 
 
 def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: float = 1e-3,
-                plain_first: bool = True):
+                plain_first: bool = True, gpu_scale: np.ndarray = None, rtol: float = 1e-5):
     """run(follow[, grad_noise]) -> an oracle sweep result (oracle.realq_sweep
     with that follow).
 
@@ -96,7 +96,9 @@ def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: fl
     n_conditioned, every other one as unexplained.  Returns (plain result,
     followed result, report); the report carries the plain comparison
     (plain_frac_equal, plain_n_mismatch), the decisions followed, and the
-    probes' per-group moves of the scales as fol["probe_scale_move"].
+    probes' per-group moves of the scales as fol["probe_scale_move"] (the
+    probes also run when gpu_scale is given and a scale differs from the
+    followed run's by more than rtol).
     plain_first=False skips the plain run (where the oracle is slow): the
     oracle runs once, with the follow, and the plain entries are None."""
     if plain_first:
@@ -104,20 +106,23 @@ def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: fl
         rep0 = code_report(gpu_codes, plain, gpu_zero, tau)
     else:
         plain, rep0 = None, {"frac_equal": None, "n_mismatch": None, "n_zero_mismatch": None}
-    if plain_first and rep0["n_mismatch"] == 0 and rep0["n_zero_mismatch"] == 0:
-        rep0.update(plain_frac_equal=rep0["frac_equal"], plain_n_mismatch=0, n_followed=0, n_followed_zero=0,
-                    n_unexplained=0, n_conditioned=0)
-        return plain, plain, rep0
     follow = {"codes": np.asarray(gpu_codes, dtype=np.int64),
               "zero": None if gpu_zero is None else np.asarray(gpu_zero, dtype=np.int64), "tau": tau}
-    fol = run(follow)
+    if plain_first and rep0["n_mismatch"] == 0 and rep0["n_zero_mismatch"] == 0:
+        fol = plain
+    else:
+        fol = run(follow)
     rep = code_report(gpu_codes, fol, gpu_zero, tau)
     rep.update(plain_frac_equal=rep0["frac_equal"], plain_n_mismatch=rep0["n_mismatch"],
                n_followed=int(fol["n_followed"]), n_followed_zero=int(fol["n_followed_zero"]), n_conditioned=0)
     mism = gpu_codes != fol["codes"]
     zmism = np.zeros_like(fol["zero"], dtype=bool) if gpu_zero is None else \
         np.asarray(gpu_zero, dtype=np.int64) != fol["zero"]
-    if mism.any() or zmism.any():
+    scale_off = False
+    if gpu_scale is not None:
+        so = fol["scale"].astype(np.float64)
+        scale_off = bool((np.abs(np.asarray(gpu_scale, dtype=np.float64) - so) > rtol * np.abs(so)).any())
+    if mism.any() or zmism.any() or scale_off:
         m, n = gpu_codes.shape
         eta = probe_eta(m, n)
         dx = np.zeros((m, n))
@@ -176,14 +181,17 @@ def adam_scale_bound(orc_scale: np.ndarray, n: int, qkw: dict, lr: float, steps:
     return np.broadcast_to(4.0 * lr * taken / maxq + 1e-12, orc_scale.shape)
 
 
-def check_codes_and_scales(orc, codes, zero, scale, n, qkw, bgd, lr=0.0, steps=1, what="", plain_first=True):
+def check_codes_and_scales(orc, codes, zero, scale, n, qkw, bgd, lr=0.0, steps=1, what="", plain_first=True,
+                           probe_scales=True):
     """The codes bar on the CUDA path's branch (follow_ties: >= 99.9 %
     identical, none unexplained, decisions the arithmetic does not
     determine at most 1e-5 of the codes plus one) and the scales within 1e-5
     relative, apart from groups within the probes' move and groups within
     the Adam-sign allowance of reading R18 (counted; at most 0.1 % of the
-    groups plus one).  Returns (plain, followed, report)."""
-    plain, fol, rep = follow_ties(orc, codes, zero, plain_first=plain_first)
+    groups plus one).  probe_scales=False runs the probes for codes only
+    (where the oracle is slow).  Returns (plain, followed, report)."""
+    plain, fol, rep = follow_ties(orc, codes, zero, plain_first=plain_first,
+                                  gpu_scale=scale if probe_scales else None)
     frac, med, s_bad, s_allow = scale_agreement(scale, fol["scale"],
                                                 adam_bound=adam_scale_bound(fol["scale"], n, qkw, lr, steps)
                                                 if bgd else None, probe_move=fol.get("probe_scale_move"))

@@ -161,7 +161,8 @@ def test_sweeps_against_the_oracle(shape_run, oracle_H):
         # (one oracle run, on the CUDA path's branch at rounding ties)
         _, fol, rep = check_codes_and_scales(orc, codes, o["zero"].cpu().numpy(), o["scale"].cpu().numpy(),
                                              md.n, qkw, True, wl.lr, wl.steps_per_block,
-                                             f"{wl.name} {md.name} {md.m}x{md.n} ", plain_first=False)
+                                             f"{wl.name} {md.name} {md.m}x{md.n} ", plain_first=False,
+                                             probe_scales=False)
         assert o["adam_t"] == fol["adam_t"] == (nb - 1) * wl.steps_per_block
         # the surrogate (Eq. fisher_loss at the layer level, the last block's
         # F_eff): the CUDA path's own value of its output against the
