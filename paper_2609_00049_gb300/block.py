@@ -48,6 +48,14 @@ from . import (BLOCK_MODULES, REALQ_BF16, REALQ_OPT_ADAM, QuantCfg, bgd_cfg, rea
                realq_scale_moment, realq_workspace_status, workspace)
 
 
+def _prepare_ws(n: int, dev) -> torch.Tensor:
+    """A preparation workspace whose status words read as "no failure" (the
+    failing column -1, no timeout) before the first preparation."""
+    ws = workspace(realq_prepare_workspace_size(n), dev).zero_()
+    ws[:4].fill_(0xFF)
+    return ws
+
+
 @dataclass
 class BlockInput:
     """Calibration input X̂ of T tokens and n channels (token-major)."""
@@ -131,7 +139,7 @@ class BlockQuantizer:
             self.state[name] = dict(
                 H=torch.empty(n, n, device=dev), U=torch.empty(n, n, device=dev), Hbar=torch.empty(n, n, device=dev),
                 dead=torch.empty(n, dtype=torch.uint8, device=dev),
-                pws=workspace(realq_prepare_workspace_size(n), dev).fill_(0xFF),  # status word -1: no failure
+                pws=_prepare_ws(n, dev),
                 hws=workspace(realq_hessian_workspace_size(n, spec.T, REALQ_BF16, act_quant is not None), dev))
             if minibatch_tokens and a_loss_clip is None:
                 nmb = -(-spec.T // minibatch_tokens)

@@ -313,12 +313,14 @@ realq_status_t realq_hessian_prepare_deferred(realq_stream_t stream, int64_t n, 
 }
 
 realq_status_t realq_prepare_status(realq_stream_t stream, void *ws, size_t ws_bytes, int64_t *fail_col) {
-    if (!ws || ws_bytes < sizeof(int) || !fail_col) return fail(REALQ_ERR_INVALID_ARG, "prepare_status: bad argument");
-    int st = -1;
-    REALQ_CUDA_TRY(cudaMemcpyAsync(&st, ws, sizeof(int), cudaMemcpyDeviceToHost, S(stream)));
+    if (!ws || ws_bytes < 2 * sizeof(int) || !fail_col)
+        return fail(REALQ_ERR_INVALID_ARG, "prepare_status: bad argument");
+    int st[2] = {-1, 0};
+    REALQ_CUDA_TRY(cudaMemcpyAsync(st, ws, 2 * sizeof(int), cudaMemcpyDeviceToHost, S(stream)));
     REALQ_CUDA_TRY(cudaStreamSynchronize(S(stream)));
-    *fail_col = st;
-    if (st >= 0) return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", st);
+    *fail_col = st[0];
+    if (st[1] & ST_TIMEOUT) return fail(REALQ_ERR_TIMEOUT, "a bounded device-side wait gave up (prepare)");
+    if (st[0] >= 0) return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", st[0]);
     return REALQ_OK;
 }
 

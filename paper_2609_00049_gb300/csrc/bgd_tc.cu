@@ -24,6 +24,9 @@
 //             moments and the displacement, and writing the step's hi / lo
 //             planes for the next M update
 //   TC_ACCUM  M += acc (the running product of one row group)
+//   TC_SYRK   M[i][j] -= acc for j >= i only (a symmetric rank-K update of
+//             the upper triangle of M; tiles wholly below the diagonal exit
+//             at once)
 //   TC_BGD_PG the gradient factor of a row group whose OBS used its own
 //             H̄_g:  p = M + lambda_g (A_disp - (W - W0)) - acc (+ W0 Dbar),
 //             acc = ΔW (H̄_g - H̄); written like TC_BGD_P
@@ -180,6 +183,21 @@ __device__ __forceinline__ void accum_rows4(const TcEpi &e, int64_t gi0, int64_t
     }
 }
 
+// TC_SYRK for 4 rows x 4 columns: M -= acc on and above the diagonal
+__device__ __forceinline__ void syrk_rows4(const TcEpi &e, int64_t gi0, int64_t gj, const float *t, int tp) {
+    float4 mp[4];
+#pragma unroll
+    for (int u = 0; u < 4; ++u) mp[u] = ld4(e.M + (gi0 + u) * e.ldw + gj);
+#pragma unroll
+    for (int u = 0; u < 4; ++u) {
+        const float *tr = t + u * tp;
+        const int64_t gi = gi0 + u;
+        st4(e.M + gi * e.ldw + gj,
+            make_float4(gj + 0 >= gi ? mp[u].x - tr[0] : mp[u].x, gj + 1 >= gi ? mp[u].y - tr[1] : mp[u].y,
+                        gj + 2 >= gi ? mp[u].z - tr[2] : mp[u].z, gj + 3 >= gi ? mp[u].w - tr[3] : mp[u].w));
+    }
+}
+
 __device__ __forceinline__ float adam_step(const TcEpi &e, float g, float &m, float &v) {
     if (e.sgd) return e.lr * g;
     m = e.b1 * m + (1.f - e.b1) * g;
@@ -232,6 +250,10 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
         e.M[i * e.ldw + e.col0 + j] += v;
         return;
     }
+    if (e.mode == TC_SYRK) {
+        if (j >= i) e.M[i * e.ldw + j] -= v;
+        return;
+    }
     const int64_t col = e.col0 + j;
     const int64_t w = i * e.ldw + col;
     // TC_ADAM
@@ -271,9 +293,16 @@ __global__ void __launch_bounds__(THREADS, 1)
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TN;
+    // a symmetric update touches the upper triangle only: a tile wholly
+    // below the diagonal has nothing to do (uniform over the CTA, before any
+    // barrier or allocation)
+    if (MODE == TC_SYRK && j0 + TN <= i0) return;
     // K split over blockIdx.z: this CTA takes K range [kz0, kz0 + Kz)
     const int64_t kz0 = kchunk > 0 ? (int64_t)blockIdx.z * kchunk : 0;
-    const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+    int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+    // a triangular B (zero beyond the output column): this tile's K range
+    // ends at its last column (the wrapper takes no K split with it)
+    if (e.b_tri && Kz > j0 + TN) Kz = j0 + TN;
     const int nk = (int)((Kz + KS - 1) / KS);
 
     if (threadIdx.x == 0) {
@@ -396,6 +425,7 @@ __global__ void __launch_bounds__(THREADS, 1)
                     if (MODE == TC_ADAM) adam_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
                     else if (MODE == TC_BGD_P) bgd_p_rows4(e, i0 + rb, M, gj, T + rb * TP + cc, TP);
                     else if (MODE == TC_BGD_PG) bgd_pg_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
+                    else if (MODE == TC_SYRK) syrk_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
                     else accum_rows4(e, i0 + rb, gj, T + rb * TP + cc, TP);
                 } else {
                     for (int u = 0; u < 4; ++u) {
@@ -559,6 +589,69 @@ realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const flo
     return check_launch("tf32_split");
 }
 
+namespace {
+// dst[c * ldd + r] = planes of src[r * lds + c], 32 x 32 tiles through shared memory
+__global__ void trans_planes_kernel(int64_t rows, int64_t cols, const float *src, int64_t lds, float *dh, float *dl,
+                                    int64_t ldd, int64_t tiles_c) {
+    __shared__ float tile[32][33];
+    const int tx = threadIdx.x, ty = threadIdx.y;
+    const int64_t tr = blockIdx.x / tiles_c, tcol = blockIdx.x % tiles_c;
+    const int64_t c = tcol * 32 + tx;
+#pragma unroll
+    for (int q = 0; q < 32; q += 8) {
+        const int64_t r = tr * 32 + ty + q;
+        tile[ty + q][tx] = (r < rows && c < cols) ? src[r * lds + c] : 0.f;
+    }
+    __syncthreads();
+    const int64_t r = tr * 32 + tx;
+#pragma unroll
+    for (int q = 0; q < 32; q += 8) {
+        const int64_t cc = tcol * 32 + ty + q;
+        if (cc < cols && r < rows) {
+            const float v = tile[tx][ty + q];
+            const float h = tc::tf32_hi(v);
+            dh[cc * ldd + r] = h;
+            dl[cc * ldd + r] = v - h;
+        }
+    }
+}
+
+__global__ void split_rows_kernel(int64_t rows, int64_t cols, const float *src, int64_t lds, float *hi, float *lo,
+                                  int64_t ldd, int64_t pad) {
+    const int64_t i = (int64_t)blockIdx.x * blockDim.x + threadIdx.x;
+    if (i >= rows * pad) return;
+    const int64_t r = i / pad, c = i % pad;
+    const float v = c < cols ? src[r * lds + c] : 0.f;
+    const float h = tc::tf32_hi(v);
+    hi[r * ldd + c] = h;
+    lo[r * ldd + c] = v - h;
+}
+}  // namespace
+
+realq_status_t tc_trans_planes(cudaStream_t s, int64_t rows, int64_t cols, const float *src, int64_t lds,
+                               float *dh, float *dl, int64_t ldd) {
+    if (rows <= 0 || cols <= 0) return REALQ_OK;
+    const int64_t tr = ceil_div(rows, 32), tcn = ceil_div(cols, 32);
+    {
+        Launch L("tf32_split", s);
+        trans_planes_kernel<<<(unsigned)(tr * tcn), dim3(32, 8), 0, s>>>(rows, cols, src, lds, dh, dl, ldd, tcn);
+    }
+    return check_launch("tf32_split");
+}
+
+realq_status_t tc_split_rows(cudaStream_t s, int64_t rows, int64_t cols, const float *src, int64_t lds, float *hi,
+                             float *lo, int64_t ldd, int64_t pad) {
+    if (rows <= 0 || cols <= 0) return REALQ_OK;
+    if (cols > pad || pad > ldd)
+        return fail(REALQ_ERR_INVALID_ARG, "tf32 split: %lld columns padded to %lld in rows of %lld", (long long)cols,
+                    (long long)pad, (long long)ldd);
+    {
+        Launch L("tf32_split", s);
+        split_rows_kernel<<<(unsigned)ceil_div(rows * pad, 256), 256, 0, s>>>(rows, cols, src, lds, hi, lo, ldd, pad);
+    }
+    return check_launch("tf32_split");
+}
+
 realq_status_t tc_trail_planes(cudaStream_t s, int64_t m, const float *Et, int64_t ldet, int64_t n, const float *U,
                                int64_t bs, int64_t be, int kb, int B, float *Eh, float *El, float *Ph, float *Pl) {
     if (kb <= 0 || kb % 32 != 0 || kb > B || be > n || bs + kb > n)
@@ -618,6 +711,7 @@ realq_status_t launch_tf32x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N
     REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ADAM, TN>), SM));
     REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ACCUM, TN>), SM));
     REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_PG, TN>), SM));
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_SYRK, TN>), SM));
     const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
     const dim3 grid((unsigned)ceil_div(N, TN), (unsigned)ceil_div(M, TB), nz);
     switch (e.mode) {
@@ -636,6 +730,10 @@ realq_status_t launch_tf32x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N
         case TC_ACCUM:
             gemm_tf32x3_kernel<TC_ACCUM, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
                                                                        kchunk, exact);
+            break;
+        case TC_SYRK:
+            gemm_tf32x3_kernel<TC_SYRK, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
+                                                                      kchunk, exact);
             break;
         default:
             gemm_tf32x3_kernel<TC_BGD_PG, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
@@ -677,7 +775,10 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     if (kchunk < 0 || (kchunk % Tile<128>::KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
         return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name,
                     Tile<128>::KS);
-    if (e.mode < TC_STORE || e.mode > TC_BGD_PG) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
+    if (e.mode < TC_STORE || e.mode > TC_SYRK) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
+    if (e.mode == TC_SYRK && (a_row0 != 0 || b_row0 != 0 || M != N))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: a symmetric update takes a square product from row 0", name);
+    if (e.b_tri && kchunk > 0) return fail(REALQ_ERR_INVALID_ARG, "%s: a triangular B takes no K split", name);
     const MapPair &mp = *reinterpret_cast<const MapPair *>(maps.storage);
     const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));

@@ -51,7 +51,7 @@ struct GemmArgs {
 realq_status_t gemm_f32(cudaStream_t s, AMode am, EpiMode em, const GemmArgs &g, const char *name);
 
 // ------------------------------------------- tensor-core tf32x3 GEMM ---
-enum TcMode { TC_STORE = 0, TC_BGD_P = 1, TC_ADAM = 2, TC_ACCUM = 3, TC_BGD_PG = 4 };
+enum TcMode { TC_STORE = 0, TC_BGD_P = 1, TC_ADAM = 2, TC_ACCUM = 3, TC_BGD_PG = 4, TC_SYRK = 5 };
 struct TcEpi {
     int mode;
     float *C; int64_t ldc;                                   // TC_STORE
@@ -62,6 +62,7 @@ struct TcEpi {
     float *Wm; float *mA; float *vA; float *D; float *Sh; float *Sl;  // TC_ADAM (ldw, col0 shared)
     float lr, b1, b2, eps, bc1, bc2; int sgd;
     int64_t czs;                                             // TC_STORE with a K split: C of split z at C + z czs
+    int b_tri;   // B(j, k) = 0 for k > j (K range relative to the output column): a CTA's K ends at its last column
 };
 // The operand maps of one product, for both tile shapes of the kernel
 // (128 x 128 outputs with 32-wide K slices, 128 x 256 with 16-wide slices).
@@ -72,6 +73,15 @@ bool tc_gemm_eligible(int64_t m, int64_t n);
 // Tile shape of the tf32x3 products: 0 chosen per launch by its grid, 1 always
 // 128 x 128, 2 always 128 x 256 (process-wide).
 void tc_set_tile_mode(int mode);
+// hi / lo planes of the transpose of the rows x cols block at src (row stride
+// lds): dst[c * ldd + r] for r < rows, c < cols.
+realq_status_t tc_trans_planes(cudaStream_t s, int64_t rows, int64_t cols, const float *src, int64_t lds,
+                               float *dh, float *dl, int64_t ldd);
+// hi / lo planes of the rows x cols block at src (row stride lds), written
+// to hi / lo with row stride ldd: columns 0..pad-1 of each row, those from
+// cols on zero (pad >= cols, ldd >= pad).
+realq_status_t tc_split_rows(cudaStream_t s, int64_t rows, int64_t cols, const float *src, int64_t lds, float *hi,
+                             float *lo, int64_t ldd, int64_t pad);
 // The operands of the lazy batch update W[:, be:] -= E_b U[bs:be, be:] as
 // K-major tf32 planes: Eh/El = hi/lo of -E_b (m x B, from Et, kb x m with
 // leading dimension ldet; skipped when Et is NULL), Ph/Pl = hi/lo of

@@ -267,6 +267,19 @@ constexpr size_t prepare_bytes_split(int64_t n, int slices) {
            align256((size_t)slices * n * NB * sizeof(float));
 }
 constexpr size_t prepare_bytes(int64_t n) { return prepare_bytes_split(n, 1); }
+// tf32 hi / lo planes of two panels (n x NB each), for the rank-NB updates on
+// the tensor cores (two sets: a step's panel is split while the previous
+// step's update may still read the other set)
+constexpr size_t tc_panel_bytes(int64_t n) { return 4 * align256((size_t)n * NB * sizeof(float)); }
+// the triangular inverse's product on the tensor cores: planes of U^T (n x n,
+// filled block column by block column as U's row blocks become final) and of
+// the row block R[K, K+1:] (NB x n, at its global columns)
+constexpr size_t tc_trtri_bytes(int64_t n) {
+    return 2 * align256((size_t)n * n * sizeof(float)) + 2 * align256((size_t)NB * n * sizeof(float));
+}
+// the rank-NB update above the diagonal takes the tensor cores from this many
+// rows on (below it the fp32 tiles, whose work is small)
+constexpr int64_t kTcUpdateRows = 512;
 
 // Scratch of the allocation-free entry point, sized for n <= REALQ_PREPARE_NOALLOC_MAX_N.
 // Every GPU that loads the library holds it until the process exits.
@@ -288,7 +301,9 @@ realq_status_t noalloc_scratch(void **out) {
 
 }  // namespace
 
-size_t prepare_ws_bytes(int64_t n) { return prepare_bytes_split(n, KSPLIT_MAX); }
+size_t prepare_ws_bytes(int64_t n) {
+    return prepare_bytes_split(n, KSPLIT_MAX) + tc_panel_bytes(n) + tc_trtri_bytes(n);
+}
 
 realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, const float *H, float *U, float *Hbar,
                             uint8_t *dead, int64_t *fail_col, void *ws, size_t ws_bytes, bool overlap, bool sync);
@@ -364,11 +379,41 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
     float *lam = cv.take<float>(1);
     float *Vd = cv.take<float>((size_t)NB * NB);
     float *panel = cv.take<float>(0);
+    // the wide rank-NB updates on the tensor cores when the workspace has
+    // room for the panel planes besides one panel slice (otherwise the fp32
+    // tiles) and n suits the product
+    const bool tc_update = n % 4 == 0 && n > kTcUpdateRows && tc_gemm_eligible(n, n) &&
+                           ws_bytes >= prepare_bytes_split(n, 1) + tc_panel_bytes(n);
+    const bool tc_trtri = tc_update && ws_bytes >= prepare_bytes_split(n, 1) + tc_panel_bytes(n) + tc_trtri_bytes(n);
+    const size_t reserve = (tc_update ? tc_panel_bytes(n) : 0) + (tc_trtri ? tc_trtri_bytes(n) : 0);
     // as many K slices of the panel product as the workspace holds
     int slices = 1;
-    while (slices < KSPLIT_MAX && prepare_bytes_split(n, slices + 1) <= ws_bytes) ++slices;
+    while (slices < KSPLIT_MAX && prepare_bytes_split(n, slices + 1) + reserve <= ws_bytes) ++slices;
     const int64_t plane = n * NB;
+    float *Pp[4] = {nullptr, nullptr, nullptr, nullptr};   // set 0 hi, lo; set 1 hi, lo
+    float *UTh = nullptr, *UTl = nullptr, *Rh = nullptr, *Rl = nullptr;
+    TcMaps pmaps[2], tmaps;
+    if (tc_update) {
+        Carve pc(reinterpret_cast<unsigned char *>(ws) + prepare_bytes_split(n, slices));
+        for (int i = 0; i < 4; ++i) Pp[i] = pc.take<float>((size_t)n * NB);
+        for (int st = 0; st < 2; ++st)
+            REALQ_TRY(tc_make_maps(&pmaps[st], Pp[2 * st], Pp[2 * st + 1], n, NB, NB, Pp[2 * st], Pp[2 * st + 1], n,
+                                   NB, NB));
+        if (tc_trtri) {
+            UTh = pc.take<float>((size_t)n * n);
+            UTl = pc.take<float>((size_t)n * n);
+            Rh = pc.take<float>((size_t)NB * n);
+            Rl = pc.take<float>((size_t)NB * n);
+            // A: the row block R[K, K+1:] (NB rows, columns at their global
+            // index); B: rows of U^T, so that both take K from column k1 on
+            REALQ_TRY(tc_make_maps(&tmaps, Rh, Rl, NB, n, n, UTh, UTl, n, n, n));
+        }
+    }
+    // status[0]: the failing column (-1: none); status[1]: timeout bits of
+    // the tensor-core updates (the same 256-byte slot of the workspace)
+    int *status_tc = status + 1;
     REALQ_CUDA_TRY(cudaMemsetAsync(status, 0xFF, sizeof(int), s));
+    REALQ_CUDA_TRY(cudaMemsetAsync(status_tc, 0, sizeof(int), s));
     const int64_t tot = n * n;
     {
         Launch L("prepare_init", s);
@@ -388,6 +433,12 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
     // Row block K of U touches rows >= k0 only, the later Cholesky steps rows
     // < k0 only: with overlap, the U row work runs on an auxiliary stream that
     // starts after the diagonal step of K (which wrote U_KK into A[K, K]).
+    if (tc_trtri) {
+        // U^T's planes are filled on and below the diagonal, block column by
+        // block column; what lies above it is read as zeros
+        REALQ_CUDA_TRY(cudaMemsetAsync(UTh, 0, (size_t)n * n * sizeof(float), s));
+        REALQ_CUDA_TRY(cudaMemsetAsync(UTl, 0, (size_t)n * n * sizeof(float), s));
+    }
     AuxStream *aux = nullptr;
     if (overlap && nbk > 1) REALQ_TRY(aux_for(s, nbk, &aux));
     cudaStream_t rs = aux ? aux->stream : s;
@@ -406,7 +457,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
             chol_diag_kernel<<<1, 128, 0, s>>>(n, U, k0, kb, status, Vd);
         }
         REALQ_TRY(check_launch("chol_diag"));
-        if (aux && k1 < n) {
+        if (aux && (k1 < n || tc_trtri)) {
             REALQ_CUDA_TRY(cudaEventRecord(aux->steps[K], s));
             REALQ_CUDA_TRY(cudaStreamWaitEvent(rs, aux->steps[K], 0));
         }
@@ -440,7 +491,18 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
             REALQ_TRY(check_launch("chol_update"));
             if (nwide > 0) {
                 cudaStream_t ws_ = aux ? aux->wide : s;
-                {
+                const int64_t kw = k0 - NB;   // rows and columns of the wide part
+                if (tc_update && kw >= kTcUpdateRows) {
+                    // U[0:kw, 0:kw] (upper) -= P P^T with P = R[0:kw, K], as
+                    // a tf32x3 symmetric product on the tensor cores
+                    const int st = K & 1;
+                    REALQ_TRY(tc_split_rows(ws_, kw, kb, U + k0, n, Pp[2 * st], Pp[2 * st + 1], NB, NB));
+                    TcEpi e{};
+                    e.mode = TC_SYRK;
+                    e.M = U;
+                    e.ldw = n;
+                    REALQ_TRY(tc_gemm_tf32x3(ws_, pmaps[st], kw, kw, NB, 0, 0, e, status_tc, "chol_update_tc"));
+                } else {
                     Launch L("chol_update", ws_);
                     chol_update_kernel<<<(unsigned)nwide, 256, 0, ws_>>>(n, U, k0, kb, 0);
                 }
@@ -452,7 +514,27 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
                 }
             }
         }
-        if (k1 < n) {
+        if (k1 < n && tc_trtri) {
+            const int64_t r = n - k1;
+            // X = R[K, K+1:] U[K+1:, K+1:] on the tensor cores: the planes of
+            // the row block, then X = R_K (U^T)^T with U^T's rows k1.. (a
+            // column tile's K range ends at its last column: U is upper)
+            REALQ_TRY(tc_split_rows(rs, kb, r, U + k0 * n + k1, n, Rh + k1, Rl + k1, n, r));
+            TcEpi e{};
+            e.mode = TC_STORE;
+            e.C = panel;
+            e.ldc = n;
+            e.b_tri = 1;
+            REALQ_TRY(tc_gemm_tf32x3(rs, tmaps, kb, r, r, (int)k1, (int)k1, e, status_tc, "trtri_trmm_tc"));
+            // U[K, K+1:] = -U_KK X, U_KK read from A[K, K] (upper, zeros below)
+            GemmArgs h{};
+            h.M = kb; h.N = r; h.K = kb;
+            h.A = U + k0 * n + k0; h.lda = n;
+            h.B = panel; h.ldb = n; h.nsum_b = 1; h.bplane = plane;
+            h.C = U + k0 * n + k1; h.ldc = n;
+            h.alpha = -1.f;
+            REALQ_TRY(gemm_f32(rs, A_ROW, EPI_STORE, h, "trtri_panel"));
+        } else if (k1 < n) {
             const int64_t r = n - k1;
             // X = R[K, K+1:] U[K+1:, K+1:] (U upper: a column tile's K range ends
             // at its last column), K split into fixed-order slices
@@ -474,6 +556,10 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
             h.alpha = -1.f;
             REALQ_TRY(gemm_f32(rs, A_ROW, EPI_STORE, h, "trtri_panel"));
         }
+        // row block K of U is final: its transpose joins U^T's planes for the
+        // later steps' products
+        if (tc_trtri)
+            REALQ_TRY(tc_trans_planes(rs, kb, n - k0, U + k0 * n + k0, n, UTh + k0 * n + k0, UTl + k0 * n + k0, n));
     }
     if (aux) {
         REALQ_CUDA_TRY(cudaEventRecord(aux->ev[1], rs));
@@ -486,11 +572,13 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
         }
     }
     if (!sync) return REALQ_OK;  // the failing column stays in the workspace's first word
-    int host_status = -1;
-    REALQ_CUDA_TRY(cudaMemcpyAsync(&host_status, status, sizeof(int), cudaMemcpyDeviceToHost, s));
+    int host_status[2] = {-1, 0};
+    REALQ_CUDA_TRY(cudaMemcpyAsync(host_status, status, 2 * sizeof(int), cudaMemcpyDeviceToHost, s));
     REALQ_CUDA_TRY(cudaStreamSynchronize(s));
-    *fail_col = host_status;
-    if (host_status >= 0) return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", host_status);
+    *fail_col = host_status[0];
+    if (host_status[1] & ST_TIMEOUT) return fail(REALQ_ERR_TIMEOUT, "a bounded device-side wait gave up (prepare)");
+    if (host_status[0] >= 0)
+        return fail(REALQ_ERR_NOT_SPD, "damped Hessian not positive definite at column %d", host_status[0]);
     return REALQ_OK;
 }
 

@@ -86,7 +86,11 @@ def test_hessian_bf16_and_cross_moment(n, T):
 
 
 # --------------------------------------------------------------- prepare ---
-@pytest.mark.parametrize("n,dead", [(256, ()), (300, (5, 77, 299)), (64, ())])
+# n = 1500 and 2052 take the tensor-core rank-64 updates and the tensor-core
+# triangular-inverse product (n > 512, n % 4 == 0), 2052 with a ragged first
+# 4-column panel; 1498 (n % 4 != 0) keeps the fp32 tiles
+@pytest.mark.parametrize("n,dead", [(256, ()), (300, (5, 77, 299)), (64, ()), (1500, (3, 700)), (2052, ()),
+                                    (1498, ())])
 def test_prepare_matches_oracle(n, dead):
     case = synth.layer_case(22, 4, n, 4 * n, outliers=3, dead_cols=dead)
     Href, T = oracle.hessian_sum([case.Xhat])
