@@ -123,15 +123,22 @@ def test_fullsize_sweeps_against_oracle(block_run, oracle_H):
         o = bq.out[md.name]
         assert o["adam_t"] == orc["adam_t"] == nb - 1
         codes = unpack(o["codes"].cpu().numpy(), md.n)
-        plain, _, _ = check_codes_and_scales(orc, codes, o["zero"].cpu().numpy(), o["scale"].cpu().numpy(), md.n,
-                                             qkw, True, wl.lr, wl.steps_per_block, f"{md.name} {md.m}x{md.n} ")
-        L_or = token_surrogate(oracle, plain["deq"], W0, _x64, x_bits[md.input], F_np[md.name])
+        plain, fol, _ = check_codes_and_scales(orc, codes, o["zero"].cpu().numpy(), o["scale"].cpu().numpy(),
+                                               md.n, qkw, True, wl.lr, wl.steps_per_block, f"{md.name} {md.m}x{md.n} ")
+        # the surrogate of the oracle's result on the CUDA path's branch at
+        # rounding ties (the one the codes are compared with; the plain run's
+        # is printed: at lr 3e-4 a few ties taken the other way move the loss
+        # by about 1e-3)
+        L_or = token_surrogate(oracle, fol["deq"], W0, _x64, x_bits[md.input], F_np[md.name])
+        L_plain = L_or if fol is plain else token_surrogate(oracle, plain["deq"], W0, _x64, x_bits[md.input],
+                                                            F_np[md.name])
         ws = rq.workspace(rq.realq_surrogate_workspace_size(md.m, md.n))
         loss = torch.zeros(1, device="cuda")
         rq.realq_surrogate_loss(o["W"], torch.from_numpy(W0.astype(np.float32)).cuda(), bq.state[md.input]["Hbar"],
                                 torch.from_numpy(F_np[md.name]).cuda(), loss, ws)
         L_gpu = float(loss.item())
-        print(f"{md.name}: surrogate gpu {L_gpu:.6e} oracle {L_or:.6e} (rel {abs(L_gpu - L_or) / L_or:.2e})")
+        print(f"{md.name}: surrogate gpu {L_gpu:.6e} oracle {L_or:.6e} (rel {abs(L_gpu - L_or) / L_or:.2e}); "
+              f"plain oracle {L_plain:.6e} (rel {abs(L_gpu - L_plain) / L_plain:.2e})")
         assert abs(L_gpu - L_or) <= 1e-3 * L_or
 
 
