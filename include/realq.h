@@ -520,6 +520,15 @@ void realq_graph_destroy(realq_graph_t graph);
  * for other values.  No counterpart in the paper. */
 realq_status_t realq_set_tensor_tile(int mode);
 
+/* Tuning: the kernel of the column-serial quantize-and-compensate step.  1
+ * (default): warps pipelined through shared-memory progress flags where the
+ * group parameters are taken at the block start or before it; 0: the kernel
+ * whose warps meet at a block-wide barrier after every 32 columns.  Both
+ * perform the same operations in the same order (identical results).
+ * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
+ * the paper. */
+realq_status_t realq_set_quant_kernel(int mode);
+
 /* The learning rate of decoder block i (1-based) of L under the paper's
  * reverse-cosine schedule over transformer blocks (App. "Full Setup",
  * Eq. reverse_cosine; the first block's rate is 0.01 of the final one, App.

@@ -807,6 +807,12 @@ realq_status_t realq_set_tensor_tile(int mode) {
     return REALQ_OK;
 }
 
+realq_status_t realq_set_quant_kernel(int mode) {
+    if (mode < 0 || mode > 1) return fail(REALQ_ERR_INVALID_ARG, "set_quant_kernel: mode 0 or 1");
+    quant_set_kernel(mode);
+    return REALQ_OK;
+}
+
 // ------------------------------------------------------------ schedules ---
 realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out) {
     if (!lr_out || L < 1 || i < 1 || i > L || !std::isfinite(lr_final))

@@ -73,6 +73,10 @@ bool tc_gemm_eligible(int64_t m, int64_t n);
 // Tile shape of the tf32x3 products: 0 chosen per launch by its grid, 1 always
 // 128 x 128, 2 always 128 x 256 (process-wide).
 void tc_set_tile_mode(int mode);
+// The column-serial quantizer: 1 the pipelined kernel where the group
+// parameters come at the block start or before it (default), 0 the
+// barrier-phased kernel everywhere (process-wide).
+void quant_set_kernel(int mode);
 // hi / lo planes of the transpose of the rows x cols block at src (row stride
 // lds): dst[c * ldd + r] for r < rows, c < cols.
 realq_status_t tc_trans_planes(cudaStream_t s, int64_t rows, int64_t cols, const float *src, int64_t lds,

@@ -274,6 +274,231 @@ __global__ void __launch_bounds__(B) quant_block_kernel(const QArgs a) {
     if (bad) atomicOr(a.status, ST_NONFINITE);
 }
 
+// The same column-serial quantize + in-block OBS as quant_block_kernel, with
+// the phases pipelined: warp w applies sub-block s's errors in chunks of 8
+// columns as soon as warp s has published them (a per-warp progress flag in
+// shared memory) and starts its own chain right after, instead of every warp
+// waiting at a CTA barrier for the slowest one after every phase.  Each
+// weight still receives exactly the updates of the plain column loop in the
+// same order (sub-blocks in order, columns in order), so the results are the
+// kernel's above bit for bit.  U's diagonal block is staged as its 32 x 32
+// blocks on or above the diagonal only (row pitch 36 keeps float4 reads
+// aligned), which leaves room for three CTAs per SM beside the error
+// buffers.  Group parameters at the block start (G = B) or before it (G = 0).
+template <int B>
+struct QPipe {
+    static constexpr int NW = B / 32;
+    static constexpr int NSLOT = NW * (NW + 1) / 2;
+    static constexpr int P = 36;
+    static constexpr int NBUF = NW > 1 ? NW - 1 : 1;
+    static constexpr size_t floats = (size_t)NSLOT * 32 * P + B + (size_t)NBUF * QB_ROWS * 33 + 2 * NW * QB_ROWS + NW;
+};
+
+// slot of the 32 x 32 block (s, w), s <= w, in row-major order of the upper triangle
+__device__ __forceinline__ int qslot(int s, int w, int nw) { return s * nw - s * (s - 1) / 2 + (w - s); }
+
+template <int B, int G>
+__global__ void __launch_bounds__(B) quant_block_pipe_kernel(const QArgs a) {
+    static_assert(G == 0 || G == B, "group parameters at the block start or before it");
+    using QP = QPipe<B>;
+    constexpr int NW = QP::NW, P = QP::P;
+    extern __shared__ __align__(16) float qsm[];
+    float *Ut = qsm;                                   // NSLOT x 32 x P
+    float *invd = Ut + QP::NSLOT * 32 * P;             // B
+    float *Es = invd + B;                              // NBUF x QB_ROWS x 33
+    float *mm = Es + QP::NBUF * QB_ROWS * 33;          // 2 x NW x QB_ROWS
+    volatile int *flags = reinterpret_cast<volatile int *>(mm + 2 * NW * QB_ROWS);   // NW
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int kb = a.kb;
+    if (threadIdx.x < NW) flags[threadIdx.x] = 0;
+    // U's blocks on or above the diagonal: slot (s, w) row jj col c holds
+    // U[bs + 32 s + jj][bs + 32 w + c] where that lies strictly above the
+    // diagonal of the block, else 0
+    for (int idx = threadIdx.x; idx < QP::NSLOT * 32 * 8; idx += blockDim.x) {
+        const int slot = idx / 256, rr = (idx / 8) % 32, c4 = (idx % 8) * 4;
+        int s = 0, w = 0;
+        for (int t = 0, k = 0; t < NW; ++t)
+            for (int u = t; u < NW; ++u, ++k)
+                if (k == slot) { s = t; w = u; }
+        const int j = s * 32 + rr;
+        float v[4];
+        if ((a.n & 3) == 0 && kb == B) {
+            const float4 q = *reinterpret_cast<const float4 *>(a.U + (a.bs + j) * a.n + a.bs + w * 32 + c4);
+            v[0] = q.x; v[1] = q.y; v[2] = q.z; v[3] = q.w;
+        } else {
+#pragma unroll
+            for (int e = 0; e < 4; ++e) {
+                const int k = w * 32 + c4 + e;
+                v[e] = (j < kb && k < kb) ? a.U[(a.bs + j) * a.n + a.bs + k] : 0.f;
+            }
+        }
+        float *d = Ut + slot * 32 * P + rr * P + c4;
+#pragma unroll
+        for (int e = 0; e < 4; ++e) d[e] = (s < w || c4 + e > rr) ? v[e] : 0.f;
+    }
+    for (int j = threadIdx.x; j < B; j += blockDim.x)
+        invd[j] = (j < kb) ? 1.f / a.U[(a.bs + j) * a.n + a.bs + j] : 0.f;
+
+    const int64_t i = (int64_t)blockIdx.x * QB_ROWS + lane;   // this lane's row
+    const bool live = i < a.m;
+    const int c0 = warp * 32;                                   // this warp's first column
+    float r[32];
+    {
+        const float *wrow = a.W + (live ? i : 0) * a.n + a.bs + c0;
+        if ((a.n & 3) == 0 && c0 + 32 <= kb) {
+#pragma unroll
+            for (int c = 0; c < 32; c += 4) {
+                const float4 v = live ? *reinterpret_cast<const float4 *>(wrow + c) : make_float4(0.f, 0.f, 0.f, 0.f);
+                r[c] = v.x; r[c + 1] = v.y; r[c + 2] = v.z; r[c + 3] = v.w;
+            }
+        } else {
+#pragma unroll
+            for (int c = 0; c < 32; ++c) r[c] = (live && c0 + c < kb) ? wrow[c] : 0.f;
+        }
+    }
+    float sc = 1.f, zr = 0.f;
+    if (G == 0 && live) {
+        const int gi = (int)(a.bs / a.g);
+        sc = a.scale[i * a.ngroups + gi];
+        zr = (float)a.zero[i * a.ngroups + gi];
+    }
+    if (G == B) {
+        // one group: min / max over the block's columns from every warp
+        float mn = 0.f, mx = 0.f;
+#pragma unroll
+        for (int c = 0; c < 32; ++c)
+            if (c0 + c < kb) {
+                mn = fminf(mn, r[c]);
+                mx = fmaxf(mx, r[c]);
+            }
+        mm[warp * QB_ROWS + lane] = mn;
+        mm[(NW + warp) * QB_ROWS + lane] = mx;
+    }
+    __syncthreads();
+    if (G == B) {
+        if (warp == 0) {
+            float mn = 0.f, mx = 0.f;
+            for (int w = 0; w < NW; ++w) {
+                mn = fminf(mn, mm[w * QB_ROWS + lane]);
+                mx = fmaxf(mx, mm[(NW + w) * QB_ROWS + lane]);
+            }
+            grid_params(mn, mx, a.bits, a.sym, sc, zr);
+            if (live) {
+                const int gi = (int)(a.bs / a.g);
+                a.scale[i * a.ngroups + gi] = sc;
+                a.zero[i * a.ngroups + gi] = (uint8_t)zr;
+            }
+            // (each lane overwrites only partials it has already read)
+            mm[lane] = sc;
+            mm[QB_ROWS + lane] = zr;
+        }
+        __syncthreads();
+        sc = mm[lane];
+        zr = mm[QB_ROWS + lane];
+    }
+
+    const float maxq = (float)((1 << a.bits) - 1);
+    bool bad = false, late = false;
+    if (c0 < kb) {
+        // the errors of every earlier sub-block, chunk by chunk as published
+#pragma unroll 1
+        for (int s = 0; s < warp; ++s) {
+            const float *E = Es + s * QB_ROWS * 33;
+#pragma unroll 1
+            for (int ch = 0; ch < 4; ++ch) {
+                if (lane == 0) {
+                    uint32_t it = 0;
+                    while (flags[s] < ch + 1) {
+                        if (++it > (1u << 22)) {
+                            late = true;
+                            break;
+                        }
+                        __nanosleep(32);
+                    }
+                }
+                __syncwarp();
+                __threadfence_block();
+#pragma unroll 1
+                for (int jj = ch * 8; jj < ch * 8 + 8; ++jj) {
+                    const float ej = E[lane * 33 + jj];
+                    const float *urow = Ut + qslot(s, warp, NW) * 32 * P + jj * P;
+#pragma unroll
+                    for (int c = 0; c < 32; c += 4) {
+                        const float4 u = *reinterpret_cast<const float4 *>(urow + c);
+                        r[c] = fmaf(-ej, u.x, r[c]);
+                        r[c + 1] = fmaf(-ej, u.y, r[c + 1]);
+                        r[c + 2] = fmaf(-ej, u.z, r[c + 2]);
+                        r[c + 3] = fmaf(-ej, u.w, r[c + 3]);
+                    }
+                }
+            }
+        }
+        // this warp's own columns, one after the other
+        const bool publish = c0 + 32 < kb && warp < NW - 1;
+        float *Eo = Es + (warp < QP::NBUF ? warp : 0) * QB_ROWS * 33;
+        const float *ud = Ut + qslot(warp, warp, NW) * 32 * P;
+        uint32_t packed[4] = {0u, 0u, 0u, 0u};
+        // rint(w / sc) through the reciprocal, as in quant_block_kernel
+        const float rcp = __frcp_rn(sc);
+#pragma unroll
+        for (int jj = 0; jj < 32; ++jj) {
+            const int j = c0 + jj;
+            float err = 0.f;
+            uint32_t qi = 0;
+            if (j < kb) {
+                const float w = r[jj];
+                bad |= !isfinite(w);
+                const float x = __fmul_rn(w, rcp);
+                float qx = rintf(x);
+                const float gap = 0.5f - fabsf(x - qx);
+                if (!(gap > 2.4e-7f * fabsf(x) + 1e-30f)) qx = rintf(w / sc);
+                float q = qx + zr;
+                q = fminf(fmaxf(q, 0.f), maxq);
+                const float dq = sc * (q - zr);
+                err = (w - dq) * invd[j];
+                r[jj] = dq;
+                qi = (uint32_t)q;
+#pragma unroll
+                for (int kk = jj + 1; kk < 32; ++kk) r[kk] = fmaf(-err, ud[jj * P + kk], r[kk]);
+            }
+            if (publish) Eo[lane * 33 + jj] = err;
+            if (live && j < kb) a.Et[(int64_t)j * a.ldet + i] = err;
+            packed[jj >> 3] |= (qi & 15u) << ((jj & 7) * 4);
+            if (publish && (jj & 7) == 7) {
+                __syncwarp();
+                if (lane == 0) {
+                    __threadfence_block();
+                    flags[warp] = (jj >> 3) + 1;
+                }
+            }
+        }
+        if (live) {
+            uint8_t *crow = a.codes + i * a.ncb + (a.bs + c0) / 2;
+            if (c0 + 32 <= kb && (((uintptr_t)crow) & 15) == 0) {
+                *reinterpret_cast<uint4 *>(crow) = make_uint4(packed[0], packed[1], packed[2], packed[3]);
+            } else {
+                for (int jj = 0; jj < 32 && c0 + jj < kb; jj += 2)
+                    crow[jj / 2] = (uint8_t)((packed[jj >> 3] >> ((jj & 7) * 4)) & 0xFFu);
+            }
+        }
+        if (live) {
+            float *wout = a.W + i * a.n + a.bs + c0;
+            if ((a.n & 3) == 0 && c0 + 32 <= kb) {
+#pragma unroll
+                for (int c = 0; c < 32; c += 4)
+                    *reinterpret_cast<float4 *>(wout + c) = make_float4(r[c], r[c + 1], r[c + 2], r[c + 3]);
+            } else {
+#pragma unroll
+                for (int c = 0; c < 32; ++c)
+                    if (c0 + c < kb) wout[c] = r[c];
+            }
+        }
+    }
+    late = __shfl_sync(0xffffffffu, late ? 1 : 0, 0) != 0;
+    if (bad) atomicOr(a.status, ST_NONFINITE);
+    if (late && lane == 0) atomicOr(a.status, ST_TIMEOUT);
+}
+
 // One optimizer step on the free columns c0..n-1; the applied step is also
 // accumulated into D (the optimizer displacement) when D is given.
 __global__ void adam_kernel(int64_t m, int64_t r, int64_t n, int64_t c0, const float *G, float *W, float *mA,
@@ -374,8 +599,28 @@ realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
     return check_launch("quant_block");
 }
 
+int g_quant_kernel = 1;   // 1: the pipelined quantizer where it applies, 0: the barrier-phased one
+}  // namespace
+
+void quant_set_kernel(int mode) { g_quant_kernel = mode; }
+
+namespace {
+
+template <int B, int G>
+realq_status_t launch_qb_pipe(cudaStream_t s, const QArgs &qa) {
+    const size_t smem = QPipe<B>::floats * sizeof(float);
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(quant_block_pipe_kernel<B, G>), (int)smem));
+    {
+        Launch L("quant_block", s);
+        quant_block_pipe_kernel<B, G><<<ceil_div(qa.m, QB_ROWS), B, smem, s>>>(qa);
+    }
+    return check_launch("quant_block");
+}
+
 template <int B>
 realq_status_t launch_qb_g(cudaStream_t s, const QArgs &qa, int Gk) {
+    if (g_quant_kernel == 1 && Gk == 0) return launch_qb_pipe<B, 0>(s, qa);
+    if (g_quant_kernel == 1 && Gk == B) return launch_qb_pipe<B, B>(s, qa);
     if (Gk == 0) return launch_qb<B, 0>(s, qa);
     if (Gk == B) return launch_qb<B, B>(s, qa);
     if (B >= 64 && Gk == B / 2) return launch_qb<B, (B >= 64 ? B / 2 : B)>(s, qa);

@@ -902,3 +902,28 @@ def test_tensor_tiles_match_the_oracle(tile):
         test_token_block_gd_with_output_clipping(0.95, 2, 2)
     finally:
         rq.realq_set_tensor_tile(0)
+
+
+# --------------------------------------------------- the quantizer kernels ---
+@pytest.mark.parametrize("qkw,m,n", [(dict(group_size=128, block_size=128), 200, 384),
+                                     (dict(group_size=0, block_size=64, symmetric=1), 96, 200),
+                                     (dict(group_size=32, block_size=32), 64, 96),
+                                     (dict(group_size=128, block_size=128), 1024, 520)])
+def test_quantizer_kernels_agree_bit_for_bit(qkw, m, n):
+    # the pipelined column-serial kernel and the barrier-phased one perform
+    # the same operations in the same order: the whole sweep (with Block-GD,
+    # ragged last blocks, per-row groups, 1024 rows = 32 CTAs) is the same
+    # bits with either
+    case = synth.layer_case(77, m, n, 3 * n, outliers=2)
+    H, _, T = layer.accumulate([dev(case.Xhat)], n)
+    prep = layer.prepare(H, T)
+    outs = []
+    for mode in (0, 1):
+        rq.realq_set_quant_kernel(mode)
+        try:
+            outs.append(layer.quantize(dev(case.W0), prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4), F=dev(case.F)))
+            torch.cuda.synchronize()
+        finally:
+            rq.realq_set_quant_kernel(1)
+    for k in ("codes", "scale", "zero", "W"):
+        assert torch.equal(getattr(outs[0], k), getattr(outs[1], k)), k
