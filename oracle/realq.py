@@ -154,6 +154,11 @@ def _round(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int):
     return q, x64, margin
 
 
+def _round32(a: np.ndarray) -> None:
+    """In place: every entry rounded to the nearest single-precision value."""
+    a[...] = a.astype(np.float32)
+
+
 def _dequant(q: np.ndarray, scale: np.ndarray, zero: np.ndarray) -> np.ndarray:
     return (scale.astype(np.float32) * (q.astype(np.float32) - zero.astype(np.float32))).astype(np.float32)
 
@@ -381,7 +386,7 @@ def pack_codes(codes: np.ndarray) -> np.ndarray:
 # ---------------------------------------------------------------------------
 def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetric=False,
                 damp_frac=0.01, bgd=None, F=None, F_next=None, D_sum=None, record=True, obs_hessians=None,
-                follow=None, columns=None, grad_noise=None):
+                follow=None, columns=None, grad_noise=None, state32=False):
     """Quantize W0 column by column with OBS feedback and Block-GD after each block.
 
     bgd: None for the plain column sweep (GPTQ), else a dict with keys
@@ -448,6 +453,12 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     decisions the sweep's arithmetic does not determine at that precision.
     The returned "x" holds every column's w / scale before rounding, "zf"
     every group's -xmin / scale.
+
+    state32: a second sensitivity probe (not part of the method): the sweep's
+    state (the Hessian, each downdated inverse, the weights after every
+    compensation and every optimizer step, the gradient and Adam's moments)
+    is rounded to single precision after every update, one realization of
+    the rounding that an fp32 implementation carries along.
     """
     W0 = np.asarray(W0, dtype=np.float64)
     m, n = W0.shape
@@ -471,6 +482,10 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
     for rows, _, dg in groups:
         W[rows, dg] = 0.0
     Hinvs = [np.linalg.inv(Hdg) for _, Hdg, _ in groups]
+    r32 = _round32 if state32 else (lambda a: None)
+    for Hinv in Hinvs:
+        r32(Hinv)
+    r32(W)
     ngroups = -(-n // g)
     codes = np.zeros((m, n), dtype=np.int64)
     scale = np.zeros((m, ngroups), dtype=np.float32)
@@ -516,8 +531,10 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             hinv_diag[k, j] = d
             # Eq. (gptq_update): W[:, j+1:] -= delta_j H^-1[j, j+1:] / [H^-1]_jj
             native.outer_sub(W[rows, j + 1:], e[rows] / d, Hinv[j, j + 1:])
+            r32(W[rows, j + 1:])
             # remove j from the free set: Schur-complement downdate of H^-1
             native.outer_sub(Hinv[j + 1:, j + 1:], Hinv[j + 1:, j], Hinv[j, j + 1:], d)
+            r32(Hinv[j + 1:, j + 1:])
         W[:, j] = dq
 
         be = j + 1
@@ -562,8 +579,14 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
                 if bgd.get("optimizer", "adam") == "sgd":
                     opt.t += 1
                     W[:, be:] -= bgd["lr"] * G
+                    r32(W[:, be:])
                 else:
+                    if state32:
+                        G = G.astype(np.float32).astype(np.float64)
                     W[:, be:] -= opt.direction(G, slice(be, n))
+                    r32(W[:, be:])
+                    r32(opt.m[:, be:])
+                    r32(opt.v[:, be:])
             if gfn is not None:
                 after = gfn(W, alpha, (b_global - 1) * steps + steps - 1)[0] if record else None
             else:

@@ -69,18 +69,23 @@ class OracleSweep:
 
 # The sensitivity probe: how far the sweep's pre-rounding values move when
 # every Block-GD gradient entry moves by eta times the magnitude of its terms
-# (oracle.gradient_error_scale), eta the rounding of an fp32 accumulation over
-# the two contractions of the gradient (P over n inputs, G over m outputs) plus
-# the tf32x3 splitting error of one product.  Two seeded probes; a decision
-# whose margin is within PROBE_K times the larger move is not determined by
-# the method's arithmetic at fp32 precision (Adam's m / sqrt(v) amplifies the
-# rounding of a gradient entry whose moments nearly cancel).
+# (oracle.gradient_error_scale), with every rounding decision held at the
+# compared run's (so that the move is the continuous one, not a cascade from
+# a decision the probe takes the other way).  eta is the error of the
+# gradient's evaluation on the tensor cores: the tf32x3 splitting error of a
+# product (2^-21) plus the accumulation in the tensor memory, which loses
+# about one unit in the last place per accumulated MMA (K = 8 per MMA, three
+# MMAs per K step) over the two contractions of the gradient (P over at most n
+# inputs, G over m outputs).  Two seeded probes; a decision whose margin is
+# within PROBE_K times the larger move is not determined by the method's
+# arithmetic at that precision (Adam's m / sqrt(v) amplifies the error of a
+# gradient entry whose moments nearly cancel).
 PROBE_K = 10.0
 PROBE_SEEDS = (101, 202)
 
 
 def probe_eta(m: int, n: int) -> float:
-    return 2.0 ** -24 * float(np.sqrt(m + n)) + 2.0 ** -21
+    return 2.0 ** -24 * 3.0 * (m + n) / 8.0 + 2.0 ** -21
 
 
 def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: float = 1e-3,
@@ -128,8 +133,9 @@ def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: fl
         dx = np.zeros((m, n))
         dz = np.zeros_like(fol["zf"])
         ds = np.zeros(fol["scale"].shape)
+        held = {"codes": fol["codes"], "zero": fol["zero"], "tau": 0.5}
         for seed in PROBE_SEEDS:
-            pr = run(follow, grad_noise={"seed": seed, "eta": eta})
+            pr = run(held, grad_noise={"seed": seed, "eta": eta})
             dx = np.maximum(dx, np.abs(pr["x"] - fol["x"]))
             dz = np.maximum(dz, np.abs(pr["zf"] - fol["zf"]))
             ds = np.maximum(ds, np.abs(pr["scale"].astype(np.float64) - fol["scale"].astype(np.float64)))
