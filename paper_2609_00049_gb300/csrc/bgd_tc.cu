@@ -292,7 +292,23 @@ __global__ void __launch_bounds__(THREADS, 1)
     volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int64_t i0 = (int64_t)blockIdx.y * TB, j0 = (int64_t)blockIdx.x * TN;
+    // Tiles in groups of up to 8 row tiles: consecutive CTAs walk down a
+    // group's rows before moving right, so that the CTAs resident at one time
+    // cover a compact block of the output and share their A rows and B rows
+    // through L2 (row-major order had each wave stream every B row of the
+    // product from DRAM again).  A bijection of the tiles: every tile is
+    // computed exactly as before.
+    int64_t ti, tj;
+    {
+        const int64_t nx = gridDim.x, ny = gridDim.y;
+        const int64_t pid = (int64_t)blockIdx.y * nx + blockIdx.x;
+        constexpr int64_t GROUP = 8;
+        const int64_t per = GROUP * nx, first = (pid / per) * GROUP;
+        const int64_t gm = (ny - first) < GROUP ? (ny - first) : GROUP;
+        ti = first + (pid % per) % gm;
+        tj = (pid % per) / gm;
+    }
+    const int64_t i0 = ti * TB, j0 = tj * TN;
     // a symmetric update touches the upper triangle only: a tile wholly
     // below the diagonal has nothing to do (uniform over the CTA, before any
     // barrier or allocation)
