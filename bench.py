@@ -407,8 +407,16 @@ def work_models(wl, args=None):
     per_step["quant_block"] = ("hbm", serial_bytes, "GB/s")
     prep_flops = sum(2 * s.n ** 3 // 3 for s in wl.inputs.values())
     per_step["chol_diag"] = ("alu", sum(s.n * 64 * 64 for s in wl.inputs.values()), "TFLOP/s")
-    per_step["trtri_trmm"] = ("alu", prep_flops // 2, "TFLOP/s")
-    per_step["chol_update"] = ("alu", prep_flops // 2, "TFLOP/s")
+    # the rank-64 updates: the look-ahead column on fp32 tiles (2 k0 64^2 flop
+    # per step, about 64 n^2 in all), the rest on the tensor cores; the
+    # triangular inverse's product on the tensor cores, or on fp32 tiles
+    # where the workspace lacks the planes of U^T
+    tc_prep = [s for s in wl.inputs.values() if s.n > 512 and s.n % 4 == 0]
+    per_step["chol_update"] = ("alu", sum(64 * s.n ** 2 for s in wl.inputs.values()) +
+                               sum(s.n ** 3 // 3 for s in wl.inputs.values() if s not in tc_prep), "TFLOP/s")
+    per_step["chol_update_tc"] = ("tf32x3", sum(s.n ** 3 // 3 - 64 * s.n ** 2 for s in tc_prep), "TFLOP/s")
+    per_step["trtri_trmm_tc"] = ("tf32x3", sum(s.n ** 3 // 3 for s in tc_prep), "TFLOP/s")
+    per_step["trtri_trmm"] = ("alu", sum(s.n ** 3 // 3 for s in wl.inputs.values() if s not in tc_prep), "TFLOP/s")
     return per_step
 
 
@@ -460,7 +468,7 @@ def roofline_table(wl, prof, steps, peaks, args=None, top=8):
     if not prof:
         return []
     models = work_models(wl, args)
-    rows = sorted(((n, v) for n, v in prof.items() if n in models and v[1] > 0 and v[0] > 0),
+    rows = sorted(((n, v) for n, v in prof.items() if n in models and models[n][1] > 0 and v[1] > 0 and v[0] > 0),
                   key=lambda kv: -kv[1][1])[:top]
     out = []
     for n, (launches, ms) in rows:

@@ -15,9 +15,10 @@ import synth  # noqa: E402
 
 # {kernel family: (launches, total ms)} over 40 steps
 PROF = {"bgd_g_gemm_adam": (5560, 194.618), "chol_diag": (4480, 145.768), "hessian_syrk_tc": (160, 125.379),
-        "trtri_trmm": (4320, 116.026), "chol_update": (8480, 114.924), "bgd_p_gemm": (2920, 111.765),
+        "trtri_trmm_tc": (4320, 116.026), "chol_update": (8480, 114.924), "bgd_p_gemm": (2920, 111.765),
         "quant_block": (3200, 97.391), "trtri_panel": (4320, 80.342), "trailing_update": (2920, 67.88),
-        "chol_panel": (4320, 44.897), "bgd_g_gsum_adam": (2920, 26.335), "hessian_reduce": (160, 17.334)}
+        "chol_update_tc": (4320, 44.897), "bgd_g_gsum_adam": (2920, 26.335), "hessian_reduce": (160, 17.334),
+        "trtri_trmm": (10, 0.5)}
 ARGS = argparse.Namespace(saliency_groups=0, act_bits=0, a_loss_clip=None, minibatch_seqs=0)
 PEAKS = {"hbm_gbs": 6764.0, "bf16_tflops": 1888.7, "bf16_tflops_sustained": 1708.1, "sm_max_mhz": 2070.0,
          "source": "measured"}
@@ -43,6 +44,7 @@ def test_table_by_device_time():
     names = [e["kernel"] for e in t]
     assert names[0] == "bgd_g_gemm_adam" and len(t) == 8
     assert "bgd_g_gsum_adam" not in names and "hessian_reduce" not in names    # no work model
+    assert "trtri_trmm" not in names     # no work on the fp32 tiles at these widths
     ms = [PROF[n][1] for n in names]
     assert ms == sorted(ms, reverse=True)
     for e in t:
