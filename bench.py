@@ -631,6 +631,7 @@ def window_bench(args, peaks):
                 "Wv": w(Hkv * dh, d), "Wo": w(d, H * dh), "g2": (1 + 0.1 * torch.randn(d, generator=g)).cuda(),
                 "Wg": w(f, d), "Wu": w(f, d), "Wd": w(d, f)}
 
+    rq.realq_set_block_products(args.block_products)
     Wl, Wn = block(), block()
     x = torch.randn(S, L, d, generator=g).cuda()
     x_hat = x + 0.05 * torch.randn(S, L, d, generator=g).cuda()
@@ -656,17 +657,25 @@ def window_bench(args, peaks):
     e1.record(stream)
     torch.cuda.synchronize()
     ms = e0.elapsed_time(e1) / args.steps
+    rq.realq_workspace_status(ws)
     # one forward pass: the seven projections and the causal attention
     # (q.k and p.v over half the sequence on average); a backward is about
     # two forwards; a call runs four forwards and two backwards
     fwd = 2 * T * (2 * d * H * dh + 2 * d * Hkv * dh + 3 * d * f) + 2 * T * L * H * dh
     flop = 8 * fwd
-    alu = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
     tf = flop / (ms / 1e3) / 1e12
+    if args.block_products:
+        # the projections as tf32x3 tensor-core products (the attention stays
+        # on the CUDA cores)
+        peak = peaks["bf16_tflops_sustained"] * (1.1 / 2.25) / 3.0
+        src, bound = f"fp32 via 3 tf32 passes: sustained bf16 x 1.1/2.25 / 3, {peaks['source']}", "tensor"
+    else:
+        peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
+        src, bound = "fp32 ALU: 152 SMs x 128 lanes x 2 x max clock", "alu"
     print(json.dumps({"kernel": "block_module_window", "d": d, "heads": H, "kv_heads": Hkv, "head_dim": dh,
-                      "ffn": f, "seqs": S, "seq_len": L, "ms_per_call": ms, "achieved": tf, "unit": "TFLOP/s",
-                      "peak": alu, "frac": tf / alu, "peak_source": "fp32 ALU: 152 SMs x 128 lanes x 2 x max clock",
-                      "bound": "alu"}))
+                      "ffn": f, "seqs": S, "seq_len": L, "block_products": args.block_products,
+                      "ms_per_call": ms, "achieved": tf, "unit": "TFLOP/s", "peak": peak, "frac": tf / peak,
+                      "peak_source": src, "bound": bound}))
 
 
 def main():
@@ -700,6 +709,8 @@ def main():
     ap.add_argument("--ffn", type=int, default=3072)
     ap.add_argument("--seqs", type=int, default=2)
     ap.add_argument("--seq-len", type=int, default=2048)
+    ap.add_argument("--block-products", type=int, choices=[0, 1], default=1,
+                    help="window: the block ops' products on tf32x3 tensor cores (1) or fp32 CUDA cores (0)")
     ap.add_argument("--n", type=int, default=2048)
     ap.add_argument("--m", type=int, default=1024)
     ap.add_argument("--tokens", type=int, default=65536)

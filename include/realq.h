@@ -430,7 +430,7 @@ realq_status_t realq_surrogate_loss(realq_stream_t stream, int64_t m, int64_t n,
 size_t realq_surrogate_workspace_size(int64_t m, int64_t n);
 
 /* Synchronizes `stream`, returns the device status word recorded at the start
- * of a Hessian or quantize workspace (REALQ_OK, REALQ_ERR_TIMEOUT,
+ * of a Hessian, quantize or block-ops workspace (REALQ_OK, REALQ_ERR_TIMEOUT,
  * REALQ_ERR_NONFINITE) and clears it. */
 realq_status_t realq_workspace_status(realq_stream_t stream, void *ws, size_t ws_bytes);
 
@@ -482,6 +482,42 @@ realq_status_t realq_graph_launch(realq_graph_t graph, realq_stream_t stream);
 int64_t realq_graph_kernels(realq_graph_t graph);
 void realq_graph_destroy(realq_graph_t graph);
 
+/* Tuning: the output tile of the fp32-accurate (tf32x3) tensor-core
+ * products of Block-GD and the lazy batch update.  0 (default): chosen per
+ * launch from its grid (128 x 256 when its waves on the SMs take less time
+ * than 128 x 128's), 1: always 128 x 128, 2: always 128 x 256.  Results do
+ * not depend on it beyond the fp32 accumulation order of the tensor pipe.
+ * Process-wide; not for use while other threads launch.  REALQ_ERR_INVALID_ARG
+ * for other values.  No counterpart in the paper. */
+realq_status_t realq_set_tensor_tile(int mode);
+
+/* Tuning: the kernel of the column-serial quantize-and-compensate step.  1
+ * (default): warps pipelined through shared-memory progress flags where the
+ * group parameters are taken at the block start or before it; 0: the kernel
+ * whose warps meet at a block-wide barrier after every 32 columns.  Both
+ * perform the same operations in the same order (identical results).
+ * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
+ * the paper. */
+realq_status_t realq_set_quant_kernel(int mode);
+
+/* Tuning: the products of the block ops (realq_block_*, and the window
+ * quantization's loss).  1 (default): tf32x3 tensor-core products where the
+ * operands fit the workspace's plane scratch; 0: fp32 CUDA-core tiles for
+ * all.  Both are fp32-accurate; results differ by fp32 rounding.
+ * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
+ * the paper. */
+realq_status_t realq_set_block_products(int mode);
+
+/* The learning rate of decoder block i (1-based) of L under the paper's
+ * reverse-cosine schedule over transformer blocks (App. "Full Setup",
+ * Eq. reverse_cosine; the first block's rate is 0.01 of the final one, App.
+ * "REAL-Q Learning Rates"):
+ *   eta_i = eta_base + (eta_final - eta_base) sin(pi/2 (i - 1) / (L - 1)),
+ *   eta_base = 0.01 eta_final;  eta_final when L = 1.
+ * Host arithmetic in double; *lr_out (host) receives it.  1 <= i <= L and a
+ * finite lr_final required, else REALQ_ERR_INVALID_ARG. */
+realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out);
+
 /* ---- The next decoder block of the exact two-block sliding window ----
  * Sec. 4.4, Eq. (slide_window): while block l is quantized, the loss blends
  * block l's Fisher loss with block l+1's, and the latter is back-propagated
@@ -507,38 +543,17 @@ void realq_graph_destroy(realq_graph_t graph);
  *   F_next    device fp32 d x d (the next block's Fisher).
  *   loss      device fp32 scalar, or NULL.
  *   ws        device workspace of realq_block_workspace_size(dims, S, L)
- *             bytes, 256-byte aligned; it holds the forward caches.
- * Computed in fp32 with fp32 accumulation (the loss summed in double).
+ *             bytes, 256-byte aligned; it holds the forward caches.  Its
+ *             first int is a status word that each call clears at its start
+ *             and that a timed-out bounded wait of a tensor-core product
+ *             sets (read it with realq_workspace_status).
+ * The projections and products run as fp32-accurate tf32x3 tensor-core
+ * products (operands split into tf32 hi / lo planes, three MMAs per step,
+ * fp32 accumulation); a product whose operand does not fit the workspace's
+ * plane scratch runs on fp32 CUDA-core tiles.  Everything else is fp32 (the
+ * loss summed in double).
  * Asynchronous on `stream`; argument errors are returned before any launch.
  * S L is at most 4194240 tokens.  Outputs may not alias inputs. */
-/* Tuning: the output tile of the fp32-accurate (tf32x3) tensor-core
- * products of Block-GD and the lazy batch update.  0 (default): chosen per
- * launch from its grid (128 x 256 when its waves on the SMs take less time
- * than 128 x 128's), 1: always 128 x 128, 2: always 128 x 256.  Results do
- * not depend on it beyond the fp32 accumulation order of the tensor pipe.
- * Process-wide; not for use while other threads launch.  REALQ_ERR_INVALID_ARG
- * for other values.  No counterpart in the paper. */
-realq_status_t realq_set_tensor_tile(int mode);
-
-/* Tuning: the kernel of the column-serial quantize-and-compensate step.  1
- * (default): warps pipelined through shared-memory progress flags where the
- * group parameters are taken at the block start or before it; 0: the kernel
- * whose warps meet at a block-wide barrier after every 32 columns.  Both
- * perform the same operations in the same order (identical results).
- * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
- * the paper. */
-realq_status_t realq_set_quant_kernel(int mode);
-
-/* The learning rate of decoder block i (1-based) of L under the paper's
- * reverse-cosine schedule over transformer blocks (App. "Full Setup",
- * Eq. reverse_cosine; the first block's rate is 0.01 of the final one, App.
- * "REAL-Q Learning Rates"):
- *   eta_i = eta_base + (eta_final - eta_base) sin(pi/2 (i - 1) / (L - 1)),
- *   eta_base = 0.01 eta_final;  eta_final when L = 1.
- * Host arithmetic in double; *lr_out (host) receives it.  1 <= i <= L and a
- * finite lr_final required, else REALQ_ERR_INVALID_ARG. */
-realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, double *lr_out);
-
 typedef struct {
     int64_t d, n_heads, n_kv, head_dim, ffn;
     float rms_eps;    /* 1e-6 */

@@ -173,7 +173,7 @@ def quantize(w: np.ndarray, scale: np.ndarray, zero: np.ndarray, bits: int = 4):
     return q, _dequant(q, scale, zero).astype(np.float64), margin
 
 
-def _follow_tie(mine: np.ndarray, value: np.ndarray, margin: np.ndarray, other: np.ndarray, tau: float,
+def _follow_tie(mine: np.ndarray, value: np.ndarray, margin: np.ndarray, other: np.ndarray, tau,
                 offset, lo: int, hi: int):
     """Where this run's rounding of `value` is a tie (margin < tau) and another
     run of the sweep took the other neighbour, take that one.  The two
@@ -433,7 +433,9 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
 
     follow: None, or the rounding decisions of another run of the same sweep
     as a dict with "codes" (m x n ints), optionally "zero" (m x ngroups ints)
-    and "tau" (grid steps, default 1e-3).  quant(.) rounds to the nearest
+    and "tau" (grid steps, default 1e-3: a scalar, or an m x n array of
+    per-decision tolerances with "tau_zero" an m x ngroups one for the zero
+    points).  quant(.) rounds to the nearest
     grid point, and where w / scale (or -xmin / scale for the zero point)
     lies within tau of a rounding boundary both neighbours are the correctly
     rounded result up to the rounding of the operands (reading C3 of the
@@ -505,6 +507,10 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
 
     maxq = 2 ** bits - 1
     tau = 1e-3 if follow is None else follow.get("tau", 1e-3)
+    tau_codes = np.broadcast_to(np.asarray(tau, dtype=np.float64), (m, n))
+    tz = None if follow is None else follow.get("tau_zero")
+    tau_zero = np.broadcast_to(np.asarray((tau if np.ndim(tau) == 0 else 1e-3) if tz is None else tz,
+                                          dtype=np.float64), (m, ngroups))
     n_followed = n_followed_zero = 0
     for j in range(n if columns is None else min(int(columns), n)):
         if j % g == 0:
@@ -512,13 +518,13 @@ def realq_sweep(W0, H_sum, T, *, bits=4, group_size=128, block_size=128, symmetr
             scale[:, gi], zero[:, gi], zmargin[:, gi], zf = _grid(W[:, j:j + g], bits, symmetric)
             zfval[:, gi] = zf
             if follow is not None and follow.get("zero") is not None and not symmetric:
-                zero[:, gi], took = _follow_tie(zero[:, gi], zf, zmargin[:, gi], follow["zero"][:, gi], tau, 0,
-                                                0, maxq)
+                zero[:, gi], took = _follow_tie(zero[:, gi], zf, zmargin[:, gi], follow["zero"][:, gi],
+                                                tau_zero[:, gi], 0, 0, maxq)
                 n_followed_zero += int(took.sum())
         gi = j // g
         q, x, mg = _round(W[:, j], scale[:, gi], zero[:, gi], bits)
         if follow is not None:
-            q, took = _follow_tie(q, x, mg, follow["codes"][:, j], tau, zero[:, gi], 0, maxq)
+            q, took = _follow_tie(q, x, mg, follow["codes"][:, j], tau_codes[:, j], zero[:, gi], 0, maxq)
             n_followed += int(took.sum())
         dq = _dequant(q, scale[:, gi], zero[:, gi]).astype(np.float64)
         e = W[:, j] - dq                       # residual delta_j of Eq. (gptq_update)

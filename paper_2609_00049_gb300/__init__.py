@@ -29,7 +29,7 @@ __all__ = [
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
-    "realq_profile_collect", "realq_reverse_cosine_lr", "realq_set_tensor_tile", "realq_set_quant_kernel", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
+    "realq_profile_collect", "realq_reverse_cosine_lr", "realq_set_tensor_tile", "realq_set_quant_kernel", "realq_set_block_products", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
     "realq_block_window", "BLOCK_MODULES", "realq_block_module_workspace_size", "realq_block_head_workspace_size",
     "realq_block_module_window", "realq_block_head_kl", "realq_block_module_kl",
     "realq_quantize_window_workspace_size", "realq_quantize_layer_window", "realq_block_module_inputs",
@@ -143,6 +143,7 @@ _SIGS = {
     "realq_block_workspace_size": ([ctypes.POINTER(BlockDims), _i64, _i64], _sz),
     "realq_set_tensor_tile": ([_int], _int),
     "realq_set_quant_kernel": ([_int], _int),
+    "realq_set_block_products": ([_int], _int),
     "realq_reverse_cosine_lr": ([_i64, _i64, _f64, ctypes.POINTER(ctypes.c_double)], _int),
     "realq_block_forward": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
                              _vp, _sz], _int),
@@ -656,6 +657,12 @@ def realq_set_quant_kernel(mode: int) -> None:
     """Kernel of the column-serial quantizer: 1 pipelined (default), 0 with
     block-wide barriers (identical results)."""
     _check(lib().realq_set_quant_kernel(int(mode)))
+
+
+def realq_set_block_products(mode: int) -> None:
+    """Products of the block ops: 1 tf32x3 tensor cores where the operands fit
+    the workspace's plane scratch (default), 0 fp32 CUDA-core tiles."""
+    _check(lib().realq_set_block_products(int(mode)))
 
 
 def realq_reverse_cosine_lr(i: int, L: int, lr_final: float) -> float:

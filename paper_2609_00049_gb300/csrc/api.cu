@@ -629,6 +629,7 @@ static realq_status_t window_step(cudaStream_t s, SweepPlan &p, int64_t b, void 
     if (w.cfg.B_total > 1) alpha = (float)(1.0 - (double)(b_global - 1) / (double)(w.cfg.B_total - 1));
     float *bl = w.block_loss ? w.block_loss + 2 * b : nullptr;
     const int64_t steps = w.cfg.steps_per_block, k0 = (b_global - 1) * steps;
+    const BlockStatusScope into_sweep(p.status);
     for (int64_t k = 0; k < steps; ++k) {
         // the loss and its gradient at the current weights (the dequantized
         // columns < be and the free ones) on the step's mini-batch

@@ -451,7 +451,9 @@ __global__ void __launch_bounds__(THREADS, 1)
                         for (int q = 0; q < 4; ++q) {
                             if (gj + q >= N) break;
                             float &t = T[rr * TP + cc + q];
-                            if (MODE == TC_STORE) e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] = t;
+                            if (MODE == TC_STORE)
+                                e.C[(int64_t)blockIdx.z * e.czs + gi * e.ldc + gj + q] =
+                                    e.affine ? e.alpha_s * t + (e.R ? e.R[gi * e.ldr + gj + q] : 0.f) : t;
                             else if (MODE == TC_BGD_P) t = bgd_p_value(e, gi, gj + q, t);
                             else if (MODE == TC_BGD_PG) t = bgd_pg_value(e, gi, gj + q, t);
                             else epi_apply(e, gi, gj + q, t);
@@ -795,6 +797,8 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     if (e.mode == TC_SYRK && (a_row0 != 0 || b_row0 != 0 || M != N))
         return fail(REALQ_ERR_INVALID_ARG, "%s: a symmetric update takes a square product from row 0", name);
     if (e.b_tri && kchunk > 0) return fail(REALQ_ERR_INVALID_ARG, "%s: a triangular B takes no K split", name);
+    if (e.affine && (kchunk > 0 || e.mode != TC_STORE))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: the affine store takes no K split", name);
     const MapPair &mp = *reinterpret_cast<const MapPair *>(maps.storage);
     const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));

@@ -17,10 +17,24 @@ __global__ void __launch_bounds__(256) map_kernel(int64_t count, Fn fn) {
 }
 
 // Each step returns nonzero once a launch has failed; the first failure's
-// status is kept and nothing more is launched.
+// status is kept and nothing more is launched.  With plane scratch (planes:
+// four buffers of cap floats) the projections whose shapes the tensor-core
+// path takes run as tf32x3 products on tcgen05: the operands are split into
+// K-major tf32 hi / lo planes (transposed where stored the other way) and
+// C = alpha A B + R is formed in the product's epilogue; the others, and
+// every product without scratch, run on the fp32 CUDA-core tiles.
 struct DevExec {
     cudaStream_t s;
+    float *planes = nullptr;
+    size_t cap = 0;
+    int *err = nullptr;   // status word of the products' bounded waits
     realq_status_t st = REALQ_OK;
+
+    bool tc_ok(const blk::Gemm &g) const {
+        return planes && g.M >= 32 && g.N >= 32 && g.M % 4 == 0 && g.N % 4 == 0 && g.K >= 32 && g.K % 4 == 0 &&
+               (size_t)g.M * g.K <= cap && (size_t)g.N * g.K <= cap && g.M < (1ll << 31) && g.N < (1ll << 31) &&
+               g.K < (1ll << 31);
+    }
 
     template <class Fn>
     int map(int64_t count, const Fn &fn, const char *name) {
@@ -36,6 +50,28 @@ struct DevExec {
 
     int gemm(const blk::Gemm &g, const char *name) {
         if (st != REALQ_OK) return 1;
+        if (tc_ok(g)) {
+            float *Ah = planes, *Al = planes + cap, *Bh = planes + 2 * cap, *Bl = planes + 3 * cap;
+            // A (M x K): rows of A, or A stored K x M (column i of the stored matrix)
+            st = g.a_kmajor ? tc_trans_planes(s, g.K, g.M, g.A, g.lda, Ah, Al, g.K)
+                            : tc_split_rows(s, g.M, g.K, g.A, g.lda, Ah, Al, g.K, g.K);
+            // B (K x N, row-major): its columns as rows of K
+            if (st == REALQ_OK) st = tc_trans_planes(s, g.K, g.N, g.B, g.ldb, Bh, Bl, g.K);
+            TcMaps maps;
+            if (st == REALQ_OK) st = tc_make_maps(&maps, Ah, Al, g.M, g.K, g.K, Bh, Bl, g.N, g.K, g.K);
+            if (st == REALQ_OK) {
+                TcEpi e{};
+                e.mode = TC_STORE;
+                e.C = g.C;
+                e.ldc = g.ldc;
+                e.affine = 1;
+                e.alpha_s = g.alpha;
+                e.R = g.R;
+                e.ldr = g.ldr;
+                st = tc_gemm_tf32x3(s, maps, g.M, g.N, g.K, 0, 0, e, err, name);
+            }
+            return st != REALQ_OK;
+        }
         GemmArgs a{};
         a.M = g.M; a.N = g.N; a.K = g.K;
         a.A = g.A; a.lda = g.lda;
@@ -117,11 +153,55 @@ realq_status_t check_head(const float *gf, const float *Wh, int64_t vocab, const
     return REALQ_OK;
 }
 
+// Every block workspace starts with the tensor-core scratch: a status word
+// (its first int; kAlign bytes) and four operand planes of tc_cap floats,
+// enough for every projection of the block (M K and N K at most
+// max(T, d) max(d, H dh, f)) and, with a head, for the logits product
+// (max(T, V) d).  Products with a larger operand run on the CUDA cores.
+size_t tc_cap(const blk::Dims &dm, int64_t vocab) {
+    const size_t T = (size_t)dm.T(), d = (size_t)dm.d;
+    const size_t wide = std::max(d, std::max((size_t)dm.qw(), (size_t)dm.f));
+    size_t cap = std::max(T, d) * wide;
+    if (vocab > 0) cap = std::max(cap, std::max(T, (size_t)vocab) * d);
+    return (cap + 63) / 64 * 64;   // each plane 256-byte aligned
+}
+
+size_t tc_scratch(const blk::Dims &dm, int64_t vocab) { return kAlign + 4 * blk::rnd(tc_cap(dm, vocab) * 4); }
+
 size_t module_ws(const blk::Dims &dm, int64_t vocab) {
     if (vocab > 0)
-        return blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr) +
+        return tc_scratch(dm, vocab) + blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr) +
                blk::carve_head(dm, vocab, nullptr, nullptr);
-    return 2 * blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr);
+    return tc_scratch(dm, 0) + 2 * blk::carve(dm, nullptr, nullptr) + blk::carve_module(dm, nullptr, nullptr);
+}
+
+size_t block_ws(const blk::Dims &dm) { return tc_scratch(dm, 0) + blk::carve(dm, nullptr, nullptr); }
+
+size_t head_ws(const blk::Dims &dm, int64_t vocab) {
+    return tc_scratch(dm, vocab) + blk::carve_head(dm, vocab, nullptr, nullptr);
+}
+
+// the status word recorded by the block ops' products; the window
+// quantization driver points it at its sweep's own status word for the
+// calls it makes
+thread_local int *g_status_override = nullptr;
+
+int g_block_tc = 1;   // realq_set_block_products
+
+// An executor on the scratch at the start of ws; returns the rest of ws.
+// The status word is cleared at the start of the call unless overridden.
+char *exec_at(DevExec *X, void *ws, const blk::Dims &dm, int64_t vocab) {
+    char *p = static_cast<char *>(ws);
+    X->cap = tc_cap(dm, vocab);
+    X->planes = g_block_tc ? reinterpret_cast<float *>(p + kAlign) : nullptr;
+    if (g_status_override) {
+        X->err = g_status_override;
+    } else {
+        X->err = reinterpret_cast<int *>(p);
+        const cudaError_t r = cudaMemsetAsync(p, 0, sizeof(int), X->s);
+        if (r != cudaSuccess) X->st = fail(REALQ_ERR_CUDA, "block ops: %s", cudaGetErrorString(r));
+    }
+    return p + tc_scratch(dm, vocab);
 }
 
 }  // namespace
@@ -156,6 +236,9 @@ realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_bloc
     return REALQ_OK;
 }
 
+BlockStatusScope::BlockStatusScope(int *status) : prev(g_status_override) { g_status_override = status; }
+BlockStatusScope::~BlockStatusScope() { g_status_override = prev; }
+
 realq_status_t adam_cols(cudaStream_t s, int64_t m, int64_t n, int64_t c0, const float *G, float *W, float *mA,
                          float *vA, float lr, float b1, float b2, float eps, int64_t t, int sgd) {
     const int64_t r = n - c0;
@@ -176,11 +259,17 @@ using namespace realq;
 
 extern "C" {
 
+realq_status_t realq_set_block_products(int mode) {
+    if (mode != 0 && mode != 1) return fail(REALQ_ERR_INVALID_ARG, "set_block_products: mode must be 0 or 1");
+    g_block_tc = mode;
+    return REALQ_OK;
+}
+
 size_t realq_block_workspace_size(const realq_block_dims_t *dims, int64_t S, int64_t L) {
     if (!dims || S <= 0 || L <= 0 || dims->head_dim <= 0) return 0;
     const blk::Dims dm{S, L, dims->d, dims->n_heads, dims->n_kv, dims->head_dim, dims->ffn, dims->rms_eps,
                        dims->rope_base};
-    return blk::carve(dm, nullptr, nullptr);
+    return block_ws(dm);
 }
 
 realq_status_t realq_block_forward(realq_stream_t stream, const realq_block_dims_t *dims,
@@ -189,13 +278,10 @@ realq_status_t realq_block_forward(realq_stream_t stream, const realq_block_dims
     blk::Dims dm{};
     REALQ_TRY(check_block(dims, weights, S, L, "block_forward", &dm));
     if (!x || !y) return fail(REALQ_ERR_INVALID_ARG, "block_forward: NULL x or y");
-    const size_t need = blk::carve(dm, nullptr, nullptr);
-    if (!ws || ws_bytes < need || reinterpret_cast<uintptr_t>(ws) % kAlign)
-        return fail(REALQ_ERR_WORKSPACE, "block_forward: workspace of %zu bytes (%zu-byte aligned) required", need,
-                    kAlign);
-    blk::Buffers B{};
-    blk::carve(dm, ws, &B);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, block_ws(dm), "block_forward"));
     DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::Buffers B{};
+    blk::carve(dm, exec_at(&X, ws, dm, 0), &B);
     const blk::Weights W = weights_of(weights);
     blk::setup(X, dm, W, B);
     blk::forward(X, dm, W, B, x, y);
@@ -209,13 +295,10 @@ realq_status_t realq_block_window(realq_stream_t stream, const realq_block_dims_
     blk::Dims dm{};
     REALQ_TRY(check_block(dims, weights, S, L, "block_window", &dm));
     if (!h_ref || !dh || !F_next || !g_h) return fail(REALQ_ERR_INVALID_ARG, "block_window: NULL argument");
-    const size_t need = blk::carve(dm, nullptr, nullptr);
-    if (!ws || ws_bytes < need || reinterpret_cast<uintptr_t>(ws) % kAlign)
-        return fail(REALQ_ERR_WORKSPACE, "block_window: workspace of %zu bytes (%zu-byte aligned) required", need,
-                    kAlign);
-    blk::Buffers B{};
-    blk::carve(dm, ws, &B);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, block_ws(dm), "block_window"));
     DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::Buffers B{};
+    blk::carve(dm, exec_at(&X, ws, dm, 0), &B);
     const blk::Weights W = weights_of(weights);
     blk::setup(X, dm, W, B);
     blk::window(X, dm, W, B, h_ref, dh, F_next, g_h, loss);
@@ -231,10 +314,10 @@ realq_status_t realq_block_module_inputs(realq_stream_t stream, const realq_bloc
     if (module < blk::M_Q || module > blk::M_DOWN)
         return fail(REALQ_ERR_INVALID_ARG, "%s: module must be 0..6 (q, k, v, o, gate, up, down)", who);
     if (!x || !X_out) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x or X_out", who);
-    REALQ_TRY(check_ws_block(ws, ws_bytes, blk::carve(dm, nullptr, nullptr), who));
-    blk::Buffers B{};
-    blk::carve(dm, ws, &B);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, block_ws(dm), who));
     DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::Buffers B{};
+    blk::carve(dm, exec_at(&X, ws, dm, 0), &B);
     blk::module_input(X, dm, weights_of(weights), B, x, module, X_out);
     return X.st;
 }
@@ -249,7 +332,7 @@ size_t realq_block_module_workspace_size(const realq_block_dims_t *dims, int64_t
 size_t realq_block_head_workspace_size(int64_t d, int64_t S, int64_t L, int64_t vocab) {
     if (d <= 0 || S <= 0 || L <= 0 || vocab <= 0) return 0;
     const blk::Dims dm{S, L, d, 1, 1, 2, 1, 1e-6f, 10000.f};
-    return blk::carve_head(dm, vocab, nullptr, nullptr);
+    return head_ws(dm, vocab);
 }
 
 realq_status_t realq_block_module_window(realq_stream_t stream, const realq_block_dims_t *dims,
@@ -268,13 +351,13 @@ realq_status_t realq_block_module_window(realq_stream_t stream, const realq_bloc
     if (!x || !F_this || !F_next) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x, F_this or F_next", who);
     if (!(alpha >= 0.f && alpha <= 1.f)) return fail(REALQ_ERR_INVALID_ARG, "%s: alpha must be in [0, 1]", who);
     REALQ_TRY(check_ws_block(ws, ws_bytes, module_ws(dm, 0), who));
+    DevExec X{static_cast<cudaStream_t>(stream)};
     blk::Buffers Bl{}, Bn{};
     blk::ModuleBuffers M{};
-    char *p = static_cast<char *>(ws);
+    char *p = exec_at(&X, ws, dm, 0);
     p += blk::carve(dm, p, &Bl);
     p += blk::carve(dm, p, &Bn);
     blk::carve_module(dm, p, &M);
-    DevExec X{static_cast<cudaStream_t>(stream)};
     const blk::Weights Wref = weights_of(this_block);
     const blk::Weights Wcur = weights_of(this_block_hat ? this_block_hat : this_block);
     blk::module_window(X, dm, Wref, blk::with_module(Wcur, module, W_module), weights_of(next_block), Bl, Bn, M, x,
@@ -292,10 +375,10 @@ realq_status_t realq_block_head_kl(realq_stream_t stream, int64_t d, int64_t S, 
     const blk::Dims dm{S, L, d, 1, 1, 2, 1, rms_eps, 10000.f};
     REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
     if (!h_ref || !dh || !g_h) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL h_ref, dh or g_h", who);
-    REALQ_TRY(check_ws_block(ws, ws_bytes, blk::carve_head(dm, vocab, nullptr, nullptr), who));
-    blk::HeadBuffers H{};
-    blk::carve_head(dm, vocab, ws, &H);
+    REALQ_TRY(check_ws_block(ws, ws_bytes, head_ws(dm, vocab), who));
     DevExec X{static_cast<cudaStream_t>(stream)};
+    blk::HeadBuffers H{};
+    blk::carve_head(dm, vocab, exec_at(&X, ws, dm, vocab), &H);
     blk::kl_head(X, dm, blk::Head{gf, Wh, vocab}, H, h_ref, dh, g_h, loss);
     return X.st;
 }
@@ -314,14 +397,14 @@ realq_status_t realq_block_module_kl(realq_stream_t stream, const realq_block_di
     REALQ_TRY(check_head(gf, Wh, vocab, dm, who));
     if (!x) return fail(REALQ_ERR_INVALID_ARG, "%s: NULL x", who);
     REALQ_TRY(check_ws_block(ws, ws_bytes, module_ws(dm, vocab), who));
+    DevExec X{static_cast<cudaStream_t>(stream)};
     blk::Buffers Bl{};
     blk::ModuleBuffers M{};
     blk::HeadBuffers H{};
-    char *p = static_cast<char *>(ws);
+    char *p = exec_at(&X, ws, dm, vocab);
     p += blk::carve(dm, p, &Bl);
     p += blk::carve_module(dm, p, &M);
     blk::carve_head(dm, vocab, p, &H);
-    DevExec X{static_cast<cudaStream_t>(stream)};
     const blk::Weights Wref = weights_of(this_block);
     const blk::Weights Wcur = weights_of(this_block_hat ? this_block_hat : this_block);
     blk::module_kl(X, dm, Wref, blk::with_module(Wcur, module, W_module), Bl, M, blk::Head{gf, Wh, vocab}, H, x,

@@ -63,6 +63,8 @@ struct TcEpi {
     float lr, b1, b2, eps, bc1, bc2; int sgd;
     int64_t czs;                                             // TC_STORE with a K split: C of split z at C + z czs
     int b_tri;   // B(j, k) = 0 for k > j (K range relative to the output column): a CTA's K ends at its last column
+    // TC_STORE without a K split: C = alpha_s acc + R (R nullable, row stride ldr) when affine is set
+    int affine; float alpha_s; const float *R; int64_t ldr;
 };
 // The operand maps of one product, for both tile shapes of the kernel
 // (128 x 128 outputs with 32-wide K slices, 128 x 256 with 16-wide slices).
@@ -155,6 +157,14 @@ realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_bloc
 // One Adam (or SGD) step of Eq. block_gd_update on the columns c0.. of the
 // m x n weights W with a full-width m x n gradient G (the block ops' module
 // gradient): PyTorch-form Adam with bias corrections for step t >= 1.
+// While one lives, the block ops called on this thread record a timed-out
+// wait of their tensor-core products in *status (the caller's status word)
+// instead of the status word at the start of their own workspace.
+struct BlockStatusScope {
+    explicit BlockStatusScope(int *status);
+    ~BlockStatusScope();
+    int *prev;
+};
 realq_status_t adam_cols(cudaStream_t s, int64_t m, int64_t n, int64_t c0, const float *G, float *W, float *mA,
                          float *vA, float lr, float b1, float b2, float eps, int64_t t, int sgd);
 realq_status_t prepare_noalloc(cudaStream_t s, int64_t n, int64_t T, float damp, const float *H, float *U, float *Hbar,

@@ -82,6 +82,7 @@ class OracleSweep:
 # gradient entry whose moments nearly cancel).
 PROBE_K = 10.0
 PROBE_SEEDS = (101, 202)
+PROBE_ROUNDS = 3
 
 
 def probe_eta(m: int, n: int) -> float:
@@ -98,7 +99,10 @@ def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: fl
     own rounding ties.  If codes still differ, the followed run is repeated
     under the sensitivity probe: a remaining mismatch whose margin is within
     PROBE_K times the probes' move of that value is counted as
-    n_conditioned, every other one as unexplained.  Returns (plain result,
+    n_conditioned, every other one as unexplained; while unexplained ones
+    remain, the oracle reruns taking the CUDA path's decision at the
+    conditioned ones too (their tolerance widened to the probes' reach) and
+    compares again, PROBE_ROUNDS probe passes at most.  Returns (plain result,
     followed result, report); the report carries the plain comparison
     (plain_frac_equal, plain_n_mismatch), the decisions followed, and the
     probes' per-group moves of the scales as fol["probe_scale_move"] (the
@@ -130,20 +134,47 @@ def follow_ties(run, gpu_codes: np.ndarray, gpu_zero: np.ndarray = None, tau: fl
     if mism.any() or zmism.any() or scale_off:
         m, n = gpu_codes.shape
         eta = probe_eta(m, n)
-        dx = np.zeros((m, n))
-        dz = np.zeros_like(fol["zf"])
-        ds = np.zeros(fol["scale"].shape)
-        held = {"codes": fol["codes"], "zero": fol["zero"], "tau": 0.5}
-        for seed in PROBE_SEEDS:
-            pr = run(held, grad_noise={"seed": seed, "eta": eta})
-            dx = np.maximum(dx, np.abs(pr["x"] - fol["x"]))
-            dz = np.maximum(dz, np.abs(pr["zf"] - fol["zf"]))
-            ds = np.maximum(ds, np.abs(pr["scale"].astype(np.float64) - fol["scale"].astype(np.float64)))
-        cond = mism & (fol["margin"] <= PROBE_K * dx)
-        zcond = zmism & (fol["zero_margin"] <= PROBE_K * dz)
-        fol = dict(fol, probe_scale_move=ds)
-        rep["n_conditioned"] = int(cond.sum() + zcond.sum())
+        tau_c = np.full((m, n), tau)
+        tau_z = np.full(fol["zero"].shape, tau)
+        raised = np.zeros((m, n), dtype=bool)
+        zraised = np.zeros(fol["zero"].shape, dtype=bool)
+        for it in range(PROBE_ROUNDS):
+            dx = np.zeros((m, n))
+            dz = np.zeros_like(fol["zf"])
+            ds = np.zeros(fol["scale"].shape)
+            held = {"codes": fol["codes"], "zero": fol["zero"], "tau": 0.5}
+            for seed in PROBE_SEEDS:
+                pr = run(held, grad_noise={"seed": seed, "eta": eta})
+                dx = np.maximum(dx, np.abs(pr["x"] - fol["x"]))
+                dz = np.maximum(dz, np.abs(pr["zf"] - fol["zf"]))
+                ds = np.maximum(ds, np.abs(pr["scale"].astype(np.float64) - fol["scale"].astype(np.float64)))
+            cond = mism & (fol["margin"] <= PROBE_K * dx)
+            zcond = zmism & (fol["zero_margin"] <= PROBE_K * dz)
+            fol = dict(fol, probe_scale_move=ds)
+            new, znew = cond & ~raised, zcond & ~zraised
+            if not ((mism & ~cond).any() or (zmism & ~zcond).any()) or not (new.any() or znew.any()) \
+                    or it == PROBE_ROUNDS - 1:
+                break
+            # a mismatch left after the conditioned ones is downstream of one
+            # of them (the rest of its row, every row through Block-GD): the
+            # comparison follows the CUDA path there too, with the decision's
+            # tolerance widened to the probes' reach, and compares again
+            tau_c[new] = np.maximum(tau_c[new], PROBE_K * dx[new] * (1.0 + 1e-9))
+            tau_z[znew] = np.maximum(tau_z[znew], PROBE_K * dz[znew] * (1.0 + 1e-9))
+            raised |= new
+            zraised |= znew
+            fol = run(dict(follow, tau=tau_c, tau_zero=tau_z))
+            mism = gpu_codes != fol["codes"]
+            zmism = np.zeros_like(fol["zero"], dtype=bool) if gpu_zero is None else \
+                np.asarray(gpu_zero, dtype=np.int64) != fol["zero"]
+            rep.update(code_report(gpu_codes, fol, gpu_zero, tau))
+            rep["n_followed"] = int(fol["n_followed"])
+            rep["n_followed_zero"] = int(fol["n_followed_zero"])
+        # every decision the comparison took from the CUDA path beyond the
+        # ties counts, with the mismatches the probes explain in the last run
+        rep["n_conditioned"] = int((raised | cond).sum() + (zraised | zcond).sum())
         rep["n_unexplained"] = int((mism & ~cond).sum() + (zmism & ~zcond).sum())
+        rep["probe_rounds"] = it + 1
     else:
         rep["n_unexplained"] = 0
     return plain, fol, rep

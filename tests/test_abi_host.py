@@ -210,7 +210,11 @@ def test_block_module_and_head_entry_points_reject_bad_arguments(L):
         return L.realq_block_module_window(None, ctypes.byref(ok), ctypes.byref(w), hat, ctypes.byref(w), 2, 8, fake,
                                            None, module, fake, alpha, F, fake, fake, None, fake, nbytes)
 
-    assert rq.realq_block_module_workspace_size(ok, 2, 8) > 2 * rq.realq_block_workspace_size(ok, 2, 8)
+    # every block workspace starts with a status word and four tensor-core
+    # operand planes of max(T, d) max(d, H dh, f) floats (T = 16, d = 64, f = 96)
+    planes = 256 + 4 * max(16, 64) * max(64, 4 * 16, 96) * 4
+    assert rq.realq_block_workspace_size(ok, 2, 8) > planes
+    assert rq.realq_block_module_workspace_size(ok, 2, 8) > 2 * rq.realq_block_workspace_size(ok, 2, 8) - planes
     assert rq.realq_block_module_workspace_size(ok, 2, 8, 1000) > 2 * 8 * 1000 * 8
     assert rq.realq_block_head_workspace_size(64, 2, 8, 1000) > 2 * 8 * 1000 * 8
     assert win(module=7) == rq.REALQ_ERR_INVALID_ARG

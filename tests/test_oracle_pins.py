@@ -426,6 +426,29 @@ def test_following_a_decision_changes_only_its_row_from_there_on():
     assert not np.array_equal(a["deq"][i0, j0:], b["deq"][i0, j0:])
 
 
+def test_per_decision_tolerances_follow_only_where_they_are_wide():
+    # tau as an m x n array: the decision at (i0, j0) may follow (tau 0.5
+    # there), none other may (tau 0), so a run whose codes all differ by one
+    # level changes (i0, j0) and nothing before it in its row or in other rows
+    W0, X = _correlated_case(9, 6, 40, 200)
+    H, T = oracle.hessian_sum([X])
+    a = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8)
+    i0, j0 = 2, 21
+    other = np.where(a["codes"] < 15, a["codes"] + 1, a["codes"] - 1)
+    tau = np.zeros(a["codes"].shape)
+    tau[i0, j0] = 0.5
+    b = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8, follow={"codes": other, "tau": tau})
+    assert b["n_followed"] == 1 and b["codes"][i0, j0] == other[i0, j0]
+    keep = np.ones_like(a["codes"], dtype=bool)
+    keep[i0, j0:] = False
+    assert np.array_equal(a["codes"][keep], b["codes"][keep])
+    # a zero tolerance everywhere follows nothing, whatever the other run says
+    c = oracle.realq_sweep(W0, H, T, group_size=8, block_size=8,
+                           follow={"codes": other, "zero": a["zero"] + 1, "tau": np.zeros_like(tau),
+                                   "tau_zero": np.zeros(a["zero"].shape)})
+    assert c["n_followed"] == 0 and c["n_followed_zero"] == 0 and np.array_equal(a["codes"], c["codes"])
+
+
 # ---------------------------------------------------------------------------
 # Brute force over all int4 codes of a 4 x 8 layer (diagonal Fisher: rows
 # decouple).  The surrogate evaluator agrees with the independent C evaluator;
