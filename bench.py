@@ -143,6 +143,7 @@ def gpu_arm(args, wl, rank, world):
     dev = torch.device("cuda", int(os.environ.get("LOCAL_RANK", 0)))
     torch.cuda.set_device(dev)
     rq.lib()
+    rq.realq_set_bgd_products(args.bgd_products)
     stream = torch.cuda.current_stream()
     dist = None
     if world > 1:
@@ -400,8 +401,24 @@ def work_models(wl, args=None):
         per_step["tok_clip"] = ("hbm", clip_b, "GB/s")
         per_step["tok_xconv"] = ("hbm", conv_b, "GB/s")
         per_step["tok_grad_t"] = ("hbm", gt_b, "GB/s")
-    per_step["bgd_p_gemm"] = ("tf32x3", bgd_p, "TFLOP/s")
-    per_step["bgd_g_gemm_adam"] = ("tf32x3", bgd_g, "TFLOP/s")
+    # the plain Block-GD products run as f16x3 where m, n and the block are
+    # multiples of 8 (and the precision switch is on); the row-grouped,
+    # mini-batch and token forms as tf32x3
+    plain = not (ng or getattr(args, "minibatch_seqs", 0))
+    f16 = plain and getattr(args, "bgd_products", 1) == 1 and wl.block_size % 8 == 0 and all(
+        md.m % 8 == 0 and md.n % 8 == 0 for md in wl.modules)
+    per_step["bgd_p_gemm"] = ("f16x3" if f16 else "tf32x3", bgd_p, "TFLOP/s")
+    per_step["bgd_g_gemm_adam"] = ("f16x3" if f16 else "tf32x3", bgd_g, "TFLOP/s")
+    if f16:
+        # the step's and P^T's fp16 planes, per block: read the fp32 values
+        # twice (row maximum, then split) and write two 2-byte planes
+        f16_split = 0
+        for md in wl.modules:
+            m, n, B = md.m, md.n, wl.block_size
+            for b in range(-(-n // B)):
+                r = n - min((b + 1) * B, n)
+                f16_split += 12 * m * (n - b * B) * (b > 0) + 12 * m * r
+        per_step["f16_split"] = ("hbm", f16_split, "GB/s")
     per_step["trailing_update"] = ("tf32x3", trail, "TFLOP/s")
     per_step["trailing_planes"] = ("hbm", trail_planes, "GB/s")
     per_step["quant_block"] = ("hbm", serial_bytes, "GB/s")
@@ -440,6 +457,13 @@ def roofline_entry(wl, name, launches, ms, steps, peaks, per_step):
         achieved = total / secs / 1e12
         peak = peaks["bf16_tflops_sustained"] * (1.1 / 2.25) / 3.0
         peak_note = f"fp32 via 3 tf32 passes: sustained bf16 x 1.1/2.25 / 3, {peaks['source']}"
+    elif bound == "f16x3":
+        # fp32-accurate contraction as three fp16 tensor passes over
+        # power-of-two row-scaled planes: fp16 runs at the bf16 rate
+        bound = "tensor"
+        achieved = total / secs / 1e12
+        peak = peaks["bf16_tflops_sustained"] / 3.0
+        peak_note = f"fp32 via 3 fp16 passes: sustained bf16 / 3, {peaks['source']}"
     elif bound == "alu":
         achieved = total / secs / 1e12
         peak = fp32_alu_tflops
@@ -559,6 +583,7 @@ def kernel_bench(args):
     from paper_2609_00049_gb300 import build as rqbuild
     rqbuild.build()
     rq.lib()
+    rq.realq_set_bgd_products(args.bgd_products)
     from paper_2609_00049_gb300 import layer
     peaks = load_peaks()
     if args.kernel == "window":
@@ -693,6 +718,8 @@ def main():
                     help="mini-batch Block-GD with this many 2048-token sequences per step (0: full batch)")
     ap.add_argument("--saliency-groups", type=int, default=0,
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
+    ap.add_argument("--bgd-products", type=int, choices=[0, 1], default=1,
+                    help="the plain Block-GD products as f16x3 (1, where the shapes allow) or tf32x3 (0)")
     ap.add_argument("--a-loss-clip", type=float, default=None,
                     help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
     ap.add_argument("--clock-log", default=None, help="directory for the raw clock samples (default: temp dir)")
@@ -709,7 +736,7 @@ def main():
     ap.add_argument("--ffn", type=int, default=3072)
     ap.add_argument("--seqs", type=int, default=2)
     ap.add_argument("--seq-len", type=int, default=2048)
-    ap.add_argument("--block-products", type=int, choices=[0, 1], default=1,
+    ap.add_argument("--block-products", type=int, choices=[0, 1], default=0,
                     help="window: the block ops' products on tf32x3 tensor cores (1) or fp32 CUDA cores (0)")
     ap.add_argument("--n", type=int, default=2048)
     ap.add_argument("--m", type=int, default=1024)

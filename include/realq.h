@@ -312,7 +312,11 @@ realq_status_t realq_scale_moment(realq_stream_t stream, int64_t n, int64_t T_to
  *               P_R = (bgd_disp Hbar)_R + lambda (bgd_disp - (W - W0))_R
  *                     (+ (W0 Dbar)_R),  0 on dead channels,
  *             the same value as ((W - W0) Hbar)_R without its cancellation;
- *             G = F_eff P_R.
+ *             G = F_eff P_R.  Both products run on the tensor cores with
+ *             fp32-level accuracy: as f16x3 (each operand row scaled by a
+ *             power of two and split into fp16 hi / lo planes, three kind::f16
+ *             MMAs per step) when m and n are multiples of 8, else as tf32x3
+ *             (see realq_set_bgd_products).
  *   codes     m x ceil(n/2) bytes, two codes per byte, even column in the low
  *             nibble.  scale (fp32) and zero (uint8): m x ngroups, ngroups =
  *             ceil(n / group_size) (1 when group_size = 0).
@@ -491,19 +495,35 @@ void realq_graph_destroy(realq_graph_t graph);
  * for other values.  No counterpart in the paper. */
 realq_status_t realq_set_tensor_tile(int mode);
 
-/* Tuning: the kernel of the column-serial quantize-and-compensate step.  1
- * (default): warps pipelined through shared-memory progress flags where the
- * group parameters are taken at the block start or before it; 0: the kernel
- * whose warps meet at a block-wide barrier after every 32 columns.  Both
- * perform the same operations in the same order (identical results).
+/* Tuning: the kernel of the column-serial quantize-and-compensate step.  0
+ * (default): the kernel whose warps meet at a block-wide barrier after every
+ * 32 columns; 1: warps pipelined through shared-memory progress flags where
+ * the group parameters are taken at the block start or before it (more
+ * instructions per warp for its polling and chunked updates: slower on
+ * GB300, 41 against 31 us per 8192-row block).  Both perform the same
+ * operations in the same order (identical results).
  * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
  * the paper. */
 realq_status_t realq_set_quant_kernel(int mode);
 
+/* Tuning: the plain Block-GD products (the gradient factor P and G = F_eff P
+ * of realq_quantize_layer and the traced sweep).  1 (default): f16x3 where m
+ * and n are multiples of 8 (fp16 planes with power-of-two row scales: the
+ * same 22 significant bits per operand as tf32x3 at twice the tensor rate);
+ * 0: tf32x3.  The row-grouped, mini-batch and token-form sweeps always take
+ * tf32x3.  Results differ by fp32-level rounding.  Process-wide; read when
+ * a sweep starts.  REALQ_ERR_INVALID_ARG for other values.  No counterpart
+ * in the paper. */
+realq_status_t realq_set_bgd_products(int mode);
+
 /* Tuning: the products of the block ops (realq_block_*, and the window
- * quantization's loss).  1 (default): tf32x3 tensor-core products where the
- * operands fit the workspace's plane scratch; 0: fp32 CUDA-core tiles for
- * all.  Both are fp32-accurate; results differ by fp32 rounding.
+ * quantization's loss).  0 (default): fp32 CUDA-core tiles for all; 1:
+ * tf32x3 tensor-core products where the operands fit the workspace's plane
+ * scratch.  tf32x3 keeps 22 significant bits of each operand against fp32's
+ * 24, and the window's loss (a difference of two forward passes) magnifies
+ * that about tenfold: its gradient moves a few group scales of a window
+ * sweep by more than 1e-5, while the projections are under 1 % of the
+ * window's time (the attention is the rest).
  * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
  * the paper. */
 realq_status_t realq_set_block_products(int mode);
@@ -547,11 +567,9 @@ realq_status_t realq_reverse_cosine_lr(int64_t i, int64_t L, double lr_final, do
  *             first int is a status word that each call clears at its start
  *             and that a timed-out bounded wait of a tensor-core product
  *             sets (read it with realq_workspace_status).
- * The projections and products run as fp32-accurate tf32x3 tensor-core
- * products (operands split into tf32 hi / lo planes, three MMAs per step,
- * fp32 accumulation); a product whose operand does not fit the workspace's
- * plane scratch runs on fp32 CUDA-core tiles.  Everything else is fp32 (the
- * loss summed in double).
+ * Computed in fp32 with fp32 accumulation (the loss summed in double); with
+ * realq_set_block_products(1) the projections and products whose operands
+ * fit the workspace's plane scratch run as tf32x3 tensor-core products.
  * Asynchronous on `stream`; argument errors are returned before any launch.
  * S L is at most 4194240 tokens.  Outputs may not alias inputs. */
 typedef struct {

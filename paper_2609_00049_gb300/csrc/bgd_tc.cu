@@ -53,17 +53,23 @@ constexpr int THREADS = 256;                  // 8 warps; warp 0 lane 0 loads, w
 // the pipe.  A 128 x 256 tile reuses each A row for twice the columns
 // (about 145 bytes per cycle): it takes 16-wide K slices (64-byte rows,
 // 64-byte swizzle) so that a 4-deep ring of both planes still fits.
-template <int TN>
+//
+// With fp16 planes (F16) a slice row holds twice the elements in the same
+// bytes, each MMA (kind::f16, K = 16) advances 32 bytes as a tf32 MMA (K = 8)
+// does, and the f16 rate is twice the tf32 rate: the same kernel at twice the
+// flops per byte of shared memory.
+template <int TN, bool F16 = false>
 struct Tile {
-    static constexpr int KS = TN == 256 ? 16 : 32;            // fp32 per K slice
+    static constexpr int KB = TN == 256 ? 64 : 128;            // bytes per row of a K slice
+    static constexpr int KS = KB / (F16 ? 2 : 4);              // elements per K slice
     static constexpr int STAGES = TN == 256 ? 4 : 3;
     static constexpr uint32_t SWZ = TN == 256 ? tc::SW_64B : tc::SW_128B;
     static constexpr uint32_t SBO = TN == 256 ? 512 : 1024;   // 8 rows of one swizzle atom
-    static constexpr int PLANE_A = TB * KS * 4;
-    static constexpr int PLANE_B = TN * KS * 4;
+    static constexpr int PLANE_A = TB * KB;
+    static constexpr int PLANE_B = TN * KB;
     static constexpr int STAGE_BYTES = 2 * PLANE_A + 2 * PLANE_B;   // A hi, A lo, B hi, B lo
     static constexpr int SMEM = STAGES * STAGE_BYTES + 1024 + 256;
-    static constexpr uint32_t IDESC = tc::idesc_tf32_f32(TB, TN);
+    static constexpr uint32_t IDESC = F16 ? tc::idesc_f16_f32(TB, TN) : tc::idesc_tf32_f32(TB, TN);
     static_assert(STAGES * STAGE_BYTES >= TB * (TN + 1) * 4, "epilogue tile must fit the ring");
 };
 
@@ -234,7 +240,12 @@ __device__ __forceinline__ void adam_rows4(const TcEpi &e, int64_t gi0, int64_t 
         }
         st4(e.Wm + wi, make_float4(w[u].x - st.x, w[u].y - st.y, w[u].z - st.z, w[u].w - st.w));
         st4(e.D + wi, make_float4(d[u].x - st.x, d[u].y - st.y, d[u].z - st.z, d[u].w - st.w));
-        // the displacement moved by -st: its planes feed the next M update
+        // the displacement moved by -st: its planes (or, for f16 planes, -st
+        // itself, split later) feed the next M update
+        if (!e.Sl) {
+            st4(e.Sh + wi, make_float4(-st.x, -st.y, -st.z, -st.w));
+            continue;
+        }
         const float4 sh = make_float4(tc::tf32_hi(-st.x), tc::tf32_hi(-st.y), tc::tf32_hi(-st.z), tc::tf32_hi(-st.w));
         st4(e.Sh + wi, sh);
         st4(e.Sl + wi, make_float4(-st.x - sh.x, -st.y - sh.y, -st.z - sh.z, -st.w - sh.w));
@@ -269,18 +280,23 @@ __device__ __forceinline__ void epi_apply(const TcEpi &e, int64_t i, int64_t j, 
     }
     e.Wm[w] -= step;
     e.D[w] -= step;
+    if (!e.Sl) {
+        e.Sh[w] = -step;
+        return;
+    }
     const float sh = tc::tf32_hi(-step);
     e.Sh[w] = sh;
     e.Sl[w] = -step - sh;
 }
 
 // MODE = e.mode, fixed at compile time: one kernel per epilogue (and so one
-// name per role in a profiler's launch list); TN = the tile's width.
-template <int MODE, int TN>
+// name per role in a profiler's launch list); TN = the tile's width; F16 =
+// fp16 planes with row scales (f16x3) instead of tf32 planes.
+template <int MODE, int TN, bool F16>
 __global__ void __launch_bounds__(THREADS, 1)
-    gemm_tf32x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
+    gemm_x3_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
                        int a_row0, const TcEpi e, int *err, int kchunk, int exact) {
-    using TL = Tile<TN>;
+    using TL = Tile<TN, F16>;
     constexpr int KS = TL::KS, STAGES = TL::STAGES, PLANE_A = TL::PLANE_A, PLANE_B = TL::PLANE_B;
     constexpr int STAGE_BYTES = TL::STAGE_BYTES;
     extern __shared__ uint8_t smem_raw[];
@@ -378,15 +394,21 @@ __global__ void __launch_bounds__(THREADS, 1)
             tc::fence_after_sync();
             const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
 #pragma unroll
-            for (int k = 0; k < KS / 8; ++k) {
-                // K step k: 8 fp32 = 32 bytes into every row of the swizzle atom
+            for (int k = 0; k < TL::KB / 32; ++k) {
+                // K step k: 32 bytes (8 fp32 or 16 fp16) into every row of the swizzle atom
                 const uint64_t ah = tc::smem_desc(base + k * 32, 16, TL::SBO, TL::SWZ);
                 const uint64_t al = tc::smem_desc(base + PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
                 const uint64_t bh = tc::smem_desc(base + 2 * PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
                 const uint64_t bl = tc::smem_desc(base + 2 * PLANE_A + PLANE_B + k * 32, 16, TL::SBO, TL::SWZ);
-                tc::mma_tf32_ss(tmem, ah, bh, TL::IDESC, (it > 0 || k > 0) ? 1u : 0u);
-                if (!(exact & 2)) tc::mma_tf32_ss(tmem, ah, bl, TL::IDESC, 1u);
-                if (!(exact & 1)) tc::mma_tf32_ss(tmem, al, bh, TL::IDESC, 1u);
+                if constexpr (F16) {
+                    tc::mma_f16_ss(tmem, ah, bh, TL::IDESC, (it > 0 || k > 0) ? 1u : 0u);
+                    if (!(exact & 2)) tc::mma_f16_ss(tmem, ah, bl, TL::IDESC, 1u);
+                    if (!(exact & 1)) tc::mma_f16_ss(tmem, al, bh, TL::IDESC, 1u);
+                } else {
+                    tc::mma_tf32_ss(tmem, ah, bh, TL::IDESC, (it > 0 || k > 0) ? 1u : 0u);
+                    if (!(exact & 2)) tc::mma_tf32_ss(tmem, ah, bl, TL::IDESC, 1u);
+                    if (!(exact & 1)) tc::mma_tf32_ss(tmem, al, bh, TL::IDESC, 1u);
+                }
             }
             tc::mma_commit(tc::smem_u32(&empty[s]));
         }
@@ -418,8 +440,18 @@ __global__ void __launch_bounds__(THREADS, 1)
 #pragma unroll
                 for (int q = 0; q < 32; ++q) v[q] = 0u;
             }
+            if (F16 && e.ainv && nk > 0) {
+                // back from the operands' row scales (powers of two: exact)
+                const float sa = i0 + row < M ? e.ainv[i0 + row] : 0.f;
 #pragma unroll
-            for (int q = 0; q < 32; ++q) T[row * TP + c0 + q] = __uint_as_float(v[q]);
+                for (int q = 0; q < 32; ++q) {
+                    const int64_t gj = j0 + c0 + q;
+                    T[row * TP + c0 + q] = gj < N ? __uint_as_float(v[q]) * (sa * e.binv[gj]) : 0.f;
+                }
+            } else {
+#pragma unroll
+                for (int q = 0; q < 32; ++q) T[row * TP + c0 + q] = __uint_as_float(v[q]);
+            }
         }
     }
     __syncthreads();
@@ -474,6 +506,10 @@ __global__ void __launch_bounds__(THREADS, 1)
                 const int64_t gi = i0 + rr;
                 if (gi >= M) break;
                 const float pv = T[rr * TP + cc];
+                if (!e.Ptl) {
+                    e.Pth[gj * e.ldp + gi] = pv;   // split into f16 planes afterwards
+                    continue;
+                }
                 const float hi = tc::tf32_hi(pv);
                 e.Pth[gj * e.ldp + gi] = hi;
                 e.Ptl[gj * e.ldp + gi] = pv - hi;
@@ -503,6 +539,10 @@ __global__ void gsum_adam_kernel(int64_t m, int64_t N, int nz, const float *part
     }
     e.Wm[w] -= st;
     e.D[w] -= st;
+    if (!e.Sl) {
+        e.Sh[w] = -st;
+        return;
+    }
     const float sh = tc::tf32_hi(-st);
     e.Sh[w] = sh;
     e.Sl[w] = -st - sh;
@@ -716,49 +756,134 @@ realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, i
             r = encode_tmap_2d_f32(&m->b_lo, b_lo, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 4, ks, bn, swz);
     }
     if (r != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled (tf32 planes) failed (%d)", (int)r);
+    out->f16 = 0;
+    return REALQ_OK;
+}
+
+realq_status_t tc_make_maps_f16(TcMaps *out, const __half *a_hi, const __half *a_lo, int64_t a_rows, int64_t a_k,
+                                int64_t lda, const __half *b_hi, const __half *b_lo, int64_t b_rows, int64_t b_k,
+                                int64_t ldb) {
+    MapPair *mp = reinterpret_cast<MapPair *>(out->storage);
+    if ((lda & 7) || (ldb & 7) || ((reinterpret_cast<uintptr_t>(a_hi) | reinterpret_cast<uintptr_t>(a_lo) |
+                                    reinterpret_cast<uintptr_t>(b_hi) | reinterpret_cast<uintptr_t>(b_lo)) & 15))
+        return fail(REALQ_ERR_INVALID_ARG, "f16 planes: row strides of 8 elements and 16-byte bases required");
+    CUresult r = CUDA_SUCCESS;
+    // the same byte boxes as the tf32 planes': twice the elements per row
+    for (int w = 0; w < 2 && r == CUDA_SUCCESS; ++w) {
+        Maps *m = w ? &mp->wide : &mp->narrow;
+        const uint32_t ks = w ? Tile<256, true>::KS : Tile<128, true>::KS, bn = w ? 256 : 128;
+        const int swz = w ? 2 : 1;
+        r = encode_tmap_2d_f16(&m->a_hi, a_hi, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 2, ks, TB, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f16(&m->a_lo, a_lo, (uint64_t)a_k, (uint64_t)a_rows, (uint64_t)lda * 2, ks, TB, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f16(&m->b_hi, b_hi, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 2, ks, bn, swz);
+        if (r == CUDA_SUCCESS)
+            r = encode_tmap_2d_f16(&m->b_lo, b_lo, (uint64_t)b_k, (uint64_t)b_rows, (uint64_t)ldb * 2, ks, bn, swz);
+    }
+    if (r != CUDA_SUCCESS) return fail(REALQ_ERR_CUDA, "cuTensorMapEncodeTiled (f16 planes) failed (%d)", (int)r);
+    out->f16 = 1;
     return REALQ_OK;
 }
 
 namespace {
-template <int TN>
-realq_status_t launch_tf32x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
-                             const TcEpi &e, int *err, int a_row0, int kchunk, int exact) {
-    constexpr int SM = Tile<TN>::SMEM;
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_STORE, TN>), SM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_P, TN>), SM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ADAM, TN>), SM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_ACCUM, TN>), SM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_BGD_PG, TN>), SM));
-    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_tf32x3_kernel<TC_SYRK, TN>), SM));
+// One CTA per row: the row's largest magnitude over [c0, c1), the power of
+// two s that puts it in [2^14, 2^15) (from its exponent field; clamped so
+// that s and 1/s are normal floats), then the fp16 planes of s v.  The
+// largest scaled value stays below 2^15 after rounding, within fp16's range.
+__global__ void __launch_bounds__(256) split_f16_rows_kernel(int64_t c0, int64_t c1, const float *x, const float *y,
+                                                             float alpha, int64_t lds, __half *hi, __half *lo,
+                                                             int64_t ldd, float *inv) {
+    __shared__ float red[8];
+    const int64_t r = blockIdx.x;
+    const float *xr = x + r * lds;
+    const float *yr = y ? y + r * lds : nullptr;
+    float mx = 0.f;
+    for (int64_t c = c0 + threadIdx.x; c < c1; c += 256) {
+        const float v = yr ? alpha * xr[c] + (1.f - alpha) * yr[c] : xr[c];
+        mx = fmaxf(mx, fabsf(v));
+    }
+    for (int o = 16; o > 0; o >>= 1) mx = fmaxf(mx, __shfl_xor_sync(0xffffffffu, mx, o));
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = mx;
+    __syncthreads();
+    mx = red[0];
+    for (int w = 1; w < 8; ++w) mx = fmaxf(mx, red[w]);
+    // mx < 2^(e - 126) for biased exponent e: s = 2^(141 - e)
+    const int e = (int)((__float_as_uint(mx) >> 23) & 0xFFu);
+    int k = mx == 0.f ? 0 : 141 - e;
+    k = k < -126 ? -126 : (k > 126 ? 126 : k);
+    const float sc = __uint_as_float((uint32_t)(k + 127) << 23);
+    if (threadIdx.x == 0) inv[r] = __uint_as_float((uint32_t)(127 - k) << 23);
+    __half *hr = hi + r * ldd, *lr = lo + r * ldd;
+    for (int64_t c = c0 + threadIdx.x; c < c1; c += 256) {
+        const float v = (yr ? alpha * xr[c] + (1.f - alpha) * yr[c] : xr[c]) * sc;
+        const __half h = __float2half_rn(v);
+        hr[c] = h;
+        lr[c] = __float2half_rn(v - __half2float(h));
+    }
+}
+
+int g_bgd_products = 1;   // 1: f16x3 for the plain Block-GD products where the shapes allow, 0: tf32x3
+}  // namespace
+
+void bgd_set_products(int mode) { g_bgd_products = mode; }
+int bgd_products() { return g_bgd_products; }
+
+realq_status_t tc_split_f16_rows(cudaStream_t s, int64_t rows, int64_t c0, int64_t c1, const float *x, const float *y,
+                                 float alpha, int64_t lds, __half *hi, __half *lo, int64_t ldd, float *inv) {
+    if (rows <= 0 || c1 <= c0) return REALQ_OK;
+    if (rows > 0x7FFFFFFFll) return fail(REALQ_ERR_INVALID_ARG, "f16 split: too many rows");
+    {
+        Launch L("f16_split", s);
+        split_f16_rows_kernel<<<(unsigned)rows, 256, 0, s>>>(c0, c1, x, y, alpha, lds, hi, lo, ldd, inv);
+    }
+    return check_launch("f16_split");
+}
+
+namespace {
+template <int MODE, int TN, bool F16>
+void launch_mode(cudaStream_t s, const Maps &m, dim3 grid, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
+                 const TcEpi &e, int *err, int a_row0, int kchunk, int exact) {
+    gemm_x3_kernel<MODE, TN, F16><<<grid, THREADS, Tile<TN, F16>::SMEM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e,
+                                                                             err, kchunk, exact);
+}
+
+template <int TN, bool F16>
+realq_status_t launch_x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off, int b_row0,
+                         const TcEpi &e, int *err, int a_row0, int kchunk, int exact) {
+    constexpr int SM = Tile<TN, F16>::SMEM;
     const unsigned nz = kchunk > 0 ? (unsigned)ceil_div(K, kchunk) : 1u;
     const dim3 grid((unsigned)ceil_div(N, TN), (unsigned)ceil_div(M, TB), nz);
-    switch (e.mode) {
-        case TC_STORE:
-            gemm_tf32x3_kernel<TC_STORE, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                       kchunk, exact);
-            break;
-        case TC_BGD_P:
-            gemm_tf32x3_kernel<TC_BGD_P, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                       kchunk, exact);
-            break;
-        case TC_ADAM:
-            gemm_tf32x3_kernel<TC_ADAM, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                      kchunk, exact);
-            break;
-        case TC_ACCUM:
-            gemm_tf32x3_kernel<TC_ACCUM, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                       kchunk, exact);
-            break;
-        case TC_SYRK:
-            gemm_tf32x3_kernel<TC_SYRK, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                      kchunk, exact);
-            break;
-        default:
-            gemm_tf32x3_kernel<TC_BGD_PG, TN><<<grid, THREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err,
-                                                                        kchunk, exact);
-            break;
+    if constexpr (F16) {
+        // the f16x3 products: the plain Block-GD gradient factor, the G
+        // product with its optimizer step, and its K-split slices
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_STORE, TN, true>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_BGD_P, TN, true>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_ADAM, TN, true>), SM));
+        switch (e.mode) {
+            case TC_STORE: launch_mode<TC_STORE, TN, true>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_BGD_P: launch_mode<TC_BGD_P, TN, true>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_ADAM: launch_mode<TC_ADAM, TN, true>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            default: return fail(REALQ_ERR_INVALID_ARG, "f16x3 product: epilogue mode %d not built", e.mode);
+        }
+        return REALQ_OK;
+    } else {
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_STORE, TN, false>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_BGD_P, TN, false>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_ADAM, TN, false>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_ACCUM, TN, false>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_BGD_PG, TN, false>), SM));
+        REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_x3_kernel<TC_SYRK, TN, false>), SM));
+        switch (e.mode) {
+            case TC_STORE: launch_mode<TC_STORE, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_BGD_P: launch_mode<TC_BGD_P, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_ADAM: launch_mode<TC_ADAM, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_ACCUM: launch_mode<TC_ACCUM, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            case TC_SYRK: launch_mode<TC_SYRK, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+            default: launch_mode<TC_BGD_PG, TN, false>(s, m, grid, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact); break;
+        }
+        return REALQ_OK;
     }
-    return REALQ_OK;
 }
 
 int g_tile_mode = 0;   // 0: by the grid (wide_tiles_pay), 1: always 128 x 128, 2: always 128 x 256
@@ -785,14 +910,20 @@ bool wide_tiles_pay(int64_t M, int64_t N, unsigned nz) {
 
 void tc_set_tile_mode(int mode) { g_tile_mode = mode; }
 
-realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
+realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
                               int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk,
                               int exact) {
     if (M <= 0 || N <= 0) return REALQ_OK;
-    if ((k_off & 3) != 0) return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of 4", name);
-    if (kchunk < 0 || (kchunk % Tile<128>::KS) != 0 || (kchunk > 0 && e.mode != TC_STORE))
-        return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name,
-                    Tile<128>::KS);
+    const bool f16 = maps.f16 != 0;
+    // the x coordinate of every TMA box: 16-byte aligned
+    if ((k_off & (f16 ? 7 : 3)) != 0)
+        return fail(REALQ_ERR_INVALID_ARG, "%s: K offset must be a multiple of %d", name, f16 ? 8 : 4);
+    const int ks = f16 ? Tile<128, true>::KS : Tile<128>::KS;
+    if (kchunk < 0 || (kchunk % ks) != 0 || (kchunk > 0 && e.mode != TC_STORE))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: a K split takes a multiple of %d and the store epilogue", name, ks);
+    if (f16 && (e.b_tri || (e.mode != TC_STORE && e.mode != TC_BGD_P && e.mode != TC_ADAM) || !e.ainv || !e.binv))
+        return fail(REALQ_ERR_INVALID_ARG, "%s: f16x3 takes the store, gradient-factor or Adam epilogue with row "
+                    "scales", name);
     if (e.mode < TC_STORE || e.mode > TC_SYRK) return fail(REALQ_ERR_INVALID_ARG, "%s: bad epilogue mode", name);
     if (e.mode == TC_SYRK && (a_row0 != 0 || b_row0 != 0 || M != N))
         return fail(REALQ_ERR_INVALID_ARG, "%s: a symmetric update takes a square product from row 0", name);
@@ -804,8 +935,13 @@ realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));
     {
         Launch L(name, s);
-        if (wide) REALQ_TRY(launch_tf32x3<256>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact));
-        else REALQ_TRY(launch_tf32x3<128>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact));
+        if (f16) {
+            if (wide) REALQ_TRY((launch_x3<256, true>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
+            else REALQ_TRY((launch_x3<128, true>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
+        } else {
+            if (wide) REALQ_TRY((launch_x3<256, false>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
+            else REALQ_TRY((launch_x3<128, false>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
+        }
     }
     return check_launch(name);
 }

@@ -68,7 +68,7 @@ struct DevExec {
                 e.alpha_s = g.alpha;
                 e.R = g.R;
                 e.ldr = g.ldr;
-                st = tc_gemm_tf32x3(s, maps, g.M, g.N, g.K, 0, 0, e, err, name);
+                st = tc_gemm_x3(s, maps, g.M, g.N, g.K, 0, 0, e, err, name);
             }
             return st != REALQ_OK;
         }
@@ -186,7 +186,7 @@ size_t head_ws(const blk::Dims &dm, int64_t vocab) {
 // calls it makes
 thread_local int *g_status_override = nullptr;
 
-int g_block_tc = 1;   // realq_set_block_products
+int g_block_tc = 0;   // realq_set_block_products
 
 // An executor on the scratch at the start of ws; returns the rest of ws.
 // The status word is cleared at the start of the call unless overridden.

@@ -318,6 +318,12 @@ static CUresult encode_tmap_2d(CUtensorMapDataType dt, CUtensorMap *map, const v
                     CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE);
 }
 
+CUresult encode_tmap_2d_f16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
+                            uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle) {
+    return encode_tmap_2d(CU_TENSOR_MAP_DATA_TYPE_FLOAT16, map, base, inner, outer, row_stride_bytes, box_inner,
+                          box_outer, swizzle);
+}
+
 bool hessian_tc_eligible(int64_t n, int64_t T, const void *X) {
     return n >= 64 && n % 8 == 0 && (reinterpret_cast<uintptr_t>(X) & 15) == 0 && T > 0 && T < (1ll << 31) &&
            n < (1ll << 31);

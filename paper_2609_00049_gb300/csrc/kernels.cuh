@@ -65,19 +65,25 @@ struct TcEpi {
     int b_tri;   // B(j, k) = 0 for k > j (K range relative to the output column): a CTA's K ends at its last column
     // TC_STORE without a K split: C = alpha_s acc + R (R nullable, row stride ldr) when affine is set
     int affine; float alpha_s; const float *R; int64_t ldr;
+    // f16x3 maps: the accumulator is in units of the operands' power-of-two
+    // row scales; output (i, j) is acc ainv[i] binv[j] (both null otherwise).
+    // With them, TC_BGD_P writes P^T in fp32 to Pth (Ptl null) and TC_ADAM
+    // the step's negation in fp32 to Sh (Sl null), to be split afterwards.
+    const float *ainv; const float *binv;
 };
 // The operand maps of one product, for both tile shapes of the kernel
 // (128 x 128 outputs with 32-wide K slices, 128 x 256 with 16-wide slices).
 struct TcMaps {
     alignas(64) unsigned char storage[8 * 128];
+    int f16 = 0;   // fp16 planes (f16x3) instead of tf32 planes
 };
 bool tc_gemm_eligible(int64_t m, int64_t n);
 // Tile shape of the tf32x3 products: 0 chosen per launch by its grid, 1 always
 // 128 x 128, 2 always 128 x 256 (process-wide).
 void tc_set_tile_mode(int mode);
-// The column-serial quantizer: 1 the pipelined kernel where the group
-// parameters come at the block start or before it (default), 0 the
-// barrier-phased kernel everywhere (process-wide).
+// The column-serial quantizer: 0 the barrier-phased kernel everywhere
+// (default), 1 the pipelined kernel where the group parameters come at the
+// block start or before it (process-wide).
 void quant_set_kernel(int mode);
 // hi / lo planes of the transpose of the rows x cols block at src (row stride
 // lds): dst[c * ldd + r] for r < rows, c < cols.
@@ -96,10 +102,26 @@ realq_status_t tc_trail_planes(cudaStream_t s, int64_t m, const float *Et, int64
                                int64_t bs, int64_t be, int kb, int B, float *Eh, float *El, float *Ph, float *Pl);
 realq_status_t tc_split(cudaStream_t s, int64_t count, const float *x, const float *y, float alpha, float *hi,
                         float *lo);
+// The maps of an f16x3 product: fp16 hi / lo planes, K-major, row strides
+// lda / ldb (multiples of 8 elements, 16-byte aligned bases).
+realq_status_t tc_make_maps_f16(TcMaps *out, const __half *a_hi, const __half *a_lo, int64_t a_rows, int64_t a_k,
+                                int64_t lda, const __half *b_hi, const __half *b_lo, int64_t b_rows, int64_t b_k,
+                                int64_t ldb);
+// fp16 hi / lo planes of rows of x (or of alpha x + (1 - alpha) y), columns
+// c0 .. c1 - 1 (row stride lds), written at the same columns of hi / lo (row
+// stride ldd), each row scaled by a power of two s_r that puts its largest
+// magnitude in [2^14, 2^15): hi = fp16(s_r v), lo = fp16(s_r v - hi);
+// inv[r] = 1 / s_r.
+realq_status_t tc_split_f16_rows(cudaStream_t s, int64_t rows, int64_t c0, int64_t c1, const float *x, const float *y,
+                                 float alpha, int64_t lds, __half *hi, __half *lo, int64_t ldd, float *inv);
+// Precision of the plain Block-GD products (process-wide): 1 f16x3 where the
+// shapes allow (default), 0 tf32x3 everywhere.
+void bgd_set_products(int mode);
+int bgd_products();
 realq_status_t tc_make_maps(TcMaps *out, const float *a_hi, const float *a_lo, int64_t a_rows, int64_t a_k,
                             int64_t lda, const float *b_hi, const float *b_lo, int64_t b_rows, int64_t b_k,
                             int64_t ldb);
-realq_status_t tc_gemm_tf32x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
+realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
                               int b_row0, const TcEpi &e, int *err, const char *name, int a_row0 = 0, int kchunk = 0,
                               int exact = 0);   // exact & 1: A exact in tf32 (no low plane), & 2: B
 // g = sum_z part[z] (fixed order) and one optimizer step on the m x N block at
@@ -200,6 +222,11 @@ struct SweepPlan {
     // tensor-core path: hi / lo planes and tensor maps
     int tc;
     float *Sh, *Sl, *Hh, *Hl, *Fh, *Fl, *Pth, *Ptl;
+    // f16x3 (the plain Block-GD products): the step and P^T in fp32 in Sh /
+    // Pth, the fp16 hi / lo planes of the step, P^T, H̄ and F_eff in Sl, Ptl,
+    // Hh and Fh, and their row scales' inverses
+    int f16;
+    float *scS, *scF, *scH, *scP;
     float *M;        // M = A H̄ (per row group: A H̄_g), kept current for the free columns
     int64_t step_c;  // first column of the last optimizer step not yet in M (n: none)
     TcMaps mapsP, mapsG;

@@ -501,7 +501,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
                     e.mode = TC_SYRK;
                     e.M = U;
                     e.ldw = n;
-                    REALQ_TRY(tc_gemm_tf32x3(ws_, pmaps[st], kw, kw, NB, 0, 0, e, status_tc, "chol_update_tc"));
+                    REALQ_TRY(tc_gemm_x3(ws_, pmaps[st], kw, kw, NB, 0, 0, e, status_tc, "chol_update_tc"));
                 } else {
                     Launch L("chol_update", ws_);
                     chol_update_kernel<<<(unsigned)nwide, 256, 0, ws_>>>(n, U, k0, kb, 0);
@@ -525,7 +525,7 @@ realq_status_t prepare_impl(cudaStream_t s, int64_t n, double norm, float damp, 
             e.C = panel;
             e.ldc = n;
             e.b_tri = 1;
-            REALQ_TRY(tc_gemm_tf32x3(rs, tmaps, kb, r, r, (int)k1, (int)k1, e, status_tc, "trtri_trmm_tc"));
+            REALQ_TRY(tc_gemm_x3(rs, tmaps, kb, r, r, (int)k1, (int)k1, e, status_tc, "trtri_trmm_tc"));
             // U[K, K+1:] = -U_KK X, U_KK read from A[K, K] (upper, zeros below)
             GemmArgs h{};
             h.M = kb; h.N = r; h.K = kb;

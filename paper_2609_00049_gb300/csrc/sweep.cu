@@ -599,7 +599,7 @@ realq_status_t launch_qb(cudaStream_t s, const QArgs &qa) {
     return check_launch("quant_block");
 }
 
-int g_quant_kernel = 1;   // 1: the pipelined quantizer where it applies, 0: the barrier-phased one
+int g_quant_kernel = 0;   // 0: the barrier-phased quantizer (default), 1: the pipelined one where it applies
 }  // namespace
 
 void quant_set_kernel(int mode) { g_quant_kernel = mode; }
@@ -654,6 +654,7 @@ size_t sweep_ws_bytes(int64_t m, int64_t n, int block, int has_bgd, int has_fnex
         if (block > 0 && tc_gemm_eligible(m, n)) {
             b += 5 * mn + 2 * nn + 2 * align_up((size_t)m * m * sizeof(float));
             b += align_up((size_t)kGSplit * m * block * sizeof(float));
+            b += align_up((size_t)(2 * m + 2 * n) * sizeof(float));   // row scales of the f16 planes
             if (rgroups > 0) b += 2 * mn + 4 * (size_t)rgroups * nn;
             if (nmb > 0) b += (rgroups > 0 ? 0 : 2 * mn) + 2 * (size_t)nmb * nn;
             if (tmb > 0) {
@@ -690,6 +691,8 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
     }
     p.P = p.G = p.Feff = p.R0 = nullptr;
     p.Sh = p.Sl = p.Hh = p.Hl = p.Fh = p.Fl = p.Pth = p.Ptl = p.M = nullptr;
+    p.f16 = 0;
+    p.scS = p.scF = p.scH = p.scP = nullptr;
     p.HGh = p.HGl = p.GGh = p.GGl = p.DWh = p.DWl = p.MBh = p.MBl = nullptr;
     p.lam_g = p.grouped ? cv.take<float>((size_t)p.rgroups) : nullptr;
     p.step_c = p.n;
@@ -707,6 +710,16 @@ void sweep_carve(SweepPlan &p, void *ws, int has_bgd, int has_fnext, int has_dba
             p.Fh = cv.take<float>((size_t)p.m * p.m);
             p.Fl = cv.take<float>((size_t)p.m * p.m);
             p.Gpart = cv.take<float>((size_t)kGSplit * p.m * p.block);
+            float *scl = cv.take<float>((size_t)(2 * p.m + 2 * p.n));
+            // the plain Block-GD products as f16x3 (fp16 planes with row
+            // scales): twice the tf32 rate at the same accuracy; the
+            // row-grouped, mini-batch and token forms keep tf32 planes
+            p.f16 = bgd_products() == 1 && !p.grouped && p.nmb == 0 && p.tmb == 0 && p.m % 8 == 0 && p.n % 8 == 0 &&
+                    p.block % 8 == 0;
+            p.scS = scl;
+            p.scF = scl + p.m;
+            p.scH = scl + 2 * p.m;
+            p.scP = scl + 2 * p.m + p.n;
             if (p.nmb > 0) {
                 p.MBh = cv.take<float>((size_t)p.nmb * p.n * p.n);
                 p.MBl = cv.take<float>((size_t)p.nmb * p.n * p.n);
@@ -843,6 +856,18 @@ static realq_status_t bgd_one(cudaStream_t s, SweepPlan &p, int64_t c0, const fl
     return check_launch("bgd_adam");
 }
 
+// The fp16 planes of the f16x3 products, in the regions of the tf32 ones
+// (each region holds m n, n n or m m floats: room for both fp16 planes).
+static __half *h16(float *region) { return reinterpret_cast<__half *>(region); }
+static __half *S16h(const SweepPlan &p) { return h16(p.Sl); }
+static __half *S16l(const SweepPlan &p) { return h16(p.Sl) + (size_t)p.m * p.n; }
+static __half *P16h(const SweepPlan &p) { return h16(p.Ptl); }
+static __half *P16l(const SweepPlan &p) { return h16(p.Ptl) + (size_t)p.m * p.n; }
+static __half *H16h(const SweepPlan &p) { return h16(p.Hh); }
+static __half *H16l(const SweepPlan &p) { return h16(p.Hh) + (size_t)p.n * p.n; }
+static __half *F16h(const SweepPlan &p) { return h16(p.Fh); }
+static __half *F16l(const SweepPlan &p) { return h16(p.Fh) + (size_t)p.m * p.m; }
+
 // G = F_eff P on the free columns c0.. and one Adam step on them.  On the
 // last step of a block the next block's columns (c0 .. c0 + B) run first, K
 // split into slices whose fixed-order sum takes the step, and the rest (fused
@@ -855,13 +880,17 @@ static realq_status_t g_adam(cudaStream_t s, SweepPlan &p, int64_t c0, bool last
     TcEpi g{};
     g.mode = TC_ADAM;
     g.ldw = p.n; g.col0 = c0;
-    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.Sl;
+    g.Wm = p.W; g.mA = p.adam_m; g.vA = p.adam_v; g.D = p.disp; g.Sh = p.Sh; g.Sl = p.f16 ? nullptr : p.Sl;
+    if (p.f16) {
+        g.ainv = p.scF;
+        g.binv = p.scP;
+    }
     g.lr = p.lr; g.b1 = p.beta1; g.b2 = p.beta2; g.eps = p.eps;
     g.bc1 = (float)(1.0 - std::pow((double)p.beta1, (double)t));
     g.bc2 = (float)(1.0 - std::pow((double)p.beta2, (double)t));
     g.sgd = p.optimizer == REALQ_OPT_SGD;
     const int64_t nb = std::min<int64_t>(p.block, r);
-    if (!last) return tc_gemm_tf32x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
+    if (!last) return tc_gemm_x3(s, p.mapsG, p.m, r, p.m, 0, 0, g, p.status, "bgd_g_gemm_adam");
     // (the split below is the same arithmetic with or without the side
     // stream, so a sweep resumed at any block gives the same bits)
     cudaStream_t ws = (p.wide && r > nb) ? p.wide : s;
@@ -872,17 +901,20 @@ static realq_status_t g_adam(cudaStream_t s, SweepPlan &p, int64_t c0, bool last
     // the next block's columns: few tiles with K = m, so K is split into
     // kGSplit slices (more CTAs, shorter chains), summed in a fixed order by
     // the pass that takes the optimizer step
-    const int kchunk = (int)((ceil_div(p.m, kGSplit) + 31) / 32 * 32);
+    const int ks = p.f16 ? 64 : 32;
+    const int kchunk = (int)((ceil_div(p.m, kGSplit) + ks - 1) / ks * ks);
     const int nz = ceil_div(p.m, kchunk);
     TcEpi st{};
     st.mode = TC_STORE;
     st.C = p.Gpart; st.ldc = nb; st.czs = p.m * nb;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsG, p.m, nb, p.m, 0, 0, st, p.status, "bgd_g_gemm_adam", 0, kchunk));
+    st.ainv = g.ainv; st.binv = g.binv;
+    REALQ_TRY(tc_gemm_x3(s, p.mapsG, p.m, nb, p.m, 0, 0, st, p.status, "bgd_g_gemm_adam", 0, kchunk));
     REALQ_TRY(tc_gsum_adam(s, p.m, nb, nz, p.Gpart, g));
     if (r <= nb) return REALQ_OK;
     TcEpi gw = g;
     gw.col0 = c0 + nb;
-    REALQ_TRY(tc_gemm_tf32x3(ws, p.mapsG, p.m, r - nb, p.m, 0, (int)nb, gw, p.status, "bgd_g_gemm_adam"));
+    if (p.f16) gw.binv = p.scP + nb;
+    REALQ_TRY(tc_gemm_x3(ws, p.mapsG, p.m, r - nb, p.m, 0, (int)nb, gw, p.status, "bgd_g_gemm_adam"));
     if (ws != s) {
         REALQ_CUDA_TRY(cudaEventRecord(p.wide_done, p.wide));
         p.wide_pending = 1;
@@ -952,7 +984,16 @@ static realq_status_t bgd_one_tc(cudaStream_t s, SweepPlan &p, int64_t c0, bool 
     e.Ad = p.disp; e.W = p.W; e.W0 = p.W0; e.w0_bf16 = p.w_dtype == REALQ_BF16;
     e.dead = p.dead; e.lam = p.lam; e.R0 = p.R0; e.ldw = p.n; e.col0 = c0;
     e.Pth = p.Pth; e.Ptl = p.Ptl; e.ldp = p.m; e.M = p.M;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
+    if (p.f16) {
+        // the last step's fp16 planes over its columns [k0, n) (K of this
+        // product); P^T comes out in fp32 and is split for the G product
+        REALQ_TRY(tc_split_f16_rows(s, p.m, k0, p.n, p.Sh, nullptr, 1.f, p.n, S16h(p), S16l(p), p.n, p.scS));
+        e.Ptl = nullptr;
+        e.ainv = p.scS;
+        e.binv = p.scH + c0;
+    }
+    REALQ_TRY(tc_gemm_x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_p_gemm"));
+    if (p.f16) REALQ_TRY(tc_split_f16_rows(s, r, 0, p.m, p.Pth, nullptr, 1.f, p.m, P16h(p), P16l(p), p.m, p.scP));
     REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
     return REALQ_OK;
@@ -979,7 +1020,7 @@ static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c
             TcEpi e{};
             e.mode = TC_ACCUM;
             e.M = p.M + row0 * p.n; e.ldw = p.n; e.col0 = c0;
-            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMg[gr], rows, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm",
+            REALQ_TRY(tc_gemm_x3(s, p.mapsMg[gr], rows, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm",
                                      (int)row0));
         }
         TcEpi q{};
@@ -989,7 +1030,7 @@ static realq_status_t bgd_one_tc_grouped(cudaStream_t s, SweepPlan &p, int64_t c
         q.dead = p.dead_g + (size_t)gr * p.n; q.lam = p.lam_g + gr; q.R0 = p.R0 ? p.R0 + row0 * p.n : nullptr;
         q.ldw = p.n; q.col0 = c0; q.M = p.M + row0 * p.n;
         q.Pth = p.Pth + row0; q.Ptl = p.Ptl + row0; q.ldp = p.m;
-        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsQg[gr], rows, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm", (int)row0));
+        REALQ_TRY(tc_gemm_x3(s, p.mapsQg[gr], rows, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm", (int)row0));
     }
     REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
@@ -1010,7 +1051,7 @@ static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, in
         TcEpi e{};
         e.mode = TC_ACCUM;
         e.M = p.M; e.ldw = p.n; e.col0 = c0;
-        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm"));
+        REALQ_TRY(tc_gemm_x3(s, p.mapsP, p.m, r, p.n - k0, (int)k0, (int)c0, e, p.status, "bgd_m_gemm"));
     }
     TcEpi q{};
     q.mode = TC_BGD_PG;
@@ -1018,7 +1059,7 @@ static realq_status_t bgd_one_tc_mb(cudaStream_t s, SweepPlan &p, int64_t c0, in
     q.dead = p.dead; q.lam = p.lam; q.R0 = nullptr;
     q.ldw = p.n; q.col0 = c0; q.M = p.M;
     q.Pth = p.Pth; q.Ptl = p.Ptl; q.ldp = p.m;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMB[kmb], p.m, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm"));
+    REALQ_TRY(tc_gemm_x3(s, p.mapsMB[kmb], p.m, r, p.n, 0, (int)c0, q, p.status, "bgd_p_gemm"));
     REALQ_TRY(g_adam(s, p, c0, last));
     p.step_c = c0;
     return REALQ_OK;
@@ -1043,12 +1084,12 @@ static realq_status_t bgd_one_tokens(cudaStream_t s, SweepPlan &p, int64_t c0, i
     TcEpi e1{};
     e1.mode = TC_STORE;
     e1.C = p.Dk; e1.ldc = p.m;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT1[kmb], Tk, p.m, p.n, 0, 0, e1, p.status, "tok_residual_gemm", 0, 0, 1));
+    REALQ_TRY(tc_gemm_x3(s, p.mapsT1[kmb], Tk, p.m, p.n, 0, 0, e1, p.status, "tok_residual_gemm", 0, 0, 1));
     REALQ_TRY(tok_clip(s, Tk, p.m, p.Dk, p.rank_q, p.Yh, p.Yl));
     TcEpi e2{};
     e2.mode = TC_STORE;
     e2.C = p.Zk; e2.ldc = p.m;
-    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT2[kmb], Tk, p.m, p.m, 0, 0, e2, p.status, "tok_fisher_gemm"));
+    REALQ_TRY(tc_gemm_x3(s, p.mapsT2[kmb], Tk, p.m, p.m, 0, 0, e2, p.status, "tok_fisher_gemm"));
     REALQ_TRY(tok_gt(s, Tk, p.m, p.Dk, p.Zk, (float)(1.0 / (double)Tk), p.Yh, p.Yl, p.tmb));
     REALQ_CUDA_TRY(cudaMemsetAsync(p.Gc, 0, (size_t)p.m * r * sizeof(float), s));
     TcEpi e3{};
@@ -1056,7 +1097,7 @@ static realq_status_t bgd_one_tokens(cudaStream_t s, SweepPlan &p, int64_t c0, i
     e3.M = p.Gc; e3.ldw = r; e3.col0 = 0;
     constexpr int64_t kChunk = 8192;
     for (int64_t k0 = 0; k0 < Tk; k0 += kChunk)
-        REALQ_TRY(tc_gemm_tf32x3(s, p.mapsT3[kmb], p.m, r, std::min<int64_t>(kChunk, Tk - k0), (int)k0, (int)c0, e3,
+        REALQ_TRY(tc_gemm_x3(s, p.mapsT3[kmb], p.m, r, std::min<int64_t>(kChunk, Tk - k0), (int)k0, (int)c0, e3,
                                  p.status, "tok_grad_gemm", 0, 0, 2));
     const int64_t t = ++(*p.adam_t);
     const double bc1 = 1.0 - std::pow((double)p.beta1, (double)t);
@@ -1165,7 +1206,7 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
             e.M = p.W + row0 * p.n;
             e.ldw = p.n;
             e.col0 = be;
-            REALQ_TRY(tc_gemm_tf32x3(s, p.mapsTr, rows, p.n - be, kb, 0, 0, e, p.status, "trailing_update",
+            REALQ_TRY(tc_gemm_x3(s, p.mapsTr, rows, p.n - be, kb, 0, 0, e, p.status, "trailing_update",
                                      (int)row0));
         }
     }
@@ -1188,8 +1229,11 @@ realq_status_t sweep_block(cudaStream_t s, SweepPlan &p, int64_t b) {
         // F_eff planes: split once for a plain F, per block under the sliding window
         const float a_eff = p.F_next ? alpha : 1.f;
         if (!p.f_split_alpha_valid || p.f_split_alpha != a_eff) {
-            REALQ_TRY(tc_split(s, p.m * p.m, p.F, (p.F_next && a_eff != 1.f) ? p.F_next : nullptr, a_eff, p.Fh,
-                               p.Fl));
+            const float *Fn = (p.F_next && a_eff != 1.f) ? p.F_next : nullptr;
+            if (p.f16)
+                REALQ_TRY(tc_split_f16_rows(s, p.m, 0, p.m, p.F, Fn, a_eff, p.m, F16h(p), F16l(p), p.m, p.scF));
+            else
+                REALQ_TRY(tc_split(s, p.m * p.m, p.F, Fn, a_eff, p.Fh, p.Fl));
             p.f_split_alpha_valid = 1;
             p.f_split_alpha = a_eff;
         }
@@ -1229,9 +1273,16 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
         // planes of H̄ and the tensor maps of both GEMMs; M = A H̄ from the
         // caller's displacement (zero on a fresh sweep; a resumed sweep takes
         // nothing from an earlier workspace)
-        REALQ_TRY(tc_split(s, p.n * p.n, p.Hbar, nullptr, 1.f, p.Hh, p.Hl));
-        REALQ_TRY(tc_make_maps(&p.mapsP, p.Sh, p.Sl, p.m, p.n, p.n, p.Hh, p.Hl, p.n, p.n, p.n));
-        REALQ_TRY(tc_make_maps(&p.mapsG, p.Fh, p.Fl, p.m, p.m, p.m, p.Pth, p.Ptl, p.n, p.m, p.m));
+        if (p.f16) {
+            // (H̄ is symmetric: row j of its planes is column j of H̄)
+            REALQ_TRY(tc_split_f16_rows(s, p.n, 0, p.n, p.Hbar, nullptr, 1.f, p.n, H16h(p), H16l(p), p.n, p.scH));
+            REALQ_TRY(tc_make_maps_f16(&p.mapsP, S16h(p), S16l(p), p.m, p.n, p.n, H16h(p), H16l(p), p.n, p.n, p.n));
+            REALQ_TRY(tc_make_maps_f16(&p.mapsG, F16h(p), F16l(p), p.m, p.m, p.m, P16h(p), P16l(p), p.n, p.m, p.m));
+        } else {
+            REALQ_TRY(tc_split(s, p.n * p.n, p.Hbar, nullptr, 1.f, p.Hh, p.Hl));
+            REALQ_TRY(tc_make_maps(&p.mapsP, p.Sh, p.Sl, p.m, p.n, p.n, p.Hh, p.Hl, p.n, p.n, p.n));
+            REALQ_TRY(tc_make_maps(&p.mapsG, p.Fh, p.Fl, p.m, p.m, p.m, p.Pth, p.Ptl, p.n, p.m, p.m));
+        }
         p.f_split_alpha_valid = 0;
         p.step_c = p.n;
         if (p.grouped) {
@@ -1283,7 +1334,10 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
         if (fresh) {
             REALQ_CUDA_TRY(cudaMemsetAsync(p.M, 0, (size_t)p.m * p.n * sizeof(float), s));
         } else {
-            REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Sh, p.Sl));
+            if (p.f16)
+                REALQ_TRY(tc_split_f16_rows(s, p.m, 0, p.n, p.disp, nullptr, 1.f, p.n, S16h(p), S16l(p), p.n, p.scS));
+            else
+                REALQ_TRY(tc_split(s, p.m * p.n, p.disp, nullptr, 1.f, p.Sh, p.Sl));
             if (p.grouped) {
                 for (int gr = 0; gr < p.rgroups; ++gr) {
                     const int64_t row0 = gr * p.rg_rows, rows = std::min<int64_t>(p.rg_rows, p.m - row0);
@@ -1291,14 +1345,18 @@ realq_status_t sweep_prologue_r0(cudaStream_t s, SweepPlan &p, bool fresh) {
                     TcEpi e{};
                     e.mode = TC_STORE;
                     e.C = p.M + row0 * p.n; e.ldc = p.n;
-                    REALQ_TRY(tc_gemm_tf32x3(s, p.mapsMg[gr], rows, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm",
+                    REALQ_TRY(tc_gemm_x3(s, p.mapsMg[gr], rows, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm",
                                              (int)row0));
                 }
             } else {
                 TcEpi e{};
                 e.mode = TC_STORE;
                 e.C = p.M; e.ldc = p.n;
-                REALQ_TRY(tc_gemm_tf32x3(s, p.mapsP, p.m, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm"));
+                if (p.f16) {
+                    e.ainv = p.scS;
+                    e.binv = p.scH;
+                }
+                REALQ_TRY(tc_gemm_x3(s, p.mapsP, p.m, p.n, p.n, 0, 0, e, p.status, "bgd_m_gemm"));
             }
         }
     }

@@ -124,6 +124,14 @@ __host__ __device__ constexpr uint32_t idesc_tf32_f32(uint32_t M, uint32_t N) {
            | ((N >> 3) << 17) | ((M >> 4) << 24);
 }
 
+// kind::f16 with fp16 operands and fp32 accumulation, both operands K-major.
+__host__ __device__ constexpr uint32_t idesc_f16_f32(uint32_t M, uint32_t N) {
+    return (1u << 4)            // D format: f32
+           | (0u << 7)          // A format: f16
+           | (0u << 10)         // B format: f16
+           | ((N >> 3) << 17) | ((M >> 4) << 24);
+}
+
 __device__ __forceinline__ void mma_tf32_ss(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
                                             uint32_t accumulate) {
     asm volatile(
@@ -158,6 +166,12 @@ __device__ __forceinline__ void mma_bf16_ss(uint32_t tmem_d, uint64_t adesc, uin
         : "memory");
 }
 
+// kind::f16 (the operand type, f16 or bf16, is in the instruction descriptor)
+__device__ __forceinline__ void mma_f16_ss(uint32_t tmem_d, uint64_t adesc, uint64_t bdesc, uint32_t idesc,
+                                           uint32_t accumulate) {
+    mma_bf16_ss(tmem_d, adesc, bdesc, idesc, accumulate);
+}
+
 // Arrive on `bar` once every tcgen05.mma issued so far by this thread is done.
 __device__ __forceinline__ void mma_commit(uint32_t bar) {
     asm volatile("tcgen05.commit.cta_group::1.mbarrier::arrive::one.shared::cluster.b64 [%0];" ::"r"(bar) : "memory");
@@ -184,6 +198,8 @@ CUresult encode_tmap_2d_bf16(CUtensorMap *map, const void *base, uint64_t inner,
                              uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle128);
 // swizzle: 0 none, 1 128-byte, 2 64-byte
 CUresult encode_tmap_2d_f32(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
+                            uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle);
+CUresult encode_tmap_2d_f16(CUtensorMap *map, const void *base, uint64_t inner, uint64_t outer,
                             uint64_t row_stride_bytes, uint32_t box_inner, uint32_t box_outer, int swizzle);
 
 }  // namespace realq

@@ -19,7 +19,8 @@ PROF = {"bgd_g_gemm_adam": (5560, 194.618), "chol_diag": (4480, 145.768), "hessi
         "quant_block": (3200, 97.391), "trtri_panel": (4320, 80.342), "trailing_update": (2920, 67.88),
         "chol_update_tc": (4320, 44.897), "bgd_g_gsum_adam": (2920, 26.335), "hessian_reduce": (160, 17.334),
         "trtri_trmm": (10, 0.5)}
-ARGS = argparse.Namespace(saliency_groups=0, act_bits=0, a_loss_clip=None, minibatch_seqs=0)
+# (the profile was recorded with the Block-GD products as tf32x3)
+ARGS = argparse.Namespace(saliency_groups=0, act_bits=0, a_loss_clip=None, minibatch_seqs=0, bgd_products=0)
 PEAKS = {"hbm_gbs": 6764.0, "bf16_tflops": 1888.7, "bf16_tflops_sustained": 1708.1, "sm_max_mhz": 2070.0,
          "source": "measured"}
 
@@ -36,6 +37,20 @@ def test_dominant_entry():
     assert r["peak"] == pytest.approx(1708.1 * 1.1 / 2.25 / 3)
     assert r["frac"] == pytest.approx(r["achieved"] / r["peak"])
     assert r["traffic"] == bench.NCU_TRAFFIC[("qwen3-0.6b", "bgd_g_gemm_adam")]
+
+
+def test_f16x3_products_take_the_fp16_peak():
+    # with the products as f16x3 the peak is the fp16 (= bf16) tensor rate
+    # over three passes, and the planes' split pass is modelled; the
+    # row-grouped variant keeps tf32x3
+    wl = synth.workloads()["qwen3-0.6b"]
+    a = argparse.Namespace(**{**vars(ARGS), "bgd_products": 1})
+    r = bench.roofline(wl, PROF, 40, PEAKS, a)
+    assert r["kernel"] == "bgd_g_gemm_adam" and r["peak"] == pytest.approx(1708.1 / 3)
+    models = bench.work_models(wl, a)
+    assert models["bgd_p_gemm"][0] == "f16x3" and models["f16_split"][0] == "hbm"
+    g = argparse.Namespace(**{**vars(a), "saliency_groups": 4})
+    assert bench.work_models(wl, g)["bgd_g_gemm_adam"][0] == "tf32x3" and "f16_split" not in bench.work_models(wl, g)
 
 
 def test_table_by_device_time():

@@ -877,6 +877,33 @@ def test_traced_block_losses(with_next):
         assert abs(got[blk, 1] - after) <= 1e-3 * abs(after)
 
 
+# ----------------------------------------------- Block-GD product precision ---
+@pytest.mark.parametrize("products,tile", [(0, 0), (1, 1), (1, 2)])
+def test_bgd_products_match_the_oracle(products, tile):
+    # the plain Block-GD products as tf32x3 (0) and as f16x3 (1, the default
+    # where m, n and the block are multiples of 8: fp16 planes with
+    # power-of-two row scales) on either output tile: shapes no multiple of a
+    # tile, a dead channel, the sliding window with perturbed inputs, bf16
+    # weights, and a sweep resumed mid-way (M rebuilt from the displacement)
+    rq.realq_set_bgd_products(products)
+    rq.realq_set_tensor_tile(tile)
+    try:
+        case = synth.layer_case(27, 200, 328, 1500, outliers=2, dead_cols=(7,))
+        for qkw in (dict(group_size=64, block_size=64), dict(group_size=128, block_size=128)):
+            orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4)
+            _check(orc, out, case, qkw, True, prep=prep, W0=W0, lr=2e-4)
+        case = synth.layer_case(26, 96, 320, 1200, with_next=True, perturbed=True)
+        qkw = dict(group_size=64, block_size=64)
+        orc, out, prep, W0 = _oracle_and_gpu(case, qkw, bgd=2e-4, with_next=True, b_global_start=3, B_total=9,
+                                             use_dbar=True)
+        _check(orc, out, case, qkw, True, lr=2e-4)
+        test_bf16_weights()
+        test_resume_matches_single_call()
+    finally:
+        rq.realq_set_bgd_products(1)
+        rq.realq_set_tensor_tile(0)
+
+
 # ------------------------------------------------- tensor-core tile shapes ---
 @pytest.mark.parametrize("tile", [1, 2])
 def test_tensor_tiles_match_the_oracle(tile):
@@ -924,6 +951,6 @@ def test_quantizer_kernels_agree_bit_for_bit(qkw, m, n):
             outs.append(layer.quantize(dev(case.W0), prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4), F=dev(case.F)))
             torch.cuda.synchronize()
         finally:
-            rq.realq_set_quant_kernel(1)
+            rq.realq_set_quant_kernel(0)
     for k in ("codes", "scale", "zero", "W"):
         assert torch.equal(getattr(outs[0], k), getattr(outs[1], k)), k

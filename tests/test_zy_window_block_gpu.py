@@ -165,9 +165,10 @@ def test_module_window_matches_the_oracle(case, current, module):
 @pytest.mark.parametrize("module", ("q_proj", "down_proj"))
 def test_block_products_on_tensor_cores_agree_with_the_cuda_core_tiles(module):
     # the same module window with the block ops' products as tf32x3 tensor-core
-    # products (default) and on the fp32 CUDA-core tiles: both fp32-accurate,
-    # so the gradients agree to a few fp32 roundings of their scale (the
-    # window's difference of two forward passes amplifies them about tenfold)
+    # products and on the fp32 CUDA-core tiles (default): each within 1e-4 of
+    # the oracle's scale (the window's difference of two forward passes
+    # amplifies the products' rounding about tenfold), so within 1e-4 of each
+    # other
     case = CASES[4]
     S, L, d, H, Hkv, dh, f = case
     r, P, W, dims, _ = _case(9, *case)
@@ -179,7 +180,7 @@ def test_block_products_on_tensor_cores_agree_with_the_cuda_core_tiles(module):
     ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L))
     out = []
     try:
-        for mode in (1, 0):
+        for mode in (1, 0):   # (0 last: the default stays set)
             rq.realq_set_block_products(mode)
             grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
             loss = torch.zeros(1, dtype=torch.float32, device="cuda")
@@ -188,14 +189,14 @@ def test_block_products_on_tensor_cores_agree_with_the_cuda_core_tiles(module):
             rq.realq_workspace_status(ws)
             out.append((grad, loss.item(), rq.realq_launch_count() - n0))
     finally:
-        rq.realq_set_block_products(1)
+        rq.realq_set_block_products(0)
     (g1, l1, n1), (g0, l0, n0) = out
     # the tensor path splits each product's operands into planes first
     assert n1 > n0, (n1, n0)
-    assert abs(l1 - l0) <= 1e-5 * abs(l0), (l1, l0)
+    assert abs(l1 - l0) <= 1e-4 * abs(l0), (l1, l0)
     err = (g1 - g0).abs().max().item() / g0.abs().max().item()
     print(f"\n{module}: tensor vs CUDA-core gradient {err:.2e} of its scale, launches {n1} vs {n0}")
-    assert err <= 2e-5
+    assert err <= 1e-4
 
 
 def test_head_kl_matches_the_oracle():
