@@ -516,6 +516,14 @@ realq_status_t realq_set_quant_kernel(int mode);
  * in the paper. */
 realq_status_t realq_set_bgd_products(int mode);
 
+/* Tuning: the causal attention of the block ops.  1 (default): tiled
+ * kernels (64 rows of a CTA against 32-wide tiles streamed through shared
+ * memory, online softmax; fp32 on the CUDA cores); 0: one thread per query
+ * or key row.  The same arithmetic up to the fp32 summation order.
+ * Process-wide.  REALQ_ERR_INVALID_ARG for other values.  No counterpart in
+ * the paper. */
+realq_status_t realq_set_block_attention(int mode);
+
 /* Tuning: the products of the block ops (realq_block_*, and the window
  * quantization's loss).  0 (default): fp32 CUDA-core tiles for all; 1:
  * tf32x3 tensor-core products where the operands fit the workspace's plane

@@ -16,6 +16,8 @@ __global__ void __launch_bounds__(256) map_kernel(int64_t count, Fn fn) {
     if (i < count) fn(i);
 }
 
+int g_attn_tiled = 1;   // realq_set_block_attention
+
 // Each step returns nonzero once a launch has failed; the first failure's
 // status is kept and nothing more is launched.  With plane scratch (planes:
 // four buffers of cap floats) the projections whose shapes the tensor-core
@@ -45,6 +47,33 @@ struct DevExec {
             map_kernel<<<(unsigned)ceil_div(count, 256), 256, 0, s>>>(count, fn);
         }
         st = check_launch(name);
+        return st != REALQ_OK;
+    }
+
+    // The attention passes run as tiled kernels (attention.cu) unless the
+    // per-row bodies are selected (realq_set_block_attention).
+    int map(int64_t count, const blk::AttnFwd &f, const char *name) {
+        if (!g_attn_tiled) return map<blk::AttnFwd>(count, f, name);
+        if (st != REALQ_OK) return 1;
+        if (count <= 0) return 0;
+        st = attn_fwd_tiled(s, count / (f.a.H * f.a.L), f.a.L, f.a.H, f.a.Hkv, f.a.dh, f.q, f.k, f.v, f.o, f.lse,
+                            name);
+        return st != REALQ_OK;
+    }
+    int map(int64_t count, const blk::AttnBwdQ &f, const char *name) {
+        if (!g_attn_tiled) return map<blk::AttnBwdQ>(count, f, name);
+        if (st != REALQ_OK) return 1;
+        if (count <= 0) return 0;
+        st = attn_bwd_q_tiled(s, count / (f.a.H * f.a.L), f.a.L, f.a.H, f.a.Hkv, f.a.dh, f.q, f.k, f.v, f.go, f.lse,
+                              f.D, f.gq, name);
+        return st != REALQ_OK;
+    }
+    int map(int64_t count, const blk::AttnBwdKV &f, const char *name) {
+        if (!g_attn_tiled) return map<blk::AttnBwdKV>(count, f, name);
+        if (st != REALQ_OK) return 1;
+        if (count <= 0) return 0;
+        st = attn_bwd_kv_tiled(s, count / (f.a.Hkv * f.a.L), f.a.L, f.a.H, f.a.Hkv, f.a.dh, f.q, f.k, f.v, f.go,
+                               f.lse, f.D, f.gk, f.gv, name);
         return st != REALQ_OK;
     }
 
@@ -258,6 +287,12 @@ realq_status_t adam_cols(cudaStream_t s, int64_t m, int64_t n, int64_t c0, const
 using namespace realq;
 
 extern "C" {
+
+realq_status_t realq_set_block_attention(int mode) {
+    if (mode != 0 && mode != 1) return fail(REALQ_ERR_INVALID_ARG, "set_block_attention: mode must be 0 or 1");
+    g_attn_tiled = mode;
+    return REALQ_OK;
+}
 
 realq_status_t realq_set_block_products(int mode) {
     if (mode != 0 && mode != 1) return fail(REALQ_ERR_INVALID_ARG, "set_block_products: mode must be 0 or 1");

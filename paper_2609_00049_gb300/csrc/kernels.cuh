@@ -179,6 +179,16 @@ realq_status_t block_loss_check(const realq_block_dims_t *dims, const realq_bloc
 // One Adam (or SGD) step of Eq. block_gd_update on the columns c0.. of the
 // m x n weights W with a full-width m x n gradient G (the block ops' module
 // gradient): PyTorch-form Adam with bias corrections for step t >= 1.
+// The block ops' causal attention, tiled (attention.cu): the forward (o and
+// lse), the query gradient and the key / value gradients.
+realq_status_t attn_fwd_tiled(cudaStream_t st, int64_t S, int64_t L, int64_t H, int64_t Hkv, int64_t dh,
+                              const float *q, const float *k, const float *v, float *o, float *lse, const char *name);
+realq_status_t attn_bwd_q_tiled(cudaStream_t st, int64_t S, int64_t L, int64_t H, int64_t Hkv, int64_t dh,
+                                const float *q, const float *k, const float *v, const float *go, const float *lse,
+                                const float *D, float *gq, const char *name);
+realq_status_t attn_bwd_kv_tiled(cudaStream_t st, int64_t S, int64_t L, int64_t H, int64_t Hkv, int64_t dh,
+                                 const float *q, const float *k, const float *v, const float *go, const float *lse,
+                                 const float *D, float *gk, float *gv, const char *name);
 // While one lives, the block ops called on this thread record a timed-out
 // wait of their tensor-core products in *status (the caller's status word)
 // instead of the status word at the start of their own workspace.

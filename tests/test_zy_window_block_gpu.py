@@ -199,6 +199,42 @@ def test_block_products_on_tensor_cores_agree_with_the_cuda_core_tiles(module):
     assert err <= 1e-4
 
 
+@pytest.mark.parametrize("case", [(2, 150, 128, 4, 2, 64, 256), (1, 130, 256, 2, 1, 128, 384),
+                                  (1, 70, 256, 2, 2, 256, 256)])
+def test_tiled_attention_matches_the_oracle_and_the_row_bodies(case):
+    # the tiled attention kernels (64-row tiles, 32-wide streamed tiles,
+    # ragged sequence ends, head widths 64 / 128 / 256, grouped and plain
+    # key/value heads) through the module window's forward and backward
+    # passes, against the oracle and against the per-row bodies
+    S, L, d, H, Hkv, dh, f = case
+    r, P, W, dims, _ = _case(11, *case)
+    _, Pn, Wn, _, _ = _case(111, *case)
+    x = _f32(r.standard_normal((S, L, d)))
+    F, Fn = _spd(r, d), _spd(r, d)
+    ws = rq.workspace(rq.realq_block_module_workspace_size(dims, S, L))
+    for module in ("q_proj", "v_proj"):
+        name = ob._MODULE_WEIGHT[module]
+        Wm = _f32(P[name] + 0.05 * r.standard_normal(P[name].shape))
+        want_loss, want_g = ob.sliding_window_module(module, Wm, x, P, Pn, 0.6, F, Fn)
+        out = []
+        try:
+            for tiled in (0, 1):   # (1 last: the default stays set)
+                rq.realq_set_block_attention(tiled)
+                grad = torch.empty(Wm.shape, dtype=torch.float32, device="cuda")
+                loss = torch.zeros(1, dtype=torch.float32, device="cuda")
+                rq.realq_block_module_window(dims, W, Wn, _dev(x), module, _dev(Wm), 0.6, _dev(F), _dev(Fn), grad, ws,
+                                             loss=loss)
+                out.append((grad.cpu().numpy(), loss.item()))
+        finally:
+            rq.realq_set_block_attention(1)
+        for got, got_loss in out:
+            assert abs(got_loss - want_loss) <= 1e-4 * abs(want_loss), (module, got_loss, want_loss)
+            np.testing.assert_allclose(got, want_g, rtol=0, atol=1e-4 * np.abs(want_g).max())
+        gap = np.abs(out[0][0] - out[1][0]).max() / np.abs(want_g).max()
+        print(f"\n{case} {module}: tiled vs per-row attention {gap:.2e} of the gradient's scale")
+        assert gap <= 1e-4
+
+
 def test_head_kl_matches_the_oracle():
     r = np.random.default_rng(5)
     S, L, d, V = 4, 33, 64, 1000
