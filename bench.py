@@ -40,11 +40,6 @@ NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
     ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
-    # the Block-GD G product: per block the next block's columns as a K split
-    # (store epilogue) and the other free columns with the fused Adam step;
-    # 695 launches of a Qwen3-0.6B block over 5 steps, 37.46 MB of DRAM
-    # traffic per launch on average
-    ("qwen3-0.6b", "bgd_g_gemm_adam"): 37455628,
 }
 
 
@@ -309,6 +304,10 @@ def gpu_arm(args, wl, rank, world):
     if rank == 0:
         peaks = load_peaks()
         roof = roofline(wl, prof, prof_steps, peaks, args)
+        # a side measurement outside the timed region: one Block-GD gradient
+        # of the exact two-block window on a decoder-block shape (the sweep
+        # variant whose loss runs through the block ops)
+        window = None if args.no_window else window_measure(args, peaks, 3, 1)
         result = {
             "metric": METRIC, "value": value, "unit": UNIT, "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": ms_total / args.steps, "higher_is_better": True,
@@ -337,7 +336,7 @@ def gpu_arm(args, wl, rank, world):
             "profile_steps": prof_steps if prof else 0,
             "kernels": {k: {"launches": v[0], "ms": round(v[1], 3)} for k, v in
                                            sorted(prof.items(), key=lambda kv: -kv[1][1])},
-            "gpu_launches": int(launches), "clocks": clk, "e2e": e2e,
+            "gpu_launches": int(launches), "clocks": clk, "e2e": e2e, "window": window,
         }
     if dist is not None:
         dist.destroy_process_group()
@@ -636,11 +635,16 @@ def kernel_bench(args):
 
 
 def window_bench(args, peaks):
+    """Prints window_measure's JSON line (--kernel window)."""
+    print(json.dumps(window_measure(args, peaks, args.steps, args.warmup)))
+
+
+def window_measure(args, peaks, steps, warmup):
     """Times one Block-GD gradient of the exact two-block window
     (realq_block_module_window for down_proj: block l's reference and
     current passes, the next block's two passes and its backward, block l's
     backward to the module) on one decoder-block shape, with seeded random
-    weights and inputs.  Prints one JSON line."""
+    weights and inputs.  Returns a dict."""
     import torch
     import paper_2609_00049_gb300 as rq
     d, H, Hkv, dh, f = args.d, args.heads, args.kv_heads, args.head_dim, args.ffn
@@ -672,16 +676,16 @@ def window_bench(args, peaks):
     def run():
         rq.realq_block_module_window(dims, Wl, Wn, x, "down_proj", Wm, 0.5, F, F, grad, ws, loss=loss,
                                      x_hat=x_hat)
-    for _ in range(args.warmup):
+    for _ in range(warmup):
         run()
     torch.cuda.synchronize()
     e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     e0.record(stream)
-    for _ in range(args.steps):
+    for _ in range(steps):
         run()
     e1.record(stream)
     torch.cuda.synchronize()
-    ms = e0.elapsed_time(e1) / args.steps
+    ms = e0.elapsed_time(e1) / steps
     rq.realq_workspace_status(ws)
     # one forward pass: the seven projections and the causal attention
     # (q.k and p.v over half the sequence on average); a backward is about
@@ -697,10 +701,9 @@ def window_bench(args, peaks):
     else:
         peak = 152 * 128 * 2 * peaks.get("sm_max_mhz", 2070.0) * 1e6 / 1e12
         src, bound = "fp32 ALU: 152 SMs x 128 lanes x 2 x max clock", "alu"
-    print(json.dumps({"kernel": "block_module_window", "d": d, "heads": H, "kv_heads": Hkv, "head_dim": dh,
-                      "ffn": f, "seqs": S, "seq_len": L, "block_products": args.block_products,
-                      "ms_per_call": ms, "achieved": tf, "unit": "TFLOP/s", "peak": peak, "frac": tf / peak,
-                      "peak_source": src, "bound": bound}))
+    return {"kernel": "block_module_window", "d": d, "heads": H, "kv_heads": Hkv, "head_dim": dh, "ffn": f,
+            "seqs": S, "seq_len": L, "block_products": args.block_products, "steps": steps, "ms_per_call": ms,
+            "achieved": tf, "unit": "TFLOP/s", "peak": peak, "frac": tf / peak, "peak_source": src, "bound": bound}
 
 
 def main():
@@ -724,6 +727,7 @@ def main():
                     help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
     ap.add_argument("--clock-log", default=None, help="directory for the raw clock samples (default: temp dir)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-window", action="store_true", help="skip the window gradient's side measurement")
     ap.add_argument("--no-profile", action="store_true", help="skip the event-profiled pass")
     ap.add_argument("--no-graph", action="store_true", help="launch the block step eagerly instead of as a CUDA graph")
     ap.add_argument("--kernel", choices=["hessian", "prepare", "sweep", "window"], default=None,

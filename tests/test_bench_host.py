@@ -36,7 +36,8 @@ def test_dominant_entry():
     assert r["achieved"] == pytest.approx(work * 40 / 0.194618 / 1e12)
     assert r["peak"] == pytest.approx(1708.1 * 1.1 / 2.25 / 3)
     assert r["frac"] == pytest.approx(r["achieved"] / r["peak"])
-    assert r["traffic"] == bench.NCU_TRAFFIC[("qwen3-0.6b", "bgd_g_gemm_adam")]
+    # (no counters of the current G kernel for this workload)
+    assert r["traffic"] is bench.NCU_TRAFFIC.get(("qwen3-0.6b", "bgd_g_gemm_adam"))
 
 
 def test_f16x3_products_take_the_fp16_peak():
