@@ -29,7 +29,7 @@ __all__ = [
     "realq_quantize_workspace_size", "realq_bgd_refine", "realq_bgd_workspace_size",
     "realq_surrogate_loss", "realq_surrogate_workspace_size", "realq_workspace_status",
     "realq_status_string", "realq_last_error", "realq_launch_count", "realq_profile_enable",
-    "realq_profile_collect", "realq_reverse_cosine_lr", "realq_set_tensor_tile", "realq_set_quant_kernel", "realq_set_block_products", "realq_set_bgd_products", "realq_set_block_attention", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
+    "realq_profile_collect", "realq_reverse_cosine_lr", "realq_set_tensor_tile", "realq_set_quant_kernel", "realq_set_block_products", "realq_set_bgd_products", "realq_set_tensor_overlap", "realq_set_block_attention", "BlockDims", "block_dims", "realq_block_workspace_size", "realq_block_forward",
     "realq_block_window", "BLOCK_MODULES", "realq_block_module_workspace_size", "realq_block_head_workspace_size",
     "realq_block_module_window", "realq_block_head_kl", "realq_block_module_kl",
     "realq_quantize_window_workspace_size", "realq_quantize_layer_window", "realq_block_module_inputs",
@@ -145,6 +145,7 @@ _SIGS = {
     "realq_set_quant_kernel": ([_int], _int),
     "realq_set_block_products": ([_int], _int),
     "realq_set_bgd_products": ([_int], _int),
+    "realq_set_tensor_overlap": ([_int], _int),
     "realq_set_block_attention": ([_int], _int),
     "realq_reverse_cosine_lr": ([_i64, _i64, _f64, ctypes.POINTER(ctypes.c_double)], _int),
     "realq_block_forward": ([_vp, ctypes.POINTER(BlockDims), ctypes.POINTER(BlockWeights), _i64, _i64, _vp, _vp,
@@ -665,6 +666,12 @@ def realq_set_bgd_products(mode: int) -> None:
     """The plain Block-GD products: 1 f16x3 where m and n are multiples of 8
     (default), 0 tf32x3."""
     _check(lib().realq_set_bgd_products(int(mode)))
+
+
+def realq_set_tensor_overlap(mode: int) -> None:
+    """Wide-tile f16x3 products: 1 persistent with the epilogue overlapped
+    (default), 0 one tile per CTA (identical results)."""
+    _check(lib().realq_set_tensor_overlap(int(mode)))
 
 
 def realq_set_block_attention(mode: int) -> None:

@@ -808,6 +808,12 @@ realq_status_t realq_set_tensor_tile(int mode) {
     return REALQ_OK;
 }
 
+realq_status_t realq_set_tensor_overlap(int mode) {
+    if (mode < 0 || mode > 1) return fail(REALQ_ERR_INVALID_ARG, "set_tensor_overlap: mode 0 or 1");
+    tc_set_overlap(mode);
+    return REALQ_OK;
+}
+
 realq_status_t realq_set_bgd_products(int mode) {
     if (mode < 0 || mode > 1) return fail(REALQ_ERR_INVALID_ARG, "set_bgd_products: mode 0 or 1");
     bgd_set_products(mode);

@@ -522,6 +522,285 @@ __global__ void __launch_bounds__(THREADS, 1)
     if (warp == 0) tc::tmem_dealloc(tmem, TN);
 }
 
+// ---------------------------------------------------------------------------
+// Persistent f16x3 products with the epilogue overlapped (the plain Block-GD
+// G and P products and the K-split slices of the next block's G).  One CTA
+// per SM walks the tiles (t = blockIdx.x, + gridDim.x, ... in the grouped
+// order above, K-split slices last) with three roles: warp 0 issues the TMA
+// loads of the ring, warp 1 the MMAs, and warps 2..9 run the epilogue.  The
+// accumulator is double-buffered in TMEM (2 x 256 columns): while the
+// epilogue warps drain tile t's accumulator, the MMAs of tile t + 1 fill the
+// other one, so the tensor pipe does not wait for the epilogue's global
+// traffic.  The epilogue reads TMEM straight into registers, one output row
+// per thread and 32 consecutive columns per load, and applies the same
+// per-element operations as the tile kernel (the products' bits are the
+// same; the order of the MMAs of a tile is unchanged).  Every wait is
+// bounded; a wait that gives up raises the CTA's abort flag, the roles
+// leave their loops, the MMAs already issued are drained and TMEM is freed.
+constexpr int PTHREADS = 320;
+constexpr int PEPI_WARPS = 8;
+
+__device__ __forceinline__ void persistent_tile(int64_t t, int tiles_m, int tiles_n, int &z, int64_t &i0,
+                                                int64_t &j0) {
+    const int64_t per = (int64_t)tiles_m * tiles_n;
+    z = (int)(t / per);
+    const int64_t pid = t % per;
+    constexpr int64_t GROUP = 8;
+    const int64_t pg = GROUP * tiles_n, first = (pid / pg) * GROUP;
+    const int64_t gm = (tiles_m - first) < GROUP ? (tiles_m - first) : GROUP;
+    i0 = (first + (pid % pg) % gm) * TB;
+    j0 = ((pid % pg) / gm) * 256;
+}
+
+// The epilogue of 8 consecutive columns gj .. gj + 7 of row gi (all inside
+// the output when full, else column by column); v holds the unscaled
+// products, already multiplied by the rows' inverse scales.
+template <int MODE>
+__device__ __forceinline__ void persistent_epi8(const TcEpi &e, int z, int64_t gi, int64_t gj, int64_t N,
+                                                float (&v)[8]) {
+    const bool full = gj + 7 < N;
+    if (MODE == TC_STORE) {
+        float *c = e.C + (int64_t)z * e.czs + gi * e.ldc + gj;
+        if (full) {
+            st4(c, make_float4(v[0], v[1], v[2], v[3]));
+            st4(c + 4, make_float4(v[4], v[5], v[6], v[7]));
+        } else {
+            for (int q = 0; q < 8 && gj + q < N; ++q) c[q] = v[q];
+        }
+        return;
+    }
+    if (MODE == TC_ADAM) {
+        const int64_t w = gi * e.ldw + e.col0 + gj;
+        if (full) {
+            float4 m4[2], v4[2], w4[2], d4[2];
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                if (!e.sgd) {
+                    m4[h] = ld4(e.mA + w + 4 * h);
+                    v4[h] = ld4(e.vA + w + 4 * h);
+                }
+                w4[h] = ld4(e.Wm + w + 4 * h);
+                d4[h] = ld4(e.D + w + 4 * h);
+            }
+#pragma unroll
+            for (int h = 0; h < 2; ++h) {
+                float *mm = reinterpret_cast<float *>(&m4[h]), *vv = reinterpret_cast<float *>(&v4[h]);
+                float *ww = reinterpret_cast<float *>(&w4[h]), *dd = reinterpret_cast<float *>(&d4[h]);
+                float st[4];
+#pragma unroll
+                for (int q = 0; q < 4; ++q) {
+                    float a = e.sgd ? 0.f : mm[q], b = e.sgd ? 0.f : vv[q];
+                    st[q] = adam_step(e, v[4 * h + q], a, b);
+                    mm[q] = a;
+                    vv[q] = b;
+                    ww[q] -= st[q];
+                    dd[q] -= st[q];
+                }
+                if (!e.sgd) {
+                    st4(e.mA + w + 4 * h, m4[h]);
+                    st4(e.vA + w + 4 * h, v4[h]);
+                }
+                st4(e.Wm + w + 4 * h, w4[h]);
+                st4(e.D + w + 4 * h, d4[h]);
+                st4(e.Sh + w + 4 * h, make_float4(-st[0], -st[1], -st[2], -st[3]));
+            }
+        } else {
+            for (int q = 0; q < 8 && gj + q < N; ++q) epi_apply(e, gi, gj + q, v[q]);
+        }
+        return;
+    }
+    // TC_BGD_P: M += acc, P = M + lambda (A - (W - W0)) (+ R0), 0 on dead
+    // channels, written transposed (consecutive lanes: consecutive rows)
+    for (int q = 0; q < 8 && gj + q < N; ++q) e.Pth[(gj + q) * e.ldp + gi] = bgd_p_value(e, gi, gj + q, v[q]);
+}
+
+template <int MODE>
+__global__ void __launch_bounds__(PTHREADS, 1)
+    gemm_f16x3_persistent_kernel(const __grid_constant__ Maps maps, int64_t M, int64_t N, int64_t K, int k_off,
+                                 int b_row0, int a_row0, const TcEpi e, int *err, int kchunk, int tiles_m,
+                                 int tiles_n, int nz) {
+    using TL = Tile<256, true>;
+    constexpr int KS = TL::KS, STAGES = TL::STAGES, PLANE_A = TL::PLANE_A, PLANE_B = TL::PLANE_B;
+    constexpr int STAGE_BYTES = TL::STAGE_BYTES;
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
+    uint64_t *empty = full + STAGES;
+    uint64_t *tfull = empty + STAGES;     // [2]: MMAs of an accumulator done
+    uint64_t *tempty = tfull + 2;         // [2]: the epilogue has read an accumulator
+    uint64_t *drain = tempty + 2;         // the MMA thread's last commit
+    uint32_t *tslot = reinterpret_cast<uint32_t *>(drain + 1);
+    volatile int *abort_flag = reinterpret_cast<volatile int *>(tslot + 1);
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int64_t ntiles = (int64_t)tiles_m * tiles_n * nz;
+    if (threadIdx.x == 0) {
+        for (int s = 0; s < STAGES; ++s) {
+            tc::mbar_init(tc::smem_u32(&full[s]), 1);
+            tc::mbar_init(tc::smem_u32(&empty[s]), 1);
+        }
+        for (int a = 0; a < 2; ++a) {
+            tc::mbar_init(tc::smem_u32(&tfull[a]), 1);
+            tc::mbar_init(tc::smem_u32(&tempty[a]), PEPI_WARPS);
+        }
+        tc::mbar_init(tc::smem_u32(drain), 1);
+        *abort_flag = 0;
+        tc::fence_barrier_init();
+        tc::prefetch_tmap(&maps.a_hi);
+        tc::prefetch_tmap(&maps.a_lo);
+        tc::prefetch_tmap(&maps.b_hi);
+        tc::prefetch_tmap(&maps.b_lo);
+    }
+    if (warp == 0) tc::tmem_alloc(tc::smem_u32(tslot), 512);
+    tc::fence_before_sync();
+    __syncthreads();
+    tc::fence_after_sync();
+    const uint32_t tmem = *tslot;
+
+    if (warp == 0) {
+        if (lane == 0) {
+            // ---------------- TMA producer ----------------
+            uint32_t it = 0;
+            for (int64_t t = blockIdx.x; t < ntiles && !*abort_flag; t += gridDim.x) {
+                int z;
+                int64_t i0, j0;
+                persistent_tile(t, tiles_m, tiles_n, z, i0, j0);
+                const int64_t kz0 = kchunk > 0 ? (int64_t)z * kchunk : 0;
+                const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+                const int nk = (int)((Kz + KS - 1) / KS);
+                for (int kk = 0; kk < nk; ++kk, ++it) {
+                    const int s = (int)(it % STAGES);
+                    const uint32_t r = it / STAGES;
+                    if (!tc::mbar_wait(tc::smem_u32(&empty[s]), (r & 1u) ^ 1u, abort_flag)) {
+                        *abort_flag = 1;
+                        break;
+                    }
+                    const uint32_t fb = tc::smem_u32(&full[s]);
+                    tc::mbar_arrive_expect_tx(fb, STAGE_BYTES);
+                    const int x = k_off + (int)kz0 + kk * KS;
+                    const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
+                    tc::tma_load_2d(base, &maps.a_hi, fb, x, a_row0 + (int)i0);
+                    tc::tma_load_2d(base + PLANE_A, &maps.a_lo, fb, x, a_row0 + (int)i0);
+                    tc::tma_load_2d(base + 2 * PLANE_A, &maps.b_hi, fb, x, b_row0 + (int)j0);
+                    tc::tma_load_2d(base + 2 * PLANE_A + PLANE_B, &maps.b_lo, fb, x, b_row0 + (int)j0);
+                }
+            }
+            if (*abort_flag) {
+                // let the copies in flight land before the CTA leaves
+                int never = 0;
+                for (uint32_t k = (it > (uint32_t)STAGES ? it - STAGES : 0u); k < it; ++k)
+                    tc::mbar_wait(tc::smem_u32(&full[k % STAGES]), (k / STAGES) & 1u, &never, 100000000ull);
+            }
+        }
+    } else if (warp == 1) {
+        if (lane == 0) {
+            // ---------------- MMA issuer ----------------
+            uint32_t it = 0;
+            int lt = 0;
+            for (int64_t t = blockIdx.x; t < ntiles && !*abort_flag; t += gridDim.x, ++lt) {
+                int z;
+                int64_t i0, j0;
+                persistent_tile(t, tiles_m, tiles_n, z, i0, j0);
+                const int64_t kz0 = kchunk > 0 ? (int64_t)z * kchunk : 0;
+                const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+                const int nk = (int)((Kz + KS - 1) / KS);
+                const int acc = lt & 1;
+                // the epilogue has read this accumulator's previous tile
+                if (!tc::mbar_wait(tc::smem_u32(&tempty[acc]), (((uint32_t)lt >> 1) & 1u) ^ 1u, abort_flag)) {
+                    *abort_flag = 1;
+                    break;
+                }
+                tc::fence_after_sync();
+                const uint32_t td = tmem + (uint32_t)(acc * 256);
+                bool ok = true;
+                for (int kk = 0; kk < nk; ++kk, ++it) {
+                    const int s = (int)(it % STAGES);
+                    const uint32_t r = it / STAGES;
+                    if (!tc::mbar_wait(tc::smem_u32(&full[s]), r & 1u, abort_flag)) {
+                        ok = false;
+                        break;
+                    }
+                    tc::fence_after_sync();
+                    const uint32_t base = tc::smem_u32(smem + s * STAGE_BYTES);
+#pragma unroll
+                    for (int k = 0; k < TL::KB / 32; ++k) {
+                        const uint64_t ah = tc::smem_desc(base + k * 32, 16, TL::SBO, TL::SWZ);
+                        const uint64_t al = tc::smem_desc(base + PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
+                        const uint64_t bh = tc::smem_desc(base + 2 * PLANE_A + k * 32, 16, TL::SBO, TL::SWZ);
+                        const uint64_t bl = tc::smem_desc(base + 2 * PLANE_A + PLANE_B + k * 32, 16, TL::SBO, TL::SWZ);
+                        tc::mma_f16_ss(td, ah, bh, TL::IDESC, (kk > 0 || k > 0) ? 1u : 0u);
+                        tc::mma_f16_ss(td, ah, bl, TL::IDESC, 1u);
+                        tc::mma_f16_ss(td, al, bh, TL::IDESC, 1u);
+                    }
+                    tc::mma_commit(tc::smem_u32(&empty[s]));
+                }
+                if (!ok) {
+                    *abort_flag = 1;
+                    break;
+                }
+                // (K = 0: no MMA; the epilogue reads zeros for nk = 0)
+                if (nk > 0) tc::mma_commit(tc::smem_u32(&tfull[acc]));
+                else tc::mbar_arrive(tc::smem_u32(&tfull[acc]));
+            }
+            // every MMA issued has retired before TMEM is freed
+            tc::mma_commit(tc::smem_u32(drain));
+            int never = 0;
+            tc::mbar_wait(tc::smem_u32(drain), 0u, &never, 100000000ull);
+        }
+    } else {
+        // ---------------- epilogue (warps 2..9) ----------------
+        const int quarter = warp & 3, half = (warp - 2) >> 2;
+        const int row = quarter * 32 + lane;
+        int lt = 0;
+        for (int64_t t = blockIdx.x; t < ntiles; t += gridDim.x, ++lt) {
+            int z;
+            int64_t i0, j0;
+            persistent_tile(t, tiles_m, tiles_n, z, i0, j0);
+            const int64_t kz0 = kchunk > 0 ? (int64_t)z * kchunk : 0;
+            const int64_t Kz = kchunk > 0 ? ((K - kz0) < kchunk ? (K - kz0) : kchunk) : K;
+            const int acc = lt & 1;
+            // (the warp agrees on the outcome: its TMEM loads are warp-wide)
+            const bool got = tc::mbar_wait(tc::smem_u32(&tfull[acc]), ((uint32_t)lt >> 1) & 1u, abort_flag);
+            if (!__all_sync(0xffffffffu, got)) {
+                *abort_flag = 1;
+                break;
+            }
+            tc::fence_after_sync();
+            const int64_t gi = i0 + row;
+            // (K = 0: nothing was issued into the accumulator; the products are 0)
+            const bool none = Kz <= 0;
+            const float sa = (gi < M && !none) ? e.ainv[gi] : 0.f;
+#pragma unroll 1
+            for (int c0 = half * 128; c0 < half * 128 + 128; c0 += 32) {
+                uint32_t v[32];
+                tc::tmem_ld_32x32b_x32(tmem + ((uint32_t)(quarter * 32) << 16) + (uint32_t)(acc * 256 + c0), v);
+                if (c0 == half * 128 + 96) {
+                    // this warp's last read of the accumulator: hand it back
+                    tc::fence_before_sync();
+                    __syncwarp();
+                    if (lane == 0) tc::mbar_arrive(tc::smem_u32(&tempty[acc]));
+                }
+                if (gi >= M) continue;
+#pragma unroll
+                for (int g8 = 0; g8 < 32; g8 += 8) {
+                    const int64_t gj = j0 + c0 + g8;
+                    if (gj >= N) break;
+                    float x[8];
+#pragma unroll
+                    for (int q = 0; q < 8; ++q)
+                        x[q] = (gj + q < N && !none) ? __uint_as_float(v[g8 + q]) * (sa * e.binv[gj + q]) : 0.f;
+                    persistent_epi8<MODE>(e, z, gi, gj, N, x);
+                }
+            }
+        }
+    }
+    __syncwarp();
+    tc::fence_before_sync();
+    __syncthreads();
+    if (threadIdx.x == 0 && *abort_flag && err) atomicOr(err, ST_TIMEOUT);
+    if (warp == 0) tc::tmem_dealloc(tmem, 512);
+}
+
 // g = sum over the K splits (z = 0, 1, ... in order), then the TC_ADAM
 // epilogue on element (i, j) of the m x N block at column e.col0
 __global__ void gsum_adam_kernel(int64_t m, int64_t N, int nz, const float *part, const TcEpi e) {
@@ -887,6 +1166,36 @@ realq_status_t launch_x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N, in
 }
 
 int g_tile_mode = 0;   // 0: by the grid (wide_tiles_pay), 1: always 128 x 128, 2: always 128 x 256
+int g_overlap = 1;     // the persistent f16x3 kernel for wide-tile f16x3 products
+
+int sm_count() {
+    static int sms = 0;
+    if (sms == 0) {
+        int dev = 0, c = 0;
+        if (cudaGetDevice(&dev) == cudaSuccess &&
+            cudaDeviceGetAttribute(&c, cudaDevAttrMultiProcessorCount, dev) == cudaSuccess && c > 0)
+            sms = c;
+    }
+    return sms;
+}
+
+template <int MODE>
+realq_status_t launch_persistent(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off,
+                                 int b_row0, const TcEpi &e, int *err, int a_row0, int kchunk) {
+    constexpr int SM = Tile<256, true>::SMEM;
+    REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_f16x3_persistent_kernel<MODE>), SM));
+    const int64_t tiles_m = ceil_div(M, TB), tiles_n = ceil_div(N, 256);
+    const int64_t nz = kchunk > 0 ? ceil_div(K, kchunk) : 1;
+    const int64_t ntiles = tiles_m * tiles_n * nz;
+    const int sms = sm_count();
+    if (sms <= 0) return fail(REALQ_ERR_CUDA, "persistent product: no SM count");
+    if (tiles_m > 0x7FFFFFFF || tiles_n > 0x7FFFFFFF || nz > 0x7FFFFFFF)
+        return fail(REALQ_ERR_UNSUPPORTED, "persistent product: too many tiles");
+    const unsigned grid = (unsigned)(ntiles < sms ? ntiles : sms);
+    gemm_f16x3_persistent_kernel<MODE><<<grid, PTHREADS, SM, s>>>(m, M, N, K, k_off, b_row0, a_row0, e, err, kchunk,
+                                                                  (int)tiles_m, (int)tiles_n, (int)nz);
+    return REALQ_OK;
+}
 
 // The 128 x 256 tile does twice a narrow tile's work in about 1.55 narrow
 // tile times (its measured rate over the narrow one's, at the shared-memory
@@ -909,6 +1218,7 @@ bool wide_tiles_pay(int64_t M, int64_t N, unsigned nz) {
 }  // namespace
 
 void tc_set_tile_mode(int mode) { g_tile_mode = mode; }
+void tc_set_overlap(int mode) { g_overlap = mode; }
 
 realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t N, int64_t K, int k_off,
                               int b_row0, const TcEpi &e, int *err, const char *name, int a_row0, int kchunk,
@@ -935,7 +1245,13 @@ realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));
     {
         Launch L(name, s);
-        if (f16) {
+        if (f16 && wide && g_overlap) {
+            switch (e.mode) {
+                case TC_STORE: REALQ_TRY(launch_persistent<TC_STORE>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
+                case TC_BGD_P: REALQ_TRY(launch_persistent<TC_BGD_P>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
+                default: REALQ_TRY(launch_persistent<TC_ADAM>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
+            }
+        } else if (f16) {
             if (wide) REALQ_TRY((launch_x3<256, true>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
             else REALQ_TRY((launch_x3<128, true>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
         } else {

@@ -904,6 +904,34 @@ def test_bgd_products_match_the_oracle(products, tile):
         rq.realq_set_tensor_tile(0)
 
 
+@pytest.mark.parametrize("qkw,m,n,bf16", [(dict(group_size=128, block_size=128), 200, 328, False),
+                                          (dict(group_size=64, block_size=64), 1024, 1536, True),
+                                          (dict(group_size=128, block_size=128), 512, 2048, False)])
+def test_persistent_products_are_bit_identical(qkw, m, n, bf16):
+    # the wide-tile f16x3 products as persistent kernels (the epilogue of one
+    # tile overlapping the next tile's MMAs, two TMEM accumulators) and as one
+    # tile per CTA: the same MMAs per tile and the same epilogue arithmetic,
+    # so the whole sweep with Block-GD (ragged tiles, several tiles per CTA,
+    # the K-split store of the next block's columns) gives the same bits
+    case = synth.layer_case(79, m, n, 2 * n, outliers=2, bf16=bf16)
+    H, _, T = layer.accumulate([dev(case.Xhat)], n)
+    prep = layer.prepare(H, T)
+    W0 = dev(case.W0, torch.bfloat16) if bf16 else dev(case.W0)
+    outs = []
+    rq.realq_set_tensor_tile(2)
+    try:
+        for mode in (0, 1):   # (1 last: the default stays set)
+            rq.realq_set_tensor_overlap(mode)
+            outs.append(layer.quantize(W0, prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4, steps_per_block=2),
+                                       F=dev(case.F)))
+            torch.cuda.synchronize()
+    finally:
+        rq.realq_set_tensor_overlap(1)
+        rq.realq_set_tensor_tile(0)
+    for k in ("codes", "scale", "zero", "W"):
+        assert torch.equal(getattr(outs[0], k), getattr(outs[1], k)), k
+
+
 # ------------------------------------------------- tensor-core tile shapes ---
 @pytest.mark.parametrize("tile", [1, 2])
 def test_tensor_tiles_match_the_oracle(tile):
