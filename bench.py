@@ -139,6 +139,7 @@ def gpu_arm(args, wl, rank, world):
     torch.cuda.set_device(dev)
     rq.lib()
     rq.realq_set_bgd_products(args.bgd_products)
+    rq.realq_set_tensor_overlap(args.tensor_overlap)
     stream = torch.cuda.current_stream()
     dist = None
     if world > 1:
@@ -583,6 +584,7 @@ def kernel_bench(args):
     rqbuild.build()
     rq.lib()
     rq.realq_set_bgd_products(args.bgd_products)
+    rq.realq_set_tensor_overlap(args.tensor_overlap)
     from paper_2609_00049_gb300 import layer
     peaks = load_peaks()
     if args.kernel == "window":
@@ -723,6 +725,9 @@ def main():
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--bgd-products", type=int, choices=[0, 1], default=1,
                     help="the plain Block-GD products as f16x3 (1, where the shapes allow) or tf32x3 (0)")
+    ap.add_argument("--tensor-overlap", type=int, choices=[0, 1], default=1,
+                    help="wide-tile f16x3 products as persistent kernels with the epilogue overlapped (1) or one "
+                         "tile per CTA (0)")
     ap.add_argument("--a-loss-clip", type=float, default=None,
                     help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
     ap.add_argument("--clock-log", default=None, help="directory for the raw clock samples (default: temp dir)")
