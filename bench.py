@@ -40,6 +40,11 @@ NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
     ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
+    # the f16x3 G product of the LLaMA-3.1-70B block: three fused-Adam
+    # launches of down_proj captured in the bench step (one-pass DRAM
+    # counters: 14.28-14.50 GB each, 4.64 GB per TFLOP), scaled to the
+    # family's average launch (1.128 TFLOP)
+    ("llama3.1-70b", "bgd_g_gemm_adam"): 5234000000,
 }
 
 
