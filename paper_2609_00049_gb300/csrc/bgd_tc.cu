@@ -552,66 +552,77 @@ __device__ __forceinline__ void persistent_tile(int64_t t, int tiles_m, int tile
     j0 = ((pid % pg) / gm) * 256;
 }
 
-// The epilogue of 8 consecutive columns gj .. gj + 7 of row gi (all inside
-// the output when full, else column by column); v holds the unscaled
-// products, already multiplied by the rows' inverse scales.
+constexpr int PSTAGES = 3;             // ring stages (the rest of shared memory stages the epilogue)
+constexpr int PSTAGE_PITCH = 33;       // a warp's 32 x 32 staging block, padded
+
+// One 32 x 32 block of the output (rows gi0 .., columns gj0 ..), staged in
+// st[r * 33 + c] (row r, column c) by the warp that drained it from TMEM:
+// the lanes walk columns, so that the global accesses of a row coalesce.
+// Rows at or past M and columns at or past N are skipped.
 template <int MODE>
-__device__ __forceinline__ void persistent_epi8(const TcEpi &e, int z, int64_t gi, int64_t gj, int64_t N,
-                                                float (&v)[8]) {
-    const bool full = gj + 7 < N;
+__device__ __forceinline__ void persistent_block(const TcEpi &e, int z, int64_t gi0, int64_t gj0, int64_t M,
+                                                 int64_t N, float *st, int lane) {
+    const int64_t gj = gj0 + lane;
+    const bool col_ok = gj < N;
     if (MODE == TC_STORE) {
-        float *c = e.C + (int64_t)z * e.czs + gi * e.ldc + gj;
-        if (full) {
-            st4(c, make_float4(v[0], v[1], v[2], v[3]));
-            st4(c + 4, make_float4(v[4], v[5], v[6], v[7]));
-        } else {
-            for (int q = 0; q < 8 && gj + q < N; ++q) c[q] = v[q];
+#pragma unroll 4
+        for (int r = 0; r < 32; ++r) {
+            const int64_t gi = gi0 + r;
+            if (gi < M && col_ok) e.C[(int64_t)z * e.czs + gi * e.ldc + gj] = st[r * PSTAGE_PITCH + lane];
         }
         return;
     }
     if (MODE == TC_ADAM) {
-        const int64_t w = gi * e.ldw + e.col0 + gj;
-        if (full) {
-            float4 m4[2], v4[2], w4[2], d4[2];
+        // four rows at a time: their loads are issued before any store
+        for (int r0 = 0; r0 < 32; r0 += 4) {
+            float mv[4], vv[4], wv[4], dv[4];
+            int64_t w[4];
+            bool ok[4];
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                if (!e.sgd) {
-                    m4[h] = ld4(e.mA + w + 4 * h);
-                    v4[h] = ld4(e.vA + w + 4 * h);
+            for (int u = 0; u < 4; ++u) {
+                const int64_t gi = gi0 + r0 + u;
+                ok[u] = gi < M && col_ok;
+                w[u] = gi * e.ldw + e.col0 + gj;
+                mv[u] = vv[u] = wv[u] = dv[u] = 0.f;
+                if (ok[u]) {
+                    if (!e.sgd) {
+                        mv[u] = e.mA[w[u]];
+                        vv[u] = e.vA[w[u]];
+                    }
+                    wv[u] = e.Wm[w[u]];
+                    dv[u] = e.D[w[u]];
                 }
-                w4[h] = ld4(e.Wm + w + 4 * h);
-                d4[h] = ld4(e.D + w + 4 * h);
             }
 #pragma unroll
-            for (int h = 0; h < 2; ++h) {
-                float *mm = reinterpret_cast<float *>(&m4[h]), *vv = reinterpret_cast<float *>(&v4[h]);
-                float *ww = reinterpret_cast<float *>(&w4[h]), *dd = reinterpret_cast<float *>(&d4[h]);
-                float st[4];
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    float a = e.sgd ? 0.f : mm[q], b = e.sgd ? 0.f : vv[q];
-                    st[q] = adam_step(e, v[4 * h + q], a, b);
-                    mm[q] = a;
-                    vv[q] = b;
-                    ww[q] -= st[q];
-                    dd[q] -= st[q];
-                }
+            for (int u = 0; u < 4; ++u) {
+                if (!ok[u]) continue;
+                const float stp = adam_step(e, st[(r0 + u) * PSTAGE_PITCH + lane], mv[u], vv[u]);
                 if (!e.sgd) {
-                    st4(e.mA + w + 4 * h, m4[h]);
-                    st4(e.vA + w + 4 * h, v4[h]);
+                    e.mA[w[u]] = mv[u];
+                    e.vA[w[u]] = vv[u];
                 }
-                st4(e.Wm + w + 4 * h, w4[h]);
-                st4(e.D + w + 4 * h, d4[h]);
-                st4(e.Sh + w + 4 * h, make_float4(-st[0], -st[1], -st[2], -st[3]));
+                e.Wm[w[u]] = wv[u] - stp;
+                e.D[w[u]] = dv[u] - stp;
+                e.Sh[w[u]] = -stp;
             }
-        } else {
-            for (int q = 0; q < 8 && gj + q < N; ++q) epi_apply(e, gi, gj + q, v[q]);
         }
         return;
     }
-    // TC_BGD_P: M += acc, P = M + lambda (A - (W - W0)) (+ R0), 0 on dead
-    // channels, written transposed (consecutive lanes: consecutive rows)
-    for (int q = 0; q < 8 && gj + q < N; ++q) e.Pth[(gj + q) * e.ldp + gi] = bgd_p_value(e, gi, gj + q, v[q]);
+    // TC_BGD_P: the gradient factor per element (lanes over columns), put
+    // back into the staging block, then written transposed with the lanes
+    // over rows (consecutive rows of P^T's column are consecutive in memory)
+#pragma unroll 4
+    for (int r = 0; r < 32; ++r) {
+        const int64_t gi = gi0 + r;
+        if (gi < M && col_ok) st[r * PSTAGE_PITCH + lane] = bgd_p_value(e, gi, gj, st[r * PSTAGE_PITCH + lane]);
+    }
+    __syncwarp();
+    const int64_t gi = gi0 + lane;
+    if (gi < M) {
+#pragma unroll 4
+        for (int c = 0; c < 32; ++c)
+            if (gj0 + c < N) e.Pth[(gj0 + c) * e.ldp + gi] = st[lane * PSTAGE_PITCH + c];
+    }
 }
 
 template <int MODE>
@@ -620,11 +631,12 @@ __global__ void __launch_bounds__(PTHREADS, 1)
                                  int b_row0, int a_row0, const TcEpi e, int *err, int kchunk, int tiles_m,
                                  int tiles_n, int nz) {
     using TL = Tile<256, true>;
-    constexpr int KS = TL::KS, STAGES = TL::STAGES, PLANE_A = TL::PLANE_A, PLANE_B = TL::PLANE_B;
+    constexpr int KS = TL::KS, STAGES = PSTAGES, PLANE_A = TL::PLANE_A, PLANE_B = TL::PLANE_B;
     constexpr int STAGE_BYTES = TL::STAGE_BYTES;
     extern __shared__ uint8_t smem_raw[];
     uint8_t *smem = reinterpret_cast<uint8_t *>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint64_t *full = reinterpret_cast<uint64_t *>(smem + STAGES * STAGE_BYTES);
+    float *stage_all = reinterpret_cast<float *>(smem + STAGES * STAGE_BYTES);   // 8 warps x 32 x 33
+    uint64_t *full = reinterpret_cast<uint64_t *>(stage_all + PEPI_WARPS * 32 * PSTAGE_PITCH);
     uint64_t *empty = full + STAGES;
     uint64_t *tfull = empty + STAGES;     // [2]: MMAs of an accumulator done
     uint64_t *tempty = tfull + 2;         // [2]: the epilogue has read an accumulator
@@ -770,6 +782,7 @@ __global__ void __launch_bounds__(PTHREADS, 1)
             // (K = 0: nothing was issued into the accumulator; the products are 0)
             const bool none = Kz <= 0;
             const float sa = (gi < M && !none) ? e.ainv[gi] : 0.f;
+            float *st = stage_all + (warp - 2) * 32 * PSTAGE_PITCH;
 #pragma unroll 1
             for (int c0 = half * 128; c0 < half * 128 + 128; c0 += 32) {
                 uint32_t v[32];
@@ -780,17 +793,18 @@ __global__ void __launch_bounds__(PTHREADS, 1)
                     __syncwarp();
                     if (lane == 0) tc::mbar_arrive(tc::smem_u32(&tempty[acc]));
                 }
-                if (gi >= M) continue;
+                if (j0 + c0 >= N) continue;
+                // this lane's row of the 32 x 32 block, unscaled, into the
+                // staging block; then the block with the lanes over columns
 #pragma unroll
-                for (int g8 = 0; g8 < 32; g8 += 8) {
-                    const int64_t gj = j0 + c0 + g8;
-                    if (gj >= N) break;
-                    float x[8];
-#pragma unroll
-                    for (int q = 0; q < 8; ++q)
-                        x[q] = (gj + q < N && !none) ? __uint_as_float(v[g8 + q]) * (sa * e.binv[gj + q]) : 0.f;
-                    persistent_epi8<MODE>(e, z, gi, gj, N, x);
+                for (int q = 0; q < 32; ++q) {
+                    const int64_t gj = j0 + c0 + q;
+                    st[lane * PSTAGE_PITCH + q] =
+                        (gj < N && !none) ? __uint_as_float(v[q]) * (sa * e.binv[gj]) : 0.f;
                 }
+                __syncwarp();
+                persistent_block<MODE>(e, z, i0 + quarter * 32, j0 + c0, M, N, st, lane);
+                __syncwarp();
             }
         }
     }
@@ -1182,7 +1196,7 @@ int sm_count() {
 template <int MODE>
 realq_status_t launch_persistent(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off,
                                  int b_row0, const TcEpi &e, int *err, int a_row0, int kchunk) {
-    constexpr int SM = Tile<256, true>::SMEM;
+    constexpr int SM = PSTAGES * Tile<256, true>::STAGE_BYTES + PEPI_WARPS * 32 * PSTAGE_PITCH * 4 + 1024 + 256;
     REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_f16x3_persistent_kernel<MODE>), SM));
     const int64_t tiles_m = ceil_div(M, TB), tiles_n = ceil_div(N, 256);
     const int64_t nz = kchunk > 0 ? ceil_div(K, kchunk) : 1;

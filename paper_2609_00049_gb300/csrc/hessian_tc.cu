@@ -63,15 +63,36 @@ __host__ __device__ inline int64_t lower_tiles(int nti) {
     return c;
 }
 
+// The lower tiles in groups of 8 row blocks: a group's tiles column by
+// column (within a column, its rows that reach it), so that the CTAs resident
+// at one time cover a compact block of the product and share their channel
+// blocks through L2.  A bijection onto {(ti, tj): tj <= ti / 2, ti < nti}.
 __device__ __forceinline__ void lower_tile(int64_t idx, int nti, int &ti, int &tj) {
-    int r = 0;
-    for (; r < nti; ++r) {
-        const int64_t c = r / 2 + 1;
-        if (idx < c) break;
+    constexpr int G = 8;
+    int r0 = 0;
+    for (;; r0 += G) {
+        const int r1 = min(r0 + G, nti);
+        int64_t c = 0;
+        for (int r = r0; r < r1; ++r) c += r / 2 + 1;
+        if (idx < c || r1 >= nti) break;
         idx -= c;
     }
-    ti = r;
-    tj = (int)idx;
+    const int r1 = min(r0 + G, nti);
+    for (int j = 0;; ++j) {
+        const int lo = max(r0, 2 * j);
+        const int cnt = r1 > lo ? r1 - lo : 0;
+        if (cnt == 0) {   // (not reached for idx < lower_tiles(nti))
+            ti = r1 - 1;
+            tj = 0;
+            return;
+        }
+        if (idx < cnt) {
+            ti = lo + (int)idx;
+            tj = j;
+            return;
+        }
+        idx -= cnt;
+    }
 }
 
 __global__ void __launch_bounds__(THREADS, 1)
