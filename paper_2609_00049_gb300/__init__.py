@@ -669,8 +669,8 @@ def realq_set_bgd_products(mode: int) -> None:
 
 
 def realq_set_tensor_overlap(mode: int) -> None:
-    """Wide-tile f16x3 products: 1 persistent with the epilogue overlapped
-    (default), 0 one tile per CTA (identical results)."""
+    """The wide-tile f16x3 G product: 1 persistent with the epilogue
+    overlapped (default), 0 one tile per CTA (identical results)."""
     _check(lib().realq_set_tensor_overlap(int(mode)))
 
 

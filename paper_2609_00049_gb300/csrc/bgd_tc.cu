@@ -1259,12 +1259,11 @@ realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));
     {
         Launch L(name, s);
-        if (f16 && wide && g_overlap) {
-            switch (e.mode) {
-                case TC_STORE: REALQ_TRY(launch_persistent<TC_STORE>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
-                case TC_BGD_P: REALQ_TRY(launch_persistent<TC_BGD_P>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
-                default: REALQ_TRY(launch_persistent<TC_ADAM>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk)); break;
-            }
+        if (f16 && wide && g_overlap && e.mode == TC_ADAM) {
+            // (measured on the 70B step: the G product 4.5 % faster persistent;
+            // the gradient-factor product 10 % slower with the 3-stage ring
+            // the staged epilogue leaves room for, so it keeps the tile kernel)
+            REALQ_TRY(launch_persistent<TC_ADAM>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk));
         } else if (f16) {
             if (wide) REALQ_TRY((launch_x3<256, true>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
             else REALQ_TRY((launch_x3<128, true>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
