@@ -40,11 +40,6 @@ NCU_TRAFFIC = {
     # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
     # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
     ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
-    # the f16x3 G product of the LLaMA-3.1-70B block: three fused-Adam
-    # launches of down_proj captured in the bench step (one-pass DRAM
-    # counters: 14.28-14.50 GB each, 4.64 GB per TFLOP), scaled to the
-    # family's average launch (1.128 TFLOP)
-    ("llama3.1-70b", "bgd_g_gemm_adam"): 5234000000,
 }
 
 
@@ -730,9 +725,9 @@ def main():
                     help="saliency-weighted grouped Hessians with this many row groups (0: one Hessian per input)")
     ap.add_argument("--bgd-products", type=int, choices=[0, 1], default=1,
                     help="the plain Block-GD products as f16x3 (1, where the shapes allow) or tf32x3 (0)")
-    ap.add_argument("--tensor-overlap", type=int, choices=[0, 1], default=1,
-                    help="wide-tile f16x3 products as persistent kernels with the epilogue overlapped (1) or one "
-                         "tile per CTA (0)")
+    ap.add_argument("--tensor-overlap", type=int, choices=[0, 1, 2], default=1,
+                    help="wide-tile f16x3 products as persistent kernels with the epilogue overlapped: 1 the G "
+                         "product, 2 G and P, 0 none (one tile per CTA)")
     ap.add_argument("--a-loss-clip", type=float, default=None,
                     help="with --minibatch-seqs: token-form Block-GD gradient with per-token output clipping")
     ap.add_argument("--clock-log", default=None, help="directory for the raw clock samples (default: temp dir)")

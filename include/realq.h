@@ -520,10 +520,10 @@ realq_status_t realq_set_bgd_products(int mode);
  * 128 x 256 tiles.  1 (default): a persistent kernel, one CTA per SM walking
  * the tiles, a TMA warp, an MMA warp and eight epilogue warps, with two TMEM
  * accumulators so that a tile's epilogue overlaps the next tile's main
- * loop; 0: one tile per CTA, the epilogue after the main loop.  The same
- * MMAs in the same order per tile and the same epilogue arithmetic
- * (identical results).  Process-wide.  REALQ_ERR_INVALID_ARG for other
- * values.  No counterpart in the paper. */
+ * loop; 2: the gradient-factor product P as well; 0: one tile per CTA, the
+ * epilogue after the main loop.  The same MMAs in the same order per tile
+ * and the same epilogue arithmetic (identical results).  Process-wide.
+ * REALQ_ERR_INVALID_ARG for other values.  No counterpart in the paper. */
 realq_status_t realq_set_tensor_overlap(int mode);
 
 /* Tuning: the causal attention of the block ops.  1 (default): tiled

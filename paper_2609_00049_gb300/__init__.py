@@ -669,8 +669,9 @@ def realq_set_bgd_products(mode: int) -> None:
 
 
 def realq_set_tensor_overlap(mode: int) -> None:
-    """The wide-tile f16x3 G product: 1 persistent with the epilogue
-    overlapped (default), 0 one tile per CTA (identical results)."""
+    """Wide-tile f16x3 products as persistent kernels with the epilogue
+    overlapped: 1 the G product (default), 2 G and P, 0 none (one tile per
+    CTA; identical results)."""
     _check(lib().realq_set_tensor_overlap(int(mode)))
 
 

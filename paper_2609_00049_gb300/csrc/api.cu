@@ -809,7 +809,7 @@ realq_status_t realq_set_tensor_tile(int mode) {
 }
 
 realq_status_t realq_set_tensor_overlap(int mode) {
-    if (mode < 0 || mode > 1) return fail(REALQ_ERR_INVALID_ARG, "set_tensor_overlap: mode 0 or 1");
+    if (mode < 0 || mode > 2) return fail(REALQ_ERR_INVALID_ARG, "set_tensor_overlap: mode 0, 1 or 2");
     tc_set_overlap(mode);
     return REALQ_OK;
 }

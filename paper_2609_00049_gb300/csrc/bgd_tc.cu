@@ -552,7 +552,7 @@ __device__ __forceinline__ void persistent_tile(int64_t t, int tiles_m, int tile
     j0 = ((pid % pg) / gm) * 256;
 }
 
-constexpr int PSTAGES = 3;             // ring stages (the rest of shared memory stages the epilogue)
+constexpr int PSTAGES = 4;             // ring stages (the rest of shared memory stages the epilogue)
 constexpr int PSTAGE_PITCH = 33;       // a warp's 32 x 32 staging block, padded
 
 // One 32 x 32 block of the output (rows gi0 .., columns gj0 ..), staged in
@@ -1180,7 +1180,7 @@ realq_status_t launch_x3(cudaStream_t s, const Maps &m, int64_t M, int64_t N, in
 }
 
 int g_tile_mode = 0;   // 0: by the grid (wide_tiles_pay), 1: always 128 x 128, 2: always 128 x 256
-int g_overlap = 1;     // the persistent f16x3 kernel for wide-tile f16x3 products
+int g_overlap = 1;     // persistent f16x3 kernels: 1 for the G product, 2 for G and the gradient factor
 
 int sm_count() {
     static int sms = 0;
@@ -1197,6 +1197,7 @@ template <int MODE>
 realq_status_t launch_persistent(cudaStream_t s, const Maps &m, int64_t M, int64_t N, int64_t K, int k_off,
                                  int b_row0, const TcEpi &e, int *err, int a_row0, int kchunk) {
     constexpr int SM = PSTAGES * Tile<256, true>::STAGE_BYTES + PEPI_WARPS * 32 * PSTAGE_PITCH * 4 + 1024 + 256;
+    static_assert(SM <= 232448, "shared memory of the persistent kernel");
     REALQ_TRY(set_smem_limit(reinterpret_cast<const void *>(gemm_f16x3_persistent_kernel<MODE>), SM));
     const int64_t tiles_m = ceil_div(M, TB), tiles_n = ceil_div(N, 256);
     const int64_t nz = kchunk > 0 ? ceil_div(K, kchunk) : 1;
@@ -1259,11 +1260,10 @@ realq_status_t tc_gemm_x3(cudaStream_t s, const TcMaps &maps, int64_t M, int64_t
     const bool wide = g_tile_mode == 2 || (g_tile_mode == 0 && wide_tiles_pay(M, N, nz));
     {
         Launch L(name, s);
-        if (f16 && wide && g_overlap && e.mode == TC_ADAM) {
-            // (measured on the 70B step: the G product 4.5 % faster persistent;
-            // the gradient-factor product 10 % slower with the 3-stage ring
-            // the staged epilogue leaves room for, so it keeps the tile kernel)
+        if (f16 && wide && g_overlap >= 1 && e.mode == TC_ADAM) {
             REALQ_TRY(launch_persistent<TC_ADAM>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk));
+        } else if (f16 && wide && g_overlap == 2 && e.mode == TC_BGD_P) {
+            REALQ_TRY(launch_persistent<TC_BGD_P>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk));
         } else if (f16) {
             if (wide) REALQ_TRY((launch_x3<256, true>(s, mp.wide, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));
             else REALQ_TRY((launch_x3<128, true>(s, mp.narrow, M, N, K, k_off, b_row0, e, err, a_row0, kchunk, exact)));

@@ -83,7 +83,8 @@ bool tc_gemm_eligible(int64_t m, int64_t n);
 void tc_set_tile_mode(int mode);
 // 1 (default): the wide-tile f16x3 G product (fused Adam epilogue) runs as a
 // persistent kernel that overlaps each tile's epilogue with the next tile's
-// main loop; 0: one tile per CTA (process-wide).
+// main loop; 2: the gradient-factor product too; 0: one tile per CTA
+// (process-wide).
 void tc_set_overlap(int mode);
 // The column-serial quantizer: 0 the barrier-phased kernel everywhere
 // (default), 1 the pipelined kernel where the group parameters come at the

@@ -920,7 +920,7 @@ def test_persistent_products_are_bit_identical(qkw, m, n, bf16):
     outs = []
     rq.realq_set_tensor_tile(2)
     try:
-        for mode in (0, 1):   # (1 last: the default stays set)
+        for mode in (0, 2, 1):   # (1 last: the default stays set)
             rq.realq_set_tensor_overlap(mode)
             outs.append(layer.quantize(W0, prep, rq.quant_cfg(**qkw), rq.bgd_cfg(2e-4, steps_per_block=2),
                                        F=dev(case.F)))
@@ -928,8 +928,9 @@ def test_persistent_products_are_bit_identical(qkw, m, n, bf16):
     finally:
         rq.realq_set_tensor_overlap(1)
         rq.realq_set_tensor_tile(0)
-    for k in ("codes", "scale", "zero", "W"):
-        assert torch.equal(getattr(outs[0], k), getattr(outs[1], k)), k
+    for o in outs[1:]:
+        for k in ("codes", "scale", "zero", "W"):
+            assert torch.equal(getattr(outs[0], k), getattr(o, k)), k
 
 
 # ------------------------------------------------- tensor-core tile shapes ---
