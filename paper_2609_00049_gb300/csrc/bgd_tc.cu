@@ -524,7 +524,7 @@ __global__ void __launch_bounds__(THREADS, 1)
 
 // ---------------------------------------------------------------------------
 // Persistent f16x3 products with the epilogue overlapped (the plain Block-GD
-// G and P products and the K-split slices of the next block's G).  One CTA
+// G product; the gradient factor P with realq_set_tensor_overlap(2)).  One CTA
 // per SM walks the tiles (t = blockIdx.x, + gridDim.x, ... in the grouped
 // order above, K-split slices last) with three roles: warp 0 issues the TMA
 // loads of the ring, warp 1 the MMAs, and warps 2..9 run the epilogue.  The
@@ -562,16 +562,10 @@ constexpr int PSTAGE_PITCH = 33;       // a warp's 32 x 32 staging block, padded
 template <int MODE>
 __device__ __forceinline__ void persistent_block(const TcEpi &e, int z, int64_t gi0, int64_t gj0, int64_t M,
                                                  int64_t N, float *st, int lane) {
+    static_assert(MODE == TC_ADAM || MODE == TC_BGD_P, "persistent epilogues: Adam and the gradient factor");
     const int64_t gj = gj0 + lane;
     const bool col_ok = gj < N;
-    if (MODE == TC_STORE) {
-#pragma unroll 4
-        for (int r = 0; r < 32; ++r) {
-            const int64_t gi = gi0 + r;
-            if (gi < M && col_ok) e.C[(int64_t)z * e.czs + gi * e.ldc + gj] = st[r * PSTAGE_PITCH + lane];
-        }
-        return;
-    }
+    (void)z;
     if (MODE == TC_ADAM) {
         // four rows at a time: their loads are issued before any store
         for (int r0 = 0; r0 < 32; r0 += 4) {
