@@ -37,9 +37,6 @@ UNIT = "columns/s"
 # dram bytes per launch from ncu captures (profiles/), keyed by (workload, kernel); None
 # when the kernel changed after its capture.
 NCU_TRAFFIC = {
-    # the four Hessian launches of a Qwen3-0.6B block step (n = 1024, 2048,
-    # 1024, 3072 at T = 262,144): 6.095 GB in total, averaged per launch
-    ("qwen3-0.6b", "hessian_syrk_tc"): 1523751616,
 }
 
 
