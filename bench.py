@@ -37,6 +37,11 @@ UNIT = "columns/s"
 # dram bytes per launch from ncu captures (profiles/), keyed by (workload, kernel); None
 # when the kernel changed after its capture.
 NCU_TRAFFIC = {
+    # the G product of the LLaMA-3.1-70B block (the persistent f16x3 kernel
+    # with the fused Adam step): three down_proj launches captured in the
+    # bench step with one-pass DRAM counters (14.29-14.51 GB each, 4.64 GB
+    # per TFLOP), scaled to the family's average launch (1.128 TFLOP)
+    ("llama3.1-70b", "bgd_g_gemm_adam"): 5234000000,
 }
 
 
