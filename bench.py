@@ -42,6 +42,14 @@ NCU_TRAFFIC = {
     # bench step with one-pass DRAM counters (14.29-14.51 GB each, 4.64 GB
     # per TFLOP), scaled to the family's average launch (1.128 TFLOP)
     ("llama3.1-70b", "bgd_g_gemm_adam"): 5234000000,
+    # the gradient-factor product P of the same block: three down_proj
+    # launches (28.4-30.7 GB each, 3.30 GB per TFLOP), scaled to the family's
+    # average launch (1.995 TFLOP)
+    ("llama3.1-70b", "bgd_p_gemm"): 6584000000,
+    # the four Hessians of one step of the same block, one-pass counters:
+    # down_in (n = 28,672) 1010 GB, the three n = 8192 inputs 58-66 GB each;
+    # averaged per launch
+    ("llama3.1-70b", "hessian_syrk_tc"): 296200000000,
 }
 
 
