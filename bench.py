@@ -49,7 +49,7 @@ NCU_TRAFFIC = {
     # the four Hessians of one step of the same block, one-pass counters:
     # down_in (n = 28,672) 1010 GB, the three n = 8192 inputs 58-66 GB each;
     # averaged per launch
-    ("llama3.1-70b", "hessian_syrk_tc"): 296200000000,
+    ("llama3.1-70b", "hessian_syrk_tc"): 299400000000,
 }
 
 
